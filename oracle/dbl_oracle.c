@@ -1,0 +1,501 @@
+/*
+ * dbl_oracle.c -- plain, slow, fp64 CPU reference for the ResNet-18 training
+ * step of the hybrid dual-batch / cyclic-progressive scheme
+ * (arXiv 2509.26092).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the
+ * CPU-baseline leg of the benchmark may load this code.  It shares nothing
+ * with the CUDA library: no headers, no helpers, no tables.
+ *
+ * Every routine is the textbook definition written out as loops, in double
+ * precision, with no blocking, fusion or reordering beyond what the
+ * definition states.  OpenMP only splits independent output elements (or
+ * independent images for the scatter-form adjoint) across threads; each
+ * output is still summed in one fixed order.
+ *
+ * Layouts: activations NHWC, conv weights KRSC, all row-major.
+ *
+ * Paper passages followed:
+ *   - mini-batch SGD with the batch-mean gradient: Sec. 2.2, Eq. 1;
+ *   - model-update factor (1 for large-batch workers, d_S/d_L or
+ *     sqrt(d_S/d_L) for small-batch workers): Sec. 3.4;
+ *   - asynchronous pushes applied by the server as they arrive: Sec. 2.4
+ *     (ASP) and Sec. 3.1;
+ *   - resolution changes of cyclic progressive learning: Sec. 4.1;
+ *   - ResNet-18 (convolutions, BatchNorm, ReLU, residual, global pooling and
+ *     one fully connected layer): Sec. 5.1.1 and Sec. 6.
+ * Readings where the paper is silent (momentum form, push order, resize
+ * convention, max-pool tie rule, BN epsilon) are the ones listed in the
+ * design notes; each is restated at the routine that takes it.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define IDX4(a, b, c, d, B, C, D) ((((int64_t)(a) * (B) + (b)) * (C) + (c)) * (D) + (d))
+
+static int out_dim(int in, int k, int stride, int pad) { return (in + 2 * pad - k) / stride + 1; }
+
+/* ------------------------------------------------------------------------ */
+/* bf16 storage rounding.                                                    */
+/* bfloat16 keeps fp32's 8-bit exponent and 8 significand bits (7 stored).  */
+/* Round-to-nearest-even of a double to that grid, written from the format's */
+/* definition: normal numbers have a quantum of 2^(e-8) for |x| in          */
+/* [2^(e-1), 2^e); below 2^-126 the quantum is fixed at 2^-133.             */
+/* ------------------------------------------------------------------------ */
+double orc_round_bf16(double x)
+{
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    frexp(x, &e); /* |x| in [2^(e-1), 2^e) */
+    int qexp = e - 8;
+    if (e - 1 < -126) qexp = -133;
+    double scaled = ldexp(x, -qexp);
+    double r = nearbyint(scaled); /* default rounding mode: ties to even */
+    double y = ldexp(r, qexp);
+    /* overflow beyond the largest finite bf16 (0x7F7F) rounds to infinity */
+    const double bmax = ldexp(255.0, 120); /* (2 - 2^-7) * 2^127 */
+    if (fabs(y) > bmax) y = copysign(INFINITY, x);
+    return y;
+}
+
+void orc_round_bf16_array(double* a, int64_t n)
+{
+    for (int64_t i = 0; i < n; ++i) a[i] = orc_round_bf16(a[i]);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Convolution (cross-correlation, zero padding), Sec. 5.1.1 ResNet-18.      */
+/*   y[n,p,q,k] = sum_{r,s,c} x[n, p*st + r - pad, q*st + s - pad, c] w[k,r,s,c] */
+/*   P = floor((H + 2 pad - R)/st) + 1.                                      */
+/* ------------------------------------------------------------------------ */
+void orc_conv2d_fwd(const double* x, const double* w, double* y, int N, int H, int W, int C, int K,
+                    int R, int S, int st, int pad)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, S, st, pad);
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < P; ++p)
+            for (int q = 0; q < Q; ++q)
+                for (int k = 0; k < K; ++k) {
+                    double acc = 0.0;
+                    for (int r = 0; r < R; ++r) {
+                        const int h = p * st + r - pad;
+                        if (h < 0 || h >= H) continue;
+                        for (int s = 0; s < S; ++s) {
+                            const int ww = q * st + s - pad;
+                            if (ww < 0 || ww >= W) continue;
+                            const double* xp = x + IDX4(n, h, ww, 0, H, W, C);
+                            const double* wp = w + IDX4(k, r, s, 0, R, S, C);
+                            for (int c = 0; c < C; ++c) acc += xp[c] * wp[c];
+                        }
+                    }
+                    y[IDX4(n, p, q, k, P, Q, K)] = acc;
+                }
+}
+
+/* Data gradient: the adjoint of the forward map, written in scatter form   */
+/* (each dy element sends dy*w to every input it read).  Images are         */
+/* independent, so the scatter is race-free per image.                      */
+void orc_conv2d_dgrad(const double* dy, const double* w, double* dx, int N, int H, int W, int C, int K,
+                      int R, int S, int st, int pad)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, S, st, pad);
+    memset(dx, 0, sizeof(double) * (size_t)N * H * W * C);
+#pragma omp parallel for schedule(static)
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < P; ++p)
+            for (int q = 0; q < Q; ++q)
+                for (int k = 0; k < K; ++k) {
+                    const double g = dy[IDX4(n, p, q, k, P, Q, K)];
+                    for (int r = 0; r < R; ++r) {
+                        const int h = p * st + r - pad;
+                        if (h < 0 || h >= H) continue;
+                        for (int s = 0; s < S; ++s) {
+                            const int ww = q * st + s - pad;
+                            if (ww < 0 || ww >= W) continue;
+                            double* xp = dx + IDX4(n, h, ww, 0, H, W, C);
+                            const double* wp = w + IDX4(k, r, s, 0, R, S, C);
+                            for (int c = 0; c < C; ++c) xp[c] += g * wp[c];
+                        }
+                    }
+                }
+}
+
+/* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] x[n, p*st+r-pad, q*st+s-pad, c]. */
+void orc_conv2d_wgrad(const double* x, const double* dy, double* dw, int N, int H, int W, int C, int K,
+                      int R, int S, int st, int pad)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, S, st, pad);
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int k = 0; k < K; ++k)
+        for (int r = 0; r < R; ++r)
+            for (int s = 0; s < S; ++s)
+                for (int c = 0; c < C; ++c) {
+                    double acc = 0.0;
+                    for (int n = 0; n < N; ++n)
+                        for (int p = 0; p < P; ++p) {
+                            const int h = p * st + r - pad;
+                            if (h < 0 || h >= H) continue;
+                            for (int q = 0; q < Q; ++q) {
+                                const int ww = q * st + s - pad;
+                                if (ww < 0 || ww >= W) continue;
+                                acc += dy[IDX4(n, p, q, k, P, Q, K)] * x[IDX4(n, h, ww, c, H, W, C)];
+                            }
+                        }
+                    dw[IDX4(k, r, s, c, R, S, C)] = acc;
+                }
+}
+
+/* Single-element evaluators, for sampled checks at full size.               */
+double orc_conv2d_fwd_at(const double* x, const double* w, int N, int H, int W, int C, int K, int R, int S,
+                         int st, int pad, int n, int p, int q, int k)
+{
+    (void)N; (void)K;
+    double acc = 0.0;
+    for (int r = 0; r < R; ++r) {
+        const int h = p * st + r - pad;
+        if (h < 0 || h >= H) continue;
+        for (int s = 0; s < S; ++s) {
+            const int ww = q * st + s - pad;
+            if (ww < 0 || ww >= W) continue;
+            for (int c = 0; c < C; ++c) acc += x[IDX4(n, h, ww, c, H, W, C)] * w[IDX4(k, r, s, c, R, S, C)];
+        }
+    }
+    return acc;
+}
+
+/* dx at one input element, gathered: the outputs (p,q) whose window placed  */
+/* tap (r,s) on (h,w) are those with p*st = h + pad - r (exact division).    */
+double orc_conv2d_dgrad_at(const double* dy, const double* w, int N, int H, int W, int C, int K, int R, int S,
+                           int st, int pad, int n, int h, int ww, int c)
+{
+    (void)N;
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, S, st, pad);
+    double acc = 0.0;
+    for (int r = 0; r < R; ++r) {
+        const int ph = h + pad - r;
+        if (ph < 0 || ph % st) continue;
+        const int p = ph / st;
+        if (p >= P) continue;
+        for (int s = 0; s < S; ++s) {
+            const int qw = ww + pad - s;
+            if (qw < 0 || qw % st) continue;
+            const int q = qw / st;
+            if (q >= Q) continue;
+            for (int k = 0; k < K; ++k) acc += dy[IDX4(n, p, q, k, P, Q, K)] * w[IDX4(k, r, s, c, R, S, C)];
+        }
+    }
+    return acc;
+}
+
+double orc_conv2d_wgrad_at(const double* x, const double* dy, int N, int H, int W, int C, int K, int R, int S,
+                           int st, int pad, int k, int r, int s, int c)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, S, st, pad);
+    double acc = 0.0;
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < P; ++p) {
+            const int h = p * st + r - pad;
+            if (h < 0 || h >= H) continue;
+            for (int q = 0; q < Q; ++q) {
+                const int ww = q * st + s - pad;
+                if (ww < 0 || ww >= W) continue;
+                acc += dy[IDX4(n, p, q, k, P, Q, K)] * x[IDX4(n, h, ww, c, H, W, C)];
+            }
+        }
+    return acc;
+}
+
+/* ------------------------------------------------------------------------ */
+/* BatchNorm in training mode over the M = N*H*W rows of a [M, C] matrix.    */
+/* mean_c = (1/M) sum y, var_c = (1/M) sum (y - mean)^2 (biased),            */
+/* xhat = (y - mean)/sqrt(var + eps), out = gamma*xhat + beta [+ res],       */
+/* then ReLU (max(0, .)) when relu != 0.                                     */
+/* ------------------------------------------------------------------------ */
+void orc_bn_fwd(const double* y, int64_t M, int C, const double* gamma, const double* beta, double eps,
+                const double* res, int relu, double* out, double* mean, double* invstd)
+{
+#pragma omp parallel for schedule(static)
+    for (int c = 0; c < C; ++c) {
+        double s = 0.0;
+        for (int64_t m = 0; m < M; ++m) s += y[m * C + c];
+        const double mu = s / (double)M;
+        double v = 0.0;
+        for (int64_t m = 0; m < M; ++m) {
+            const double d = y[m * C + c] - mu;
+            v += d * d;
+        }
+        v /= (double)M;
+        mean[c] = mu;
+        invstd[c] = 1.0 / sqrt(v + eps);
+    }
+#pragma omp parallel for schedule(static)
+    for (int64_t m = 0; m < M; ++m)
+        for (int c = 0; c < C; ++c) {
+            double o = gamma[c] * (y[m * C + c] - mean[c]) * invstd[c] + beta[c];
+            if (res) o += res[m * C + c];
+            if (relu && !(o > 0.0)) o = 0.0;
+            out[m * C + c] = o;
+        }
+}
+
+/* Backward of orc_bn_fwd.  g = (dout [+ dout2]) * [out > 0] (ReLU'(0) = 0), */
+/* the gradient reaching gamma*xhat + beta [+ res].                          */
+/*   dbeta = sum g, dgamma = sum g*xhat,                                     */
+/*   dy = gamma*invstd*(g - dbeta/M - xhat*dgamma/M),                        */
+/*   dres = g (the residual branch's gradient).                              */
+void orc_bn_bwd(const double* dout, const double* dout2, const double* out, int relu, const double* y, int64_t M,
+                int C, const double* gamma, const double* mean, const double* invstd, double* dy, double* dres,
+                double* dgamma, double* dbeta)
+{
+#pragma omp parallel for schedule(static)
+    for (int c = 0; c < C; ++c) {
+        double sg = 0.0, sgx = 0.0;
+        for (int64_t m = 0; m < M; ++m) {
+            double g = dout[m * C + c] + (dout2 ? dout2[m * C + c] : 0.0);
+            if (relu && !(out[m * C + c] > 0.0)) g = 0.0;
+            const double xh = (y[m * C + c] - mean[c]) * invstd[c];
+            sg += g;
+            sgx += g * xh;
+        }
+        dbeta[c] = sg;
+        dgamma[c] = sgx;
+        for (int64_t m = 0; m < M; ++m) {
+            double g = dout[m * C + c] + (dout2 ? dout2[m * C + c] : 0.0);
+            if (relu && !(out[m * C + c] > 0.0)) g = 0.0;
+            const double xh = (y[m * C + c] - mean[c]) * invstd[c];
+            dy[m * C + c] = gamma[c] * invstd[c] * (g - sg / (double)M - xh * sgx / (double)M);
+            if (dres) dres[m * C + c] = g;
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Max pooling, window R x R, stride st, padding pad (ImageNet stem: 3,2,1). */
+/* Padding counts as -infinity.  Tie rule (paper silent): the first maximum  */
+/* in row-major (r, s) window order is the argmax and takes all the gradient.*/
+/* ------------------------------------------------------------------------ */
+void orc_maxpool_fwd(const double* x, int N, int H, int W, int C, int R, int st, int pad, double* y, int32_t* arg)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, R, st, pad);
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < P; ++p)
+            for (int q = 0; q < Q; ++q)
+                for (int c = 0; c < C; ++c) {
+                    double best = -INFINITY;
+                    int bi = -1;
+                    for (int r = 0; r < R; ++r)
+                        for (int s = 0; s < R; ++s) {
+                            const int h = p * st + r - pad, ww = q * st + s - pad;
+                            if (h < 0 || h >= H || ww < 0 || ww >= W) continue;
+                            const double v = x[IDX4(n, h, ww, c, H, W, C)];
+                            if (v > best) {
+                                best = v;
+                                bi = r * R + s;
+                            }
+                        }
+                    y[IDX4(n, p, q, c, P, Q, C)] = best;
+                    if (arg) arg[IDX4(n, p, q, c, P, Q, C)] = bi;
+                }
+}
+
+void orc_maxpool_bwd(const double* dy, const int32_t* arg, int N, int H, int W, int C, int R, int st, int pad,
+                     double* dx)
+{
+    const int P = out_dim(H, R, st, pad), Q = out_dim(W, R, st, pad);
+    memset(dx, 0, sizeof(double) * (size_t)N * H * W * C);
+#pragma omp parallel for schedule(static)
+    for (int n = 0; n < N; ++n)
+        for (int p = 0; p < P; ++p)
+            for (int q = 0; q < Q; ++q)
+                for (int c = 0; c < C; ++c) {
+                    const int a = arg[IDX4(n, p, q, c, P, Q, C)];
+                    const int h = p * st + a / R - pad, ww = q * st + a % R - pad;
+                    dx[IDX4(n, h, ww, c, H, W, C)] += dy[IDX4(n, p, q, c, P, Q, C)];
+                }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Head: global average pooling (Sec. 6 notes the global pooling layer that  */
+/* makes the network resolution-agnostic), one fully connected layer with   */
+/* bias (Sec. 5.1.1), softmax cross-entropy averaged over the batch         */
+/* (the 1/n of Eq. 1).                                                       */
+/* ------------------------------------------------------------------------ */
+void orc_avgpool_fwd(const double* x, int N, int HW, int C, double* f)
+{
+    for (int n = 0; n < N; ++n)
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int i = 0; i < HW; ++i) s += x[((int64_t)n * HW + i) * C + c];
+            f[(int64_t)n * C + c] = s / (double)HW;
+        }
+}
+
+void orc_avgpool_bwd(const double* df, int N, int HW, int C, double* dx)
+{
+    for (int n = 0; n < N; ++n)
+        for (int i = 0; i < HW; ++i)
+            for (int c = 0; c < C; ++c) dx[((int64_t)n * HW + i) * C + c] = df[(int64_t)n * C + c] / (double)HW;
+}
+
+/* logits[n,j] = sum_c f[n,c] W[j,c] + b[j] */
+void orc_fc_fwd(const double* f, const double* Wt, const double* b, int N, int C, int J, double* logits)
+{
+    for (int n = 0; n < N; ++n)
+        for (int j = 0; j < J; ++j) {
+            double s = b[j];
+            for (int c = 0; c < C; ++c) s += f[(int64_t)n * C + c] * Wt[(int64_t)j * C + c];
+            logits[(int64_t)n * J + j] = s;
+        }
+}
+
+/* dW[j,c] = sum_n dl[n,j] f[n,c]; db[j] = sum_n dl[n,j]; df[n,c] = sum_j dl[n,j] W[j,c] */
+void orc_fc_bwd(const double* dl, const double* f, const double* Wt, int N, int C, int J, double* dW, double* db,
+                double* df)
+{
+    for (int j = 0; j < J; ++j) {
+        double sb = 0.0;
+        for (int n = 0; n < N; ++n) sb += dl[(int64_t)n * J + j];
+        db[j] = sb;
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int n = 0; n < N; ++n) s += dl[(int64_t)n * J + j] * f[(int64_t)n * C + c];
+            dW[(int64_t)j * C + c] = s;
+        }
+    }
+    for (int n = 0; n < N; ++n)
+        for (int c = 0; c < C; ++c) {
+            double s = 0.0;
+            for (int j = 0; j < J; ++j) s += dl[(int64_t)n * J + j] * Wt[(int64_t)j * C + c];
+            df[(int64_t)n * C + c] = s;
+        }
+}
+
+/* loss = (1/N) sum_n [ log sum_j exp(l[n,j]) - l[n, label_n] ];            */
+/* dlogits[n,j] = (softmax(l[n])_j - [j == label_n]) / N.                    */
+double orc_softmax_ce(const double* logits, const int32_t* labels, int N, int J, double* dlogits)
+{
+    double loss = 0.0;
+    for (int n = 0; n < N; ++n) {
+        const double* l = logits + (int64_t)n * J;
+        double mx = l[0];
+        for (int j = 1; j < J; ++j)
+            if (l[j] > mx) mx = l[j];
+        double z = 0.0;
+        for (int j = 0; j < J; ++j) z += exp(l[j] - mx);
+        const double lse = mx + log(z);
+        loss += lse - l[labels[n]];
+        for (int j = 0; j < J; ++j) {
+            const double p = exp(l[j] - lse);
+            dlogits[(int64_t)n * J + j] = (p - (j == labels[n] ? 1.0 : 0.0)) / (double)N;
+        }
+    }
+    return loss / (double)N;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Parameter-server merge of the two workers' pushes (Sec. 3.4 with Eq. 1). */
+/* Each push i carries its worker's batch-mean gradient g_i and is scaled by */
+/* the model-update factor f_i (f_L = 1, f_S = d_S/d_L or its square root).  */
+/* The server's optimizer is SGD with momentum in the form                  */
+/*     u <- mu*u - lr*f_i*g_i ;  w <- w + u                                  */
+/* (reduces to Eq. 1 when mu = 0).  Under ASP the server applies each push  */
+/* as it arrives (Sec. 2.4):                                                 */
+/*   order 0: large push, then small push (two momentum steps),             */
+/*   order 1: small push, then large push,                                   */
+/*   order 2: both pushes summed into one step (the synchronous reading).   */
+/* A NULL gradient is a worker that did not push in this round.             */
+/* ------------------------------------------------------------------------ */
+void orc_ps_merge(double* w, double* u, const double* gL, const double* gS, int64_t n, double lr, double mu,
+                  double fL, double fS, int order)
+{
+    for (int64_t i = 0; i < n; ++i) {
+        double wi = w[i], ui = u[i];
+        if (order == 2) {
+            double g = 0.0;
+            if (gL) g += fL * gL[i];
+            if (gS) g += fS * gS[i];
+            ui = mu * ui - lr * g;
+            wi = wi + ui;
+        } else {
+            const double* first = order == 0 ? gL : gS;
+            const double* second = order == 0 ? gS : gL;
+            const double ff = order == 0 ? fL : fS, fs = order == 0 ? fS : fL;
+            if (first) {
+                ui = mu * ui - lr * ff * first[i];
+                wi = wi + ui;
+            }
+            if (second) {
+                ui = mu * ui - lr * fs * second[i];
+                wi = wi + ui;
+            }
+        }
+        w[i] = wi;
+        u[i] = ui;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Bilinear downsampling for the low-resolution sub-stages (Sec. 4.1).      */
+/* Convention (paper silent): half-pixel centres, no antialiasing, edge     */
+/* clamp.  Output j of an axis samples source coordinate                    */
+/*     src = (j + 1/2) * in/out - 1/2 = ((2j+1)*in - out) / (2*out),        */
+/* taken in exact integers: i0 = floor(num/den), lambda = (num - i0*den)/den,*/
+/* i1 = min(i0 + 1, in - 1).  Negative src (upsampling only) clamps to 0.   */
+/* ------------------------------------------------------------------------ */
+int orc_resize_taps(int in, int out, int32_t* i0, int32_t* i1, double* lam)
+{
+    if (in <= 0 || out <= 0) return -1;
+    for (int j = 0; j < out; ++j) {
+        const int64_t num = (int64_t)(2 * j + 1) * in - out;
+        const int64_t den = 2 * (int64_t)out;
+        int64_t a;
+        double l;
+        if (num <= 0) {
+            a = 0;
+            l = 0.0;
+        } else {
+            a = num / den;
+            l = (double)(num - a * den) / (double)den;
+        }
+        if (a > in - 1) {
+            a = in - 1;
+            l = 0.0;
+        }
+        i0[j] = (int32_t)a;
+        i1[j] = (int32_t)(a + 1 < in ? a + 1 : in - 1);
+        lam[j] = l;
+    }
+    return 0;
+}
+
+/* out[n,y,x,c] = (1-ly)[(1-lx) a + lx b] + ly[(1-lx) c + lx d] */
+int orc_bilinear_resize(const double* in, int N, int Hi, int Wi, int C, double* out, int Ho, int Wo)
+{
+    int32_t *y0 = malloc(sizeof(int32_t) * Ho), *y1 = malloc(sizeof(int32_t) * Ho);
+    int32_t *x0 = malloc(sizeof(int32_t) * Wo), *x1 = malloc(sizeof(int32_t) * Wo);
+    double *ly = malloc(sizeof(double) * Ho), *lx = malloc(sizeof(double) * Wo);
+    int rc = -1;
+    if (!y0 || !y1 || !x0 || !x1 || !ly || !lx) goto done;
+    orc_resize_taps(Hi, Ho, y0, y1, ly);
+    orc_resize_taps(Wi, Wo, x0, x1, lx);
+    for (int n = 0; n < N; ++n)
+        for (int yy = 0; yy < Ho; ++yy)
+            for (int xx = 0; xx < Wo; ++xx)
+                for (int c = 0; c < C; ++c) {
+                    const double a = in[IDX4(n, y0[yy], x0[xx], c, Hi, Wi, C)];
+                    const double b = in[IDX4(n, y0[yy], x1[xx], c, Hi, Wi, C)];
+                    const double cc = in[IDX4(n, y1[yy], x0[xx], c, Hi, Wi, C)];
+                    const double d = in[IDX4(n, y1[yy], x1[xx], c, Hi, Wi, C)];
+                    const double top = (1.0 - lx[xx]) * a + lx[xx] * b;
+                    const double bot = (1.0 - lx[xx]) * cc + lx[xx] * d;
+                    out[IDX4(n, yy, xx, c, Ho, Wo, C)] = (1.0 - ly[yy]) * top + ly[yy] * bot;
+                }
+    rc = 0;
+done:
+    free(y0); free(y1); free(x0); free(x1); free(ly); free(lx);
+    return rc;
+}
