@@ -1,0 +1,238 @@
+/*
+ * dbl.h -- C ABI of libdbl.so: the GB300 (sm_103a) kernels of one training
+ * step of the hybrid dual-batch / cyclic-progressive learning scheme
+ * (arXiv 2509.26092) on ResNet-18.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Every call returns DBL_OK (0) or a negative DBL_ERR_* code; the text of
+ *    the last error on the calling thread is available from dbl_last_error().
+ *  - Device pointers are owned by the caller (PyTorch allocates them); the
+ *    library never allocates or frees device memory.  Scratch space is passed
+ *    in as `ws`/`ws_bytes`, sized by the matching *_workspace_bytes() call.
+ *  - Work is enqueued on the caller's CUDA stream, passed as `void*`
+ *    (a cudaStream_t; NULL is the legacy default stream).  No call
+ *    synchronises the device or the stream, so calls can be captured into a
+ *    CUDA graph.  Exceptions, marked "host" or "synchronous", are stated.
+ *  - Tensors are dense row-major.  Activations are NHWC bfloat16, conv
+ *    weights are KRSC, master weights and gradients are fp32.  Every tensor
+ *    base address must be 16-byte aligned and every NHWC channel count a
+ *    multiple of 8 (a 16-byte pixel row); violations return DBL_ERR_INVALID
+ *    before anything is launched.  There is no slow fallback path.
+ *  - Kernels that wait on an asynchronous copy give up after a bounded time,
+ *    record DBL_ERR_TIMEOUT in a device-side status word and return; read it
+ *    with dbl_device_status().
+ */
+#ifndef DBL_H
+#define DBL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DBL_API __attribute__((visibility("default")))
+#else
+#define DBL_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    DBL_OK = 0,
+    DBL_ERR_INVALID = -1,     /* null pointer, misaligned, inconsistent shape        */
+    DBL_ERR_UNSUPPORTED = -2, /* well-formed request outside what the kernels cover  */
+    DBL_ERR_CUDA = -3,        /* a CUDA call or launch failed                        */
+    DBL_ERR_TIMEOUT = -4,     /* a device-side wait gave up (see dbl_device_status)  */
+    DBL_ERR_WORKSPACE = -5    /* ws_bytes smaller than *_workspace_bytes()           */
+};
+
+enum { DBL_F32 = 0, DBL_BF16 = 1 }; /* element types for dbl_progressive_resize */
+
+/* Text of the last error raised on the calling thread ("" if none). Host. */
+DBL_API const char* dbl_last_error(void);
+
+/* Library version, major*10000 + minor*100 + patch.  Host. */
+DBL_API int dbl_version(void);
+
+/* Synchronous: reads and clears the device-side status word of the current
+ * device (DBL_OK or DBL_ERR_TIMEOUT), after synchronising the device.  For
+ * tests and diagnostics only; never call it inside a captured graph. */
+DBL_API int dbl_device_status(int32_t* status);
+
+/* ========================================================================
+ * Convolution passes as implicit GEMM on the tensor cores.
+ *
+ * The ResNet-18 of the paper (Sec. 5.1.1) is built from these three passes;
+ * the training step needs the forward pass and, through Eq. 1 (the gradient
+ * of the batch-mean loss), the data and weight gradients.
+ *
+ *   y[n,p,q,k] = sum_{r,s,c} x[n, p*stride + r - pad, q*stride + s - pad, c] * w[k,r,s,c]
+ *   P = (h + 2*pad - r)/stride + 1,  Q = (w + 2*pad - s)/stride + 1
+ *
+ * x: [n,h,w,c] bf16, w: [k,r,s,c] bf16, y: [n,P,Q,k] bf16, all NHWC/KRSC.
+ * Supported: r == s, c and k multiples of 64, or the stem case c == 8
+ * (3 colour channels zero-padded to 8) for the forward and weight passes.
+ * ======================================================================== */
+typedef struct {
+    int32_t n, h, w, c; /* input activation shape (NHWC)                    */
+    int32_t k, r, s;    /* output channels and filter size (KRSC weights)   */
+    int32_t stride, pad;
+} dbl_conv_shape;
+
+enum { DBL_PASS_FWD = 0, DBL_PASS_DGRAD = 1, DBL_PASS_WGRAD = 2 };
+
+/* Bytes of scratch the given pass needs for this shape (0 if none).  Host. */
+DBL_API size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass);
+
+/* Forward pass.  Writes y (bf16, rounded to nearest even from the fp32
+ * accumulator).  If ch_sum/ch_sumsq are non-NULL, also writes the per-output-
+ * channel sums of the stored (rounded) y and of its squares over all n*P*Q
+ * rows, [k] fp32 each: the batch statistics BatchNorm needs in training
+ * mode.  Overwrites ch_sum/ch_sumsq (no accumulation). */
+DBL_API int dbl_conv_fwd(const dbl_conv_shape* shape, const void* x_bf16, const void* w_bf16, void* y_bf16,
+                 float* ch_sum, float* ch_sumsq, void* ws, size_t ws_bytes, void* stream);
+
+/* Data gradient: dx = d(sum y*dy)/dx, the adjoint of the forward pass in its
+ * input.  dy: [n,P,Q,k] bf16; dx: [n,h,w,c] bf16 (fully overwritten).
+ * Supported for stride 1, and for stride 2 with even h and w. */
+DBL_API int dbl_conv_dgrad(const dbl_conv_shape* shape, const void* dy_bf16, const void* w_bf16, void* dx_bf16, void* ws,
+                   size_t ws_bytes, void* stream);
+
+/* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*stride+r-pad, q*stride+s-pad, c],
+ * fp32 [k,r,s,c].  accumulate != 0 adds to dw instead of overwriting it.
+ * The split over n*P*Q is reduced in a fixed order (deterministic). */
+DBL_API int dbl_conv_wgrad(const dbl_conv_shape* shape, const void* x_bf16, const void* dy_bf16, float* dw_f32,
+                   int accumulate, void* ws, size_t ws_bytes, void* stream);
+
+/* ========================================================================
+ * BatchNorm (training mode) + residual + ReLU, the non-convolution layers of
+ * ResNet-18 (Sec. 5.1.1).
+ *
+ *   mean = ch_sum/count, var = ch_sumsq/count - mean^2 (biased),
+ *   invstd = 1/sqrt(var + eps),
+ *   out = [ReLU]( gamma*(y - mean)*invstd + beta [+ residual] )
+ *
+ * y, residual, out: [count, c] bf16 (NHWC flattened); gamma, beta, ch_sum,
+ * ch_sumsq, save_mean, save_invstd: [c] fp32.  ReLU'(0) is taken as 0.
+ * ======================================================================== */
+typedef struct {
+    int64_t count; /* rows: n*h*w                  */
+    int32_t c;     /* channels, a multiple of 8    */
+    float eps;     /* variance epsilon (1e-5)      */
+    int32_t relu;  /* nonzero: apply ReLU          */
+} dbl_bn_shape;
+
+/* Per-channel sum and sum of squares of y over all rows, [c] fp32 each.
+ * (dbl_conv_fwd already provides them for its own output.) */
+DBL_API int dbl_bn_stats(const dbl_bn_shape* shape, const void* y_bf16, float* ch_sum, float* ch_sumsq, void* stream);
+
+/* Normalise + affine + optional residual + optional ReLU; writes out (bf16)
+ * and the batch mean and 1/sqrt(var+eps) used (needed by the backward). */
+DBL_API int dbl_bn_relu_fused(const dbl_bn_shape* shape, const void* y_bf16, const float* ch_sum, const float* ch_sumsq,
+                      const float* gamma, const float* beta, const void* residual_bf16 /* or NULL */,
+                      void* out_bf16, float* save_mean, float* save_invstd, void* stream);
+
+/* Bytes of scratch dbl_bn_relu_fused_bwd needs.  Host. */
+DBL_API size_t dbl_bn_workspace_bytes(const dbl_bn_shape* shape);
+
+/* Backward of dbl_bn_relu_fused.  The incoming gradient is dout [+ dout2]
+ * (a tensor read by two consumers, e.g. a block output feeding the next
+ * block's convolution and its shortcut), masked by ReLU through out > 0 when
+ * shape->relu is set:  g = (dout + dout2) * [out > 0].  Then
+ *   dbeta = sum g, dgamma = sum g*xhat, xhat = (y - mean)*invstd,
+ *   dy = gamma*invstd*(g - dbeta/count - xhat*dgamma/count),
+ * and, if dresidual is non-NULL, dresidual = g (the residual branch's
+ * gradient).  dy, dresidual: bf16 [count, c]; dgamma, dbeta: fp32 [c]
+ * (overwritten).  The channel sums are reduced in a fixed order. */
+DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf16, const void* dout2_bf16 /* or NULL */,
+                          const void* y_bf16, const void* out_bf16, const float* gamma, const float* save_mean,
+                          const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
+                          float* dgamma, float* dbeta, void* ws, size_t ws_bytes, void* stream);
+
+/* ========================================================================
+ * Stem max pooling (ImageNet ResNet-18): 3x3 window, stride 2, padding 1,
+ * padding counted as -infinity.  x: [n,h,w,c] bf16, y: [n,P,Q,c] bf16,
+ * argmax: [n,P,Q,c] uint8, the window index r*3+s of the first maximum in
+ * row-major window order (the tie rule).  The backward routes each of
+ * dy [+ dy2] to its argmax and sums what lands on each input: dx [n,h,w,c].
+ * ======================================================================== */
+DBL_API int dbl_maxpool_fwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* x_bf16, void* y_bf16, uint8_t* argmax,
+                    void* stream);
+DBL_API int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy_bf16, const void* dy2_bf16,
+                    const uint8_t* argmax, void* dx_bf16, void* stream);
+
+/* ========================================================================
+ * Head forward + backward in one call: global average pooling (the pooling
+ * that makes the network resolution-agnostic, Sec. 6), one fully connected
+ * layer (Sec. 5.1.1) and softmax cross-entropy averaged over the batch (the
+ * 1/n of Eq. 1).
+ *   feat[n,c] = mean_hw x,  logits = feat*fc_w^T + fc_b,
+ *   loss = mean_n (logsumexp(logits_n) - logits_n[label_n]),
+ *   dlogits = (softmax - onehot)/n,  dfc_w = dlogits^T feat,  dfc_b = sum_n dlogits,
+ *   dx[n,i,c] = (dlogits*fc_w)[n,c] / hw.
+ * x: [n,hw,c] bf16; fc_w: [classes,c] fp32; fc_b: [classes] fp32;
+ * labels: [n] int32 in [0,classes); loss: one fp32 on the device;
+ * dfc_w, dfc_b: fp32 (overwritten); dx: [n,hw,c] bf16.
+ * ======================================================================== */
+DBL_API size_t dbl_head_workspace_bytes(int32_t n, int32_t c, int32_t classes);
+DBL_API int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x_bf16, const float* fc_w,
+                     const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx_bf16,
+                     void* ws, size_t ws_bytes, void* stream);
+
+/* ========================================================================
+ * Parameter-server merge of the two workers' pushes (Sec. 3.4, with the SGD
+ * of Eq. 1 and momentum).  Each push i brings its worker's batch-mean
+ * gradient g_i, scaled by the model-update factor f_i (1 for the large-batch
+ * worker; d_S/d_L or sqrt(d_S/d_L) for the small-batch worker):
+ *     u <- momentum*u - lr*f_i*g_i ;  w <- w + u
+ * order 0: large push then small push (ASP arrival order, Sec. 2.4);
+ * order 1: small then large; order 2: one step on f_L*g_L + f_S*g_S.
+ * A NULL gradient is a worker that did not push (both NULL is invalid).
+ * w, u: fp32 [n], updated in place; w16_out (or NULL): bf16 copy of the new
+ * w, the weights the workers pull for their next step.
+ * ======================================================================== */
+typedef struct {
+    float lr, momentum, f_large, f_small;
+    int32_t order;
+} dbl_merge_params;
+
+DBL_API int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const float* g_large, const float* g_small, int64_t n,
+                            const dbl_merge_params* params, void* stream);
+
+/* ========================================================================
+ * Progressive resizing for the low-resolution sub-stages of cyclic
+ * progressive learning (Sec. 4.1): bilinear, half-pixel centres, no
+ * antialiasing, downsampling only.  Output j of an axis reads source
+ * i0 = floor(num/den), i1 = min(i0+1, in-1), weight lambda = (num - i0*den)/den
+ * with num = (2j+1)*in - out, den = 2*out, all in exact integers.
+ * in: [n,h_in,w_in,c] (DBL_F32 or DBL_BF16); out: [n,h_out,w_out,c_out_stride]
+ * (DBL_F32 or DBL_BF16) with channels c..c_out_stride-1 set to zero.
+ * h_out == h_in is a plain cast/pad; h_out > h_in is DBL_ERR_UNSUPPORTED.
+ * ======================================================================== */
+DBL_API int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
+                           int out_dtype, int32_t h_out, int32_t w_out, int32_t c_out_stride, void* stream);
+
+/* Host: the integer taps above for one axis (i0, i1, lambda: [out] each). */
+DBL_API int dbl_resize_taps(int32_t in, int32_t out, int32_t* i0, int32_t* i1, float* lambda);
+
+/* ========================================================================
+ * Host-side planner of dual-batch learning (Sec. 3.3-3.4).
+ * ======================================================================== */
+/* Model-update factor of a small-batch worker: d_S/d_L, or sqrt(d_S/d_L)
+ * when sqrt_scheme != 0 (Sec. 3.4).  Returns NaN for d_large <= 0. */
+DBL_API double dbl_update_factor(double d_small, double d_large, int sqrt_scheme);
+
+/* Eqs. 4-8: given the extra-time ratio k > 1, data amount d, worker counts,
+ * the time-model coefficients a, b (per-batch time a*x + b, Eq. 2) and the
+ * large batch B_L, returns d_L = k*d/n, d_S = (d - n_L*d_L)/n_S,
+ * B_S = b/((a + b/B_L)*d_L/d_S - a) and f_S = d_S/d_L (scheme 1) or its root.
+ * DBL_ERR_INVALID if n_small < 1 or the inputs give no positive B_S. */
+DBL_API int dbl_plan(double k, double d, int32_t n_small, int32_t n_large, double a, double b, double batch_large,
+             int sqrt_scheme, double* d_large, double* d_small, double* batch_small, double* f_small);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DBL_H */

@@ -1,0 +1,346 @@
+// bn.cu -- training-mode BatchNorm + residual + ReLU, forward and backward,
+// for the ResNet-18 of Sec. 5.1.1.  All kernels are HBM-bound streaming
+// passes over [count, C] bf16 tensors with 16-byte (8-channel) vectors.
+//
+// Forward (one pass, 6 B/element with a residual): the batch statistics come
+// from the convolution epilogue (or dbl_bn_stats); every CTA turns them into
+// per-channel scale/shift in shared memory, then
+//     out = ReLU(y*scale + shift [+ res]).
+// Backward (two passes): a reduce pass of sum(g) and sum(g*xhat) per channel
+// into per-CTA partials, a tiny fixed-order finalize, and an apply pass
+//     dy = gamma*invstd*(g - sum(g)/count - xhat*sum(g*xhat)/count).
+#include "dbl_internal.cuh"
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxC = 2048;
+
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
+{
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 t = __bfloat1622float2(h[k]);
+        f[2 * k] = t.x;
+        f[2 * k + 1] = t.y;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&f)[8])
+{
+    uint4 v;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(f[2 * k], f[2 * k + 1]);
+    return v;
+}
+
+// ----------------------------------------------------------------------------- statistics
+__global__ void __launch_bounds__(kThreads) bn_stats_kernel(const __nv_bfloat16* __restrict__ y, int64_t count, int C,
+                                                            float* __restrict__ sum, float* __restrict__ sumsq)
+{
+    const int groups = C / 8;
+    const int g = threadIdx.x % groups;
+    const int rstep = kThreads / groups;
+    float s[8] = {}, q[8] = {};
+    for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += (int64_t)gridDim.x * rstep) {
+        float f[8];
+        unpack8(__ldg(reinterpret_cast<const uint4*>(y + r * C) + g), f);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            s[k] += f[k];
+            q[k] = fmaf(f[k], f[k], q[k]);
+        }
+    }
+    __shared__ float red[kThreads][17];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        red[threadIdx.x][k] = s[k];
+        red[threadIdx.x][8 + k] = q[k];
+    }
+    __syncthreads();
+    if (threadIdx.x < groups) {
+        float ts[8] = {}, tq[8] = {};
+        for (int t = threadIdx.x; t < rstep * groups; t += groups)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                ts[k] += red[t][k];
+                tq[k] += red[t][8 + k];
+            }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            atomicAdd(sum + 8 * threadIdx.x + k, ts[k]);
+            atomicAdd(sumsq + 8 * threadIdx.x + k, tq[k]);
+        }
+    }
+}
+
+// ----------------------------------------------------------------------------- forward apply
+__global__ void __launch_bounds__(kThreads)
+    bn_apply_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ res,
+                    __nv_bfloat16* __restrict__ out, int64_t count, int C, float eps, int relu,
+                    const float* __restrict__ sum, const float* __restrict__ sumsq, const float* __restrict__ gamma,
+                    const float* __restrict__ beta, float* __restrict__ save_mean, float* __restrict__ save_invstd)
+{
+    __shared__ float sc[kMaxC], sh[kMaxC];
+    const double inv_n = 1.0 / (double)count;
+    for (int c = threadIdx.x; c < C; c += kThreads) {
+        const double mean = (double)sum[c] * inv_n;
+        double var = (double)sumsq[c] * inv_n - mean * mean;
+        if (var < 0.0) var = 0.0;
+        const float invstd = (float)(1.0 / sqrt(var + (double)eps));
+        const float scale = gamma[c] * invstd;
+        sc[c] = scale;
+        sh[c] = beta[c] - (float)mean * scale;
+        if (blockIdx.x == 0) {
+            save_mean[c] = (float)mean;
+            save_invstd[c] = invstd;
+        }
+    }
+    __syncthreads();
+    const int64_t nvec = count * C / 8;
+    for (int64_t v = (int64_t)blockIdx.x * kThreads + threadIdx.x; v < nvec; v += (int64_t)gridDim.x * kThreads) {
+        const int c0 = (int)((v * 8) % C);
+        float f[8];
+        unpack8(__ldcs(reinterpret_cast<const uint4*>(y) + v), f);
+        float r[8] = {};
+        if (res) unpack8(__ldcs(reinterpret_cast<const uint4*>(res) + v), r);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            float o = fmaf(f[k], sc[c0 + k], sh[c0 + k]) + r[k];
+            f[k] = (relu && !(o > 0.f)) ? 0.f : o;
+        }
+        reinterpret_cast<uint4*>(out)[v] = pack8(f);
+    }
+}
+
+// ----------------------------------------------------------------------------- backward
+// g = (dout [+ dout2]) * [out > 0]
+__device__ __forceinline__ void load_g(const __nv_bfloat16* dout, const __nv_bfloat16* dout2,
+                                       const __nv_bfloat16* out, int relu, int64_t v, float (&g)[8])
+{
+    unpack8(__ldg(reinterpret_cast<const uint4*>(dout) + v), g);
+    if (dout2) {
+        float h[8];
+        unpack8(__ldg(reinterpret_cast<const uint4*>(dout2) + v), h);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) g[k] += h[k];
+    }
+    if (relu) {
+        float o[8];
+        unpack8(__ldg(reinterpret_cast<const uint4*>(out) + v), o);
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (!(o[k] > 0.f)) g[k] = 0.f;
+    }
+}
+
+// Each CTA reduces a contiguous range of rows into partial[blk][0..C) (sum g)
+// and partial[blk][C..2C) (sum g*xhat).
+__global__ void __launch_bounds__(kThreads)
+    bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
+                         const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int64_t count,
+                         int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
+                         int64_t rows_per_blk, float* __restrict__ partial)
+{
+    const int groups = C / 8;
+    const int g = threadIdx.x % groups;
+    const int rstep = kThreads / groups;
+    float mu[8], is[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        mu[k] = mean[8 * g + k];
+        is[k] = invstd[8 * g + k];
+    }
+    float sg[8] = {}, sgx[8] = {};
+    const int64_t r0 = (int64_t)blockIdx.x * rows_per_blk;
+    const int64_t r1 = min(count, r0 + rows_per_blk);
+    for (int64_t r = r0 + threadIdx.x / groups; r < r1; r += rstep) {
+        const int64_t v = r * groups + g;
+        float gg[8], yy[8];
+        load_g(dout, dout2, out, relu, v, gg);
+        unpack8(__ldg(reinterpret_cast<const uint4*>(y) + v), yy);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            sg[k] += gg[k];
+            sgx[k] = fmaf(gg[k], (yy[k] - mu[k]) * is[k], sgx[k]);
+        }
+    }
+    __shared__ float red[kThreads][17];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        red[threadIdx.x][k] = sg[k];
+        red[threadIdx.x][8 + k] = sgx[k];
+    }
+    __syncthreads();
+    if (threadIdx.x < groups) {
+        float ts[8] = {}, tx[8] = {};
+        for (int t = threadIdx.x; t < rstep * groups; t += groups)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                ts[k] += red[t][k];
+                tx[k] += red[t][8 + k];
+            }
+        float* p = partial + (int64_t)blockIdx.x * 2 * C;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            p[8 * threadIdx.x + k] = ts[k];
+            p[C + 8 * threadIdx.x + k] = tx[k];
+        }
+    }
+}
+
+// Fixed-order sum of the partials (double), then dgamma/dbeta and the three
+// per-channel coefficients of the apply pass.
+__global__ void bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C, int64_t count,
+                                       const float* __restrict__ gamma, const float* __restrict__ invstd,
+                                       float* __restrict__ dgamma, float* __restrict__ dbeta, float* __restrict__ coef)
+{
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    double sg = 0.0, sgx = 0.0;
+    for (int b = 0; b < nblk; ++b) {
+        sg += partial[(int64_t)b * 2 * C + c];
+        sgx += partial[(int64_t)b * 2 * C + C + c];
+    }
+    dbeta[c] = (float)sg;
+    dgamma[c] = (float)sgx;
+    coef[c] = gamma[c] * invstd[c];
+    coef[C + c] = (float)(sg / (double)count);
+    coef[2 * C + c] = (float)(sgx / (double)count);
+}
+
+__global__ void __launch_bounds__(kThreads)
+    bn_bwd_apply_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
+                        const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int64_t count,
+                        int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
+                        const float* __restrict__ coef, __nv_bfloat16* __restrict__ dy, __nv_bfloat16* __restrict__ dres)
+{
+    __shared__ float k1[kMaxC], k2[kMaxC], k3[kMaxC], mu[kMaxC], is[kMaxC];
+    for (int c = threadIdx.x; c < C; c += kThreads) {
+        k1[c] = coef[c];
+        k2[c] = coef[C + c];
+        k3[c] = coef[2 * C + c];
+        mu[c] = mean[c];
+        is[c] = invstd[c];
+    }
+    __syncthreads();
+    const int64_t nvec = count * C / 8;
+    for (int64_t v = (int64_t)blockIdx.x * kThreads + threadIdx.x; v < nvec; v += (int64_t)gridDim.x * kThreads) {
+        const int c0 = (int)((v * 8) % C);
+        float g[8], yy[8], d[8];
+        load_g(dout, dout2, out, relu, v, g);
+        unpack8(__ldg(reinterpret_cast<const uint4*>(y) + v), yy);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int c = c0 + k;
+            const float xh = (yy[k] - mu[c]) * is[c];
+            d[k] = k1[c] * (g[k] - k2[c] - xh * k3[c]);
+        }
+        reinterpret_cast<uint4*>(dy)[v] = pack8(d);
+        if (dres) reinterpret_cast<uint4*>(dres)[v] = pack8(g);
+    }
+}
+
+int bn_grid(int64_t nvec)
+{
+    int64_t b = (nvec + kThreads - 1) / kThreads;
+    const int64_t cap = (int64_t)dbl::sm_count() * 8;
+    if (b > cap) b = cap;
+    return (int)(b < 1 ? 1 : b);
+}
+
+int check_shape(const dbl_bn_shape* s, const char* who)
+{
+    if (!s || s->count < 0 || s->c <= 0) return dbl::set_error(DBL_ERR_INVALID, "%s: bad shape", who);
+    if (s->c % 8 != 0 || s->c > kMaxC || (kThreads % (s->c / 8)) != 0)
+        return dbl::set_error(DBL_ERR_UNSUPPORTED, "%s: channel count %d (need a multiple of 8 dividing 2048)", who,
+                              s->c);
+    return DBL_OK;
+}
+
+// Backward reduce split: a fixed function of the shape, so the workspace
+// size does not depend on the device.
+int64_t bwd_blocks(int64_t count) { return count <= 0 ? 1 : (count + 255) / 256 < 1024 ? (count + 255) / 256 : 1024; }
+
+}  // namespace
+
+extern "C" {
+
+int dbl_bn_stats(const dbl_bn_shape* s, const void* y, float* ch_sum, float* ch_sumsq, void* stream)
+{
+    using namespace dbl;
+    int rc = check_shape(s, "bn_stats");
+    if (rc) return rc;
+    if (!y || !ch_sum || !ch_sumsq || !aligned16(y)) return set_error(DBL_ERR_INVALID, "bn_stats: bad pointer");
+    cudaStream_t st = as_stream(stream);
+    if ((rc = cuda_check(cudaMemsetAsync(ch_sum, 0, sizeof(float) * s->c, st), "bn_stats memset"))) return rc;
+    if ((rc = cuda_check(cudaMemsetAsync(ch_sumsq, 0, sizeof(float) * s->c, st), "bn_stats memset"))) return rc;
+    if (s->count == 0) return DBL_OK;
+    bn_stats_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(y), s->count,
+                                                                       s->c, ch_sum, ch_sumsq);
+    return launch_check("bn_stats launch");
+}
+
+int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum, const float* ch_sumsq,
+                      const float* gamma, const float* beta, const void* residual, void* out, float* save_mean,
+                      float* save_invstd, void* stream)
+{
+    using namespace dbl;
+    int rc = check_shape(s, "bn_relu_fused");
+    if (rc) return rc;
+    if (!y || !out || !ch_sum || !ch_sumsq || !gamma || !beta || !save_mean || !save_invstd)
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused: null pointer");
+    if (!aligned16(y) || !aligned16(out) || (residual && !aligned16(residual)))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused: tensors must be 16-byte aligned");
+    if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused: empty batch has no statistics");
+    bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, as_stream(stream)>>>(
+        static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
+        static_cast<__nv_bfloat16*>(out), s->count, s->c, s->eps, s->relu, ch_sum, ch_sumsq, gamma, beta, save_mean,
+        save_invstd);
+    return launch_check("bn_relu_fused launch");
+}
+
+size_t dbl_bn_workspace_bytes(const dbl_bn_shape* s)
+{
+    if (!s || s->c <= 0) return 0;
+    return sizeof(float) * ((size_t)bwd_blocks(s->count) * 2 * s->c + 3 * (size_t)s->c);
+}
+
+int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
+                          const float* gamma, const float* save_mean, const float* save_invstd, void* dy,
+                          void* dresidual, float* dgamma, float* dbeta, void* ws, size_t ws_bytes, void* stream)
+{
+    using namespace dbl;
+    int rc = check_shape(s, "bn_relu_fused_bwd");
+    if (rc) return rc;
+    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd: null pointer");
+    if (!aligned16(dout) || !aligned16(y) || !aligned16(dy) || (dout2 && !aligned16(dout2)) ||
+        (out && !aligned16(out)) || (dresidual && !aligned16(dresidual)))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd: tensors must be 16-byte aligned");
+    if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd: empty batch");
+    const size_t need = dbl_bn_workspace_bytes(s);
+    if (!ws || ws_bytes < need)
+        return set_error(DBL_ERR_WORKSPACE, "bn_relu_fused_bwd: workspace %zu < %zu bytes", ws_bytes, need);
+    const int C = s->c;
+    const int64_t nblk = bwd_blocks(s->count);
+    const int64_t rows = (s->count + nblk - 1) / nblk;
+    float* partial = static_cast<float*>(ws);
+    float* coef = partial + nblk * 2 * C;
+    cudaStream_t st = as_stream(stream);
+    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
+    bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
+                                                         save_mean, save_invstd, rows, partial);
+    if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
+    bn_bwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+                                                            dgamma, dbeta, coef);
+    if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
+    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
+        bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
+        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
+    return launch_check("bn_bwd_apply launch");
+}
+
+}  // extern "C"

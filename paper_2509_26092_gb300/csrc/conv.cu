@@ -1,0 +1,811 @@
+// conv.cu -- convolution forward, data-gradient and weight-gradient passes of
+// ResNet-18 (Sec. 5.1.1; the gradients are those of the batch-mean loss of
+// Eq. 1) as implicit GEMMs on the sm_103a tensor cores.
+//
+// One kernel template serves every pass.  A CTA owns a 128 x BN tile of the
+// GEMM result D, accumulated in tensor memory (TMEM) by tcgen05.mma with bf16
+// operands and fp32 accumulation:
+//
+//   pass   D rows (M)          D cols (N)     reduction            A operand            B operand
+//   fwd    output pixels n,p,q out channel k  taps x in channels   im2col(x), K-major   w [k][rsc], K-major
+//   dgrad  input pixels n,h,w  in channel c   taps x out channels  im2col(dy), K-major  w [k][rs][c], MN-major
+//   wgrad  taps x in channel   out channel k  output pixels        im2col(x), MN-major  dy [pix][k], MN-major
+//
+// Operands are staged in shared memory by TMA: the activation side with
+// im2col-mode tensor maps (the bounding box handles zero padding, stride and
+// the ragged tail of the last tile), the other side with tiled tensor maps,
+// all with 128-byte swizzling (no swizzle for the 8-channel stem input).
+// Warp roles: warp 4 issues TMA loads into a STAGES-deep ring guarded by
+// full/empty mbarriers, warp 5 allocates TMEM and issues the MMAs (one thread),
+// warps 0-3 drain TMEM to global memory (bf16 rows plus BatchNorm channel
+// statistics for fwd, fp32 split-K partials for wgrad).
+//
+// Stride-2 data gradients are split into the 4 output phases (h mod 2,
+// w mod 2); each phase is a stride-1 correlation with the taps of matching
+// parity, so no MMA work is spent on the zeros of the strided input.
+// Every mbarrier wait is bounded (see dbl_internal.cuh); a wait that gives up
+// records DBL_ERR_TIMEOUT in the device status word and the CTA winds down.
+#include <algorithm>
+
+#include "dbl_internal.cuh"
+
+namespace {
+
+using namespace dbl::dev;
+
+constexpr int BM = 128;        // tile rows = TMEM lanes
+constexpr int BK = 64;         // reduction elements per stage (128 bytes of bf16)
+constexpr int kA_BYTES = BM * BK * 2;
+constexpr int kTargetCTAs = 304;  // 2 x 152 SMs: split-K sizing target (device independent)
+
+enum Mode : int { kFwd = 0, kDgrad = 1, kWgrad = 2, kFwdC8 = 3, kWgradC8 = 4 };
+
+__device__ int g_conv_status;  // DBL_OK or DBL_ERR_TIMEOUT, read by dbl_device_status()
+
+struct ConvParams {
+    int mode;
+    int M;              // D rows (for dgrad: rows of one phase)
+    int Ncols;          // D columns
+    int m_tiles, n_tiles;
+    // traversal grid of the im2col operand: (images, rows, cols) and origin of grid point (0,0)
+    int gN, gP, gQ;
+    int tstride;        // origin step per grid step
+    int base_h, base_w;
+    int cblocks;        // 64-channel blocks in the reduction (fwd: C/64, dgrad: K/64)
+    int ntaps;          // R*S
+    int S;              // filter width
+    int Cin;            // input channels (fwd B column offset, wgrad row -> (tap, c))
+    int num_kb;         // K-blocks of the whole reduction (fwd, wgrad); per phase from the table (dgrad)
+    int kb_per_split;   // wgrad split-K chunk
+    // dgrad phase tables
+    int phase_div;      // 1 or 2
+    int out_h, out_w;   // full dx spatial size
+    int phase_off[5];
+    int8_t tap_r[16], tap_s[16], tap_oh[16], tap_ow[16];
+    // outputs
+    void* out;          // bf16 rows (fwd, dgrad) or fp32 partials (wgrad)
+    int64_t ldo;        // elements between output rows
+    float* stats;       // fwd: [m_tiles][2][Ncols] or nullptr
+};
+
+__device__ __forceinline__ void report_timeout(volatile int* abort)
+{
+    *abort = 1;
+    atomicExch(&g_conv_status, DBL_ERR_TIMEOUT);
+}
+
+template <int BN, int STAGES>
+struct Cfg {
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int STAGE_BYTES = kA_BYTES + B_BYTES;
+    // + 1 KB alignment slack, + 32 KB guard so that no descriptor stride can
+    // make the tensor cores read past the CTA's shared-memory allocation
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 32768;
+    static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+};
+
+// Number of K-blocks this CTA reduces, and the first one.
+__device__ __forceinline__ void kb_range(const ConvParams& p, int split, int phase, int& kb0, int& nkb)
+{
+    if (p.mode == kDgrad) {
+        kb0 = 0;
+        nkb = (p.phase_off[phase + 1] - p.phase_off[phase]) * p.cblocks;
+    } else if (p.mode == kWgrad || p.mode == kWgradC8) {
+        kb0 = split * p.kb_per_split;
+        nkb = min(p.num_kb, kb0 + p.kb_per_split) - kb0;
+        if (nkb < 0) nkb = 0;
+    } else {
+        kb0 = 0;
+        nkb = p.num_kb;
+    }
+}
+
+template <int BN, int STAGES>
+__global__ void __launch_bounds__(192, 1)
+    conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const ConvParams p)
+{
+    using C = Cfg<BN, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accum_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
+
+    const int n_tile = blockIdx.x % p.n_tiles;
+    const int m_tile = blockIdx.x / p.n_tiles;
+    const int split = (p.mode == kWgrad || p.mode == kWgradC8) ? blockIdx.y : 0;
+    const int phase = p.mode == kDgrad ? blockIdx.y : 0;
+    int kb0, nkb;
+    kb_range(p, split, phase, kb0, nkb);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        mbar_init(&accum_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 4 && lane == 0) {
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 5) {
+        tmem_alloc(&tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    // Start of the tile's im2col traversal (fwd, dgrad): row m_tile*BM of the grid.
+    const int64_t m0 = (int64_t)m_tile * BM;
+    const int64_t gPQ = (int64_t)p.gP * p.gQ;
+
+    if (warp == 4) {
+        // ------------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int tn = 0, tp = 0, tq = 0;
+            if (p.mode == kFwd || p.mode == kDgrad || p.mode == kFwdC8) {
+                tn = (int)(m0 / gPQ);
+                const int64_t rem = m0 % gPQ;
+                tp = (int)(rem / p.gQ);
+                tq = (int)(rem % p.gQ);
+            }
+            const uint32_t tx_bytes = (uint32_t)C::STAGE_BYTES;
+            int it = 0;
+            for (; it < nkb; ++it) {
+                const int s = it % STAGES;
+                if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
+                    report_timeout(&abort_flag);
+                    break;
+                }
+                uint8_t* sa = sgen + s * C::STAGE_BYTES;
+                uint8_t* sb = sa + kA_BYTES;
+                uint64_t* fb = &full_bar[s];
+                mbar_arrive_expect_tx(fb, tx_bytes);
+                const int kb = kb0 + it;
+                if (p.mode == kFwd) {
+                    const int tap = kb / p.cblocks, cb = kb % p.cblocks;
+                    const int r = tap / p.S, sx = tap % p.S;
+                    tma_load_im2col_4d(sa, &tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h,
+                                       tn, (uint16_t)sx, (uint16_t)r);
+                    tma_load_2d(sb, &tmB, fb, tap * p.Cin + cb * 64, n_tile * BN);
+                } else if (p.mode == kDgrad) {
+                    const int t = p.phase_off[phase] + kb / p.cblocks, kbk = kb % p.cblocks;
+                    tma_load_im2col_4d(sa, &tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn,
+                                       (uint16_t)p.tap_ow[t], (uint16_t)p.tap_oh[t]);
+                    const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
+#pragma unroll
+                    for (int j = 0; j < BN / 64; ++j)
+                        tma_load_3d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, wtap, kbk * 64);
+                } else if (p.mode == kWgrad) {
+                    const int64_t pix0 = (int64_t)kb * 64;
+                    const int n = (int)(pix0 / gPQ);
+                    const int64_t rem = pix0 % gPQ;
+                    const int pp = (int)(rem / p.gQ), qq = (int)(rem % p.gQ);
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int mrow = m_tile * BM + 64 * h;
+                        int tap = mrow / p.Cin;
+                        const int c0 = mrow % p.Cin;
+                        if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
+                        tma_load_im2col_4d(sa + h * 8192, &tmA, fb, c0, qq * p.tstride + p.base_w,
+                                           pp * p.tstride + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                    }
+#pragma unroll
+                    for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, (int)pix0);
+                } else if (p.mode == kFwdC8) {
+                    // 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        int tap = kb * 8 + j;
+                        const int wcol = tap * 8;
+                        if (tap >= p.ntaps) tap = p.ntaps - 1;
+                        tma_load_im2col_4d(sa + j * 2048, &tmA, fb, 0, tq * p.tstride + p.base_w,
+                                           tp * p.tstride + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                        tma_load_2d(sb + j * (BN * 16), &tmB, fb, wcol, n_tile * BN);
+                    }
+                } else {  // kWgradC8: 16 taps x 8 channels of rows, 64 pixels
+                    const int64_t pix0 = (int64_t)kb * 64;
+                    const int n = (int)(pix0 / gPQ);
+                    const int64_t rem = pix0 % gPQ;
+                    const int pp = (int)(rem / p.gQ), qq = (int)(rem % p.gQ);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        int tap = m_tile * 16 + j;
+                        if (tap >= p.ntaps) tap = 0;
+                        tma_load_im2col_4d(sa + j * 1024, &tmA, fb, 0, qq * p.tstride + p.base_w,
+                                           pp * p.tstride + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                    }
+#pragma unroll
+                    for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, (int)pix0);
+                }
+            }
+            if (abort_flag) {
+                // let copies already issued land before the CTA's shared memory goes away:
+                // for each stage, wait (time-bounded, ignoring the abort flag) for its last issued phase
+                for (int s = 0; s < STAGES && s < it; ++s) {
+                    const int last = s + STAGES * ((it - 1 - s) / STAGES);
+                    (void)mbar_wait_drain(&full_bar[s], (last / STAGES) & 1);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 5) {
+        // ------------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
+            const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
+            const uint32_t idesc = idesc_bf16(BM, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
+            for (int it = 0; it < nkb; ++it) {
+                const int s = it % STAGES;
+                if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
+                    report_timeout(&abort_flag);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = sbase + s * C::STAGE_BYTES;
+                const uint32_t sb = sa + kA_BYTES;
+#pragma unroll
+                for (int j = 0; j < BK / 16; ++j) {
+                    uint64_t ad, bd;
+                    if (p.mode == kFwd) {
+                        ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                        bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
+                    } else if (p.mode == kDgrad) {
+                        ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                    } else if (p.mode == kWgrad) {
+                        ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
+                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                    } else if (p.mode == kFwdC8) {
+                        // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
+                        // 8-row groups 128 B apart (SBO), the two taps of one MMA 2 KB apart (LBO)
+                        ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
+                        bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
+                    } else {
+                        // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
+                        // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
+                        ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
+                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                    }
+                    mma_bf16(tmem, ad, bd, idesc, (it > 0 || j > 0) ? 1u : 0u);
+                }
+                mma_commit(&empty_bar[s]);
+            }
+            mma_commit(&accum_bar);  // arrives when every MMA issued above has completed
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------------ epilogue (warps 0-3)
+        const bool ok = mbar_wait(&accum_bar, 0, &abort_flag);
+        if (!ok) report_timeout(&abort_flag);
+        tc_fence_after();
+        const int row = warp * 32 + lane;  // TMEM lane = tile row
+        const int64_t m = m0 + row;
+        const bool valid = m < p.M;
+        const bool have_acc = nkb > 0 && ok;
+        float* st_tile = reinterpret_cast<float*>(sgen) + warp * 32 * 33;  // stats transpose scratch
+        float* colsum = reinterpret_cast<float*>(sgen) + 4 * 32 * 33;       // [4][2][BN]
+        const bool want_stats = (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
+
+        int64_t out_row = m;
+        if (p.mode == kDgrad && p.phase_div == 2) {
+            const int64_t hw = (int64_t)p.gP * p.gQ;
+            const int64_t n = m / hw, rem = m % hw;
+            const int i = (int)(rem / p.gQ), j = (int)(rem % p.gQ);
+            const int a = phase >> 1, b = phase & 1;
+            out_row = (n * p.out_h + 2 * i + a) * p.out_w + 2 * j + b;
+        }
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+            uint32_t v[32];
+            if (have_acc) {
+                tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + ch * 32, v);
+                tmem_ld_wait();
+            } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) v[k] = 0u;
+            }
+            const int col0 = n_tile * BN + ch * 32;
+            if (p.mode == kWgrad || p.mode == kWgradC8) {
+                if (valid) {
+                    float* o = static_cast<float*>(p.out) + ((int64_t)split * p.M + m) * p.ldo + col0;
+#pragma unroll
+                    for (int k = 0; k < 32; k += 4)
+                        *reinterpret_cast<float4*>(o + k) = make_float4(__uint_as_float(v[k]), __uint_as_float(v[k + 1]),
+                                                                        __uint_as_float(v[k + 2]), __uint_as_float(v[k + 3]));
+                }
+            } else {
+                uint4 pk[4];
+                __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
+                float rv[32];
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
+                    const float2 back = __bfloat1622float2(h2[k]);
+                    rv[2 * k] = back.x;
+                    rv[2 * k + 1] = back.y;
+                }
+                if (valid) {
+                    uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) o[k] = pk[k];
+                }
+                if (want_stats) {
+                    // column sums of the stored values over this warp's 32 rows
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) st_tile[lane * 33 + k] = valid ? rv[k] : 0.f;
+                    __syncwarp();
+                    float s = 0.f, q = 0.f;
+#pragma unroll 8
+                    for (int r = 0; r < 32; ++r) {
+                        const float x = st_tile[r * 33 + lane];
+                        s += x;
+                        q = fmaf(x, x, q);
+                    }
+                    colsum[(warp * 2 + 0) * BN + ch * 32 + lane] = s;
+                    colsum[(warp * 2 + 1) * BN + ch * 32 + lane] = q;
+                    __syncwarp();
+                }
+            }
+        }
+        if (want_stats) {
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            for (int c = threadIdx.x; c < BN; c += 128) {
+                float s = 0.f, q = 0.f;
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    s += colsum[(w * 2 + 0) * BN + c];
+                    q += colsum[(w * 2 + 1) * BN + c];
+                }
+                float* dst = p.stats + (int64_t)m_tile * 2 * p.Ncols;
+                dst[n_tile * BN + c] = s;
+                dst[p.Ncols + n_tile * BN + c] = q;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 5) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+// ----------------------------------------------------------------------------- reductions
+// Stage 1: per 64-tile chunk and 32 channels, fixed-order sums of the tile partials.
+__global__ void stats_reduce1_kernel(const float* __restrict__ part, int tiles, int K, double* __restrict__ lvl2)
+{
+    __shared__ double red[8][2][33];
+    const int c = blockIdx.x * 32 + threadIdx.x % 32;
+    const int lane8 = threadIdx.x / 32;
+    const int t0 = blockIdx.y * 64, t1 = min(tiles, t0 + 64);
+    double s = 0.0, q = 0.0;
+    if (c < K)
+        for (int t = t0 + lane8; t < t1; t += 8) {
+            s += part[(int64_t)t * 2 * K + c];
+            q += part[(int64_t)t * 2 * K + K + c];
+        }
+    red[lane8][0][threadIdx.x % 32] = s;
+    red[lane8][1][threadIdx.x % 32] = q;
+    __syncthreads();
+    if (threadIdx.x < 32 && c < K) {
+        double ts = 0.0, tq = 0.0;
+        for (int l = 0; l < 8; ++l) {
+            ts += red[l][0][threadIdx.x];
+            tq += red[l][1][threadIdx.x];
+        }
+        lvl2[(int64_t)blockIdx.y * 2 * K + c] = ts;
+        lvl2[(int64_t)blockIdx.y * 2 * K + K + c] = tq;
+    }
+}
+
+__global__ void stats_reduce2_kernel(const double* __restrict__ lvl2, int chunks, int K, float* __restrict__ sum,
+                                     float* __restrict__ sumsq)
+{
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= K) return;
+    double s = 0.0, q = 0.0;
+    for (int i = 0; i < chunks; ++i) {
+        s += lvl2[(int64_t)i * 2 * K + c];
+        q += lvl2[(int64_t)i * 2 * K + K + c];
+    }
+    sum[c] = (float)s;
+    sumsq[c] = (float)q;
+}
+
+// dw[k][m] (+)= sum over splits of part[split][m][k], fixed split order; 32x32 transpose tiles.
+__global__ void wgrad_reduce_kernel(const float* __restrict__ part, int splits, int M, int K, float* __restrict__ dw,
+                                    int accumulate)
+{
+    __shared__ float t[32][33];
+    const int k0 = blockIdx.x * 32, mb = blockIdx.y * 32;
+    const int tx = threadIdx.x % 32, ty = threadIdx.x / 32;  // 32 x 8 threads
+    for (int i = ty; i < 32; i += 8) {
+        const int m = mb + i, k = k0 + tx;
+        float s = 0.f;
+        if (m < M && k < K)
+            for (int sp = 0; sp < splits; ++sp) s += part[((int64_t)sp * M + m) * K + k];
+        t[i][tx] = s;
+    }
+    __syncthreads();
+    for (int i = ty; i < 32; i += 8) {
+        const int k = k0 + i, m = mb + tx;
+        if (k < K && m < M) {
+            float* d = dw + (int64_t)k * M + m;
+            *d = accumulate ? *d + t[tx][i] : t[tx][i];
+        }
+    }
+}
+
+// ----------------------------------------------------------------------------- host side
+struct Plan {
+    int mode;
+    int BN;
+    ConvParams p;
+    dim3 grid;
+    size_t ws_part = 0, ws_lvl2 = 0;  // bytes: split-K partials or tile stats; stats level 2
+    int stat_chunks = 0;
+};
+
+int out_dim(int in, int k, int st, int pad) { return (in + 2 * pad - k) / st + 1; }
+
+int choose_bn(int cols)
+{
+    if (cols % 128 == 0) return 128;
+    return 64;
+}
+
+int validate(const dbl_conv_shape* s, const char* who)
+{
+    using dbl::set_error;
+    if (!s) return set_error(DBL_ERR_INVALID, "%s: null shape", who);
+    if (s->n <= 0 || s->h <= 0 || s->w <= 0 || s->c <= 0 || s->k <= 0 || s->r <= 0 || s->s <= 0 || s->stride <= 0 ||
+        s->pad < 0)
+        return set_error(DBL_ERR_INVALID, "%s: non-positive dimension", who);
+    if (s->r != s->s) return set_error(DBL_ERR_UNSUPPORTED, "%s: only square filters", who);
+    if (s->c % 8) return set_error(DBL_ERR_INVALID, "%s: channels must be a multiple of 8", who);
+    if (s->k % 64) return set_error(DBL_ERR_UNSUPPORTED, "%s: output channels must be a multiple of 64", who);
+    if (s->stride > 2 || s->r > 7 || s->pad > 3)
+        return set_error(DBL_ERR_UNSUPPORTED, "%s: stride <= 2, filter <= 7, pad <= 3 supported", who);
+    if (out_dim(s->h, s->r, s->stride, s->pad) <= 0 || out_dim(s->w, s->s, s->stride, s->pad) <= 0)
+        return set_error(DBL_ERR_INVALID, "%s: empty output", who);
+    return DBL_OK;
+}
+
+int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
+{
+    using dbl::set_error;
+    int rc = validate(s, pass == DBL_PASS_FWD ? "conv_fwd" : pass == DBL_PASS_DGRAD ? "conv_dgrad" : "conv_wgrad");
+    if (rc) return rc;
+    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    ConvParams& p = pl.p;
+    memset(&p, 0, sizeof(p));
+    const bool c8 = s->c == 8;
+    if (!c8 && s->c % 64) return set_error(DBL_ERR_UNSUPPORTED, "conv: input channels must be 8 or a multiple of 64");
+    p.ntaps = s->r * s->s;
+    p.S = s->s;
+    p.Cin = s->c;
+    if (pass == DBL_PASS_FWD) {
+        pl.mode = p.mode = c8 ? kFwdC8 : kFwd;
+        if (c8 && p.ntaps > 56) return set_error(DBL_ERR_UNSUPPORTED, "conv_fwd: stem filter too large");
+        p.M = s->n * P * Q;
+        p.Ncols = s->k;
+        pl.BN = c8 ? 64 : choose_bn(s->k);
+        p.m_tiles = (p.M + BM - 1) / BM;
+        p.n_tiles = s->k / pl.BN;
+        p.gN = s->n;
+        p.gP = P;
+        p.gQ = Q;
+        p.tstride = s->stride;
+        p.base_h = p.base_w = -s->pad;
+        p.cblocks = c8 ? 1 : s->c / 64;
+        p.num_kb = c8 ? (p.ntaps + 7) / 8 : p.ntaps * p.cblocks;
+        p.ldo = s->k;
+        pl.grid = dim3(p.m_tiles * p.n_tiles, 1, 1);
+        pl.ws_part = (size_t)p.m_tiles * 2 * s->k * sizeof(float);
+        pl.stat_chunks = (p.m_tiles + 63) / 64;
+        pl.ws_lvl2 = (size_t)pl.stat_chunks * 2 * s->k * sizeof(double);
+    } else if (pass == DBL_PASS_DGRAD) {
+        if (c8) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: the 8-channel stem has no data gradient path");
+        pl.mode = p.mode = kDgrad;
+        p.Ncols = s->c;
+        pl.BN = choose_bn(s->c);
+        p.n_tiles = s->c / pl.BN;
+        p.cblocks = s->k / 64;
+        p.ldo = s->c;
+        p.out_h = s->h;
+        p.out_w = s->w;
+        p.gN = s->n;
+        if (s->stride == 1) {
+            if (P != s->h || Q != s->w)
+                return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride 1 needs 'same' padding (P == H)");
+            p.phase_div = 1;
+            p.M = s->n * s->h * s->w;
+            p.gP = s->h;
+            p.gQ = s->w;
+            p.base_h = p.base_w = -(s->r - 1 - s->pad);
+            int t = 0;
+            p.phase_off[0] = 0;
+            for (int r2 = 0; r2 < s->r; ++r2)
+                for (int s2 = 0; s2 < s->s; ++s2) {
+                    if (t >= 16) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: too many taps");
+                    // im2col offset (r2, s2) reads dy at h - (R-1-pad) + r2 = h + pad - r with r = R-1-r2
+                    p.tap_oh[t] = (int8_t)r2;
+                    p.tap_ow[t] = (int8_t)s2;
+                    p.tap_r[t] = (int8_t)(s->r - 1 - r2);
+                    p.tap_s[t] = (int8_t)(s->s - 1 - s2);
+                    ++t;
+                }
+            p.phase_off[1] = t;
+            pl.grid = dim3((unsigned)(((p.M + BM - 1) / BM) * p.n_tiles), 1, 1);
+        } else {
+            if ((s->h & 1) || (s->w & 1) || P * 2 != s->h || Q * 2 != s->w)
+                return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride 2 needs even H, W with P = H/2");
+            p.phase_div = 2;
+            p.gP = s->h / 2;
+            p.gQ = s->w / 2;
+            p.M = s->n * p.gP * p.gQ;
+            p.base_h = p.base_w = 0;
+            int t = 0;
+            for (int ph = 0; ph < 4; ++ph) {
+                const int a = ph >> 1, b = ph & 1;
+                p.phase_off[ph] = t;
+                for (int r = 0; r < s->r; ++r) {
+                    const int dh = a + s->pad - r;
+                    if (dh < 0 || (dh & 1)) continue;
+                    for (int c2 = 0; c2 < s->s; ++c2) {
+                        const int dw = b + s->pad - c2;
+                        if (dw < 0 || (dw & 1)) continue;
+                        if (t >= 16) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: too many taps");
+                        p.tap_r[t] = (int8_t)r;
+                        p.tap_s[t] = (int8_t)c2;
+                        p.tap_oh[t] = (int8_t)(dh / 2);
+                        p.tap_ow[t] = (int8_t)(dw / 2);
+                        ++t;
+                    }
+                }
+            }
+            p.phase_off[4] = t;
+            // taps that would read dy at a negative offset are not representable (none for ResNet-18)
+            for (int r = 0; r < s->r; ++r)
+                if (r > 1 + s->pad) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride-2 filter too large for pad");
+            pl.grid = dim3((unsigned)(((p.M + BM - 1) / BM) * p.n_tiles), 4, 1);
+        }
+        p.m_tiles = (p.M + BM - 1) / BM;
+    } else {
+        pl.mode = p.mode = c8 ? kWgradC8 : kWgrad;
+        const int64_t Mrows = (int64_t)p.ntaps * s->c;  // D rows = (tap, c)
+        p.M = (int)Mrows;
+        p.Ncols = s->k;
+        pl.BN = choose_bn(s->k);
+        if (c8) {
+            pl.BN = 64;
+            p.m_tiles = (p.ntaps + 15) / 16;
+        } else {
+            p.m_tiles = (p.M + BM - 1) / BM;
+        }
+        p.n_tiles = s->k / pl.BN;
+        p.gN = s->n;
+        p.gP = P;
+        p.gQ = Q;
+        p.tstride = s->stride;
+        p.base_h = p.base_w = -s->pad;
+        const int64_t pix = (int64_t)s->n * P * Q;
+        p.num_kb = (int)((pix + 63) / 64);
+        const int tiles = p.m_tiles * p.n_tiles;
+        int splits = (kTargetCTAs + tiles - 1) / tiles;
+        if (splits > p.num_kb) splits = p.num_kb;
+        if (splits < 1) splits = 1;
+        p.kb_per_split = (p.num_kb + splits - 1) / splits;
+        splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
+        p.ldo = s->k;
+        pl.grid = dim3((unsigned)tiles, (unsigned)splits, 1);
+        pl.ws_part = (size_t)splits * p.M * s->k * sizeof(float);
+    }
+    return DBL_OK;
+}
+
+size_t plan_ws(const Plan& pl) { return ((pl.ws_part + 255) / 256) * 256 + ((pl.ws_lvl2 + 255) / 256) * 256; }
+
+int enc_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int lower, int upper, int stride,
+               int channels, int pixels, bool swizzle)
+{
+    auto fn = dbl::encode_im2col();
+    if (!fn) return dbl::set_error(DBL_ERR_CUDA, "conv: cuTensorMapEncodeIm2col unavailable from the driver");
+    cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+    int lo[2] = {lower, lower}, hi[2] = {upper, upper};
+    cuuint32_t es[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, lo, hi,
+                    (cuuint32_t)channels, (cuuint32_t)pixels, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return dbl::set_error(DBL_ERR_CUDA, "conv: im2col tensor map encode failed (%d)", (int)r);
+    return DBL_OK;
+}
+
+int enc_tiled(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides_bytes,
+              const cuuint32_t* box, bool swizzle)
+{
+    auto fn = dbl::encode_tiled();
+    if (!fn) return dbl::set_error(DBL_ERR_CUDA, "conv: cuTensorMapEncodeTiled unavailable from the driver");
+    cuuint32_t es[5] = {1, 1, 1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims,
+                    strides_bytes, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return dbl::set_error(DBL_ERR_CUDA, "conv: tiled tensor map encode failed (%d)", (int)r);
+    return DBL_OK;
+}
+
+template <int BN, int STAGES>
+int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t st)
+{
+    using Cf = Cfg<BN, STAGES>;
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             Cf::SMEM);
+        if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
+        attr_set[dev] = true;
+    }
+    conv_igemm_kernel<BN, STAGES><<<pl.grid, 192, Cf::SMEM, st>>>(a, b, pl.p);
+    return dbl::launch_check("conv_igemm launch");
+}
+
+int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t st)
+{
+    if (pl.BN == 128) return launch_cfg<128, 4>(pl, a, b, st);
+    return launch_cfg<64, 4>(pl, a, b, st);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass)
+{
+    Plan pl;
+    if (pass < 0 || pass > 2 || make_plan(shape, pass, pl) != DBL_OK) return 0;
+    if (pass == DBL_PASS_DGRAD) return 0;
+    return plan_ws(pl);
+}
+
+int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y, float* ch_sum, float* ch_sumsq,
+                 void* ws, size_t ws_bytes, void* stream)
+{
+    using namespace dbl;
+    Plan pl;
+    int rc = make_plan(s, DBL_PASS_FWD, pl);
+    if (rc) return rc;
+    if (!x || !w || !y || !aligned16(x) || !aligned16(w) || !aligned16(y))
+        return set_error(DBL_ERR_INVALID, "conv_fwd: null or misaligned tensor");
+    if ((ch_sum == nullptr) != (ch_sumsq == nullptr))
+        return set_error(DBL_ERR_INVALID, "conv_fwd: ch_sum and ch_sumsq go together");
+    const bool stats = ch_sum != nullptr;
+    if (stats && (!ws || ws_bytes < plan_ws(pl)))
+        return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
+    CUtensorMap ta, tb;
+    const int P = out_dim(s->h, s->r, s->stride, s->pad);
+    (void)P;
+    if (pl.mode == kFwdC8) {
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -s->pad, s->pad - (s->r - 1), s->stride, 8, BM, false)))
+            return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * 8;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {8, (cuuint32_t)pl.BN};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, false))) return rc;
+    } else {
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, 64, BM, true)))
+            return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * s->c;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
+    }
+    uint8_t* wsb = static_cast<uint8_t*>(ws);
+    pl.p.out = y;
+    pl.p.stats = stats ? reinterpret_cast<float*>(wsb) : nullptr;
+    cudaStream_t st = as_stream(stream);
+    if ((rc = launch(pl, ta, tb, st))) return rc;
+    if (stats) {
+        double* lvl2 = reinterpret_cast<double*>(wsb + ((pl.ws_part + 255) / 256) * 256);
+        stats_reduce1_kernel<<<dim3((s->k + 31) / 32, pl.stat_chunks), 256, 0, st>>>(pl.p.stats, pl.p.m_tiles, s->k,
+                                                                                      lvl2);
+        if ((rc = launch_check("conv stats reduce1"))) return rc;
+        stats_reduce2_kernel<<<(s->k + 127) / 128, 128, 0, st>>>(lvl2, pl.stat_chunks, s->k, ch_sum, ch_sumsq);
+        if ((rc = launch_check("conv stats reduce2"))) return rc;
+    }
+    return DBL_OK;
+}
+
+int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void* dx, void* ws, size_t ws_bytes,
+                   void* stream)
+{
+    using namespace dbl;
+    (void)ws;
+    (void)ws_bytes;
+    Plan pl;
+    int rc = make_plan(s, DBL_PASS_DGRAD, pl);
+    if (rc) return rc;
+    if (!dy || !w || !dx || !aligned16(dy) || !aligned16(w) || !aligned16(dx))
+        return set_error(DBL_ERR_INVALID, "conv_dgrad: null or misaligned tensor");
+    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    CUtensorMap ta, tb;
+    // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
+    int lower, upper;
+    if (s->stride == 1) {
+        lower = -(s->r - 1 - s->pad);
+        upper = -s->pad;  // origin range [lower, H-1+lower] expressed against dy's extent P
+        upper = (s->h - 1 + lower) - (P - 1);
+    } else {
+        lower = 0;
+        upper = 0;
+    }
+    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, 1, 64, BM, true))) return rc;
+    // w viewed as [k][r*s][c]: inner c, then tap, then k
+    cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
+    cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
+    cuuint32_t box[3] = {64, 1, 64};
+    if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
+    pl.p.out = dx;
+    return launch(pl, ta, tb, as_stream(stream));
+}
+
+int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float* dw, int accumulate, void* ws,
+                   size_t ws_bytes, void* stream)
+{
+    using namespace dbl;
+    Plan pl;
+    int rc = make_plan(s, DBL_PASS_WGRAD, pl);
+    if (rc) return rc;
+    if (!x || !dy || !dw || !aligned16(x) || !aligned16(dy) || !aligned16(dw))
+        return set_error(DBL_ERR_INVALID, "conv_wgrad: null or misaligned tensor");
+    if (!ws || ws_bytes < plan_ws(pl))
+        return set_error(DBL_ERR_WORKSPACE, "conv_wgrad: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
+    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    CUtensorMap ta, tb;
+    const bool c8 = pl.mode == kWgradC8;
+    if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, c8 ? 8 : 64, 64,
+                         !c8)))
+        return rc;
+    cuuint64_t dims[2] = {(cuuint64_t)s->k, (cuuint64_t)s->n * P * Q};
+    cuuint64_t str[1] = {(cuuint64_t)s->k * 2};
+    cuuint32_t box[2] = {64, 64};
+    if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
+    pl.p.out = ws;
+    cudaStream_t st = as_stream(stream);
+    if ((rc = launch(pl, ta, tb, st))) return rc;
+    dim3 g((s->k + 31) / 32, (pl.p.M + 31) / 32);
+    wgrad_reduce_kernel<<<g, 256, 0, st>>>(static_cast<const float*>(ws), (int)pl.grid.y, pl.p.M, s->k, dw,
+                                           accumulate);
+    return launch_check("conv wgrad reduce");
+}
+
+int dbl_device_status(int32_t* status)
+{
+    using namespace dbl;
+    if (!status) return set_error(DBL_ERR_INVALID, "device_status: null");
+    int rc = cuda_check(cudaDeviceSynchronize(), "device_status sync");
+    if (rc) return rc;
+    int v = 0, zero = 0;
+    if ((rc = cuda_check(cudaMemcpyFromSymbol(&v, g_conv_status, sizeof(int)), "device_status read"))) return rc;
+    if ((rc = cuda_check(cudaMemcpyToSymbol(g_conv_status, &zero, sizeof(int)), "device_status clear"))) return rc;
+    *status = v;
+    return DBL_OK;
+}
+
+}  // extern "C"

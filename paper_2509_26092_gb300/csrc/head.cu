@@ -1,0 +1,345 @@
+// head.cu -- the small layers around the convolutions of ResNet-18
+// (Sec. 5.1.1): the ImageNet stem's 3x3/2 max pooling, and the head
+// (global average pooling -- Sec. 6 -- a fully connected layer and the
+// batch-mean softmax cross-entropy of Eq. 1), forward and backward.
+//
+// These are a few percent of a step's time: the max pool is a bandwidth
+// pass over the stem output, the head works on [n, 512] features.  The FC
+// products are done by a small tiled fp32 GEMM on the CUDA cores.
+#include <float.h>
+
+#include "dbl_internal.cuh"
+
+namespace {
+
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
+{
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 t = __bfloat1622float2(h[k]);
+        f[2 * k] = t.x;
+        f[2 * k + 1] = t.y;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&f)[8])
+{
+    uint4 v;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(f[2 * k], f[2 * k + 1]);
+    return v;
+}
+
+int grid_for(int64_t items, int threads, int per_sm = 8)
+{
+    int64_t b = (items + threads - 1) / threads;
+    const int64_t cap = (int64_t)dbl::sm_count() * per_sm;
+    if (b > cap) b = cap;
+    return (int)(b < 1 ? 1 : b);
+}
+
+// ----------------------------------------------------------------------------- max pool 3x3 / 2, pad 1
+__global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ x,
+                                                          __nv_bfloat16* __restrict__ y, uint8_t* __restrict__ arg,
+                                                          int n, int H, int W, int C, int P, int Q)
+{
+    const int groups = C / 8;
+    const int64_t total = (int64_t)n * P * Q * groups;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % groups);
+        int64_t pix = t / groups;
+        const int q = (int)(pix % Q);
+        pix /= Q;
+        const int p = (int)(pix % P);
+        const int b = (int)(pix / P);
+        float best[8];
+        uint8_t bi[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            best[k] = -INFINITY;
+            bi[k] = 0;
+        }
+        for (int r = 0; r < 3; ++r) {
+            const int h = 2 * p + r - 1;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < 3; ++s) {
+                const int w = 2 * q + s - 1;
+                if (w < 0 || w >= W) continue;
+                float f[8];
+                unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)b * H + h) * W + w) * C) + g), f);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    if (f[k] > best[k]) {  // strict: the first maximum in (r, s) order wins ties
+                        best[k] = f[k];
+                        bi[k] = (uint8_t)(r * 3 + s);
+                    }
+            }
+        }
+        const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
+        *reinterpret_cast<uint4*>(y + o) = pack8(best);
+        uint2 packed;
+        packed.x = bi[0] | (bi[1] << 8) | (bi[2] << 16) | ((uint32_t)bi[3] << 24);
+        packed.y = bi[4] | (bi[5] << 8) | (bi[6] << 16) | ((uint32_t)bi[7] << 24);
+        *reinterpret_cast<uint2*>(arg + o) = packed;
+    }
+}
+
+// Gather form: input (h,w) receives dy from every window (p,q) that contains
+// it and whose argmax is (h,w).  Windows are visited in (p, q) order.
+__global__ void __launch_bounds__(256)
+    maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dy, const __nv_bfloat16* __restrict__ dy2,
+                       const uint8_t* __restrict__ arg, __nv_bfloat16* __restrict__ dx, int n, int H, int W, int C,
+                       int P, int Q)
+{
+    const int groups = C / 8;
+    const int64_t total = (int64_t)n * H * W * groups;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % groups);
+        int64_t pix = t / groups;
+        const int w = (int)(pix % W);
+        pix /= W;
+        const int h = (int)(pix % H);
+        const int b = (int)(pix / H);
+        float acc[8] = {};
+        // windows p with 2p-1 <= h <= 2p+1, i.e. h/2 <= p <= (h+1)/2; tap r = h - 2p + 1
+        for (int p = h / 2; p <= min(P - 1, (h + 1) / 2); ++p) {
+            const int r = h - 2 * p + 1;
+            for (int q = w / 2; q <= min(Q - 1, (w + 1) / 2); ++q) {
+                const int s = w - 2 * q + 1;
+                const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
+                const uint2 a = *reinterpret_cast<const uint2*>(arg + o);
+                const uint8_t* ab = reinterpret_cast<const uint8_t*>(&a);
+                float f[8];
+                unpack8(__ldg(reinterpret_cast<const uint4*>(dy + o)), f);
+                if (dy2) {
+                    float f2[8];
+                    unpack8(__ldg(reinterpret_cast<const uint4*>(dy2 + o)), f2);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) f[k] += f2[k];
+                }
+                const uint8_t me = (uint8_t)(r * 3 + s);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    if (ab[k] == me) acc[k] += f[k];
+            }
+        }
+        *reinterpret_cast<uint4*>(dx + (((int64_t)b * H + h) * W + w) * C + 8 * g) = pack8(acc);
+    }
+}
+
+// ----------------------------------------------------------------------------- head
+// feat[n, c] = mean over hw of x[n, hw, c]
+__global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __restrict__ x, float* __restrict__ feat,
+                                                      int n, int hw, int C)
+{
+    const int groups = C / 8;
+    const int64_t total = (int64_t)n * groups;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % groups);
+        const int b = (int)(t / groups);
+        float acc[8] = {};
+        for (int i = 0; i < hw; ++i) {
+            float f[8];
+            unpack8(__ldg(reinterpret_cast<const uint4*>(x + ((int64_t)b * hw + i) * C) + g), f);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) acc[k] += f[k];
+        }
+        const float inv = 1.0f / (float)hw;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv;
+    }
+}
+
+// out[m, n] = sum_k A(m,k) * B(n,k) (+ bias[n]); A(m,k) = A[m*sam + k*sak], B(n,k) = B[n*sbn + k*sbk].
+constexpr int GT = 32;
+__global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__ A, int64_t sam, int64_t sak,
+                                                       const float* __restrict__ B, int64_t sbn, int64_t sbk,
+                                                       const float* __restrict__ bias, float* __restrict__ out,
+                                                       int64_t ldo, int M, int N, int K)
+{
+    __shared__ float As[GT][GT + 1], Bs[GT][GT + 1];
+    const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;  // 16x16 threads, 2x2 outputs each
+    const int m0 = blockIdx.y * GT, n0 = blockIdx.x * GT;
+    float acc[2][2] = {};
+    for (int k0 = 0; k0 < K; k0 += GT) {
+        for (int e = threadIdx.x; e < GT * GT; e += 256) {
+            const int i = e / GT, j = e % GT;
+            const int m = m0 + i, n = n0 + i, k = k0 + j;
+            As[i][j] = (m < M && k < K) ? A[m * sam + k * sak] : 0.f;
+            Bs[i][j] = (n < N && k < K) ? B[n * sbn + k * sbk] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int j = 0; j < GT; ++j) {
+            const float a0 = As[ty][j], a1 = As[ty + 16][j];
+            const float b0 = Bs[tx][j], b1 = Bs[tx + 16][j];
+            acc[0][0] = fmaf(a0, b0, acc[0][0]);
+            acc[0][1] = fmaf(a0, b1, acc[0][1]);
+            acc[1][0] = fmaf(a1, b0, acc[1][0]);
+            acc[1][1] = fmaf(a1, b1, acc[1][1]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const int m = m0 + ty + 16 * i, n = n0 + tx + 16 * j;
+            if (m < M && n < N) out[m * ldo + n] = acc[i][j] + (bias ? bias[n] : 0.f);
+        }
+}
+
+// One warp per row: loss_n = logsumexp(l) - l[label]; dl = (softmax - onehot)/n (in place).
+__global__ void softmax_ce_kernel(float* __restrict__ logits, const int32_t* __restrict__ labels, int n, int J,
+                                  float* __restrict__ row_loss)
+{
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
+    if (warp >= n) return;
+    float* l = logits + (int64_t)warp * J;
+    float mx = -FLT_MAX;
+    for (int j = lane; j < J; j += 32) mx = fmaxf(mx, l[j]);
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float z = 0.f;
+    for (int j = lane; j < J; j += 32) z += expf(l[j] - mx);
+    for (int o = 16; o; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+    const float lse = mx + logf(z);
+    const int lab = labels[warp];
+    if (lane == 0) row_loss[warp] = lse - l[lab];
+    const float invn = 1.0f / (float)n;
+    for (int j = lane; j < J; j += 32) l[j] = (expf(l[j] - lse) - (j == lab ? 1.f : 0.f)) * invn;
+}
+
+// loss = mean(row_loss) (one block, fixed order); db[j] = sum_n dl[n, j].
+__global__ void head_reduce_kernel(const float* __restrict__ row_loss, const float* __restrict__ dl, int n, int J,
+                                   float* __restrict__ loss, float* __restrict__ db)
+{
+    if (blockIdx.x == 0) {
+        __shared__ float red[256];
+        float s = 0.f;
+        for (int i = threadIdx.x; i < n; i += blockDim.x) s += row_loss[i];
+        red[threadIdx.x] = s;
+        __syncthreads();
+        for (int w = blockDim.x / 2; w; w >>= 1) {
+            if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+            __syncthreads();
+        }
+        if (threadIdx.x == 0) *loss = red[0] / (float)n;
+        return;
+    }
+    const int j = (blockIdx.x - 1) * blockDim.x + threadIdx.x;
+    if (j >= J) return;
+    float s = 0.f;
+    for (int i = 0; i < n; ++i) s += dl[(int64_t)i * J + j];
+    db[j] = s;
+}
+
+// dx[n, i, c] = df[n, c] / hw
+__global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, __nv_bfloat16* __restrict__ dx,
+                                                          int n, int hw, int C)
+{
+    const int groups = C / 8;
+    const int64_t total = (int64_t)n * hw * groups;
+    const float inv = 1.0f / (float)hw;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % groups);
+        const int b = (int)(t / groups / hw);
+        float f[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) f[k] = df[(int64_t)b * C + 8 * g + k] * inv;
+        reinterpret_cast<uint4*>(dx)[t] = pack8(f);
+    }
+}
+
+}  // namespace
+
+extern "C" {
+
+int dbl_maxpool_fwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* x, void* y, uint8_t* argmax, void* stream)
+{
+    using namespace dbl;
+    if (n < 0 || h <= 0 || w <= 0 || c <= 0 || !x || !y || !argmax)
+        return set_error(DBL_ERR_INVALID, "maxpool_fwd: bad arguments");
+    if (c % 8) return set_error(DBL_ERR_INVALID, "maxpool_fwd: channels must be a multiple of 8");
+    if (!aligned16(x) || !aligned16(y) || (reinterpret_cast<uintptr_t>(argmax) & 7))
+        return set_error(DBL_ERR_INVALID, "maxpool_fwd: misaligned pointer");
+    const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
+    if (n == 0) return DBL_OK;
+    maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q * (c / 8), 256), 256, 0, as_stream(stream)>>>(
+        static_cast<const __nv_bfloat16*>(x), static_cast<__nv_bfloat16*>(y), argmax, n, h, w, c, P, Q);
+    return launch_check("maxpool_fwd launch");
+}
+
+int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, const void* dy2,
+                    const uint8_t* argmax, void* dx, void* stream)
+{
+    using namespace dbl;
+    if (n < 0 || h <= 0 || w <= 0 || c <= 0 || !dy || !dx || !argmax)
+        return set_error(DBL_ERR_INVALID, "maxpool_bwd: bad arguments");
+    if (c % 8) return set_error(DBL_ERR_INVALID, "maxpool_bwd: channels must be a multiple of 8");
+    if (!aligned16(dy) || !aligned16(dx) || (dy2 && !aligned16(dy2)) || (reinterpret_cast<uintptr_t>(argmax) & 7))
+        return set_error(DBL_ERR_INVALID, "maxpool_bwd: misaligned pointer");
+    const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
+    if (n == 0) return DBL_OK;
+    maxpool_bwd_kernel<<<grid_for((int64_t)n * h * w * (c / 8), 256), 256, 0, as_stream(stream)>>>(
+        static_cast<const __nv_bfloat16*>(dy), static_cast<const __nv_bfloat16*>(dy2), argmax,
+        static_cast<__nv_bfloat16*>(dx), n, h, w, c, P, Q);
+    return launch_check("maxpool_bwd launch");
+}
+
+size_t dbl_head_workspace_bytes(int32_t n, int32_t c, int32_t classes)
+{
+    if (n <= 0 || c <= 0 || classes <= 0) return 0;
+    // feat [n,c], logits/dlogits [n,classes], df [n,c], row_loss [n]
+    const size_t f = (size_t)n * c * 2 + (size_t)n * classes + (size_t)n;
+    return (f * sizeof(float) + 255) / 256 * 256;
+}
+
+int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
+                     const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx,
+                     void* ws, size_t ws_bytes, void* stream)
+{
+    using namespace dbl;
+    if (n <= 0 || hw <= 0 || c <= 0 || classes <= 0 || !x || !fc_w || !fc_b || !labels || !loss || !dfc_w || !dfc_b ||
+        !dx)
+        return set_error(DBL_ERR_INVALID, "head_fwd_bwd: bad arguments");
+    if (c % 8 || !aligned16(x) || !aligned16(dx))
+        return set_error(DBL_ERR_INVALID, "head_fwd_bwd: channels must be a multiple of 8, tensors 16-byte aligned");
+    const size_t need = dbl_head_workspace_bytes(n, c, classes);
+    if (!ws || ws_bytes < need) return set_error(DBL_ERR_WORKSPACE, "head_fwd_bwd: workspace %zu < %zu", ws_bytes, need);
+    float* feat = static_cast<float*>(ws);
+    float* logits = feat + (size_t)n * c;
+    float* df = logits + (size_t)n * classes;
+    float* row_loss = df + (size_t)n * c;
+    cudaStream_t s = as_stream(stream);
+    int rc;
+    avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(x), feat, n,
+                                                                       hw, c);
+    if ((rc = launch_check("avgpool launch"))) return rc;
+    // logits = feat * W^T + b
+    dim3 g1((classes + GT - 1) / GT, (n + GT - 1) / GT);
+    gemm_f32_kernel<<<g1, 256, 0, s>>>(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c);
+    if ((rc = launch_check("fc fwd launch"))) return rc;
+    softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss);
+    if ((rc = launch_check("softmax_ce launch"))) return rc;
+    head_reduce_kernel<<<1 + (classes + 255) / 256, 256, 0, s>>>(row_loss, logits, n, classes, loss, dfc_b);
+    if ((rc = launch_check("head reduce launch"))) return rc;
+    // dW[j, c] = sum_n dl[n, j] feat[n, c]
+    dim3 g2((c + GT - 1) / GT, (classes + GT - 1) / GT);
+    gemm_f32_kernel<<<g2, 256, 0, s>>>(logits, 1, classes, feat, 1, c, nullptr, dfc_w, c, classes, c, n);
+    if ((rc = launch_check("fc dW launch"))) return rc;
+    // df[n, c] = sum_j dl[n, j] W[j, c]
+    dim3 g3((c + GT - 1) / GT, (n + GT - 1) / GT);
+    gemm_f32_kernel<<<g3, 256, 0, s>>>(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes);
+    if ((rc = launch_check("fc dX launch"))) return rc;
+    avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(df, static_cast<__nv_bfloat16*>(dx), n,
+                                                                                hw, c);
+    return launch_check("avgpool_bwd launch");
+}
+
+}  // extern "C"

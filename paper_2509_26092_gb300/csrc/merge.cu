@@ -1,0 +1,141 @@
+// merge.cu -- the parameter server's merge of the large- and small-batch
+// workers' pushes into the fp32 master weights (Sec. 3.4 with Eq. 1 and
+// momentum), plus the bf16 copy the workers pull next (Sec. 2.3).
+//
+// One pass over memory: per parameter it reads w, u, g_L, g_S (16 B) and
+// writes w, u (8 B) and the bf16 w16 (2 B), 26 B in all.  The kernel is
+// HBM-bound; it moves 4 parameters per thread per step with 128-bit loads,
+// streaming (evict-first) cache hints, and two steps in flight per thread.
+#include "dbl_internal.cuh"
+
+namespace {
+
+struct MergeArgs {
+    float* w;
+    float* u;
+    __nv_bfloat16* w16;
+    const float* gL;
+    const float* gS;
+    int64_t n;
+    float lr, mu, fL, fS;
+    int order;
+};
+
+// One momentum step per push, in the order the server receives them.
+__device__ __forceinline__ void merge_one(float& w, float& u, float gl, float gs, const MergeArgs& a, bool hasL,
+                                          bool hasS)
+{
+    if (a.order == 2) {
+        float g = 0.f;
+        if (hasL) g = a.fL * gl;
+        if (hasS) g = fmaf(a.fS, gs, g);
+        u = a.mu * u - a.lr * g;
+        w = w + u;
+        return;
+    }
+    const bool lfirst = a.order == 0;
+    const bool has1 = lfirst ? hasL : hasS, has2 = lfirst ? hasS : hasL;
+    const float g1 = lfirst ? gl : gs, g2 = lfirst ? gs : gl;
+    const float f1 = lfirst ? a.fL : a.fS, f2 = lfirst ? a.fS : a.fL;
+    if (has1) {
+        u = a.mu * u - a.lr * (f1 * g1);
+        w = w + u;
+    }
+    if (has2) {
+        u = a.mu * u - a.lr * (f2 * g2);
+        w = w + u;
+    }
+}
+
+__device__ __forceinline__ float4 ld_stream(const float* p) { return __ldcs(reinterpret_cast<const float4*>(p)); }
+
+__global__ void __launch_bounds__(256) ps_merge_kernel(MergeArgs a)
+{
+    const bool hasL = a.gL != nullptr, hasS = a.gS != nullptr;
+    const int64_t n4 = a.n >> 2;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    // two independent float4 groups per iteration keep more loads in flight
+    for (; i + stride < n4; i += 2 * stride) {
+        float4 w[2], u[2], gl[2] = {}, gs[2] = {};
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int64_t e = (i + k * stride) * 4;
+            w[k] = ld_stream(a.w + e);
+            u[k] = ld_stream(a.u + e);
+            if (hasL) gl[k] = ld_stream(a.gL + e);
+            if (hasS) gs[k] = ld_stream(a.gS + e);
+        }
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            merge_one(w[k].x, u[k].x, gl[k].x, gs[k].x, a, hasL, hasS);
+            merge_one(w[k].y, u[k].y, gl[k].y, gs[k].y, a, hasL, hasS);
+            merge_one(w[k].z, u[k].z, gl[k].z, gs[k].z, a, hasL, hasS);
+            merge_one(w[k].w, u[k].w, gl[k].w, gs[k].w, a, hasL, hasS);
+            const int64_t e = (i + k * stride) * 4;
+            __stcs(reinterpret_cast<float4*>(a.w + e), w[k]);
+            __stcs(reinterpret_cast<float4*>(a.u + e), u[k]);
+            if (a.w16) {
+                __nv_bfloat162 lo = __floats2bfloat162_rn(w[k].x, w[k].y);
+                __nv_bfloat162 hi = __floats2bfloat162_rn(w[k].z, w[k].w);
+                uint2 pk;
+                pk.x = *reinterpret_cast<uint32_t*>(&lo);
+                pk.y = *reinterpret_cast<uint32_t*>(&hi);
+                __stcs(reinterpret_cast<uint2*>(a.w16 + e), pk);
+            }
+        }
+    }
+    for (; i < n4; i += stride) {
+        const int64_t e = i * 4;
+        float4 w = ld_stream(a.w + e), u = ld_stream(a.u + e), gl = {}, gs = {};
+        if (hasL) gl = ld_stream(a.gL + e);
+        if (hasS) gs = ld_stream(a.gS + e);
+        merge_one(w.x, u.x, gl.x, gs.x, a, hasL, hasS);
+        merge_one(w.y, u.y, gl.y, gs.y, a, hasL, hasS);
+        merge_one(w.z, u.z, gl.z, gs.z, a, hasL, hasS);
+        merge_one(w.w, u.w, gl.w, gs.w, a, hasL, hasS);
+        __stcs(reinterpret_cast<float4*>(a.w + e), w);
+        __stcs(reinterpret_cast<float4*>(a.u + e), u);
+        if (a.w16) {
+            __nv_bfloat162 lo = __floats2bfloat162_rn(w.x, w.y);
+            __nv_bfloat162 hi = __floats2bfloat162_rn(w.z, w.w);
+            uint2 pk;
+            pk.x = *reinterpret_cast<uint32_t*>(&lo);
+            pk.y = *reinterpret_cast<uint32_t*>(&hi);
+            __stcs(reinterpret_cast<uint2*>(a.w16 + e), pk);
+        }
+    }
+    // scalar tail (n not a multiple of 4)
+    const int64_t t = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t < a.n && t < (n4 << 2) + 4) {
+        float w = a.w[t], u = a.u[t];
+        merge_one(w, u, hasL ? a.gL[t] : 0.f, hasS ? a.gS[t] : 0.f, a, hasL, hasS);
+        a.w[t] = w;
+        a.u[t] = u;
+        if (a.w16) a.w16[t] = __float2bfloat16_rn(w);
+    }
+}
+
+}  // namespace
+
+extern "C" int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const float* g_large, const float* g_small,
+                                       int64_t n, const dbl_merge_params* p, void* stream)
+{
+    using namespace dbl;
+    if (!w || !u || !p || n < 0) return set_error(DBL_ERR_INVALID, "ps_merge: null w/u/params or n < 0");
+    if (!g_large && !g_small) return set_error(DBL_ERR_INVALID, "ps_merge: no push (both gradients NULL)");
+    if (p->order < 0 || p->order > 2) return set_error(DBL_ERR_INVALID, "ps_merge: order must be 0, 1 or 2");
+    if (!aligned16(w) || !aligned16(u) || (g_large && !aligned16(g_large)) || (g_small && !aligned16(g_small)) ||
+        (w16_out && !aligned16(w16_out)))
+        return set_error(DBL_ERR_INVALID, "ps_merge: buffers must be 16-byte aligned");
+    if (n == 0) return DBL_OK;
+    MergeArgs a{w, u, reinterpret_cast<__nv_bfloat16*>(w16_out), g_large, g_small, n, p->lr, p->momentum,
+                p->f_large, p->f_small, p->order};
+    const int64_t n4 = n >> 2;
+    const int threads = 256;
+    int64_t want = (n4 + 2 * threads - 1) / (2 * threads);
+    const int64_t cap = (int64_t)sm_count() * 8;  // 8 resident 256-thread CTAs per SM
+    int blocks = (int)(want < cap ? (want < 1 ? 1 : want) : cap);
+    ps_merge_kernel<<<blocks, threads, 0, as_stream(stream)>>>(a);
+    return launch_check("ps_merge launch");
+}

@@ -1,0 +1,133 @@
+// resize.cu -- progressive resizing for the low-resolution sub-stages of
+// cyclic progressive learning (Sec. 4.1): bilinear downsampling with
+// half-pixel centres, fused with the cast to the network's input type and
+// the zero channel padding (3 colour channels -> 8, one 16-byte pixel).
+//
+// Taps are integer-exact: output j of an axis reads source rows
+// i0 = floor(num/den) and min(i0+1, in-1) with weight (num - i0*den)/den,
+// num = (2j+1)*in - out, den = 2*out.  When in == out this is a plain copy.
+#include "dbl_internal.cuh"
+
+namespace {
+
+struct Taps {
+    int32_t i0, i1;
+    float lam;
+};
+
+__device__ __forceinline__ Taps axis_taps(int32_t j, int32_t in, int32_t out)
+{
+    const int64_t num = (int64_t)(2 * j + 1) * in - out;
+    const int64_t den = 2 * (int64_t)out;
+    const int64_t a = num / den;
+    Taps t;
+    t.i0 = (int32_t)a;
+    t.i1 = (int32_t)(a + 1 < in ? a + 1 : in - 1);
+    t.lam = (float)(num - a * den) / (float)den;
+    return t;
+}
+
+template <typename Tin>
+__device__ __forceinline__ float ld_in(const Tin* p);
+template <>
+__device__ __forceinline__ float ld_in<float>(const float* p)
+{
+    return __ldg(p);
+}
+template <>
+__device__ __forceinline__ float ld_in<__nv_bfloat16>(const __nv_bfloat16* p)
+{
+    return __bfloat162float(*p);
+}
+
+// One thread per output pixel; channels 0..c-1 interpolated, c..cs-1 zeroed.
+template <typename Tin, typename Tout, int CMAX>
+__global__ void __launch_bounds__(256) resize_kernel(const Tin* __restrict__ in, Tout* __restrict__ out, int32_t n,
+                                                     int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
+                                                     int32_t cs)
+{
+    const int64_t total = (int64_t)n * ho * wo;
+    for (int64_t pix = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pix < total;
+         pix += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t x = (int32_t)(pix % wo);
+        const int64_t t = pix / wo;
+        const int32_t y = (int32_t)(t % ho);
+        const int32_t b = (int32_t)(t / ho);
+        const Taps ty = axis_taps(y, hi, ho), tx = axis_taps(x, wi, wo);
+        const Tin* base = in + (int64_t)b * hi * wi * c;
+        const Tin* pa = base + ((int64_t)ty.i0 * wi + tx.i0) * c;
+        const Tin* pb = base + ((int64_t)ty.i0 * wi + tx.i1) * c;
+        const Tin* pc = base + ((int64_t)ty.i1 * wi + tx.i0) * c;
+        const Tin* pd = base + ((int64_t)ty.i1 * wi + tx.i1) * c;
+        float v[CMAX];
+#pragma unroll
+        for (int ch = 0; ch < CMAX; ++ch) {
+            v[ch] = 0.f;
+            if (ch < c) {
+                const float top = (1.f - tx.lam) * ld_in(pa + ch) + tx.lam * ld_in(pb + ch);
+                const float bot = (1.f - tx.lam) * ld_in(pc + ch) + tx.lam * ld_in(pd + ch);
+                v[ch] = (1.f - ty.lam) * top + ty.lam * bot;
+            }
+        }
+        Tout* o = out + pix * cs;
+        if constexpr (sizeof(Tout) == 2 && CMAX == 8) {
+            if (cs == 8) {  // one 16-byte store per pixel
+                __nv_bfloat162 q[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) q[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+                *reinterpret_cast<uint4*>(o) = *reinterpret_cast<uint4*>(q);
+                continue;
+            }
+        }
+        for (int ch = 0; ch < cs; ++ch) {
+            const float val = ch < CMAX ? v[ch < CMAX ? ch : 0] : 0.f;
+            if constexpr (sizeof(Tout) == 2)
+                o[ch] = __float2bfloat16_rn(val);
+            else
+                o[ch] = val;
+        }
+    }
+}
+
+template <typename Tin, typename Tout>
+int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
+                  int32_t cs, cudaStream_t s)
+{
+    const int64_t total = (int64_t)n * ho * wo;
+    const int threads = 256;
+    int64_t blocks = (total + threads - 1) / threads;
+    const int64_t cap = (int64_t)dbl::sm_count() * 16;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    resize_kernel<Tin, Tout, 8><<<(int)blocks, threads, 0, s>>>(static_cast<const Tin*>(in), static_cast<Tout*>(out),
+                                                                n, hi, wi, c, ho, wo, cs);
+    return dbl::launch_check("progressive_resize launch");
+}
+
+}  // namespace
+
+extern "C" int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, int32_t h_in, int32_t w_in, int32_t c,
+                                      void* out, int out_dtype, int32_t h_out, int32_t w_out, int32_t c_out_stride,
+                                      void* stream)
+{
+    using namespace dbl;
+    if (!in || !out || n < 0 || h_in <= 0 || w_in <= 0 || c <= 0 || h_out <= 0 || w_out <= 0)
+        return set_error(DBL_ERR_INVALID, "progressive_resize: bad sizes or null pointer");
+    if (c > 8 || c_out_stride < c || c_out_stride > 8)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: supports 1..8 channels, stride c..8");
+    if (h_out > h_in || w_out > w_in)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: upsampling %dx%d -> %dx%d", h_in, w_in, h_out,
+                         w_out);
+    if ((in_dtype != DBL_F32 && in_dtype != DBL_BF16) || (out_dtype != DBL_F32 && out_dtype != DBL_BF16))
+        return set_error(DBL_ERR_INVALID, "progressive_resize: dtype must be DBL_F32 or DBL_BF16");
+    if (!aligned16(out)) return set_error(DBL_ERR_INVALID, "progressive_resize: output must be 16-byte aligned");
+    if (n == 0) return DBL_OK;
+    cudaStream_t s = as_stream(stream);
+    if (in_dtype == DBL_F32 && out_dtype == DBL_BF16)
+        return launch_resize<float, __nv_bfloat16>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+    if (in_dtype == DBL_F32 && out_dtype == DBL_F32)
+        return launch_resize<float, float>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+    if (in_dtype == DBL_BF16 && out_dtype == DBL_BF16)
+        return launch_resize<__nv_bfloat16, __nv_bfloat16>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+    return launch_resize<__nv_bfloat16, float>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+}

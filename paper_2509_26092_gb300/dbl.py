@@ -1,0 +1,221 @@
+"""ctypes binding of ``libdbl.so`` (see ``include/dbl.h``).
+
+Argument marshalling only: every function here calls the C entry point of
+the same name, passing device pointers, sizes and the CUDA stream.  Tensors
+may be given as torch tensors (their ``data_ptr()`` is passed) or as raw
+integer addresses.  A nonzero status raises ``DblError`` with the library's
+error text.  There is no fallback: if the library is not built, importing
+the functions fails.
+"""
+import ctypes
+import os
+
+from . import build_lib
+
+DBL_OK, DBL_ERR_INVALID, DBL_ERR_UNSUPPORTED, DBL_ERR_CUDA, DBL_ERR_TIMEOUT, DBL_ERR_WORKSPACE = 0, -1, -2, -3, -4, -5
+DBL_F32, DBL_BF16 = 0, 1
+DBL_PASS_FWD, DBL_PASS_DGRAD, DBL_PASS_WGRAD = 0, 1, 2
+
+
+class DblError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"libdbl error {code}: {msg}")
+        self.code = code
+
+
+class ConvShape(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int32) for f in ("n", "h", "w", "c", "k", "r", "s", "stride", "pad")]
+
+
+class BnShape(ctypes.Structure):
+    _fields_ = [("count", ctypes.c_int64), ("c", ctypes.c_int32), ("eps", ctypes.c_float), ("relu", ctypes.c_int32)]
+
+
+class MergeParams(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("momentum", ctypes.c_float), ("f_large", ctypes.c_float),
+                ("f_small", ctypes.c_float), ("order", ctypes.c_int32)]
+
+
+_lib = None
+_V = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_SZ = ctypes.c_size_t
+_D = ctypes.c_double
+
+
+def lib_path():
+    return build_lib.LIB
+
+
+def lib():
+    """Load libdbl.so (it must have been built by ``build_lib.build()``)."""
+    global _lib
+    if _lib is None:
+        path = build_lib.LIB
+        if not os.path.exists(path):
+            raise ImportError(f"{path} is missing: build it with paper_2509_26092_gb300.build_lib.build()")
+        L = ctypes.CDLL(path)
+        sig = {
+            "dbl_last_error": (ctypes.c_char_p, []),
+            "dbl_version": (ctypes.c_int, []),
+            "dbl_device_status": (ctypes.c_int, [ctypes.POINTER(_I32)]),
+            "dbl_conv_workspace_bytes": (_SZ, [ctypes.POINTER(ConvShape), ctypes.c_int]),
+            "dbl_conv_fwd": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _V, _V, _SZ, _V]),
+            "dbl_conv_dgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _SZ, _V]),
+            "dbl_conv_wgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, ctypes.c_int, _V, _SZ, _V]),
+            "dbl_bn_stats": (ctypes.c_int, [ctypes.POINTER(BnShape), _V, _V, _V, _V]),
+            "dbl_bn_relu_fused": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 10),
+            "dbl_bn_workspace_bytes": (_SZ, [ctypes.POINTER(BnShape)]),
+            "dbl_bn_relu_fused_bwd": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 12 + [_SZ, _V]),
+            "dbl_maxpool_fwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V]),
+            "dbl_maxpool_bwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V, _V]),
+            "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
+            "dbl_head_fwd_bwd": (ctypes.c_int, [_I32] * 4 + [_V] * 8 + [_V, _SZ, _V]),
+            "dbl_ps_dual_batch_merge": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams), _V]),
+            "dbl_progressive_resize": (ctypes.c_int, [_V, ctypes.c_int, _I32, _I32, _I32, _I32, _V, ctypes.c_int,
+                                                      _I32, _I32, _I32, _V]),
+            "dbl_resize_taps": (ctypes.c_int, [_I32, _I32, _V, _V, _V]),
+            "dbl_update_factor": (_D, [_D, _D, ctypes.c_int]),
+            "dbl_plan": (ctypes.c_int, [_D, _D, _I32, _I32, _D, _D, _D, ctypes.c_int] + [ctypes.POINTER(_D)] * 4),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(rc):
+    if rc != DBL_OK:
+        raise DblError(rc, lib().dbl_last_error().decode(errors="replace"))
+
+
+def dbl_last_error():
+    return lib().dbl_last_error().decode(errors="replace")
+
+
+def dbl_version():
+    return lib().dbl_version()
+
+
+def dbl_device_status():
+    """Synchronous: device-side status word (DBL_OK or DBL_ERR_TIMEOUT), then cleared."""
+    v = _I32(0)
+    _check(lib().dbl_device_status(ctypes.byref(v)))
+    return v.value
+
+
+def conv_shape(n, h, w, c, k, r, stride, pad):
+    return ConvShape(n, h, w, c, k, r, r, stride, pad)
+
+
+def dbl_conv_workspace_bytes(shape, pass_):
+    return lib().dbl_conv_workspace_bytes(ctypes.byref(shape), pass_)
+
+
+def dbl_conv_fwd(shape, x, w, y, ch_sum=None, ch_sumsq=None, ws=None, ws_bytes=0, stream=None):
+    _check(lib().dbl_conv_fwd(ctypes.byref(shape), _ptr(x), _ptr(w), _ptr(y), _ptr(ch_sum), _ptr(ch_sumsq), _ptr(ws),
+                              ws_bytes, _stream(stream)))
+
+
+def dbl_conv_dgrad(shape, dy, w, dx, ws=None, ws_bytes=0, stream=None):
+    _check(lib().dbl_conv_dgrad(ctypes.byref(shape), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws), ws_bytes,
+                                _stream(stream)))
+
+
+def dbl_conv_wgrad(shape, x, dy, dw, accumulate=False, ws=None, ws_bytes=0, stream=None):
+    _check(lib().dbl_conv_wgrad(ctypes.byref(shape), _ptr(x), _ptr(dy), _ptr(dw), int(bool(accumulate)), _ptr(ws),
+                                ws_bytes, _stream(stream)))
+
+
+def bn_shape(count, c, eps=1e-5, relu=True):
+    return BnShape(count, c, eps, int(bool(relu)))
+
+
+def dbl_bn_stats(shape, y, ch_sum, ch_sumsq, stream=None):
+    _check(lib().dbl_bn_stats(ctypes.byref(shape), _ptr(y), _ptr(ch_sum), _ptr(ch_sumsq), _stream(stream)))
+
+
+def dbl_bn_relu_fused(shape, y, ch_sum, ch_sumsq, gamma, beta, residual, out, save_mean, save_invstd, stream=None):
+    _check(lib().dbl_bn_relu_fused(ctypes.byref(shape), _ptr(y), _ptr(ch_sum), _ptr(ch_sumsq), _ptr(gamma),
+                                   _ptr(beta), _ptr(residual), _ptr(out), _ptr(save_mean), _ptr(save_invstd),
+                                   _stream(stream)))
+
+
+def dbl_bn_workspace_bytes(shape):
+    return lib().dbl_bn_workspace_bytes(ctypes.byref(shape))
+
+
+def dbl_bn_relu_fused_bwd(shape, dout, dout2, y, out, gamma, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
+                          ws, ws_bytes, stream=None):
+    _check(lib().dbl_bn_relu_fused_bwd(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out), _ptr(gamma),
+                                       _ptr(save_mean), _ptr(save_invstd), _ptr(dy), _ptr(dresidual), _ptr(dgamma),
+                                       _ptr(dbeta), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def dbl_maxpool_fwd(n, h, w, c, x, y, argmax, stream=None):
+    _check(lib().dbl_maxpool_fwd(n, h, w, c, _ptr(x), _ptr(y), _ptr(argmax), _stream(stream)))
+
+
+def dbl_maxpool_bwd(n, h, w, c, dy, dy2, argmax, dx, stream=None):
+    _check(lib().dbl_maxpool_bwd(n, h, w, c, _ptr(dy), _ptr(dy2), _ptr(argmax), _ptr(dx), _stream(stream)))
+
+
+def dbl_head_workspace_bytes(n, c, classes):
+    return lib().dbl_head_workspace_bytes(n, c, classes)
+
+
+def dbl_head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, loss, dfc_w, dfc_b, dx, ws, ws_bytes, stream=None):
+    _check(lib().dbl_head_fwd_bwd(n, hw, c, classes, _ptr(x), _ptr(fc_w), _ptr(fc_b), _ptr(labels), _ptr(loss),
+                                  _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def dbl_ps_dual_batch_merge(w, u, w16_out, g_large, g_small, n, lr, momentum, f_large, f_small, order=0,
+                            stream=None):
+    p = MergeParams(lr, momentum, f_large, f_small, order)
+    _check(lib().dbl_ps_dual_batch_merge(_ptr(w), _ptr(u), _ptr(w16_out), _ptr(g_large), _ptr(g_small), n,
+                                         ctypes.byref(p), _stream(stream)))
+
+
+def dbl_progressive_resize(inp, in_dtype, n, h_in, w_in, c, out, out_dtype, h_out, w_out, c_out_stride, stream=None):
+    _check(lib().dbl_progressive_resize(_ptr(inp), in_dtype, n, h_in, w_in, c, _ptr(out), out_dtype, h_out, w_out,
+                                        c_out_stride, _stream(stream)))
+
+
+def dbl_resize_taps(n_in, n_out):
+    import numpy as np
+    i0 = np.empty(n_out, np.int32)
+    i1 = np.empty(n_out, np.int32)
+    lam = np.empty(n_out, np.float32)
+    _check(lib().dbl_resize_taps(n_in, n_out, i0.ctypes.data, i1.ctypes.data, lam.ctypes.data))
+    return i0, i1, lam
+
+
+def dbl_update_factor(d_small, d_large, sqrt_scheme=False):
+    return lib().dbl_update_factor(d_small, d_large, int(bool(sqrt_scheme)))
+
+
+def dbl_plan(k, d, n_small, n_large, a, b, batch_large, sqrt_scheme=False):
+    out = [_D(0) for _ in range(4)]
+    _check(lib().dbl_plan(k, d, n_small, n_large, a, b, batch_large, int(bool(sqrt_scheme)),
+                          *[ctypes.byref(o) for o in out]))
+    return tuple(o.value for o in out)

@@ -1,0 +1,49 @@
+"""Helpers shared by the GPU parity tests (no arithmetic of the method here)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2509_26092_gb300 import build_lib
+
+
+def need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def load_dbl():
+    need_gpu()
+    build_lib.build()
+    from paper_2509_26092_gb300 import dbl
+    return dbl
+
+
+def to_bf16_dev(a):
+    """numpy float -> bf16 CUDA tensor (round to nearest even)."""
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).cuda()
+
+
+def to_f32_dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).cuda()
+
+
+def host(t):
+    """CUDA tensor -> float64 numpy."""
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def bf16_values(a):
+    """The float64 values of a after rounding to bf16 (the inputs both sides see)."""
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).double().numpy()
+
+
+def ws(nbytes):
+    return torch.empty(max(int(nbytes), 16), dtype=torch.uint8, device="cuda")
+
+
+def rng(seed):
+    return np.random.default_rng(seed)
+
+
+def check_status(D):
+    assert D.dbl_device_status() == D.DBL_OK

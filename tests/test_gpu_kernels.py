@@ -1,0 +1,273 @@
+"""GPU parity of each C-ABI kernel against the fp64 oracle, on seeded inputs
+that both sides see identically (bf16-rounded where the GPU reads bf16).
+
+Tolerances (max|gpu - ref| / max|ref|): 1e-2 for bf16-input / fp32-accumulate
+convolutions and the bf16 outputs of BatchNorm and the head; 1e-6 for the
+fp32 merge; resize taps bit-exact and values within one bf16 ulp.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from conftest import max_norm_rel
+from gpu_common import bf16_values, check_status, host, load_dbl, rng, to_bf16_dev, to_f32_dev, ws
+
+pytestmark = pytest.mark.gpu
+
+CONV_TOL = 1e-2
+MERGE_TOL = 1e-6
+
+
+@pytest.fixture(scope="module")
+def D():
+    return load_dbl()
+
+
+# ----------------------------------------------------------------------------- merge
+@pytest.mark.parametrize("n", [36_864, 1_001, 11_220_132])
+@pytest.mark.parametrize("order", [0, 1, 2])
+def test_merge_matches_oracle(D, n, order):
+    g = rng(n + order)
+    w0 = g.standard_normal(n).astype(np.float32)
+    u0 = (0.01 * g.standard_normal(n)).astype(np.float32)
+    gl = (0.1 * g.standard_normal(n)).astype(np.float32)
+    gs = (0.1 * g.standard_normal(n)).astype(np.float32)
+    w, u, gL, gS = (to_f32_dev(a) for a in (w0, u0, gl, gs))
+    w16 = torch.empty(n, dtype=torch.bfloat16, device="cuda")
+    D.dbl_ps_dual_batch_merge(w, u, w16, gL, gS, n, 0.2, 0.9, 1.0, 19 / 21, order)
+    rw, ru = orc.ps_merge(w0, u0, gl, gs, 0.2, 0.9, 1.0, 19 / 21, order)
+    assert max_norm_rel(host(w), rw) <= MERGE_TOL
+    assert max_norm_rel(host(u), ru) <= MERGE_TOL
+    # the pulled copy is the bf16 rounding of the new fp32 master weights
+    assert torch.equal(w16, w.to(torch.bfloat16))
+    check_status(D)
+
+
+def test_merge_single_push_and_no_w16(D):
+    n = 4099
+    g = rng(7)
+    w0, u0, gl = (g.standard_normal(n).astype(np.float32) for _ in range(3))
+    w, u, gL = to_f32_dev(w0), to_f32_dev(u0), to_f32_dev(gl)
+    D.dbl_ps_dual_batch_merge(w, u, None, gL, None, n, 0.1, 0.9, 1.0, 0.5, 0)
+    rw, ru = orc.ps_merge(w0, u0, gl, None, 0.1, 0.9, 1.0, 0.5, 0)
+    assert max_norm_rel(host(w), rw) <= MERGE_TOL
+    assert max_norm_rel(host(u), ru) <= MERGE_TOL
+
+
+# ----------------------------------------------------------------------------- resize
+@pytest.mark.parametrize("n,hin,hout", [(3, 32, 16), (3, 32, 24), (2, 32, 32), (2, 224, 128), (2, 224, 160),
+                                        (1, 17, 5)])
+def test_resize_matches_oracle(D, n, hin, hout):
+    x = rng(hin + hout).standard_normal((n, hin, hin, 3)).astype(np.float32)
+    ref = orc.bilinear_resize(x, hout, hout)
+    xd = to_f32_dev(x)
+    out = torch.full((n, hout, hout, 8), 7.0, dtype=torch.bfloat16, device="cuda")
+    D.dbl_progressive_resize(xd, D.DBL_F32, n, hin, hin, 3, out, D.DBL_BF16, hout, hout, 8)
+    got = host(out)
+    assert np.all(got[..., 3:] == 0.0)
+    # within one bf16 ulp of the exact value
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
+    assert np.all(np.abs(got[..., :3] - ref) <= ulp + 1e-30)
+    out32 = torch.empty((n, hout, hout, 3), dtype=torch.float32, device="cuda")
+    D.dbl_progressive_resize(xd, D.DBL_F32, n, hin, hin, 3, out32, D.DBL_F32, hout, hout, 3)
+    assert max_norm_rel(host(out32), ref) <= 1e-6
+
+
+# ----------------------------------------------------------------------------- BatchNorm
+@pytest.mark.parametrize("count,C,relu,res", [(4096, 64, True, True), (1000, 128, True, False),
+                                              (777, 512, False, False), (2048, 256, True, True)])
+def test_bn_fwd_bwd_match_oracle(D, count, C, relu, res):
+    g = rng(count + C)
+    y = bf16_values(g.standard_normal((count, C)) * 2.0 + 0.5)
+    r = bf16_values(g.standard_normal((count, C))) if res else None
+    gamma = (1.0 + 0.2 * g.standard_normal(C)).astype(np.float32)
+    beta = (0.1 * g.standard_normal(C)).astype(np.float32)
+    yd = to_bf16_dev(y)
+    s1 = torch.empty(C, device="cuda")
+    s2 = torch.empty(C, device="cuda")
+    shape = D.bn_shape(count, C, 1e-5, relu)
+    D.dbl_bn_stats(shape, yd, s1, s2)
+    np.testing.assert_allclose(host(s1), y.sum(0), rtol=1e-4, atol=1e-2)
+    out = torch.empty((count, C), dtype=torch.bfloat16, device="cuda")
+    mean = torch.empty(C, device="cuda")
+    istd = torch.empty(C, device="cuda")
+    D.dbl_bn_relu_fused(shape, yd, s1, s2, to_f32_dev(gamma), to_f32_dev(beta), to_bf16_dev(r) if res else None, out,
+                        mean, istd)
+    ro, rm, ri = orc.bn_fwd(y, gamma, beta, 1e-5, res=r, relu=relu)
+    assert max_norm_rel(host(out), ro) <= CONV_TOL
+    np.testing.assert_allclose(host(mean), rm, rtol=1e-5, atol=1e-5)
+    np.testing.assert_allclose(host(istd), ri, rtol=1e-4)
+    # backward, with a second upstream gradient
+    dout = bf16_values(g.standard_normal((count, C)))
+    dout2 = bf16_values(g.standard_normal((count, C)))
+    out_h = host(out)
+    dy = torch.empty_like(out)
+    dres = torch.empty_like(out)
+    dg = torch.empty(C, device="cuda")
+    db = torch.empty(C, device="cuda")
+    wsb = D.dbl_bn_workspace_bytes(shape)
+    D.dbl_bn_relu_fused_bwd(shape, to_bf16_dev(dout), to_bf16_dev(dout2), yd, out, to_f32_dev(gamma), mean, istd, dy,
+                            dres, dg, db, ws(wsb), wsb)
+    rdy, rdg, rdb, rdres = orc.bn_bwd(dout, out_h, y, gamma, host(mean), host(istd), relu=relu, dout2=dout2,
+                                      want_dres=True)
+    assert max_norm_rel(host(dy), rdy) <= CONV_TOL
+    assert max_norm_rel(host(dg), rdg) <= 1e-4
+    assert max_norm_rel(host(db), rdb) <= 1e-4
+    assert max_norm_rel(host(dres), rdres) <= CONV_TOL
+    check_status(D)
+
+
+# ----------------------------------------------------------------------------- max pool
+@pytest.mark.parametrize("n,h,w,c,zeros", [(2, 9, 10, 64, False), (2, 16, 16, 64, True), (1, 112, 112, 64, True)])
+def test_maxpool_matches_oracle(D, n, h, w, c, zeros):
+    g = rng(h * w + c)
+    x = g.standard_normal((n, h, w, c))
+    if zeros:  # post-ReLU-like input: many exact ties at zero
+        x = np.maximum(x, 0.0)
+    x = bf16_values(x)
+    ry, rarg = orc.maxpool_fwd(x, 3, 2, 1)
+    P, Q = ry.shape[1], ry.shape[2]
+    y = torch.empty((n, P, Q, c), dtype=torch.bfloat16, device="cuda")
+    arg = torch.empty((n, P, Q, c), dtype=torch.uint8, device="cuda")
+    xd = to_bf16_dev(x)
+    D.dbl_maxpool_fwd(n, h, w, c, xd, y, arg)
+    np.testing.assert_array_equal(host(y), ry)
+    np.testing.assert_array_equal(arg.cpu().numpy().astype(np.int32), rarg)
+    dy = bf16_values(g.standard_normal(ry.shape))
+    dy2 = bf16_values(g.standard_normal(ry.shape))
+    dx = torch.empty_like(xd)
+    D.dbl_maxpool_bwd(n, h, w, c, to_bf16_dev(dy), to_bf16_dev(dy2), arg, dx)
+    rdx = orc.maxpool_bwd(dy + dy2, rarg, x.shape, 3, 2, 1)
+    assert max_norm_rel(host(dx), rdx) <= CONV_TOL
+
+
+# ----------------------------------------------------------------------------- head
+@pytest.mark.parametrize("n,hw,c,classes", [(4, 16, 64, 10), (8, 49, 512, 1000), (256, 16, 512, 100)])
+def test_head_matches_oracle(D, n, hw, c, classes):
+    g = rng(n * classes)
+    x = bf16_values(np.maximum(g.standard_normal((n, hw, c)), 0))
+    W = (0.05 * g.standard_normal((classes, c))).astype(np.float32)
+    b = (0.01 * g.standard_normal(classes)).astype(np.float32)
+    lab = g.integers(0, classes, n).astype(np.int32)
+    loss = torch.empty(1, device="cuda")
+    dW = torch.empty((classes, c), device="cuda")
+    db = torch.empty(classes, device="cuda")
+    dx = torch.empty((n, hw, c), dtype=torch.bfloat16, device="cuda")
+    wsb = D.dbl_head_workspace_bytes(n, c, classes)
+    D.dbl_head_fwd_bwd(n, hw, c, classes, to_bf16_dev(x), to_f32_dev(W), to_f32_dev(b),
+                       torch.from_numpy(lab).cuda(), loss, dW, db, dx, ws(wsb), wsb)
+    x4 = x.reshape(n, 1, hw, c)
+    feat = orc.avgpool_fwd(x4)
+    logits = orc.fc_fwd(feat, W, b)
+    rl, dl = orc.softmax_ce(logits, lab)
+    rdW, rdb, rdf = orc.fc_bwd(dl, feat, W)
+    rdx = orc.avgpool_bwd(rdf, x4.shape).reshape(n, hw, c)
+    assert abs(loss.item() - rl) <= 1e-5 * abs(rl)
+    assert max_norm_rel(host(dW), rdW) <= 1e-4
+    assert max_norm_rel(host(db), rdb) <= 1e-4
+    assert max_norm_rel(host(dx), rdx) <= CONV_TOL
+
+
+# ----------------------------------------------------------------------------- convolutions
+FWD_CASES = [  # n, h, w, c, k, r, stride, pad
+    (2, 8, 8, 64, 64, 3, 1, 1),      # exactly one 128-row tile
+    (3, 7, 9, 64, 128, 3, 1, 1),     # ragged last tile, BN = 128
+    (2, 8, 8, 128, 64, 3, 2, 1),     # stride 2, two channel blocks
+    (2, 8, 8, 64, 128, 1, 2, 0),     # 1x1 stride-2 projection
+    (8, 16, 16, 64, 64, 3, 1, 1),    # the single-block workload (batch 8, 16x16)
+    (2, 6, 6, 8, 64, 3, 1, 1),       # CIFAR stem, 8 padded channels
+    (2, 20, 20, 8, 64, 7, 2, 3),     # ImageNet stem, 8 padded channels
+    (1, 4, 4, 256, 256, 3, 1, 1),    # deep layer, small image
+]
+
+
+def _conv_inputs(case, seed):
+    n, h, w, c, k, r, st, pad = case
+    g = rng(seed)
+    x = g.standard_normal((n, h, w, c))
+    if c == 8:
+        x[..., 3:] = 0.0  # 3 colour channels padded to 8
+    wt = g.standard_normal((k, r, r, c)) * np.sqrt(2.0 / (r * r * c))
+    return bf16_values(x), bf16_values(wt)
+
+
+@pytest.mark.parametrize("case", FWD_CASES)
+def test_conv_fwd_matches_oracle(D, case):
+    n, h, w, c, k, r, st, pad = case
+    x, wt = _conv_inputs(case, 11)
+    ref = orc.conv2d_fwd(x, wt, st, pad)
+    P, Q = ref.shape[1], ref.shape[2]
+    shape = D.conv_shape(n, h, w, c, k, r, st, pad)
+    y = torch.full((n, P, Q, k), float("nan"), dtype=torch.bfloat16, device="cuda")
+    s1 = torch.empty(k, device="cuda")
+    s2 = torch.empty(k, device="cuda")
+    wsb = D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_FWD)
+    D.dbl_conv_fwd(shape, to_bf16_dev(x), to_bf16_dev(wt), y, s1, s2, ws(wsb), wsb)
+    got = host(y)
+    assert np.all(np.isfinite(got))
+    assert max_norm_rel(got, ref) <= CONV_TOL
+    # channel statistics are those of the stored outputs
+    flat = got.reshape(-1, k)
+    np.testing.assert_allclose(host(s1), flat.sum(0), rtol=1e-4, atol=1e-3 * np.abs(flat).max())
+    np.testing.assert_allclose(host(s2), (flat ** 2).sum(0), rtol=1e-4, atol=1e-3)
+    check_status(D)
+
+
+DGRAD_CASES = [
+    (2, 8, 8, 64, 64, 3, 1, 1),
+    (3, 6, 10, 64, 64, 3, 1, 1),     # ragged
+    (2, 8, 8, 128, 64, 3, 2, 1),     # stride-2 phases, BN = 128
+    (2, 8, 8, 64, 128, 1, 2, 0),     # 1x1 stride 2: three phases are all zero
+    (2, 16, 16, 64, 128, 3, 2, 1),
+    (1, 4, 4, 256, 256, 3, 1, 1),
+]
+
+
+@pytest.mark.parametrize("case", DGRAD_CASES)
+def test_conv_dgrad_matches_oracle(D, case):
+    n, h, w, c, k, r, st, pad = case
+    x, wt = _conv_inputs(case, 12)
+    P, Q = orc.out_dim(h, r, st, pad), orc.out_dim(w, r, st, pad)
+    dy = bf16_values(rng(13).standard_normal((n, P, Q, k)))
+    ref = orc.conv2d_dgrad(dy, wt, x.shape, st, pad)
+    shape = D.conv_shape(n, h, w, c, k, r, st, pad)
+    dx = torch.full((n, h, w, c), float("nan"), dtype=torch.bfloat16, device="cuda")
+    D.dbl_conv_dgrad(shape, to_bf16_dev(dy), to_bf16_dev(wt), dx)
+    got = host(dx)
+    assert np.all(np.isfinite(got))
+    assert max_norm_rel(got, ref) <= CONV_TOL
+    check_status(D)
+
+
+WGRAD_CASES = [
+    (2, 8, 8, 64, 64, 3, 1, 1),
+    (5, 7, 7, 64, 64, 3, 1, 1),      # ragged pixel count
+    (2, 8, 8, 128, 64, 3, 2, 1),
+    (2, 8, 8, 64, 128, 1, 2, 0),
+    (2, 6, 6, 8, 64, 3, 1, 1),       # CIFAR stem
+    (2, 20, 20, 8, 64, 7, 2, 3),     # ImageNet stem
+    (1, 4, 4, 256, 256, 3, 1, 1),
+    (8, 16, 16, 64, 64, 3, 1, 1),
+]
+
+
+@pytest.mark.parametrize("case", WGRAD_CASES)
+def test_conv_wgrad_matches_oracle(D, case):
+    n, h, w, c, k, r, st, pad = case
+    x, wt = _conv_inputs(case, 14)
+    P, Q = orc.out_dim(h, r, st, pad), orc.out_dim(w, r, st, pad)
+    dy = bf16_values(rng(15).standard_normal((n, P, Q, k)))
+    ref = orc.conv2d_wgrad(x, dy, wt.shape, st, pad)
+    shape = D.conv_shape(n, h, w, c, k, r, st, pad)
+    wsb = D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_WGRAD)
+    dw = torch.full((k, r, r, c), float("nan"), dtype=torch.float32, device="cuda")
+    xd, dyd = to_bf16_dev(x), to_bf16_dev(dy)
+    D.dbl_conv_wgrad(shape, xd, dyd, dw, False, ws(wsb), wsb)
+    got = host(dw)
+    assert np.all(np.isfinite(got))
+    assert max_norm_rel(got, ref) <= CONV_TOL
+    # accumulate mode adds onto what is there
+    D.dbl_conv_wgrad(shape, xd, dyd, dw, True, ws(wsb), wsb)
+    assert max_norm_rel(host(dw), 2 * ref) <= CONV_TOL
+    check_status(D)
