@@ -1,0 +1,457 @@
+#!/usr/bin/env python
+"""Benchmark of the ResNet-18 hybrid dual-batch training step on GB300.
+
+Default workload (``imagenet_hybrid``): ImageNet-shaped ResNet-18 (7x7/2 stem,
+3x3/2 max pool, 1000 classes), synthetic 224x224 images resized by the
+library's bilinear downsampler to the cyclic-progressive sub-stage
+resolutions 128, 160 and 224; at each resolution a large-batch worker
+(batch 512) and a small-batch worker (batch 128) run concurrently on two CUDA
+streams and the parameter server merges both pushes into the fp32 master
+weights (11.7 M parameters) with the model-update factor f_S = 19/21.
+
+One benchmark step is one dual-batch iteration at each of the three
+resolutions (1920 images).  ``value`` is images/s over the whole job (all
+ranks); ``per_resolution`` breaks it down.  Each rank runs an independent
+replica (the path has no cross-GPU exchange on one box), so scaling is weak.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+"""
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "ResNet-18 train-step images/s per resolution; conv TFLOP/s vs bf16 peak"
+
+CONFIGS = {
+    # variant, classes, native resolution, sub-stage resolutions, large / small batch per stage
+    "imagenet_hybrid": dict(variant="imagenet", classes=1000, native=224, stages=(128, 160, 224),
+                            large=(512, 512, 512), small=(128, 128, 128),
+                            desc="ImageNet-shaped ResNet-18 hybrid: 224 px images resized to 128/160/224, "
+                                 "large worker 512 + small worker 128 on two streams, PS merge each iteration"),
+    "cifar_hybrid": dict(variant="cifar", classes=100, native=32, stages=(16, 24, 32), large=(1024, 512, 256),
+                         small=(256, 128, 64),
+                         desc="CIFAR-shaped ResNet-18 cyclic progressive sweep 16/24/32 px, dual batch, PS merge"),
+    "cifar_step": dict(variant="cifar", classes=100, native=32, stages=(32,), large=(256,), small=(None,),
+                       desc="CIFAR-shaped ResNet-18, one train step at 32x32, batch 256, single push"),
+    "imagenet_step": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(256,), small=(None,),
+                          desc="ImageNet-shaped ResNet-18, one train step at 224x224, batch 256, single push"),
+    "imagenet_small": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(32,), small=(8,),
+                           desc="small ImageNet-shaped dual-batch iteration for profiling"),
+}
+DEFAULT_CONFIG = "imagenet_hybrid"
+F_SMALL = 19.0 / 21.0  # d_S/d_L for one large and one small worker at k = 1.05 (Eqs. 4-6)
+LR, MOMENTUM = 0.2, 0.9
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", 0)), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _conv_source_hash():
+    h = hashlib.sha256()
+    for name in ("conv.cu", "dbl_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2509_26092_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def _traffic_record(config):
+    """DRAM bytes of the conv kernel per step from a committed ncu summary, if it is current."""
+    path = os.path.join(ROOT, "profiles", "conv_igemm_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        if rec.get("source_hash") != _conv_source_hash() or rec.get("config") != config:
+            return None
+        return rec.get("dram_bytes_per_launch_avg")
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ------------------------------------------------------------------------------------------ oracle timing
+def _oracle_setup(cfg):
+    import numpy as np
+
+    import oracle as orc
+    from oracle import resnet18 as OR
+    from paper_2509_26092_gb300 import synth
+
+    table = OR.layer_table(cfg["variant"], cfg["classes"])
+    params = {k: v.astype(np.float64) for k, v in synth.params(table, seed=0).items()}
+    vel = {k: np.zeros_like(v) for k, v in params.items()}
+    img = synth.images(3, cfg["native"], cfg["native"], 3, seed=0).astype(np.float64)
+    lab = synth.labels(3, cfg["classes"], seed=0)
+    orc.lib()
+    return dict(params=params, vel=vel, img=img, lab=lab)
+
+
+def _oracle_iteration(cfg, st, res):
+    """One dual-batch iteration of the fp64 oracle at resolution res: large batch 2, small batch 1."""
+    from oracle import resnet18 as OR
+    t0 = time.perf_counter()
+    st["params"], st["vel"], *_ = OR.dual_batch_iteration(st["params"], st["vel"], st["img"][:2], st["lab"][:2],
+                                                          st["img"][2:], st["lab"][2:], res, cfg["variant"], LR,
+                                                          MOMENTUM, 1.0, F_SMALL, order=0)
+    return 3, time.perf_counter() - t0
+
+
+def time_oracle(cfg):
+    """The fp64 CPU oracle on a bounded sample of the workload, timed on this
+    host's cores: one dual-batch iteration (large batch 2, small batch 1) at
+    each sub-stage resolution."""
+    st = _oracle_setup(cfg)
+    images, secs = 0, 0.0
+    for res in cfg["stages"]:
+        n, dt = _oracle_iteration(cfg, st, res)
+        images += n
+        secs += dt
+    sample = (f"one dual-batch iteration (large batch 2, small batch 1) at each of "
+              f"{', '.join(str(r) for r in cfg['stages'])} px, {cfg['variant']} ResNet-18, fp64")
+    return images / secs, secs, images, sample
+
+
+def run_reference(args, cfg):
+    """The reference arm: the fp64 CPU oracle, as it stands, on this host's cores.
+    Each step is one dual-batch iteration (large batch 2, small batch 1) at the
+    next sub-stage resolution of the cycle."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    st = _oracle_setup(cfg)
+    stages = cfg["stages"]
+    images, secs = 0, 0.0
+    for i in range(args.warmup + args.steps):
+        n, dt = _oracle_iteration(cfg, st, stages[i % len(stages)])
+        if i >= args.warmup:
+            images += n
+            secs += dt
+    value = images / secs
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    sample = (f"{args.steps} dual-batch iterations (large batch 2, small batch 1) cycling through "
+              f"{', '.join(str(r) for r in stages)} px, {cfg['variant']} ResNet-18, fp64 CPU oracle")
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "images/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1000.0 * secs / args.steps, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.config, "description": cfg["desc"], "reference": "fp64 CPU oracle"},
+            "cpu_baseline": {"value": round(value, 4), "unit": "images/s", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------------------------------ GPU arm
+def build_pipeline(cfg, device):
+    import torch
+
+    from paper_2509_26092_gb300 import dbl as D
+    from paper_2509_26092_gb300 import resnet18 as R
+    from paper_2509_26092_gb300 import synth
+
+    spec = R.ResNet18Spec(cfg["variant"], cfg["classes"])
+    server = R.ServerState(spec, synth.params(spec.table(), seed=0), synth.momentum_state(spec.table(), 0.0, seed=0))
+    bl_max = max(cfg["large"])
+    bs_max = max([b for b in cfg["small"] if b] or [0])
+    nat = cfg["native"]
+    host_l = torch.from_numpy(synth.images(bl_max, nat, nat, 3, seed=1, name="large")).pin_memory()
+    host_s = torch.from_numpy(synth.images(bs_max, nat, nat, 3, seed=1, name="small")).pin_memory() if bs_max else None
+    lab_l = torch.from_numpy(synth.labels(bl_max, cfg["classes"], seed=1, name="large")).pin_memory()
+    lab_s = torch.from_numpy(synth.labels(bs_max, cfg["classes"], seed=1, name="small")).pin_memory() if bs_max else None
+    stages = []
+    for res, bl, bs in zip(cfg["stages"], cfg["large"], cfg["small"]):
+        large = R.Worker(spec, bl, res, device)
+        small = R.Worker(spec, bs, res, device) if bs else None
+        it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_large=1.0, f_small=F_SMALL)
+        it.set_inputs(host_l[:bl].to(device), lab_l[:bl].to(device),
+                      host_s[:bs].to(device) if bs else None, lab_s[:bs].to(device) if bs else None)
+        n0 = D.dbl_kernel_launches()
+        it.capture()
+        launches = D.dbl_kernel_launches() - n0
+        # capture() enqueues one eager warm-up iteration and one captured iteration
+        stages.append(dict(res=res, it=it, large=large, small=small, launches=launches // 2,
+                           images=bl + (bs or 0)))
+    return dict(spec=server.spec, server=server, stages=stages, host_l=host_l, host_s=host_s, lab_l=lab_l,
+                lab_s=lab_s)
+
+
+def conv_roofline(stage, reps=3):
+    """Time each convolution pass of the stage's workers alone with CUDA events;
+    return (algorithmic conv FLOPs of one iteration, seconds per iteration)."""
+    import torch
+
+    from paper_2509_26092_gb300 import dbl as D
+    s = torch.cuda.current_stream()
+    flops, secs = 0.0, 0.0
+    for wk in (stage["large"], stage["small"]):
+        if wk is None:
+            continue
+        stem = wk.spec.stem.name
+        bufs = _conv_buffers(wk)
+        for name, shp in wk.conv_shapes():
+            x, y, dy, dx, w16, g = bufs[name]
+            st_sum = torch.empty(shp.k, device=x.device)
+            st_sq = torch.empty(shp.k, device=x.device)
+            P = (shp.h + 2 * shp.pad - shp.r) // shp.stride + 1
+            cin = wk.spec.stem.cin_logical if name == stem else shp.c
+            f1 = 2.0 * shp.n * P * P * shp.k * shp.r * shp.s * cin
+            passes = [("fwd", lambda: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            if name != stem:
+                passes.append(("dgrad", lambda: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
+            passes.append(("wgrad", lambda: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
+            for _, fn in passes:
+                fn()
+                ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+                ev[0].record(s)
+                for _ in range(reps):
+                    fn()
+                ev[1].record(s)
+                torch.cuda.synchronize()
+                secs += ev[0].elapsed_time(ev[1]) / 1000.0 / reps
+                flops += f1
+    return flops, secs
+
+
+def _conv_buffers(wk):
+    """Per conv layer: (input, output, output-gradient, input-gradient, bf16 weights, fp32 gradient slice)."""
+    spec = wk.spec
+    srv_w16 = wk._bench_w16
+    out = {}
+    st = spec.stem
+    out[st.name] = (wk.x0, wk.stem_y, wk.stem_dy, None, spec.view(srv_w16, "conv1.w"), spec.view(wk.grad, "conv1.w"))
+    cur = wk.pool_out if spec.variant == "imagenet" else wk.stem_a
+    for d in wk.blocks:
+        b = d["spec"]
+        out[b.pre + ".conv1"] = (cur, d["h1"], d["dh1"], d["din"], spec.view(srv_w16, b.pre + ".conv1.w"),
+                                 spec.view(wk.grad, b.pre + ".conv1.w"))
+        out[b.pre + ".conv2"] = (d["o1"], d["h2"], d["dh2"], d["do1"], spec.view(srv_w16, b.pre + ".conv2.w"),
+                                 spec.view(wk.grad, b.pre + ".conv2.w"))
+        if b.proj:
+            out[b.pre + ".down"] = (cur, d["hs"], d["dhs"], d["din2"], spec.view(srv_w16, b.pre + ".down.w"),
+                                    spec.view(wk.grad, b.pre + ".down.w"))
+        cur = d["out"]
+    return out
+
+
+def run_ours(args, cfg):
+    import torch
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+    from paper_2509_26092_gb300 import build_lib
+    build_lib.build()
+    from paper_2509_26092_gb300 import dbl as D
+
+    pipe = build_pipeline(cfg, device)
+    stages = pipe["stages"]
+    images_per_step = sum(s["images"] for s in stages)
+
+    def step():
+        for st in stages:
+            st["it"].run()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if ws > 1:
+            torch.distributed.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    assert D.dbl_device_status() == D.DBL_OK, "a device-side wait timed out during warm-up"
+    clocks = ClockSampler(local)
+    clocks.start()
+    stream = torch.cuda.current_stream()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    t0.record(stream)
+    for _ in range(args.steps):
+        step()
+    t1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    ms = t0.elapsed_time(t1)
+    if ws > 1:
+        tt = torch.tensor([ms], device=device)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_per_step = ms / args.steps
+    value = images_per_step * ws * args.steps / (ms / 1000.0)
+    gpu_launches = sum(s["launches"] for s in stages) * args.steps
+
+    # per-resolution throughput (each stage's graph replayed alone)
+    per_res = {}
+    for st in stages:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(2, args.steps)
+        e0.record(stream)
+        for _ in range(reps):
+            st["it"].run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        per_res[str(st["res"])] = round(st["images"] * reps / (e0.elapsed_time(e1) / 1000.0), 1)
+
+    # end to end through the public API: pinned host images -> device, iteration, loss back to host
+    h2d = d2h = 0
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    e0.record(stream)
+    for _ in range(args.steps):
+        for st in stages:
+            it, bl, bs = st["it"], st["large"].batch, st["small"].batch if st["small"] else 0
+            it.set_inputs(pipe["host_l"][:bl], pipe["lab_l"][:bl], pipe["host_s"][:bs] if bs else None,
+                          pipe["lab_s"][:bs] if bs else None, non_blocking=True)
+            it.run()
+            losses = [st["large"].loss.to("cpu", non_blocking=False)]
+            if st["small"] is not None:
+                losses.append(st["small"].loss.to("cpu", non_blocking=False))
+        if h2d == 0:
+            for st in stages:
+                bl, bs = st["large"].batch, st["small"].batch if st["small"] else 0
+                h2d += (bl + bs) * cfg["native"] ** 2 * 3 * 4 + (bl + bs) * 4
+                d2h += 4 * (2 if bs else 1)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    if ws > 1:
+        tt = torch.tensor([e2e_ms], device=device)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_value = images_per_step * ws * args.steps / (e2e_ms / 1000.0)
+    assert D.dbl_device_status() == D.DBL_OK, "a device-side wait timed out during the timed region"
+
+    # roofline of the dominant kernel: the implicit-GEMM convolution, full-resolution stage, timed alone
+    hbm, bf16, bf16_sus, src = _peaks()
+    top = max(stages, key=lambda s: s["res"])
+    for wk in (top["large"], top["small"]):
+        if wk is not None:
+            wk._bench_w16 = pipe["server"].w16
+    flops, secs = conv_roofline(top)
+    achieved = flops / secs / 1e12
+    roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16, "unit": "TFLOP/s",
+                "frac": round(achieved / bf16, 4), "traffic": _traffic_record(args.config),
+                "kernel": "conv_igemm_kernel (fwd/dgrad/wgrad, every layer of both workers at "
+                          f"{top['res']} px, each ABI call timed alone)", "peak_source": src}
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        v, dt, images, sample = time_oracle(cfg)
+        cpu = {"value": round(v, 4), "unit": "images/s", "cores": int(os.environ.get("OMP_NUM_THREADS",
+                                                                                      os.cpu_count() or 1)),
+               "kind": "oracle", "sample": sample, "seconds": round(dt, 2)}
+    if rank == 0:
+        line = {"metric": METRIC, "value": round(value, 1), "unit": "images/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3), "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": args.config, "description": cfg["desc"],
+                           "stages_px": list(cfg["stages"]), "large_batch": list(cfg["large"]),
+                           "small_batch": list(cfg["small"]), "images_per_step": images_per_step,
+                           "params": pipe["spec"].n_params(), "f_small": F_SMALL, "lr": LR, "momentum": MOMENTUM,
+                           "l2": "working set (activations, several GB) larger than L2; no explicit flush",
+                           "parallelism": f"{ws} independent replica(s), 2 worker streams each"},
+                "per_resolution": per_res, "roofline": roofline, "cpu_baseline": cpu,
+                "e2e": {"value": round(e2e_value, 1), "unit": "images/s", "h2d_bytes_per_step": h2d,
+                        "d2h_bytes_per_step": d2h},
+                "clocks": clk, "gpu_launches": gpu_launches,
+                "conv_tflops_step": round(sum(s["large"].conv_flops() + (s["small"].conv_flops() if s["small"] else 0)
+                                              for s in stages) / (ms_per_step / 1000.0) / 1e12, 1)}
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    cfg = CONFIGS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, cfg)
+    return run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -56,6 +56,11 @@ DBL_API const char* dbl_last_error(void);
 /* Library version, major*10000 + minor*100 + patch.  Host. */
 DBL_API int dbl_version(void);
 
+/* Number of kernel launches this library has issued from the host since it
+ * was loaded (all threads, all devices).  Launches replayed from a captured
+ * CUDA graph are not counted again.  Host; for instrumentation. */
+DBL_API int64_t dbl_kernel_launches(void);
+
 /* Synchronous: reads and clears the device-side status word of the current
  * device (DBL_OK or DBL_ERR_TIMEOUT), after synchronising the device.  For
  * tests and diagnostics only; never call it inside a captured graph. */

@@ -5,6 +5,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "dbl_internal.cuh"
@@ -12,6 +13,9 @@
 namespace dbl {
 
 static thread_local char g_err[512] = "";
+static std::atomic<int64_t> g_launches{0};
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int set_error(int code, const char* fmt, ...)
 {
@@ -67,6 +71,8 @@ extern "C" {
 const char* dbl_last_error(void) { return dbl::g_err; }
 
 int dbl_version(void) { return 100; /* 0.1.0 */ }
+
+int64_t dbl_kernel_launches(void) { return dbl::g_launches.load(std::memory_order_relaxed); }
 
 int dbl_resize_taps(int32_t in, int32_t out, int32_t* i0, int32_t* i1, float* lambda)
 {

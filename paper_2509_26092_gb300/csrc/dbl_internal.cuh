@@ -22,8 +22,16 @@ inline int cuda_check(cudaError_t e, const char* what)
     return set_error(DBL_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-// Launch-error check after a kernel launch (does not synchronise).
-inline int launch_check(const char* what) { return cuda_check(cudaGetLastError(), what); }
+// Counts one kernel launch (see dbl_kernel_launches).
+void count_launch();
+
+// Launch-error check after a kernel launch (does not synchronise); every
+// launch site calls it exactly once, which is also how launches are counted.
+inline int launch_check(const char* what)
+{
+    count_launch();
+    return cuda_check(cudaGetLastError(), what);
+}
 
 inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
 

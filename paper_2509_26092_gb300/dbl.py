@@ -59,6 +59,7 @@ def lib():
         sig = {
             "dbl_last_error": (ctypes.c_char_p, []),
             "dbl_version": (ctypes.c_int, []),
+            "dbl_kernel_launches": (_I64, []),
             "dbl_device_status": (ctypes.c_int, [ctypes.POINTER(_I32)]),
             "dbl_conv_workspace_bytes": (_SZ, [ctypes.POINTER(ConvShape), ctypes.c_int]),
             "dbl_conv_fwd": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _V, _V, _SZ, _V]),
@@ -115,6 +116,11 @@ def dbl_last_error():
 
 def dbl_version():
     return lib().dbl_version()
+
+
+def dbl_kernel_launches():
+    """Kernel launches issued by the library from the host so far."""
+    return lib().dbl_kernel_launches()
 
 
 def dbl_device_status():

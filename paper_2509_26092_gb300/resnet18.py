@@ -1,0 +1,438 @@
+"""ResNet-18 training step of the hybrid dual-batch / cyclic-progressive scheme
+on one GB300, driven through the C ABI of ``libdbl.so``.
+
+What runs where
+---------------
+Every arithmetic step is a ``libdbl`` kernel; this module only allocates
+device memory (through PyTorch), lays out the flat parameter buffers and
+enqueues ABI calls on CUDA streams:
+
+* the parameter server (Sec. 2.3) holds fp32 master weights ``w``, the
+  momentum buffer ``u`` and the bf16 copy ``w16`` the workers pull, each one
+  flat contiguous buffer;
+* a worker (Sec. 3.1) owns the activations of one batch size at one
+  resolution and writes its batch-mean gradient into its own flat fp32
+  buffer (same layout as ``w``);
+* a dual-batch iteration runs the large-batch and the small-batch worker on
+  two streams of the same GPU, joins them with an event, and merges both
+  pushes into the master weights with the model-update factor (Sec. 3.4);
+* the resolution of a cyclic-progressive sub-stage (Sec. 4.1) is produced by
+  ``dbl_progressive_resize`` from the native-resolution images.
+
+ResNet-18 (Sec. 5.1.1): stem convolution (3x3/1 for CIFAR-shaped inputs,
+7x7/2 + 3x3/2 max pooling for ImageNet-shaped inputs), four stages of two
+BasicBlocks (64/128/256/512 channels; the first block of stages 2-4 has
+stride 2 and a 1x1 stride-2 projection shortcut with BatchNorm), global
+average pooling and one fully connected layer.  The 3 colour channels are
+zero-padded to 8 so that a pixel is one 16-byte row.
+
+Convolutions read the bf16 weights ``w16``; BatchNorm and the fully connected
+layer read the fp32 master weights directly (they are tiny).
+"""
+from dataclasses import dataclass, field
+
+import torch
+
+from . import dbl as D
+
+WIDTHS = (64, 128, 256, 512)
+ALIGN = 64  # parameter tensors start on 256-byte boundaries
+
+
+@dataclass
+class ConvSpec:
+    name: str
+    cin: int       # channels as stored (the stem's 3 colour channels padded to 8)
+    cin_logical: int
+    cout: int
+    r: int
+    stride: int
+    pad: int
+
+
+@dataclass
+class BlockSpec:
+    pre: str
+    cin: int
+    cout: int
+    stride: int
+    proj: bool
+
+
+@dataclass
+class ParamEntry:
+    name: str
+    shape: tuple          # stored shape
+    logical: tuple        # shape the method defines (stem: 3 input channels)
+    fan_in: object
+    offset: int
+    numel: int = field(init=False)
+
+    def __post_init__(self):
+        n = 1
+        for s in self.shape:
+            n *= s
+        self.numel = n
+
+
+class ResNet18Spec:
+    """Layer list and flat parameter layout of a ResNet-18 variant."""
+
+    def __init__(self, variant="cifar", classes=100, widths=WIDTHS):
+        if variant not in ("cifar", "imagenet"):
+            raise ValueError(variant)
+        self.variant, self.classes, self.widths = variant, classes, tuple(widths)
+        r, st, pad = (3, 1, 1) if variant == "cifar" else (7, 2, 3)
+        self.stem = ConvSpec("conv1", 8, 3, widths[0], r, st, pad)
+        self.blocks = []
+        cin = widths[0]
+        for li, wd in enumerate(widths):
+            for bi in range(2):
+                stride = 2 if (li > 0 and bi == 0) else 1
+                self.blocks.append(BlockSpec(f"layer{li + 1}.{bi}", cin, wd, stride, stride != 1 or cin != wd))
+                cin = wd
+        self.entries = []
+        off = 0
+
+        def add(name, shape, logical, fan_in):
+            nonlocal off
+            e = ParamEntry(name, tuple(shape), tuple(logical), fan_in, off)
+            self.entries.append(e)
+            off += (e.numel + ALIGN - 1) // ALIGN * ALIGN
+
+        def conv(cs):
+            add(cs.name + ".w", (cs.cout, cs.r, cs.r, cs.cin), (cs.cout, cs.r, cs.r, cs.cin_logical),
+                cs.r * cs.r * cs.cin_logical)
+
+        def bn(name, c):
+            add(name + ".g", (c,), (c,), None)
+            add(name + ".b", (c,), (c,), None)
+
+        conv(self.stem)
+        bn("bn1", widths[0])
+        for b in self.blocks:
+            conv(ConvSpec(b.pre + ".conv1", b.cin, b.cin, b.cout, 3, b.stride, 1))
+            bn(b.pre + ".bn1", b.cout)
+            conv(ConvSpec(b.pre + ".conv2", b.cout, b.cout, b.cout, 3, 1, 1))
+            bn(b.pre + ".bn2", b.cout)
+            if b.proj:
+                conv(ConvSpec(b.pre + ".down", b.cin, b.cin, b.cout, 1, b.stride, 0))
+                bn(b.pre + ".downbn", b.cout)
+        add("fc.w", (classes, cin), (classes, cin), cin)
+        add("fc.b", (classes,), (classes,), None)
+        self.n_flat = off
+        self.by_name = {e.name: e for e in self.entries}
+
+    def table(self):
+        """(name, logical shape, fan_in) of every parameter tensor, for the input generator."""
+        return [(e.name, e.logical, e.fan_in) for e in self.entries]
+
+    def n_params(self):
+        """Parameters the method defines (without the stem's channel padding)."""
+        n = 0
+        for e in self.entries:
+            k = 1
+            for s in e.logical:
+                k *= s
+            n += k
+        return n
+
+    def view(self, flat, name):
+        e = self.by_name[name]
+        return flat[e.offset:e.offset + e.numel].view(e.shape)
+
+    def pack(self, tensors, device="cuda", dtype=torch.float32):
+        """Flat buffer from {name: array of the logical shape} (stem channels zero-padded)."""
+        flat = torch.zeros(self.n_flat, dtype=dtype, device=device)
+        for e in self.entries:
+            t = torch.as_tensor(tensors[e.name], dtype=dtype)
+            v = self.view(flat, e.name)
+            if tuple(t.shape) == e.shape:
+                v.copy_(t)
+            else:
+                v.zero_()
+                v[..., :t.shape[-1]].copy_(t)
+        return flat
+
+    def unpack(self, flat):
+        """{name: host float64 array of the logical shape} from a flat buffer."""
+        out = {}
+        for e in self.entries:
+            v = self.view(flat, e.name)
+            if e.shape != e.logical:
+                v = v[..., :e.logical[-1]]
+            out[e.name] = v.detach().double().cpu().numpy().copy()
+        return out
+
+
+def conv_out(n, r, st, pad):
+    return (n + 2 * pad - r) // st + 1
+
+
+class ServerState:
+    """The parameter server's global model: fp32 master w, momentum u, bf16 pull copy w16."""
+
+    def __init__(self, spec, params, momentum_state=None, device="cuda"):
+        self.spec = spec
+        self.w = spec.pack(params, device)
+        self.u = (spec.pack(momentum_state, device) if momentum_state is not None
+                  else torch.zeros_like(self.w))
+        self.w16 = self.w.to(torch.bfloat16)
+
+
+class Worker:
+    """Activations, gradients and scratch of one worker at one (batch, resolution)."""
+
+    def __init__(self, spec, batch, res, device="cuda", eps=1e-5):
+        self.spec, self.batch, self.res, self.eps = spec, batch, res, eps
+        dev = device
+        bf = torch.bfloat16
+        B = batch
+
+        def act(h, c):
+            return torch.empty((B, h, h, c), dtype=bf, device=dev)
+
+        def vec(c):
+            return torch.empty(c, dtype=torch.float32, device=dev)
+
+        self.x0 = act(res, 8)
+        st = spec.stem
+        p = conv_out(res, st.r, st.stride, st.pad)
+        self.stem_hw = p
+        self.stem_y, self.stem_a, self.stem_da, self.stem_dy = act(p, st.cout), act(p, st.cout), None, act(p, st.cout)
+        self.stem_stats = [vec(st.cout) for _ in range(4)]  # sum, sumsq, mean, invstd
+        h = p
+        if spec.variant == "imagenet":
+            q = conv_out(p, 3, 2, 1)
+            self.pool_out = act(q, st.cout)
+            self.pool_arg = torch.empty((B, q, q, st.cout), dtype=torch.uint8, device=dev)
+            self.stem_da = act(p, st.cout)
+            h = q
+        self.blocks = []
+        for b in spec.blocks:
+            ho = conv_out(h, 3, b.stride, 1)
+            d = dict(spec=b, hin=h, hout=ho)
+            for k in ("h1", "o1", "h2", "out", "dh2", "do1", "dh1", "din", "din2"):
+                d[k] = act(ho if k not in ("din", "din2") else h, b.cout if k not in ("din", "din2") else b.cin)
+            if b.proj:
+                d["hs"], d["sc"], d["dhs"] = act(ho, b.cout), act(ho, b.cout), act(ho, b.cout)
+            for k in ("bn1", "bn2", "downbn"):
+                d[k] = [vec(b.cout) for _ in range(4)]
+            self.blocks.append(d)
+            h = ho
+        self.final_hw = h
+        self.dfeat = act(h, spec.widths[-1])
+        self.grad = torch.zeros(spec.n_flat, dtype=torch.float32, device=dev)
+        self.loss = torch.zeros(1, dtype=torch.float32, device=dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.ws = torch.empty(self._ws_bytes(), dtype=torch.uint8, device=dev)
+
+    # ------------------------------------------------------------------ shapes
+    def conv_shapes(self):
+        """(name, dbl_conv_shape) of every convolution of this worker, in forward order."""
+        B, spec = self.batch, self.spec
+        st = spec.stem
+        out = [(st.name, D.conv_shape(B, self.res, self.res, st.cin, st.cout, st.r, st.stride, st.pad))]
+        for d in self.blocks:
+            b = d["spec"]
+            out.append((b.pre + ".conv1", D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)))
+            out.append((b.pre + ".conv2", D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)))
+            if b.proj:
+                out.append((b.pre + ".down", D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)))
+        return out
+
+    def _ws_bytes(self):
+        need = D.dbl_head_workspace_bytes(self.batch, self.spec.widths[-1], self.spec.classes)
+        for _, s in self.conv_shapes():
+            for ps in (D.DBL_PASS_FWD, D.DBL_PASS_DGRAD, D.DBL_PASS_WGRAD):
+                need = max(need, D.dbl_conv_workspace_bytes(s, ps))
+        for d in self.blocks:
+            need = max(need, D.dbl_bn_workspace_bytes(D.bn_shape(self.batch * d["hout"] ** 2, d["spec"].cout)))
+        need = max(need, D.dbl_bn_workspace_bytes(D.bn_shape(self.batch * self.stem_hw ** 2, self.spec.stem.cout)))
+        return int(need) + 256
+
+    def conv_flops(self):
+        """Algorithmic conv FLOPs of one step: 2*M*N*K per pass, unpadded channels,
+        forward + data gradient (not the stem) + weight gradient."""
+        total = 0
+        for name, s in self.conv_shapes():
+            P = conv_out(s.h, s.r, s.stride, s.pad)
+            cin = self.spec.stem.cin_logical if name == self.spec.stem.name else s.c
+            f = 2 * s.n * P * P * s.k * s.r * s.s * cin
+            total += f * (2 if name == self.spec.stem.name else 3)
+        return total
+
+    # ------------------------------------------------------------------ the step
+    def enqueue_step(self, server, images, native_res, stream):
+        """Resize, forward, loss, backward; gradients land in self.grad (batch means).
+
+        images: fp32 [B, native_res, native_res, 3] on the device; labels in self.labels.
+        """
+        spec, B, eps = self.spec, self.batch, self.eps
+        s = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+        ws, wsb = self.ws, self.ws.numel()
+        W16, W, G = server.w16, server.w, self.grad
+
+        def wv(name):
+            return spec.view(W16, name)
+
+        def pv(name):
+            return spec.view(W, name)
+
+        def gv(name):
+            return spec.view(G, name)
+
+        D.dbl_progressive_resize(images, D.DBL_F32, B, native_res, native_res, 3, self.x0, D.DBL_BF16, self.res,
+                                 self.res, 8, s)
+        # ---- forward
+        st = spec.stem
+        shp = D.conv_shape(B, self.res, self.res, st.cin, st.cout, st.r, st.stride, st.pad)
+        s_sum, s_sq, s_mean, s_istd = self.stem_stats
+        D.dbl_conv_fwd(shp, self.x0, wv("conv1.w"), self.stem_y, s_sum, s_sq, ws, wsb, s)
+        bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)
+        D.dbl_bn_relu_fused(bns, self.stem_y, s_sum, s_sq, pv("bn1.g"), pv("bn1.b"), None, self.stem_a, s_mean, s_istd,
+                            s)
+        cur = self.stem_a
+        if spec.variant == "imagenet":
+            D.dbl_maxpool_fwd(B, self.stem_hw, self.stem_hw, st.cout, self.stem_a, self.pool_out, self.pool_arg, s)
+            cur = self.pool_out
+        for d in self.blocks:
+            b = d["spec"]
+            d["x"] = cur
+            cnt = B * d["hout"] ** 2
+            s1 = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)
+            st1 = d["bn1"]
+            D.dbl_conv_fwd(s1, cur, wv(b.pre + ".conv1.w"), d["h1"], st1[0], st1[1], ws, wsb, s)
+            D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, True), d["h1"], st1[0], st1[1], pv(b.pre + ".bn1.g"),
+                                pv(b.pre + ".bn1.b"), None, d["o1"], st1[2], st1[3], s)
+            s2 = D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)
+            st2 = d["bn2"]
+            D.dbl_conv_fwd(s2, d["o1"], wv(b.pre + ".conv2.w"), d["h2"], st2[0], st2[1], ws, wsb, s)
+            if b.proj:
+                sd = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)
+                std = d["downbn"]
+                D.dbl_conv_fwd(sd, cur, wv(b.pre + ".down.w"), d["hs"], std[0], std[1], ws, wsb, s)
+                D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, False), d["hs"], std[0], std[1],
+                                    pv(b.pre + ".downbn.g"), pv(b.pre + ".downbn.b"), None, d["sc"], std[2], std[3], s)
+                res = d["sc"]
+            else:
+                res = cur
+            D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, True), d["h2"], st2[0], st2[1], pv(b.pre + ".bn2.g"),
+                                pv(b.pre + ".bn2.b"), res, d["out"], st2[2], st2[3], s)
+            cur = d["out"]
+        # ---- head: pooling, FC, softmax cross-entropy and their backward
+        C = spec.widths[-1]
+        D.dbl_head_fwd_bwd(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"), self.labels, self.loss,
+                           gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
+        # ---- backward
+        dout, dout2 = self.dfeat, None
+        for d in reversed(self.blocks):
+            b = d["spec"]
+            cnt = B * d["hout"] ** 2
+            st1, st2, std = d["bn1"], d["bn2"], d["downbn"]
+            dres = None if b.proj else d["din2"]
+            D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), dout, dout2, d["h2"], d["out"],
+                                    pv(b.pre + ".bn2.g"), st2[2], st2[3], d["dh2"], dres, gv(b.pre + ".bn2.g"),
+                                    gv(b.pre + ".bn2.b"), ws, wsb, s)
+            s2 = D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)
+            D.dbl_conv_wgrad(s2, d["o1"], d["dh2"], gv(b.pre + ".conv2.w"), False, ws, wsb, s)
+            D.dbl_conv_dgrad(s2, d["dh2"], wv(b.pre + ".conv2.w"), d["do1"], None, 0, s)
+            D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), d["do1"], None, d["h1"], d["o1"],
+                                    pv(b.pre + ".bn1.g"), st1[2], st1[3], d["dh1"], None, gv(b.pre + ".bn1.g"),
+                                    gv(b.pre + ".bn1.b"), ws, wsb, s)
+            s1 = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)
+            D.dbl_conv_wgrad(s1, d["x"], d["dh1"], gv(b.pre + ".conv1.w"), False, ws, wsb, s)
+            D.dbl_conv_dgrad(s1, d["dh1"], wv(b.pre + ".conv1.w"), d["din"], None, 0, s)
+            if b.proj:
+                # the shortcut BatchNorm sees the same masked gradient as bn2
+                D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), dout, dout2, d["hs"], d["out"],
+                                        pv(b.pre + ".downbn.g"), std[2], std[3], d["dhs"], None,
+                                        gv(b.pre + ".downbn.g"), gv(b.pre + ".downbn.b"), ws, wsb, s)
+                sd = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)
+                D.dbl_conv_wgrad(sd, d["x"], d["dhs"], gv(b.pre + ".down.w"), False, ws, wsb, s)
+                D.dbl_conv_dgrad(sd, d["dhs"], wv(b.pre + ".down.w"), d["din2"], None, 0, s)
+            dout, dout2 = d["din"], d["din2"]
+        bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)
+        if spec.variant == "imagenet":
+            D.dbl_maxpool_bwd(B, self.stem_hw, self.stem_hw, st.cout, dout, dout2, self.pool_arg, self.stem_da, s)
+            D.dbl_bn_relu_fused_bwd(bns, self.stem_da, None, self.stem_y, self.stem_a, pv("bn1.g"), s_mean, s_istd,
+                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s)
+        else:
+            D.dbl_bn_relu_fused_bwd(bns, dout, dout2, self.stem_y, self.stem_a, pv("bn1.g"), s_mean, s_istd,
+                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s)
+        D.dbl_conv_wgrad(shp, self.x0, self.stem_dy, gv("conv1.w"), False, ws, wsb, s)
+
+
+class DualBatchIteration:
+    """One parameter-server iteration of the hybrid scheme on one GPU.
+
+    The large-batch worker runs on stream L and the small-batch worker on
+    stream S, concurrently; the merge (Sec. 3.4) runs on stream L once both
+    have pushed, in the arrival order given by ``order``.  Either worker may be
+    None (a single push).  ``capture()`` records the iteration as a CUDA graph.
+    """
+
+    def __init__(self, server, large, small, native_res, lr=0.2, momentum=0.9, f_large=1.0, f_small=19.0 / 21.0,
+                 order=0):
+        self.server, self.large, self.small = server, large, small
+        self.native_res = native_res
+        self.lr, self.momentum, self.f_large, self.f_small, self.order = lr, momentum, f_large, f_small, order
+        self.stream_l = torch.cuda.Stream()
+        self.stream_s = torch.cuda.Stream()
+        self.images_l = self.images_s = None
+        self.graph = None
+
+    def set_inputs(self, images_l, labels_l, images_s=None, labels_s=None, non_blocking=False):
+        """fp32 images at the native resolution and int32 labels (device or pinned host
+        tensors), copied into the iteration's device buffers on the current stream."""
+        dev = self.server.w.device
+        if self.large is not None:
+            if self.images_l is None:
+                self.images_l = torch.empty(images_l.shape, dtype=torch.float32, device=dev)
+            self.images_l.copy_(images_l, non_blocking=non_blocking)
+            self.large.labels.copy_(labels_l, non_blocking=non_blocking)
+        if self.small is not None:
+            if self.images_s is None:
+                self.images_s = torch.empty(images_s.shape, dtype=torch.float32, device=dev)
+            self.images_s.copy_(images_s, non_blocking=non_blocking)
+            self.small.labels.copy_(labels_s, non_blocking=non_blocking)
+
+    def _enqueue(self):
+        cur = torch.cuda.current_stream()
+        sL, sS = self.stream_l, self.stream_s
+        sL.wait_stream(cur)
+        sS.wait_stream(cur)
+        if self.large is not None:
+            self.large.enqueue_step(self.server, self.images_l, self.native_res, sL)
+        if self.small is not None:
+            self.small.enqueue_step(self.server, self.images_s, self.native_res, sS)
+        sL.wait_stream(sS)  # the server applies the pushes once both have arrived
+        srv = self.server
+        D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, self.large.grad if self.large else None,
+                                  self.small.grad if self.small else None, srv.spec.n_flat, self.lr, self.momentum,
+                                  self.f_large, self.f_small, self.order, sL.cuda_stream)
+        cur.wait_stream(sL)
+
+    def run(self):
+        if self.graph is not None:
+            self.graph.replay()
+        else:
+            self._enqueue()
+
+    def capture(self):
+        """Record one iteration (both workers, the join and the merge) as a CUDA graph."""
+        self._enqueue()  # warm-up outside capture: kernel attributes, lazy loading
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            with torch.cuda.graph(g, stream=s):
+                self._enqueue()
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        self.graph = g
+        return g
+
+    def images_per_iteration(self):
+        return (self.large.batch if self.large else 0) + (self.small.batch if self.small else 0)

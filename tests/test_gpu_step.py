@@ -1,0 +1,121 @@
+"""Whole-step GPU parity: the ResNet-18 training step and the two-stream
+dual-batch iteration run through libdbl, against the fp64 oracle with bf16
+rounding at the same storage points.
+
+Loss and every parameter gradient are compared per tensor at the conv-path
+tolerance (max-norm relative error <= 1e-2).  The merge is compared on the
+GPU's own pushed gradients (identical fp32 inputs) at 1e-6.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from conftest import max_norm_rel
+from gpu_common import load_dbl
+from oracle import resnet18 as OR
+from paper_2509_26092_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+
+
+@pytest.fixture(scope="module")
+def R():
+    load_dbl()
+    from paper_2509_26092_gb300 import resnet18
+    return resnet18
+
+
+def _compare_grads(spec, grad_flat, ref_grads):
+    got = spec.unpack(grad_flat)
+    worst = (0.0, None)
+    for name, g in ref_grads.items():
+        e = max_norm_rel(got[name], g)
+        worst = max(worst, (e, name))
+        assert e <= TOL, f"{name}: {e:.3e}"
+    return worst
+
+
+@pytest.mark.parametrize("variant,classes,batch,res", [("cifar", 100, 8, 32), ("imagenet", 1000, 8, 96)])
+def test_train_step_matches_oracle(R, variant, classes, batch, res):
+    spec = R.ResNet18Spec(variant, classes)
+    params = synth.params(spec.table(), seed=3, random_bn=True)
+    img = synth.images(batch, res, res, 3, seed=3)
+    lab = synth.labels(batch, classes, seed=3)
+    server = R.ServerState(spec, params)
+    wk = R.Worker(spec, batch, res)
+    it = R.DualBatchIteration(server, wk, None, res)
+    it.set_inputs(torch.from_numpy(img).cuda(), torch.from_numpy(lab).cuda())
+    s = torch.cuda.current_stream()
+    wk.enqueue_step(server, it.images_l, res, s)
+    torch.cuda.synchronize()
+    D = load_dbl()
+    assert D.dbl_device_status() == D.DBL_OK
+    ref = OR.train_step({k: v.astype(np.float64) for k, v in params.items()}, img.astype(np.float64), lab, variant,
+                        bf16_storage=True)
+    assert abs(wk.loss.item() - ref["loss"]) <= TOL * abs(ref["loss"])
+    worst = _compare_grads(spec, wk.grad, ref["grads"])
+    print(f"{variant}: loss {wk.loss.item():.6f} vs {ref['loss']:.6f}; worst grad {worst[1]} {worst[0]:.2e}")
+
+
+def test_dual_batch_iteration_matches_oracle(R):
+    # native 32x32 images, sub-stage resolution 24: large worker batch 6, small worker batch 2
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=5, random_bn=True)
+    u0 = synth.momentum_state(spec.table(), 0.01, seed=5)
+    img = synth.images(8, 32, 32, 3, seed=5)
+    lab = synth.labels(8, 100, seed=5)
+    server = R.ServerState(spec, params, u0)
+    large, small = R.Worker(spec, 6, 24), R.Worker(spec, 2, 24)
+    fS = 19.0 / 21.0
+    it = R.DualBatchIteration(server, large, small, 32, lr=0.2, momentum=0.9, f_large=1.0, f_small=fS, order=0)
+    it.set_inputs(torch.from_numpy(img[2:]).cuda(), torch.from_numpy(lab[2:]).cuda(), torch.from_numpy(img[:2]).cuda(),
+                  torch.from_numpy(lab[:2]).cuda())
+    w_before = server.w.clone()
+    u_before = server.u.clone()
+    it.run()
+    torch.cuda.synchronize()
+    p64 = {k: v.astype(np.float64) for k, v in params.items()}
+    u64 = {k: v.astype(np.float64) for k, v in u0.items()}
+    nw, nu, lL, lS, gL, gS = OR.dual_batch_iteration(p64, u64, img[2:], lab[2:], img[:2], lab[:2], 24, "cifar", 0.2,
+                                                     0.9, 1.0, fS, order=0, bf16_storage=True)
+    assert abs(large.loss.item() - lL) <= TOL * abs(lL)
+    assert abs(small.loss.item() - lS) <= TOL * abs(lS)
+    _compare_grads(spec, large.grad, gL)
+    _compare_grads(spec, small.grad, gS)
+    # the server's merge, given the pushes the GPU workers produced
+    rw, ru = orc.ps_merge(w_before.double().cpu().numpy(), u_before.double().cpu().numpy(),
+                          large.grad.double().cpu().numpy(), small.grad.double().cpu().numpy(), 0.2, 0.9, 1.0, fS, 0)
+    assert max_norm_rel(server.w.double().cpu().numpy(), rw) <= 1e-6
+    assert max_norm_rel(server.u.double().cpu().numpy(), ru) <= 1e-6
+    assert torch.equal(server.w16, server.w.to(torch.bfloat16))
+    # and against the oracle's own end-to-end iteration
+    got_w = spec.unpack(server.w)
+    for name in nw:
+        assert max_norm_rel(got_w[name] - p64[name], nw[name] - p64[name]) <= TOL, name
+
+
+def test_graph_replay_equals_eager(R):
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=7)
+    img = torch.from_numpy(synth.images(12, 32, 32, 3, seed=7)).cuda()
+    lab = torch.from_numpy(synth.labels(12, 100, seed=7)).cuda()
+    outs = []
+    for use_graph in (False, True):
+        server = R.ServerState(spec, params)
+        it = R.DualBatchIteration(server, R.Worker(spec, 8, 16), R.Worker(spec, 4, 16), 32)
+        it.set_inputs(img[4:], lab[4:], img[:4], lab[:4])
+        if use_graph:
+            w0, u0 = server.w.clone(), server.u.clone()
+            it.capture()  # runs one eager warm-up iteration first
+            server.w.copy_(w0)
+            server.u.copy_(u0)
+            server.w16.copy_(w0.to(torch.bfloat16))
+        for _ in range(2):
+            it.run()
+        torch.cuda.synchronize()
+        outs.append(server.w.clone())
+    # deterministic kernels: replay and eager launches give identical bits
+    assert torch.equal(outs[0], outs[1])
