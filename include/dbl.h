@@ -156,6 +156,30 @@ DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf
                           const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
                           float* dgamma, float* dbeta, void* ws, size_t ws_bytes, void* stream);
 
+/* Same computation as dbl_bn_relu_fused_bwd, for callers that cannot hand
+ * the library a workspace: their memory comes from an allocator they do not
+ * control (a host framework that owns every device allocation), or their
+ * device-memory footprint must be fixed once the process has started.  The
+ * paper has no counterpart; this is a property of the library, not of the
+ * method.
+ *
+ * The scratch lives in one statically sized device array inside libdbl.so
+ * (4.2 MB, held on every device that loads the library until the process
+ * exits).  Limit: c <= DBL_BN_NOALLOC_MAX_C (512); larger c returns
+ * DBL_ERR_UNSUPPORTED before anything is launched.  The first call on a
+ * device looks up the array's device address (cudaGetSymbolAddress) with that
+ * device current; make that first call before any stream capture.  No
+ * device memory is allocated or freed by any call.  All calls share the one
+ * array, so calls whose kernels overlap on the GPU (two streams, two host
+ * threads) race on it; serialise them.  Nothing in the array needs to start
+ * at zero: each call writes every element it later reads. */
+#define DBL_BN_NOALLOC_MAX_C 512
+DBL_API int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* shape, const void* dout_bf16,
+                                          const void* dout2_bf16 /* or NULL */, const void* y_bf16,
+                                          const void* out_bf16, const float* gamma, const float* save_mean,
+                                          const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
+                                          float* dgamma, float* dbeta, void* stream);
+
 /* ========================================================================
  * Stem max pooling (ImageNet ResNet-18): 3x3 window, stride 2, padding 1,
  * padding counted as -infinity.  x: [n,h,w,c] bf16, y: [n,P,Q,c] bf16,

@@ -9,6 +9,8 @@
 // Backward (two passes): a reduce pass of sum(g) and sum(g*xhat) per channel
 // into per-CTA partials, a tiny fixed-order finalize, and an apply pass
 //     dy = gamma*invstd*(g - sum(g)/count - xhat*sum(g*xhat)/count).
+#include <mutex>
+
 #include "dbl_internal.cuh"
 
 namespace {
@@ -344,3 +346,81 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
 }
 
 }  // extern "C"
+
+// ----------------------------------------------------------------------------- workspace-free variant
+// For callers that cannot pass a workspace (see dbl_bn_relu_fused_bwd_noalloc
+// in dbl.h): the per-CTA partials and the per-channel coefficients live in
+// one file-scope device array sized for the largest channel count accepted.
+namespace {
+
+constexpr int kNoallocMaxBlocks = 1024;  // bwd_blocks() never exceeds this
+constexpr size_t kNoallocFloats =
+    (size_t)kNoallocMaxBlocks * 2 * DBL_BN_NOALLOC_MAX_C + 3 * (size_t)DBL_BN_NOALLOC_MAX_C;
+
+static __device__ __align__(256) float g_bn_noalloc_scratch[kNoallocFloats];
+
+// Device address of the array, looked up once per device with that device current.
+// (In host code the array's name is only a stand-in, never a device address.)
+float* noalloc_scratch(int* rc)
+{
+    static std::mutex mu;
+    static float* ptr[64] = {nullptr};
+    int dev = 0;
+    if ((*rc = dbl::cuda_check(cudaGetDevice(&dev), "bn_bwd_noalloc: cudaGetDevice"))) return nullptr;
+    if (dev < 0 || dev >= 64) {
+        *rc = dbl::set_error(DBL_ERR_UNSUPPORTED, "bn_bwd_noalloc: device index %d out of range", dev);
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ptr[dev]) {
+        void* p = nullptr;
+        if ((*rc = dbl::cuda_check(cudaGetSymbolAddress(&p, g_bn_noalloc_scratch),
+                                   "bn_bwd_noalloc: cudaGetSymbolAddress")))
+            return nullptr;
+        ptr[dev] = static_cast<float*>(p);
+    }
+    *rc = DBL_OK;
+    return ptr[dev];
+}
+
+}  // namespace
+
+extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* dout, const void* dout2,
+                                              const void* y, const void* out, const float* gamma,
+                                              const float* save_mean, const float* save_invstd, void* dy,
+                                              void* dresidual, float* dgamma, float* dbeta, void* stream)
+{
+    using namespace dbl;
+    int rc = check_shape(s, "bn_relu_fused_bwd_noalloc");
+    if (rc) return rc;
+    if (s->c > DBL_BN_NOALLOC_MAX_C)
+        return set_error(DBL_ERR_UNSUPPORTED,
+                         "bn_relu_fused_bwd_noalloc: %d channels exceed the static scratch limit of %d", s->c,
+                         DBL_BN_NOALLOC_MAX_C);
+    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: null pointer");
+    if (!aligned16(dout) || !aligned16(y) || !aligned16(dy) || (dout2 && !aligned16(dout2)) ||
+        (out && !aligned16(out)) || (dresidual && !aligned16(dresidual)))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: tensors must be 16-byte aligned");
+    if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: empty batch");
+    const int C = s->c;
+    const int64_t nblk = bwd_blocks(s->count);
+    if (nblk > kNoallocMaxBlocks || (size_t)nblk * 2 * C + 3 * (size_t)C > kNoallocFloats)
+        return set_error(DBL_ERR_UNSUPPORTED, "bn_relu_fused_bwd_noalloc: shape exceeds the static scratch");
+    float* partial = noalloc_scratch(&rc);
+    if (rc) return rc;
+    float* coef = partial + nblk * 2 * C;  // written by the finalize kernel before the apply kernel reads it
+    const int64_t rows = (s->count + nblk - 1) / nblk;
+    cudaStream_t st = as_stream(stream);
+    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
+    bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
+                                                         save_mean, save_invstd, rows, partial);
+    if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
+    bn_bwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+                                                            dgamma, dbeta, coef);
+    if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
+    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
+        bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
+        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
+    return launch_check("bn_bwd_noalloc apply launch");
+}

@@ -69,6 +69,7 @@ def lib():
             "dbl_bn_relu_fused": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 10),
             "dbl_bn_workspace_bytes": (_SZ, [ctypes.POINTER(BnShape)]),
             "dbl_bn_relu_fused_bwd": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 12 + [_SZ, _V]),
+            "dbl_bn_relu_fused_bwd_noalloc": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 12),
             "dbl_maxpool_fwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V]),
             "dbl_maxpool_bwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V, _V]),
             "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
@@ -176,6 +177,15 @@ def dbl_bn_relu_fused_bwd(shape, dout, dout2, y, out, gamma, save_mean, save_inv
     _check(lib().dbl_bn_relu_fused_bwd(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out), _ptr(gamma),
                                        _ptr(save_mean), _ptr(save_invstd), _ptr(dy), _ptr(dresidual), _ptr(dgamma),
                                        _ptr(dbeta), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def dbl_bn_relu_fused_bwd_noalloc(shape, dout, dout2, y, out, gamma, save_mean, save_invstd, dy, dresidual, dgamma,
+                                  dbeta, stream=None):
+    """dbl_bn_relu_fused_bwd without a workspace argument: the scratch is a fixed array inside
+    the library (channels <= 512; calls must not overlap on the GPU)."""
+    _check(lib().dbl_bn_relu_fused_bwd_noalloc(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out),
+                                               _ptr(gamma), _ptr(save_mean), _ptr(save_invstd), _ptr(dy),
+                                               _ptr(dresidual), _ptr(dgamma), _ptr(dbeta), _stream(stream)))
 
 
 def dbl_maxpool_fwd(n, h, w, c, x, y, argmax, stream=None):
