@@ -308,6 +308,38 @@ def _conv_buffers(wk):
     return out
 
 
+def run_profile_iteration(args, cfg):
+    """One eager dual-batch iteration per stage and nothing else: the command ncu
+    captures for the launch list and the per-kernel captures."""
+    import torch
+
+    from paper_2509_26092_gb300 import build_lib
+    build_lib.build()
+    from paper_2509_26092_gb300 import dbl as D
+    from paper_2509_26092_gb300 import resnet18 as R
+    from paper_2509_26092_gb300 import synth
+
+    torch.cuda.set_device(0)
+    spec = R.ResNet18Spec(cfg["variant"], cfg["classes"])
+    server = R.ServerState(spec, synth.params(spec.table(), seed=0))
+    nat = cfg["native"]
+    n0 = D.dbl_kernel_launches()
+    for res, bl, bs in zip(cfg["stages"], cfg["large"], cfg["small"]):
+        large = R.Worker(spec, bl, res)
+        small = R.Worker(spec, bs, res) if bs else None
+        it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_small=F_SMALL)
+        it.set_inputs(torch.from_numpy(synth.images(bl, nat, nat, 3, seed=1)).cuda(),
+                      torch.from_numpy(synth.labels(bl, cfg["classes"], seed=1)).cuda(),
+                      torch.from_numpy(synth.images(bs, nat, nat, 3, seed=2)).cuda() if bs else None,
+                      torch.from_numpy(synth.labels(bs, cfg["classes"], seed=2)).cuda() if bs else None)
+        it.run()
+        torch.cuda.synchronize()
+        del it, large, small
+    assert D.dbl_device_status() == D.DBL_OK
+    print(json.dumps({"profile_iteration": args.config, "launches": D.dbl_kernel_launches() - n0}), flush=True)
+    return 0
+
+
 def run_ours(args, cfg):
     import torch
     ws, rank, local = _dist()
@@ -446,10 +478,14 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-iteration", action="store_true",
+                    help="run one eager iteration per stage and exit (the command ncu profiles)")
     args = ap.parse_args()
     cfg = CONFIGS[args.config]
     if args.impl == "reference":
         return run_reference(args, cfg)
+    if args.profile_iteration:
+        return run_profile_iteration(args, cfg)
     return run_ours(args, cfg)
 
 
