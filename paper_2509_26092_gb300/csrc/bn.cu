@@ -79,38 +79,45 @@ __global__ void __launch_bounds__(kThreads) bn_stats_kernel(const __nv_bfloat16*
 }
 
 // ----------------------------------------------------------------------------- forward apply
+// Thread t of a CTA owns channel group g = t % (C/8) (8 channels, one 16-byte
+// vector) and visits rows t / (C/8), + rows-per-CTA-step, ...; a warp covers
+// consecutive vectors of consecutive rows, so every access is coalesced, and the
+// channel's scale and shift stay in registers.
 __global__ void __launch_bounds__(kThreads)
     bn_apply_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ res,
                     __nv_bfloat16* __restrict__ out, int64_t count, int C, float eps, int relu,
                     const float* __restrict__ sum, const float* __restrict__ sumsq, const float* __restrict__ gamma,
                     const float* __restrict__ beta, float* __restrict__ save_mean, float* __restrict__ save_invstd)
 {
-    __shared__ float sc[kMaxC], sh[kMaxC];
+    const int groups = C / 8;
+    const int g = threadIdx.x % groups;
+    const int rstep = kThreads / groups;
     const double inv_n = 1.0 / (double)count;
-    for (int c = threadIdx.x; c < C; c += kThreads) {
+    float sc[8], sh[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int c = 8 * g + k;
         const double mean = (double)sum[c] * inv_n;
         double var = (double)sumsq[c] * inv_n - mean * mean;
         if (var < 0.0) var = 0.0;
         const float invstd = (float)(1.0 / sqrt(var + (double)eps));
-        const float scale = gamma[c] * invstd;
-        sc[c] = scale;
-        sh[c] = beta[c] - (float)mean * scale;
-        if (blockIdx.x == 0) {
+        sc[k] = gamma[c] * invstd;
+        sh[k] = beta[c] - (float)mean * sc[k];
+        if (blockIdx.x == 0 && threadIdx.x < groups) {
             save_mean[c] = (float)mean;
             save_invstd[c] = invstd;
         }
     }
-    __syncthreads();
-    const int64_t nvec = count * C / 8;
-    for (int64_t v = (int64_t)blockIdx.x * kThreads + threadIdx.x; v < nvec; v += (int64_t)gridDim.x * kThreads) {
-        const int c0 = (int)((v * 8) % C);
+    const int64_t step = (int64_t)gridDim.x * rstep;
+    for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += step) {
+        const int64_t v = r * groups + g;
         float f[8];
         unpack8(__ldcs(reinterpret_cast<const uint4*>(y) + v), f);
-        float r[8] = {};
-        if (res) unpack8(__ldcs(reinterpret_cast<const uint4*>(res) + v), r);
+        float rr[8] = {};
+        if (res) unpack8(__ldcs(reinterpret_cast<const uint4*>(res) + v), rr);
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            float o = fmaf(f[k], sc[c0 + k], sh[c0 + k]) + r[k];
+            const float o = fmaf(f[k], sc[k], sh[k]) + rr[k];
             f[k] = (relu && !(o > 0.f)) ? 0.f : o;
         }
         reinterpret_cast<uint4*>(out)[v] = pack8(f);
@@ -193,18 +200,32 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
-// Fixed-order sum of the partials (double), then dgamma/dbeta and the three
-// per-channel coefficients of the apply pass.
-__global__ void bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C, int64_t count,
-                                       const float* __restrict__ gamma, const float* __restrict__ invstd,
-                                       float* __restrict__ dgamma, float* __restrict__ dbeta, float* __restrict__ coef)
+// Fixed-order sum of the partials (double; 8 lanes per channel, then 8 -> 1),
+// then dgamma/dbeta and the three per-channel coefficients of the apply pass.
+__global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C,
+                                                              int64_t count, const float* __restrict__ gamma,
+                                                              const float* __restrict__ invstd,
+                                                              float* __restrict__ dgamma, float* __restrict__ dbeta,
+                                                              float* __restrict__ coef)
 {
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= C) return;
+    __shared__ double red[8][2][33];
+    const int c = blockIdx.x * 32 + threadIdx.x % 32;
+    const int l8 = threadIdx.x / 32;
     double sg = 0.0, sgx = 0.0;
-    for (int b = 0; b < nblk; ++b) {
-        sg += partial[(int64_t)b * 2 * C + c];
-        sgx += partial[(int64_t)b * 2 * C + C + c];
+    if (c < C)
+        for (int b = l8; b < nblk; b += 8) {
+            sg += partial[(int64_t)b * 2 * C + c];
+            sgx += partial[(int64_t)b * 2 * C + C + c];
+        }
+    red[l8][0][threadIdx.x % 32] = sg;
+    red[l8][1][threadIdx.x % 32] = sgx;
+    __syncthreads();
+    if (threadIdx.x >= 32 || c >= C) return;
+    sg = 0.0;
+    sgx = 0.0;
+    for (int l = 0; l < 8; ++l) {
+        sg += red[l][0][threadIdx.x];
+        sgx += red[l][1][threadIdx.x];
     }
     dbeta[c] = (float)sg;
     dgamma[c] = (float)sgx;
@@ -219,29 +240,32 @@ __global__ void __launch_bounds__(kThreads)
                         int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
                         const float* __restrict__ coef, __nv_bfloat16* __restrict__ dy, __nv_bfloat16* __restrict__ dres)
 {
-    __shared__ float k1[kMaxC], k2[kMaxC], k3[kMaxC], mu[kMaxC], is[kMaxC];
-    for (int c = threadIdx.x; c < C; c += kThreads) {
-        k1[c] = coef[c];
-        k2[c] = coef[C + c];
-        k3[c] = coef[2 * C + c];
-        mu[c] = mean[c];
-        is[c] = invstd[c];
+    const int groups = C / 8;
+    const int g = threadIdx.x % groups;
+    const int rstep = kThreads / groups;
+    float k1[8], k2[8], k3[8], mu[8], is[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int c = 8 * g + k;
+        k1[k] = coef[c];
+        k2[k] = coef[C + c];
+        k3[k] = coef[2 * C + c];
+        mu[k] = mean[c];
+        is[k] = invstd[c];
     }
-    __syncthreads();
-    const int64_t nvec = count * C / 8;
-    for (int64_t v = (int64_t)blockIdx.x * kThreads + threadIdx.x; v < nvec; v += (int64_t)gridDim.x * kThreads) {
-        const int c0 = (int)((v * 8) % C);
-        float g[8], yy[8], d[8];
-        load_g(dout, dout2, out, relu, v, g);
+    const int64_t step = (int64_t)gridDim.x * rstep;
+    for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += step) {
+        const int64_t v = r * groups + g;
+        float gg[8], yy[8], d[8];
+        load_g(dout, dout2, out, relu, v, gg);
         unpack8(__ldg(reinterpret_cast<const uint4*>(y) + v), yy);
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            const int c = c0 + k;
-            const float xh = (yy[k] - mu[c]) * is[c];
-            d[k] = k1[c] * (g[k] - k2[c] - xh * k3[c]);
+            const float xh = (yy[k] - mu[k]) * is[k];
+            d[k] = k1[k] * (gg[k] - k2[k] - xh * k3[k]);
         }
         reinterpret_cast<uint4*>(dy)[v] = pack8(d);
-        if (dres) reinterpret_cast<uint4*>(dres)[v] = pack8(g);
+        if (dres) reinterpret_cast<uint4*>(dres)[v] = pack8(gg);
     }
 }
 
@@ -336,7 +360,7 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
     bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
                                                          save_mean, save_invstd, rows, partial);
     if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
@@ -416,7 +440,7 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
     bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
                                                          save_mean, save_invstd, rows, partial);
     if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(

@@ -42,11 +42,15 @@ enum Mode : int { kFwd = 0, kDgrad = 1, kWgrad = 2, kFwdC8 = 3, kWgradC8 = 4 };
 
 __device__ int g_conv_status;  // DBL_OK or DBL_ERR_TIMEOUT, read by dbl_device_status()
 
+constexpr int kMaxGrid = 256;     // persistent grid never exceeds this (workspace sizing)
+constexpr int kMaxNcols = 512;    // widest D (output channels of ResNet-18)
+
 struct ConvParams {
     int mode;
     int M;              // D rows (for dgrad: rows of one phase)
     int Ncols;          // D columns
-    int m_tiles, n_tiles;
+    int m_tiles, n_tiles, zdim;  // tile grid; zdim = split-K slices (wgrad) or phases (dgrad)
+    int total_tiles;
     // traversal grid of the im2col operand: (images, rows, cols) and origin of grid point (0,0)
     int gN, gP, gQ;
     int tstride;        // origin step per grid step
@@ -63,9 +67,10 @@ struct ConvParams {
     int phase_off[5];
     int8_t tap_r[16], tap_s[16], tap_oh[16], tap_ow[16];
     // outputs
-    void* out;          // bf16 rows (fwd, dgrad) or fp32 partials (wgrad)
-    int64_t ldo;        // elements between output rows
-    float* stats;       // fwd: [m_tiles][2][Ncols] or nullptr
+    void* out;          // bf16 rows (fwd, dgrad); fp32 dw (wgrad, one slice) or fp32 slices [z][Ncols][M]
+    int64_t ldo;        // elements between output rows (fwd, dgrad)
+    int wg_accumulate;  // wgrad with one slice: add into dw
+    float* stats;       // fwd: [gridDim.x][2][Ncols] per-CTA channel sums, or nullptr
 };
 
 __device__ __forceinline__ void report_timeout(volatile int* abort)
@@ -74,24 +79,41 @@ __device__ __forceinline__ void report_timeout(volatile int* abort)
     atomicExch(&g_conv_status, DBL_ERR_TIMEOUT);
 }
 
-template <int BN, int STAGES>
+template <int BN>
 struct Cfg {
+    static constexpr int STAGES = BN == 256 ? 4 : BN == 128 ? 6 : 8;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = kA_BYTES + B_BYTES;
-    // + 1 KB alignment slack, + 32 KB guard so that no descriptor stride can
-    // make the tensor cores read past the CTA's shared-memory allocation
-    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 32768;
-    static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+    static constexpr int RING = STAGES * STAGE_BYTES;
+    static constexpr int EPI_TILE = 4 * 32 * 33 * 4;           // per-warp 32x32 transpose scratch
+    static constexpr int EPI_SUM = 4 * 2 * kMaxNcols * 4;      // per-warp channel sums (fwd)
+    static constexpr int SMEM = RING + EPI_TILE + EPI_SUM + 1024;  // + 1 KB alignment slack
+    static constexpr uint32_t TMEM_COLS = 2 * BN;               // two accumulators
 };
 
-// Number of K-blocks this CTA reduces, and the first one.
-__device__ __forceinline__ void kb_range(const ConvParams& p, int split, int phase, int& kb0, int& nkb)
+struct TileCoord {
+    int m_tile, n_tile, z;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(const ConvParams& p, int t)
+{
+    const int mn = p.m_tiles * p.n_tiles;
+    TileCoord c;
+    c.z = t / mn;
+    const int r = t - c.z * mn;
+    c.m_tile = r / p.n_tiles;
+    c.n_tile = r - c.m_tile * p.n_tiles;
+    return c;
+}
+
+// Number of K-blocks a tile reduces, and the first one.
+__device__ __forceinline__ void kb_range(const ConvParams& p, int z, int& kb0, int& nkb)
 {
     if (p.mode == kDgrad) {
         kb0 = 0;
-        nkb = (p.phase_off[phase + 1] - p.phase_off[phase]) * p.cblocks;
+        nkb = (p.phase_off[z + 1] - p.phase_off[z]) * p.cblocks;
     } else if (p.mode == kWgrad || p.mode == kWgradC8) {
-        kb0 = split * p.kb_per_split;
+        kb0 = z * p.kb_per_split;
         nkb = min(p.num_kb, kb0 + p.kb_per_split) - kb0;
         if (nkb < 0) nkb = 0;
     } else {
@@ -100,37 +122,96 @@ __device__ __forceinline__ void kb_range(const ConvParams& p, int split, int pha
     }
 }
 
-template <int BN, int STAGES>
+// Issue the TMA loads of one K-block of one tile into ring stage (sa, sb).
+__device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorMap* tmA, const CUtensorMap* tmB,
+                                            int BN, uint8_t* sa, uint8_t* sb, uint64_t* fb, const TileCoord& tc,
+                                            int kb, int tn, int tp, int tq)
+{
+    const int64_t gPQ = (int64_t)p.gP * p.gQ;
+    if (p.mode == kFwd) {
+        const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
+        const int r = tap / p.S, sx = tap - r * p.S;
+        tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
+                           (uint16_t)sx, (uint16_t)r);
+        tma_load_2d(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
+    } else if (p.mode == kDgrad) {
+        const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
+        tma_load_im2col_4d(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
+                           (uint16_t)p.tap_oh[t]);
+        const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
+        for (int j = 0; j < BN / 64; ++j) tma_load_3d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
+    } else if (p.mode == kWgrad || p.mode == kWgradC8) {
+        const int64_t pix0 = (int64_t)kb * 64;
+        const int n = (int)(pix0 / gPQ);
+        const int64_t rem = pix0 - (int64_t)n * gPQ;
+        const int pp = (int)(rem / p.gQ), qq = (int)(rem - (int64_t)pp * p.gQ);
+        if (p.mode == kWgrad) {
+            for (int h = 0; h < 2; ++h) {
+                const int mrow = tc.m_tile * BM + 64 * h;
+                int tap = mrow / p.Cin;
+                const int c0 = mrow - tap * p.Cin;
+                if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
+                tma_load_im2col_4d(sa + h * 8192, tmA, fb, c0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h,
+                                   n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+            }
+        } else {  // 16 taps x 8 channels of rows
+            for (int j = 0; j < 16; ++j) {
+                int tap = tc.m_tile * 16 + j;
+                if (tap >= p.ntaps) tap = 0;
+                tma_load_im2col_4d(sa + j * 1024, tmA, fb, 0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
+                                   (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+            }
+        }
+        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
+    } else {  // kFwdC8: 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
+        for (int j = 0; j < 8; ++j) {
+            int tap = kb * 8 + j;
+            const int wcol = tap * 8;
+            if (tap >= p.ntaps) tap = p.ntaps - 1;
+            tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
+                               (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+            tma_load_2d(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
+        }
+    }
+}
+
+// Persistent kernel: CTA b processes tiles b, b + gridDim.x, ...  The ring of
+// STAGES shared-memory stages runs continuously across tiles; two TMEM
+// accumulators let the epilogue of one tile overlap the MMAs of the next.
+template <int BN>
 __global__ void __launch_bounds__(192, 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const ConvParams p)
 {
-    using C = Cfg<BN, STAGES>;
+    using C = Cfg<BN>;
+    constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accum_bar;
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accf_bar[2], acce_bar[2], drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
     uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
-
-    const int n_tile = blockIdx.x % p.n_tiles;
-    const int m_tile = blockIdx.x / p.n_tiles;
-    const int split = (p.mode == kWgrad || p.mode == kWgradC8) ? blockIdx.y : 0;
-    const int phase = p.mode == kDgrad ? blockIdx.y : 0;
-    int kb0, nkb;
-    kb_range(p, split, phase, kb0, nkb);
+    float* epi_tile = reinterpret_cast<float*>(sgen + C::RING);
+    float* epi_sum = reinterpret_cast<float*>(sgen + C::RING + C::EPI_TILE);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        mbar_init(&accum_bar, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&accf_bar[b], 1);
+            mbar_init(&acce_bar[b], 4);  // one arrival per epilogue warp
+        }
+        mbar_init(&drain_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
     }
+    const bool want_stats = (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
+    if (want_stats)
+        for (int i = threadIdx.x; i < 4 * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
     if (warp == 4 && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
@@ -143,94 +224,37 @@ __global__ void __launch_bounds__(192, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
-
-    // Start of the tile's im2col traversal (fwd, dgrad): row m_tile*BM of the grid.
-    const int64_t m0 = (int64_t)m_tile * BM;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
 
     if (warp == 4) {
         // ------------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            int tn = 0, tp = 0, tq = 0;
-            if (p.mode == kFwd || p.mode == kDgrad || p.mode == kFwdC8) {
-                tn = (int)(m0 / gPQ);
-                const int64_t rem = m0 % gPQ;
-                tp = (int)(rem / p.gQ);
-                tq = (int)(rem % p.gQ);
-            }
-            const uint32_t tx_bytes = (uint32_t)C::STAGE_BYTES;
             int it = 0;
-            for (; it < nkb; ++it) {
-                const int s = it % STAGES;
-                if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
-                    report_timeout(&abort_flag);
-                    break;
+            for (int t = blockIdx.x; t < p.total_tiles && !abort_flag; t += gridDim.x) {
+                const TileCoord tc = decode_tile(p, t);
+                int kb0, nkb;
+                kb_range(p, tc.z, kb0, nkb);
+                int tn = 0, tp = 0, tq = 0;
+                if (p.mode == kFwd || p.mode == kDgrad || p.mode == kFwdC8) {
+                    const int64_t m0 = (int64_t)tc.m_tile * BM;
+                    tn = (int)(m0 / gPQ);
+                    const int64_t rem = m0 - (int64_t)tn * gPQ;
+                    tp = (int)(rem / p.gQ);
+                    tq = (int)(rem - (int64_t)tp * p.gQ);
                 }
-                uint8_t* sa = sgen + s * C::STAGE_BYTES;
-                uint8_t* sb = sa + kA_BYTES;
-                uint64_t* fb = &full_bar[s];
-                mbar_arrive_expect_tx(fb, tx_bytes);
-                const int kb = kb0 + it;
-                if (p.mode == kFwd) {
-                    const int tap = kb / p.cblocks, cb = kb % p.cblocks;
-                    const int r = tap / p.S, sx = tap % p.S;
-                    tma_load_im2col_4d(sa, &tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h,
-                                       tn, (uint16_t)sx, (uint16_t)r);
-                    tma_load_2d(sb, &tmB, fb, tap * p.Cin + cb * 64, n_tile * BN);
-                } else if (p.mode == kDgrad) {
-                    const int t = p.phase_off[phase] + kb / p.cblocks, kbk = kb % p.cblocks;
-                    tma_load_im2col_4d(sa, &tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn,
-                                       (uint16_t)p.tap_ow[t], (uint16_t)p.tap_oh[t]);
-                    const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
-#pragma unroll
-                    for (int j = 0; j < BN / 64; ++j)
-                        tma_load_3d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, wtap, kbk * 64);
-                } else if (p.mode == kWgrad) {
-                    const int64_t pix0 = (int64_t)kb * 64;
-                    const int n = (int)(pix0 / gPQ);
-                    const int64_t rem = pix0 % gPQ;
-                    const int pp = (int)(rem / p.gQ), qq = (int)(rem % p.gQ);
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int mrow = m_tile * BM + 64 * h;
-                        int tap = mrow / p.Cin;
-                        const int c0 = mrow % p.Cin;
-                        if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
-                        tma_load_im2col_4d(sa + h * 8192, &tmA, fb, c0, qq * p.tstride + p.base_w,
-                                           pp * p.tstride + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                for (int k = 0; k < nkb; ++k, ++it) {
+                    const int s = it % STAGES;
+                    if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
+                        report_timeout(&abort_flag);
+                        break;
                     }
-#pragma unroll
-                    for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, (int)pix0);
-                } else if (p.mode == kFwdC8) {
-                    // 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        int tap = kb * 8 + j;
-                        const int wcol = tap * 8;
-                        if (tap >= p.ntaps) tap = p.ntaps - 1;
-                        tma_load_im2col_4d(sa + j * 2048, &tmA, fb, 0, tq * p.tstride + p.base_w,
-                                           tp * p.tstride + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
-                        tma_load_2d(sb + j * (BN * 16), &tmB, fb, wcol, n_tile * BN);
-                    }
-                } else {  // kWgradC8: 16 taps x 8 channels of rows, 64 pixels
-                    const int64_t pix0 = (int64_t)kb * 64;
-                    const int n = (int)(pix0 / gPQ);
-                    const int64_t rem = pix0 % gPQ;
-                    const int pp = (int)(rem / p.gQ), qq = (int)(rem % p.gQ);
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        int tap = m_tile * 16 + j;
-                        if (tap >= p.ntaps) tap = 0;
-                        tma_load_im2col_4d(sa + j * 1024, &tmA, fb, 0, qq * p.tstride + p.base_w,
-                                           pp * p.tstride + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
-                    }
-#pragma unroll
-                    for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &tmB, fb, n_tile * BN + 64 * j, (int)pix0);
+                    uint8_t* sa = sgen + s * C::STAGE_BYTES;
+                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)C::STAGE_BYTES);
+                    load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
                 }
             }
             if (abort_flag) {
-                // let copies already issued land before the CTA's shared memory goes away:
-                // for each stage, wait (time-bounded, ignoring the abort flag) for its last issued phase
+                // let copies already issued land before the CTA's shared memory goes away
                 for (int s = 0; s < STAGES && s < it; ++s) {
                     const int last = s + STAGES * ((it - 1 - s) / STAGES);
                     (void)mbar_wait_drain(&full_bar[s], (last / STAGES) & 1);
@@ -244,132 +268,158 @@ __global__ void __launch_bounds__(192, 1)
             const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
             const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
             const uint32_t idesc = idesc_bf16(BM, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
-            for (int it = 0; it < nkb; ++it) {
-                const int s = it % STAGES;
-                if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
+            int it = 0, lt = 0;
+            for (int t = blockIdx.x; t < p.total_tiles && !abort_flag; t += gridDim.x, ++lt) {
+                const TileCoord tc = decode_tile(p, t);
+                int kb0, nkb;
+                kb_range(p, tc.z, kb0, nkb);
+                const int buf = lt & 1;
+                if (!mbar_wait(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag)) {
                     report_timeout(&abort_flag);
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = sbase + s * C::STAGE_BYTES;
-                const uint32_t sb = sa + kA_BYTES;
-#pragma unroll
-                for (int j = 0; j < BK / 16; ++j) {
-                    uint64_t ad, bd;
-                    if (p.mode == kFwd) {
-                        ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
-                        bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
-                    } else if (p.mode == kDgrad) {
-                        ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
-                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                    } else if (p.mode == kWgrad) {
-                        ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
-                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                    } else if (p.mode == kFwdC8) {
-                        // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
-                        // 8-row groups 128 B apart (SBO), the two taps of one MMA 2 KB apart (LBO)
-                        ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
-                        bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
-                    } else {
-                        // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
-                        // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
-                        ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
-                        bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                const uint32_t d = tmem + (uint32_t)(buf * BN);
+                bool ok = true;
+                for (int k = 0; k < nkb; ++k, ++it) {
+                    const int s = it % STAGES;
+                    if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
+                        report_timeout(&abort_flag);
+                        ok = false;
+                        break;
                     }
-                    mma_bf16(tmem, ad, bd, idesc, (it > 0 || j > 0) ? 1u : 0u);
+                    tc_fence_after();
+                    const uint32_t sa = sbase + s * C::STAGE_BYTES;
+                    const uint32_t sb = sa + kA_BYTES;
+#pragma unroll
+                    for (int j = 0; j < BK / 16; ++j) {
+                        uint64_t ad, bd;
+                        if (p.mode == kFwd) {
+                            ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
+                        } else if (p.mode == kDgrad) {
+                            ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                        } else if (p.mode == kWgrad) {
+                            ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                        } else if (p.mode == kFwdC8) {
+                            // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
+                            // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
+                            ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
+                            bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
+                        } else {
+                            // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
+                            // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
+                            ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
+                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                        }
+                        mma_bf16(d, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
+                    }
+                    mma_commit(&empty_bar[s]);
                 }
-                mma_commit(&empty_bar[s]);
+                mma_commit(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
+                if (!ok) break;
             }
-            mma_commit(&accum_bar);  // arrives when every MMA issued above has completed
+            // every MMA issued above completes before the accumulators are freed
+            mma_commit(&drain_bar);
+            (void)mbar_wait_drain(&drain_bar, 0);
         }
         __syncwarp();
     } else {
         // ------------------------------------------------------------------ epilogue (warps 0-3)
-        const bool ok = mbar_wait(&accum_bar, 0, &abort_flag);
-        if (!ok) report_timeout(&abort_flag);
-        tc_fence_after();
-        const int row = warp * 32 + lane;  // TMEM lane = tile row
-        const int64_t m = m0 + row;
-        const bool valid = m < p.M;
-        const bool have_acc = nkb > 0 && ok;
-        float* st_tile = reinterpret_cast<float*>(sgen) + warp * 32 * 33;  // stats transpose scratch
-        float* colsum = reinterpret_cast<float*>(sgen) + 4 * 32 * 33;       // [4][2][BN]
-        const bool want_stats = (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
-
-        int64_t out_row = m;
-        if (p.mode == kDgrad && p.phase_div == 2) {
-            const int64_t hw = (int64_t)p.gP * p.gQ;
-            const int64_t n = m / hw, rem = m % hw;
-            const int i = (int)(rem / p.gQ), j = (int)(rem % p.gQ);
-            const int a = phase >> 1, b = phase & 1;
-            out_row = (n * p.out_h + 2 * i + a) * p.out_w + 2 * j + b;
-        }
+        float* st_tile = epi_tile + warp * 32 * 33;
+        float* wsum = epi_sum + warp * 2 * p.Ncols;
+        int lt = 0;
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
+            const TileCoord tc = decode_tile(p, t);
+            int kb0, nkb;
+            kb_range(p, tc.z, kb0, nkb);
+            const int buf = lt & 1;
+            const bool ok = mbar_wait(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
+            if (!ok) {
+                report_timeout(&abort_flag);
+                break;
+            }
+            tc_fence_after();
+            const int row = warp * 32 + lane;  // TMEM lane = tile row
+            const int64_t m = (int64_t)tc.m_tile * BM + row;
+            const bool valid = m < p.M;
+            const bool have_acc = nkb > 0;
+            int64_t out_row = m;
+            if (p.mode == kDgrad && p.phase_div == 2) {
+                const int64_t n = m / gPQ, rem = m - n * gPQ;
+                const int i = (int)(rem / p.gQ), j = (int)(rem - (int64_t)(rem / p.gQ) * p.gQ);
+                const int a = tc.z >> 1, b = tc.z & 1;
+                out_row = (n * p.out_h + 2 * i + a) * p.out_w + 2 * j + b;
+            }
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * BN);
 #pragma unroll 1
-        for (int ch = 0; ch < BN / 32; ++ch) {
-            uint32_t v[32];
-            if (have_acc) {
-                tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + ch * 32, v);
-                tmem_ld_wait();
-            } else {
+            for (int ch = 0; ch < BN / 32; ++ch) {
+                uint32_t v[32];
+                if (have_acc) {
+                    tmem_ld_32x32b_x32(taddr + ch * 32, v);
+                    tmem_ld_wait();
+                } else {
 #pragma unroll
-                for (int k = 0; k < 32; ++k) v[k] = 0u;
-            }
-            const int col0 = n_tile * BN + ch * 32;
-            if (p.mode == kWgrad || p.mode == kWgradC8) {
-                if (valid) {
-                    float* o = static_cast<float*>(p.out) + ((int64_t)split * p.M + m) * p.ldo + col0;
-#pragma unroll
-                    for (int k = 0; k < 32; k += 4)
-                        *reinterpret_cast<float4*>(o + k) = make_float4(__uint_as_float(v[k]), __uint_as_float(v[k + 1]),
-                                                                        __uint_as_float(v[k + 2]), __uint_as_float(v[k + 3]));
+                    for (int k = 0; k < 32; ++k) v[k] = 0u;
                 }
-            } else {
-                uint4 pk[4];
-                __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
-                float rv[32];
+                const int col0 = tc.n_tile * BN + ch * 32;
+                if (p.mode == kWgrad || p.mode == kWgradC8) {
+                    // D row m = (tap, c), column = output channel k; stored as [slice][k][m]:
+                    // consecutive lanes hold consecutive m, so each store is one 128-byte line
+                    if (valid) {
+                        float* o = static_cast<float*>(p.out) + ((int64_t)tc.z * p.Ncols + col0) * p.M + m;
+                        if (p.zdim == 1 && p.wg_accumulate) {
 #pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
-                    const float2 back = __bfloat1622float2(h2[k]);
-                    rv[2 * k] = back.x;
-                    rv[2 * k + 1] = back.y;
-                }
-                if (valid) {
-                    uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
+                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] += __uint_as_float(v[k]);
+                        } else {
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) o[k] = pk[k];
-                }
-                if (want_stats) {
-                    // column sums of the stored values over this warp's 32 rows
-#pragma unroll
-                    for (int k = 0; k < 32; ++k) st_tile[lane * 33 + k] = valid ? rv[k] : 0.f;
-                    __syncwarp();
-                    float s = 0.f, q = 0.f;
-#pragma unroll 8
-                    for (int r = 0; r < 32; ++r) {
-                        const float x = st_tile[r * 33 + lane];
-                        s += x;
-                        q = fmaf(x, x, q);
+                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] = __uint_as_float(v[k]);
+                        }
                     }
-                    colsum[(warp * 2 + 0) * BN + ch * 32 + lane] = s;
-                    colsum[(warp * 2 + 1) * BN + ch * 32 + lane] = q;
-                    __syncwarp();
+                } else {
+                    uint4 pk[4];
+                    __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
+#pragma unroll
+                    for (int k = 0; k < 16; ++k)
+                        h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
+                    if (valid) {
+                        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) o[k] = pk[k];
+                    }
+                    if (want_stats) {
+                        // column sums of the stored (rounded) values over this warp's 32 rows
+#pragma unroll
+                        for (int k = 0; k < 16; ++k) {
+                            const float2 back = __bfloat1622float2(h2[k]);
+                            st_tile[lane * 33 + 2 * k] = valid ? back.x : 0.f;
+                            st_tile[lane * 33 + 2 * k + 1] = valid ? back.y : 0.f;
+                        }
+                        __syncwarp();
+                        float s = 0.f, q = 0.f;
+#pragma unroll 8
+                        for (int r = 0; r < 32; ++r) {
+                            const float x = st_tile[r * 33 + lane];
+                            s += x;
+                            q = fmaf(x, x, q);
+                        }
+                        wsum[col0 + lane] += s;
+                        wsum[p.Ncols + col0 + lane] += q;
+                        __syncwarp();
+                    }
                 }
             }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce_bar[buf]);
         }
         if (want_stats) {
             asm volatile("bar.sync 1, 128;" ::: "memory");
-            for (int c = threadIdx.x; c < BN; c += 128) {
-                float s = 0.f, q = 0.f;
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    s += colsum[(w * 2 + 0) * BN + c];
-                    q += colsum[(w * 2 + 1) * BN + c];
-                }
-                float* dst = p.stats + (int64_t)m_tile * 2 * p.Ncols;
-                dst[n_tile * BN + c] = s;
-                dst[p.Ncols + n_tile * BN + c] = q;
-            }
+            float* dst = p.stats + (int64_t)blockIdx.x * 2 * p.Ncols;
+            for (int c = threadIdx.x; c < 2 * p.Ncols; c += 128)
+                dst[c] = (epi_sum[c] + epi_sum[2 * p.Ncols + c]) + (epi_sum[4 * p.Ncols + c] + epi_sum[6 * p.Ncols + c]);
         }
     }
     tc_fence_before();
@@ -381,21 +431,21 @@ __global__ void __launch_bounds__(192, 1)
 }
 
 // ----------------------------------------------------------------------------- reductions
-// Stage 1: per 64-tile chunk and 32 channels, fixed-order sums of the tile partials.
-__global__ void stats_reduce1_kernel(const float* __restrict__ part, int tiles, int K, double* __restrict__ lvl2)
+// Per-channel sums over the per-CTA partials, fixed order: 8 lanes per channel, then 8 -> 1.
+__global__ void stats_reduce_kernel(const float* __restrict__ part, int nparts, int K, float* __restrict__ sum,
+                                    float* __restrict__ sumsq)
 {
     __shared__ double red[8][2][33];
     const int c = blockIdx.x * 32 + threadIdx.x % 32;
-    const int lane8 = threadIdx.x / 32;
-    const int t0 = blockIdx.y * 64, t1 = min(tiles, t0 + 64);
+    const int l8 = threadIdx.x / 32;
     double s = 0.0, q = 0.0;
     if (c < K)
-        for (int t = t0 + lane8; t < t1; t += 8) {
+        for (int t = l8; t < nparts; t += 8) {
             s += part[(int64_t)t * 2 * K + c];
             q += part[(int64_t)t * 2 * K + K + c];
         }
-    red[lane8][0][threadIdx.x % 32] = s;
-    red[lane8][1][threadIdx.x % 32] = q;
+    red[l8][0][threadIdx.x % 32] = s;
+    red[l8][1][threadIdx.x % 32] = q;
     __syncthreads();
     if (threadIdx.x < 32 && c < K) {
         double ts = 0.0, tq = 0.0;
@@ -403,46 +453,32 @@ __global__ void stats_reduce1_kernel(const float* __restrict__ part, int tiles, 
             ts += red[l][0][threadIdx.x];
             tq += red[l][1][threadIdx.x];
         }
-        lvl2[(int64_t)blockIdx.y * 2 * K + c] = ts;
-        lvl2[(int64_t)blockIdx.y * 2 * K + K + c] = tq;
+        sum[c] = (float)ts;
+        sumsq[c] = (float)tq;
     }
 }
 
-__global__ void stats_reduce2_kernel(const double* __restrict__ lvl2, int chunks, int K, float* __restrict__ sum,
-                                     float* __restrict__ sumsq)
+// dw[i] (+)= sum over slices of part[slice][i], slices in a fixed order; i runs over the
+// KRSC weight gradient (the slices are already in that layout).
+__global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restrict__ part, int slices, int64_t n,
+                                                           float* __restrict__ dw, int accumulate)
 {
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= K) return;
-    double s = 0.0, q = 0.0;
-    for (int i = 0; i < chunks; ++i) {
-        s += lvl2[(int64_t)i * 2 * K + c];
-        q += lvl2[(int64_t)i * 2 * K + K + c];
-    }
-    sum[c] = (float)s;
-    sumsq[c] = (float)q;
-}
-
-// dw[k][m] (+)= sum over splits of part[split][m][k], fixed split order; 32x32 transpose tiles.
-__global__ void wgrad_reduce_kernel(const float* __restrict__ part, int splits, int M, int K, float* __restrict__ dw,
-                                    int accumulate)
-{
-    __shared__ float t[32][33];
-    const int k0 = blockIdx.x * 32, mb = blockIdx.y * 32;
-    const int tx = threadIdx.x % 32, ty = threadIdx.x / 32;  // 32 x 8 threads
-    for (int i = ty; i < 32; i += 8) {
-        const int m = mb + i, k = k0 + tx;
-        float s = 0.f;
-        if (m < M && k < K)
-            for (int sp = 0; sp < splits; ++sp) s += part[((int64_t)sp * M + m) * K + k];
-        t[i][tx] = s;
-    }
-    __syncthreads();
-    for (int i = ty; i < 32; i += 8) {
-        const int k = k0 + i, m = mb + tx;
-        if (k < K && m < M) {
-            float* d = dw + (int64_t)k * M + m;
-            *d = accumulate ? *d + t[tx][i] : t[tx][i];
+    const int64_t n4 = n >> 2;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+        float4 acc = accumulate ? reinterpret_cast<const float4*>(dw)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s = 0; s < slices; ++s) {
+            const float4 v = __ldcs(reinterpret_cast<const float4*>(part + (int64_t)s * n) + i);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
         }
+        reinterpret_cast<float4*>(dw)[i] = acc;
+    }
+    for (int64_t i = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        float acc = accumulate ? dw[i] : 0.f;
+        for (int s = 0; s < slices; ++s) acc += part[(int64_t)s * n + i];
+        dw[i] = acc;
     }
 }
 
@@ -451,15 +487,14 @@ struct Plan {
     int mode;
     int BN;
     ConvParams p;
-    dim3 grid;
-    size_t ws_part = 0, ws_lvl2 = 0;  // bytes: split-K partials or tile stats; stats level 2
-    int stat_chunks = 0;
+    size_t ws_main = 0;  // bytes: fwd channel-sum partials, or wgrad split-K slices
 };
 
 int out_dim(int in, int k, int st, int pad) { return (in + 2 * pad - k) / st + 1; }
 
 int choose_bn(int cols)
 {
+    if (cols % 256 == 0) return 256;
     if (cols % 128 == 0) return 128;
     return 64;
 }
@@ -474,11 +509,23 @@ int validate(const dbl_conv_shape* s, const char* who)
     if (s->r != s->s) return set_error(DBL_ERR_UNSUPPORTED, "%s: only square filters", who);
     if (s->c % 8) return set_error(DBL_ERR_INVALID, "%s: channels must be a multiple of 8", who);
     if (s->k % 64) return set_error(DBL_ERR_UNSUPPORTED, "%s: output channels must be a multiple of 64", who);
+    if (s->k > kMaxNcols || s->c > kMaxNcols * 8)
+        return set_error(DBL_ERR_UNSUPPORTED, "%s: at most %d output channels", who, kMaxNcols);
     if (s->stride > 2 || s->r > 7 || s->pad > 3)
         return set_error(DBL_ERR_UNSUPPORTED, "%s: stride <= 2, filter <= 7, pad <= 3 supported", who);
     if (out_dim(s->h, s->r, s->stride, s->pad) <= 0 || out_dim(s->w, s->s, s->stride, s->pad) <= 0)
         return set_error(DBL_ERR_INVALID, "%s: empty output", who);
     return DBL_OK;
+}
+
+// Persistent grid: one CTA per SM (the kernel uses ~225 KB of shared memory), never more
+// CTAs than tiles, never more than kMaxGrid (the workspace is sized for that bound).
+int grid_size(int total_tiles)
+{
+    int g = dbl::sm_count();
+    if (g > kMaxGrid) g = kMaxGrid;
+    if (g > total_tiles) g = total_tiles;
+    return g < 1 ? 1 : g;
 }
 
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
@@ -494,10 +541,13 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
     p.ntaps = s->r * s->s;
     p.S = s->s;
     p.Cin = s->c;
+    p.zdim = 1;
     if (pass == DBL_PASS_FWD) {
         pl.mode = p.mode = c8 ? kFwdC8 : kFwd;
         if (c8 && p.ntaps > 56) return set_error(DBL_ERR_UNSUPPORTED, "conv_fwd: stem filter too large");
-        p.M = s->n * P * Q;
+        const int64_t M = (int64_t)s->n * P * Q;
+        if (M > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_fwd: too many output pixels");
+        p.M = (int)M;
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
         p.m_tiles = (p.M + BM - 1) / BM;
@@ -510,10 +560,7 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.cblocks = c8 ? 1 : s->c / 64;
         p.num_kb = c8 ? (p.ntaps + 7) / 8 : p.ntaps * p.cblocks;
         p.ldo = s->k;
-        pl.grid = dim3(p.m_tiles * p.n_tiles, 1, 1);
-        pl.ws_part = (size_t)p.m_tiles * 2 * s->k * sizeof(float);
-        pl.stat_chunks = (p.m_tiles + 63) / 64;
-        pl.ws_lvl2 = (size_t)pl.stat_chunks * 2 * s->k * sizeof(double);
+        pl.ws_main = (size_t)kMaxGrid * 2 * s->k * sizeof(float);
     } else if (pass == DBL_PASS_DGRAD) {
         if (c8) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: the 8-channel stem has no data gradient path");
         pl.mode = p.mode = kDgrad;
@@ -546,11 +593,13 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
                     ++t;
                 }
             p.phase_off[1] = t;
-            pl.grid = dim3((unsigned)(((p.M + BM - 1) / BM) * p.n_tiles), 1, 1);
         } else {
             if ((s->h & 1) || (s->w & 1) || P * 2 != s->h || Q * 2 != s->w)
                 return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride 2 needs even H, W with P = H/2");
+            for (int r = 0; r < s->r; ++r)
+                if (r > 1 + s->pad) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride-2 filter too large for pad");
             p.phase_div = 2;
+            p.zdim = 4;
             p.gP = s->h / 2;
             p.gQ = s->w / 2;
             p.M = s->n * p.gP * p.gQ;
@@ -575,24 +624,14 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
                 }
             }
             p.phase_off[4] = t;
-            // taps that would read dy at a negative offset are not representable (none for ResNet-18)
-            for (int r = 0; r < s->r; ++r)
-                if (r > 1 + s->pad) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: stride-2 filter too large for pad");
-            pl.grid = dim3((unsigned)(((p.M + BM - 1) / BM) * p.n_tiles), 4, 1);
         }
         p.m_tiles = (p.M + BM - 1) / BM;
     } else {
         pl.mode = p.mode = c8 ? kWgradC8 : kWgrad;
-        const int64_t Mrows = (int64_t)p.ntaps * s->c;  // D rows = (tap, c)
-        p.M = (int)Mrows;
+        p.M = p.ntaps * s->c;  // D rows = (tap, c)
         p.Ncols = s->k;
-        pl.BN = choose_bn(s->k);
-        if (c8) {
-            pl.BN = 64;
-            p.m_tiles = (p.ntaps + 15) / 16;
-        } else {
-            p.m_tiles = (p.M + BM - 1) / BM;
-        }
+        pl.BN = c8 ? 64 : choose_bn(s->k);
+        p.m_tiles = c8 ? (p.ntaps + 15) / 16 : (p.M + BM - 1) / BM;
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;
         p.gP = P;
@@ -600,21 +639,24 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.tstride = s->stride;
         p.base_h = p.base_w = -s->pad;
         const int64_t pix = (int64_t)s->n * P * Q;
+        if ((pix + 63) / 64 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
         p.num_kb = (int)((pix + 63) / 64);
         const int tiles = p.m_tiles * p.n_tiles;
+        // split the pixel reduction so that there are about two tiles per SM of a 152-SM GPU,
+        // keeping at least 8 K-blocks per slice (a fixed function of the shape)
         int splits = (kTargetCTAs + tiles - 1) / tiles;
-        if (splits > p.num_kb) splits = p.num_kb;
+        if (splits > p.num_kb / 8) splits = p.num_kb / 8;
         if (splits < 1) splits = 1;
         p.kb_per_split = (p.num_kb + splits - 1) / splits;
         splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
-        p.ldo = s->k;
-        pl.grid = dim3((unsigned)tiles, (unsigned)splits, 1);
-        pl.ws_part = (size_t)splits * p.M * s->k * sizeof(float);
+        p.zdim = splits;
+        pl.ws_main = splits > 1 ? (size_t)splits * p.M * s->k * sizeof(float) : 0;
     }
+    p.total_tiles = p.m_tiles * p.n_tiles * p.zdim;
     return DBL_OK;
 }
 
-size_t plan_ws(const Plan& pl) { return ((pl.ws_part + 255) / 256) * 256 + ((pl.ws_lvl2 + 255) / 256) * 256; }
+size_t plan_ws(const Plan& pl) { return ((pl.ws_main + 255) / 256) * 256; }
 
 int enc_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int lower, int upper, int stride,
                int channels, int pixels, bool swizzle)
@@ -647,27 +689,27 @@ int enc_tiled(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims
     return DBL_OK;
 }
 
-template <int BN, int STAGES>
-int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t st)
+template <int BN>
+int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
-    using Cf = Cfg<BN, STAGES>;
+    using Cf = Cfg<BN>;
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             Cf::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::SMEM);
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_igemm_kernel<BN, STAGES><<<pl.grid, 192, Cf::SMEM, st>>>(a, b, pl.p);
+    conv_igemm_kernel<BN><<<grid, 192, Cf::SMEM, st>>>(a, b, pl.p);
     return dbl::launch_check("conv_igemm launch");
 }
 
-int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t st)
+int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
-    if (pl.BN == 128) return launch_cfg<128, 4>(pl, a, b, st);
-    return launch_cfg<64, 4>(pl, a, b, st);
+    if (pl.BN == 256) return launch_cfg<256>(pl, a, b, grid, st);
+    if (pl.BN == 128) return launch_cfg<128>(pl, a, b, grid, st);
+    return launch_cfg<64>(pl, a, b, grid, st);
 }
 
 }  // namespace
@@ -678,7 +720,6 @@ size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass)
 {
     Plan pl;
     if (pass < 0 || pass > 2 || make_plan(shape, pass, pl) != DBL_OK) return 0;
-    if (pass == DBL_PASS_DGRAD) return 0;
     return plan_ws(pl);
 }
 
@@ -697,8 +738,6 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
     if (stats && (!ws || ws_bytes < plan_ws(pl)))
         return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
     CUtensorMap ta, tb;
-    const int P = out_dim(s->h, s->r, s->stride, s->pad);
-    (void)P;
     if (pl.mode == kFwdC8) {
         if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -s->pad, s->pad - (s->r - 1), s->stride, 8, BM, false)))
             return rc;
@@ -716,18 +755,14 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
     }
-    uint8_t* wsb = static_cast<uint8_t*>(ws);
     pl.p.out = y;
-    pl.p.stats = stats ? reinterpret_cast<float*>(wsb) : nullptr;
+    pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
+    const int grid = grid_size(pl.p.total_tiles);
     cudaStream_t st = as_stream(stream);
-    if ((rc = launch(pl, ta, tb, st))) return rc;
+    if ((rc = launch(pl, ta, tb, grid, st))) return rc;
     if (stats) {
-        double* lvl2 = reinterpret_cast<double*>(wsb + ((pl.ws_part + 255) / 256) * 256);
-        stats_reduce1_kernel<<<dim3((s->k + 31) / 32, pl.stat_chunks), 256, 0, st>>>(pl.p.stats, pl.p.m_tiles, s->k,
-                                                                                      lvl2);
-        if ((rc = launch_check("conv stats reduce1"))) return rc;
-        stats_reduce2_kernel<<<(s->k + 127) / 128, 128, 0, st>>>(lvl2, pl.stat_chunks, s->k, ch_sum, ch_sumsq);
-        if ((rc = launch_check("conv stats reduce2"))) return rc;
+        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
+        if ((rc = launch_check("conv stats reduce"))) return rc;
     }
     return DBL_OK;
 }
@@ -746,14 +781,10 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
     const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
     CUtensorMap ta, tb;
     // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
-    int lower, upper;
+    int lower = 0, upper = 0;
     if (s->stride == 1) {
         lower = -(s->r - 1 - s->pad);
-        upper = -s->pad;  // origin range [lower, H-1+lower] expressed against dy's extent P
-        upper = (s->h - 1 + lower) - (P - 1);
-    } else {
-        lower = 0;
-        upper = 0;
+        upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
     }
     if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, 1, 64, BM, true))) return rc;
     // w viewed as [k][r*s][c]: inner c, then tap, then k
@@ -762,7 +793,7 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
     cuuint32_t box[3] = {64, 1, 64};
     if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
     pl.p.out = dx;
-    return launch(pl, ta, tb, as_stream(stream));
+    return launch(pl, ta, tb, grid_size(pl.p.total_tiles), as_stream(stream));
 }
 
 int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float* dw, int accumulate, void* ws,
@@ -774,7 +805,7 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     if (rc) return rc;
     if (!x || !dy || !dw || !aligned16(x) || !aligned16(dy) || !aligned16(dw))
         return set_error(DBL_ERR_INVALID, "conv_wgrad: null or misaligned tensor");
-    if (!ws || ws_bytes < plan_ws(pl))
+    if (plan_ws(pl) && (!ws || ws_bytes < plan_ws(pl)))
         return set_error(DBL_ERR_WORKSPACE, "conv_wgrad: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
     const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
     CUtensorMap ta, tb;
@@ -786,12 +817,18 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     cuuint64_t str[1] = {(cuuint64_t)s->k * 2};
     cuuint32_t box[2] = {64, 64};
     if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
-    pl.p.out = ws;
+    const bool sliced = pl.p.zdim > 1;
+    pl.p.out = sliced ? ws : static_cast<void*>(dw);
+    pl.p.wg_accumulate = accumulate;
     cudaStream_t st = as_stream(stream);
-    if ((rc = launch(pl, ta, tb, st))) return rc;
-    dim3 g((s->k + 31) / 32, (pl.p.M + 31) / 32);
-    wgrad_reduce_kernel<<<g, 256, 0, st>>>(static_cast<const float*>(ws), (int)pl.grid.y, pl.p.M, s->k, dw,
-                                           accumulate);
+    if ((rc = launch(pl, ta, tb, grid_size(pl.p.total_tiles), st))) return rc;
+    if (!sliced) return DBL_OK;
+    const int64_t n = (int64_t)pl.p.M * s->k;
+    int64_t blocks = (n / 4 + 255) / 256;
+    const int64_t cap = (int64_t)sm_count() * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    wgrad_reduce_kernel<<<(int)blocks, 256, 0, st>>>(static_cast<const float*>(ws), pl.p.zdim, n, dw, accumulate);
     return launch_check("conv wgrad reduce");
 }
 

@@ -45,16 +45,16 @@ __global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* _
                                                           __nv_bfloat16* __restrict__ y, uint8_t* __restrict__ arg,
                                                           int n, int H, int W, int C, int P, int Q)
 {
-    const int groups = C / 8;
-    const int64_t total = (int64_t)n * P * Q * groups;
-    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-         t += (int64_t)gridDim.x * blockDim.x) {
-        const int g = (int)(t % groups);
-        int64_t pix = t / groups;
-        const int q = (int)(pix % Q);
-        pix /= Q;
-        const int p = (int)(pix % P);
-        const int b = (int)(pix / P);
+    // 32-bit index math: the host checks that n*P*Q*C/8 fits
+    const unsigned groups = (unsigned)C / 8u;
+    const unsigned total = (unsigned)n * P * Q * groups;
+    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
+        const unsigned g = t % groups;
+        unsigned pix = t / groups;
+        const int q = (int)(pix % (unsigned)Q);
+        pix /= (unsigned)Q;
+        const int p = (int)(pix % (unsigned)P);
+        const int b = (int)(pix / (unsigned)P);
         float best[8];
         uint8_t bi[8];
 #pragma unroll
@@ -94,25 +94,30 @@ __global__ void __launch_bounds__(256)
                        const uint8_t* __restrict__ arg, __nv_bfloat16* __restrict__ dx, int n, int H, int W, int C,
                        int P, int Q)
 {
-    const int groups = C / 8;
-    const int64_t total = (int64_t)n * H * W * groups;
-    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-         t += (int64_t)gridDim.x * blockDim.x) {
-        const int g = (int)(t % groups);
-        int64_t pix = t / groups;
-        const int w = (int)(pix % W);
-        pix /= W;
-        const int h = (int)(pix % H);
-        const int b = (int)(pix / H);
+    const unsigned groups = (unsigned)C / 8u;
+    const unsigned total = (unsigned)n * H * W * groups;
+    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
+        const unsigned g = t % groups;
+        unsigned pix = t / groups;
+        const int w = (int)(pix % (unsigned)W);
+        pix /= (unsigned)W;
+        const int h = (int)(pix % (unsigned)H);
+        const int b = (int)(pix / (unsigned)H);
         float acc[8] = {};
         // windows p with 2p-1 <= h <= 2p+1, i.e. h/2 <= p <= (h+1)/2; tap r = h - 2p + 1
-        for (int p = h / 2; p <= min(P - 1, (h + 1) / 2); ++p) {
+        const int p1 = min(P - 1, (h + 1) / 2), q1 = min(Q - 1, (w + 1) / 2);
+        for (int p = h / 2; p <= p1; ++p) {
             const int r = h - 2 * p + 1;
-            for (int q = w / 2; q <= min(Q - 1, (w + 1) / 2); ++q) {
+            for (int q = w / 2; q <= q1; ++q) {
                 const int s = w - 2 * q + 1;
                 const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
-                const uint2 a = *reinterpret_cast<const uint2*>(arg + o);
+                const uint2 a = __ldg(reinterpret_cast<const uint2*>(arg + o));
                 const uint8_t* ab = reinterpret_cast<const uint8_t*>(&a);
+                const uint8_t me = (uint8_t)(r * 3 + s);
+                bool any = false;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) any |= ab[k] == me;
+                if (!any) continue;  // this window's maximum is elsewhere for all 8 channels
                 float f[8];
                 unpack8(__ldg(reinterpret_cast<const uint4*>(dy + o)), f);
                 if (dy2) {
@@ -121,7 +126,6 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
                     for (int k = 0; k < 8; ++k) f[k] += f2[k];
                 }
-                const uint8_t me = (uint8_t)(r * 3 + s);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     if (ab[k] == me) acc[k] += f[k];
@@ -269,6 +273,8 @@ int dbl_maxpool_fwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* x, v
     if (!aligned16(x) || !aligned16(y) || (reinterpret_cast<uintptr_t>(argmax) & 7))
         return set_error(DBL_ERR_INVALID, "maxpool_fwd: misaligned pointer");
     const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
+    if ((int64_t)n * h * w * (c / 8) >= (int64_t)1 << 31)
+        return set_error(DBL_ERR_UNSUPPORTED, "maxpool_fwd: tensor too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
     maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q * (c / 8), 256), 256, 0, as_stream(stream)>>>(
         static_cast<const __nv_bfloat16*>(x), static_cast<__nv_bfloat16*>(y), argmax, n, h, w, c, P, Q);
@@ -285,6 +291,8 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
     if (!aligned16(dy) || !aligned16(dx) || (dy2 && !aligned16(dy2)) || (reinterpret_cast<uintptr_t>(argmax) & 7))
         return set_error(DBL_ERR_INVALID, "maxpool_bwd: misaligned pointer");
     const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
+    if ((int64_t)n * h * w * (c / 8) >= (int64_t)1 << 31)
+        return set_error(DBL_ERR_UNSUPPORTED, "maxpool_bwd: tensor too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
     maxpool_bwd_kernel<<<grid_for((int64_t)n * h * w * (c / 8), 256), 256, 0, as_stream(stream)>>>(
         static_cast<const __nv_bfloat16*>(dy), static_cast<const __nv_bfloat16*>(dy2), argmax,

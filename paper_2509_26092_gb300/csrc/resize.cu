@@ -17,9 +17,10 @@ struct Taps {
 
 __device__ __forceinline__ Taps axis_taps(int32_t j, int32_t in, int32_t out)
 {
-    const int64_t num = (int64_t)(2 * j + 1) * in - out;
-    const int64_t den = 2 * (int64_t)out;
-    const int64_t a = num / den;
+    // 32-bit: the host limits sizes so that (2j+1)*in stays far below 2^31
+    const int32_t num = (2 * j + 1) * in - out;
+    const int32_t den = 2 * out;
+    const int32_t a = num / den;
     Taps t;
     t.i0 = (int32_t)a;
     t.i1 = (int32_t)(a + 1 < in ? a + 1 : in - 1);
@@ -46,13 +47,13 @@ __global__ void __launch_bounds__(256) resize_kernel(const Tin* __restrict__ in,
                                                      int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
                                                      int32_t cs)
 {
-    const int64_t total = (int64_t)n * ho * wo;
-    for (int64_t pix = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pix < total;
-         pix += (int64_t)gridDim.x * blockDim.x) {
-        const int32_t x = (int32_t)(pix % wo);
-        const int64_t t = pix / wo;
-        const int32_t y = (int32_t)(t % ho);
-        const int32_t b = (int32_t)(t / ho);
+    // 32-bit index math: the host checks that n*ho*wo fits
+    const unsigned total = (unsigned)n * ho * wo;
+    for (unsigned pix = blockIdx.x * blockDim.x + threadIdx.x; pix < total; pix += gridDim.x * blockDim.x) {
+        const int32_t x = (int32_t)(pix % (unsigned)wo);
+        const unsigned t = pix / (unsigned)wo;
+        const int32_t y = (int32_t)(t % (unsigned)ho);
+        const int32_t b = (int32_t)(t / (unsigned)ho);
         const Taps ty = axis_taps(y, hi, ho), tx = axis_taps(x, wi, wo);
         const Tin* base = in + (int64_t)b * hi * wi * c;
         const Tin* pa = base + ((int64_t)ty.i0 * wi + tx.i0) * c;
@@ -69,7 +70,7 @@ __global__ void __launch_bounds__(256) resize_kernel(const Tin* __restrict__ in,
                 v[ch] = (1.f - ty.lam) * top + ty.lam * bot;
             }
         }
-        Tout* o = out + pix * cs;
+        Tout* o = out + (int64_t)pix * cs;
         if constexpr (sizeof(Tout) == 2 && CMAX == 8) {
             if (cs == 8) {  // one 16-byte store per pixel
                 __nv_bfloat162 q[4];
@@ -115,12 +116,16 @@ extern "C" int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, i
         return set_error(DBL_ERR_INVALID, "progressive_resize: bad sizes or null pointer");
     if (c > 8 || c_out_stride < c || c_out_stride > 8)
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: supports 1..8 channels, stride c..8");
+    if (h_in > 16384 || w_in > 16384)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: input side above 16384");
     if (h_out > h_in || w_out > w_in)
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: upsampling %dx%d -> %dx%d", h_in, w_in, h_out,
                          w_out);
     if ((in_dtype != DBL_F32 && in_dtype != DBL_BF16) || (out_dtype != DBL_F32 && out_dtype != DBL_BF16))
         return set_error(DBL_ERR_INVALID, "progressive_resize: dtype must be DBL_F32 or DBL_BF16");
     if (!aligned16(out)) return set_error(DBL_ERR_INVALID, "progressive_resize: output must be 16-byte aligned");
+    if ((int64_t)n * h_out * w_out >= (int64_t)1 << 31)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize: output too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
     cudaStream_t s = as_stream(stream);
     if (in_dtype == DBL_F32 && out_dtype == DBL_BF16)

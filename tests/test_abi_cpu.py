@@ -71,7 +71,7 @@ def test_update_factor_and_plan_match_oracle(D):
 def test_workspace_sizes_are_host_computable(D):
     s = D.conv_shape(8, 16, 16, 64, 64, 3, 1, 1)
     assert D.dbl_conv_workspace_bytes(s, D.DBL_PASS_FWD) > 0
-    assert D.dbl_conv_workspace_bytes(s, D.DBL_PASS_WGRAD) >= 576 * 64 * 4
+    assert D.dbl_conv_workspace_bytes(s, D.DBL_PASS_WGRAD) >= 0
     assert D.dbl_conv_workspace_bytes(D.conv_shape(8, 16, 16, 64, 60, 3, 1, 1), D.DBL_PASS_FWD) == 0  # unsupported
     assert D.dbl_bn_workspace_bytes(D.bn_shape(1000, 64)) > 0
     assert D.dbl_head_workspace_bytes(4, 512, 100) > 0
@@ -91,7 +91,8 @@ def test_invalid_arguments_rejected_before_launch(D):
     assert L.dbl_conv_fwd(ctypes.byref(s), 16, 16, 16, None, None, None, 0, None) == D.DBL_ERR_INVALID
     s = D.ConvShape(2, 8, 8, 64, 64, 3, 1, 1, 1)
     assert L.dbl_conv_fwd(ctypes.byref(s), 16, 16, 16, None, None, None, 0, None) == D.DBL_ERR_UNSUPPORTED
-    s = D.ConvShape(2, 8, 8, 64, 64, 3, 3, 1, 1)
+    s = D.ConvShape(8, 32, 32, 64, 64, 3, 3, 1, 1)  # 8192 pixels: the reduction is split, needing a workspace
+    assert D.dbl_conv_workspace_bytes(s, D.DBL_PASS_WGRAD) > 0
     assert L.dbl_conv_wgrad(ctypes.byref(s), 16, 16, 16, 0, None, 0, None) == D.DBL_ERR_WORKSPACE
     s = D.ConvShape(2, 8, 8, 8, 64, 7, 7, 2, 3)
     assert L.dbl_conv_dgrad(ctypes.byref(s), 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED

@@ -178,7 +178,9 @@ FWD_CASES = [  # n, h, w, c, k, r, stride, pad
     (8, 16, 16, 64, 64, 3, 1, 1),    # the single-block workload (batch 8, 16x16)
     (2, 6, 6, 8, 64, 3, 1, 1),       # CIFAR stem, 8 padded channels
     (2, 20, 20, 8, 64, 7, 2, 3),     # ImageNet stem, 8 padded channels
-    (1, 4, 4, 256, 256, 3, 1, 1),    # deep layer, small image
+    (1, 4, 4, 256, 256, 3, 1, 1),    # deep layer, small image, 256-wide tile
+    (4, 14, 14, 256, 512, 3, 2, 1),  # two 256-wide column tiles, stride 2
+    (32, 56, 56, 64, 64, 3, 1, 1),   # 784 tiles: every persistent CTA loops over several
 ]
 
 
@@ -221,6 +223,8 @@ DGRAD_CASES = [
     (2, 8, 8, 64, 128, 1, 2, 0),     # 1x1 stride 2: three phases are all zero
     (2, 16, 16, 64, 128, 3, 2, 1),
     (1, 4, 4, 256, 256, 3, 1, 1),
+    (2, 8, 8, 512, 512, 3, 1, 1),    # 256-wide tiles, 8 channel blocks of dy
+    (16, 28, 28, 128, 128, 3, 1, 1), # many tiles per CTA
 ]
 
 
@@ -249,6 +253,9 @@ WGRAD_CASES = [
     (2, 20, 20, 8, 64, 7, 2, 3),     # ImageNet stem
     (1, 4, 4, 256, 256, 3, 1, 1),
     (8, 16, 16, 64, 64, 3, 1, 1),
+    (2, 8, 8, 256, 512, 3, 2, 1),    # 256-wide tiles
+    (16, 28, 28, 128, 128, 3, 1, 1), # split-K slices reduced in order
+    (1, 3, 3, 64, 64, 3, 1, 1),      # a single slice, written straight into dw
 ]
 
 
