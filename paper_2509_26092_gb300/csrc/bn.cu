@@ -92,21 +92,29 @@ __global__ void __launch_bounds__(kThreads)
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
+    // statistics -> per-channel scale and shift, once per CTA (fp64 is slow on this GPU:
+    // one thread per channel, not one per thread and channel)
+    __shared__ float s_sc[kMaxC], s_sh[kMaxC];
     const double inv_n = 1.0 / (double)count;
-    float sc[8], sh[8];
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-        const int c = 8 * g + k;
+    for (int c = threadIdx.x; c < C; c += kThreads) {
         const double mean = (double)sum[c] * inv_n;
         double var = (double)sumsq[c] * inv_n - mean * mean;
         if (var < 0.0) var = 0.0;
         const float invstd = (float)(1.0 / sqrt(var + (double)eps));
-        sc[k] = gamma[c] * invstd;
-        sh[k] = beta[c] - (float)mean * sc[k];
-        if (blockIdx.x == 0 && threadIdx.x < groups) {
+        const float scale = gamma[c] * invstd;
+        s_sc[c] = scale;
+        s_sh[c] = beta[c] - (float)mean * scale;
+        if (blockIdx.x == 0) {
             save_mean[c] = (float)mean;
             save_invstd[c] = invstd;
         }
+    }
+    __syncthreads();
+    float sc[8], sh[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        sc[k] = s_sc[8 * g + k];
+        sh[k] = s_sh[8 * g + k];
     }
     const int64_t step = (int64_t)gridDim.x * rstep;
     for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += step) {

@@ -79,16 +79,26 @@ __device__ __forceinline__ void report_timeout(volatile int* abort)
     atomicExch(&g_conv_status, DBL_ERR_TIMEOUT);
 }
 
+// A ring stage holds two consecutive 64-element K-blocks ("sub-blocks"), so one
+// barrier round trip of the producer and of the MMA thread covers twice the MMA
+// work; mbarrier waits and TMA issues cost a thread on the order of a hundred
+// cycles each, which a single 64-wide K-block cannot hide at N <= 128.
+constexpr int kSub = 2;           // K-blocks per ring stage
+constexpr int kProducers = 2;     // producer warps; producer p fills the stages of iterations it % 2 == p
+
 template <int BN>
 struct Cfg {
-    static constexpr int STAGES = BN == 256 ? 4 : BN == 128 ? 6 : 8;
     static constexpr int B_BYTES = BN * BK * 2;
-    static constexpr int STAGE_BYTES = kA_BYTES + B_BYTES;
+    static constexpr int SUB_BYTES = kA_BYTES + B_BYTES;        // one K-block of A and B
+    static constexpr int STAGE_BYTES = kSub * SUB_BYTES;
+    static constexpr int STAGES = (196608 / STAGE_BYTES) < 2 ? 2 : (196608 / STAGE_BYTES);
     static constexpr int RING = STAGES * STAGE_BYTES;
     static constexpr int EPI_TILE = 4 * 32 * 33 * 4;           // per-warp 32x32 transpose scratch
     static constexpr int EPI_SUM = 4 * 2 * kMaxNcols * 4;      // per-warp channel sums (fwd)
     static constexpr int SMEM = RING + EPI_TILE + EPI_SUM + 1024;  // + 1 KB alignment slack
     static constexpr uint32_t TMEM_COLS = 2 * BN;               // two accumulators
+    static constexpr int THREADS = 32 * (4 + kProducers + 1);   // epilogue, producers, MMA
+    static constexpr int MMA_WARP = 4 + kProducers;
 };
 
 struct TileCoord {
@@ -176,10 +186,11 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
 }
 
 // Persistent kernel: CTA b processes tiles b, b + gridDim.x, ...  The ring of
-// STAGES shared-memory stages runs continuously across tiles; two TMEM
-// accumulators let the epilogue of one tile overlap the MMAs of the next.
+// STAGES shared-memory stages (two K-blocks each) runs continuously across
+// tiles; two producer warps fill alternate stages; two TMEM accumulators let
+// the epilogue of one tile overlap the MMAs of the next.
 template <int BN>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const ConvParams p)
 {
@@ -212,11 +223,11 @@ __global__ void __launch_bounds__(192, 1)
     const bool want_stats = (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
     if (want_stats)
         for (int i = threadIdx.x; i < 4 * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
-    if (warp == 4 && lane == 0) {
+    if (warp >= 4 && warp < 4 + kProducers && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
     }
-    if (warp == 5) {
+    if (warp == C::MMA_WARP) {
         tmem_alloc(&tmem_slot, C::TMEM_COLS);
         tmem_relinquish();
     }
@@ -226,10 +237,11 @@ __global__ void __launch_bounds__(192, 1)
     const uint32_t tmem = tmem_slot;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
 
-    if (warp == 4) {
-        // ------------------------------------------------------------------ TMA producer
+    if (warp >= 4 && warp < 4 + kProducers) {
+        // ------------------------------------------------------------------ TMA producers
+        const int prod = warp - 4;
         if (lane == 0) {
-            int it = 0;
+            int it = 0, last_it = -1;
             for (int t = blockIdx.x; t < p.total_tiles && !abort_flag; t += gridDim.x) {
                 const TileCoord tc = decode_tile(p, t);
                 int kb0, nkb;
@@ -242,27 +254,33 @@ __global__ void __launch_bounds__(192, 1)
                     tp = (int)(rem / p.gQ);
                     tq = (int)(rem - (int64_t)tp * p.gQ);
                 }
-                for (int k = 0; k < nkb; ++k, ++it) {
+                const int nst = (nkb + kSub - 1) / kSub;
+                for (int k = 0; k < nst; ++k, ++it) {
+                    if (it % kProducers != prod) continue;
                     const int s = it % STAGES;
                     if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
                         report_timeout(&abort_flag);
                         break;
                     }
-                    uint8_t* sa = sgen + s * C::STAGE_BYTES;
-                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)C::STAGE_BYTES);
-                    load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
+                    const int nsub = min(kSub, nkb - k * kSub);
+                    uint8_t* st = sgen + s * C::STAGE_BYTES;
+                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)(nsub * C::SUB_BYTES));
+                    for (int j = 0; j < nsub; ++j) {
+                        uint8_t* sa = st + j * C::SUB_BYTES;
+                        load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k * kSub + j, tn, tp,
+                                    tq);
+                    }
+                    last_it = it;
                 }
             }
             if (abort_flag) {
-                // let copies already issued land before the CTA's shared memory goes away
-                for (int s = 0; s < STAGES && s < it; ++s) {
-                    const int last = s + STAGES * ((it - 1 - s) / STAGES);
-                    (void)mbar_wait_drain(&full_bar[s], (last / STAGES) & 1);
-                }
+                // let copies this producer issued land before the CTA's shared memory goes away
+                for (int i = last_it; i >= 0 && i > last_it - STAGES * kProducers; i -= kProducers)
+                    (void)mbar_wait_drain(&full_bar[i % STAGES], (i / STAGES) & 1);
             }
         }
         __syncwarp();
-    } else if (warp == 5) {
+    } else if (warp == C::MMA_WARP) {
         // ------------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
@@ -281,7 +299,8 @@ __global__ void __launch_bounds__(192, 1)
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(buf * BN);
                 bool ok = true;
-                for (int k = 0; k < nkb; ++k, ++it) {
+                const int nst = (nkb + kSub - 1) / kSub;
+                for (int k = 0; k < nst; ++k, ++it) {
                     const int s = it % STAGES;
                     if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
                         report_timeout(&abort_flag);
@@ -289,32 +308,35 @@ __global__ void __launch_bounds__(192, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = sbase + s * C::STAGE_BYTES;
-                    const uint32_t sb = sa + kA_BYTES;
+                    const int nsub = min(kSub, nkb - k * kSub);
+                    for (int jj = 0; jj < nsub; ++jj) {
+                        const uint32_t sa = sbase + s * C::STAGE_BYTES + jj * C::SUB_BYTES;
+                        const uint32_t sb = sa + kA_BYTES;
 #pragma unroll
-                    for (int j = 0; j < BK / 16; ++j) {
-                        uint64_t ad, bd;
-                        if (p.mode == kFwd) {
-                            ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
-                        } else if (p.mode == kDgrad) {
-                            ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                        } else if (p.mode == kWgrad) {
-                            ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                        } else if (p.mode == kFwdC8) {
-                            // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
-                            // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
-                            ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
-                            bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
-                        } else {
-                            // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
-                            // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
-                            ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
-                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                        for (int j = 0; j < BK / 16; ++j) {
+                            uint64_t ad, bd;
+                            if (p.mode == kFwd) {
+                                ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                                bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
+                            } else if (p.mode == kDgrad) {
+                                ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                            } else if (p.mode == kWgrad) {
+                                ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
+                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                            } else if (p.mode == kFwdC8) {
+                                // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
+                                // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
+                                ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
+                                bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
+                            } else {
+                                // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
+                                // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
+                                ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
+                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                            }
+                            mma_bf16(d, ad, bd, idesc, (k > 0 || jj > 0 || j > 0) ? 1u : 0u);
                         }
-                        mma_bf16(d, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
                     }
                     mma_commit(&empty_bar[s]);
                 }
@@ -424,7 +446,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == C::MMA_WARP) {
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
@@ -701,7 +723,7 @@ int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int g
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_igemm_kernel<BN><<<grid, 192, Cf::SMEM, st>>>(a, b, pl.p);
+    conv_igemm_kernel<BN><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
     return dbl::launch_check("conv_igemm launch");
 }
 
