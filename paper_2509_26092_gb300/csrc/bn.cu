@@ -208,33 +208,29 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
-// Fixed-order sum of the partials (double; 8 lanes per channel, then 8 -> 1),
-// then dgamma/dbeta and the three per-channel coefficients of the apply pass.
+// Fixed-order sum of the partials: one warp per channel, lane l sums blocks
+// l, l+32, ... in double, then a fixed butterfly across the warp; then dgamma,
+// dbeta and the three per-channel coefficients of the apply pass.
 __global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C,
                                                               int64_t count, const float* __restrict__ gamma,
                                                               const float* __restrict__ invstd,
                                                               float* __restrict__ dgamma, float* __restrict__ dbeta,
                                                               float* __restrict__ coef)
 {
-    __shared__ double red[8][2][33];
-    const int c = blockIdx.x * 32 + threadIdx.x % 32;
-    const int l8 = threadIdx.x / 32;
+    const int c = blockIdx.x * 8 + threadIdx.x / 32;
+    const int lane = threadIdx.x % 32;
+    if (c >= C) return;
     double sg = 0.0, sgx = 0.0;
-    if (c < C)
-        for (int b = l8; b < nblk; b += 8) {
-            sg += partial[(int64_t)b * 2 * C + c];
-            sgx += partial[(int64_t)b * 2 * C + C + c];
-        }
-    red[l8][0][threadIdx.x % 32] = sg;
-    red[l8][1][threadIdx.x % 32] = sgx;
-    __syncthreads();
-    if (threadIdx.x >= 32 || c >= C) return;
-    sg = 0.0;
-    sgx = 0.0;
-    for (int l = 0; l < 8; ++l) {
-        sg += red[l][0][threadIdx.x];
-        sgx += red[l][1][threadIdx.x];
+    for (int b = lane; b < nblk; b += 32) {
+        sg += partial[(int64_t)b * 2 * C + c];
+        sgx += partial[(int64_t)b * 2 * C + C + c];
     }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        sg += __shfl_xor_sync(0xffffffffu, sg, o);
+        sgx += __shfl_xor_sync(0xffffffffu, sgx, o);
+    }
+    if (lane != 0) return;
     dbeta[c] = (float)sg;
     dgamma[c] = (float)sgx;
     coef[c] = gamma[c] * invstd[c];
@@ -296,7 +292,7 @@ int check_shape(const dbl_bn_shape* s, const char* who)
 
 // Backward reduce split: a fixed function of the shape, so the workspace
 // size does not depend on the device.
-int64_t bwd_blocks(int64_t count) { return count <= 0 ? 1 : (count + 255) / 256 < 1024 ? (count + 255) / 256 : 1024; }
+int64_t bwd_blocks(int64_t count) { return count <= 0 ? 1 : (count + 255) / 256 < 512 ? (count + 255) / 256 : 512; }
 
 }  // namespace
 
@@ -368,7 +364,7 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
     bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
                                                          save_mean, save_invstd, rows, partial);
     if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
@@ -448,7 +444,7 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
     bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
                                                          save_mean, save_invstd, rows, partial);
     if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(

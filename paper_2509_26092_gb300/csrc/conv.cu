@@ -83,11 +83,13 @@ __device__ __forceinline__ void report_timeout(volatile int* abort)
 // barrier round trip of the producer and of the MMA thread covers twice the MMA
 // work; mbarrier waits and TMA issues cost a thread on the order of a hundred
 // cycles each, which a single 64-wide K-block cannot hide at N <= 128.
-constexpr int kSub = 2;           // K-blocks per ring stage
 constexpr int kProducers = 2;     // producer warps; producer p fills the stages of iterations it % 2 == p
 
 template <int BN>
 struct Cfg {
+    // 128x256 tiles already give 512 MMA cycles per K-block: one K-block per stage,
+    // four stages of latency cover; narrower tiles take two K-blocks per stage.
+    static constexpr int kSub = BN == 256 ? 1 : 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int SUB_BYTES = kA_BYTES + B_BYTES;        // one K-block of A and B
     static constexpr int STAGE_BYTES = kSub * SUB_BYTES;
@@ -254,7 +256,7 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                     tp = (int)(rem / p.gQ);
                     tq = (int)(rem - (int64_t)tp * p.gQ);
                 }
-                const int nst = (nkb + kSub - 1) / kSub;
+                const int nst = (nkb + C::kSub - 1) / C::kSub;
                 for (int k = 0; k < nst; ++k, ++it) {
                     if (it % kProducers != prod) continue;
                     const int s = it % STAGES;
@@ -262,12 +264,12 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                         report_timeout(&abort_flag);
                         break;
                     }
-                    const int nsub = min(kSub, nkb - k * kSub);
+                    const int nsub = min(C::kSub, nkb - k * C::kSub);
                     uint8_t* st = sgen + s * C::STAGE_BYTES;
                     mbar_arrive_expect_tx(&full_bar[s], (uint32_t)(nsub * C::SUB_BYTES));
                     for (int j = 0; j < nsub; ++j) {
                         uint8_t* sa = st + j * C::SUB_BYTES;
-                        load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k * kSub + j, tn, tp,
+                        load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k * C::kSub + j, tn, tp,
                                     tq);
                     }
                     last_it = it;
@@ -299,7 +301,7 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(buf * BN);
                 bool ok = true;
-                const int nst = (nkb + kSub - 1) / kSub;
+                const int nst = (nkb + C::kSub - 1) / C::kSub;
                 for (int k = 0; k < nst; ++k, ++it) {
                     const int s = it % STAGES;
                     if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
@@ -308,7 +310,7 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    const int nsub = min(kSub, nkb - k * kSub);
+                    const int nsub = min(C::kSub, nkb - k * C::kSub);
                     for (int jj = 0; jj < nsub; ++jj) {
                         const uint32_t sa = sbase + s * C::STAGE_BYTES + jj * C::SUB_BYTES;
                         const uint32_t sb = sa + kA_BYTES;

@@ -87,37 +87,36 @@ __global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* _
     }
 }
 
-// Gather form: input (h,w) receives dy from every window (p,q) that contains
-// it and whose argmax is (h,w).  Windows are visited in (p, q) order.
+// Gather form over 2x2 blocks of input pixels: block (i, j) = rows 2i..2i+1,
+// cols 2j..2j+1 is covered by windows (i..i+1, j..j+1); window (p, q) reaches
+// input (h, w) at tap (h - 2p + 1, w - 2q + 1).  Each window's argmax and
+// gradient are read once per block, and every input pixel sums its windows in
+// (p, q) order.
 __global__ void __launch_bounds__(256)
     maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dy, const __nv_bfloat16* __restrict__ dy2,
                        const uint8_t* __restrict__ arg, __nv_bfloat16* __restrict__ dx, int n, int H, int W, int C,
                        int P, int Q)
 {
     const unsigned groups = (unsigned)C / 8u;
-    const unsigned total = (unsigned)n * H * W * groups;
+    const int BH = (H + 1) / 2, BW = (W + 1) / 2;
+    const unsigned total = (unsigned)n * BH * BW * groups;
     for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
         const unsigned g = t % groups;
         unsigned pix = t / groups;
-        const int w = (int)(pix % (unsigned)W);
-        pix /= (unsigned)W;
-        const int h = (int)(pix % (unsigned)H);
-        const int b = (int)(pix / (unsigned)H);
-        float acc[8] = {};
-        // windows p with 2p-1 <= h <= 2p+1, i.e. h/2 <= p <= (h+1)/2; tap r = h - 2p + 1
-        const int p1 = min(P - 1, (h + 1) / 2), q1 = min(Q - 1, (w + 1) / 2);
-        for (int p = h / 2; p <= p1; ++p) {
-            const int r = h - 2 * p + 1;
-            for (int q = w / 2; q <= q1; ++q) {
-                const int s = w - 2 * q + 1;
+        const int j = (int)(pix % (unsigned)BW);
+        pix /= (unsigned)BW;
+        const int i = (int)(pix % (unsigned)BH);
+        const int b = (int)(pix / (unsigned)BH);
+        float acc[4][8] = {};
+        for (int dp = 0; dp < 2; ++dp) {
+            const int p = i + dp;
+            if (p >= P) continue;
+            for (int dq = 0; dq < 2; ++dq) {
+                const int q = j + dq;
+                if (q >= Q) continue;
                 const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
                 const uint2 a = __ldg(reinterpret_cast<const uint2*>(arg + o));
                 const uint8_t* ab = reinterpret_cast<const uint8_t*>(&a);
-                const uint8_t me = (uint8_t)(r * 3 + s);
-                bool any = false;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) any |= ab[k] == me;
-                if (!any) continue;  // this window's maximum is elsewhere for all 8 channels
                 float f[8];
                 unpack8(__ldg(reinterpret_cast<const uint4*>(dy + o)), f);
                 if (dy2) {
@@ -127,11 +126,32 @@ __global__ void __launch_bounds__(256)
                     for (int k = 0; k < 8; ++k) f[k] += f2[k];
                 }
 #pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    if (ab[k] == me) acc[k] += f[k];
+                for (int dh = 0; dh < 2; ++dh) {
+                    const int r = 2 * i + dh - 2 * p + 1;  // tap row of input row 2i+dh in window row p
+                    if (r < 0 || r > 2) continue;
+#pragma unroll
+                    for (int dw = 0; dw < 2; ++dw) {
+                        const int sx = 2 * j + dw - 2 * q + 1;
+                        if (sx < 0 || sx > 2) continue;
+                        const uint8_t me = (uint8_t)(r * 3 + sx);
+#pragma unroll
+                        for (int k = 0; k < 8; ++k)
+                            if (ab[k] == me) acc[dh * 2 + dw][k] += f[k];
+                    }
+                }
             }
         }
-        *reinterpret_cast<uint4*>(dx + (((int64_t)b * H + h) * W + w) * C + 8 * g) = pack8(acc);
+#pragma unroll
+        for (int dh = 0; dh < 2; ++dh) {
+            const int h = 2 * i + dh;
+            if (h >= H) continue;
+#pragma unroll
+            for (int dw = 0; dw < 2; ++dw) {
+                const int w = 2 * j + dw;
+                if (w >= W) continue;
+                *reinterpret_cast<uint4*>(dx + (((int64_t)b * H + h) * W + w) * C + 8 * g) = pack8(acc[dh * 2 + dw]);
+            }
+        }
     }
 }
 
@@ -294,7 +314,8 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
     if ((int64_t)n * h * w * (c / 8) >= (int64_t)1 << 31)
         return set_error(DBL_ERR_UNSUPPORTED, "maxpool_bwd: tensor too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
-    maxpool_bwd_kernel<<<grid_for((int64_t)n * h * w * (c / 8), 256), 256, 0, as_stream(stream)>>>(
+    maxpool_bwd_kernel<<<grid_for((int64_t)n * ((h + 1) / 2) * ((w + 1) / 2) * (c / 8), 256), 256, 0,
+                         as_stream(stream)>>>(
         static_cast<const __nv_bfloat16*>(dy), static_cast<const __nv_bfloat16*>(dy2), argmax,
         static_cast<__nv_bfloat16*>(dx), n, h, w, c, P, Q);
     return launch_check("maxpool_bwd launch");
