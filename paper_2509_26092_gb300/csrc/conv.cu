@@ -79,28 +79,35 @@ __device__ __forceinline__ void report_timeout(volatile int* abort)
     atomicExch(&g_conv_status, DBL_ERR_TIMEOUT);
 }
 
-// A ring stage holds two consecutive 64-element K-blocks ("sub-blocks"), so one
-// barrier round trip of the producer and of the MMA thread covers twice the MMA
-// work; mbarrier waits and TMA issues cost a thread on the order of a hundred
-// cycles each, which a single 64-wide K-block cannot hide at N <= 128.
 constexpr int kProducers = 2;     // producer warps; producer p fills the stages of iterations it % 2 == p
 
-template <int BN>
+enum Family : int { kFamFwd = 0, kFamWgrad = 1 };  // fwd/dgrad/stem-fwd, and the two weight-gradient modes
+
+// Per (tile width, family) geometry.  mbarrier round trips and TMA issues cost a
+// thread on the order of a hundred cycles each, so every ring stage is sized to
+// carry at least ~384 cycles of MMA work per handful of TMA ops:
+//   forward family, BN <= 128: a tile is 256 rows in two 128-row accumulators
+//     that share one B tile; one 256-pixel im2col op feeds both;
+//   weight-gradient family: a K-block is 128 pixels (8 MMA K-steps).
+template <int BN, int FAM>
 struct Cfg {
-    // 128x256 tiles already give 512 MMA cycles per K-block: one K-block per stage,
-    // four stages of latency cover; narrower tiles take two K-blocks per stage.
-    static constexpr int kSub = BN == 256 ? 1 : 2;
-    static constexpr int B_BYTES = BN * BK * 2;
-    static constexpr int SUB_BYTES = kA_BYTES + B_BYTES;        // one K-block of A and B
-    static constexpr int STAGE_BYTES = kSub * SUB_BYTES;
-    static constexpr int STAGES = (196608 / STAGE_BYTES) < 2 ? 2 : (196608 / STAGE_BYTES);
+    static constexpr int ACC = (FAM == kFamFwd && BN <= 128) ? 2 : 1;  // 128-row accumulators per tile
+    static constexpr int BMT = 128 * ACC;                               // tile rows
+    static constexpr int KB = FAM == kFamFwd ? 64 : 128;                // reduction elements per stage
+    static constexpr int KSTEPS = KB / 16;
+    static constexpr int A_BYTES = BMT * KB * 2;
+    static constexpr int B_BYTES = BN * KB * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES = (196608 / STAGE_BYTES) < 4 ? (196608 / STAGE_BYTES) : 4;
     static constexpr int RING = STAGES * STAGE_BYTES;
     static constexpr int EPI_TILE = 4 * 32 * 33 * 4;           // per-warp 32x32 transpose scratch
     static constexpr int EPI_SUM = 4 * 2 * kMaxNcols * 4;      // per-warp channel sums (fwd)
     static constexpr int SMEM = RING + EPI_TILE + EPI_SUM + 1024;  // + 1 KB alignment slack
-    static constexpr uint32_t TMEM_COLS = 2 * BN;               // two accumulators
+    static constexpr uint32_t TMEM_COLS = 2 * ACC * BN;         // two tiles in flight
     static constexpr int THREADS = 32 * (4 + kProducers + 1);   // epilogue, producers, MMA
     static constexpr int MMA_WARP = 4 + kProducers;
+    static_assert(STAGES >= 2, "ring too shallow");
+    static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
 };
 
 struct TileCoord {
@@ -135,25 +142,40 @@ __device__ __forceinline__ void kb_range(const ConvParams& p, int z, int& kb0, i
 }
 
 // Issue the TMA loads of one K-block of one tile into ring stage (sa, sb).
+template <int BN, int FAM>
 __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorMap* tmA, const CUtensorMap* tmB,
-                                            int BN, uint8_t* sa, uint8_t* sb, uint64_t* fb, const TileCoord& tc,
-                                            int kb, int tn, int tp, int tq)
+                                            uint8_t* sa, uint8_t* sb, uint64_t* fb, const TileCoord& tc, int kb, int tn,
+                                            int tp, int tq)
 {
+    using C = Cfg<BN, FAM>;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
-    if (p.mode == kFwd) {
-        const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
-        const int r = tap / p.S, sx = tap - r * p.S;
-        tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
-                           (uint16_t)sx, (uint16_t)r);
-        tma_load_2d(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
-    } else if (p.mode == kDgrad) {
-        const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
-        tma_load_im2col_4d(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
-                           (uint16_t)p.tap_oh[t]);
-        const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
-        for (int j = 0; j < BN / 64; ++j) tma_load_3d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
-    } else if (p.mode == kWgrad || p.mode == kWgradC8) {
-        const int64_t pix0 = (int64_t)kb * 64;
+    if constexpr (FAM == kFamFwd) {
+        if (p.mode == kFwd) {
+            const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
+            const int r = tap / p.S, sx = tap - r * p.S;
+            tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
+                               (uint16_t)sx, (uint16_t)r);
+            tma_load_2d(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
+        } else if (p.mode == kDgrad) {
+            const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
+            tma_load_im2col_4d(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
+                               (uint16_t)p.tap_oh[t]);
+            const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
+            for (int j = 0; j < BN / 64; ++j)
+                tma_load_3d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
+        } else {  // kFwdC8: 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
+            for (int j = 0; j < 8; ++j) {
+                int tap = kb * 8 + j;
+                const int wcol = tap * 8;
+                if (tap >= p.ntaps) tap = p.ntaps - 1;
+                tma_load_im2col_4d(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride + p.base_w,
+                                   tp * p.tstride + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_2d(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
+            }
+        }
+    } else {
+        // weight gradient: a K-block is 128 output pixels
+        const int64_t pix0 = (int64_t)kb * 128;
         const int n = (int)(pix0 / gPQ);
         const int64_t rem = pix0 - (int64_t)n * gPQ;
         const int pp = (int)(rem / p.gQ), qq = (int)(rem - (int64_t)pp * p.gQ);
@@ -163,27 +185,18 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
                 int tap = mrow / p.Cin;
                 const int c0 = mrow - tap * p.Cin;
                 if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
-                tma_load_im2col_4d(sa + h * 8192, tmA, fb, c0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h,
-                                   n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_im2col_4d(sa + h * 16384, tmA, fb, c0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
+                                   (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
-        } else {  // 16 taps x 8 channels of rows
+        } else {  // kWgradC8: 16 taps x 8 channels of rows
             for (int j = 0; j < 16; ++j) {
                 int tap = tc.m_tile * 16 + j;
                 if (tap >= p.ntaps) tap = 0;
-                tma_load_im2col_4d(sa + j * 1024, tmA, fb, 0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
+                tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
                                    (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         }
-        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
-    } else {  // kFwdC8: 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
-        for (int j = 0; j < 8; ++j) {
-            int tap = kb * 8 + j;
-            const int wcol = tap * 8;
-            if (tap >= p.ntaps) tap = p.ntaps - 1;
-            tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
-                               (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
-            tma_load_2d(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
-        }
+        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 16384, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
     }
 }
 
@@ -191,12 +204,12 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
 // STAGES shared-memory stages (two K-blocks each) runs continuously across
 // tiles; two producer warps fill alternate stages; two TMEM accumulators let
 // the epilogue of one tile overlap the MMAs of the next.
-template <int BN>
-__global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
+template <int BN, int FAM>
+__global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const ConvParams p)
 {
-    using C = Cfg<BN>;
+    using C = Cfg<BN, FAM>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accf_bar[2], acce_bar[2], drain_bar;
@@ -249,29 +262,23 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                 int kb0, nkb;
                 kb_range(p, tc.z, kb0, nkb);
                 int tn = 0, tp = 0, tq = 0;
-                if (p.mode == kFwd || p.mode == kDgrad || p.mode == kFwdC8) {
-                    const int64_t m0 = (int64_t)tc.m_tile * BM;
+                if (FAM == kFamFwd) {
+                    const int64_t m0 = (int64_t)tc.m_tile * C::BMT;
                     tn = (int)(m0 / gPQ);
                     const int64_t rem = m0 - (int64_t)tn * gPQ;
                     tp = (int)(rem / p.gQ);
                     tq = (int)(rem - (int64_t)tp * p.gQ);
                 }
-                const int nst = (nkb + C::kSub - 1) / C::kSub;
-                for (int k = 0; k < nst; ++k, ++it) {
+                for (int k = 0; k < nkb; ++k, ++it) {
                     if (it % kProducers != prod) continue;
                     const int s = it % STAGES;
                     if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
                         report_timeout(&abort_flag);
                         break;
                     }
-                    const int nsub = min(C::kSub, nkb - k * C::kSub);
-                    uint8_t* st = sgen + s * C::STAGE_BYTES;
-                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)(nsub * C::SUB_BYTES));
-                    for (int j = 0; j < nsub; ++j) {
-                        uint8_t* sa = st + j * C::SUB_BYTES;
-                        load_kblock(p, &tmA, &tmB, BN, sa, sa + kA_BYTES, &full_bar[s], tc, kb0 + k * C::kSub + j, tn, tp,
-                                    tq);
-                    }
+                    uint8_t* sa = sgen + s * C::STAGE_BYTES;
+                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)C::STAGE_BYTES);
+                    load_kblock<BN, FAM>(p, &tmA, &tmB, sa, sa + C::A_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
                     last_it = it;
                 }
             }
@@ -299,10 +306,9 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(buf * BN);
+                const uint32_t d = tmem + (uint32_t)(buf * C::ACC * BN);
                 bool ok = true;
-                const int nst = (nkb + C::kSub - 1) / C::kSub;
-                for (int k = 0; k < nst; ++k, ++it) {
+                for (int k = 0; k < nkb; ++k, ++it) {
                     const int s = it % STAGES;
                     if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
                         report_timeout(&abort_flag);
@@ -310,34 +316,35 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    const int nsub = min(C::kSub, nkb - k * C::kSub);
-                    for (int jj = 0; jj < nsub; ++jj) {
-                        const uint32_t sa = sbase + s * C::STAGE_BYTES + jj * C::SUB_BYTES;
-                        const uint32_t sb = sa + kA_BYTES;
+                    const uint32_t sa = sbase + s * C::STAGE_BYTES;
+                    const uint32_t sb = sa + C::A_BYTES;
 #pragma unroll
-                        for (int j = 0; j < BK / 16; ++j) {
+                    for (int j = 0; j < C::KSTEPS; ++j) {
+#pragma unroll
+                        for (int a = 0; a < C::ACC; ++a) {
                             uint64_t ad, bd;
                             if (p.mode == kFwd) {
-                                ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
+                                ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
                                 bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
                             } else if (p.mode == kDgrad) {
-                                ad = smem_desc(sa + 32 * j, 16, 1024, kSwizzle128B);
-                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                            } else if (p.mode == kWgrad) {
-                                ad = smem_desc(sa + 2048 * j, 8192, 1024, kSwizzle128B);
+                                ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
                                 bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
                             } else if (p.mode == kFwdC8) {
                                 // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
                                 // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
-                                ad = smem_desc(sa + 4096 * j, 2048, 128, kSwizzleNone);
+                                ad = smem_desc(sa + a * 2048 + 2 * (C::BMT * 16) * j, C::BMT * 16, 128, kSwizzleNone);
                                 bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
+                            } else if (p.mode == kWgrad) {
+                                // MN-major, 128-byte swizzle: 64-wide atoms 16 KB apart (LBO)
+                                ad = smem_desc(sa + 2048 * j, 16384, 1024, kSwizzle128B);
+                                bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
                             } else {
                                 // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
-                                // next 8 pixels 128 B apart (LBO), next tap 1 KB apart (SBO)
-                                ad = smem_desc(sa + 256 * j, 128, 1024, kSwizzleNone);
-                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                                // next 8 pixels 128 B apart (LBO), next tap 2 KB apart (SBO)
+                                ad = smem_desc(sa + 256 * j, 128, 2048, kSwizzleNone);
+                                bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
                             }
-                            mma_bf16(d, ad, bd, idesc, (k > 0 || jj > 0 || j > 0) ? 1u : 0u);
+                            mma_bf16(d + a * BN, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
                         }
                     }
                     mma_commit(&empty_bar[s]);
@@ -366,18 +373,20 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                 break;
             }
             tc_fence_after();
-            const int row = warp * 32 + lane;  // TMEM lane = tile row
-            const int64_t m = (int64_t)tc.m_tile * BM + row;
-            const bool valid = m < p.M;
+            const int row = warp * 32 + lane;  // TMEM lane = row within a 128-row accumulator
             const bool have_acc = nkb > 0;
+#pragma unroll 1
+            for (int a = 0; a < C::ACC; ++a) {
+            const int64_t m = (int64_t)tc.m_tile * C::BMT + a * 128 + row;
+            const bool valid = m < p.M;
             int64_t out_row = m;
             if (p.mode == kDgrad && p.phase_div == 2) {
                 const int64_t n = m / gPQ, rem = m - n * gPQ;
                 const int i = (int)(rem / p.gQ), j = (int)(rem - (int64_t)(rem / p.gQ) * p.gQ);
-                const int a = tc.z >> 1, b = tc.z & 1;
-                out_row = (n * p.out_h + 2 * i + a) * p.out_w + 2 * j + b;
+                const int pa = tc.z >> 1, pb = tc.z & 1;
+                out_row = (n * p.out_h + 2 * i + pa) * p.out_w + 2 * j + pb;
             }
-            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * BN);
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * C::ACC + a) * BN);
 #pragma unroll 1
             for (int ch = 0; ch < BN / 32; ++ch) {
                 uint32_t v[32];
@@ -434,6 +443,7 @@ __global__ void __launch_bounds__(Cfg<BN>::THREADS, 1)
                         __syncwarp();
                     }
                 }
+            }
             }
             tc_fence_before();
             __syncwarp();
@@ -516,6 +526,8 @@ struct Plan {
 
 int out_dim(int in, int k, int st, int pad) { return (in + 2 * pad - k) / st + 1; }
 
+int fwd_tile_rows(int BN);
+
 int choose_bn(int cols)
 {
     if (cols % 256 == 0) return 256;
@@ -574,7 +586,7 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.M = (int)M;
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
-        p.m_tiles = (p.M + BM - 1) / BM;
+        p.m_tiles = (p.M + fwd_tile_rows(pl.BN) - 1) / fwd_tile_rows(pl.BN);
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;
         p.gP = P;
@@ -649,7 +661,7 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
             }
             p.phase_off[4] = t;
         }
-        p.m_tiles = (p.M + BM - 1) / BM;
+        p.m_tiles = (p.M + fwd_tile_rows(pl.BN) - 1) / fwd_tile_rows(pl.BN);
     } else {
         pl.mode = p.mode = c8 ? kWgradC8 : kWgrad;
         p.M = p.ntaps * s->c;  // D rows = (tap, c)
@@ -663,13 +675,13 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.tstride = s->stride;
         p.base_h = p.base_w = -s->pad;
         const int64_t pix = (int64_t)s->n * P * Q;
-        if ((pix + 63) / 64 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
-        p.num_kb = (int)((pix + 63) / 64);
+        if ((pix + 127) / 128 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
+        p.num_kb = (int)((pix + 127) / 128);  // K-blocks of 128 output pixels
         const int tiles = p.m_tiles * p.n_tiles;
         // split the pixel reduction so that there are about two tiles per SM of a 152-SM GPU,
-        // keeping at least 8 K-blocks per slice (a fixed function of the shape)
+        // keeping at least 4 K-blocks (512 pixels) per slice (a fixed function of the shape)
         int splits = (kTargetCTAs + tiles - 1) / tiles;
-        if (splits > p.num_kb / 8) splits = p.num_kb / 8;
+        if (splits > p.num_kb / 4) splits = p.num_kb / 4;
         if (splits < 1) splits = 1;
         p.kb_per_split = (p.num_kb + splits - 1) / splits;
         splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
@@ -713,28 +725,38 @@ int enc_tiled(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims
     return DBL_OK;
 }
 
-template <int BN>
+template <int BN, int FAM>
 int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
-    using Cf = Cfg<BN>;
+    using Cf = Cfg<BN, FAM>;
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cf::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN, FAM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             Cf::SMEM);
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_igemm_kernel<BN><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
+    conv_igemm_kernel<BN, FAM><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
     return dbl::launch_check("conv_igemm launch");
 }
 
 int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
-    if (pl.BN == 256) return launch_cfg<256>(pl, a, b, grid, st);
-    if (pl.BN == 128) return launch_cfg<128>(pl, a, b, grid, st);
-    return launch_cfg<64>(pl, a, b, grid, st);
+    const bool wg = pl.mode == kWgrad || pl.mode == kWgradC8;
+    if (wg) {
+        if (pl.BN == 256) return launch_cfg<256, kFamWgrad>(pl, a, b, grid, st);
+        if (pl.BN == 128) return launch_cfg<128, kFamWgrad>(pl, a, b, grid, st);
+        return launch_cfg<64, kFamWgrad>(pl, a, b, grid, st);
+    }
+    if (pl.BN == 256) return launch_cfg<256, kFamFwd>(pl, a, b, grid, st);
+    if (pl.BN == 128) return launch_cfg<128, kFamFwd>(pl, a, b, grid, st);
+    return launch_cfg<64, kFamFwd>(pl, a, b, grid, st);
 }
+
+// Rows of one tile of the forward family (see Cfg).
+int fwd_tile_rows(int BN) { return BN <= 128 ? 256 : 128; }
 
 }  // namespace
 
@@ -763,7 +785,8 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
     CUtensorMap ta, tb;
     if (pl.mode == kFwdC8) {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -s->pad, s->pad - (s->r - 1), s->stride, 8, BM, false)))
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -s->pad, s->pad - (s->r - 1), s->stride, 8,
+                             fwd_tile_rows(pl.BN), false)))
             return rc;
         const int64_t rsc = (int64_t)s->r * s->s * 8;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
@@ -771,7 +794,8 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         cuuint32_t box[2] = {8, (cuuint32_t)pl.BN};
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, false))) return rc;
     } else {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, 64, BM, true)))
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, 64,
+                             fwd_tile_rows(pl.BN), true)))
             return rc;
         const int64_t rsc = (int64_t)s->r * s->s * s->c;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
@@ -810,7 +834,7 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
         lower = -(s->r - 1 - s->pad);
         upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
     }
-    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, 1, 64, BM, true))) return rc;
+    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, 1, 64, fwd_tile_rows(pl.BN), true))) return rc;
     // w viewed as [k][r*s][c]: inner c, then tap, then k
     cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
     cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
@@ -834,12 +858,12 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
     CUtensorMap ta, tb;
     const bool c8 = pl.mode == kWgradC8;
-    if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, c8 ? 8 : 64, 64,
+    if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, c8 ? 8 : 64, 128,
                          !c8)))
         return rc;
     cuuint64_t dims[2] = {(cuuint64_t)s->k, (cuuint64_t)s->n * P * Q};
     cuuint64_t str[1] = {(cuuint64_t)s->k * 2};
-    cuuint32_t box[2] = {64, 64};
+    cuuint32_t box[2] = {64, 128};
     if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
     const bool sliced = pl.p.zdim > 1;
     pl.p.out = sliced ? ws : static_cast<void*>(dw);
