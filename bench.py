@@ -267,9 +267,7 @@ def conv_roofline(stage, reps=3):
             x, y, dy, dx, w16, g = bufs[name]
             st_sum = torch.empty(shp.k, device=x.device)
             st_sq = torch.empty(shp.k, device=x.device)
-            P = (shp.h + 2 * shp.pad - shp.r) // shp.stride + 1
-            cin = wk.spec.stem.cin_logical if name == stem else shp.c
-            f1 = 2.0 * shp.n * P * P * shp.k * shp.r * shp.s * cin
+            f1 = float(wk.layer_flops(name, shp))
             passes = [("fwd", lambda: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
             if name != stem:
                 passes.append(("dgrad", lambda: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))

@@ -73,17 +73,22 @@ DBL_API int dbl_device_status(int32_t* status);
  * the training step needs the forward pass and, through Eq. 1 (the gradient
  * of the batch-mean loss), the data and weight gradients.
  *
- *   y[n,p,q,k] = sum_{r,s,c} x[n, p*stride + r - pad, q*stride + s - pad, c] * w[k,r,s,c]
- *   P = (h + 2*pad - r)/stride + 1,  Q = (w + 2*pad - s)/stride + 1
+ *   y[n,p,q,k] = sum_{r,s,c} x[n, p*stride_h + r - pad_h, q*stride_w + s - pad_w, c] * w[k,r,s,c]
+ *   P = (h + 2*pad_h - r)/stride_h + 1,  Q = (w + 2*pad_w - s)/stride_w + 1
  *
  * x: [n,h,w,c] bf16, w: [k,r,s,c] bf16, y: [n,P,Q,k] bf16, all NHWC/KRSC.
- * Supported: r == s, c and k multiples of 64, or the stem case c == 8
- * (3 colour channels zero-padded to 8) for the forward and weight passes.
+ * Supported: c and k multiples of 64 (any r, s <= 8 with stride <= 2 and
+ * pad <= 3 per axis for the forward and weight passes; square filters with
+ * equal strides and pads for the data gradient), or c == 8 (3 colour
+ * channels zero-padded to 8) for the forward and weight passes.  The stem of
+ * ResNet-18 is run as an r x 1 convolution over the input unrolled along W
+ * (see dbl_progressive_resize_stem).
  * ======================================================================== */
 typedef struct {
     int32_t n, h, w, c; /* input activation shape (NHWC)                    */
     int32_t k, r, s;    /* output channels and filter size (KRSC weights)   */
-    int32_t stride, pad;
+    int32_t stride, pad;       /* along H (and along W when stride_w == 0)   */
+    int32_t stride_w, pad_w;   /* along W; stride_w == 0: same as stride/pad */
 } dbl_conv_shape;
 
 enum { DBL_PASS_FWD = 0, DBL_PASS_DGRAD = 1, DBL_PASS_WGRAD = 2 };
@@ -242,6 +247,20 @@ DBL_API int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const flo
  * ======================================================================== */
 DBL_API int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
                            int out_dtype, int32_t h_out, int32_t w_out, int32_t c_out_stride, void* stream);
+
+/* The same resize, written in the layout the tensor-core stem consumes: the
+ * resized image unrolled along W for a stem with `taps` filter columns,
+ * column stride stride_w and padding pad_w.  Output position (n, h, q) holds
+ * the resized pixels at columns q*stride_w + t - pad_w, t = 0..7, each with
+ * 8 channels (t >= taps, columns outside the image and channels >= c are
+ * zero):  out[n][h][q][t][ch], bf16, Q = (w_out + 2*pad_w - taps)/stride_w + 1.
+ * A taps x taps stem convolution of the resized image then equals an
+ * r x 1 convolution (stride along H only, 64 channels) of this tensor with
+ * the weights stored as [k][r][8][8] (taps and channels zero-padded).
+ * in: [n,h_in,w_in,c] fp32, c <= 8, taps <= 8. */
+DBL_API int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
+                                        int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
+                                        void* stream);
 
 /* Host: the integer taps above for one axis (i0, i1, lambda: [out] each). */
 DBL_API int dbl_resize_taps(int32_t in, int32_t out, int32_t* i0, int32_t* i1, float* lambda);

@@ -53,7 +53,7 @@ struct ConvParams {
     int total_tiles;
     // traversal grid of the im2col operand: (images, rows, cols) and origin of grid point (0,0)
     int gN, gP, gQ;
-    int tstride;        // origin step per grid step
+    int tstride_h, tstride_w;  // origin step per grid step
     int base_h, base_w;
     int cblocks;        // 64-channel blocks in the reduction (fwd: C/64, dgrad: K/64)
     int ntaps;          // R*S
@@ -153,7 +153,7 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
         if (p.mode == kFwd) {
             const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
             const int r = tap / p.S, sx = tap - r * p.S;
-            tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride + p.base_w, tp * p.tstride + p.base_h, tn,
+            tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
                                (uint16_t)sx, (uint16_t)r);
             tma_load_2d(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
         } else if (p.mode == kDgrad) {
@@ -168,8 +168,8 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
                 int tap = kb * 8 + j;
                 const int wcol = tap * 8;
                 if (tap >= p.ntaps) tap = p.ntaps - 1;
-                tma_load_im2col_4d(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride + p.base_w,
-                                   tp * p.tstride + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_im2col_4d(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride_w + p.base_w,
+                                   tp * p.tstride_h + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
                 tma_load_2d(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
             }
         }
@@ -185,14 +185,14 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
                 int tap = mrow / p.Cin;
                 const int c0 = mrow - tap * p.Cin;
                 if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
-                tma_load_im2col_4d(sa + h * 16384, tmA, fb, c0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
+                tma_load_im2col_4d(sa + h * 16384, tmA, fb, c0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
                                    (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         } else {  // kWgradC8: 16 taps x 8 channels of rows
             for (int j = 0; j < 16; ++j) {
                 int tap = tc.m_tile * 16 + j;
                 if (tap >= p.ntaps) tap = 0;
-                tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, qq * p.tstride + p.base_w, pp * p.tstride + p.base_h, n,
+                tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
                                    (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         }
@@ -535,21 +535,32 @@ int choose_bn(int cols)
     return 64;
 }
 
+// Strides and pads per axis (stride_w == 0 means: the same as along H).
+struct Geom {
+    int sh, sw, ph, pw;
+};
+
+Geom geom(const dbl_conv_shape* s)
+{
+    Geom g{s->stride, s->stride_w ? s->stride_w : s->stride, s->pad, s->stride_w ? s->pad_w : s->pad};
+    return g;
+}
+
 int validate(const dbl_conv_shape* s, const char* who)
 {
     using dbl::set_error;
     if (!s) return set_error(DBL_ERR_INVALID, "%s: null shape", who);
-    if (s->n <= 0 || s->h <= 0 || s->w <= 0 || s->c <= 0 || s->k <= 0 || s->r <= 0 || s->s <= 0 || s->stride <= 0 ||
-        s->pad < 0)
+    const Geom g = geom(s);
+    if (s->n <= 0 || s->h <= 0 || s->w <= 0 || s->c <= 0 || s->k <= 0 || s->r <= 0 || s->s <= 0 || g.sh <= 0 ||
+        g.sw <= 0 || g.ph < 0 || g.pw < 0)
         return set_error(DBL_ERR_INVALID, "%s: non-positive dimension", who);
-    if (s->r != s->s) return set_error(DBL_ERR_UNSUPPORTED, "%s: only square filters", who);
     if (s->c % 8) return set_error(DBL_ERR_INVALID, "%s: channels must be a multiple of 8", who);
     if (s->k % 64) return set_error(DBL_ERR_UNSUPPORTED, "%s: output channels must be a multiple of 64", who);
     if (s->k > kMaxNcols || s->c > kMaxNcols * 8)
         return set_error(DBL_ERR_UNSUPPORTED, "%s: at most %d output channels", who, kMaxNcols);
-    if (s->stride > 2 || s->r > 7 || s->pad > 3)
-        return set_error(DBL_ERR_UNSUPPORTED, "%s: stride <= 2, filter <= 7, pad <= 3 supported", who);
-    if (out_dim(s->h, s->r, s->stride, s->pad) <= 0 || out_dim(s->w, s->s, s->stride, s->pad) <= 0)
+    if (g.sh > 2 || g.sw > 2 || s->r > 8 || s->s > 8 || g.ph > 3 || g.pw > 3)
+        return set_error(DBL_ERR_UNSUPPORTED, "%s: stride <= 2, filter <= 8, pad <= 3 per axis supported", who);
+    if (out_dim(s->h, s->r, g.sh, g.ph) <= 0 || out_dim(s->w, s->s, g.sw, g.pw) <= 0)
         return set_error(DBL_ERR_INVALID, "%s: empty output", who);
     return DBL_OK;
 }
@@ -569,7 +580,8 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
     using dbl::set_error;
     int rc = validate(s, pass == DBL_PASS_FWD ? "conv_fwd" : pass == DBL_PASS_DGRAD ? "conv_dgrad" : "conv_wgrad");
     if (rc) return rc;
-    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    const Geom g = geom(s);
+    const int P = out_dim(s->h, s->r, g.sh, g.ph), Q = out_dim(s->w, s->s, g.sw, g.pw);
     ConvParams& p = pl.p;
     memset(&p, 0, sizeof(p));
     const bool c8 = s->c == 8;
@@ -591,14 +603,18 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.gN = s->n;
         p.gP = P;
         p.gQ = Q;
-        p.tstride = s->stride;
-        p.base_h = p.base_w = -s->pad;
+        p.tstride_h = g.sh;
+        p.tstride_w = g.sw;
+        p.base_h = -g.ph;
+        p.base_w = -g.pw;
         p.cblocks = c8 ? 1 : s->c / 64;
         p.num_kb = c8 ? (p.ntaps + 7) / 8 : p.ntaps * p.cblocks;
         p.ldo = s->k;
         pl.ws_main = (size_t)kMaxGrid * 2 * s->k * sizeof(float);
     } else if (pass == DBL_PASS_DGRAD) {
         if (c8) return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: the 8-channel stem has no data gradient path");
+        if (s->r != s->s || g.sh != g.sw || g.ph != g.pw)
+            return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad: square filters with equal strides and pads only");
         pl.mode = p.mode = kDgrad;
         p.Ncols = s->c;
         pl.BN = choose_bn(s->c);
@@ -672,8 +688,10 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.gN = s->n;
         p.gP = P;
         p.gQ = Q;
-        p.tstride = s->stride;
-        p.base_h = p.base_w = -s->pad;
+        p.tstride_h = g.sh;
+        p.tstride_w = g.sw;
+        p.base_h = -g.ph;
+        p.base_w = -g.pw;
         const int64_t pix = (int64_t)s->n * P * Q;
         if ((pix + 127) / 128 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
         p.num_kb = (int)((pix + 127) / 128);  // K-blocks of 128 output pixels
@@ -694,15 +712,18 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
 
 size_t plan_ws(const Plan& pl) { return ((pl.ws_main + 255) / 256) * 256; }
 
-int enc_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int lower, int upper, int stride,
-               int channels, int pixels, bool swizzle)
+// im2col tensor map over an NHWC tensor.  Bounding-box corners and traversal
+// strides are given per spatial axis; the driver takes them innermost axis
+// first (W, then H), like the tensor dimensions.
+int enc_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int lower_h, int upper_h, int lower_w,
+               int upper_w, int stride_h, int stride_w, int channels, int pixels, bool swizzle)
 {
     auto fn = dbl::encode_im2col();
     if (!fn) return dbl::set_error(DBL_ERR_CUDA, "conv: cuTensorMapEncodeIm2col unavailable from the driver");
     cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
     cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
-    int lo[2] = {lower, lower}, hi[2] = {upper, upper};
-    cuuint32_t es[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+    int lo[2] = {lower_w, lower_h}, hi[2] = {upper_w, upper_h};
+    cuuint32_t es[4] = {1, (cuuint32_t)stride_w, (cuuint32_t)stride_h, 1};
     CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, lo, hi,
                     (cuuint32_t)channels, (cuuint32_t)pixels, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
@@ -784,9 +805,10 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
     if (stats && (!ws || ws_bytes < plan_ws(pl)))
         return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
     CUtensorMap ta, tb;
+    const Geom g = geom(s);
     if (pl.mode == kFwdC8) {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -s->pad, s->pad - (s->r - 1), s->stride, 8,
-                             fwd_tile_rows(pl.BN), false)))
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
+                             g.sw, 8, fwd_tile_rows(pl.BN), false)))
             return rc;
         const int64_t rsc = (int64_t)s->r * s->s * 8;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
@@ -794,8 +816,8 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         cuuint32_t box[2] = {8, (cuuint32_t)pl.BN};
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, false))) return rc;
     } else {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, 64,
-                             fwd_tile_rows(pl.BN), true)))
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
+                             g.sw, 64, fwd_tile_rows(pl.BN), true)))
             return rc;
         const int64_t rsc = (int64_t)s->r * s->s * s->c;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
@@ -834,7 +856,8 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
         lower = -(s->r - 1 - s->pad);
         upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
     }
-    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, 1, 64, fwd_tile_rows(pl.BN), true))) return rc;
+    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, lower, upper, 1, 1, 64, fwd_tile_rows(pl.BN), true)))
+        return rc;
     // w viewed as [k][r*s][c]: inner c, then tap, then k
     cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
     cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
@@ -855,11 +878,12 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
         return set_error(DBL_ERR_INVALID, "conv_wgrad: null or misaligned tensor");
     if (plan_ws(pl) && (!ws || ws_bytes < plan_ws(pl)))
         return set_error(DBL_ERR_WORKSPACE, "conv_wgrad: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
-    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    const Geom g = geom(s);
+    const int P = out_dim(s->h, s->r, g.sh, g.ph), Q = out_dim(s->w, s->s, g.sw, g.pw);
     CUtensorMap ta, tb;
     const bool c8 = pl.mode == kWgradC8;
-    if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -s->pad, s->pad - (s->r - 1), s->stride, c8 ? 8 : 64, 128,
-                         !c8)))
+    if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh, g.sw,
+                         c8 ? 8 : 64, 128, !c8)))
         return rc;
     cuuint64_t dims[2] = {(cuuint64_t)s->k, (cuuint64_t)s->n * P * Q};
     cuuint64_t str[1] = {(cuuint64_t)s->k * 2};

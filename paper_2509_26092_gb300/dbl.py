@@ -24,7 +24,7 @@ class DblError(RuntimeError):
 
 
 class ConvShape(ctypes.Structure):
-    _fields_ = [(f, ctypes.c_int32) for f in ("n", "h", "w", "c", "k", "r", "s", "stride", "pad")]
+    _fields_ = [(f, ctypes.c_int32) for f in ("n", "h", "w", "c", "k", "r", "s", "stride", "pad", "stride_w", "pad_w")]
 
 
 class BnShape(ctypes.Structure):
@@ -78,6 +78,8 @@ def lib():
             "dbl_progressive_resize": (ctypes.c_int, [_V, ctypes.c_int, _I32, _I32, _I32, _I32, _V, ctypes.c_int,
                                                       _I32, _I32, _I32, _V]),
             "dbl_resize_taps": (ctypes.c_int, [_I32, _I32, _V, _V, _V]),
+            "dbl_progressive_resize_stem": (ctypes.c_int, [_V, _I32, _I32, _I32, _I32, _V, _I32, _I32, _I32, _I32,
+                                                           _I32, _V]),
             "dbl_update_factor": (_D, [_D, _D, ctypes.c_int]),
             "dbl_plan": (ctypes.c_int, [_D, _D, _I32, _I32, _D, _D, _D, ctypes.c_int] + [ctypes.POINTER(_D)] * 4),
         }
@@ -131,8 +133,9 @@ def dbl_device_status():
     return v.value
 
 
-def conv_shape(n, h, w, c, k, r, stride, pad):
-    return ConvShape(n, h, w, c, k, r, r, stride, pad)
+def conv_shape(n, h, w, c, k, r, stride, pad, s=None, stride_w=0, pad_w=0):
+    """dbl_conv_shape; s defaults to r, stride_w == 0 means the same stride and pad along W."""
+    return ConvShape(n, h, w, c, k, r, r if s is None else s, stride, pad, stride_w, pad_w)
 
 
 def dbl_conv_workspace_bytes(shape, pass_):
@@ -215,6 +218,11 @@ def dbl_ps_dual_batch_merge(w, u, w16_out, g_large, g_small, n, lr, momentum, f_
 def dbl_progressive_resize(inp, in_dtype, n, h_in, w_in, c, out, out_dtype, h_out, w_out, c_out_stride, stream=None):
     _check(lib().dbl_progressive_resize(_ptr(inp), in_dtype, n, h_in, w_in, c, _ptr(out), out_dtype, h_out, w_out,
                                         c_out_stride, _stream(stream)))
+
+
+def dbl_progressive_resize_stem(inp, n, h_in, w_in, c, out, h_out, w_out, taps, stride_w, pad_w, stream=None):
+    _check(lib().dbl_progressive_resize_stem(_ptr(inp), n, h_in, w_in, c, _ptr(out), h_out, w_out, taps, stride_w, pad_w,
+                                             _stream(stream)))
 
 
 def dbl_resize_taps(n_in, n_out):

@@ -23,8 +23,14 @@ ResNet-18 (Sec. 5.1.1): stem convolution (3x3/1 for CIFAR-shaped inputs,
 7x7/2 + 3x3/2 max pooling for ImageNet-shaped inputs), four stages of two
 BasicBlocks (64/128/256/512 channels; the first block of stages 2-4 has
 stride 2 and a 1x1 stride-2 projection shortcut with BatchNorm), global
-average pooling and one fully connected layer.  The 3 colour channels are
-zero-padded to 8 so that a pixel is one 16-byte row.
+average pooling and one fully connected layer.
+
+The stem runs on the tensor cores as an R x 1 convolution: the input
+preparation (``dbl_progressive_resize_stem``) writes the resized image unrolled
+along W, 8 filter columns x 8 channels (3 colour channels, zero-padded) per
+output column, so the stem weights are stored as [64][R][8][8] (filter columns
+and channels zero-padded) and the R x R stem equals an R x 1 convolution of
+64-channel rows with stride (stride, 1).
 
 Convolutions read the bf16 weights ``w16``; BatchNorm and the fully connected
 layer read the fp32 master weights directly (they are tiny).
@@ -83,7 +89,7 @@ class ResNet18Spec:
             raise ValueError(variant)
         self.variant, self.classes, self.widths = variant, classes, tuple(widths)
         r, st, pad = (3, 1, 1) if variant == "cifar" else (7, 2, 3)
-        self.stem = ConvSpec("conv1", 8, 3, widths[0], r, st, pad)
+        self.stem = ConvSpec("conv1", 64, 3, widths[0], r, st, pad)  # 64 = 8 unrolled columns x 8 channels
         self.blocks = []
         cin = widths[0]
         for li, wd in enumerate(widths):
@@ -101,6 +107,10 @@ class ResNet18Spec:
             off += (e.numel + ALIGN - 1) // ALIGN * ALIGN
 
         def conv(cs):
+            if cs is self.stem:  # stored [k][r][8 columns][8 channels], logical [k][r][r][3]
+                add(cs.name + ".w", (cs.cout, cs.r, 8, 8), (cs.cout, cs.r, cs.r, cs.cin_logical),
+                    cs.r * cs.r * cs.cin_logical)
+                return
             add(cs.name + ".w", (cs.cout, cs.r, cs.r, cs.cin), (cs.cout, cs.r, cs.r, cs.cin_logical),
                 cs.r * cs.r * cs.cin_logical)
 
@@ -142,25 +152,22 @@ class ResNet18Spec:
         return flat[e.offset:e.offset + e.numel].view(e.shape)
 
     def pack(self, tensors, device="cuda", dtype=torch.float32):
-        """Flat buffer from {name: array of the logical shape} (stem channels zero-padded)."""
+        """Flat buffer from {name: array of the logical shape} (stem padding zero)."""
         flat = torch.zeros(self.n_flat, dtype=dtype, device=device)
         for e in self.entries:
             t = torch.as_tensor(tensors[e.name], dtype=dtype)
+            if tuple(t.shape) != e.logical:
+                raise ValueError(f"{e.name}: shape {tuple(t.shape)} != {e.logical}")
             v = self.view(flat, e.name)
-            if tuple(t.shape) == e.shape:
-                v.copy_(t)
-            else:
-                v.zero_()
-                v[..., :t.shape[-1]].copy_(t)
+            v.zero_()
+            v[tuple(slice(0, d) for d in e.logical)].copy_(t)
         return flat
 
     def unpack(self, flat):
         """{name: host float64 array of the logical shape} from a flat buffer."""
         out = {}
         for e in self.entries:
-            v = self.view(flat, e.name)
-            if e.shape != e.logical:
-                v = v[..., :e.logical[-1]]
+            v = self.view(flat, e.name)[tuple(slice(0, d) for d in e.logical)]
             out[e.name] = v.detach().double().cpu().numpy().copy()
         return out
 
@@ -195,10 +202,11 @@ class Worker:
         def vec(c):
             return torch.empty(c, dtype=torch.float32, device=dev)
 
-        self.x0 = act(res, 8)
         st = spec.stem
         p = conv_out(res, st.r, st.stride, st.pad)
         self.stem_hw = p
+        # stem input unrolled along W: [B, res, P, 8 columns x 8 channels]
+        self.x0 = torch.empty((B, res, p, 64), dtype=bf, device=dev)
         self.stem_y, self.stem_a, self.stem_da, self.stem_dy = act(p, st.cout), act(p, st.cout), None, act(p, st.cout)
         self.stem_stats = [vec(st.cout) for _ in range(4)]  # sum, sumsq, mean, invstd
         h = p
@@ -231,8 +239,7 @@ class Worker:
     def conv_shapes(self):
         """(name, dbl_conv_shape) of every convolution of this worker, in forward order."""
         B, spec = self.batch, self.spec
-        st = spec.stem
-        out = [(st.name, D.conv_shape(B, self.res, self.res, st.cin, st.cout, st.r, st.stride, st.pad))]
+        out = [(self.spec.stem.name, self.stem_shape())]
         for d in self.blocks:
             b = d["spec"]
             out.append((b.pre + ".conv1", D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)))
@@ -251,16 +258,26 @@ class Worker:
         need = max(need, D.dbl_bn_workspace_bytes(D.bn_shape(self.batch * self.stem_hw ** 2, self.spec.stem.cout)))
         return int(need) + 256
 
+    def stem_shape(self):
+        """The stem as an R x 1 convolution of the W-unrolled input (stride along H only)."""
+        st = self.spec.stem
+        return D.conv_shape(self.batch, self.res, self.stem_hw, 64, st.cout, st.r, st.stride, st.pad, s=1, stride_w=1,
+                            pad_w=0)
+
+    def layer_flops(self, name, s):
+        """Algorithmic FLOPs of one pass of a conv layer: 2*M*N*K over the unpadded problem
+        (for the stem: R x R taps of 3 colour channels)."""
+        st = self.spec.stem
+        if name == st.name:
+            return 2 * self.batch * self.stem_hw * self.stem_hw * st.cout * st.r * st.r * st.cin_logical
+        P = conv_out(s.h, s.r, s.stride, s.pad)
+        Q = conv_out(s.w, s.s, s.stride_w or s.stride, s.pad_w if s.stride_w else s.pad)
+        return 2 * s.n * P * Q * s.k * s.r * s.s * s.c
+
     def conv_flops(self):
-        """Algorithmic conv FLOPs of one step: 2*M*N*K per pass, unpadded channels,
-        forward + data gradient (not the stem) + weight gradient."""
-        total = 0
-        for name, s in self.conv_shapes():
-            P = conv_out(s.h, s.r, s.stride, s.pad)
-            cin = self.spec.stem.cin_logical if name == self.spec.stem.name else s.c
-            f = 2 * s.n * P * P * s.k * s.r * s.s * cin
-            total += f * (2 if name == self.spec.stem.name else 3)
-        return total
+        """Algorithmic conv FLOPs of one step: forward + data gradient (not the stem) + weight gradient."""
+        return sum(self.layer_flops(name, s) * (2 if name == self.spec.stem.name else 3)
+                   for name, s in self.conv_shapes())
 
     # ------------------------------------------------------------------ the step
     def enqueue_step(self, server, images, native_res, stream):
@@ -282,11 +299,11 @@ class Worker:
         def gv(name):
             return spec.view(G, name)
 
-        D.dbl_progressive_resize(images, D.DBL_F32, B, native_res, native_res, 3, self.x0, D.DBL_BF16, self.res,
-                                 self.res, 8, s)
-        # ---- forward
         st = spec.stem
-        shp = D.conv_shape(B, self.res, self.res, st.cin, st.cout, st.r, st.stride, st.pad)
+        D.dbl_progressive_resize_stem(images, B, native_res, native_res, 3, self.x0, self.res, self.res, st.r,
+                                      st.stride, st.pad, s)
+        # ---- forward
+        shp = self.stem_shape()
         s_sum, s_sq, s_mean, s_istd = self.stem_stats
         D.dbl_conv_fwd(shp, self.x0, wv("conv1.w"), self.stem_y, s_sum, s_sq, ws, wsb, s)
         bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)

@@ -47,3 +47,20 @@ def rng(seed):
 
 def check_status(D):
     assert D.dbl_device_status() == D.DBL_OK
+
+
+def stem_fold(x_u, r, stride, pad, width):
+    """Logical NHWC stem input [n, h, width, 8] from the W-unrolled tensor
+    [n, h, P, 8 taps, 8 channels] (x_u[..., q, t, :] is column q*stride + t - pad).
+    Checks that every copy of a column holds the same values."""
+    n, h, P = x_u.shape[0], x_u.shape[1], x_u.shape[2]
+    x_u = x_u.reshape(n, h, P, 8, 8)
+    out = np.full((n, h, width, 8), np.nan)
+    for q in range(P):
+        for t in range(r):
+            w = q * stride + t - pad
+            if 0 <= w < width:
+                if not np.all(np.isnan(out[:, :, w, :])):
+                    assert np.array_equal(out[:, :, w, :], x_u[:, :, q, t, :]), "unrolled copies disagree"
+                out[:, :, w, :] = x_u[:, :, q, t, :]
+    return out

@@ -89,7 +89,9 @@ def test_invalid_arguments_rejected_before_launch(D):
     # conv: unsupported channel counts, non-square filters, bad workspace
     s = D.ConvShape(2, 8, 8, 60, 64, 3, 3, 1, 1)
     assert L.dbl_conv_fwd(ctypes.byref(s), 16, 16, 16, None, None, None, 0, None) == D.DBL_ERR_INVALID
-    s = D.ConvShape(2, 8, 8, 64, 64, 3, 1, 1, 1)
+    s = D.ConvShape(2, 8, 8, 64, 64, 3, 1, 1, 1)  # non-square: fine forward, not for the data gradient
+    assert L.dbl_conv_dgrad(ctypes.byref(s), 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
+    s = D.ConvShape(2, 8, 8, 64, 64, 3, 3, 3, 1)  # stride 3
     assert L.dbl_conv_fwd(ctypes.byref(s), 16, 16, 16, None, None, None, 0, None) == D.DBL_ERR_UNSUPPORTED
     s = D.ConvShape(8, 32, 32, 64, 64, 3, 3, 1, 1)  # 8192 pixels: the reduction is split, needing a workspace
     assert D.dbl_conv_workspace_bytes(s, D.DBL_PASS_WGRAD) > 0
@@ -98,6 +100,8 @@ def test_invalid_arguments_rejected_before_launch(D):
     assert L.dbl_conv_dgrad(ctypes.byref(s), 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
     # resize: upsampling
     assert L.dbl_progressive_resize(16, 0, 1, 8, 8, 3, 16, 1, 16, 16, 8, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 8, 8, 3, 16, 16, 16, 7, 2, 3, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 3, 16, 16, 16, 9, 2, 3, None) == D.DBL_ERR_UNSUPPORTED
     # BN: channel count that is not a multiple of 8
     b = D.BnShape(100, 12, 1e-5, 1)
     assert L.dbl_bn_relu_fused(ctypes.byref(b), 16, 16, 16, 16, 16, None, 16, 16, 16, None) == D.DBL_ERR_UNSUPPORTED

@@ -11,7 +11,7 @@ import torch
 
 import oracle as orc
 from conftest import max_norm_rel
-from gpu_common import bf16_values, check_status, host, load_dbl, rng, to_bf16_dev, to_f32_dev, ws
+from gpu_common import bf16_values, check_status, host, load_dbl, rng, stem_fold, to_bf16_dev, to_f32_dev, ws
 
 pytestmark = pytest.mark.gpu
 
@@ -72,6 +72,68 @@ def test_resize_matches_oracle(D, n, hin, hout):
     out32 = torch.empty((n, hout, hout, 3), dtype=torch.float32, device="cuda")
     D.dbl_progressive_resize(xd, D.DBL_F32, n, hin, hin, 3, out32, D.DBL_F32, hout, hout, 3)
     assert max_norm_rel(host(out32), ref) <= 1e-6
+
+
+@pytest.mark.parametrize("n,hin,hout,r,st,pad", [(2, 224, 160, 7, 2, 3), (3, 32, 24, 3, 1, 1), (2, 224, 224, 7, 2, 3),
+                                                 (1, 20, 13, 7, 2, 3)])
+def test_resize_stem_unrolls_the_resized_image(D, n, hin, hout, r, st, pad):
+    x = rng(hin + hout + r).standard_normal((n, hin, hin, 3)).astype(np.float32)
+    ref = orc.bilinear_resize(x, hout, hout)
+    P = (hout + 2 * pad - r) // st + 1
+    out = torch.full((n, hout, P, 64), 7.0, dtype=torch.bfloat16, device="cuda")
+    D.dbl_progressive_resize_stem(to_f32_dev(x), n, hin, hin, 3, out, hout, hout, r, st, pad)
+    xu = host(out).reshape(n, hout, P, 8, 8)
+    assert np.all(xu[..., r:, :] == 0.0)      # taps past the filter width
+    assert np.all(xu[..., 3:] == 0.0)         # padded colour channels
+    for q in range(P):                        # columns outside the image
+        for t in range(r):
+            if not 0 <= q * st + t - pad < hout:
+                assert np.all(xu[:, :, q, t, :] == 0.0)
+    got = stem_fold(xu, r, st, pad, hout)[..., :3]
+    covered = ~np.isnan(got[0, 0, :, 0])
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
+    assert np.all(np.abs(got[:, :, covered] - ref[:, :, covered]) <= ulp[:, :, covered] + 1e-30)
+    check_status(D)
+
+
+STEM_CASES = [  # n, h (square input), r, stride, pad
+    (2, 20, 7, 2, 3),    # ImageNet stem on a small image
+    (3, 10, 3, 1, 1),    # CIFAR stem
+    (4, 64, 7, 2, 3),    # several tiles
+]
+
+
+def _stem_inputs(n, h, r, seed):
+    g = rng(seed)
+    x = bf16_values(g.standard_normal((n, h, h, 3)))
+    wt = bf16_values(g.standard_normal((64, r, r, 3)) * np.sqrt(2.0 / (r * r * 3)))
+    w_store = np.zeros((64, r, 8, 8))
+    w_store[:, :, :r, :3] = wt
+    return x, wt, w_store
+
+
+@pytest.mark.parametrize("case", STEM_CASES)
+def test_unrolled_stem_fwd_and_wgrad_match_oracle(D, case):
+    n, h, r, st, pad = case
+    x, wt, w_store = _stem_inputs(n, h, r, 21)
+    P = (h + 2 * pad - r) // st + 1
+    xu = torch.empty((n, h, P, 64), dtype=torch.bfloat16, device="cuda")
+    D.dbl_progressive_resize_stem(to_f32_dev(x), n, h, h, 3, xu, h, h, r, st, pad)  # same size: exact copy
+    shape = D.conv_shape(n, h, P, 64, 64, r, st, pad, s=1, stride_w=1, pad_w=0)
+    y = torch.full((n, P, P, 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    s1, s2 = torch.empty(64, device="cuda"), torch.empty(64, device="cuda")
+    wsb = max(D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_FWD), D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_WGRAD))
+    D.dbl_conv_fwd(shape, xu, to_bf16_dev(w_store), y, s1, s2, ws(wsb), wsb)
+    ref = orc.conv2d_fwd(x, wt, st, pad)
+    assert max_norm_rel(host(y), ref) <= CONV_TOL
+    dy = bf16_values(rng(22).standard_normal((n, P, P, 64)))
+    dw = torch.full((64, r, 8, 8), float("nan"), device="cuda")
+    D.dbl_conv_wgrad(shape, xu, to_bf16_dev(dy), dw, False, ws(wsb), wsb)
+    got = host(dw)
+    assert np.all(got[:, :, r:, :] == 0.0) and np.all(got[..., 3:] == 0.0)  # padding gets no gradient
+    rdw = orc.conv2d_wgrad(x, dy, wt.shape, st, pad)
+    assert max_norm_rel(got[:, :, :r, :3], rdw) <= CONV_TOL
+    check_status(D)
 
 
 # ----------------------------------------------------------------------------- BatchNorm

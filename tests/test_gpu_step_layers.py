@@ -13,7 +13,7 @@ import torch
 
 import oracle as orc
 from conftest import max_norm_rel
-from gpu_common import load_dbl
+from gpu_common import load_dbl, stem_fold
 from paper_2509_26092_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -50,8 +50,10 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
     eps = wk.eps
     # ---------------- forward
     st = spec.stem
-    x0 = h(wk.x0)
-    chk("stem.conv", h(wk.stem_y), orc.conv2d_fwd(x0, W16["conv1.w"], st.stride, st.pad))
+    x0 = stem_fold(h(wk.x0), st.r, st.stride, st.pad, res)[..., :3]  # the logical stem input
+    assert not np.any(np.isnan(x0))
+    w_stem = W16["conv1.w"][:, :, :st.r, :3]
+    chk("stem.conv", h(wk.stem_y), orc.conv2d_fwd(x0, w_stem, st.stride, st.pad))
     o, m, s = orc.bn_fwd(h(wk.stem_y), P["bn1.g"], P["bn1.b"], eps, relu=True)
     chk("stem.bn", h(wk.stem_a), o)
     chk("stem.bn.mean", h(wk.stem_stats[2]), m, 1e-4)
@@ -130,8 +132,9 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
         dys, dgs, dbs, _ = orc.bn_bwd(dout, h(wk.stem_a), h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3],
                                       dout2=dout2)
     chk("stem.bn.bwd", h(wk.stem_dy), dys)
-    wst = orc.conv2d_wgrad(x0, h(wk.stem_dy), W16["conv1.w"].shape, st.stride, st.pad)
-    chk("stem.wgrad", G["conv1.w"][..., :3], wst[..., :3])
-    assert np.all(G["conv1.w"][..., 3:] == 0.0)  # padded input channels get no gradient
+    wst = orc.conv2d_wgrad(x0, h(wk.stem_dy), w_stem.shape, st.stride, st.pad)
+    chk("stem.wgrad", G["conv1.w"][:, :, :st.r, :3], wst)
+    # padded filter columns and input channels get no gradient
+    assert np.all(G["conv1.w"][:, :, st.r:, :] == 0.0) and np.all(G["conv1.w"][..., 3:] == 0.0)
     worst = sorted(errs.items(), key=lambda kv: -kv[1])[:6]
     print(f"\n{variant}: {len(errs)} layer checks; worst " + ", ".join(f"{k}={v:.2e}" for k, v in worst))
