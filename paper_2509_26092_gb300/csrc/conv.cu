@@ -35,7 +35,6 @@ using namespace dbl::dev;
 
 constexpr int BM = 128;        // tile rows = TMEM lanes
 constexpr int BK = 64;         // reduction elements per stage (128 bytes of bf16)
-constexpr int kA_BYTES = BM * BK * 2;
 constexpr int kTargetCTAs = 304;  // 2 x 152 SMs: split-K sizing target (device independent)
 
 enum Mode : int { kFwd = 0, kDgrad = 1, kWgrad = 2, kFwdC8 = 3, kWgradC8 = 4 };
@@ -153,24 +152,24 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
         if (p.mode == kFwd) {
             const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
             const int r = tap / p.S, sx = tap - r * p.S;
-            tma_load_im2col_4d(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
+            tma_load_im2col_4d_elect(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
                                (uint16_t)sx, (uint16_t)r);
-            tma_load_2d(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
+            tma_load_2d_elect(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
         } else if (p.mode == kDgrad) {
             const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
-            tma_load_im2col_4d(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
+            tma_load_im2col_4d_elect(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
                                (uint16_t)p.tap_oh[t]);
             const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
             for (int j = 0; j < BN / 64; ++j)
-                tma_load_3d(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
+                tma_load_3d_elect(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
         } else {  // kFwdC8: 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
             for (int j = 0; j < 8; ++j) {
                 int tap = kb * 8 + j;
                 const int wcol = tap * 8;
                 if (tap >= p.ntaps) tap = p.ntaps - 1;
-                tma_load_im2col_4d(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride_w + p.base_w,
+                tma_load_im2col_4d_elect(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride_w + p.base_w,
                                    tp * p.tstride_h + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
-                tma_load_2d(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
+                tma_load_2d_elect(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
             }
         }
     } else {
@@ -185,18 +184,18 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
                 int tap = mrow / p.Cin;
                 const int c0 = mrow - tap * p.Cin;
                 if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
-                tma_load_im2col_4d(sa + h * 16384, tmA, fb, c0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
+                tma_load_im2col_4d_elect(sa + h * 16384, tmA, fb, c0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
                                    (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         } else {  // kWgradC8: 16 taps x 8 channels of rows
             for (int j = 0; j < 16; ++j) {
                 int tap = tc.m_tile * 16 + j;
                 if (tap >= p.ntaps) tap = 0;
-                tma_load_im2col_4d(sa + j * 2048, tmA, fb, 0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
+                tma_load_im2col_4d_elect(sa + j * 2048, tmA, fb, 0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
                                    (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         }
-        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 16384, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
+        for (int j = 0; j < BN / 64; ++j) tma_load_2d_elect(sb + j * 16384, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
     }
 }
 
@@ -253,110 +252,110 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
 
     if (warp >= 4 && warp < 4 + kProducers) {
-        // ------------------------------------------------------------------ TMA producers
+        // ------------------------------------------------------------------ TMA producers (whole warp, one lane issues)
         const int prod = warp - 4;
-        if (lane == 0) {
-            int it = 0, last_it = -1;
-            for (int t = blockIdx.x; t < p.total_tiles && !abort_flag; t += gridDim.x) {
-                const TileCoord tc = decode_tile(p, t);
-                int kb0, nkb;
-                kb_range(p, tc.z, kb0, nkb);
-                int tn = 0, tp = 0, tq = 0;
-                if (FAM == kFamFwd) {
-                    const int64_t m0 = (int64_t)tc.m_tile * C::BMT;
-                    tn = (int)(m0 / gPQ);
-                    const int64_t rem = m0 - (int64_t)tn * gPQ;
-                    tp = (int)(rem / p.gQ);
-                    tq = (int)(rem - (int64_t)tp * p.gQ);
-                }
-                for (int k = 0; k < nkb; ++k, ++it) {
-                    if (it % kProducers != prod) continue;
-                    const int s = it % STAGES;
-                    if (!mbar_wait(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag)) {
-                        report_timeout(&abort_flag);
-                        break;
-                    }
-                    uint8_t* sa = sgen + s * C::STAGE_BYTES;
-                    mbar_arrive_expect_tx(&full_bar[s], (uint32_t)C::STAGE_BYTES);
-                    load_kblock<BN, FAM>(p, &tmA, &tmB, sa, sa + C::A_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
-                    last_it = it;
-                }
+        int it = 0, last_it = -1;
+        bool failed = false;
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+            const TileCoord tc = decode_tile(p, t);
+            int kb0, nkb;
+            kb_range(p, tc.z, kb0, nkb);
+            int tn = 0, tp = 0, tq = 0;
+            if (FAM == kFamFwd) {
+                const int64_t m0 = (int64_t)tc.m_tile * C::BMT;
+                tn = (int)(m0 / gPQ);
+                const int64_t rem = m0 - (int64_t)tn * gPQ;
+                tp = (int)(rem / p.gQ);
+                tq = (int)(rem - (int64_t)tp * p.gQ);
             }
-            if (abort_flag) {
-                // let copies this producer issued land before the CTA's shared memory goes away
-                for (int i = last_it; i >= 0 && i > last_it - STAGES * kProducers; i -= kProducers)
-                    (void)mbar_wait_drain(&full_bar[i % STAGES], (i / STAGES) & 1);
+            for (int k = 0; k < nkb; ++k, ++it) {
+                if (it % kProducers != prod) continue;
+                const int s = it % STAGES;
+                const uint32_t ok = mbar_wait_warp(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag);
+                if (__any_sync(0xffffffffu, ok == 0u)) {
+                    failed = true;
+                    break;
+                }
+                uint8_t* sa = sgen + s * C::STAGE_BYTES;
+                mbar_arrive_expect_tx_elect(&full_bar[s], (uint32_t)C::STAGE_BYTES);
+                load_kblock<BN, FAM>(p, &tmA, &tmB, sa, sa + C::A_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
+                last_it = it;
             }
+            if (failed) break;
         }
-        __syncwarp();
+        if (failed) {
+            if (lane == 0) report_timeout(&abort_flag);
+            // let copies this producer issued land before the CTA's shared memory goes away
+            for (int i = last_it; i >= 0 && i > last_it - STAGES * kProducers; i -= kProducers)
+                (void)mbar_drain_warp(&full_bar[i % STAGES], (i / STAGES) & 1);
+        }
     } else if (warp == C::MMA_WARP) {
-        // ------------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
-            const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
-            const uint32_t idesc = idesc_bf16(BM, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
-            int it = 0, lt = 0;
-            for (int t = blockIdx.x; t < p.total_tiles && !abort_flag; t += gridDim.x, ++lt) {
-                const TileCoord tc = decode_tile(p, t);
-                int kb0, nkb;
-                kb_range(p, tc.z, kb0, nkb);
-                const int buf = lt & 1;
-                if (!mbar_wait(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag)) {
-                    report_timeout(&abort_flag);
+        // ------------------------------------------------------------------ MMA issuer (whole warp, one lane issues)
+        const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
+        const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
+        const uint32_t idesc = idesc_bf16(BM, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
+        int it = 0, lt = 0;
+        bool failed = false;
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
+            const TileCoord tc = decode_tile(p, t);
+            int kb0, nkb;
+            kb_range(p, tc.z, kb0, nkb);
+            const int buf = lt & 1;
+            const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                failed = true;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d = tmem + (uint32_t)(buf * C::ACC * BN);
+            for (int k = 0; k < nkb; ++k, ++it) {
+                const int s = it % STAGES;
+                const uint32_t okk = mbar_wait_warp(&full_bar[s], (it / STAGES) & 1, &abort_flag);
+                if (__any_sync(0xffffffffu, okk == 0u)) {
+                    failed = true;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(buf * C::ACC * BN);
-                bool ok = true;
-                for (int k = 0; k < nkb; ++k, ++it) {
-                    const int s = it % STAGES;
-                    if (!mbar_wait(&full_bar[s], (it / STAGES) & 1, &abort_flag)) {
-                        report_timeout(&abort_flag);
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t sa = sbase + s * C::STAGE_BYTES;
-                    const uint32_t sb = sa + C::A_BYTES;
+                const uint32_t sa = sbase + s * C::STAGE_BYTES;
+                const uint32_t sb = sa + C::A_BYTES;
 #pragma unroll
-                    for (int j = 0; j < C::KSTEPS; ++j) {
+                for (int j = 0; j < C::KSTEPS; ++j) {
 #pragma unroll
-                        for (int a = 0; a < C::ACC; ++a) {
-                            uint64_t ad, bd;
-                            if (p.mode == kFwd) {
-                                ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
-                                bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
-                            } else if (p.mode == kDgrad) {
-                                ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
-                                bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                            } else if (p.mode == kFwdC8) {
-                                // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
-                                // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
-                                ad = smem_desc(sa + a * 2048 + 2 * (C::BMT * 16) * j, C::BMT * 16, 128, kSwizzleNone);
-                                bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
-                            } else if (p.mode == kWgrad) {
-                                // MN-major, 128-byte swizzle: 64-wide atoms 16 KB apart (LBO)
-                                ad = smem_desc(sa + 2048 * j, 16384, 1024, kSwizzle128B);
-                                bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
-                            } else {
-                                // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
-                                // next 8 pixels 128 B apart (LBO), next tap 2 KB apart (SBO)
-                                ad = smem_desc(sa + 256 * j, 128, 2048, kSwizzleNone);
-                                bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
-                            }
-                            mma_bf16(d + a * BN, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
+                    for (int a = 0; a < C::ACC; ++a) {
+                        uint64_t ad, bd;
+                        if (p.mode == kFwd) {
+                            ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
+                        } else if (p.mode == kDgrad) {
+                            ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
+                        } else if (p.mode == kFwdC8) {
+                            // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
+                            // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
+                            ad = smem_desc(sa + a * 2048 + 2 * (C::BMT * 16) * j, C::BMT * 16, 128, kSwizzleNone);
+                            bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
+                        } else if (p.mode == kWgrad) {
+                            // MN-major, 128-byte swizzle: 64-wide atoms 16 KB apart (LBO)
+                            ad = smem_desc(sa + 2048 * j, 16384, 1024, kSwizzle128B);
+                            bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
+                        } else {
+                            // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
+                            // next 8 pixels 128 B apart (LBO), next tap 2 KB apart (SBO)
+                            ad = smem_desc(sa + 256 * j, 128, 2048, kSwizzleNone);
+                            bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
                         }
+                        mma_bf16_elect(d + a * BN, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
                     }
-                    mma_commit(&empty_bar[s]);
                 }
-                mma_commit(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
-                if (!ok) break;
+                mma_commit_elect(&empty_bar[s]);
             }
-            // every MMA issued above completes before the accumulators are freed
-            mma_commit(&drain_bar);
-            (void)mbar_wait_drain(&drain_bar, 0);
+            mma_commit_elect(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
+            if (failed) break;
         }
-        __syncwarp();
+        if (failed && lane == 0) report_timeout(&abort_flag);
+        // every MMA issued above completes before the accumulators are freed
+        mma_commit_elect(&drain_bar);
+        (void)mbar_drain_warp(&drain_bar, 0);
     } else {
         // ------------------------------------------------------------------ epilogue (warps 0-3)
         float* st_tile = epi_tile + warp * 32 * 33;
@@ -367,9 +366,9 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
             const int buf = lt & 1;
-            const bool ok = mbar_wait(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
-            if (!ok) {
-                report_timeout(&abort_flag);
+            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                if (lane == 0) report_timeout(&abort_flag);
                 break;
             }
             tc_fence_after();

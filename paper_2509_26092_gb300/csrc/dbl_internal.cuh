@@ -139,6 +139,98 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity)
     return false;
 }
 
+// Warp-uniform forms for the MMA and TMA issuing warps.  All 32 lanes run
+// the same straight-line code: the wait loop lives inside one asm block (no
+// lane-dependent C++ control flow around the tcgen05/TMA issue, which would
+// otherwise slow the issue rate about threefold), and the single-thread
+// operations are issued by the lane that elect.sync picks (the lowest active
+// lane, so the same lane every time in a converged warp).
+//
+// Bounded wait: returns 1 once the phase with the given parity has
+// completed, 0 if *abort is (or becomes) nonzero, or if the poll or time
+// limit ran out, in which case it sets *abort itself so that every other
+// wait of the CTA gives up promptly.  abort points to shared memory.
+__device__ __forceinline__ uint32_t mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t"
+        ".reg .pred P1, P2;\n\t"
+        ".reg .u32 cnt, fl;\n\t"
+        ".reg .u64 t0, t1;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 P1, [%1], %2;\n\t"
+        "@P1 bra WAIT_END;\n\t"
+        "mov.u32 cnt, 0;\n\t"
+        "mov.u64 t0, %%globaltimer;\n"
+        "WAIT_POLL:\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 P1, [%1], %2;\n\t"
+        "@P1 bra WAIT_END;\n\t"
+        "add.u32 cnt, cnt, 1;\n\t"
+        "and.b32 fl, cnt, 63;\n\t"
+        "setp.ne.u32 P2, fl, 0;\n\t"
+        "@P2 bra WAIT_POLL;\n\t"
+        "setp.ge.u32 P2, cnt, %5;\n\t"
+        "@P2 bra WAIT_FAIL;\n\t"
+        "ld.volatile.shared.u32 fl, [%3];\n\t"
+        "setp.ne.u32 P2, fl, 0;\n\t"
+        "@P2 bra WAIT_END;\n\t"
+        "mov.u64 t1, %%globaltimer;\n\t"
+        "sub.u64 t1, t1, t0;\n\t"
+        "setp.lt.u64 P2, t1, %4;\n\t"
+        "@P2 bra WAIT_POLL;\n"
+        "WAIT_FAIL:\n\t"
+        "st.volatile.shared.u32 [%3], 1;\n"
+        "WAIT_END:\n\t"
+        "selp.u32 %0, 1, 0, P1;\n\t"
+        "}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(smem_u32(const_cast<int*>(abort))), "l"(kWaitLimitNs),
+          "r"(kWaitLimitPolls)
+        : "memory");
+    return ok;
+}
+
+// Warp-uniform wait on the way out of an aborted CTA: bounded by a short
+// time, not by the abort flag.  Returns 1 if the phase completed.
+__device__ __forceinline__ uint32_t mbar_drain_warp(uint64_t* bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t"
+        ".reg .pred P1, P2;\n\t"
+        ".reg .u32 cnt;\n\t"
+        ".reg .u64 t0, t1;\n\t"
+        "mov.u32 cnt, 0;\n\t"
+        "mov.u64 t0, %%globaltimer;\n"
+        "DRAIN_POLL:\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 P1, [%1], %2;\n\t"
+        "@P1 bra DRAIN_END;\n\t"
+        "add.u32 cnt, cnt, 1;\n\t"
+        "setp.ge.u32 P2, cnt, %4;\n\t"
+        "@P2 bra DRAIN_END;\n\t"
+        "mov.u64 t1, %%globaltimer;\n\t"
+        "sub.u64 t1, t1, t0;\n\t"
+        "setp.lt.u64 P2, t1, %3;\n\t"
+        "@P2 bra DRAIN_POLL;\n"
+        "DRAIN_END:\n\t"
+        "selp.u32 %0, 1, 0, P1;\n\t"
+        "}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "l"(kWaitLimitNs / 8), "r"(kWaitLimitPolls)
+        : "memory");
+    return ok;
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx_elect(uint64_t* bar, uint32_t bytes)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}" ::"r"(smem_u32(bar)),
+        "r"(bytes)
+        : "memory");
+}
+
 // ---------------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* tmap)
 {
@@ -173,6 +265,44 @@ __device__ __forceinline__ void tma_load_im2col_4d(void* dst, const void* tmap, 
     asm volatile(
         "cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8};" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w),
+        "h"(off_h)
+        : "memory");
+}
+
+// Elected-lane forms of the TMA loads above (whole warp calls, one lane issues).
+__device__ __forceinline__ void tma_load_2d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1,
+                                                  int32_t c2)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_im2col_4d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c,
+                                                         int32_t w, int32_t h, int32_t n, uint16_t off_w,
+                                                         uint16_t off_h)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8};\n\t}" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w),
         "h"(off_h)
         : "memory");
@@ -216,6 +346,30 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                  : "memory");
+}
+
+// Elected-lane forms: the whole warp calls, one lane issues.  The commit
+// tracks the MMAs issued by the elected lane, which is the same lane that
+// mma_bf16_elect uses in a converged warp.
+__device__ __forceinline__ void mma_bf16_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                               uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred E, P;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "setp.ne.b32 P, %4, 0;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, P;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_elect(uint64_t* bar)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(smem_u32(bar))
+        : "memory");
 }
 
 // 32 lanes x 32 consecutive 32-bit columns: thread i of the warp gets lane
