@@ -250,9 +250,10 @@ def build_pipeline(cfg, device):
                 lab_s=lab_s)
 
 
-def conv_roofline(stage, reps=3):
+def conv_roofline(stage, reps=3, table=None):
     """Time each convolution pass of the stage's workers alone with CUDA events;
-    return (algorithmic conv FLOPs of one iteration, seconds per iteration)."""
+    return (algorithmic conv FLOPs of one iteration, seconds per iteration).
+    If table is a list, append (worker batch, layer, pass, FLOPs, seconds) per pass."""
     import torch
 
     from paper_2509_26092_gb300 import dbl as D
@@ -272,7 +273,7 @@ def conv_roofline(stage, reps=3):
             if name != stem:
                 passes.append(("dgrad", lambda: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
             passes.append(("wgrad", lambda: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
-            for _, fn in passes:
+            for pname, fn in passes:
                 fn()
                 ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
                 ev[0].record(s)
@@ -280,8 +281,11 @@ def conv_roofline(stage, reps=3):
                     fn()
                 ev[1].record(s)
                 torch.cuda.synchronize()
-                secs += ev[0].elapsed_time(ev[1]) / 1000.0 / reps
+                t1 = ev[0].elapsed_time(ev[1]) / 1000.0 / reps
+                secs += t1
                 flops += f1
+                if table is not None:
+                    table.append((wk.batch, name, pname, f1, t1))
     return flops, secs
 
 
@@ -335,6 +339,60 @@ def run_profile_iteration(args, cfg):
         del it, large, small
     assert D.dbl_device_status() == D.DBL_OK
     print(json.dumps({"profile_iteration": args.config, "launches": D.dbl_kernel_launches() - n0}), flush=True)
+    return 0
+
+
+def run_profile_conv(args):
+    """Three launches of one convolution pass of one ResNet-18 layer (224 px input,
+    batch --profile-batch), with only that layer's operands on the device: the
+    command ncu captures for the per-kernel profiles (-k regex:conv_igemm -s 2 -c 1
+    takes the third, warm launch)."""
+    import torch
+
+    from paper_2509_26092_gb300 import build_lib
+    build_lib.build()
+    from paper_2509_26092_gb300 import dbl as D
+    from paper_2509_26092_gb300 import resnet18 as R
+
+    torch.cuda.set_device(0)
+    layer, pname = args.profile_conv.split(":")
+    spec = R.ResNet18Spec("imagenet", 1000)
+    n = args.profile_batch
+    h = R.conv_out(R.conv_out(224, spec.stem.r, spec.stem.stride, spec.stem.pad), 3, 2, 1)  # after stem and max-pool
+    shapes = {}
+    for b in spec.blocks:
+        ho = R.conv_out(h, 3, b.stride, 1)
+        shapes[b.pre + ".conv1"] = D.conv_shape(n, h, h, b.cin, b.cout, 3, b.stride, 1)
+        shapes[b.pre + ".conv2"] = D.conv_shape(n, ho, ho, b.cout, b.cout, 3, 1, 1)
+        if b.proj:
+            shapes[b.pre + ".down"] = D.conv_shape(n, h, h, b.cin, b.cout, 1, b.stride, 0)
+        h = ho
+    if layer not in shapes:
+        raise SystemExit(f"--profile-conv: unknown layer {layer!r} (one of {', '.join(shapes)})")
+    s = shapes[layer]
+    P = R.conv_out(s.h, s.r, s.stride, s.pad)
+    g = torch.Generator(device="cuda").manual_seed(0)
+    x = torch.randn(s.n, s.h, s.w, s.c, device="cuda", generator=g).to(torch.bfloat16)
+    w = (0.05 * torch.randn(s.k, s.r, s.s, s.c, device="cuda", generator=g)).to(torch.bfloat16)
+    dy = torch.randn(s.n, P, P, s.k, device="cuda", generator=g).to(torch.bfloat16)
+    ps = {"fwd": D.DBL_PASS_FWD, "dgrad": D.DBL_PASS_DGRAD, "wgrad": D.DBL_PASS_WGRAD}[pname]
+    ws = torch.empty(max(int(D.dbl_conv_workspace_bytes(s, ps)), 16), dtype=torch.uint8, device="cuda")
+    st = torch.cuda.current_stream()
+    if pname == "fwd":
+        y = torch.empty(s.n, P, P, s.k, dtype=torch.bfloat16, device="cuda")
+        ssum, ssq = torch.empty(s.k, device="cuda"), torch.empty(s.k, device="cuda")
+        fn = lambda: D.dbl_conv_fwd(s, x, w, y, ssum, ssq, ws, ws.numel(), st)
+    elif pname == "dgrad":
+        dx = torch.empty_like(x)
+        fn = lambda: D.dbl_conv_dgrad(s, dy, w, dx, None, 0, st)
+    else:
+        dw = torch.empty(s.k * s.r * s.s * s.c, device="cuda")
+        fn = lambda: D.dbl_conv_wgrad(s, x, dy, dw, False, ws, ws.numel(), st)
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    assert D.dbl_device_status() == D.DBL_OK
+    print(json.dumps({"profile_conv": args.profile_conv, "batch": n}), flush=True)
     return 0
 
 
@@ -434,7 +492,12 @@ def run_ours(args, cfg):
     for wk in (top["large"], top["small"]):
         if wk is not None:
             wk._bench_w16 = pipe["server"].w16
-    flops, secs = conv_roofline(top)
+    table = [] if args.conv_table else None
+    flops, secs = conv_roofline(top, table=table)
+    if table is not None:
+        for b, name, pname, f1, t1 in table:
+            print(f"conv {b:4d} {name:16s} {pname:5s} {t1 * 1e6:9.1f} us {f1 / t1 / 1e12:7.1f} TFLOP/s",
+                  file=sys.stderr)
     achieved = flops / secs / 1e12
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16, "unit": "TFLOP/s",
                 "frac": round(achieved / bf16, 4), "traffic": _traffic_record(args.config),
@@ -476,12 +539,19 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--conv-table", action="store_true",
+                    help="print each convolution pass's time and TFLOP/s (largest stage) to stderr")
+    ap.add_argument("--profile-conv", default=None, metavar="LAYER:PASS",
+                    help="run one conv pass of one layer three times (e.g. layer1.0.conv1:fwd) for ncu")
+    ap.add_argument("--profile-batch", type=int, default=512)
     ap.add_argument("--profile-iteration", action="store_true",
                     help="run one eager iteration per stage and exit (the command ncu profiles)")
     args = ap.parse_args()
     cfg = CONFIGS[args.config]
     if args.impl == "reference":
         return run_reference(args, cfg)
+    if args.profile_conv:
+        return run_profile_conv(args)
     if args.profile_iteration:
         return run_profile_iteration(args, cfg)
     return run_ours(args, cfg)

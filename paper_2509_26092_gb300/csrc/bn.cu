@@ -17,6 +17,9 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kMaxC = 2048;
+constexpr int kUnroll = 2;  // rows per thread whose loads are in flight together
+constexpr int kBlocksPerSM = 4;     // forward apply: 256-thread CTAs resident per SM (64 registers per thread)
+constexpr int kBwdBlocksPerSM = 3;  // backward passes (85 registers per thread)
 
 __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 {
@@ -83,9 +86,9 @@ __global__ void __launch_bounds__(kThreads) bn_stats_kernel(const __nv_bfloat16*
 // vector) and visits rows t / (C/8), + rows-per-CTA-step, ...; a warp covers
 // consecutive vectors of consecutive rows, so every access is coalesced, and the
 // channel's scale and shift stay in registers.
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, kBlocksPerSM)
     bn_apply_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ res,
-                    __nv_bfloat16* __restrict__ out, int64_t count, int C, float eps, int relu,
+                    __nv_bfloat16* __restrict__ out, int count, int C, float eps, int relu,
                     const float* __restrict__ sum, const float* __restrict__ sumsq, const float* __restrict__ gamma,
                     const float* __restrict__ beta, float* __restrict__ save_mean, float* __restrict__ save_invstd)
 {
@@ -116,75 +119,121 @@ __global__ void __launch_bounds__(kThreads)
         sc[k] = s_sc[8 * g + k];
         sh[k] = s_sh[8 * g + k];
     }
-    const int64_t step = (int64_t)gridDim.x * rstep;
-    for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += step) {
-        const int64_t v = r * groups + g;
-        float f[8];
-        unpack8(__ldcs(reinterpret_cast<const uint4*>(y) + v), f);
-        float rr[8] = {};
-        if (res) unpack8(__ldcs(reinterpret_cast<const uint4*>(res) + v), rr);
+    const int step = gridDim.x * rstep;
+    auto emit = [&](const uint4& yv, const uint4& rv, int v) {
+        float f[8], rr[8];
+        unpack8(yv, f);
+        unpack8(rv, rr);
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
             const float o = fmaf(f[k], sc[k], sh[k]) + rr[k];
             f[k] = (relu && !(o > 0.f)) ? 0.f : o;
         }
         reinterpret_cast<uint4*>(out)[v] = pack8(f);
+    };
+    const uint4 zero = make_uint4(0, 0, 0, 0);  // bf16 +0 in every lane
+    int r = blockIdx.x * rstep + threadIdx.x / groups;
+    for (; r + (kUnroll - 1) * step < count; r += kUnroll * step) {
+        uint4 yv[kUnroll], rv[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int v = (r + u * step) * groups + g;
+            yv[u] = __ldcs(reinterpret_cast<const uint4*>(y) + v);
+            rv[u] = res ? __ldcs(reinterpret_cast<const uint4*>(res) + v) : zero;
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) emit(yv[u], rv[u], (r + u * step) * groups + g);
+    }
+    for (; r < count; r += step) {
+        const int v = r * groups + g;
+        emit(__ldcs(reinterpret_cast<const uint4*>(y) + v), res ? __ldcs(reinterpret_cast<const uint4*>(res) + v) : zero,
+             v);
     }
 }
 
 // ----------------------------------------------------------------------------- backward
-// g = (dout [+ dout2]) * [out > 0]
-__device__ __forceinline__ void load_g(const __nv_bfloat16* dout, const __nv_bfloat16* dout2,
-                                       const __nv_bfloat16* out, int relu, int64_t v, float (&g)[8])
+// The raw 16-byte vectors behind one 8-channel group of g = (dout [+ dout2]) * [out > 0]
+// and of the BatchNorm input y; loaded together so that several rows' loads are in flight.
+struct Vec8 {
+    uint4 d, d2, o, y;
+};
+
+__device__ __forceinline__ void load_g_raw(const __nv_bfloat16* dout, const __nv_bfloat16* dout2,
+                                           const __nv_bfloat16* out, int relu, const __nv_bfloat16* y, int v,
+                                           Vec8& g, Vec8& yv)
 {
-    unpack8(__ldg(reinterpret_cast<const uint4*>(dout) + v), g);
-    if (dout2) {
+    g.d = __ldcs(reinterpret_cast<const uint4*>(dout) + v);
+    g.d2 = dout2 ? __ldcs(reinterpret_cast<const uint4*>(dout2) + v) : make_uint4(0, 0, 0, 0);
+    g.o = relu ? __ldcs(reinterpret_cast<const uint4*>(out) + v) : make_uint4(0, 0, 0, 0);
+    yv.y = __ldcs(reinterpret_cast<const uint4*>(y) + v);
+}
+
+__device__ __forceinline__ void combine_g(const Vec8& raw, bool two, int relu, float (&g)[8])
+{
+    unpack8(raw.d, g);
+    if (two) {
         float h[8];
-        unpack8(__ldg(reinterpret_cast<const uint4*>(dout2) + v), h);
+        unpack8(raw.d2, h);
 #pragma unroll
         for (int k = 0; k < 8; ++k) g[k] += h[k];
     }
     if (relu) {
         float o[8];
-        unpack8(__ldg(reinterpret_cast<const uint4*>(out) + v), o);
+        unpack8(raw.o, o);
 #pragma unroll
         for (int k = 0; k < 8; ++k)
             if (!(o[k] > 0.f)) g[k] = 0.f;
     }
 }
 
-// Each CTA reduces a contiguous range of rows into partial[blk][0..C) (sum g)
-// and partial[blk][C..2C) (sum g*xhat).
-__global__ void __launch_bounds__(kThreads)
+// sg += g, sgc += g*(y - mean)  (the 1/std factor is applied once per partial)
+__device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw, bool two, int relu,
+                                             const float (&mu)[8], float (&sg)[8], float (&sgc)[8])
+{
+    float gg[8], yy[8];
+    combine_g(graw, two, relu, gg);
+    unpack8(yraw.y, yy);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        sg[k] += gg[k];
+        sgc[k] = fmaf(gg[k], yy[k] - mu[k], sgc[k]);
+    }
+}
+
+// Partial blk reduces a contiguous range of rows into partial[blk][0..C) (sum g)
+// and partial[blk][C..2C) (sum g*xhat); CTA b computes partials b, b + gridDim.x, ...
+// (each in a fixed order, so the result does not depend on the grid).
+__global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
-                         const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int64_t count,
+                         const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
                          int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
-                         int64_t rows_per_blk, float* __restrict__ partial)
+                         int rows_per_blk, int nblk, float* __restrict__ partial)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
-    float mu[8], is[8];
+    float mu[8];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-        mu[k] = mean[8 * g + k];
-        is[k] = invstd[8 * g + k];
-    }
-    float sg[8] = {}, sgx[8] = {};
-    const int64_t r0 = (int64_t)blockIdx.x * rows_per_blk;
-    const int64_t r1 = min(count, r0 + rows_per_blk);
-    for (int64_t r = r0 + threadIdx.x / groups; r < r1; r += rstep) {
-        const int64_t v = r * groups + g;
-        float gg[8], yy[8];
-        load_g(dout, dout2, out, relu, v, gg);
-        unpack8(__ldg(reinterpret_cast<const uint4*>(y) + v), yy);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            sg[k] += gg[k];
-            sgx[k] = fmaf(gg[k], (yy[k] - mu[k]) * is[k], sgx[k]);
-        }
-    }
+    for (int k = 0; k < 8; ++k) mu[k] = mean[8 * g + k];
     __shared__ float red[kThreads][17];
+    for (int blk = blockIdx.x; blk < nblk; blk += gridDim.x) {
+    float sg[8] = {}, sgx[8] = {};
+    const int r0 = blk * rows_per_blk;
+    const int r1 = min(count, r0 + rows_per_blk);
+    // kUnroll rows per iteration: all their loads are issued before any is used
+    int r = r0 + threadIdx.x / groups;
+    for (; r + (kUnroll - 1) * rstep < r1; r += kUnroll * rstep) {
+        Vec8 gg[kUnroll], yy[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) load_g_raw(dout, dout2, out, relu, y, (r + u * rstep) * groups + g, gg[u], yy[u]);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) accumulate_g(gg[u], yy[u], dout2 != nullptr, relu, mu, sg, sgx);
+    }
+    for (; r < r1; r += rstep) {
+        Vec8 gg, yy;
+        load_g_raw(dout, dout2, out, relu, y, r * groups + g, gg, yy);
+        accumulate_g(gg, yy, dout2 != nullptr, relu, mu, sg, sgx);
+    }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         red[threadIdx.x][k] = sg[k];
@@ -199,20 +248,24 @@ __global__ void __launch_bounds__(kThreads)
                 ts[k] += red[t][k];
                 tx[k] += red[t][8 + k];
             }
-        float* p = partial + (int64_t)blockIdx.x * 2 * C;
+        float* p = partial + (int64_t)blk * 2 * C;
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
             p[8 * threadIdx.x + k] = ts[k];
-            p[C + 8 * threadIdx.x + k] = tx[k];
+            p[C + 8 * threadIdx.x + k] = tx[k] * invstd[8 * threadIdx.x + k];  // sum g*(y-mean) -> sum g*xhat
         }
+    }
+    __syncthreads();
     }
 }
 
 // Fixed-order sum of the partials: one warp per channel, lane l sums blocks
 // l, l+32, ... in double, then a fixed butterfly across the warp; then dgamma,
-// dbeta and the three per-channel coefficients of the apply pass.
+// dbeta and the three per-channel coefficients (A, B, C) of the apply pass
+// dy = A*g + B*y + C.
 __global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C,
                                                               int64_t count, const float* __restrict__ gamma,
+                                                              const float* __restrict__ mean,
                                                               const float* __restrict__ invstd,
                                                               float* __restrict__ dgamma, float* __restrict__ dbeta,
                                                               float* __restrict__ coef)
@@ -233,52 +286,69 @@ __global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(const float* __res
     if (lane != 0) return;
     dbeta[c] = (float)sg;
     dgamma[c] = (float)sgx;
-    coef[c] = gamma[c] * invstd[c];
-    coef[C + c] = (float)(sg / (double)count);
-    coef[2 * C + c] = (float)(sgx / (double)count);
+    // dy = k1*(g - sum(g)/n - xhat*sum(g*xhat)/n), xhat = (y - mean)*invstd, as A*g + B*y + C
+    const double k1 = (double)gamma[c] * (double)invstd[c];
+    const double k3 = sgx / (double)count;
+    const double b = -k1 * (double)invstd[c] * k3;
+    coef[c] = (float)k1;
+    coef[C + c] = (float)b;
+    coef[2 * C + c] = (float)(-k1 * (sg / (double)count) - b * (double)mean[c]);
 }
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     bn_bwd_apply_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
-                        const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int64_t count,
+                        const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
                         int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
                         const float* __restrict__ coef, __nv_bfloat16* __restrict__ dy, __nv_bfloat16* __restrict__ dres)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
-    float k1[8], k2[8], k3[8], mu[8], is[8];
+    float ca[8], cb[8], cc[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         const int c = 8 * g + k;
-        k1[k] = coef[c];
-        k2[k] = coef[C + c];
-        k3[k] = coef[2 * C + c];
-        mu[k] = mean[c];
-        is[k] = invstd[c];
+        ca[k] = coef[c];
+        cb[k] = coef[C + c];
+        cc[k] = coef[2 * C + c];
     }
-    const int64_t step = (int64_t)gridDim.x * rstep;
-    for (int64_t r = (int64_t)blockIdx.x * rstep + threadIdx.x / groups; r < count; r += step) {
-        const int64_t v = r * groups + g;
+    const int step = gridDim.x * rstep;
+    auto emit = [&](const Vec8& graw, const Vec8& yraw, int v) {
         float gg[8], yy[8], d[8];
-        load_g(dout, dout2, out, relu, v, gg);
-        unpack8(__ldg(reinterpret_cast<const uint4*>(y) + v), yy);
+        combine_g(graw, dout2 != nullptr, relu, gg);
+        unpack8(yraw.y, yy);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const float xh = (yy[k] - mu[k]) * is[k];
-            d[k] = k1[k] * (gg[k] - k2[k] - xh * k3[k]);
-        }
-        reinterpret_cast<uint4*>(dy)[v] = pack8(d);
-        if (dres) reinterpret_cast<uint4*>(dres)[v] = pack8(gg);
+        for (int k = 0; k < 8; ++k) d[k] = fmaf(ca[k], gg[k], fmaf(cb[k], yy[k], cc[k]));
+        __stcs(reinterpret_cast<uint4*>(dy) + v, pack8(d));
+        if (dres) __stcs(reinterpret_cast<uint4*>(dres) + v, pack8(gg));
+    };
+    int r = blockIdx.x * rstep + threadIdx.x / groups;
+    for (; r + (kUnroll - 1) * step < count; r += kUnroll * step) {
+        Vec8 gg[kUnroll], yy[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) load_g_raw(dout, dout2, out, relu, y, (r + u * step) * groups + g, gg[u], yy[u]);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) emit(gg[u], yy[u], (r + u * step) * groups + g);
+    }
+    for (; r < count; r += step) {
+        Vec8 gg, yy;
+        load_g_raw(dout, dout2, out, relu, y, r * groups + g, gg, yy);
+        emit(gg, yy, r * groups + g);
     }
 }
 
-int bn_grid(int64_t nvec)
+int bn_grid(int64_t nvec, int per_sm = kBlocksPerSM)
 {
     int64_t b = (nvec + kThreads - 1) / kThreads;
-    const int64_t cap = (int64_t)dbl::sm_count() * 8;
+    const int64_t cap = (int64_t)dbl::sm_count() * per_sm;
     if (b > cap) b = cap;
     return (int)(b < 1 ? 1 : b);
+}
+
+int reduce_grid(int64_t nblk)
+{
+    const int64_t cap = (int64_t)dbl::sm_count() * kBwdBlocksPerSM;
+    return (int)(nblk < cap ? nblk : cap);
 }
 
 int check_shape(const dbl_bn_shape* s, const char* who)
@@ -287,12 +357,22 @@ int check_shape(const dbl_bn_shape* s, const char* who)
     if (s->c % 8 != 0 || s->c > kMaxC || (kThreads % (s->c / 8)) != 0)
         return dbl::set_error(DBL_ERR_UNSUPPORTED, "%s: channel count %d (need a multiple of 8 dividing 2048)", who,
                               s->c);
+    // the streaming kernels index 16-byte vectors (and rows, plus one grid step) in 32 bits
+    if (s->count * (s->c / 8) + (int64_t)kThreads * dbl::sm_count() * kBlocksPerSM * kUnroll >= ((int64_t)1 << 31))
+        return dbl::set_error(DBL_ERR_UNSUPPORTED, "%s: %lld x %d elements exceed the 2^31-vector limit", who,
+                              (long long)s->count, s->c);
     return DBL_OK;
 }
 
-// Backward reduce split: a fixed function of the shape, so the workspace
-// size does not depend on the device.
-int64_t bwd_blocks(int64_t count) { return count <= 0 ? 1 : (count + 255) / 256 < 512 ? (count + 255) / 256 : 512; }
+// Backward reduce split: a fixed function of the shape (so the workspace size
+// and the summation order do not depend on the device): one CTA per 2048
+// 8-channel vectors (8 per thread), at most 1024 CTAs.
+int64_t bwd_blocks(int64_t count, int C)
+{
+    if (count <= 0 || C <= 0) return 1;
+    const int64_t b = (count * (C / 8) + 2047) / 2048;
+    return b < 1 ? 1 : b > 1024 ? 1024 : b;
+}
 
 }  // namespace
 
@@ -335,7 +415,7 @@ int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum,
 size_t dbl_bn_workspace_bytes(const dbl_bn_shape* s)
 {
     if (!s || s->c <= 0) return 0;
-    return sizeof(float) * ((size_t)bwd_blocks(s->count) * 2 * s->c + 3 * (size_t)s->c);
+    return sizeof(float) * ((size_t)bwd_blocks(s->count, s->c) * 2 * s->c + 3 * (size_t)s->c);
 }
 
 int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
@@ -355,19 +435,21 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
     if (!ws || ws_bytes < need)
         return set_error(DBL_ERR_WORKSPACE, "bn_relu_fused_bwd: workspace %zu < %zu bytes", ws_bytes, need);
     const int C = s->c;
-    const int64_t nblk = bwd_blocks(s->count);
-    const int64_t rows = (s->count + nblk - 1) / nblk;
+    const int64_t nblk = bwd_blocks(s->count, s->c);
+    const int rows = (int)((s->count + nblk - 1) / nblk);
     float* partial = static_cast<float*>(ws);
     float* coef = partial + nblk * 2 * C;
     cudaStream_t st = as_stream(stream);
     auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
-    bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
-                                                         save_mean, save_invstd, rows, partial);
+    bn_bwd_reduce_kernel<<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C,
+                                                                 s->relu, save_mean, save_invstd, rows, (int)nblk,
+                                                                 partial);
     if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_mean,
+                                                            save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
-    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
+    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
         bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
         static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
     return launch_check("bn_bwd_apply launch");
@@ -432,22 +514,24 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
         return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: tensors must be 16-byte aligned");
     if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: empty batch");
     const int C = s->c;
-    const int64_t nblk = bwd_blocks(s->count);
+    const int64_t nblk = bwd_blocks(s->count, s->c);
     if (nblk > kNoallocMaxBlocks || (size_t)nblk * 2 * C + 3 * (size_t)C > kNoallocFloats)
         return set_error(DBL_ERR_UNSUPPORTED, "bn_relu_fused_bwd_noalloc: shape exceeds the static scratch");
     float* partial = noalloc_scratch(&rc);
     if (rc) return rc;
     float* coef = partial + nblk * 2 * C;  // written by the finalize kernel before the apply kernel reads it
-    const int64_t rows = (s->count + nblk - 1) / nblk;
+    const int rows = (int)((s->count + nblk - 1) / nblk);
     cudaStream_t st = as_stream(stream);
     auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
-    bn_bwd_reduce_kernel<<<(int)nblk, kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu,
-                                                         save_mean, save_invstd, rows, partial);
+    bn_bwd_reduce_kernel<<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C,
+                                                                 s->relu, save_mean, save_invstd, rows, (int)nblk,
+                                                                 partial);
     if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_invstd,
+    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_mean,
+                                                            save_invstd,
                                                             dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
-    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8), kThreads, 0, st>>>(
+    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
         bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
         static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
     return launch_check("bn_bwd_noalloc apply launch");
