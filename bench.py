@@ -70,14 +70,15 @@ def _conv_source_hash():
 
 
 def _traffic_record(config):
-    """DRAM bytes of the conv kernel per step from a committed ncu summary, if it is current."""
+    """DRAM bytes (read + write) of all conv-kernel launches of one iteration at the largest
+    stage, from a committed ncu summary, if it was taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "conv_igemm_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
         if rec.get("source_hash") != _conv_source_hash() or rec.get("config") != config:
             return None
-        return rec.get("dram_bytes_per_launch_avg")
+        return rec.get("dram_bytes_per_iteration")
     except Exception:
         return None
 
@@ -259,6 +260,8 @@ def conv_roofline(stage, reps=3, table=None):
     from paper_2509_26092_gb300 import dbl as D
     s = torch.cuda.current_stream()
     flops, secs = 0.0, 0.0
+    nbytes = lambda *ts: sum(t.numel() * t.element_size() for t in ts)
+    algo_bytes = 0  # unique operand bytes of every pass (inputs + weights + outputs)
     for wk in (stage["large"], stage["small"]):
         if wk is None:
             continue
@@ -270,9 +273,12 @@ def conv_roofline(stage, reps=3, table=None):
             st_sq = torch.empty(shp.k, device=x.device)
             f1 = float(wk.layer_flops(name, shp))
             passes = [("fwd", lambda: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            algo_bytes += nbytes(x, w16, y)
             if name != stem:
                 passes.append(("dgrad", lambda: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
+                algo_bytes += nbytes(dy, w16, dx)
             passes.append(("wgrad", lambda: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
+            algo_bytes += nbytes(x, dy, g)
             for pname, fn in passes:
                 fn()
                 ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
@@ -286,7 +292,7 @@ def conv_roofline(stage, reps=3, table=None):
                 flops += f1
                 if table is not None:
                     table.append((wk.batch, name, pname, f1, t1))
-    return flops, secs
+    return flops, secs, algo_bytes
 
 
 def _conv_buffers(wk):
@@ -327,6 +333,8 @@ def run_profile_iteration(args, cfg):
     nat = cfg["native"]
     n0 = D.dbl_kernel_launches()
     for res, bl, bs in zip(cfg["stages"], cfg["large"], cfg["small"]):
+        if args.profile_res and res != args.profile_res:
+            continue
         large = R.Worker(spec, bl, res)
         small = R.Worker(spec, bs, res) if bs else None
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_small=F_SMALL)
@@ -493,7 +501,7 @@ def run_ours(args, cfg):
         if wk is not None:
             wk._bench_w16 = pipe["server"].w16
     table = [] if args.conv_table else None
-    flops, secs = conv_roofline(top, table=table)
+    flops, secs, algo_bytes = conv_roofline(top, table=table)
     if table is not None:
         for b, name, pname, f1, t1 in table:
             print(f"conv {b:4d} {name:16s} {pname:5s} {t1 * 1e6:9.1f} us {f1 / t1 / 1e12:7.1f} TFLOP/s",
@@ -501,6 +509,10 @@ def run_ours(args, cfg):
     achieved = flops / secs / 1e12
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16, "unit": "TFLOP/s",
                 "frac": round(achieved / bf16, 4), "traffic": _traffic_record(args.config),
+                "algorithmic_bytes": int(algo_bytes),
+                "scope": f"one dual-batch iteration at {top['res']} px: every conv pass of both workers "
+                         "(achieved = algorithmic FLOPs / summed CUDA-event time of the passes; traffic = ncu "
+                         "DRAM bytes of the same launches, null if the kernel changed since the capture)",
                 "kernel": "conv_igemm_kernel (fwd/dgrad/wgrad, every layer of both workers at "
                           f"{top['res']} px, each ABI call timed alone)", "peak_source": src}
     cpu = None
@@ -544,6 +556,8 @@ def main():
     ap.add_argument("--profile-conv", default=None, metavar="LAYER:PASS",
                     help="run one conv pass of one layer three times (e.g. layer1.0.conv1:fwd) for ncu")
     ap.add_argument("--profile-batch", type=int, default=512)
+    ap.add_argument("--profile-res", type=int, default=0,
+                    help="with --profile-iteration: run only the stage at this resolution")
     ap.add_argument("--profile-iteration", action="store_true",
                     help="run one eager iteration per stage and exit (the command ncu profiles)")
     args = ap.parse_args()
