@@ -169,7 +169,7 @@ DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf
  * method.
  *
  * The scratch lives in one statically sized device array inside libdbl.so
- * (4.2 MB, held on every device that loads the library until the process
+ * (2.1 MB, held on every device that loads the library until the process
  * exits).  Limit: c <= DBL_BN_NOALLOC_MAX_C (512); larger c returns
  * DBL_ERR_UNSUPPORTED before anything is launched.  The first call on a
  * device looks up the array's device address (cudaGetSymbolAddress) with that

@@ -15,6 +15,9 @@
 
 namespace {
 
+using dbl::dev::colsum_fixed_order;
+using dbl::dev::kColsumGroups;
+
 constexpr int kThreads = 256;
 constexpr int kMaxC = 2048;
 constexpr int kUnroll = 2;  // rows per thread whose loads are in flight together
@@ -259,31 +262,20 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     }
 }
 
-// Fixed-order sum of the partials: one warp per channel, lane l sums blocks
-// l, l+32, ... in double, then a fixed butterfly across the warp; then dgamma,
-// dbeta and the three per-channel coefficients (A, B, C) of the apply pass
-// dy = A*g + B*y + C.
-__global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(const float* __restrict__ partial, int nblk, int C,
-                                                              int64_t count, const float* __restrict__ gamma,
-                                                              const float* __restrict__ mean,
-                                                              const float* __restrict__ invstd,
-                                                              float* __restrict__ dgamma, float* __restrict__ dbeta,
-                                                              float* __restrict__ coef)
+// Fixed-order sum of the partials [nblk][2][C] (colsum_fixed_order; block b
+// covers channels 32b .. 32b+31), then dgamma, dbeta and the three per-channel
+// coefficients (A, B, C) of the apply pass dy = A*g + B*y + C.
+__global__ void __launch_bounds__(32 * kColsumGroups) bn_bwd_finalize_kernel(
+    const float* __restrict__ partial, int nblk, int C, int64_t count, const float* __restrict__ gamma,
+    const float* __restrict__ mean, const float* __restrict__ invstd, float* __restrict__ dgamma,
+    float* __restrict__ dbeta, float* __restrict__ coef)
 {
-    const int c = blockIdx.x * 8 + threadIdx.x / 32;
-    const int lane = threadIdx.x % 32;
-    if (c >= C) return;
-    double sg = 0.0, sgx = 0.0;
-    for (int b = lane; b < nblk; b += 32) {
-        sg += partial[(int64_t)b * 2 * C + c];
-        sgx += partial[(int64_t)b * 2 * C + C + c];
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-        sg += __shfl_xor_sync(0xffffffffu, sg, o);
-        sgx += __shfl_xor_sync(0xffffffffu, sgx, o);
-    }
-    if (lane != 0) return;
+    __shared__ double red[kColsumGroups * 32];
+    const int c0 = blockIdx.x * 32;
+    const double sg = colsum_fixed_order(partial, nblk, 2 * (int64_t)C, c0, C, red);
+    const double sgx = colsum_fixed_order(partial + C, nblk, 2 * (int64_t)C, c0, C, red);
+    const int c = c0 + threadIdx.x;
+    if (threadIdx.x >= 32 || c >= C) return;
     dbeta[c] = (float)sg;
     dgamma[c] = (float)sgx;
     // dy = k1*(g - sum(g)/n - xhat*sum(g*xhat)/n), xhat = (y - mean)*invstd, as A*g + B*y + C
@@ -365,13 +357,13 @@ int check_shape(const dbl_bn_shape* s, const char* who)
 }
 
 // Backward reduce split: a fixed function of the shape (so the workspace size
-// and the summation order do not depend on the device): one CTA per 2048
-// 8-channel vectors (8 per thread), at most 1024 CTAs.
+// and the summation order do not depend on the device): one partial per 2048
+// 8-channel vectors (8 per thread), at most 512 partials.
 int64_t bwd_blocks(int64_t count, int C)
 {
     if (count <= 0 || C <= 0) return 1;
     const int64_t b = (count * (C / 8) + 2047) / 2048;
-    return b < 1 ? 1 : b > 1024 ? 1024 : b;
+    return b < 1 ? 1 : b > 512 ? 512 : b;
 }
 
 }  // namespace
@@ -445,9 +437,8 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
                                                                  s->relu, save_mean, save_invstd, rows, (int)nblk,
                                                                  partial);
     if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_mean,
-                                                            save_invstd,
-                                                            dgamma, dbeta, coef);
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma,
+                                                                         save_mean, save_invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
         bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
@@ -463,7 +454,7 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
 // one file-scope device array sized for the largest channel count accepted.
 namespace {
 
-constexpr int kNoallocMaxBlocks = 1024;  // bwd_blocks() never exceeds this
+constexpr int kNoallocMaxBlocks = 512;  // bwd_blocks() never exceeds this
 constexpr size_t kNoallocFloats =
     (size_t)kNoallocMaxBlocks * 2 * DBL_BN_NOALLOC_MAX_C + 3 * (size_t)DBL_BN_NOALLOC_MAX_C;
 
@@ -527,9 +518,8 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
                                                                  s->relu, save_mean, save_invstd, rows, (int)nblk,
                                                                  partial);
     if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 7) / 8, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, save_mean,
-                                                            save_invstd,
-                                                            dgamma, dbeta, coef);
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma,
+                                                                         save_mean, save_invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
     bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
         bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,

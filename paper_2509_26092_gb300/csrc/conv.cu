@@ -34,7 +34,6 @@ namespace {
 using namespace dbl::dev;
 
 constexpr int BM = 128;        // tile rows = TMEM lanes
-constexpr int BK = 64;         // reduction elements per stage (128 bytes of bf16)
 constexpr int kTargetCTAs = 304;  // 2 x 152 SMs: split-K sizing target (device independent)
 
 enum Mode : int { kFwd = 0, kDgrad = 1, kWgrad = 2, kFwdC8 = 3, kWgradC8 = 4 };
@@ -70,6 +69,11 @@ struct ConvParams {
     int64_t ldo;        // elements between output rows (fwd, dgrad)
     int wg_accumulate;  // wgrad with one slice: add into dw
     float* stats;       // fwd: [gridDim.x][2][Ncols] per-CTA channel sums, or nullptr
+    // window kernel (3x3, stride 1, pad 1): the batch as one column of zero-padded images
+    int win_H, win_W;         // image height and width (= output height and width)
+    int win_Hp, win_Wp;       // padded height and width (H + 2, W + 2)
+    int win_srows;            // padded rows loaded per strip
+    int win_strip_bytes;      // bytes of one strip buffer (a multiple of 1024)
 };
 
 __device__ __forceinline__ void report_timeout(volatile int* abort)
@@ -199,6 +203,107 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
     }
 }
 
+// Epilogue of the bf16-output passes for one 32-column chunk of this thread's
+// accumulator row: round to bf16 and store the row chunk (if the row is a real
+// output); back[] receives the stored values (zeros for rows that are not outputs).
+__device__ __forceinline__ void store_row_chunk_bf16(const ConvParams& p, const uint32_t (&v)[32], bool valid,
+                                                     int64_t out_row, int col0, float (&back)[32])
+{
+    uint4 pk[4];
+    __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
+        const float2 f = __bfloat1622float2(h2[k]);
+        back[2 * k] = valid ? f.x : 0.f;
+        back[2 * k + 1] = valid ? f.y : 0.f;
+    }
+    if (valid) {
+        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) o[k] = pk[k];
+    }
+}
+
+// BatchNorm channel sums (sum y, sum y^2) of the stored forward outputs, kept
+// in registers across the tiles of a CTA instead of being reduced across the
+// warp for every tile (which costs shared-memory bandwidth that the mainloop
+// needs).  Thread (warp, lane) adds the values of its own accumulator row.
+// For BN > 64 the rows are first folded pairwise across lanes (LEVELS
+// shuffle steps), so that every thread holds 128 sums: after the folding,
+// value k of chunk ch belongs to column ch*32 + (lane & (32 - V)) + k.
+// flush() reduces over the lanes through the warp's 32x33 scratch and adds the
+// column totals to the warp's channel sums (once per CTA, and whenever the
+// CTA moves to another column tile).
+template <int BN>
+struct RowStats {
+    static constexpr int NCH = BN / 32;
+    static constexpr int LEVELS = BN <= 64 ? 0 : (BN <= 128 ? 1 : 2);
+    static constexpr int V = 32 >> LEVELS;
+    float s[NCH][V], q[NCH][V];
+
+    __device__ __forceinline__ void zero()
+    {
+#pragma unroll
+        for (int c = 0; c < NCH; ++c)
+#pragma unroll
+            for (int k = 0; k < V; ++k) s[c][k] = q[c][k] = 0.f;
+    }
+
+    template <int N, int O>
+    __device__ __forceinline__ static void fold(float (&a)[32], float (&b)[32], int lane)
+    {
+        const bool up = (lane & O) != 0;
+#pragma unroll
+        for (int k = 0; k < N / 2; ++k) {
+            const float sa = up ? a[k] : a[k + N / 2], ka = up ? a[k + N / 2] : a[k];
+            const float sb = up ? b[k] : b[k + N / 2], kb = up ? b[k + N / 2] : b[k];
+            a[k] = ka + __shfl_xor_sync(0xffffffffu, sa, O);
+            b[k] = kb + __shfl_xor_sync(0xffffffffu, sb, O);
+        }
+    }
+
+    // x: the stored values of chunk ch of this thread's row (call with ch a compile-time
+    // constant after unrolling).  Every lane of the warp must call it.
+    __device__ __forceinline__ void add(int ch, const float (&x)[32], int lane)
+    {
+        float a[32], b[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+            a[k] = x[k];
+            b[k] = x[k] * x[k];
+        }
+        if constexpr (LEVELS >= 1) fold<32, 16>(a, b, lane);
+        if constexpr (LEVELS >= 2) fold<16, 8>(a, b, lane);
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+            s[ch][k] += a[k];
+            q[ch][k] += b[k];
+        }
+    }
+
+    // wsum: this warp's [2][Ncols] channel sums; col_base: first column of the tile.
+    __device__ __forceinline__ void flush(float* st_tile, float* wsum, int ncols, int col_base, int lane)
+    {
+        const int hb = lane & (32 - V), kk = lane & (V - 1);
+#pragma unroll
+        for (int c = 0; c < NCH; ++c) {
+#pragma unroll
+            for (int w = 0; w < 2; ++w) {
+#pragma unroll
+                for (int k = 0; k < V; ++k) st_tile[lane * 33 + k] = w ? q[c][k] : s[c][k];
+                __syncwarp();
+                float tot = 0.f;
+#pragma unroll
+                for (int u = 0; u < V; ++u) tot += st_tile[(hb + u) * 33 + kk];
+                __syncwarp();
+                wsum[w * ncols + col_base + c * 32 + lane] += tot;
+            }
+        }
+        zero();
+    }
+};
+
 // Persistent kernel: CTA b processes tiles b, b + gridDim.x, ...  The ring of
 // STAGES shared-memory stages (two K-blocks each) runs continuously across
 // tiles; two producer warps fill alternate stages; two TMEM accumulators let
@@ -234,7 +339,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         abort_flag = 0;
         fence_mbar_init();
     }
-    const bool want_stats = (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
+    const bool want_stats = FAM == kFamFwd && (p.mode == kFwd || p.mode == kFwdC8) && p.stats != nullptr;
     if (want_stats)
         for (int i = threadIdx.x; i < 4 * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
     if (warp >= 4 && warp < 4 + kProducers && lane == 0) {
@@ -360,6 +465,9 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         // ------------------------------------------------------------------ epilogue (warps 0-3)
         float* st_tile = epi_tile + warp * 32 * 33;
         float* wsum = epi_sum + warp * 2 * p.Ncols;
+        RowStats<BN> rs;
+        rs.zero();
+        int stats_ntile = -1;  // column tile the register sums belong to
         int lt = 0;
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
             const TileCoord tc = decode_tile(p, t);
@@ -374,80 +482,69 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
             tc_fence_after();
             const int row = warp * 32 + lane;  // TMEM lane = row within a 128-row accumulator
             const bool have_acc = nkb > 0;
+            if (want_stats && stats_ntile != tc.n_tile) {
+                if (stats_ntile >= 0) rs.flush(st_tile, wsum, p.Ncols, stats_ntile * BN, lane);
+                stats_ntile = tc.n_tile;
+            }
 #pragma unroll 1
             for (int a = 0; a < C::ACC; ++a) {
-            const int64_t m = (int64_t)tc.m_tile * C::BMT + a * 128 + row;
-            const bool valid = m < p.M;
-            int64_t out_row = m;
-            if (p.mode == kDgrad && p.phase_div == 2) {
-                const int64_t n = m / gPQ, rem = m - n * gPQ;
-                const int i = (int)(rem / p.gQ), j = (int)(rem - (int64_t)(rem / p.gQ) * p.gQ);
-                const int pa = tc.z >> 1, pb = tc.z & 1;
-                out_row = (n * p.out_h + 2 * i + pa) * p.out_w + 2 * j + pb;
-            }
-            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * C::ACC + a) * BN);
+                const int64_t m = (int64_t)tc.m_tile * C::BMT + a * 128 + row;
+                const bool valid = m < p.M;
+                const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * C::ACC + a) * BN);
+                if constexpr (FAM == kFamWgrad) {
 #pragma unroll 1
-            for (int ch = 0; ch < BN / 32; ++ch) {
-                uint32_t v[32];
-                if (have_acc) {
-                    tmem_ld_32x32b_x32(taddr + ch * 32, v);
-                    tmem_ld_wait();
-                } else {
-#pragma unroll
-                    for (int k = 0; k < 32; ++k) v[k] = 0u;
-                }
-                const int col0 = tc.n_tile * BN + ch * 32;
-                if (p.mode == kWgrad || p.mode == kWgradC8) {
-                    // D row m = (tap, c), column = output channel k; stored as [slice][k][m]:
-                    // consecutive lanes hold consecutive m, so each store is one 128-byte line
-                    if (valid) {
-                        float* o = static_cast<float*>(p.out) + ((int64_t)tc.z * p.Ncols + col0) * p.M + m;
-                        if (p.zdim == 1 && p.wg_accumulate) {
-#pragma unroll
-                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] += __uint_as_float(v[k]);
+                    for (int ch = 0; ch < BN / 32; ++ch) {
+                        uint32_t v[32];
+                        if (have_acc) {
+                            tmem_ld_32x32b_x32(taddr + ch * 32, v);
+                            tmem_ld_wait();
                         } else {
 #pragma unroll
-                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] = __uint_as_float(v[k]);
+                            for (int k = 0; k < 32; ++k) v[k] = 0u;
+                        }
+                        const int col0 = tc.n_tile * BN + ch * 32;
+                        // D row m = (tap, c), column = output channel k; stored as [slice][k][m]:
+                        // consecutive lanes hold consecutive m, so each store is one 128-byte line
+                        if (valid) {
+                            float* o = static_cast<float*>(p.out) + ((int64_t)tc.z * p.Ncols + col0) * p.M + m;
+                            if (p.zdim == 1 && p.wg_accumulate) {
+#pragma unroll
+                                for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] += __uint_as_float(v[k]);
+                            } else {
+#pragma unroll
+                                for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] = __uint_as_float(v[k]);
+                            }
                         }
                     }
                 } else {
-                    uint4 pk[4];
-                    __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
-#pragma unroll
-                    for (int k = 0; k < 16; ++k)
-                        h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
-                    if (valid) {
-                        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
-#pragma unroll
-                        for (int k = 0; k < 4; ++k) o[k] = pk[k];
+                    int64_t out_row = m;
+                    if (p.mode == kDgrad && p.phase_div == 2) {
+                        const int64_t n = m / gPQ, rem = m - n * gPQ;
+                        const int i = (int)(rem / p.gQ), j = (int)(rem - (int64_t)(rem / p.gQ) * p.gQ);
+                        const int pa = tc.z >> 1, pb = tc.z & 1;
+                        out_row = (n * p.out_h + 2 * i + pa) * p.out_w + 2 * j + pb;
                     }
-                    if (want_stats) {
-                        // column sums of the stored (rounded) values over this warp's 32 rows
 #pragma unroll
-                        for (int k = 0; k < 16; ++k) {
-                            const float2 back = __bfloat1622float2(h2[k]);
-                            st_tile[lane * 33 + 2 * k] = valid ? back.x : 0.f;
-                            st_tile[lane * 33 + 2 * k + 1] = valid ? back.y : 0.f;
+                    for (int ch = 0; ch < BN / 32; ++ch) {
+                        uint32_t v[32];
+                        if (have_acc) {
+                            tmem_ld_32x32b_x32(taddr + ch * 32, v);
+                            tmem_ld_wait();
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < 32; ++k) v[k] = 0u;
                         }
-                        __syncwarp();
-                        float s = 0.f, q = 0.f;
-#pragma unroll 8
-                        for (int r = 0; r < 32; ++r) {
-                            const float x = st_tile[r * 33 + lane];
-                            s += x;
-                            q = fmaf(x, x, q);
-                        }
-                        wsum[col0 + lane] += s;
-                        wsum[p.Ncols + col0 + lane] += q;
-                        __syncwarp();
+                        float back[32];
+                        store_row_chunk_bf16(p, v, valid, out_row, tc.n_tile * BN + ch * 32, back);
+                        if (want_stats) rs.add(ch, back, lane);
                     }
                 }
-            }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acce_bar[buf]);
         }
+        if (want_stats && stats_ntile >= 0) rs.flush(st_tile, wsum, p.Ncols, stats_ntile * BN, lane);
         if (want_stats) {
             asm volatile("bar.sync 1, 128;" ::: "memory");
             float* dst = p.stats + (int64_t)blockIdx.x * 2 * p.Ncols;
@@ -463,55 +560,372 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
     }
 }
 
-// ----------------------------------------------------------------------------- reductions
-// Per-channel sums over the per-CTA partials, fixed order: 8 lanes per channel, then 8 -> 1.
-__global__ void stats_reduce_kernel(const float* __restrict__ part, int nparts, int K, float* __restrict__ sum,
-                                    float* __restrict__ sumsq)
+// ----------------------------------------------------------------------------- window kernel
+// 3x3, stride-1, pad-1 correlation (the forward pass, and the data gradient
+// with the taps flipped) without im2col.  Position (h, w) of image n of the
+// zero-padded input is row g = n*Hp + h of a column of padded rows, and
+// padded position L = g*Wp + w.  Output (h, w) of image n is computed at
+// L = (n*Hp + h)*Wp + w, and its tap (r, s) reads padded position L + r*Wp + s.
+// So a tile of 256 consecutive L needs one strip of padded rows (TMA loads
+// one padded row per copy: the box starts at w = -1 and the zero fill makes
+// the padding), and each of the nine taps is the same strip addressed by a
+// descriptor that starts r*Wp + s rows later.  The 128-byte swizzle of both
+// TMA and the MMA operand fetch is a function of the absolute shared-memory
+// address, so a start at any 128-byte row reads the rows that TMA wrote.  Rows
+// with h >= H or w >= W are computed and not stored (the padding's share of
+// the work: 7% at 56x56, 13% at 28x28).
+// Warp roles: warp 4 loads strips (two buffers), warp 5 loads weights (all
+// nine taps once per CTA when they fit, RES; else a ring of per-tap tiles),
+// warp 6 issues the MMAs, warps 0-3 drain TMEM as in conv_igemm_kernel.
+constexpr int kWinACC = 2;               // 128-row accumulators per tile
+constexpr int kWinBMT = 128 * kWinACC;   // padded positions per tile
+constexpr int kWinBStages = 4;           // weight-tile ring depth when not resident
+constexpr int kWinThreads = 224;
+constexpr int kEpiTileBytes = 4 * 32 * 33 * 4;
+
+template <int BN>
+struct WinCfg {
+    static constexpr int B_TILE = BN * 64 * 2;  // one tap x one 64-channel block of weights
+    static constexpr uint32_t TMEM_COLS = 2 * kWinACC * BN;
+};
+
+// One tap x 64-channel block of weights: K-major [BN out][64 in] for the forward
+// pass, MN-major [64 k][BN c] blocks of 64 for the data gradient (flipped tap).
+template <int BN, bool DG>
+__device__ __forceinline__ void win_load_wtile(const ConvParams& p, const CUtensorMap* tmB, uint8_t* dst, uint64_t* bar,
+                                               int tap, int cb, int n_tile)
 {
-    __shared__ double red[8][2][33];
-    const int c = blockIdx.x * 32 + threadIdx.x % 32;
-    const int l8 = threadIdx.x / 32;
-    double s = 0.0, q = 0.0;
-    if (c < K)
-        for (int t = l8; t < nparts; t += 8) {
-            s += part[(int64_t)t * 2 * K + c];
-            q += part[(int64_t)t * 2 * K + K + c];
-        }
-    red[l8][0][threadIdx.x % 32] = s;
-    red[l8][1][threadIdx.x % 32] = q;
-    __syncthreads();
-    if (threadIdx.x < 32 && c < K) {
-        double ts = 0.0, tq = 0.0;
-        for (int l = 0; l < 8; ++l) {
-            ts += red[l][0][threadIdx.x];
-            tq += red[l][1][threadIdx.x];
-        }
-        sum[c] = (float)ts;
-        sumsq[c] = (float)tq;
+    if constexpr (DG) {
+        const int wtap = 8 - tap;
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j) tma_load_3d_elect(dst + j * 8192, tmB, bar, n_tile * BN + 64 * j, wtap, cb * 64);
+    } else {
+        tma_load_2d_elect(dst, tmB, bar, tap * p.Cin + cb * 64, n_tile * BN);
     }
 }
 
-// dw[i] (+)= sum over slices of part[slice][i], slices in a fixed order; i runs over the
-// KRSC weight gradient (the slices are already in that layout).
+template <int BN, bool DG, bool RES>
+__global__ void __launch_bounds__(kWinThreads, 1)
+    conv_win_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const ConvParams p)
+{
+    using C = WinCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t sfull[2], sempty[2], bfull[kWinBStages], bempty[kWinBStages], accf_bar[2],
+        acce_bar[2], drain_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
+    const int CB = p.cblocks;
+    const int b_bytes = RES ? 9 * CB * C::B_TILE : kWinBStages * C::B_TILE;
+    uint8_t* strip = sgen + b_bytes;
+    float* epi_tile = reinterpret_cast<float*>(strip + 2 * p.win_strip_bytes);
+    float* epi_sum = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(epi_tile) + kEpiTileBytes);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&sfull[i], 1);
+            mbar_init(&sempty[i], 1);
+            mbar_init(&accf_bar[i], 1);
+            mbar_init(&acce_bar[i], 4);  // one arrival per epilogue warp
+        }
+        for (int i = 0; i < kWinBStages; ++i) {
+            mbar_init(&bfull[i], 1);
+            mbar_init(&bempty[i], 1);
+        }
+        mbar_init(&drain_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    const bool want_stats = p.mode == kFwd && p.stats != nullptr;
+    if (want_stats)
+        for (int i = threadIdx.x; i < 4 * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
+    if ((warp == 4 || warp == 5) && lane == 0) {
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 6) {
+        tmem_alloc(&tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    const int Wp = p.win_Wp;
+
+    if (warp == 4) {
+        // ------------------------------------------------------------------ strip producer
+        int it = 0;
+        bool failed = false;
+        const uint32_t strip_tx = (uint32_t)(p.win_srows * Wp * 128);
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+            const TileCoord tc = decode_tile(p, t);
+            const int g0 = tc.m_tile * kWinBMT / Wp;
+            for (int cb = 0; cb < CB; ++cb, ++it) {
+                const int s = it & 1;
+                const uint32_t ok = mbar_wait_warp(&sempty[s], ((it >> 1) & 1) ^ 1, &abort_flag);
+                if (__any_sync(0xffffffffu, ok == 0u)) {
+                    failed = true;
+                    break;
+                }
+                uint8_t* dst = strip + s * p.win_strip_bytes;
+                mbar_arrive_expect_tx_elect(&sfull[s], strip_tx);
+                for (int r = 0; r < p.win_srows; ++r) {
+                    const int g = g0 + r;
+                    const int n = g / p.win_Hp, hp = g - n * p.win_Hp;
+                    // padded row hp of image n = input row hp - 1 (rows -1 and H, and images past
+                    // the batch, are outside the tensor and arrive as zeros)
+                    tma_load_4d_elect(dst + r * Wp * 128, &tmA, &sfull[s], cb * 64, -1, hp - 1, n);
+                }
+            }
+            if (failed) break;
+        }
+        if (failed) {
+            if (lane == 0) report_timeout(&abort_flag);
+            for (int i = it - 1; i >= 0 && i >= it - 2; --i) (void)mbar_drain_warp(&sfull[i & 1], (i >> 1) & 1);
+        }
+    } else if (warp == 5) {
+        // ------------------------------------------------------------------ weight producer
+        if (RES) {
+            mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(9 * CB * C::B_TILE));
+            for (int tap = 0; tap < 9; ++tap)
+                for (int cb = 0; cb < CB; ++cb)
+                    win_load_wtile<BN, DG>(p, &tmB, sgen + (tap * CB + cb) * C::B_TILE, &bfull[0], tap, cb, 0);
+            (void)mbar_drain_warp(&bfull[0], 0);
+        } else {
+            int bt = 0;
+            bool failed = false;
+            for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
+                const TileCoord tc = decode_tile(p, t);
+                for (int cb = 0; cb < CB && !failed; ++cb)
+                    for (int tap = 0; tap < 9; ++tap, ++bt) {
+                        const int s = bt % kWinBStages;
+                        const uint32_t ok =
+                            mbar_wait_warp(&bempty[s], ((bt / kWinBStages) & 1) ^ 1, &abort_flag);
+                        if (__any_sync(0xffffffffu, ok == 0u)) {
+                            failed = true;
+                            break;
+                        }
+                        mbar_arrive_expect_tx_elect(&bfull[s], (uint32_t)C::B_TILE);
+                        win_load_wtile<BN, DG>(p, &tmB, sgen + s * C::B_TILE, &bfull[s], tap, cb, tc.n_tile);
+                    }
+            }
+            if (failed) {
+                if (lane == 0) report_timeout(&abort_flag);
+                for (int i = bt - 1; i >= 0 && i >= bt - kWinBStages; --i)
+                    (void)mbar_drain_warp(&bfull[i % kWinBStages], (i / kWinBStages) & 1);
+            }
+        }
+    } else if (warp == 6) {
+        // ------------------------------------------------------------------ MMA issuer
+        const uint32_t idesc = idesc_bf16(BM, BN, 0u, DG ? 1u : 0u);
+        int it = 0, bt = 0, lt = 0;
+        bool failed = false;
+        if (RES) {
+            const uint32_t ok = mbar_wait_warp(&bfull[0], 0, &abort_flag);
+            failed = __any_sync(0xffffffffu, ok == 0u);
+        }
+        for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
+            const TileCoord tc = decode_tile(p, t);
+            const int buf = lt & 1;
+            const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                failed = true;
+                break;
+            }
+            tc_fence_after();
+            const int L0 = tc.m_tile * kWinBMT;
+            const int off0 = L0 - (L0 / Wp) * Wp;  // tile start within the strip's first row
+            const uint32_t d = tmem + (uint32_t)(buf * kWinACC * BN);
+            for (int cb = 0; cb < CB && !failed; ++cb, ++it) {
+                const int s = it & 1;
+                const uint32_t oks = mbar_wait_warp(&sfull[s], (it >> 1) & 1, &abort_flag);
+                if (__any_sync(0xffffffffu, oks == 0u)) {
+                    failed = true;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = sbase + (uint32_t)(b_bytes + s * p.win_strip_bytes);
+#pragma unroll 1
+                for (int tap = 0; tap < 9; ++tap) {
+                    const int r = tap / 3, sx = tap - 3 * r;
+                    uint32_t sb;
+                    int bs = 0;
+                    if (RES) {
+                        sb = sbase + (uint32_t)((tap * CB + cb) * C::B_TILE);
+                    } else {
+                        bs = bt % kWinBStages;
+                        const uint32_t okb = mbar_wait_warp(&bfull[bs], (bt / kWinBStages) & 1, &abort_flag);
+                        if (__any_sync(0xffffffffu, okb == 0u)) {
+                            failed = true;
+                            break;
+                        }
+                        tc_fence_after();
+                        sb = sbase + (uint32_t)(bs * C::B_TILE);
+                    }
+                    const uint32_t a0 = sa + (uint32_t)((off0 + r * Wp + sx) * 128);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+#pragma unroll
+                        for (int a = 0; a < kWinACC; ++a) {
+                            const uint64_t ad = smem_desc(a0 + a * 128 * 128 + 32 * j, 16, 1024, kSwizzle128B);
+                            const uint64_t bd = DG ? smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B)
+                                                   : smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
+                            mma_bf16_elect(d + a * BN, ad, bd, idesc, (cb > 0 || tap > 0 || j > 0) ? 1u : 0u);
+                        }
+                    }
+                    if (!RES) {
+                        mma_commit_elect(&bempty[bs]);
+                        ++bt;
+                    }
+                }
+                mma_commit_elect(&sempty[s]);
+            }
+            mma_commit_elect(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
+        }
+        if (failed && lane == 0) report_timeout(&abort_flag);
+        mma_commit_elect(&drain_bar);
+        (void)mbar_drain_warp(&drain_bar, 0);
+    } else {
+        // ------------------------------------------------------------------ epilogue (warps 0-3)
+        float* st_tile = epi_tile + warp * 32 * 33;
+        float* wsum = epi_sum + warp * 2 * p.Ncols;
+        RowStats<BN> rs;
+        rs.zero();
+        const int img = p.win_Hp * Wp;
+        int lt = 0;
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
+            const TileCoord tc = decode_tile(p, t);
+            const int buf = lt & 1;
+            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                if (lane == 0) report_timeout(&abort_flag);
+                break;
+            }
+            tc_fence_after();
+            const int row = warp * 32 + lane;
+#pragma unroll 1
+            for (int a = 0; a < kWinACC; ++a) {
+                const int L = tc.m_tile * kWinBMT + a * 128 + row;
+                const int n = L / img, rem = L - n * img;
+                const int hp = rem / Wp, wp = rem - hp * Wp;
+                const bool valid = n < p.gN && hp < p.win_H && wp < p.win_W;
+                const int64_t out_row = ((int64_t)n * p.win_H + hp) * p.win_W + wp;
+                const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * kWinACC + a) * BN);
+#pragma unroll
+                for (int ch = 0; ch < BN / 32; ++ch) {
+                    uint32_t v[32];
+                    tmem_ld_32x32b_x32(taddr + ch * 32, v);
+                    tmem_ld_wait();
+                    float back[32];
+                    store_row_chunk_bf16(p, v, valid, out_row, tc.n_tile * BN + ch * 32, back);
+                    if (want_stats) rs.add(ch, back, lane);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce_bar[buf]);
+        }
+        if (want_stats) {
+            rs.flush(st_tile, wsum, p.Ncols, 0, lane);  // the window kernel has one column tile
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            float* dst = p.stats + (int64_t)blockIdx.x * 2 * p.Ncols;
+            for (int c = threadIdx.x; c < 2 * p.Ncols; c += 128)
+                dst[c] = (epi_sum[c] + epi_sum[2 * p.Ncols + c]) + (epi_sum[4 * p.Ncols + c] + epi_sum[6 * p.Ncols + c]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 6) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+// ----------------------------------------------------------------------------- reductions
+// Per-channel sums over the per-CTA partials [nparts][2][K], fixed order
+// (colsum_fixed_order); block b covers channels 32b .. 32b+31 of both halves.
+__global__ void __launch_bounds__(32 * kColsumGroups) stats_reduce_kernel(const float* __restrict__ part, int nparts,
+                                                                         int K, float* __restrict__ sum,
+                                                                         float* __restrict__ sumsq)
+{
+    __shared__ double red[kColsumGroups * 32];
+    const int c0 = blockIdx.x * 32;
+    const double s = colsum_fixed_order(part, nparts, 2 * (int64_t)K, c0, K, red);
+    const double q = colsum_fixed_order(part + K, nparts, 2 * (int64_t)K, c0, K, red);
+    const int c = c0 + threadIdx.x;
+    if (threadIdx.x < 32 && c < K) {
+        sum[c] = (float)s;
+        sumsq[c] = (float)q;
+    }
+}
+
+// dw[i] (+)= sum over slices of part[slice][i] in a fixed order; i runs over
+// the KRSC weight gradient (the slices are already in that layout).  LANES
+// threads share one float4 of dw: thread j sums slices j, j+LANES, ... (four
+// loads in flight), then a fixed shuffle tree adds the LANES partial sums.
+// LANES = 1 for a few slices, 8 for many (the 64-channel layers split K ~60 ways).
+template <int LANES>
 __global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restrict__ part, int slices, int64_t n,
                                                            float* __restrict__ dw, int accumulate)
 {
+    const int j = threadIdx.x % LANES;
     const int64_t n4 = n >> 2;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
-        float4 acc = accumulate ? reinterpret_cast<const float4*>(dw)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s = 0; s < slices; ++s) {
+    const int64_t groups = blockDim.x / LANES;
+    // the loop bound is the same for the whole block, so every shuffle sees all 32 lanes
+    for (int64_t base = (int64_t)blockIdx.x * groups; base < n4; base += (int64_t)gridDim.x * groups) {
+        const int64_t i = base + threadIdx.x / LANES;
+        const int sl = i < n4 ? slices : 0;  // groups past the end add nothing and store nothing
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        int s = j;
+        for (; s + 3 * LANES < sl; s += 4 * LANES) {
+            float4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                v[u] = __ldcs(reinterpret_cast<const float4*>(part + (int64_t)(s + u * LANES) * n) + i);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                acc.x += v[u].x;
+                acc.y += v[u].y;
+                acc.z += v[u].z;
+                acc.w += v[u].w;
+            }
+        }
+        for (; s < sl; s += LANES) {
             const float4 v = __ldcs(reinterpret_cast<const float4*>(part + (int64_t)s * n) + i);
             acc.x += v.x;
             acc.y += v.y;
             acc.z += v.z;
             acc.w += v.w;
         }
-        reinterpret_cast<float4*>(dw)[i] = acc;
+#pragma unroll
+        for (int o = LANES / 2; o; o >>= 1) {
+            acc.x += __shfl_xor_sync(0xffffffffu, acc.x, o, LANES);
+            acc.y += __shfl_xor_sync(0xffffffffu, acc.y, o, LANES);
+            acc.z += __shfl_xor_sync(0xffffffffu, acc.z, o, LANES);
+            acc.w += __shfl_xor_sync(0xffffffffu, acc.w, o, LANES);
+        }
+        if (j == 0 && i < n4) {
+            float4* d = reinterpret_cast<float4*>(dw) + i;
+            if (accumulate) {
+                const float4 o = *d;
+                acc.x += o.x;
+                acc.y += o.y;
+                acc.z += o.z;
+                acc.w += o.w;
+            }
+            *d = acc;
+        }
     }
-    for (int64_t i = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        float acc = accumulate ? dw[i] : 0.f;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (int64_t i = (n4 << 2) + t; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        float acc = 0.f;
         for (int s = 0; s < slices; ++s) acc += part[(int64_t)s * n + i];
-        dw[i] = acc;
+        dw[i] = accumulate ? dw[i] + acc : acc;
     }
 }
 
@@ -521,7 +935,12 @@ struct Plan {
     int BN;
     ConvParams p;
     size_t ws_main = 0;  // bytes: fwd channel-sum partials, or wgrad split-K slices
+    bool win = false;    // conv_win_kernel (3x3 stride-1 correlation over padded strips)
+    bool res = false;    // window kernel with all weights resident in shared memory
+    size_t smem = 0;     // window kernel dynamic shared memory
 };
+
+
 
 int out_dim(int in, int k, int st, int pad) { return (in + 2 * pad - k) / st + 1; }
 
@@ -574,6 +993,52 @@ int grid_size(int total_tiles)
     return g < 1 ? 1 : g;
 }
 
+// Dynamic shared memory the window kernel may use (227 KB per CTA, less the
+// static barriers and 1 KB of alignment slack).
+constexpr size_t kWinSmemMax = 232448 - 2048;
+
+// Window-kernel eligibility and geometry (see conv_win_kernel): 3x3 filters,
+// stride 1 and pad 1 on both axes, 64-channel blocks of the reduced operand
+// (red_c), 64 or 128 output channels, images 8..254 wide.
+bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, Plan& pl)
+{
+    const Geom g = geom(s);
+    if (s->r != 3 || s->s != 3 || g.sh != 1 || g.sw != 1 || g.ph != 1 || g.pw != 1) return false;
+    if (red_c % 64 != 0 || (out_c != 64 && out_c != 128)) return false;
+    const int Wp = s->w + 2, Hp = s->h + 2;
+    if (Wp < 10 || Wp > 256) return false;
+    const int64_t L = (int64_t)s->n * Hp * Wp;
+    if (L > INT32_MAX / 4) return false;
+    // a tile's rows start anywhere in a padded row and reach 2*Wp + 2 positions past its end
+    const int srows = kWinBMT / Wp + 4;
+    const int strip = ((srows * Wp * 128 + 1023) / 1024) * 1024;
+    const int BN = out_c, CB = red_c / 64;
+    const bool res = BN == 64 && CB == 1;
+    const int b_bytes = res ? 9 * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128;
+    const size_t smem = (size_t)b_bytes + 2 * (size_t)strip + kEpiTileBytes + 4 * 2 * (size_t)out_c * 4 + 1024;
+    if (smem > kWinSmemMax) return false;
+    ConvParams& p = pl.p;
+    pl.win = true;
+    pl.res = res;
+    pl.BN = BN;
+    pl.smem = smem;
+    p.win_H = s->h;
+    p.win_W = s->w;
+    p.win_Hp = Hp;
+    p.win_Wp = Wp;
+    p.win_srows = srows;
+    p.win_strip_bytes = strip;
+    p.M = s->n * s->h * s->w;
+    p.m_tiles = (int)((L + kWinBMT - 1) / kWinBMT);
+    p.n_tiles = 1;
+    p.cblocks = CB;
+    p.gN = s->n;
+    p.Ncols = out_c;
+    p.ldo = out_c;
+    p.Cin = red_c;
+    return true;
+}
+
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
 {
     using dbl::set_error;
@@ -589,7 +1054,12 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
     p.S = s->s;
     p.Cin = s->c;
     p.zdim = 1;
-    if (pass == DBL_PASS_FWD) {
+    if (pass == DBL_PASS_FWD && !c8 && win_setup(s, s->c, s->k, pl)) {
+        pl.mode = p.mode = kFwd;
+        pl.ws_main = (size_t)kMaxGrid * 2 * s->k * sizeof(float);
+    } else if (pass == DBL_PASS_DGRAD && s->c % 64 == 0 && win_setup(s, s->k, s->c, pl)) {
+        pl.mode = p.mode = kDgrad;
+    } else if (pass == DBL_PASS_FWD) {
         pl.mode = p.mode = c8 ? kFwdC8 : kFwd;
         if (c8 && p.ntaps > 56) return set_error(DBL_ERR_UNSUPPORTED, "conv_fwd: stem filter too large");
         const int64_t M = (int64_t)s->n * P * Q;
@@ -775,6 +1245,42 @@ int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid,
     return launch_cfg<64, kFamFwd>(pl, a, b, grid, st);
 }
 
+template <int BN, bool DG, bool RES>
+int launch_win_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+{
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(conv_win_kernel<BN, DG, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kWinSmemMax);
+        if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
+        attr_set[dev] = true;
+    }
+    conv_win_kernel<BN, DG, RES><<<grid, kWinThreads, pl.smem, st>>>(a, b, pl.p);
+    return dbl::launch_check("conv_win launch");
+}
+
+int launch_win(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+{
+    const bool dg = pl.mode == kDgrad;
+    if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false>(pl, a, b, grid, st)
+                                : launch_win_cfg<128, false, false>(pl, a, b, grid, st);
+    if (pl.res) return dg ? launch_win_cfg<64, true, true>(pl, a, b, grid, st)
+                          : launch_win_cfg<64, false, true>(pl, a, b, grid, st);
+    return dg ? launch_win_cfg<64, true, false>(pl, a, b, grid, st) : launch_win_cfg<64, false, false>(pl, a, b, grid, st);
+}
+
+// Tensor map of the window kernel's strip operand: one padded row (Wp pixels
+// x 64 channels, starting at w = -1) of an NHWC tensor per copy.
+int enc_win_rows(CUtensorMap* m, const void* base, int N, int H, int W, int C, int Wp)
+{
+    cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t str[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)Wp, 1, 1};
+    return enc_tiled(m, base, 4, dims, str, box, true);
+}
+
 // Rows of one tile of the forward family (see Cfg).
 int fwd_tile_rows(int BN) { return BN <= 128 ? 256 : 128; }
 
@@ -805,7 +1311,14 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
     CUtensorMap ta, tb;
     const Geom g = geom(s);
-    if (pl.mode == kFwdC8) {
+    if (pl.win) {
+        if ((rc = enc_win_rows(&ta, x, s->n, s->h, s->w, s->c, pl.p.win_Wp))) return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * s->c;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
+    } else if (pl.mode == kFwdC8) {
         if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
                              g.sw, 8, fwd_tile_rows(pl.BN), false)))
             return rc;
@@ -828,9 +1341,9 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
     pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
     const int grid = grid_size(pl.p.total_tiles);
     cudaStream_t st = as_stream(stream);
-    if ((rc = launch(pl, ta, tb, grid, st))) return rc;
+    if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, grid, st))) return rc;
     if (stats) {
-        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
+        stats_reduce_kernel<<<(s->k + 31) / 32, 32 * kColsumGroups, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
         if ((rc = launch_check("conv stats reduce"))) return rc;
     }
     return DBL_OK;
@@ -849,21 +1362,27 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
         return set_error(DBL_ERR_INVALID, "conv_dgrad: null or misaligned tensor");
     const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
     CUtensorMap ta, tb;
-    // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
-    int lower = 0, upper = 0;
-    if (s->stride == 1) {
-        lower = -(s->r - 1 - s->pad);
-        upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
+    if (pl.win) {
+        if ((rc = enc_win_rows(&ta, dy, s->n, P, Q, s->k, pl.p.win_Wp))) return rc;
+    } else {
+        // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
+        int lower = 0, upper = 0;
+        if (s->stride == 1) {
+            lower = -(s->r - 1 - s->pad);
+            upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
+        }
+        if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, lower, upper, 1, 1, 64, fwd_tile_rows(pl.BN),
+                             true)))
+            return rc;
     }
-    if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, lower, upper, 1, 1, 64, fwd_tile_rows(pl.BN), true)))
-        return rc;
     // w viewed as [k][r*s][c]: inner c, then tap, then k
     cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
     cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
     cuuint32_t box[3] = {64, 1, 64};
     if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
     pl.p.out = dx;
-    return launch(pl, ta, tb, grid_size(pl.p.total_tiles), as_stream(stream));
+    const int grid = grid_size(pl.p.total_tiles);
+    return pl.win ? launch_win(pl, ta, tb, grid, as_stream(stream)) : launch(pl, ta, tb, grid, as_stream(stream));
 }
 
 int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float* dw, int accumulate, void* ws,
@@ -895,11 +1414,15 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     if ((rc = launch(pl, ta, tb, grid_size(pl.p.total_tiles), st))) return rc;
     if (!sliced) return DBL_OK;
     const int64_t n = (int64_t)pl.p.M * s->k;
-    int64_t blocks = (n / 4 + 255) / 256;
+    const int lanes = pl.p.zdim > 8 ? 8 : 1;
+    int64_t blocks = (n / 4 + 256 / lanes - 1) / (256 / lanes);
     const int64_t cap = (int64_t)sm_count() * 8;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    wgrad_reduce_kernel<<<(int)blocks, 256, 0, st>>>(static_cast<const float*>(ws), pl.p.zdim, n, dw, accumulate);
+    if (lanes == 8)
+        wgrad_reduce_kernel<8><<<(int)blocks, 256, 0, st>>>(static_cast<const float*>(ws), pl.p.zdim, n, dw, accumulate);
+    else
+        wgrad_reduce_kernel<1><<<(int)blocks, 256, 0, st>>>(static_cast<const float*>(ws), pl.p.zdim, n, dw, accumulate);
     return launch_check("conv wgrad reduce");
 }
 

@@ -231,6 +231,52 @@ __device__ __forceinline__ void mbar_arrive_expect_tx_elect(uint64_t* bar, uint3
         : "memory");
 }
 
+// ---------------------------------------------------------------------------- fixed-order column sums
+// Column sums of a row-major fp32 matrix part[nrows][ld] for the 32 columns
+// col0 .. col0+31, by a block of 32 x kColsumGroups threads: thread (g, lane)
+// sums rows g, g + kColsumGroups, ... of column col0 + lane in fp32 with
+// Kahan compensation (16 loads in flight before the adds), then one thread
+// per column adds the groups 0..kColsumGroups-1 in order, in double.  (FP64
+// arithmetic is slow on this GPU, so only the last kColsumGroups adds use it.)
+// The order depends only on nrows, so the result is the same on every launch
+// and every GPU.  Returns the column sum in threads with g == 0 (other threads
+// return 0); every thread of the block must call it (it synchronises the block).
+constexpr int kColsumGroups = 32;
+
+__device__ __forceinline__ void kahan_add(float& sum, float& comp, float v)
+{
+    const float y = v - comp;
+    const float t = sum + y;
+    comp = (t - sum) - y;
+    sum = t;
+}
+
+__device__ __forceinline__ double colsum_fixed_order(const float* __restrict__ part, int nrows, int64_t ld,
+                                                     int col0, int ncols, double* red /* [kColsumGroups][32] */)
+{
+    const int lane = threadIdx.x % 32, g = threadIdx.x / 32;
+    const int col = col0 + lane;
+    float sum = 0.f, comp = 0.f;
+    if (col < ncols) {
+        int t = g;
+        for (; t + 15 * kColsumGroups < nrows; t += 16 * kColsumGroups) {
+            float v[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) v[u] = __ldg(part + (int64_t)(t + u * kColsumGroups) * ld + col);
+#pragma unroll
+            for (int u = 0; u < 16; ++u) kahan_add(sum, comp, v[u]);
+        }
+        for (; t < nrows; t += kColsumGroups) kahan_add(sum, comp, __ldg(part + (int64_t)t * ld + col));
+    }
+    red[g * 32 + lane] = (double)sum - (double)comp;
+    __syncthreads();
+    double total = 0.0;
+    if (g == 0)
+        for (int k = 0; k < kColsumGroups; ++k) total += red[k * 32 + lane];
+    __syncthreads();
+    return total;
+}
+
 // ---------------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* tmap)
 {
@@ -291,6 +337,18 @@ __device__ __forceinline__ void tma_load_3d_elect(void* dst, const void* tmap, u
         "@E cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%3, %4, %5}], [%2];\n\t}" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1,
+                                                  int32_t c2, int32_t c3)
+{
+    asm volatile(
+        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "@E cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
         : "memory");
 }
 

@@ -243,6 +243,10 @@ FWD_CASES = [  # n, h, w, c, k, r, stride, pad
     (1, 4, 4, 256, 256, 3, 1, 1),    # deep layer, small image, 256-wide tile
     (4, 14, 14, 256, 512, 3, 2, 1),  # two 256-wide column tiles, stride 2
     (32, 56, 56, 64, 64, 3, 1, 1),   # 784 tiles: every persistent CTA loops over several
+    # 3x3 stride-1 window kernel: strips of zero-padded rows, taps as shifted descriptors
+    (4, 28, 28, 128, 128, 3, 1, 1),  # streamed 128-wide weight tiles, two channel blocks
+    (5, 5, 13, 128, 64, 3, 1, 1),    # streamed 64-wide tiles; a tile spans several small images
+    (1, 3, 254, 64, 64, 3, 1, 1),    # widest padded row a copy can carry (256 pixels)
 ]
 
 
@@ -287,6 +291,8 @@ DGRAD_CASES = [
     (1, 4, 4, 256, 256, 3, 1, 1),
     (2, 8, 8, 512, 512, 3, 1, 1),    # 256-wide tiles, 8 channel blocks of dy
     (16, 28, 28, 128, 128, 3, 1, 1), # many tiles per CTA
+    (5, 5, 13, 64, 128, 3, 1, 1),    # window kernel, 64-wide streamed tiles over two dy channel blocks
+    (2, 9, 30, 64, 64, 3, 1, 1),     # window kernel, resident flipped weights, non-square image
 ]
 
 
