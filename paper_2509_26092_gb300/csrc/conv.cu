@@ -72,8 +72,9 @@ struct ConvParams {
     // window kernel (3x3, stride 1, pad 1): the batch as one column of zero-padded images
     int win_H, win_W;         // image height and width (= output height and width)
     int win_Hp, win_Wp;       // padded height and width (H + 2, W + 2)
-    int win_srows;            // padded rows loaded per strip
-    int win_strip_bytes;      // bytes of one strip buffer (a multiple of 1024)
+    int win_srows;            // padded rows loaded per strip (weight gradient: x strip)
+    int win_dyrows;           // weight gradient: padded rows of the dy strip
+    int win_strip_bytes;      // bytes of one strip buffer, or of one x + dy stage (a multiple of 1024)
 };
 
 __device__ __forceinline__ void report_timeout(volatile int* abort)
@@ -846,6 +847,190 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     }
 }
 
+// ----------------------------------------------------------------------------- window weight gradient
+// dW[k][r][s][c] = sum over positions L of dy[L][k] * x_pad[L + r*Wp + s][c] for 3x3 stride-1
+// layers with 64 input and 64 output channels, in the padded position space of conv_win_kernel:
+// dy is zero at the positions that are not outputs (its strip rows are read with w from 0 to
+// Wp-1 and h from 0 to Hp-1, and the zero fill of TMA covers w >= W and h >= H).
+// A CTA owns all 576 x 64 outputs, as five 128 x 64 TMEM accumulators (tap pairs (0,1), (2,3),
+// (4,5), (6,7), (8, -)), and one contiguous range of K-blocks of 256 positions (split-K over
+// CTAs, fixed-order reduce afterwards).  Per K-block it loads one x strip and one dy strip; all
+// nine taps read the same x strip.  A operand (x, MN-major: a 128-byte strip row holds the 64
+// channels of one position) of tap pair (t0, t1): start row off(t0) + 16j for K-step j, second
+// 64-row half LBO = (off(t1) - off(t0)) rows further; the fifth pair's second half is computed
+// and not stored.  B operand (dy, MN-major): start row 16j.
+constexpr int kWgWinKB = 256;  // positions per K-block
+constexpr int kWgWinAcc = 5;   // 128-row accumulators (tap pairs)
+
+__global__ void __launch_bounds__(kWinThreads, 1)
+    conv_wgwin_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmDY,
+                      const ConvParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[2], empty_bar[2], accf_bar, acce_bar, drain_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
+    const int Wp = p.win_Wp;
+    const int xalign = ((p.win_srows * Wp * 128 + 1023) / 1024) * 1024;  // dy strip offset in a stage
+    const int stage_bytes = p.win_strip_bytes;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&full_bar[i], 2);  // one expect_tx arrival per producer warp
+            mbar_init(&empty_bar[i], 1);
+        }
+        mbar_init(&accf_bar, 1);
+        mbar_init(&acce_bar, 4);
+        mbar_init(&drain_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if ((warp == 4 || warp == 5) && lane == 0) tma_prefetch_desc(warp == 4 ? &tmX : &tmDY);
+    if (warp == 6) {
+        tmem_alloc(&tmem_slot, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 4 || warp == 5) {
+        // ------------------------------------------------------------------ producers: x rows (4), dy rows (5)
+        const bool is_x = warp == 4;
+        const int rows = is_x ? p.win_srows : p.win_dyrows;
+        const uint32_t tx = (uint32_t)(rows * Wp * 128);
+        int it = 0;
+        bool failed = false;
+        for (int z = blockIdx.x; z < p.zdim && !failed; z += gridDim.x) {
+            const int kb0 = z * p.kb_per_split, kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+            for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                const int s = it & 1;
+                const uint32_t ok = mbar_wait_warp(&empty_bar[s], ((it >> 1) & 1) ^ 1, &abort_flag);
+                if (__any_sync(0xffffffffu, ok == 0u)) {
+                    failed = true;
+                    break;
+                }
+                uint8_t* dst = sgen + s * stage_bytes + (is_x ? 0 : xalign);
+                const int g0 = kb * kWgWinKB / Wp;
+                mbar_arrive_expect_tx_elect(&full_bar[s], tx);
+                for (int r = 0; r < rows; ++r) {
+                    const int g = g0 + r;
+                    const int n = g / p.win_Hp, hp = g - n * p.win_Hp;
+                    if (is_x)
+                        tma_load_4d_elect(dst + r * Wp * 128, &tmX, &full_bar[s], 0, -1, hp - 1, n);
+                    else
+                        tma_load_4d_elect(dst + r * Wp * 128, &tmDY, &full_bar[s], 0, 0, hp, n);
+                }
+            }
+        }
+        if (failed) {
+            if (lane == 0) report_timeout(&abort_flag);
+            for (int i = it - 1; i >= 0 && i >= it - 2; --i) (void)mbar_drain_warp(&full_bar[i & 1], (i >> 1) & 1);
+        }
+    } else if (warp == 6) {
+        // ------------------------------------------------------------------ MMA issuer
+        const uint32_t idesc = idesc_bf16(BM, 64, 1u, 1u);
+        int it = 0, lt = 0;
+        bool failed = false;
+        for (int z = blockIdx.x; z < p.zdim && !failed; z += gridDim.x, ++lt) {
+            const uint32_t ok = mbar_wait_warp(&acce_bar, (lt & 1) ^ 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                failed = true;
+                break;
+            }
+            tc_fence_after();
+            const int kb0 = z * p.kb_per_split, kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+            for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                const int s = it & 1;
+                const uint32_t okf = mbar_wait_warp(&full_bar[s], (it >> 1) & 1, &abort_flag);
+                if (__any_sync(0xffffffffu, okf == 0u)) {
+                    failed = true;
+                    break;
+                }
+                tc_fence_after();
+                const int P0 = kb * kWgWinKB;
+                const int off = P0 - (P0 / Wp) * Wp;
+                const uint32_t xa = sbase + (uint32_t)(s * stage_bytes), ya = xa + (uint32_t)xalign;
+#pragma unroll 1
+                for (int j = 0; j < kWgWinKB / 16; ++j) {
+                    const uint64_t bd = smem_desc(ya + (uint32_t)((off + 16 * j) * 128), 16384, 1024, kSwizzle128B);
+#pragma unroll
+                    for (int pp = 0; pp < kWgWinAcc; ++pp) {
+                        const int t0 = 2 * pp, t1 = 2 * pp + 1;
+                        const int o0 = (t0 / 3) * Wp + t0 % 3;
+                        const int o1 = t1 < 9 ? (t1 / 3) * Wp + t1 % 3 : o0 + 1;
+                        const uint64_t ad =
+                            smem_desc(xa + (uint32_t)((off + o0 + 16 * j) * 128), (uint32_t)((o1 - o0) * 128), 1024,
+                                      kSwizzle128B);
+                        mma_bf16_elect(tmem + (uint32_t)(pp * 64), ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
+                    }
+                }
+                mma_commit_elect(&empty_bar[s]);
+            }
+            mma_commit_elect(&accf_bar);  // arrives when this split's MMAs have completed
+        }
+        if (failed && lane == 0) report_timeout(&abort_flag);
+        mma_commit_elect(&drain_bar);
+        (void)mbar_drain_warp(&drain_bar, 0);
+    } else {
+        // ------------------------------------------------------------------ epilogue (warps 0-3)
+        const int i = warp * 32 + lane;  // TMEM lane = accumulator row
+        int lt = 0;
+        for (int z = blockIdx.x; z < p.zdim; z += gridDim.x, ++lt) {
+            const uint32_t ok = mbar_wait_warp(&accf_bar, lt & 1, &abort_flag);
+            if (__any_sync(0xffffffffu, ok == 0u)) {
+                if (lane == 0) report_timeout(&abort_flag);
+                break;
+            }
+            tc_fence_after();
+            const int kb0 = z * p.kb_per_split;
+            const bool have_acc = min(p.num_kb, kb0 + p.kb_per_split) > kb0;
+#pragma unroll 1
+            for (int pp = 0; pp < kWgWinAcc; ++pp) {
+                const int tap = 2 * pp + (i >> 6), c = i & 63;
+                const bool valid = tap < 9;
+                const int m = tap * 64 + c;  // row of dW viewed as [k][(r, s, c)]
+#pragma unroll 1
+                for (int ch = 0; ch < 2; ++ch) {
+                    uint32_t v[32];
+                    if (have_acc) {
+                        tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(pp * 64 + ch * 32), v);
+                        tmem_ld_wait();
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) v[k] = 0u;
+                    }
+                    if (valid) {
+                        // [slice][k][m]: consecutive lanes hold consecutive m, one 128-byte line per store
+                        float* o = static_cast<float*>(p.out) + ((int64_t)(p.zdim > 1 ? z : 0) * 64 + ch * 32) * p.M + m;
+                        if (p.zdim == 1 && p.wg_accumulate) {
+#pragma unroll
+                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] += __uint_as_float(v[k]);
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < 32; ++k) o[(int64_t)k * p.M] = __uint_as_float(v[k]);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce_bar);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 6) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
 // ----------------------------------------------------------------------------- reductions
 // Per-channel sums over the per-CTA partials [nparts][2][K], fixed order
 // (colsum_fixed_order); block b covers channels 32b .. 32b+31 of both halves.
@@ -1039,6 +1224,50 @@ bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, Plan& pl)
     return true;
 }
 
+// Window weight-gradient eligibility and geometry (see conv_wgwin_kernel): 3x3
+// filters, stride 1 and pad 1, 64 input and 64 output channels, images 8..254 wide.
+bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
+{
+    const Geom g = geom(s);
+    if (s->r != 3 || s->s != 3 || g.sh != 1 || g.sw != 1 || g.ph != 1 || g.pw != 1) return false;
+    if (s->c != 64 || s->k != 64) return false;
+    const int Wp = s->w + 2, Hp = s->h + 2;
+    if (Wp < 10 || Wp > 256) return false;
+    const int64_t L = (int64_t)s->n * Hp * Wp;
+    if (L > INT32_MAX / 4) return false;
+    // a K-block starts anywhere in a padded row; x reaches 2*Wp + 3 positions past its end
+    // (the unused tenth tap), dy none
+    const int xrows = (kWgWinKB + 3 * Wp + 1) / Wp + 1;
+    const int dyrows = (kWgWinKB + Wp - 2) / Wp + 1;
+    const int xalign = ((xrows * Wp * 128 + 1023) / 1024) * 1024;
+    const int stage = xalign + ((dyrows * Wp * 128 + 1023) / 1024) * 1024;
+    const size_t smem = 2 * (size_t)stage + 1024;
+    if (smem > kWinSmemMax) return false;
+    ConvParams& p = pl.p;
+    pl.win = true;
+    pl.BN = 64;
+    pl.smem = smem;
+    pl.mode = p.mode = kWgrad;
+    p.win_H = s->h;
+    p.win_W = s->w;
+    p.win_Hp = Hp;
+    p.win_Wp = Wp;
+    p.win_srows = xrows;
+    p.win_dyrows = dyrows;
+    p.win_strip_bytes = stage;
+    p.M = 9 * 64;
+    p.Ncols = 64;
+    p.m_tiles = p.n_tiles = 1;
+    p.gN = s->n;
+    p.num_kb = (int)((L + kWgWinKB - 1) / kWgWinKB);
+    // one contiguous range of K-blocks per CTA of a persistent grid
+    int splits = grid_size(p.num_kb);
+    p.kb_per_split = (p.num_kb + splits - 1) / splits;
+    p.zdim = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
+    pl.ws_main = p.zdim > 1 ? (size_t)p.zdim * p.M * 64 * sizeof(float) : 0;
+    return true;
+}
+
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
 {
     using dbl::set_error;
@@ -1059,6 +1288,8 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         pl.ws_main = (size_t)kMaxGrid * 2 * s->k * sizeof(float);
     } else if (pass == DBL_PASS_DGRAD && s->c % 64 == 0 && win_setup(s, s->k, s->c, pl)) {
         pl.mode = p.mode = kDgrad;
+    } else if (pass == DBL_PASS_WGRAD && wgwin_setup(s, pl)) {
+        // conv_wgwin_kernel: tiles are the split-K ranges
     } else if (pass == DBL_PASS_FWD) {
         pl.mode = p.mode = c8 ? kFwdC8 : kFwd;
         if (c8 && p.ntaps > 56) return set_error(DBL_ERR_UNSUPPORTED, "conv_fwd: stem filter too large");
@@ -1399,6 +1630,26 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     const Geom g = geom(s);
     const int P = out_dim(s->h, s->r, g.sh, g.ph), Q = out_dim(s->w, s->s, g.sw, g.pw);
     CUtensorMap ta, tb;
+    cudaStream_t st = as_stream(stream);
+    const bool sliced = pl.p.zdim > 1;
+    if (pl.win) {
+        if ((rc = enc_win_rows(&ta, x, s->n, s->h, s->w, s->c, pl.p.win_Wp))) return rc;
+        if ((rc = enc_win_rows(&tb, dy, s->n, P, Q, s->k, pl.p.win_Wp))) return rc;
+        pl.p.out = sliced ? ws : static_cast<void*>(dw);
+        pl.p.wg_accumulate = accumulate;
+        static bool attr_set[64] = {false};
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+            if ((rc = cuda_check(cudaFuncSetAttribute(conv_wgwin_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      (int)kWinSmemMax),
+                                 "conv: set smem attribute")))
+                return rc;
+            attr_set[dev] = true;
+        }
+        conv_wgwin_kernel<<<grid_size(pl.p.zdim), kWinThreads, pl.smem, st>>>(ta, tb, pl.p);
+        if ((rc = launch_check("conv_wgwin launch"))) return rc;
+    } else {
     const bool c8 = pl.mode == kWgradC8;
     if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh, g.sw,
                          c8 ? 8 : 64, 128, !c8)))
@@ -1407,11 +1658,10 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     cuuint64_t str[1] = {(cuuint64_t)s->k * 2};
     cuuint32_t box[2] = {64, 128};
     if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
-    const bool sliced = pl.p.zdim > 1;
     pl.p.out = sliced ? ws : static_cast<void*>(dw);
     pl.p.wg_accumulate = accumulate;
-    cudaStream_t st = as_stream(stream);
     if ((rc = launch(pl, ta, tb, grid_size(pl.p.total_tiles), st))) return rc;
+    }
     if (!sliced) return DBL_OK;
     const int64_t n = (int64_t)pl.p.M * s->k;
     const int lanes = pl.p.zdim > 8 ? 8 : 1;

@@ -324,6 +324,9 @@ WGRAD_CASES = [
     (2, 8, 8, 256, 512, 3, 2, 1),    # 256-wide tiles
     (16, 28, 28, 128, 128, 3, 1, 1), # split-K slices reduced in order
     (1, 3, 3, 64, 64, 3, 1, 1),      # a single slice, written straight into dw
+    # window weight gradient (64 -> 64, 3x3 stride 1): x and dy strips, five tap-pair accumulators
+    (32, 56, 56, 64, 64, 3, 1, 1),   # the layer1 shape at batch 32: one K-range per CTA
+    (3, 5, 30, 64, 64, 3, 1, 1),     # K-blocks spanning several small non-square images
 ]
 
 
