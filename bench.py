@@ -375,19 +375,24 @@ def run_profile_conv(args):
         if b.proj:
             shapes[b.pre + ".down"] = D.conv_shape(n, h, h, b.cin, b.cout, 1, b.stride, 0)
         h = ho
+    st_, lay = spec.stem, spec.stem_layout  # the stem as a convolution of its unrolled 224 px input
+    hs = R.conv_out(224, st_.r, st_.stride, st_.pad)
+    shapes[st_.name] = D.conv_shape(n, lay.rows(224, hs), hs, 64, st_.cout, lay.taps, lay.conv_stride, lay.conv_pad,
+                                    s=1, stride_w=1, pad_w=0)
     if layer not in shapes:
         raise SystemExit(f"--profile-conv: unknown layer {layer!r} (one of {', '.join(shapes)})")
     s = shapes[layer]
     P = R.conv_out(s.h, s.r, s.stride, s.pad)
+    Q = R.conv_out(s.w, s.s, s.stride_w or s.stride, s.pad_w if s.stride_w else s.pad)
     g = torch.Generator(device="cuda").manual_seed(0)
     x = torch.randn(s.n, s.h, s.w, s.c, device="cuda", generator=g).to(torch.bfloat16)
     w = (0.05 * torch.randn(s.k, s.r, s.s, s.c, device="cuda", generator=g)).to(torch.bfloat16)
-    dy = torch.randn(s.n, P, P, s.k, device="cuda", generator=g).to(torch.bfloat16)
+    dy = torch.randn(s.n, P, Q, s.k, device="cuda", generator=g).to(torch.bfloat16)
     ps = {"fwd": D.DBL_PASS_FWD, "dgrad": D.DBL_PASS_DGRAD, "wgrad": D.DBL_PASS_WGRAD}[pname]
     ws = torch.empty(max(int(D.dbl_conv_workspace_bytes(s, ps)), 16), dtype=torch.uint8, device="cuda")
     st = torch.cuda.current_stream()
     if pname == "fwd":
-        y = torch.empty(s.n, P, P, s.k, dtype=torch.bfloat16, device="cuda")
+        y = torch.empty(s.n, P, Q, s.k, dtype=torch.bfloat16, device="cuda")
         ssum, ssq = torch.empty(s.k, device="cuda"), torch.empty(s.k, device="cuda")
         fn = lambda: D.dbl_conv_fwd(s, x, w, y, ssum, ssq, ws, ws.numel(), st)
     elif pname == "dgrad":
@@ -405,6 +410,7 @@ def run_profile_conv(args):
 
 
 def run_ours(args, cfg):
+    import numpy as np
     import torch
     ws, rank, local = _dist()
     if ws > 1:
@@ -465,27 +471,43 @@ def run_ours(args, cfg):
         torch.cuda.synchronize()
         per_res[str(st["res"])] = round(st["images"] * reps / (e0.elapsed_time(e1) / 1000.0), 1)
 
-    # end to end through the public API: pinned host images -> device, iteration, loss back to host
+    # end to end through the public API: pinned host images -> device (on a copy stream, each
+    # stage's copy overlapping the compute of the stages before it), iteration, losses back to
+    # pinned host memory; step k's losses are read on the host after step k+1 is enqueued
     h2d = d2h = 0
+    copy_stream = torch.cuda.Stream()
+    loss_host = [torch.zeros(2 * len(stages), dtype=torch.float32).pin_memory() for _ in range(2)]
+    loss_seen = []
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     e0.record(stream)
-    for _ in range(args.steps):
+    prev = None
+    for k in range(args.steps):
         for st in stages:
             it, bl, bs = st["it"], st["large"].batch, st["small"].batch if st["small"] else 0
             it.set_inputs(pipe["host_l"][:bl], pipe["lab_l"][:bl], pipe["host_s"][:bs] if bs else None,
-                          pipe["lab_s"][:bs] if bs else None, non_blocking=True)
-            it.run()
-            losses = [st["large"].loss.to("cpu", non_blocking=False)]
-            if st["small"] is not None:
-                losses.append(st["small"].loss.to("cpu", non_blocking=False))
+                          pipe["lab_s"][:bs] if bs else None, non_blocking=True, stream=copy_stream)
+        buf = loss_host[k % 2]
+        n_out = 0
+        for st in stages:
+            st["it"].run()
+            n_out += st["it"].losses_to_host(buf[n_out:])
+        done = torch.cuda.Event()
+        done.record(stream)
+        if prev is not None:
+            prev[0].synchronize()
+            loss_seen.append(prev[1][:prev[2]].tolist())
+        prev = (done, buf, n_out)
         if h2d == 0:
             for st in stages:
                 bl, bs = st["large"].batch, st["small"].batch if st["small"] else 0
                 h2d += (bl + bs) * cfg["native"] ** 2 * 3 * 4 + (bl + bs) * 4
                 d2h += 4 * (2 if bs else 1)
+    prev[0].synchronize()
+    loss_seen.append(prev[1][:prev[2]].tolist())
     e1.record(stream)
     barrier()
+    assert len(loss_seen) == args.steps and all(np.isfinite(v).all() for v in map(np.asarray, loss_seen))
     e2e_ms = e0.elapsed_time(e1)
     if ws > 1:
         tt = torch.tensor([e2e_ms], device=device)

@@ -248,19 +248,34 @@ DBL_API int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const flo
 DBL_API int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
                            int out_dtype, int32_t h_out, int32_t w_out, int32_t c_out_stride, void* stream);
 
-/* The same resize, written in the layout the tensor-core stem consumes: the
- * resized image unrolled along W for a stem with `taps` filter columns,
- * column stride stride_w and padding pad_w.  Output position (n, h, q) holds
- * the resized pixels at columns q*stride_w + t - pad_w, t = 0..7, each with
- * 8 channels (t >= taps, columns outside the image and channels >= c are
- * zero):  out[n][h][q][t][ch], bf16, Q = (w_out + 2*pad_w - taps)/stride_w + 1.
- * A taps x taps stem convolution of the resized image then equals an
- * r x 1 convolution (stride along H only, 64 channels) of this tensor with
- * the weights stored as [k][r][8][8] (taps and channels zero-padded).
- * in: [n,h_in,w_in,c] fp32, c <= 8, taps <= 8. */
+/* The same resize, written in the layout the tensor-core stem consumes.
+ * Output position (n, m, q), m < rows_out, q < Q, holds row_group source rows
+ * y = row_group*m + e - pad_h (e < row_group) of the resized image, each
+ * unrolled along W for a stem with `taps` filter columns, column stride
+ * stride_w and padding pad_w: element (e, t, ch) is the resized pixel at
+ * (y, q*stride_w + t - pad_w), channel ch, for t = 0..7 and ch < 8/row_group
+ * (zero outside the image, for t >= taps and for ch >= c):
+ *   out[n][m][q][e][t][ch], bf16, 128 bytes per position,
+ *   Q = (w_out + 2*pad_w - taps)/stride_w + 1.
+ * With row_group 1 and pad_h 0 (rows_out = h_out), a taps x taps stem of
+ * stride s equals an r x 1 convolution of this tensor (stride s along H
+ * only, the stem's padding along H, 64 channels) with the weights stored as
+ * [k][r][8][8]; with row_group 2 (a stride-2 stem: pad_h = its padding and
+ * rows_out = P + ceil(r/2) - 1 for P output rows), it equals a ceil(r/2) x 1
+ * valid convolution of stride 1 with the weights stored as [k][2*ceil(r/2)][8][4]
+ * (rows r.. of that layout are not filter rows and must stay zero: their
+ * weight gradient is not part of the method, see dbl_zero_f32_2d).
+ * in: [n,h_in,w_in,c] fp32, c <= 8/row_group, taps <= 8. */
 DBL_API int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
                                         int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
-                                        void* stream);
+                                        int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream);
+
+/* Sets base[i*ld + j] = 0 for i < rows, j < cols (fp32, device memory, stream
+ * ordered).  The ResNet-18 stem uses it to keep the weight gradient of the
+ * padding rows of its row-grouped weight layout at zero, so that those
+ * weights stay zero through the parameter-server update.  Not a step of the
+ * paper's method. */
+DBL_API int dbl_zero_f32_2d(float* base, int64_t rows, int64_t cols, int64_t ld, void* stream);
 
 /* Host: the integer taps above for one axis (i0, i1, lambda: [out] each). */
 DBL_API int dbl_resize_taps(int32_t in, int32_t out, int32_t* i0, int32_t* i1, float* lambda);

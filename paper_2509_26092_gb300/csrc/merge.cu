@@ -139,3 +139,13 @@ extern "C" int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const 
     ps_merge_kernel<<<blocks, threads, 0, as_stream(stream)>>>(a);
     return launch_check("ps_merge launch");
 }
+
+extern "C" int dbl_zero_f32_2d(float* base, int64_t rows, int64_t cols, int64_t ld, void* stream)
+{
+    using namespace dbl;
+    if (!base || rows < 0 || cols < 0 || ld < cols) return set_error(DBL_ERR_INVALID, "zero_f32_2d: bad arguments");
+    if (rows == 0 || cols == 0) return DBL_OK;
+    return cuda_check(cudaMemset2DAsync(base, (size_t)ld * sizeof(float), 0, (size_t)cols * sizeof(float), (size_t)rows,
+                                        as_stream(stream)),
+                      "zero_f32_2d");
+}

@@ -105,44 +105,56 @@ int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, 
     return dbl::launch_check("progressive_resize launch");
 }
 
-// One thread per unrolled output position (n, h, q): eight column taps of eight
-// channels, 128 bytes, written as eight 16-byte stores.
+// The stem's unrolled input.  Position (n, m, q) holds rg source rows
+// y = rg*m + e - pad_h (e < rg), each as 8 column taps x (8/rg) channels:
+// element (e, t, ch) is the resized pixel at (y, q*sw + t - pw), channel ch
+// (zero outside the image, for t >= taps and for ch >= c).  One thread per
+// 16-byte chunk (8 elements): a warp's stores cover 512 contiguous bytes.
+template <int RG>
 __global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restrict__ in, __nv_bfloat16* __restrict__ out,
                                                           int32_t n, int32_t hi, int32_t wi, int32_t c, int32_t ho,
-                                                          int32_t wo, int32_t Q, int32_t taps, int32_t sw, int32_t pw)
+                                                          int32_t wo, int32_t M, int32_t Q, int32_t taps, int32_t sw,
+                                                          int32_t pw, int32_t ph)
 {
-    const unsigned total = (unsigned)n * ho * Q;
-    for (unsigned pos = blockIdx.x * blockDim.x + threadIdx.x; pos < total; pos += gridDim.x * blockDim.x) {
+    constexpr int32_t rg = RG;
+    constexpr int32_t cu = 8 / RG;     // channels per tap
+    constexpr int32_t tpc = 8 / cu;    // taps per 16-byte chunk (1 or 2); a chunk never spans two rows
+    const unsigned total = (unsigned)n * M * Q * 8;
+    for (unsigned idx = blockIdx.x * blockDim.x + threadIdx.x; idx < total; idx += gridDim.x * blockDim.x) {
+        const int32_t chunk = (int32_t)(idx & 7u);
+        const unsigned pos = idx >> 3;
         const int32_t q = (int32_t)(pos % (unsigned)Q);
         const unsigned t0 = pos / (unsigned)Q;
-        const int32_t y = (int32_t)(t0 % (unsigned)ho);
-        const int32_t b = (int32_t)(t0 / (unsigned)ho);
-        const Taps ty = axis_taps(y, hi, ho);
-        const float* base = in + (int64_t)b * hi * wi * c;
-        const float* r0 = base + (int64_t)ty.i0 * wi * c;
-        const float* r1 = base + (int64_t)ty.i1 * wi * c;
-        uint4* o = reinterpret_cast<uint4*>(out + (int64_t)pos * 64);
-#pragma unroll 1
-        for (int t = 0; t < 8; ++t) {
-            const int32_t x = q * sw + t - pw;
-            float v[8];
+        const int32_t m = (int32_t)(t0 % (unsigned)M);
+        const int32_t b = (int32_t)(t0 / (unsigned)M);
+        const int32_t e = chunk / cu, tap0 = (chunk % cu) * tpc;
+        const int32_t y = rg * m + e - ph;
+        float v[8];
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch) v[ch] = 0.f;
-            if (t < taps && x >= 0 && x < wo) {
+        for (int k = 0; k < 8; ++k) v[k] = 0.f;
+        if (y >= 0 && y < ho) {
+            const Taps ty = axis_taps(y, hi, ho);
+            const float* base = in + (int64_t)b * hi * wi * c;
+            const float* r0 = base + (int64_t)ty.i0 * wi * c;
+            const float* r1 = base + (int64_t)ty.i1 * wi * c;
+#pragma unroll
+            for (int32_t u = 0; u < tpc; ++u) {
+                const int32_t t = tap0 + u, x = q * sw + t - pw;
+                if (t >= taps || x < 0 || x >= wo) continue;
                 const Taps tx = axis_taps(x, wi, wo);
 #pragma unroll
-                for (int ch = 0; ch < 8; ++ch)
-                    if (ch < c) {
-                        const float top = (1.f - tx.lam) * __ldg(r0 + tx.i0 * c + ch) + tx.lam * __ldg(r0 + tx.i1 * c + ch);
-                        const float bot = (1.f - tx.lam) * __ldg(r1 + tx.i0 * c + ch) + tx.lam * __ldg(r1 + tx.i1 * c + ch);
-                        v[ch] = (1.f - ty.lam) * top + ty.lam * bot;
-                    }
+                for (int32_t ch = 0; ch < cu; ++ch) {
+                    if (ch >= c) break;
+                    const float top = (1.f - tx.lam) * __ldg(r0 + tx.i0 * c + ch) + tx.lam * __ldg(r0 + tx.i1 * c + ch);
+                    const float bot = (1.f - tx.lam) * __ldg(r1 + tx.i0 * c + ch) + tx.lam * __ldg(r1 + tx.i1 * c + ch);
+                    v[u * cu + ch] = (1.f - ty.lam) * top + ty.lam * bot;
+                }
             }
-            __nv_bfloat162 qv[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k) qv[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
-            o[t] = *reinterpret_cast<uint4*>(qv);
         }
+        __nv_bfloat162 qv[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) qv[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+        reinterpret_cast<uint4*>(out)[idx] = *reinterpret_cast<uint4*>(qv);
     }
 }
 
@@ -150,27 +162,36 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restric
 
 extern "C" int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
                                            int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
-                                           void* stream)
+                                           int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream)
 {
     using namespace dbl;
     if (!in || !out || n < 0 || h_in <= 0 || w_in <= 0 || c <= 0 || h_out <= 0 || w_out <= 0 || taps <= 0 ||
-        stride_w <= 0 || pad_w < 0)
+        stride_w <= 0 || pad_w < 0 || pad_h < 0 || rows_out <= 0)
         return set_error(DBL_ERR_INVALID, "progressive_resize_stem: bad sizes or null pointer");
-    if (c > 8 || taps > 8) return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: at most 8 channels and 8 taps");
+    if (row_group != 1 && row_group != 2)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: row_group must be 1 or 2");
+    if (c > 8 / row_group || taps > 8)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: at most 8 taps and 8/row_group channels");
     if (h_out > h_in || w_out > w_in) return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: upsampling");
     if (h_in > 16384 || w_in > 16384) return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: input side above 16384");
     if (!aligned16(out)) return set_error(DBL_ERR_INVALID, "progressive_resize_stem: output must be 16-byte aligned");
     const int32_t Q = (w_out + 2 * pad_w - taps) / stride_w + 1;
     if (Q <= 0) return set_error(DBL_ERR_INVALID, "progressive_resize_stem: empty output");
-    if ((int64_t)n * h_out * Q >= (int64_t)1 << 31)
+    if ((int64_t)n * rows_out * Q * 8 >= (int64_t)1 << 31)
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: output too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
-    const int64_t total = (int64_t)n * h_out * Q;
+    const int64_t total = (int64_t)n * rows_out * Q * 8;
     int64_t blocks = (total + 255) / 256;
     const int64_t cap = (int64_t)sm_count() * 16;
     if (blocks > cap) blocks = cap;
-    resize_stem_kernel<<<(int)(blocks < 1 ? 1 : blocks), 256, 0, as_stream(stream)>>>(
-        in, static_cast<__nv_bfloat16*>(out), n, h_in, w_in, c, h_out, w_out, Q, taps, stride_w, pad_w);
+    if (row_group == 2)
+        resize_stem_kernel<2><<<(int)(blocks < 1 ? 1 : blocks), 256, 0, as_stream(stream)>>>(
+            in, static_cast<__nv_bfloat16*>(out), n, h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w,
+            pad_h);
+    else
+        resize_stem_kernel<1><<<(int)(blocks < 1 ? 1 : blocks), 256, 0, as_stream(stream)>>>(
+            in, static_cast<__nv_bfloat16*>(out), n, h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w,
+            pad_h);
     return launch_check("progressive_resize_stem launch");
 }
 

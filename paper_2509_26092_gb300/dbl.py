@@ -79,7 +79,8 @@ def lib():
                                                       _I32, _I32, _I32, _V]),
             "dbl_resize_taps": (ctypes.c_int, [_I32, _I32, _V, _V, _V]),
             "dbl_progressive_resize_stem": (ctypes.c_int, [_V, _I32, _I32, _I32, _I32, _V, _I32, _I32, _I32, _I32,
-                                                           _I32, _V]),
+                                                           _I32, _I32, _I32, _I32, _V]),
+            "dbl_zero_f32_2d": (ctypes.c_int, [_V, _I64, _I64, _I64, _V]),
             "dbl_update_factor": (_D, [_D, _D, ctypes.c_int]),
             "dbl_plan": (ctypes.c_int, [_D, _D, _I32, _I32, _D, _D, _D, ctypes.c_int] + [ctypes.POINTER(_D)] * 4),
         }
@@ -220,9 +221,16 @@ def dbl_progressive_resize(inp, in_dtype, n, h_in, w_in, c, out, out_dtype, h_ou
                                         c_out_stride, _stream(stream)))
 
 
-def dbl_progressive_resize_stem(inp, n, h_in, w_in, c, out, h_out, w_out, taps, stride_w, pad_w, stream=None):
+def dbl_progressive_resize_stem(inp, n, h_in, w_in, c, out, h_out, w_out, taps, stride_w, pad_w, row_group=1,
+                                pad_h=0, rows_out=None, stream=None):
+    if rows_out is None:
+        rows_out = h_out
     _check(lib().dbl_progressive_resize_stem(_ptr(inp), n, h_in, w_in, c, _ptr(out), h_out, w_out, taps, stride_w, pad_w,
-                                             _stream(stream)))
+                                             row_group, pad_h, rows_out, _stream(stream)))
+
+
+def dbl_zero_f32_2d(base, rows, cols, ld, stream=None):
+    _check(lib().dbl_zero_f32_2d(_ptr(base), rows, cols, ld, _stream(stream)))
 
 
 def dbl_resize_taps(n_in, n_out):

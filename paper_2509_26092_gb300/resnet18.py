@@ -25,12 +25,15 @@ BasicBlocks (64/128/256/512 channels; the first block of stages 2-4 has
 stride 2 and a 1x1 stride-2 projection shortcut with BatchNorm), global
 average pooling and one fully connected layer.
 
-The stem runs on the tensor cores as an R x 1 convolution: the input
-preparation (``dbl_progressive_resize_stem``) writes the resized image unrolled
-along W, 8 filter columns x 8 channels (3 colour channels, zero-padded) per
-output column, so the stem weights are stored as [64][R][8][8] (filter columns
-and channels zero-padded) and the R x R stem equals an R x 1 convolution of
-64-channel rows with stride (stride, 1).
+The stem runs on the tensor cores as a convolution over an unrolled input
+(``StemLayout``): the input preparation (``dbl_progressive_resize_stem``)
+writes the resized image unrolled along W, 8 filter columns per output column,
+and, for the stride-2 ImageNet stem, also groups two input rows per unrolled
+row (8 columns x 4 channels each); the 3x3/1 CIFAR stem keeps one row of 8
+columns x 8 channels.  The R x R stem then equals a ceil(R/g) x 1 convolution
+of 64-channel rows (g = rows per unrolled row), with stride 1 along W, and
+the stem weights are stored as [64][g*ceil(R/g)][8][8/g] with the filter
+zero-padded in every direction.
 
 Convolutions read the bf16 weights ``w16``; BatchNorm and the fully connected
 layer read the fp32 master weights directly (they are tiny).
@@ -54,6 +57,29 @@ class ConvSpec:
     r: int
     stride: int
     pad: int
+
+
+@dataclass
+class StemLayout:
+    """How the stem's input is unrolled for the tensor cores (see dbl_progressive_resize_stem)."""
+    rg: int           # input rows per unrolled row: 2 for a stride-2 stem, else 1
+    taps: int         # filter rows of the unrolled convolution, ceil(R / rg)
+    pad_h: int        # zero rows the input preparation writes above the image
+    conv_stride: int  # stride of the unrolled convolution along H
+    conv_pad: int     # padding of the unrolled convolution along H
+
+    @classmethod
+    def of(cls, cs):
+        rg = 2 if cs.stride == 2 else 1
+        taps = -(-cs.r // rg)
+        return cls(rg, taps, cs.pad if rg == 2 else 0, cs.stride // rg, 0 if rg == 2 else cs.pad)
+
+    def rows(self, res, p):
+        """Unrolled rows for an image of res rows and p output rows."""
+        return p + self.taps - 1 if self.rg == 2 else res
+
+    def stored_shape(self, cs):
+        return (cs.cout, self.rg * self.taps, 8, 8 // self.rg)
 
 
 @dataclass
@@ -89,7 +115,8 @@ class ResNet18Spec:
             raise ValueError(variant)
         self.variant, self.classes, self.widths = variant, classes, tuple(widths)
         r, st, pad = (3, 1, 1) if variant == "cifar" else (7, 2, 3)
-        self.stem = ConvSpec("conv1", 64, 3, widths[0], r, st, pad)  # 64 = 8 unrolled columns x 8 channels
+        self.stem = ConvSpec("conv1", 64, 3, widths[0], r, st, pad)  # 64 = one unrolled row of 128 bytes
+        self.stem_layout = StemLayout.of(self.stem)
         self.blocks = []
         cin = widths[0]
         for li, wd in enumerate(widths):
@@ -107,8 +134,8 @@ class ResNet18Spec:
             off += (e.numel + ALIGN - 1) // ALIGN * ALIGN
 
         def conv(cs):
-            if cs is self.stem:  # stored [k][r][8 columns][8 channels], logical [k][r][r][3]
-                add(cs.name + ".w", (cs.cout, cs.r, 8, 8), (cs.cout, cs.r, cs.r, cs.cin_logical),
+            if cs is self.stem:  # stored [k][g*ceil(r/g)][8 columns][8/g channels], logical [k][r][r][3]
+                add(cs.name + ".w", self.stem_layout.stored_shape(cs), (cs.cout, cs.r, cs.r, cs.cin_logical),
                     cs.r * cs.r * cs.cin_logical)
                 return
             add(cs.name + ".w", (cs.cout, cs.r, cs.r, cs.cin), (cs.cout, cs.r, cs.r, cs.cin_logical),
@@ -205,8 +232,9 @@ class Worker:
         st = spec.stem
         p = conv_out(res, st.r, st.stride, st.pad)
         self.stem_hw = p
-        # stem input unrolled along W: [B, res, P, 8 columns x 8 channels]
-        self.x0 = torch.empty((B, res, p, 64), dtype=bf, device=dev)
+        # stem input unrolled (StemLayout): [B, rows, P, 64]
+        self.stem_rows = spec.stem_layout.rows(res, p)
+        self.x0 = torch.empty((B, self.stem_rows, p, 64), dtype=bf, device=dev)
         self.stem_y, self.stem_a, self.stem_da, self.stem_dy = act(p, st.cout), act(p, st.cout), None, act(p, st.cout)
         self.stem_stats = [vec(st.cout) for _ in range(4)]  # sum, sumsq, mean, invstd
         h = p
@@ -259,10 +287,25 @@ class Worker:
         return int(need) + 256
 
     def stem_shape(self):
-        """The stem as an R x 1 convolution of the W-unrolled input (stride along H only)."""
-        st = self.spec.stem
-        return D.conv_shape(self.batch, self.res, self.stem_hw, 64, st.cout, st.r, st.stride, st.pad, s=1, stride_w=1,
-                            pad_w=0)
+        """The stem as a ceil(R/g) x 1 convolution of the unrolled input (StemLayout)."""
+        st, lay = self.spec.stem, self.spec.stem_layout
+        return D.conv_shape(self.batch, self.stem_rows, self.stem_hw, 64, st.cout, lay.taps, lay.conv_stride,
+                            lay.conv_pad, s=1, stride_w=1, pad_w=0)
+
+    def stem_prepare(self, images, native_res, stream):
+        """Resize the native images to this worker's resolution, in the stem's unrolled layout."""
+        st, lay = self.spec.stem, self.spec.stem_layout
+        D.dbl_progressive_resize_stem(images, self.batch, native_res, native_res, 3, self.x0, self.res, self.res, st.r,
+                                      st.stride, st.pad, lay.rg, lay.pad_h, self.stem_rows, stream)
+
+    def stem_wgrad(self, dy, grad_w, ws, wsb, stream):
+        """Stem weight gradient into grad_w (stored layout); rows past the filter stay zero."""
+        st, lay = self.spec.stem, self.spec.stem_layout
+        D.dbl_conv_wgrad(self.stem_shape(), self.x0, dy, grad_w, False, ws, wsb, stream)
+        rows = lay.rg * lay.taps
+        if rows > st.r:  # padding rows of the row-grouped layout: not filter weights
+            k, per_row = grad_w.shape[0], grad_w[0, 0].numel()
+            D.dbl_zero_f32_2d(grad_w[:, st.r:].data_ptr(), k, (rows - st.r) * per_row, rows * per_row, stream)
 
     def layer_flops(self, name, s):
         """Algorithmic FLOPs of one pass of a conv layer: 2*M*N*K over the unpadded problem
@@ -300,8 +343,7 @@ class Worker:
             return spec.view(G, name)
 
         st = spec.stem
-        D.dbl_progressive_resize_stem(images, B, native_res, native_res, 3, self.x0, self.res, self.res, st.r,
-                                      st.stride, st.pad, s)
+        self.stem_prepare(images, native_res, s)
         # ---- forward
         shp = self.stem_shape()
         s_sum, s_sq, s_mean, s_istd = self.stem_stats
@@ -377,7 +419,7 @@ class Worker:
         else:
             D.dbl_bn_relu_fused_bwd(bns, dout, dout2, self.stem_y, self.stem_a, pv("bn1.g"), s_mean, s_istd,
                                     self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s)
-        D.dbl_conv_wgrad(shp, self.x0, self.stem_dy, gv("conv1.w"), False, ws, wsb, s)
+        self.stem_wgrad(self.stem_dy, gv("conv1.w"), ws, wsb, s)
 
 
 class DualBatchIteration:
@@ -398,21 +440,41 @@ class DualBatchIteration:
         self.stream_s = torch.cuda.Stream()
         self.images_l = self.images_s = None
         self.graph = None
+        self._inputs_ready = None  # copy-stream event the next run() waits for
+        self._consumed = None      # compute-stream event: the last run() has read its inputs
 
-    def set_inputs(self, images_l, labels_l, images_s=None, labels_s=None, non_blocking=False):
+    def set_inputs(self, images_l, labels_l, images_s=None, labels_s=None, non_blocking=False, stream=None):
         """fp32 images at the native resolution and int32 labels (device or pinned host
-        tensors), copied into the iteration's device buffers on the current stream."""
+        tensors), copied into the iteration's device buffers.  Without ``stream`` the
+        copies go on the current stream.  With a (copy) ``stream`` they are issued there
+        once the previous run() has consumed the buffers, and the next run() waits for
+        them, so that host-to-device copies overlap the compute of other iterations."""
         dev = self.server.w.device
-        if self.large is not None:
-            if self.images_l is None:
-                self.images_l = torch.empty(images_l.shape, dtype=torch.float32, device=dev)
-            self.images_l.copy_(images_l, non_blocking=non_blocking)
-            self.large.labels.copy_(labels_l, non_blocking=non_blocking)
-        if self.small is not None:
-            if self.images_s is None:
-                self.images_s = torch.empty(images_s.shape, dtype=torch.float32, device=dev)
-            self.images_s.copy_(images_s, non_blocking=non_blocking)
-            self.small.labels.copy_(labels_s, non_blocking=non_blocking)
+        cs = stream if stream is not None else torch.cuda.current_stream()
+        if stream is not None and self._consumed is not None:
+            stream.wait_event(self._consumed)
+        with torch.cuda.stream(cs):
+            if self.large is not None:
+                if self.images_l is None:
+                    self.images_l = torch.empty(images_l.shape, dtype=torch.float32, device=dev)
+                self.images_l.copy_(images_l, non_blocking=non_blocking)
+                self.large.labels.copy_(labels_l, non_blocking=non_blocking)
+            if self.small is not None:
+                if self.images_s is None:
+                    self.images_s = torch.empty(images_s.shape, dtype=torch.float32, device=dev)
+                self.images_s.copy_(images_s, non_blocking=non_blocking)
+                self.small.labels.copy_(labels_s, non_blocking=non_blocking)
+        if stream is not None:
+            self._inputs_ready = torch.cuda.Event()
+            self._inputs_ready.record(stream)
+
+    def losses_to_host(self, out):
+        """Queue the workers' losses (large, then small) into ``out`` (pinned host fp32)
+        on the current stream; read them after that stream has passed this point."""
+        workers = [w for w in (self.large, self.small) if w is not None]
+        for i, w in enumerate(workers):
+            out[i:i + 1].copy_(w.loss, non_blocking=True)
+        return len(workers)
 
     def _enqueue(self):
         cur = torch.cuda.current_stream()
@@ -431,10 +493,16 @@ class DualBatchIteration:
         cur.wait_stream(sL)
 
     def run(self):
+        cur = torch.cuda.current_stream()
+        if self._inputs_ready is not None:
+            cur.wait_event(self._inputs_ready)
+            self._inputs_ready = None
         if self.graph is not None:
             self.graph.replay()
         else:
             self._enqueue()
+        self._consumed = torch.cuda.Event()
+        self._consumed.record(cur)
 
     def capture(self):
         """Record one iteration (both workers, the join and the merge) as a CUDA graph."""

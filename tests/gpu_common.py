@@ -49,18 +49,27 @@ def check_status(D):
     assert D.dbl_device_status() == D.DBL_OK
 
 
-def stem_fold(x_u, r, stride, pad, width):
-    """Logical NHWC stem input [n, h, width, 8] from the W-unrolled tensor
-    [n, h, P, 8 taps, 8 channels] (x_u[..., q, t, :] is column q*stride + t - pad).
-    Checks that every copy of a column holds the same values."""
-    n, h, P = x_u.shape[0], x_u.shape[1], x_u.shape[2]
-    x_u = x_u.reshape(n, h, P, 8, 8)
-    out = np.full((n, h, width, 8), np.nan)
-    for q in range(P):
-        for t in range(r):
-            w = q * stride + t - pad
-            if 0 <= w < width:
-                if not np.all(np.isnan(out[:, :, w, :])):
-                    assert np.array_equal(out[:, :, w, :], x_u[:, :, q, t, :]), "unrolled copies disagree"
-                out[:, :, w, :] = x_u[:, :, q, t, :]
+def stem_fold(x_u, r, stride, pad, width, rg=1, pad_h=0, height=None):
+    """Logical NHWC stem input [n, height, width, 8/rg] from the unrolled tensor
+    [n, rows, P, rg rows, 8 taps, 8/rg channels]: x_u[:, m, q, e, t, :] is the pixel at
+    row rg*m + e - pad_h, column q*stride + t - pad.  Pixels no position covers stay NaN.
+    Checks that every copy of a pixel holds the same values."""
+    height = width if height is None else height
+    n, rows, P = x_u.shape[0], x_u.shape[1], x_u.shape[2]
+    cu = 8 // rg
+    x_u = x_u.reshape(n, rows, P, rg, 8, cu)
+    out = np.full((n, height, width, cu), np.nan)
+    for m in range(rows):
+        for e in range(rg):
+            y = rg * m + e - pad_h
+            if not 0 <= y < height:
+                continue
+            for q in range(P):
+                for t in range(r):
+                    x = q * stride + t - pad
+                    if 0 <= x < width:
+                        v = x_u[:, m, q, e, t, :]
+                        if not np.all(np.isnan(out[:, y, x, :])):
+                            assert np.array_equal(out[:, y, x, :], v), "unrolled copies disagree"
+                        out[:, y, x, :] = v
     return out

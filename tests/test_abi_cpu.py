@@ -100,8 +100,12 @@ def test_invalid_arguments_rejected_before_launch(D):
     assert L.dbl_conv_dgrad(ctypes.byref(s), 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
     # resize: upsampling
     assert L.dbl_progressive_resize(16, 0, 1, 8, 8, 3, 16, 1, 16, 16, 8, None) == D.DBL_ERR_UNSUPPORTED
-    assert L.dbl_progressive_resize_stem(16, 1, 8, 8, 3, 16, 16, 16, 7, 2, 3, None) == D.DBL_ERR_UNSUPPORTED
-    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 3, 16, 16, 16, 9, 2, 3, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 8, 8, 3, 16, 16, 16, 7, 2, 3, 1, 0, 16, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 3, 16, 16, 16, 9, 2, 3, 1, 0, 16, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 3, 16, 16, 16, 7, 2, 3, 3, 3, 11, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 5, 16, 16, 16, 7, 2, 3, 2, 3, 11, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_progressive_resize_stem(16, 1, 16, 16, 3, 16, 16, 16, 7, 2, 3, 2, 3, 0, None) == D.DBL_ERR_INVALID
+    assert L.dbl_zero_f32_2d(16, 4, 8, 4, None) == D.DBL_ERR_INVALID
     # BN: channel count that is not a multiple of 8
     b = D.BnShape(100, 12, 1e-5, 1)
     assert L.dbl_bn_relu_fused(ctypes.byref(b), 16, 16, 16, 16, 16, None, 16, 16, 16, None) == D.DBL_ERR_UNSUPPORTED

@@ -74,25 +74,36 @@ def test_resize_matches_oracle(D, n, hin, hout):
     assert max_norm_rel(host(out32), ref) <= 1e-6
 
 
+def _stem_layout(r, st, pad):
+    from paper_2509_26092_gb300.resnet18 import ConvSpec, StemLayout
+    return StemLayout.of(ConvSpec("conv1", 64, 3, 64, r, st, pad))
+
+
 @pytest.mark.parametrize("n,hin,hout,r,st,pad", [(2, 224, 160, 7, 2, 3), (3, 32, 24, 3, 1, 1), (2, 224, 224, 7, 2, 3),
                                                  (1, 20, 13, 7, 2, 3)])
 def test_resize_stem_unrolls_the_resized_image(D, n, hin, hout, r, st, pad):
+    lay = _stem_layout(r, st, pad)
     x = rng(hin + hout + r).standard_normal((n, hin, hin, 3)).astype(np.float32)
     ref = orc.bilinear_resize(x, hout, hout)
     P = (hout + 2 * pad - r) // st + 1
-    out = torch.full((n, hout, P, 64), 7.0, dtype=torch.bfloat16, device="cuda")
-    D.dbl_progressive_resize_stem(to_f32_dev(x), n, hin, hin, 3, out, hout, hout, r, st, pad)
-    xu = host(out).reshape(n, hout, P, 8, 8)
+    rows = lay.rows(hout, P)
+    out = torch.full((n, rows, P, 64), 7.0, dtype=torch.bfloat16, device="cuda")
+    D.dbl_progressive_resize_stem(to_f32_dev(x), n, hin, hin, 3, out, hout, hout, r, st, pad, lay.rg, lay.pad_h, rows)
+    xu = host(out).reshape(n, rows, P, lay.rg, 8, 8 // lay.rg)
     assert np.all(xu[..., r:, :] == 0.0)      # taps past the filter width
     assert np.all(xu[..., 3:] == 0.0)         # padded colour channels
     for q in range(P):                        # columns outside the image
         for t in range(r):
             if not 0 <= q * st + t - pad < hout:
-                assert np.all(xu[:, :, q, t, :] == 0.0)
-    got = stem_fold(xu, r, st, pad, hout)[..., :3]
-    covered = ~np.isnan(got[0, 0, :, 0])
+                assert np.all(xu[:, :, q, :, t, :] == 0.0)
+    for m in range(rows):                     # rows outside the image
+        for e in range(lay.rg):
+            if not 0 <= lay.rg * m + e - lay.pad_h < hout:
+                assert np.all(xu[:, m, :, e] == 0.0)
+    got = stem_fold(xu, r, st, pad, hout, lay.rg, lay.pad_h)[..., :3]
+    covered = ~np.isnan(got[0, :, :, 0])
     ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
-    assert np.all(np.abs(got[:, :, covered] - ref[:, :, covered]) <= ulp[:, :, covered] + 1e-30)
+    assert np.all(np.abs(got[:, covered] - ref[:, covered]) <= ulp[:, covered] + 1e-30)
     check_status(D)
 
 
@@ -103,23 +114,26 @@ STEM_CASES = [  # n, h (square input), r, stride, pad
 ]
 
 
-def _stem_inputs(n, h, r, seed):
+def _stem_inputs(n, h, r, seed, lay):
     g = rng(seed)
     x = bf16_values(g.standard_normal((n, h, h, 3)))
     wt = bf16_values(g.standard_normal((64, r, r, 3)) * np.sqrt(2.0 / (r * r * 3)))
-    w_store = np.zeros((64, r, 8, 8))
-    w_store[:, :, :r, :3] = wt
+    w_store = np.zeros((64, lay.rg * lay.taps, 8, 8 // lay.rg))
+    w_store[:, :r, :r, :3] = wt
     return x, wt, w_store
 
 
 @pytest.mark.parametrize("case", STEM_CASES)
 def test_unrolled_stem_fwd_and_wgrad_match_oracle(D, case):
     n, h, r, st, pad = case
-    x, wt, w_store = _stem_inputs(n, h, r, 21)
+    lay = _stem_layout(r, st, pad)
+    x, wt, w_store = _stem_inputs(n, h, r, 21, lay)
     P = (h + 2 * pad - r) // st + 1
-    xu = torch.empty((n, h, P, 64), dtype=torch.bfloat16, device="cuda")
-    D.dbl_progressive_resize_stem(to_f32_dev(x), n, h, h, 3, xu, h, h, r, st, pad)  # same size: exact copy
-    shape = D.conv_shape(n, h, P, 64, 64, r, st, pad, s=1, stride_w=1, pad_w=0)
+    rows = lay.rows(h, P)
+    xu = torch.empty((n, rows, P, 64), dtype=torch.bfloat16, device="cuda")
+    D.dbl_progressive_resize_stem(to_f32_dev(x), n, h, h, 3, xu, h, h, r, st, pad, lay.rg, lay.pad_h,
+                                  rows)  # same size: exact copy
+    shape = D.conv_shape(n, rows, P, 64, 64, lay.taps, lay.conv_stride, lay.conv_pad, s=1, stride_w=1, pad_w=0)
     y = torch.full((n, P, P, 64), float("nan"), dtype=torch.bfloat16, device="cuda")
     s1, s2 = torch.empty(64, device="cuda"), torch.empty(64, device="cuda")
     wsb = max(D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_FWD), D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_WGRAD))
@@ -127,12 +141,17 @@ def test_unrolled_stem_fwd_and_wgrad_match_oracle(D, case):
     ref = orc.conv2d_fwd(x, wt, st, pad)
     assert max_norm_rel(host(y), ref) <= CONV_TOL
     dy = bf16_values(rng(22).standard_normal((n, P, P, 64)))
-    dw = torch.full((64, r, 8, 8), float("nan"), device="cuda")
+    dw = torch.full(w_store.shape, float("nan"), device="cuda")
     D.dbl_conv_wgrad(shape, xu, to_bf16_dev(dy), dw, False, ws(wsb), wsb)
+    rows_w = lay.rg * lay.taps
+    if rows_w > r:  # the padding rows of the row-grouped layout: zeroed as the worker does
+        per = 8 * (8 // lay.rg)
+        D.dbl_zero_f32_2d(dw[:, r:].data_ptr(), 64, (rows_w - r) * per, rows_w * per)
     got = host(dw)
     assert np.all(got[:, :, r:, :] == 0.0) and np.all(got[..., 3:] == 0.0)  # padding gets no gradient
+    assert np.all(got[:, r:] == 0.0)
     rdw = orc.conv2d_wgrad(x, dy, wt.shape, st, pad)
-    assert max_norm_rel(got[:, :, :r, :3], rdw) <= CONV_TOL
+    assert max_norm_rel(got[:, :r, :r, :3], rdw) <= CONV_TOL
     check_status(D)
 
 

@@ -141,3 +141,29 @@ def test_graph_replay_equals_eager(R):
         outs.append(server.w.clone())
     # deterministic kernels: replay and eager launches give identical bits
     assert torch.equal(outs[0], outs[1])
+
+
+def test_inputs_on_a_copy_stream_give_the_same_iteration(R):
+    """Host inputs copied on a separate stream (overlapping other iterations' compute)
+    reach the same model as copies on the compute stream, bit for bit."""
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=9)
+    img = torch.from_numpy(synth.images(12, 32, 32, 3, seed=9)).pin_memory()
+    lab = torch.from_numpy(synth.labels(12, 100, seed=9)).pin_memory()
+    outs = []
+    for use_copy_stream in (False, True):
+        server = R.ServerState(spec, params)
+        its = [R.DualBatchIteration(server, R.Worker(spec, 8, res), R.Worker(spec, 4, res), 32) for res in (24, 32)]
+        copy = torch.cuda.Stream() if use_copy_stream else None
+        losses = torch.zeros(8, dtype=torch.float32).pin_memory()
+        for step in range(2):
+            for it in its:  # all copies first: with a copy stream they wait only for their buffer's last reader
+                it.set_inputs(img[4:], lab[4:], img[:4], lab[:4], non_blocking=True, stream=copy)
+            n = 0
+            for it in its:
+                it.run()
+                n += it.losses_to_host(losses[n:])
+        torch.cuda.synchronize()
+        outs.append((server.w.clone(), losses.clone()))
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert torch.equal(outs[0][1], outs[1][1]) and bool(torch.all(outs[0][1][:4] > 0))  # 2 iterations x 2 workers

@@ -50,9 +50,10 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
     eps = wk.eps
     # ---------------- forward
     st = spec.stem
-    x0 = stem_fold(h(wk.x0), st.r, st.stride, st.pad, res)[..., :3]  # the logical stem input
+    lay = spec.stem_layout
+    x0 = stem_fold(h(wk.x0), st.r, st.stride, st.pad, res, lay.rg, lay.pad_h)[..., :3]  # the logical stem input
     assert not np.any(np.isnan(x0))
-    w_stem = W16["conv1.w"][:, :, :st.r, :3]
+    w_stem = W16["conv1.w"][:, :st.r, :st.r, :3]
     chk("stem.conv", h(wk.stem_y), orc.conv2d_fwd(x0, w_stem, st.stride, st.pad))
     o, m, s = orc.bn_fwd(h(wk.stem_y), P["bn1.g"], P["bn1.b"], eps, relu=True)
     chk("stem.bn", h(wk.stem_a), o)
@@ -133,7 +134,8 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
                                       dout2=dout2)
     chk("stem.bn.bwd", h(wk.stem_dy), dys)
     wst = orc.conv2d_wgrad(x0, h(wk.stem_dy), w_stem.shape, st.stride, st.pad)
-    chk("stem.wgrad", G["conv1.w"][:, :, :st.r, :3], wst)
+    chk("stem.wgrad", G["conv1.w"][:, :st.r, :st.r, :3], wst)
+    assert np.all(G["conv1.w"][:, st.r:] == 0.0)  # rows of the stored layout past the filter
     # padded filter columns and input channels get no gradient
     assert np.all(G["conv1.w"][:, :, st.r:, :] == 0.0) and np.all(G["conv1.w"][..., 3:] == 0.0)
     worst = sorted(errs.items(), key=lambda kv: -kv[1])[:6]
