@@ -155,11 +155,16 @@ DBL_API size_t dbl_bn_workspace_bytes(const dbl_bn_shape* shape);
  *   dy = gamma*invstd*(g - dbeta/count - xhat*dgamma/count),
  * and, if dresidual is non-NULL, dresidual = g (the residual branch's
  * gradient).  dy, dresidual: bf16 [count, c]; dgamma, dbeta: fp32 [c]
- * (overwritten).  The channel sums are reduced in a fixed order. */
+ * (overwritten).  The channel sums are reduced in a fixed order.
+ * out_bf16 may be NULL (with shape->relu set) when the forward pass had no
+ * residual: the mask is then recomputed from y exactly as dbl_bn_relu_fused
+ * decided it, [y*scale + shift > 0] with scale = gamma*invstd and shift =
+ * beta - mean*scale, which needs beta (otherwise beta may be NULL). */
 DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf16, const void* dout2_bf16 /* or NULL */,
-                          const void* y_bf16, const void* out_bf16, const float* gamma, const float* save_mean,
-                          const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
-                          float* dgamma, float* dbeta, void* ws, size_t ws_bytes, void* stream);
+                          const void* y_bf16, const void* out_bf16 /* or NULL */, const float* gamma,
+                          const float* beta /* or NULL */, const float* save_mean, const float* save_invstd,
+                          void* dy_bf16, void* dresidual_bf16 /* or NULL */, float* dgamma, float* dbeta, void* ws,
+                          size_t ws_bytes, void* stream);
 
 /* Same computation as dbl_bn_relu_fused_bwd, for callers that cannot hand
  * the library a workspace: their memory comes from an allocator they do not
@@ -181,7 +186,7 @@ DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf
 #define DBL_BN_NOALLOC_MAX_C 512
 DBL_API int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* shape, const void* dout_bf16,
                                           const void* dout2_bf16 /* or NULL */, const void* y_bf16,
-                                          const void* out_bf16, const float* gamma, const float* save_mean,
+                                          const void* out_bf16, const float* gamma, const float* beta, const float* save_mean,
                                           const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
                                           float* dgamma, float* dbeta, void* stream);
 

@@ -85,42 +85,49 @@ __global__ void __launch_bounds__(kThreads) bn_stats_kernel(const __nv_bfloat16*
 }
 
 // ----------------------------------------------------------------------------- forward apply
+// Batch statistics -> saved mean and 1/std, once per channel (fp64: the
+// variance is E[y^2] - E[y]^2 of sums over up to 10^8 rows).
+__global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const float* __restrict__ sum,
+                                       const float* __restrict__ sumsq, float* __restrict__ save_mean,
+                                       float* __restrict__ save_invstd)
+{
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    const double inv_n = 1.0 / (double)count;
+    const double mean = (double)sum[c] * inv_n;
+    double var = (double)sumsq[c] * inv_n - mean * mean;
+    if (var < 0.0) var = 0.0;
+    save_mean[c] = (float)mean;
+    save_invstd[c] = (float)(1.0 / sqrt(var + (double)eps));
+}
+
+// Per-channel scale and shift of out = y*scale + shift from the saved
+// statistics, in fp32 with explicit rounding (no contraction), so that every
+// CTA and the backward pass's ReLU-mask recomputation get the same bits.
+__device__ __forceinline__ void bn_scale_shift(float gamma, float beta, float mean, float invstd, float& scale,
+                                               float& shift)
+{
+    scale = __fmul_rn(gamma, invstd);
+    shift = __fsub_rn(beta, __fmul_rn(mean, scale));
+}
+
 // Thread t of a CTA owns channel group g = t % (C/8) (8 channels, one 16-byte
 // vector) and visits rows t / (C/8), + rows-per-CTA-step, ...; a warp covers
 // consecutive vectors of consecutive rows, so every access is coalesced, and the
 // channel's scale and shift stay in registers.
 __global__ void __launch_bounds__(kThreads, kBlocksPerSM)
     bn_apply_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ res,
-                    __nv_bfloat16* __restrict__ out, int count, int C, float eps, int relu,
-                    const float* __restrict__ sum, const float* __restrict__ sumsq, const float* __restrict__ gamma,
-                    const float* __restrict__ beta, float* __restrict__ save_mean, float* __restrict__ save_invstd)
+                    __nv_bfloat16* __restrict__ out, int count, int C, int relu, const float* __restrict__ gamma,
+                    const float* __restrict__ beta, const float* __restrict__ mean, const float* __restrict__ invstd)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
-    // statistics -> per-channel scale and shift, once per CTA (fp64 is slow on this GPU:
-    // one thread per channel, not one per thread and channel)
-    __shared__ float s_sc[kMaxC], s_sh[kMaxC];
-    const double inv_n = 1.0 / (double)count;
-    for (int c = threadIdx.x; c < C; c += kThreads) {
-        const double mean = (double)sum[c] * inv_n;
-        double var = (double)sumsq[c] * inv_n - mean * mean;
-        if (var < 0.0) var = 0.0;
-        const float invstd = (float)(1.0 / sqrt(var + (double)eps));
-        const float scale = gamma[c] * invstd;
-        s_sc[c] = scale;
-        s_sh[c] = beta[c] - (float)mean * scale;
-        if (blockIdx.x == 0) {
-            save_mean[c] = (float)mean;
-            save_invstd[c] = invstd;
-        }
-    }
-    __syncthreads();
     float sc[8], sh[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-        sc[k] = s_sc[8 * g + k];
-        sh[k] = s_sh[8 * g + k];
+        const int c = 8 * g + k;
+        bn_scale_shift(gamma[c], beta[c], mean[c], invstd[c], sc[k], sh[k]);
     }
     const int step = gridDim.x * rstep;
     auto emit = [&](const uint4& yv, const uint4& rv, int v) {
@@ -129,7 +136,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSM)
         unpack8(rv, rr);
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            const float o = fmaf(f[k], sc[k], sh[k]) + rr[k];
+            const float o = __fadd_rn(__fmaf_rn(f[k], sc[k], sh[k]), rr[k]);
             f[k] = (relu && !(o > 0.f)) ? 0.f : o;
         }
         reinterpret_cast<uint4*>(out)[v] = pack8(f);
@@ -155,23 +162,46 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSM)
 }
 
 // ----------------------------------------------------------------------------- backward
+// Where the ReLU mask comes from: none (no ReLU), the stored output (out > 0),
+// or, when there is no stored output (a BatchNorm without a residual), y,
+// recomputed exactly as the forward pass decided it: y*scale + shift > 0 with
+// the same fp32 operations.
+enum MaskMode : int { kMaskNone = 0, kMaskOut = 1, kMaskY = 2 };
+
 // The raw 16-byte vectors behind one 8-channel group of g = (dout [+ dout2]) * [out > 0]
 // and of the BatchNorm input y; loaded together so that several rows' loads are in flight.
 struct Vec8 {
     uint4 d, d2, o, y;
 };
 
+template <int MASK>
 __device__ __forceinline__ void load_g_raw(const __nv_bfloat16* dout, const __nv_bfloat16* dout2,
-                                           const __nv_bfloat16* out, int relu, const __nv_bfloat16* y, int v,
-                                           Vec8& g, Vec8& yv)
+                                           const __nv_bfloat16* out, const __nv_bfloat16* y, int v, Vec8& g, Vec8& yv)
 {
     g.d = __ldcs(reinterpret_cast<const uint4*>(dout) + v);
     g.d2 = dout2 ? __ldcs(reinterpret_cast<const uint4*>(dout2) + v) : make_uint4(0, 0, 0, 0);
-    g.o = relu ? __ldcs(reinterpret_cast<const uint4*>(out) + v) : make_uint4(0, 0, 0, 0);
+    g.o = MASK == kMaskOut ? __ldcs(reinterpret_cast<const uint4*>(out) + v) : make_uint4(0, 0, 0, 0);
     yv.y = __ldcs(reinterpret_cast<const uint4*>(y) + v);
 }
 
-__device__ __forceinline__ void combine_g(const Vec8& raw, bool two, int relu, float (&g)[8])
+template <int MASK>
+struct ReluMask {
+    float sc[MASK == kMaskY ? 8 : 1], sh[MASK == kMaskY ? 8 : 1];
+
+    __device__ __forceinline__ void init(const float* gamma, const float* beta, const float* mean, const float* invstd,
+                                         int g)
+    {
+        if constexpr (MASK == kMaskY) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                bn_scale_shift(gamma[8 * g + k], beta[8 * g + k], mean[8 * g + k], invstd[8 * g + k], sc[k], sh[k]);
+        }
+    }
+};
+
+template <int MASK>
+__device__ __forceinline__ void combine_g(const Vec8& raw, const float (&y)[8], bool two, const ReluMask<MASK>& m,
+                                          float (&g)[8])
 {
     unpack8(raw.d, g);
     if (two) {
@@ -180,7 +210,11 @@ __device__ __forceinline__ void combine_g(const Vec8& raw, bool two, int relu, f
 #pragma unroll
         for (int k = 0; k < 8; ++k) g[k] += h[k];
     }
-    if (relu) {
+    if constexpr (MASK == kMaskY) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (!(__fmaf_rn(y[k], m.sc[k], m.sh[k]) > 0.f)) g[k] = 0.f;
+    } else if constexpr (MASK == kMaskOut) {
         float o[8];
         unpack8(raw.o, o);
 #pragma unroll
@@ -190,12 +224,13 @@ __device__ __forceinline__ void combine_g(const Vec8& raw, bool two, int relu, f
 }
 
 // sg += g, sgc += g*(y - mean)  (the 1/std factor is applied once per partial)
-__device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw, bool two, int relu,
+template <int MASK>
+__device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw, bool two, const ReluMask<MASK>& relu,
                                              const float (&mu)[8], float (&sg)[8], float (&sgc)[8])
 {
     float gg[8], yy[8];
-    combine_g(graw, two, relu, gg);
     unpack8(yraw.y, yy);
+    combine_g(graw, yy, two, relu, gg);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         sg[k] += gg[k];
@@ -206,15 +241,19 @@ __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw,
 // Partial blk reduces a contiguous range of rows into partial[blk][0..C) (sum g)
 // and partial[blk][C..2C) (sum g*xhat); CTA b computes partials b, b + gridDim.x, ...
 // (each in a fixed order, so the result does not depend on the grid).
+template <int MASK>
 __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
                          const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
-                         int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
-                         int rows_per_blk, int nblk, float* __restrict__ partial)
+                         int C, const float* __restrict__ gamma, const float* __restrict__ beta,
+                         const float* __restrict__ mean, const float* __restrict__ invstd, int rows_per_blk, int nblk,
+                         float* __restrict__ partial)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
+    ReluMask<MASK> rm;
+    rm.init(gamma, beta, mean, invstd, g);
     float mu[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) mu[k] = mean[8 * g + k];
@@ -228,14 +267,14 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     for (; r + (kUnroll - 1) * rstep < r1; r += kUnroll * rstep) {
         Vec8 gg[kUnroll], yy[kUnroll];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) load_g_raw(dout, dout2, out, relu, y, (r + u * rstep) * groups + g, gg[u], yy[u]);
+        for (int u = 0; u < kUnroll; ++u) load_g_raw<MASK>(dout, dout2, out, y, (r + u * rstep) * groups + g, gg[u], yy[u]);
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) accumulate_g(gg[u], yy[u], dout2 != nullptr, relu, mu, sg, sgx);
+        for (int u = 0; u < kUnroll; ++u) accumulate_g(gg[u], yy[u], dout2 != nullptr, rm, mu, sg, sgx);
     }
     for (; r < r1; r += rstep) {
         Vec8 gg, yy;
-        load_g_raw(dout, dout2, out, relu, y, r * groups + g, gg, yy);
-        accumulate_g(gg, yy, dout2 != nullptr, relu, mu, sg, sgx);
+        load_g_raw<MASK>(dout, dout2, out, y, r * groups + g, gg, yy);
+        accumulate_g(gg, yy, dout2 != nullptr, rm, mu, sg, sgx);
     }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -287,15 +326,19 @@ __global__ void __launch_bounds__(32 * kColsumGroups) bn_bwd_finalize_kernel(
     coef[2 * C + c] = (float)(-k1 * (sg / (double)count) - b * (double)mean[c]);
 }
 
+template <int MASK>
 __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     bn_bwd_apply_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
                         const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
-                        int C, int relu, const float* __restrict__ mean, const float* __restrict__ invstd,
+                        int C, const float* __restrict__ gamma, const float* __restrict__ beta,
+                        const float* __restrict__ mean, const float* __restrict__ invstd,
                         const float* __restrict__ coef, __nv_bfloat16* __restrict__ dy, __nv_bfloat16* __restrict__ dres)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
+    ReluMask<MASK> rm;
+    rm.init(gamma, beta, mean, invstd, g);
     float ca[8], cb[8], cc[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -307,8 +350,8 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     const int step = gridDim.x * rstep;
     auto emit = [&](const Vec8& graw, const Vec8& yraw, int v) {
         float gg[8], yy[8], d[8];
-        combine_g(graw, dout2 != nullptr, relu, gg);
         unpack8(yraw.y, yy);
+        combine_g(graw, yy, dout2 != nullptr, rm, gg);
 #pragma unroll
         for (int k = 0; k < 8; ++k) d[k] = fmaf(ca[k], gg[k], fmaf(cb[k], yy[k], cc[k]));
         __stcs(reinterpret_cast<uint4*>(dy) + v, pack8(d));
@@ -318,13 +361,13 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     for (; r + (kUnroll - 1) * step < count; r += kUnroll * step) {
         Vec8 gg[kUnroll], yy[kUnroll];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) load_g_raw(dout, dout2, out, relu, y, (r + u * step) * groups + g, gg[u], yy[u]);
+        for (int u = 0; u < kUnroll; ++u) load_g_raw<MASK>(dout, dout2, out, y, (r + u * step) * groups + g, gg[u], yy[u]);
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) emit(gg[u], yy[u], (r + u * step) * groups + g);
     }
     for (; r < count; r += step) {
         Vec8 gg, yy;
-        load_g_raw(dout, dout2, out, relu, y, r * groups + g, gg, yy);
+        load_g_raw<MASK>(dout, dout2, out, y, r * groups + g, gg, yy);
         emit(gg, yy, r * groups + g);
     }
 }
@@ -366,6 +409,45 @@ int64_t bwd_blocks(int64_t count, int C)
     return b < 1 ? 1 : b > 512 ? 512 : b;
 }
 
+template <int MASK>
+int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
+                    const float* gamma, const float* beta, const float* mean, const float* invstd, void* dy,
+                    void* dresidual, float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk, int rows,
+                    cudaStream_t st)
+{
+    using namespace dbl;
+    const int C = s->c;
+    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
+    bn_bwd_reduce_kernel<MASK><<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y),
+                                                                       (int)s->count, C, gamma, beta, mean, invstd,
+                                                                       rows, (int)nblk, partial);
+    int rc = launch_check("bn_bwd_reduce launch");
+    if (rc) return rc;
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
+                                                                         invstd, dgamma, dbeta, coef);
+    if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
+    bn_bwd_apply_kernel<MASK><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
+        bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
+        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
+    return launch_check("bn_bwd_apply launch");
+}
+
+// The three passes of the backward pass (reduce, fixed-order finalize, apply),
+// with the ReLU mask taken from out, recomputed from y (out == NULL), or none.
+int bwd_launch(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
+               const float* gamma, const float* beta, const float* mean, const float* invstd, void* dy, void* dresidual,
+               float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk, int rows, cudaStream_t st)
+{
+    if (!s->relu)
+        return bwd_launch_mask<kMaskNone>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma,
+                                          dbeta, partial, coef, nblk, rows, st);
+    if (out)
+        return bwd_launch_mask<kMaskOut>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma,
+                                         dbeta, partial, coef, nblk, rows, st);
+    return bwd_launch_mask<kMaskY>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma, dbeta,
+                                   partial, coef, nblk, rows, st);
+}
+
 }  // namespace
 
 extern "C" {
@@ -397,10 +479,13 @@ int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum,
     if (!aligned16(y) || !aligned16(out) || (residual && !aligned16(residual)))
         return set_error(DBL_ERR_INVALID, "bn_relu_fused: tensors must be 16-byte aligned");
     if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused: empty batch has no statistics");
-    bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, as_stream(stream)>>>(
+    cudaStream_t st = as_stream(stream);
+    bn_fwd_finalize_kernel<<<(s->c + 127) / 128, 128, 0, st>>>(s->count, s->c, s->eps, ch_sum, ch_sumsq, save_mean,
+                                                             save_invstd);
+    if ((rc = launch_check("bn_fwd_finalize launch"))) return rc;
+    bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
         static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
-        static_cast<__nv_bfloat16*>(out), s->count, s->c, s->eps, s->relu, ch_sum, ch_sumsq, gamma, beta, save_mean,
-        save_invstd);
+        static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
     return launch_check("bn_relu_fused launch");
 }
 
@@ -411,13 +496,13 @@ size_t dbl_bn_workspace_bytes(const dbl_bn_shape* s)
 }
 
 int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
-                          const float* gamma, const float* save_mean, const float* save_invstd, void* dy,
+                          const float* gamma, const float* beta, const float* save_mean, const float* save_invstd, void* dy,
                           void* dresidual, float* dgamma, float* dbeta, void* ws, size_t ws_bytes, void* stream)
 {
     using namespace dbl;
     int rc = check_shape(s, "bn_relu_fused_bwd");
     if (rc) return rc;
-    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out))
+    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out && !beta))
         return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd: null pointer");
     if (!aligned16(dout) || !aligned16(y) || !aligned16(dy) || (dout2 && !aligned16(dout2)) ||
         (out && !aligned16(out)) || (dresidual && !aligned16(dresidual)))
@@ -432,18 +517,8 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
     float* partial = static_cast<float*>(ws);
     float* coef = partial + nblk * 2 * C;
     cudaStream_t st = as_stream(stream);
-    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
-    bn_bwd_reduce_kernel<<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C,
-                                                                 s->relu, save_mean, save_invstd, rows, (int)nblk,
-                                                                 partial);
-    if ((rc = launch_check("bn_bwd_reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma,
-                                                                         save_mean, save_invstd, dgamma, dbeta, coef);
-    if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
-    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
-        bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
-        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
-    return launch_check("bn_bwd_apply launch");
+    return bwd_launch(s, dout, dout2, y, out, gamma, beta, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
+                      partial, coef, nblk, rows, st);
 }
 
 }  // extern "C"
@@ -487,7 +562,7 @@ float* noalloc_scratch(int* rc)
 }  // namespace
 
 extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* dout, const void* dout2,
-                                              const void* y, const void* out, const float* gamma,
+                                              const void* y, const void* out, const float* gamma, const float* beta,
                                               const float* save_mean, const float* save_invstd, void* dy,
                                               void* dresidual, float* dgamma, float* dbeta, void* stream)
 {
@@ -498,7 +573,7 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
         return set_error(DBL_ERR_UNSUPPORTED,
                          "bn_relu_fused_bwd_noalloc: %d channels exceed the static scratch limit of %d", s->c,
                          DBL_BN_NOALLOC_MAX_C);
-    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out))
+    if (!dout || !y || !dy || !gamma || !save_mean || !save_invstd || !dgamma || !dbeta || (s->relu && !out && !beta))
         return set_error(DBL_ERR_INVALID, "bn_relu_fused_bwd_noalloc: null pointer");
     if (!aligned16(dout) || !aligned16(y) || !aligned16(dy) || (dout2 && !aligned16(dout2)) ||
         (out && !aligned16(out)) || (dresidual && !aligned16(dresidual)))
@@ -513,16 +588,6 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
     float* coef = partial + nblk * 2 * C;  // written by the finalize kernel before the apply kernel reads it
     const int rows = (int)((s->count + nblk - 1) / nblk);
     cudaStream_t st = as_stream(stream);
-    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
-    bn_bwd_reduce_kernel<<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y), s->count, C,
-                                                                 s->relu, save_mean, save_invstd, rows, (int)nblk,
-                                                                 partial);
-    if ((rc = launch_check("bn_bwd_noalloc reduce launch"))) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma,
-                                                                         save_mean, save_invstd, dgamma, dbeta, coef);
-    if ((rc = launch_check("bn_bwd_noalloc finalize launch"))) return rc;
-    bn_bwd_apply_kernel<<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
-        bd(dout), bd(dout2), bd(out), bd(y), s->count, C, s->relu, save_mean, save_invstd, coef,
-        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
-    return launch_check("bn_bwd_noalloc apply launch");
+    return bwd_launch(s, dout, dout2, y, out, gamma, beta, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
+                      partial, coef, nblk, rows, st);
 }

@@ -68,8 +68,8 @@ def lib():
             "dbl_bn_stats": (ctypes.c_int, [ctypes.POINTER(BnShape), _V, _V, _V, _V]),
             "dbl_bn_relu_fused": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 10),
             "dbl_bn_workspace_bytes": (_SZ, [ctypes.POINTER(BnShape)]),
-            "dbl_bn_relu_fused_bwd": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 12 + [_SZ, _V]),
-            "dbl_bn_relu_fused_bwd_noalloc": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 12),
+            "dbl_bn_relu_fused_bwd": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 13 + [_SZ, _V]),
+            "dbl_bn_relu_fused_bwd_noalloc": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 13),
             "dbl_maxpool_fwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V]),
             "dbl_maxpool_bwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V, _V]),
             "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
@@ -177,18 +177,19 @@ def dbl_bn_workspace_bytes(shape):
 
 
 def dbl_bn_relu_fused_bwd(shape, dout, dout2, y, out, gamma, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
-                          ws, ws_bytes, stream=None):
+                          ws, ws_bytes, stream=None, beta=None):
+    """out=None with shape.relu: the ReLU mask is recomputed from y (needs beta)."""
     _check(lib().dbl_bn_relu_fused_bwd(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out), _ptr(gamma),
-                                       _ptr(save_mean), _ptr(save_invstd), _ptr(dy), _ptr(dresidual), _ptr(dgamma),
-                                       _ptr(dbeta), _ptr(ws), ws_bytes, _stream(stream)))
+                                       _ptr(beta), _ptr(save_mean), _ptr(save_invstd), _ptr(dy), _ptr(dresidual),
+                                       _ptr(dgamma), _ptr(dbeta), _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def dbl_bn_relu_fused_bwd_noalloc(shape, dout, dout2, y, out, gamma, save_mean, save_invstd, dy, dresidual, dgamma,
-                                  dbeta, stream=None):
+                                  dbeta, stream=None, beta=None):
     """dbl_bn_relu_fused_bwd without a workspace argument: the scratch is a fixed array inside
     the library (channels <= 512; calls must not overlap on the GPU)."""
     _check(lib().dbl_bn_relu_fused_bwd_noalloc(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out),
-                                               _ptr(gamma), _ptr(save_mean), _ptr(save_invstd), _ptr(dy),
+                                               _ptr(gamma), _ptr(beta), _ptr(save_mean), _ptr(save_invstd), _ptr(dy),
                                                _ptr(dresidual), _ptr(dgamma), _ptr(dbeta), _stream(stream)))
 
 

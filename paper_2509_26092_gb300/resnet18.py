@@ -396,9 +396,10 @@ class Worker:
             s2 = D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)
             D.dbl_conv_wgrad(s2, d["o1"], d["dh2"], gv(b.pre + ".conv2.w"), False, ws, wsb, s)
             D.dbl_conv_dgrad(s2, d["dh2"], wv(b.pre + ".conv2.w"), d["do1"], None, 0, s)
-            D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), d["do1"], None, d["h1"], d["o1"],
+            # bn1 has no residual: its ReLU mask is recomputed from h1 (o1 is not read again)
+            D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), d["do1"], None, d["h1"], None,
                                     pv(b.pre + ".bn1.g"), st1[2], st1[3], d["dh1"], None, gv(b.pre + ".bn1.g"),
-                                    gv(b.pre + ".bn1.b"), ws, wsb, s)
+                                    gv(b.pre + ".bn1.b"), ws, wsb, s, beta=pv(b.pre + ".bn1.b"))
             s1 = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)
             D.dbl_conv_wgrad(s1, d["x"], d["dh1"], gv(b.pre + ".conv1.w"), False, ws, wsb, s)
             D.dbl_conv_dgrad(s1, d["dh1"], wv(b.pre + ".conv1.w"), d["din"], None, 0, s)
@@ -414,11 +415,11 @@ class Worker:
         bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)
         if spec.variant == "imagenet":
             D.dbl_maxpool_bwd(B, self.stem_hw, self.stem_hw, st.cout, dout, dout2, self.pool_arg, self.stem_da, s)
-            D.dbl_bn_relu_fused_bwd(bns, self.stem_da, None, self.stem_y, self.stem_a, pv("bn1.g"), s_mean, s_istd,
-                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s)
+            D.dbl_bn_relu_fused_bwd(bns, self.stem_da, None, self.stem_y, None, pv("bn1.g"), s_mean, s_istd,
+                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s, beta=pv("bn1.b"))
         else:
-            D.dbl_bn_relu_fused_bwd(bns, dout, dout2, self.stem_y, self.stem_a, pv("bn1.g"), s_mean, s_istd,
-                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s)
+            D.dbl_bn_relu_fused_bwd(bns, dout, dout2, self.stem_y, None, pv("bn1.g"), s_mean, s_istd,
+                                    self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s, beta=pv("bn1.b"))
         self.stem_wgrad(self.stem_dy, gv("conv1.w"), ws, wsb, s)
 
 

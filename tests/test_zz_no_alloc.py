@@ -57,7 +57,7 @@ def test_noalloc_matches_workspace_version_twice():
         got = _outputs(count, C)
         stream = torch.cuda.current_stream().cuda_stream
         rc = L.dbl_bn_relu_fused_bwd_noalloc(ctypes.byref(shape), dout.data_ptr(), dout2.data_ptr(), y.data_ptr(),
-                                             out.data_ptr(), gamma.data_ptr(), mean.data_ptr(), istd.data_ptr(),
+                                             out.data_ptr(), gamma.data_ptr(), None, mean.data_ptr(), istd.data_ptr(),
                                              got[0].data_ptr(), got[1].data_ptr(), got[2].data_ptr(),
                                              got[3].data_ptr(), stream)
         assert rc == D.DBL_OK, D.dbl_last_error()
