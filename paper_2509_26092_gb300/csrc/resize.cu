@@ -108,53 +108,87 @@ int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, 
 // The stem's unrolled input.  Position (n, m, q) holds rg source rows
 // y = rg*m + e - pad_h (e < rg), each as 8 column taps x (8/rg) channels:
 // element (e, t, ch) is the resized pixel at (y, q*sw + t - pw), channel ch
-// (zero outside the image, for t >= taps and for ch >= c).  One thread per
-// 16-byte chunk (8 elements): a warp's stores cover 512 contiguous bytes.
+// (zero outside the image, for t >= taps and for ch >= c).
+// One CTA per unrolled row (n, m): it interpolates the rg resized rows once
+// into shared memory (with pw zero columns on each side), then writes the
+// row's Q positions as 16-byte chunks (8 elements), consecutive threads on
+// consecutive chunks.
+constexpr int kStemMaxW = 1024;  // widest resized row a CTA stages (host-checked)
+
 template <int RG>
 __global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restrict__ in, __nv_bfloat16* __restrict__ out,
-                                                          int32_t n, int32_t hi, int32_t wi, int32_t c, int32_t ho,
-                                                          int32_t wo, int32_t M, int32_t Q, int32_t taps, int32_t sw,
-                                                          int32_t pw, int32_t ph)
+                                                          int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
+                                                          int32_t M, int32_t Q, int32_t taps, int32_t sw, int32_t pw,
+                                                          int32_t ph)
 {
-    constexpr int32_t rg = RG;
-    constexpr int32_t cu = 8 / RG;     // channels per tap
-    constexpr int32_t tpc = 8 / cu;    // taps per 16-byte chunk (1 or 2); a chunk never spans two rows
-    const unsigned total = (unsigned)n * M * Q * 8;
-    for (unsigned idx = blockIdx.x * blockDim.x + threadIdx.x; idx < total; idx += gridDim.x * blockDim.x) {
-        const int32_t chunk = (int32_t)(idx & 7u);
-        const unsigned pos = idx >> 3;
-        const int32_t q = (int32_t)(pos % (unsigned)Q);
-        const unsigned t0 = pos / (unsigned)Q;
-        const int32_t m = (int32_t)(t0 % (unsigned)M);
-        const int32_t b = (int32_t)(t0 / (unsigned)M);
-        const int32_t e = chunk / cu, tap0 = (chunk % cu) * tpc;
-        const int32_t y = rg * m + e - ph;
-        float v[8];
+    constexpr int32_t cu = 8 / RG;  // channels per tap
+    // staged rows: [RG][wo + 2*pw + 8][cu] fp32, column x at index x + pw (dynamic shared memory)
+    extern __shared__ __align__(16) float rows[];
+    const int32_t wst = wo + 2 * pw + 8;
+    const int32_t m = blockIdx.x % M, b = blockIdx.x / M;
+    const float* base = in + (int64_t)b * hi * wi * c;
+    // the RG source rows of this unrolled row: taps once per CTA
+    Taps ty[RG];
+    bool yin[RG];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) v[k] = 0.f;
-        if (y >= 0 && y < ho) {
-            const Taps ty = axis_taps(y, hi, ho);
-            const float* base = in + (int64_t)b * hi * wi * c;
-            const float* r0 = base + (int64_t)ty.i0 * wi * c;
-            const float* r1 = base + (int64_t)ty.i1 * wi * c;
+    for (int e = 0; e < RG; ++e) {
+        const int32_t y = RG * m + e - ph;
+        yin[e] = y >= 0 && y < ho;
+        ty[e] = axis_taps(yin[e] ? y : 0, hi, ho);
+    }
+    // one staged pixel (all its channels) per thread and iteration
+#pragma unroll 2
+    for (int32_t i = threadIdx.x; i < RG * wst; i += blockDim.x) {
+        const int32_t xs = i % wst, e = i / wst;
+        const int32_t x = xs - pw;
+        float v[cu];
 #pragma unroll
-            for (int32_t u = 0; u < tpc; ++u) {
-                const int32_t t = tap0 + u, x = q * sw + t - pw;
-                if (t >= taps || x < 0 || x >= wo) continue;
-                const Taps tx = axis_taps(x, wi, wo);
+        for (int ch = 0; ch < cu; ++ch) v[ch] = 0.f;
+        Taps tyy = ty[0];
+        bool in_y = yin[0];
 #pragma unroll
-                for (int32_t ch = 0; ch < cu; ++ch) {
-                    if (ch >= c) break;
+        for (int k = 1; k < RG; ++k)
+            if (e == k) {
+                tyy = ty[k];
+                in_y = yin[k];
+            }
+        if (in_y && x >= 0 && x < wo) {
+            const Taps tx = axis_taps(x, wi, wo);
+            const float* r0 = base + (int64_t)tyy.i0 * wi * c;
+            const float* r1 = base + (int64_t)tyy.i1 * wi * c;
+#pragma unroll
+            for (int ch = 0; ch < cu; ++ch)
+                if (ch < c) {
                     const float top = (1.f - tx.lam) * __ldg(r0 + tx.i0 * c + ch) + tx.lam * __ldg(r0 + tx.i1 * c + ch);
                     const float bot = (1.f - tx.lam) * __ldg(r1 + tx.i0 * c + ch) + tx.lam * __ldg(r1 + tx.i1 * c + ch);
-                    v[u * cu + ch] = (1.f - ty.lam) * top + ty.lam * bot;
+                    v[ch] = (1.f - tyy.lam) * top + tyy.lam * bot;
                 }
-            }
+        }
+        float* dst = rows + (int64_t)i * cu;
+        if constexpr (cu == 4) {
+            *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+        } else {
+#pragma unroll
+            for (int ch = 0; ch < cu; ++ch) dst[ch] = v[ch];
+        }
+    }
+    __syncthreads();
+    uint4* orow = reinterpret_cast<uint4*>(out) + ((int64_t)b * M + m) * Q * 8;
+    for (int32_t idx = threadIdx.x; idx < Q * 8; idx += blockDim.x) {
+        const int32_t q = idx >> 3, chunk = idx & 7;
+        const int32_t e = chunk / cu, tap0 = (chunk % cu) * (8 / cu);
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8 / cu; ++u) {
+            const int32_t t = tap0 + u;
+            const int32_t xs = q * sw + t;  // staged column of image column q*sw + t - pw
+#pragma unroll
+            for (int ch = 0; ch < cu; ++ch) v[u * cu + ch] = t < taps ? rows[(e * wst + xs) * cu + ch] : 0.f;
         }
         __nv_bfloat162 qv[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) qv[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
-        reinterpret_cast<uint4*>(out)[idx] = *reinterpret_cast<uint4*>(qv);
+        orow[idx] = *reinterpret_cast<uint4*>(qv);
     }
 }
 
@@ -177,21 +211,21 @@ extern "C" int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h
     if (!aligned16(out)) return set_error(DBL_ERR_INVALID, "progressive_resize_stem: output must be 16-byte aligned");
     const int32_t Q = (w_out + 2 * pad_w - taps) / stride_w + 1;
     if (Q <= 0) return set_error(DBL_ERR_INVALID, "progressive_resize_stem: empty output");
-    if ((int64_t)n * rows_out * Q * 8 >= (int64_t)1 << 31)
+    if ((int64_t)n * rows_out >= (int64_t)1 << 31 || (int64_t)Q * 8 >= (int64_t)1 << 31)
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: output too large for 32-bit indexing");
+    if (w_out + 2 * pad_w + 8 > kStemMaxW + 16 || (Q - 1) * stride_w + 8 > w_out + 2 * pad_w + 8)
+        return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: rows wider than %d pixels", kStemMaxW);
     if (n == 0) return DBL_OK;
-    const int64_t total = (int64_t)n * rows_out * Q * 8;
-    int64_t blocks = (total + 255) / 256;
-    const int64_t cap = (int64_t)sm_count() * 16;
-    if (blocks > cap) blocks = cap;
+    const int blocks = n * rows_out;  // one CTA per unrolled row
+    const size_t smem = (size_t)row_group * (w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels
     if (row_group == 2)
-        resize_stem_kernel<2><<<(int)(blocks < 1 ? 1 : blocks), 256, 0, as_stream(stream)>>>(
-            in, static_cast<__nv_bfloat16*>(out), n, h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w,
-            pad_h);
+        resize_stem_kernel<2><<<blocks, 256, smem, as_stream(stream)>>>(in, static_cast<__nv_bfloat16*>(out), h_in,
+                                                                        w_in, c, h_out, w_out, rows_out, Q, taps,
+                                                                        stride_w, pad_w, pad_h);
     else
-        resize_stem_kernel<1><<<(int)(blocks < 1 ? 1 : blocks), 256, 0, as_stream(stream)>>>(
-            in, static_cast<__nv_bfloat16*>(out), n, h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w,
-            pad_h);
+        resize_stem_kernel<1><<<blocks, 256, smem, as_stream(stream)>>>(in, static_cast<__nv_bfloat16*>(out), h_in,
+                                                                        w_in, c, h_out, w_out, rows_out, Q, taps,
+                                                                        stride_w, pad_w, pad_h);
     return launch_check("progressive_resize_stem launch");
 }
 
