@@ -230,8 +230,9 @@ def build_pipeline(cfg, device):
     bl_max = max(cfg["large"])
     bs_max = max([b for b in cfg["small"] if b] or [0])
     nat = cfg["native"]
-    host_l = torch.from_numpy(synth.images(bl_max, nat, nat, 3, seed=1, name="large")).pin_memory()
-    host_s = torch.from_numpy(synth.images(bs_max, nat, nat, 3, seed=1, name="small")).pin_memory() if bs_max else None
+    # decoded 8-bit pixels, as an input pipeline hands them over (standardized on the GPU)
+    host_l = torch.from_numpy(synth.images_u8(bl_max, nat, nat, 3, seed=1, name="large")).pin_memory()
+    host_s = torch.from_numpy(synth.images_u8(bs_max, nat, nat, 3, seed=1, name="small")).pin_memory() if bs_max else None
     lab_l = torch.from_numpy(synth.labels(bl_max, cfg["classes"], seed=1, name="large")).pin_memory()
     lab_s = torch.from_numpy(synth.labels(bs_max, cfg["classes"], seed=1, name="small")).pin_memory() if bs_max else None
     stages = []
@@ -338,9 +339,9 @@ def run_profile_iteration(args, cfg):
         large = R.Worker(spec, bl, res)
         small = R.Worker(spec, bs, res) if bs else None
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_small=F_SMALL)
-        it.set_inputs(torch.from_numpy(synth.images(bl, nat, nat, 3, seed=1)).cuda(),
+        it.set_inputs(torch.from_numpy(synth.images_u8(bl, nat, nat, 3, seed=1)).cuda(),
                       torch.from_numpy(synth.labels(bl, cfg["classes"], seed=1)).cuda(),
-                      torch.from_numpy(synth.images(bs, nat, nat, 3, seed=2)).cuda() if bs else None,
+                      torch.from_numpy(synth.images_u8(bs, nat, nat, 3, seed=2)).cuda() if bs else None,
                       torch.from_numpy(synth.labels(bs, cfg["classes"], seed=2)).cuda() if bs else None)
         it.run()
         torch.cuda.synchronize()
@@ -501,7 +502,7 @@ def run_ours(args, cfg):
         if h2d == 0:
             for st in stages:
                 bl, bs = st["large"].batch, st["small"].batch if st["small"] else 0
-                h2d += (bl + bs) * cfg["native"] ** 2 * 3 * 4 + (bl + bs) * 4
+                h2d += (bl + bs) * cfg["native"] ** 2 * 3 * pipe["host_l"].element_size() + (bl + bs) * 4
                 d2h += 4 * (2 if bs else 1)
     prev[0].synchronize()
     loss_seen.append(prev[1][:prev[2]].tolist())
@@ -552,6 +553,8 @@ def run_ours(args, cfg):
                            "small_batch": list(cfg["small"]), "images_per_step": images_per_step,
                            "params": pipe["spec"].n_params(), "f_small": F_SMALL, "lr": LR, "momentum": MOMENTUM,
                            "l2": "working set (activations, several GB) larger than L2; no explicit flush",
+                           "input": f"uint8 images {cfg['native']}x{cfg['native']}x3 from pinned host memory, "
+                                    "standardized per channel on the GPU",
                            "parallelism": f"{ws} independent replica(s), 2 worker streams each"},
                 "per_resolution": per_res, "roofline": roofline, "cpu_baseline": cpu,
                 "e2e": {"value": round(e2e_value, 1), "unit": "images/s", "h2d_bytes_per_step": h2d,

@@ -275,6 +275,15 @@ DBL_API int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in
                                         int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
                                         int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream);
 
+/* The same, from 8-bit pixels: in is [n,h_in,w_in,c] uint8 and the value the
+ * resize sees is p*scale[ch] + bias[ch] (fp32, rounded after the product and
+ * after the sum), the usual per-channel standardization of decoded images.
+ * scale, bias: host arrays [c], read during the call. */
+DBL_API int dbl_progressive_resize_stem_u8(const uint8_t* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c,
+                                           const float* scale, const float* bias, void* out, int32_t h_out,
+                                           int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
+                                           int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream);
+
 /* Sets base[i*ld + j] = 0 for i < rows, j < cols (fp32, device memory, stream
  * ordered).  The ResNet-18 stem uses it to keep the weight gradient of the
  * padding rows of its row-grouped weight layout at zero, so that those

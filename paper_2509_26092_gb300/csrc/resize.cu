@@ -115,18 +115,38 @@ int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, 
 // consecutive chunks.
 constexpr int kStemMaxW = 1024;  // widest resized row a CTA stages (host-checked)
 
-template <int RG>
-__global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restrict__ in, __nv_bfloat16* __restrict__ out,
+// Per-channel affine map of 8-bit pixels to the network's input values,
+// x = p*scale + bias, rounded after the product and after the sum (no
+// contraction: the same bits as the same two fp32 operations on the host).
+struct PixelNorm {
+    float scale[8], bias[8];
+};
+
+template <typename Tin>
+__device__ __forceinline__ float stem_pixel(const Tin* p, int ch, const PixelNorm& nm);
+template <>
+__device__ __forceinline__ float stem_pixel<float>(const float* p, int ch, const PixelNorm&)
+{
+    return __ldg(p);
+}
+template <>
+__device__ __forceinline__ float stem_pixel<uint8_t>(const uint8_t* p, int ch, const PixelNorm& nm)
+{
+    return __fadd_rn(__fmul_rn((float)__ldg(p), nm.scale[ch]), nm.bias[ch]);
+}
+
+template <int RG, typename Tin>
+__global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict__ in, __nv_bfloat16* __restrict__ out,
                                                           int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
                                                           int32_t M, int32_t Q, int32_t taps, int32_t sw, int32_t pw,
-                                                          int32_t ph)
+                                                          int32_t ph, const PixelNorm nm)
 {
     constexpr int32_t cu = 8 / RG;  // channels per tap
     // staged rows: [RG][wo + 2*pw + 8][cu] fp32, column x at index x + pw (dynamic shared memory)
     extern __shared__ __align__(16) float rows[];
     const int32_t wst = wo + 2 * pw + 8;
     const int32_t m = blockIdx.x % M, b = blockIdx.x / M;
-    const float* base = in + (int64_t)b * hi * wi * c;
+    const Tin* base = in + (int64_t)b * hi * wi * c;
     // the RG source rows of this unrolled row: taps once per CTA
     Taps ty[RG];
     bool yin[RG];
@@ -154,13 +174,15 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restric
             }
         if (in_y && x >= 0 && x < wo) {
             const Taps tx = axis_taps(x, wi, wo);
-            const float* r0 = base + (int64_t)tyy.i0 * wi * c;
-            const float* r1 = base + (int64_t)tyy.i1 * wi * c;
+            const Tin* r0 = base + (int64_t)tyy.i0 * wi * c;
+            const Tin* r1 = base + (int64_t)tyy.i1 * wi * c;
 #pragma unroll
             for (int ch = 0; ch < cu; ++ch)
                 if (ch < c) {
-                    const float top = (1.f - tx.lam) * __ldg(r0 + tx.i0 * c + ch) + tx.lam * __ldg(r0 + tx.i1 * c + ch);
-                    const float bot = (1.f - tx.lam) * __ldg(r1 + tx.i0 * c + ch) + tx.lam * __ldg(r1 + tx.i1 * c + ch);
+                    const float top = (1.f - tx.lam) * stem_pixel(r0 + tx.i0 * c + ch, ch, nm) +
+                                      tx.lam * stem_pixel(r0 + tx.i1 * c + ch, ch, nm);
+                    const float bot = (1.f - tx.lam) * stem_pixel(r1 + tx.i0 * c + ch, ch, nm) +
+                                      tx.lam * stem_pixel(r1 + tx.i1 * c + ch, ch, nm);
                     v[ch] = (1.f - tyy.lam) * top + tyy.lam * bot;
                 }
         }
@@ -194,9 +216,12 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const float* __restric
 
 }  // namespace
 
-extern "C" int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
-                                           int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
-                                           int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream)
+namespace {
+
+template <typename Tin>
+int resize_stem_impl(const Tin* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, const PixelNorm& nm, void* out,
+                     int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w, int32_t row_group,
+                     int32_t pad_h, int32_t rows_out, void* stream)
 {
     using namespace dbl;
     if (!in || !out || n < 0 || h_in <= 0 || w_in <= 0 || c <= 0 || h_out <= 0 || w_out <= 0 || taps <= 0 ||
@@ -219,14 +244,42 @@ extern "C" int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h
     const int blocks = n * rows_out;  // one CTA per unrolled row
     const size_t smem = (size_t)row_group * (w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels
     if (row_group == 2)
-        resize_stem_kernel<2><<<blocks, 256, smem, as_stream(stream)>>>(in, static_cast<__nv_bfloat16*>(out), h_in,
-                                                                        w_in, c, h_out, w_out, rows_out, Q, taps,
-                                                                        stride_w, pad_w, pad_h);
+        resize_stem_kernel<2, Tin><<<blocks, 256, smem, as_stream(stream)>>>(
+            in, static_cast<__nv_bfloat16*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
+            nm);
     else
-        resize_stem_kernel<1><<<blocks, 256, smem, as_stream(stream)>>>(in, static_cast<__nv_bfloat16*>(out), h_in,
-                                                                        w_in, c, h_out, w_out, rows_out, Q, taps,
-                                                                        stride_w, pad_w, pad_h);
+        resize_stem_kernel<1, Tin><<<blocks, 256, smem, as_stream(stream)>>>(
+            in, static_cast<__nv_bfloat16*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
+            nm);
     return launch_check("progressive_resize_stem launch");
+}
+
+}  // namespace
+
+extern "C" int dbl_progressive_resize_stem(const float* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c, void* out,
+                                           int32_t h_out, int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
+                                           int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream)
+{
+    const PixelNorm nm{};
+    return resize_stem_impl(in, n, h_in, w_in, c, nm, out, h_out, w_out, taps, stride_w, pad_w, row_group, pad_h,
+                            rows_out, stream);
+}
+
+extern "C" int dbl_progressive_resize_stem_u8(const uint8_t* in, int32_t n, int32_t h_in, int32_t w_in, int32_t c,
+                                              const float* scale, const float* bias, void* out, int32_t h_out,
+                                              int32_t w_out, int32_t taps, int32_t stride_w, int32_t pad_w,
+                                              int32_t row_group, int32_t pad_h, int32_t rows_out, void* stream)
+{
+    using namespace dbl;
+    if (!scale || !bias) return set_error(DBL_ERR_INVALID, "progressive_resize_stem_u8: null scale or bias");
+    if (c <= 0 || c > 8) return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem_u8: 1..8 channels");
+    PixelNorm nm{};
+    for (int ch = 0; ch < c; ++ch) {
+        nm.scale[ch] = scale[ch];
+        nm.bias[ch] = bias[ch];
+    }
+    return resize_stem_impl(in, n, h_in, w_in, c, nm, out, h_out, w_out, taps, stride_w, pad_w, row_group, pad_h,
+                            rows_out, stream);
 }
 
 extern "C" int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, int32_t h_in, int32_t w_in, int32_t c,

@@ -81,6 +81,9 @@ def lib():
             "dbl_progressive_resize_stem": (ctypes.c_int, [_V, _I32, _I32, _I32, _I32, _V, _I32, _I32, _I32, _I32,
                                                            _I32, _I32, _I32, _I32, _V]),
             "dbl_zero_f32_2d": (ctypes.c_int, [_V, _I64, _I64, _I64, _V]),
+            "dbl_progressive_resize_stem_u8": (ctypes.c_int, [_V, _I32, _I32, _I32, _I32, ctypes.POINTER(ctypes.c_float),
+                                                              ctypes.POINTER(ctypes.c_float), _V, _I32, _I32, _I32,
+                                                              _I32, _I32, _I32, _I32, _I32, _V]),
             "dbl_update_factor": (_D, [_D, _D, ctypes.c_int]),
             "dbl_plan": (ctypes.c_int, [_D, _D, _I32, _I32, _D, _D, _D, ctypes.c_int] + [ctypes.POINTER(_D)] * 4),
         }
@@ -228,6 +231,17 @@ def dbl_progressive_resize_stem(inp, n, h_in, w_in, c, out, h_out, w_out, taps, 
         rows_out = h_out
     _check(lib().dbl_progressive_resize_stem(_ptr(inp), n, h_in, w_in, c, _ptr(out), h_out, w_out, taps, stride_w, pad_w,
                                              row_group, pad_h, rows_out, _stream(stream)))
+
+
+def dbl_progressive_resize_stem_u8(inp, n, h_in, w_in, c, scale, bias, out, h_out, w_out, taps, stride_w, pad_w,
+                                   row_group=1, pad_h=0, rows_out=None, stream=None):
+    """8-bit images, standardized per channel as p*scale + bias (scale, bias: c floats)."""
+    if rows_out is None:
+        rows_out = h_out
+    sc = (ctypes.c_float * c)(*[float(v) for v in scale])
+    bi = (ctypes.c_float * c)(*[float(v) for v in bias])
+    _check(lib().dbl_progressive_resize_stem_u8(_ptr(inp), n, h_in, w_in, c, sc, bi, _ptr(out), h_out, w_out, taps,
+                                                stride_w, pad_w, row_group, pad_h, rows_out, _stream(stream)))
 
 
 def dbl_zero_f32_2d(base, rows, cols, ld, stream=None):

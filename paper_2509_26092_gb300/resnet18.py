@@ -40,11 +40,19 @@ layer read the fp32 master weights directly (they are tiny).
 """
 from dataclasses import dataclass, field
 
+import numpy as np
 import torch
 
 from . import dbl as D
 
 WIDTHS = (64, 128, 256, 512)
+# 8-bit images are standardized per channel as p*PIXEL_SCALE + PIXEL_BIAS (fp32): the
+# usual ImageNet channel means and deviations of decoded pixels (the paper does not give
+# its preprocessing constants)
+PIXEL_MEAN = (0.485 * 255, 0.456 * 255, 0.406 * 255)
+PIXEL_STD = (0.229 * 255, 0.224 * 255, 0.225 * 255)
+PIXEL_SCALE = tuple(float(np.float32(1.0) / np.float32(s)) for s in PIXEL_STD)
+PIXEL_BIAS = tuple(float(-np.float32(m) / np.float32(s)) for m, s in zip(PIXEL_MEAN, PIXEL_STD))
 ALIGN = 64  # parameter tensors start on 256-byte boundaries
 
 
@@ -293,10 +301,16 @@ class Worker:
                             lay.conv_pad, s=1, stride_w=1, pad_w=0)
 
     def stem_prepare(self, images, native_res, stream):
-        """Resize the native images to this worker's resolution, in the stem's unrolled layout."""
+        """Resize the native images (fp32 values, or uint8 pixels standardized with
+        PIXEL_SCALE / PIXEL_BIAS) to this worker's resolution, in the stem's unrolled layout."""
         st, lay = self.spec.stem, self.spec.stem_layout
-        D.dbl_progressive_resize_stem(images, self.batch, native_res, native_res, 3, self.x0, self.res, self.res, st.r,
-                                      st.stride, st.pad, lay.rg, lay.pad_h, self.stem_rows, stream)
+        if images.dtype == torch.uint8:
+            D.dbl_progressive_resize_stem_u8(images, self.batch, native_res, native_res, 3, PIXEL_SCALE, PIXEL_BIAS,
+                                             self.x0, self.res, self.res, st.r, st.stride, st.pad, lay.rg, lay.pad_h,
+                                             self.stem_rows, stream)
+        else:
+            D.dbl_progressive_resize_stem(images, self.batch, native_res, native_res, 3, self.x0, self.res, self.res,
+                                          st.r, st.stride, st.pad, lay.rg, lay.pad_h, self.stem_rows, stream)
 
     def stem_wgrad(self, dy, grad_w, ws, wsb, stream):
         """Stem weight gradient into grad_w (stored layout); rows past the filter stay zero."""
@@ -445,24 +459,27 @@ class DualBatchIteration:
         self._consumed = None      # compute-stream event: the last run() has read its inputs
 
     def set_inputs(self, images_l, labels_l, images_s=None, labels_s=None, non_blocking=False, stream=None):
-        """fp32 images at the native resolution and int32 labels (device or pinned host
-        tensors), copied into the iteration's device buffers.  Without ``stream`` the
+        """Images at the native resolution (fp32 values, or uint8 pixels) and int32 labels
+        (device or pinned host tensors), copied into the iteration's device buffers.  Without ``stream`` the
         copies go on the current stream.  With a (copy) ``stream`` they are issued there
         once the previous run() has consumed the buffers, and the next run() waits for
         them, so that host-to-device copies overlap the compute of other iterations."""
         dev = self.server.w.device
+        for have, new_t in ((self.images_l, images_l), (self.images_s, images_s)):
+            if self.graph is not None and have is not None and new_t is not None and have.dtype != new_t.dtype:
+                raise ValueError("set_inputs: the captured graph reads images of another dtype")
         cs = stream if stream is not None else torch.cuda.current_stream()
         if stream is not None and self._consumed is not None:
             stream.wait_event(self._consumed)
         with torch.cuda.stream(cs):
             if self.large is not None:
-                if self.images_l is None:
-                    self.images_l = torch.empty(images_l.shape, dtype=torch.float32, device=dev)
+                if self.images_l is None or self.images_l.dtype != images_l.dtype:
+                    self.images_l = torch.empty(images_l.shape, dtype=images_l.dtype, device=dev)
                 self.images_l.copy_(images_l, non_blocking=non_blocking)
                 self.large.labels.copy_(labels_l, non_blocking=non_blocking)
             if self.small is not None:
-                if self.images_s is None:
-                    self.images_s = torch.empty(images_s.shape, dtype=torch.float32, device=dev)
+                if self.images_s is None or self.images_s.dtype != images_s.dtype:
+                    self.images_s = torch.empty(images_s.shape, dtype=images_s.dtype, device=dev)
                 self.images_s.copy_(images_s, non_blocking=non_blocking)
                 self.small.labels.copy_(labels_s, non_blocking=non_blocking)
         if stream is not None:

@@ -26,6 +26,11 @@ def images(n, h, w, c=3, seed=0, name="images"):
     return rng(seed, name).standard_normal((n, h, w, c), dtype=np.float32)
 
 
+def images_u8(n, h, w, c=3, seed=0, name="images_u8"):
+    """[n, h, w, c] uint8, i.i.d. uniform in 0..255 (decoded 8-bit pixels)."""
+    return rng(seed, name).integers(0, 256, size=(n, h, w, c), dtype=np.uint8)
+
+
 def labels(n, classes, seed=0, name="labels"):
     """[n] int32, uniform in [0, classes)."""
     return rng(seed, name).integers(0, classes, size=n, dtype=np.int32)

@@ -107,6 +107,32 @@ def test_resize_stem_unrolls_the_resized_image(D, n, hin, hout, r, st, pad):
     check_status(D)
 
 
+@pytest.mark.parametrize("n,hin,hout", [(2, 224, 160), (3, 40, 40)])
+def test_resize_stem_from_8bit_pixels(D, n, hin, hout):
+    """8-bit pixels standardized on the GPU: the same bits as the fp32 path on pixels
+    standardized on the host with the same two fp32 operations, and the oracle's resize."""
+    from paper_2509_26092_gb300.resnet18 import PIXEL_BIAS, PIXEL_SCALE
+    r, st, pad = 7, 2, 3
+    lay = _stem_layout(r, st, pad)
+    u8 = rng(hin + 5).integers(0, 256, size=(n, hin, hin, 3), dtype=np.uint8)
+    x32 = u8.astype(np.float32) * np.asarray(PIXEL_SCALE, np.float32) + np.asarray(PIXEL_BIAS, np.float32)
+    P = (hout + 2 * pad - r) // st + 1
+    rows = lay.rows(hout, P)
+    a = torch.empty((n, rows, P, 64), dtype=torch.bfloat16, device="cuda")
+    b = torch.empty_like(a)
+    D.dbl_progressive_resize_stem_u8(torch.from_numpy(u8).cuda(), n, hin, hin, 3, PIXEL_SCALE, PIXEL_BIAS, a, hout,
+                                     hout, r, st, pad, lay.rg, lay.pad_h, rows)
+    D.dbl_progressive_resize_stem(to_f32_dev(x32), n, hin, hin, 3, b, hout, hout, r, st, pad, lay.rg, lay.pad_h, rows)
+    assert torch.equal(a, b)
+    ref = orc.bilinear_resize(x32.astype(np.float64), hout, hout)
+    got = stem_fold(host(a).reshape(n, rows, P, lay.rg, 8, 8 // lay.rg), r, st, pad, hout, lay.rg, lay.pad_h)[..., :3]
+    covered = ~np.isnan(got[0, :, :, 0])
+    # one bf16 ulp of the value, plus the fp32 rounding of interpolating O(1) inputs (values near zero)
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
+    assert np.all(np.abs(got[:, covered] - ref[:, covered]) <= ulp[:, covered] + 1e-6)
+    check_status(D)
+
+
 STEM_CASES = [  # n, h (square input), r, stride, pad
     (2, 20, 7, 2, 3),    # ImageNet stem on a small image
     (3, 10, 3, 1, 1),    # CIFAR stem

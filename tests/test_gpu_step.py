@@ -167,3 +167,22 @@ def test_inputs_on_a_copy_stream_give_the_same_iteration(R):
         outs.append((server.w.clone(), losses.clone()))
     assert torch.equal(outs[0][0], outs[1][0])
     assert torch.equal(outs[0][1], outs[1][1]) and bool(torch.all(outs[0][1][:4] > 0))  # 2 iterations x 2 workers
+
+
+def test_8bit_images_give_the_same_iteration_as_standardized_fp32(R):
+    """The iteration fed 8-bit pixels equals the iteration fed the same pixels standardized
+    on the host (p*PIXEL_SCALE + PIXEL_BIAS in fp32), bit for bit."""
+    spec = R.ResNet18Spec("imagenet", 10)
+    params = synth.params(spec.table(), seed=4)
+    u8 = synth.images_u8(6, 96, 96, 3, seed=4)
+    x32 = u8.astype(np.float32) * np.asarray(R.PIXEL_SCALE, np.float32) + np.asarray(R.PIXEL_BIAS, np.float32)
+    lab = torch.from_numpy(synth.labels(6, 10, seed=4)).cuda()
+    outs = []
+    for img in (torch.from_numpy(u8).cuda(), torch.from_numpy(x32).cuda()):
+        server = R.ServerState(spec, params)
+        it = R.DualBatchIteration(server, R.Worker(spec, 4, 64), R.Worker(spec, 2, 64), 96)
+        it.set_inputs(img[2:], lab[2:], img[:2], lab[:2])
+        it.run()
+        torch.cuda.synchronize()
+        outs.append(server.w.clone())
+    assert torch.equal(outs[0], outs[1])
