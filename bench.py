@@ -72,7 +72,7 @@ def _conv_source_hash():
 def _traffic_record(config):
     """DRAM bytes (read + write) of all conv-kernel launches of one iteration at the largest
     stage, from a committed ncu summary, if it was taken on the current kernel source."""
-    path = os.path.join(ROOT, "profiles", "conv_igemm_traffic.json")
+    path = os.path.join(ROOT, "profiles", "conv_traffic_imagenet_hybrid_224.json")
     try:
         with open(path) as f:
             rec = json.load(f)
