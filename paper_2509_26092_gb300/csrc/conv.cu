@@ -70,8 +70,11 @@ struct ConvParams {
     int wg_accumulate;  // wgrad with one slice: add into dw
     float* stats;       // fwd: [gridDim.x][2][Ncols] per-CTA channel sums, or nullptr
     // window kernel (3x3, stride 1, pad 1): the batch as one column of zero-padded images
-    int win_H, win_W;         // image height and width (= output height and width)
-    int win_Hp, win_Wp;       // padded height and width (H + 2, W + 2)
+    int win_R, win_S;         // filter taps along H and W
+    int win_ph, win_pw;       // padding along H and W (a strip row copy starts at column -pw)
+    int win_P, win_Q;         // output height and width: positions with h < P, w < Q are outputs
+    int win_Hp, win_Wp;       // padded height and width (H + 2*ph, W + 2*pw)
+    int win_tile;             // positions per tile (weight gradient: per K-block), <= 256
     int win_srows;            // padded rows loaded per strip (weight gradient: x strip)
     int win_dyrows;           // weight gradient: padded rows of the dy strip
     int win_strip_bytes;      // bytes of one strip buffer, or of one x + dy stage (a multiple of 1024)
@@ -597,7 +600,7 @@ __device__ __forceinline__ void win_load_wtile(const ConvParams& p, const CUtens
                                                int tap, int cb, int n_tile)
 {
     if constexpr (DG) {
-        const int wtap = 8 - tap;
+        const int wtap = p.win_R * p.win_S - 1 - tap;  // flipped filter
 #pragma unroll
         for (int j = 0; j < BN / 64; ++j) tma_load_3d_elect(dst + j * 8192, tmB, bar, n_tile * BN + 64 * j, wtap, cb * 64);
     } else {
@@ -621,7 +624,8 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
     uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
     const int CB = p.cblocks;
-    const int b_bytes = RES ? 9 * CB * C::B_TILE : kWinBStages * C::B_TILE;
+    const int ntaps = p.win_R * p.win_S;
+    const int b_bytes = RES ? ntaps * CB * C::B_TILE : kWinBStages * C::B_TILE;
     uint8_t* strip = sgen + b_bytes;
     float* epi_tile = reinterpret_cast<float*>(strip + 2 * p.win_strip_bytes);
     float* epi_sum = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(epi_tile) + kEpiTileBytes);
@@ -665,7 +669,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const uint32_t strip_tx = (uint32_t)(p.win_srows * Wp * 128);
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
             const TileCoord tc = decode_tile(p, t);
-            const int g0 = tc.m_tile * kWinBMT / Wp;
+            const int g0 = tc.m_tile * p.win_tile / Wp;
             for (int cb = 0; cb < CB; ++cb, ++it) {
                 const int s = it & 1;
                 const uint32_t ok = mbar_wait_warp(&sempty[s], ((it >> 1) & 1) ^ 1, &abort_flag);
@@ -678,9 +682,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 for (int r = 0; r < p.win_srows; ++r) {
                     const int g = g0 + r;
                     const int n = g / p.win_Hp, hp = g - n * p.win_Hp;
-                    // padded row hp of image n = input row hp - 1 (rows -1 and H, and images past
-                    // the batch, are outside the tensor and arrive as zeros)
-                    tma_load_4d_elect(dst + r * Wp * 128, &tmA, &sfull[s], cb * 64, -1, hp - 1, n);
+                    // padded row hp of image n = input row hp - ph from column -pw (padding rows and
+                    // columns, and images past the batch, are outside the tensor and arrive as zeros)
+                    tma_load_4d_elect(dst + r * Wp * 128, &tmA, &sfull[s], cb * 64, -p.win_pw, hp - p.win_ph, n);
                 }
             }
             if (failed) break;
@@ -692,8 +696,8 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     } else if (warp == 5) {
         // ------------------------------------------------------------------ weight producer
         if (RES) {
-            mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(9 * CB * C::B_TILE));
-            for (int tap = 0; tap < 9; ++tap)
+            mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(ntaps * CB * C::B_TILE));
+            for (int tap = 0; tap < ntaps; ++tap)
                 for (int cb = 0; cb < CB; ++cb)
                     win_load_wtile<BN, DG>(p, &tmB, sgen + (tap * CB + cb) * C::B_TILE, &bfull[0], tap, cb, 0);
             (void)mbar_drain_warp(&bfull[0], 0);
@@ -703,7 +707,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
                 const TileCoord tc = decode_tile(p, t);
                 for (int cb = 0; cb < CB && !failed; ++cb)
-                    for (int tap = 0; tap < 9; ++tap, ++bt) {
+                    for (int tap = 0; tap < ntaps; ++tap, ++bt) {
                         const int s = bt % kWinBStages;
                         const uint32_t ok =
                             mbar_wait_warp(&bempty[s], ((bt / kWinBStages) & 1) ^ 1, &abort_flag);
@@ -739,7 +743,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 break;
             }
             tc_fence_after();
-            const int L0 = tc.m_tile * kWinBMT;
+            const int L0 = tc.m_tile * p.win_tile;
             const int off0 = L0 - (L0 / Wp) * Wp;  // tile start within the strip's first row
             const uint32_t d = tmem + (uint32_t)(buf * kWinACC * BN);
             for (int cb = 0; cb < CB && !failed; ++cb, ++it) {
@@ -751,9 +755,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 }
                 tc_fence_after();
                 const uint32_t sa = sbase + (uint32_t)(b_bytes + s * p.win_strip_bytes);
+                int r = 0, sx = 0;  // (tap / S, tap % S), stepped without divisions
 #pragma unroll 1
-                for (int tap = 0; tap < 9; ++tap) {
-                    const int r = tap / 3, sx = tap - 3 * r;
+                for (int tap = 0; tap < ntaps; ++tap) {
                     uint32_t sb;
                     int bs = 0;
                     if (RES) {
@@ -783,6 +787,10 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                         mma_commit_elect(&bempty[bs]);
                         ++bt;
                     }
+                    if (++sx == p.win_S) {
+                        sx = 0;
+                        ++r;
+                    }
                 }
                 mma_commit_elect(&sempty[s]);
             }
@@ -811,11 +819,12 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int row = warp * 32 + lane;
 #pragma unroll 1
             for (int a = 0; a < kWinACC; ++a) {
-                const int L = tc.m_tile * kWinBMT + a * 128 + row;
+                const int L = tc.m_tile * p.win_tile + a * 128 + row;
                 const int n = L / img, rem = L - n * img;
                 const int hp = rem / Wp, wp = rem - hp * Wp;
-                const bool valid = n < p.gN && hp < p.win_H && wp < p.win_W;
-                const int64_t out_row = ((int64_t)n * p.win_H + hp) * p.win_W + wp;
+                // rows past the tile belong to the next tile (row-aligned tiles are shorter than 256)
+                const bool valid = a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P && wp < p.win_Q;
+                const int64_t out_row = ((int64_t)n * p.win_P + hp) * p.win_Q + wp;
                 const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * kWinACC + a) * BN);
 #pragma unroll
                 for (int ch = 0; ch < BN / 32; ++ch) {
@@ -848,20 +857,21 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 }
 
 // ----------------------------------------------------------------------------- window weight gradient
-// dW[k][r][s][c] = sum over positions L of dy[L][k] * x_pad[L + r*Wp + s][c] for 3x3 stride-1
-// layers with 64 input and 64 output channels, in the padded position space of conv_win_kernel:
-// dy is zero at the positions that are not outputs (its strip rows are read with w from 0 to
-// Wp-1 and h from 0 to Hp-1, and the zero fill of TMA covers w >= W and h >= H).
-// A CTA owns all 576 x 64 outputs, as five 128 x 64 TMEM accumulators (tap pairs (0,1), (2,3),
-// (4,5), (6,7), (8, -)), and one contiguous range of K-blocks of 256 positions (split-K over
-// CTAs, fixed-order reduce afterwards).  Per K-block it loads one x strip and one dy strip; all
-// nine taps read the same x strip.  A operand (x, MN-major: a 128-byte strip row holds the 64
-// channels of one position) of tap pair (t0, t1): start row off(t0) + 16j for K-step j, second
-// 64-row half LBO = (off(t1) - off(t0)) rows further; the fifth pair's second half is computed
-// and not stored.  B operand (dy, MN-major): start row 16j.
-constexpr int kWgWinKB = 256;  // positions per K-block
-constexpr int kWgWinAcc = 5;   // 128-row accumulators (tap pairs)
+// dW[k][r][s][c] = sum over positions L of dy[L][k] * x_pad[L + r*Wp + s][c] for stride-1
+// layers with 64 input and 64 output channels and at most 10 taps, in the padded position space
+// of conv_win_kernel: dy is zero at the positions that are not outputs (its strip rows are read
+// with w from 0 to Wp-1 and h from 0 to Hp-1, and the zero fill of TMA covers w >= Q and h >= P).
+// A CTA owns all taps*64 x 64 outputs, as ceil(taps/2) 128 x 64 TMEM accumulators (tap pairs
+// (0,1), (2,3), ...), and one contiguous range of K-blocks (256 positions, or two whole padded
+// rows when those are a multiple of 16; split-K over CTAs, fixed-order reduce afterwards).  Per
+// K-block it loads one x strip and one dy strip; all taps read the same x strip.  A operand (x,
+// MN-major: a 128-byte strip row holds the 64 channels of one position) of tap pair (t0, t1):
+// start row off(t0) + 16j for K-step j, second 64-row half LBO = (off(t1) - off(t0)) rows
+// further; for an odd tap count the last pair's second half is computed and not stored.
+// B operand (dy, MN-major): start row 16j.
+constexpr int kWgWinKB = 256;  // positions per K-block (row-aligned K-blocks may be shorter)
 
+template <int NACC>  // accumulators: ceil(taps / 2)
 __global__ void __launch_bounds__(kWinThreads, 1)
     conv_wgwin_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmDY,
                       const ConvParams p)
@@ -877,6 +887,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const int Wp = p.win_Wp;
     const int xalign = ((p.win_srows * Wp * 128 + 1023) / 1024) * 1024;  // dy strip offset in a stage
     const int stage_bytes = p.win_strip_bytes;
+    const int ntaps = p.win_R * p.win_S;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
@@ -916,13 +927,13 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     break;
                 }
                 uint8_t* dst = sgen + s * stage_bytes + (is_x ? 0 : xalign);
-                const int g0 = kb * kWgWinKB / Wp;
+                const int g0 = kb * p.win_tile / Wp;
                 mbar_arrive_expect_tx_elect(&full_bar[s], tx);
                 for (int r = 0; r < rows; ++r) {
                     const int g = g0 + r;
                     const int n = g / p.win_Hp, hp = g - n * p.win_Hp;
                     if (is_x)
-                        tma_load_4d_elect(dst + r * Wp * 128, &tmX, &full_bar[s], 0, -1, hp - 1, n);
+                        tma_load_4d_elect(dst + r * Wp * 128, &tmX, &full_bar[s], 0, -p.win_pw, hp - p.win_ph, n);
                     else
                         tma_load_4d_elect(dst + r * Wp * 128, &tmDY, &full_bar[s], 0, 0, hp, n);
                 }
@@ -935,6 +946,15 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     } else if (warp == 6) {
         // ------------------------------------------------------------------ MMA issuer
         const uint32_t idesc = idesc_bf16(BM, 64, 1u, 1u);
+        // strip-row offsets of each tap pair's two halves (the unused half of an odd last pair
+        // reads the row after its first half), once per CTA
+        int o0[NACC], o1[NACC];
+#pragma unroll
+        for (int pp = 0; pp < NACC; ++pp) {
+            const int t0 = 2 * pp, t1 = 2 * pp + 1;
+            o0[pp] = (t0 / p.win_S) * Wp + t0 % p.win_S;
+            o1[pp] = t1 < ntaps ? (t1 / p.win_S) * Wp + t1 % p.win_S : o0[pp] + 1;
+        }
         int it = 0, lt = 0;
         bool failed = false;
         for (int z = blockIdx.x; z < p.zdim && !failed; z += gridDim.x, ++lt) {
@@ -953,20 +973,16 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                const int P0 = kb * kWgWinKB;
+                const int P0 = kb * p.win_tile;
                 const int off = P0 - (P0 / Wp) * Wp;
                 const uint32_t xa = sbase + (uint32_t)(s * stage_bytes), ya = xa + (uint32_t)xalign;
 #pragma unroll 1
-                for (int j = 0; j < kWgWinKB / 16; ++j) {
+                for (int j = 0; j < p.win_tile / 16; ++j) {
                     const uint64_t bd = smem_desc(ya + (uint32_t)((off + 16 * j) * 128), 16384, 1024, kSwizzle128B);
 #pragma unroll
-                    for (int pp = 0; pp < kWgWinAcc; ++pp) {
-                        const int t0 = 2 * pp, t1 = 2 * pp + 1;
-                        const int o0 = (t0 / 3) * Wp + t0 % 3;
-                        const int o1 = t1 < 9 ? (t1 / 3) * Wp + t1 % 3 : o0 + 1;
-                        const uint64_t ad =
-                            smem_desc(xa + (uint32_t)((off + o0 + 16 * j) * 128), (uint32_t)((o1 - o0) * 128), 1024,
-                                      kSwizzle128B);
+                    for (int pp = 0; pp < NACC; ++pp) {
+                        const uint64_t ad = smem_desc(xa + (uint32_t)((off + o0[pp] + 16 * j) * 128),
+                                                      (uint32_t)((o1[pp] - o0[pp]) * 128), 1024, kSwizzle128B);
                         mma_bf16_elect(tmem + (uint32_t)(pp * 64), ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
                     }
                 }
@@ -991,9 +1007,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int kb0 = z * p.kb_per_split;
             const bool have_acc = min(p.num_kb, kb0 + p.kb_per_split) > kb0;
 #pragma unroll 1
-            for (int pp = 0; pp < kWgWinAcc; ++pp) {
+            for (int pp = 0; pp < NACC; ++pp) {
                 const int tap = 2 * pp + (i >> 6), c = i & 63;
-                const bool valid = tap < 9;
+                const bool valid = tap < ntaps;
                 const int m = tap * 64 + c;  // row of dW viewed as [k][(r, s, c)]
 #pragma unroll 1
                 for (int ch = 0; ch < 2; ++ch) {
@@ -1182,39 +1198,55 @@ int grid_size(int total_tiles)
 // static barriers and 1 KB of alignment slack).
 constexpr size_t kWinSmemMax = 232448 - 2048;
 
-// Window-kernel eligibility and geometry (see conv_win_kernel): 3x3 filters,
-// stride 1 and pad 1 on both axes, 64-channel blocks of the reduced operand
-// (red_c), 64 or 128 output channels, images 8..254 wide.
-bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, Plan& pl)
+// Positions per tile of the window kernels: 256 (any start), or, for rows of at
+// least 64 positions, the whole rows that fit in 256 (row-aligned starts need no
+// strip row for a misaligned start).
+int win_tile_positions(int Wp) { return Wp >= 64 ? (kWinBMT / Wp) * Wp : kWinBMT; }
+
+// Window-kernel eligibility and geometry (see conv_win_kernel): stride 1 on both
+// axes, 64-channel blocks of the reduced operand (red_c), 64 or 128 output
+// channels, padded rows of 10..256 positions; the data gradient (dgrad) for
+// 3x3 filters with pad 1 only (its taps are the forward taps flipped).
+bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& pl)
 {
     const Geom g = geom(s);
-    if (s->r != 3 || s->s != 3 || g.sh != 1 || g.sw != 1 || g.ph != 1 || g.pw != 1) return false;
-    if (red_c % 64 != 0 || (out_c != 64 && out_c != 128)) return false;
-    const int Wp = s->w + 2, Hp = s->h + 2;
+    if (g.sh != 1 || g.sw != 1) return false;
+    if (dgrad && (s->r != 3 || s->s != 3 || g.ph != 1 || g.pw != 1)) return false;
+    if (s->r * s->s > 16 || red_c % 64 != 0 || (out_c != 64 && out_c != 128)) return false;
+    const int Wp = s->w + 2 * g.pw, Hp = s->h + 2 * g.ph;
     if (Wp < 10 || Wp > 256) return false;
+    const int P = Hp - s->r + 1, Q = Wp - s->s + 1;
+    if (P <= 0 || Q <= 0) return false;
     const int64_t L = (int64_t)s->n * Hp * Wp;
     if (L > INT32_MAX / 4) return false;
-    // a tile's rows start anywhere in a padded row and reach 2*Wp + 2 positions past its end
-    const int srows = kWinBMT / Wp + 4;
+    const int tile = win_tile_positions(Wp);
+    // rows one tile's 256 accumulator rows read: start offset within a row, plus 255, plus the last tap's offset
+    const int max_index = (tile % Wp == 0 ? 0 : Wp - 1) + kWinBMT - 1 + (s->r - 1) * Wp + (s->s - 1);
+    const int srows = max_index / Wp + 1;
     const int strip = ((srows * Wp * 128 + 1023) / 1024) * 1024;
-    const int BN = out_c, CB = red_c / 64;
-    const bool res = BN == 64 && CB == 1;
-    const int b_bytes = res ? 9 * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128;
+    const int BN = out_c, CB = red_c / 64, ntaps = s->r * s->s;
+    const bool res = BN == 64 && CB == 1 && ntaps <= 9;
+    const int b_bytes = res ? ntaps * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128;
     const size_t smem = (size_t)b_bytes + 2 * (size_t)strip + kEpiTileBytes + 4 * 2 * (size_t)out_c * 4 + 1024;
-    if (smem > kWinSmemMax) return false;
+    if (smem > kWinSmemMax || (size_t)srows * Wp * 128 >= (1u << 20)) return false;
     ConvParams& p = pl.p;
     pl.win = true;
     pl.res = res;
     pl.BN = BN;
     pl.smem = smem;
-    p.win_H = s->h;
-    p.win_W = s->w;
+    p.win_R = s->r;
+    p.win_S = s->s;
+    p.win_ph = g.ph;
+    p.win_pw = g.pw;
+    p.win_P = P;
+    p.win_Q = Q;
     p.win_Hp = Hp;
     p.win_Wp = Wp;
+    p.win_tile = tile;
     p.win_srows = srows;
     p.win_strip_bytes = strip;
-    p.M = s->n * s->h * s->w;
-    p.m_tiles = (int)((L + kWinBMT - 1) / kWinBMT);
+    p.M = s->n * P * Q;
+    p.m_tiles = (int)((L + tile - 1) / tile);
     p.n_tiles = 1;
     p.cblocks = CB;
     p.gN = s->n;
@@ -1224,21 +1256,29 @@ bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, Plan& pl)
     return true;
 }
 
-// Window weight-gradient eligibility and geometry (see conv_wgwin_kernel): 3x3
-// filters, stride 1 and pad 1, 64 input and 64 output channels, images 8..254 wide.
+// Window weight-gradient eligibility and geometry (see conv_wgwin_kernel):
+// stride 1, 64 input and 64 output channels, at most 10 taps, padded rows of
+// 10..256 positions.
 bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
 {
     const Geom g = geom(s);
-    if (s->r != 3 || s->s != 3 || g.sh != 1 || g.sw != 1 || g.ph != 1 || g.pw != 1) return false;
+    if (g.sh != 1 || g.sw != 1) return false;
     if (s->c != 64 || s->k != 64) return false;
-    const int Wp = s->w + 2, Hp = s->h + 2;
+    const int ntaps = s->r * s->s;
+    if ((ntaps + 1) / 2 != 2 && (ntaps + 1) / 2 != 5) return false;  // the instantiated accumulator counts
+    const int Wp = s->w + 2 * g.pw, Hp = s->h + 2 * g.ph;
     if (Wp < 10 || Wp > 256) return false;
+    const int P = Hp - s->r + 1, Q = Wp - s->s + 1;
+    if (P <= 0 || Q <= 0) return false;
     const int64_t L = (int64_t)s->n * Hp * Wp;
     if (L > INT32_MAX / 4) return false;
-    // a K-block starts anywhere in a padded row; x reaches 2*Wp + 3 positions past its end
-    // (the unused tenth tap), dy none
-    const int xrows = (kWgWinKB + 3 * Wp + 1) / Wp + 1;
-    const int dyrows = (kWgWinKB + Wp - 2) / Wp + 1;
+    // K-block: two whole padded rows when that is a multiple of 16 positions (no misaligned start), else 256
+    const int kb = (Wp >= 64 && 2 * Wp <= kWgWinKB && (2 * Wp) % 16 == 0) ? 2 * Wp : kWgWinKB;
+    const int start = kb % Wp == 0 ? 0 : Wp - 1;
+    auto off = [&](int t) { return (t / s->s) * Wp + t % s->s; };
+    const int last = (ntaps % 2) ? off(ntaps - 1) + 1 : off(ntaps - 1);  // the unused half of an odd last pair
+    const int xrows = (start + kb - 1 + last) / Wp + 1;
+    const int dyrows = (start + kb - 1) / Wp + 1;
     const int xalign = ((xrows * Wp * 128 + 1023) / 1024) * 1024;
     const int stage = xalign + ((dyrows * Wp * 128 + 1023) / 1024) * 1024;
     const size_t smem = 2 * (size_t)stage + 1024;
@@ -1248,18 +1288,23 @@ bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
     pl.BN = 64;
     pl.smem = smem;
     pl.mode = p.mode = kWgrad;
-    p.win_H = s->h;
-    p.win_W = s->w;
+    p.win_R = s->r;
+    p.win_S = s->s;
+    p.win_ph = g.ph;
+    p.win_pw = g.pw;
+    p.win_P = P;
+    p.win_Q = Q;
     p.win_Hp = Hp;
     p.win_Wp = Wp;
+    p.win_tile = kb;
     p.win_srows = xrows;
     p.win_dyrows = dyrows;
     p.win_strip_bytes = stage;
-    p.M = 9 * 64;
+    p.M = ntaps * 64;
     p.Ncols = 64;
     p.m_tiles = p.n_tiles = 1;
     p.gN = s->n;
-    p.num_kb = (int)((L + kWgWinKB - 1) / kWgWinKB);
+    p.num_kb = (int)((L + kb - 1) / kb);
     // one contiguous range of K-blocks per CTA of a persistent grid
     int splits = grid_size(p.num_kb);
     p.kb_per_split = (p.num_kb + splits - 1) / splits;
@@ -1283,10 +1328,10 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
     p.S = s->s;
     p.Cin = s->c;
     p.zdim = 1;
-    if (pass == DBL_PASS_FWD && !c8 && win_setup(s, s->c, s->k, pl)) {
+    if (pass == DBL_PASS_FWD && !c8 && win_setup(s, s->c, s->k, false, pl)) {
         pl.mode = p.mode = kFwd;
         pl.ws_main = (size_t)kMaxGrid * 2 * s->k * sizeof(float);
-    } else if (pass == DBL_PASS_DGRAD && s->c % 64 == 0 && win_setup(s, s->k, s->c, pl)) {
+    } else if (pass == DBL_PASS_DGRAD && s->c % 64 == 0 && win_setup(s, s->k, s->c, true, pl)) {
         pl.mode = p.mode = kDgrad;
     } else if (pass == DBL_PASS_WGRAD && wgwin_setup(s, pl)) {
         // conv_wgwin_kernel: tiles are the split-K ranges
@@ -1502,6 +1547,22 @@ int launch_win(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int g
     return dg ? launch_win_cfg<64, true, false>(pl, a, b, grid, st) : launch_win_cfg<64, false, false>(pl, a, b, grid, st);
 }
 
+template <int NACC>
+int launch_wgwin(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t st)
+{
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(conv_wgwin_kernel<NACC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kWinSmemMax);
+        if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
+        attr_set[dev] = true;
+    }
+    conv_wgwin_kernel<NACC><<<grid_size(pl.p.zdim), kWinThreads, pl.smem, st>>>(a, b, pl.p);
+    return dbl::launch_check("conv_wgwin launch");
+}
+
 // Tensor map of the window kernel's strip operand: one padded row (Wp pixels
 // x 64 channels, starting at w = -1) of an NHWC tensor per copy.
 int enc_win_rows(CUtensorMap* m, const void* base, int N, int H, int W, int C, int Wp)
@@ -1637,18 +1698,8 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
         if ((rc = enc_win_rows(&tb, dy, s->n, P, Q, s->k, pl.p.win_Wp))) return rc;
         pl.p.out = sliced ? ws : static_cast<void*>(dw);
         pl.p.wg_accumulate = accumulate;
-        static bool attr_set[64] = {false};
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-            if ((rc = cuda_check(cudaFuncSetAttribute(conv_wgwin_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                      (int)kWinSmemMax),
-                                 "conv: set smem attribute")))
-                return rc;
-            attr_set[dev] = true;
-        }
-        conv_wgwin_kernel<<<grid_size(pl.p.zdim), kWinThreads, pl.smem, st>>>(ta, tb, pl.p);
-        if ((rc = launch_check("conv_wgwin launch"))) return rc;
+        const int nacc = (pl.p.win_R * pl.p.win_S + 1) / 2;
+        if ((rc = nacc == 5 ? launch_wgwin<5>(pl, ta, tb, st) : launch_wgwin<2>(pl, ta, tb, st))) return rc;
     } else {
     const bool c8 = pl.mode == kWgradC8;
     if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh, g.sw,

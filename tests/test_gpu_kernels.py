@@ -137,6 +137,8 @@ STEM_CASES = [  # n, h (square input), r, stride, pad
     (2, 20, 7, 2, 3),    # ImageNet stem on a small image
     (3, 10, 3, 1, 1),    # CIFAR stem
     (4, 64, 7, 2, 3),    # several tiles
+    (2, 224, 7, 2, 3),   # full size: window tiles of two 112-wide rows, two-row weight-gradient K-blocks
+    (1, 160, 7, 2, 3),   # tiles of three 80-wide rows
 ]
 
 
