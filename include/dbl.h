@@ -190,6 +190,19 @@ DBL_API int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* shape, const void*
                                           const float* save_invstd, void* dy_bf16, void* dresidual_bf16 /* or NULL */,
                                           float* dgamma, float* dbeta, void* stream);
 
+/* dbl_bn_relu_fused (no residual, relu set) followed by dbl_maxpool_fwd of
+ * its output, without storing that output: y, argmax as from
+ * dbl_maxpool_fwd of bf16(ReLU(x*scale + shift)), with the statistics
+ * finalized from ch_sum/ch_sumsq exactly as dbl_bn_relu_fused does (it also
+ * writes save_mean/save_invstd).  The ImageNet stem's BatchNorm + ReLU +
+ * 3x3/2 max pool (ResNet-18, Sec. 5.1.1).  shape: count = n*h*w rows of c
+ * channels; x: [n,h,w,c] bf16 (the BatchNorm input).  The backward pass
+ * recomputes the ReLU mask from x (dbl_bn_relu_fused_bwd with out = NULL). */
+DBL_API int dbl_bn_relu_maxpool_fwd(const dbl_bn_shape* shape, int32_t n, int32_t h, int32_t w, const void* x_bf16,
+                                    const float* ch_sum, const float* ch_sumsq, const float* gamma, const float* beta,
+                                    float* save_mean, float* save_invstd, void* y_bf16, uint8_t* argmax,
+                                    void* stream);
+
 /* ========================================================================
  * Stem max pooling (ImageNet ResNet-18): 3x3 window, stride 2, padding 1,
  * padding counted as -infinity.  x: [n,h,w,c] bf16, y: [n,P,Q,c] bf16,

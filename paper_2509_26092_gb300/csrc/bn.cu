@@ -15,6 +15,7 @@
 
 namespace {
 
+using dbl::dev::bn_scale_shift;
 using dbl::dev::colsum_fixed_order;
 using dbl::dev::kColsumGroups;
 
@@ -101,15 +102,6 @@ __global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const fl
     save_invstd[c] = (float)(1.0 / sqrt(var + (double)eps));
 }
 
-// Per-channel scale and shift of out = y*scale + shift from the saved
-// statistics, in fp32 with explicit rounding (no contraction), so that every
-// CTA and the backward pass's ReLU-mask recomputation get the same bits.
-__device__ __forceinline__ void bn_scale_shift(float gamma, float beta, float mean, float invstd, float& scale,
-                                               float& shift)
-{
-    scale = __fmul_rn(gamma, invstd);
-    shift = __fsub_rn(beta, __fmul_rn(mean, scale));
-}
 
 // Thread t of a CTA owns channel group g = t % (C/8) (8 channels, one 16-byte
 // vector) and visits rows t / (C/8), + rows-per-CTA-step, ...; a warp covers
@@ -450,6 +442,17 @@ int bwd_launch(const dbl_bn_shape* s, const void* dout, const void* dout2, const
 
 }  // namespace
 
+namespace dbl {
+
+int bn_fwd_finalize(int64_t count, int C, float eps, const float* sum, const float* sumsq, float* save_mean,
+                    float* save_invstd, cudaStream_t st)
+{
+    bn_fwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(count, C, eps, sum, sumsq, save_mean, save_invstd);
+    return launch_check("bn_fwd_finalize launch");
+}
+
+}  // namespace dbl
+
 extern "C" {
 
 int dbl_bn_stats(const dbl_bn_shape* s, const void* y, float* ch_sum, float* ch_sumsq, void* stream)
@@ -480,9 +483,7 @@ int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum,
         return set_error(DBL_ERR_INVALID, "bn_relu_fused: tensors must be 16-byte aligned");
     if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused: empty batch has no statistics");
     cudaStream_t st = as_stream(stream);
-    bn_fwd_finalize_kernel<<<(s->c + 127) / 128, 128, 0, st>>>(s->count, s->c, s->eps, ch_sum, ch_sumsq, save_mean,
-                                                             save_invstd);
-    if ((rc = launch_check("bn_fwd_finalize launch"))) return rc;
+    if ((rc = bn_fwd_finalize(s->count, s->c, s->eps, ch_sum, ch_sumsq, save_mean, save_invstd, st))) return rc;
     bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
         static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
         static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);

@@ -50,6 +50,11 @@ typedef CUresult (*PFN_encodeIm2col)(CUtensorMap*, CUtensorMapDataType, cuuint32
 PFN_encodeTiled encode_tiled();
 PFN_encodeIm2col encode_im2col();
 
+// BatchNorm forward finalize (bn.cu): channel sums over count rows -> saved mean and
+// 1/sqrt(var + eps), once per channel in fp64.  Launches on st; returns a status.
+int bn_fwd_finalize(int64_t count, int C, float eps, const float* sum, const float* sumsq, float* save_mean,
+                    float* save_invstd, cudaStream_t st);
+
 }  // namespace dbl
 
 // ---------------------------------------------------------------------------- device helpers
@@ -229,6 +234,18 @@ __device__ __forceinline__ void mbar_arrive_expect_tx_elect(uint64_t* bar, uint3
         "@E mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}" ::"r"(smem_u32(bar)),
         "r"(bytes)
         : "memory");
+}
+
+// ---------------------------------------------------------------------------- BatchNorm scale / shift
+// Per-channel scale and shift of out = y*scale + shift from the saved statistics,
+// in fp32 with explicit rounding (no contraction), so that every kernel that applies
+// the normalisation (bn.cu, the fused stem max pool in head.cu) and the backward
+// pass's ReLU-mask recomputation get the same bits.
+__device__ __forceinline__ void bn_scale_shift(float gamma, float beta, float mean, float invstd, float& scale,
+                                               float& shift)
+{
+    scale = __fmul_rn(gamma, invstd);
+    shift = __fsub_rn(beta, __fmul_rn(mean, scale));
 }
 
 // ---------------------------------------------------------------------------- fixed-order column sums

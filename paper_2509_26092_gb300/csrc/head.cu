@@ -87,6 +87,67 @@ __global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* _
     }
 }
 
+// The same max pool over the output of a training-mode BatchNorm + ReLU
+// (no residual) that is never stored: each input vector is normalised as the
+// BatchNorm pass would store it, bf16(relu(y*scale + shift)) with the same
+// fp32 operations, and then pooled, so the pooled values and the argmax are
+// those of pooling the stored BatchNorm output.
+__global__ void __launch_bounds__(256)
+    bn_relu_maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ gamma,
+                               const float* __restrict__ beta, const float* __restrict__ mean,
+                               const float* __restrict__ invstd, __nv_bfloat16* __restrict__ y,
+                               uint8_t* __restrict__ arg, int n, int H, int W, int C, int P, int Q)
+{
+    const unsigned groups = (unsigned)C / 8u;
+    const unsigned total = (unsigned)n * P * Q * groups;
+    // a thread keeps its channel group across the grid-stride loop when the stride is a multiple of groups
+    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
+        const unsigned g = t % groups;
+        unsigned pix = t / groups;
+        const int q = (int)(pix % (unsigned)Q);
+        pix /= (unsigned)Q;
+        const int p = (int)(pix % (unsigned)P);
+        const int b = (int)(pix / (unsigned)P);
+        float sc[8], sh[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            dbl::dev::bn_scale_shift(gamma[8 * g + k], beta[8 * g + k], mean[8 * g + k], invstd[8 * g + k], sc[k],
+                                     sh[k]);
+        float best[8];
+        uint8_t bi[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            best[k] = -INFINITY;
+            bi[k] = 0;
+        }
+        for (int r = 0; r < 3; ++r) {
+            const int h = 2 * p + r - 1;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < 3; ++s) {
+                const int w = 2 * q + s - 1;
+                if (w < 0 || w >= W) continue;
+                float f[8];
+                unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)b * H + h) * W + w) * C) + g), f);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float o = __fadd_rn(__fmaf_rn(f[k], sc[k], sh[k]), 0.f);
+                    const float a = __bfloat162float(__float2bfloat16_rn(o > 0.f ? o : 0.f));
+                    if (a > best[k]) {  // strict: the first maximum in (r, s) order wins ties
+                        best[k] = a;
+                        bi[k] = (uint8_t)(r * 3 + s);
+                    }
+                }
+            }
+        }
+        const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
+        *reinterpret_cast<uint4*>(y + o) = pack8(best);
+        uint2 packed;
+        packed.x = bi[0] | (bi[1] << 8) | (bi[2] << 16) | ((uint32_t)bi[3] << 24);
+        packed.y = bi[4] | (bi[5] << 8) | (bi[6] << 16) | ((uint32_t)bi[7] << 24);
+        *reinterpret_cast<uint2*>(arg + o) = packed;
+    }
+}
+
 // Gather form over 2x2 blocks of input pixels: block (i, j) = rows 2i..2i+1,
 // cols 2j..2j+1 is covered by windows (i..i+1, j..j+1); window (p, q) reaches
 // input (h, w) at tap (h - 2p + 1, w - 2q + 1).  Each window's argmax and
@@ -180,41 +241,62 @@ __global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __res
 }
 
 // out[m, n] = sum_k A(m,k) * B(n,k) (+ bias[n]); A(m,k) = A[m*sam + k*sak], B(n,k) = B[n*sbn + k*sbk].
-constexpr int GT = 32;
+// fp32 on the CUDA cores (the head is fp32 end to end): 64 x 64 output tiles, 16-deep K tiles
+// stored K-major in shared memory, 4 x 4 outputs per thread from float4 reads.  Each output is a
+// sequential fmaf over k = 0..K-1.  Tile loads are coalesced along whichever index of an operand
+// has unit stride.
+constexpr int GBM = 64, GBN = 64, GBK = 16;
+
+__device__ __forceinline__ void gemm_load_tile(const float* __restrict__ X, int64_t s_row, int64_t s_k, int row0,
+                                               int rows, int k0, int K, float (*dst)[GBM + 4])
+{
+    // dst[k][r] = X(row0 + r, k0 + k), zero outside
+    if (s_k == 1) {  // consecutive threads along k
+        for (int e = threadIdx.x; e < GBM * GBK; e += blockDim.x) {
+            const int r = e / GBK, k = e % GBK;
+            const int row = row0 + r, kk = k0 + k;
+            dst[k][r] = (row < rows && kk < K) ? __ldg(X + (int64_t)row * s_row + kk) : 0.f;
+        }
+    } else {  // consecutive threads along the row index
+        for (int e = threadIdx.x; e < GBM * GBK; e += blockDim.x) {
+            const int k = e / GBM, r = e % GBM;
+            const int row = row0 + r, kk = k0 + k;
+            dst[k][r] = (row < rows && kk < K) ? __ldg(X + (int64_t)row * s_row + (int64_t)kk * s_k) : 0.f;
+        }
+    }
+}
+
 __global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__ A, int64_t sam, int64_t sak,
                                                        const float* __restrict__ B, int64_t sbn, int64_t sbk,
                                                        const float* __restrict__ bias, float* __restrict__ out,
                                                        int64_t ldo, int M, int N, int K)
 {
-    __shared__ float As[GT][GT + 1], Bs[GT][GT + 1];
-    const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;  // 16x16 threads, 2x2 outputs each
-    const int m0 = blockIdx.y * GT, n0 = blockIdx.x * GT;
-    float acc[2][2] = {};
-    for (int k0 = 0; k0 < K; k0 += GT) {
-        for (int e = threadIdx.x; e < GT * GT; e += 256) {
-            const int i = e / GT, j = e % GT;
-            const int m = m0 + i, n = n0 + i, k = k0 + j;
-            As[i][j] = (m < M && k < K) ? A[m * sam + k * sak] : 0.f;
-            Bs[i][j] = (n < N && k < K) ? B[n * sbn + k * sbk] : 0.f;
-        }
+    __shared__ __align__(16) float As[GBK][GBM + 4], Bs[GBK][GBN + 4];
+    const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;  // thread owns rows 4ty.., columns 4tx..
+    const int m0 = blockIdx.y * GBM, n0 = blockIdx.x * GBN;
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < K; k0 += GBK) {
+        gemm_load_tile(A, sam, sak, m0, M, k0, K, As);
+        gemm_load_tile(B, sbn, sbk, n0, N, k0, K, Bs);
         __syncthreads();
-#pragma unroll 8
-        for (int j = 0; j < GT; ++j) {
-            const float a0 = As[ty][j], a1 = As[ty + 16][j];
-            const float b0 = Bs[tx][j], b1 = Bs[tx + 16][j];
-            acc[0][0] = fmaf(a0, b0, acc[0][0]);
-            acc[0][1] = fmaf(a0, b1, acc[0][1]);
-            acc[1][0] = fmaf(a1, b0, acc[1][0]);
-            acc[1][1] = fmaf(a1, b1, acc[1][1]);
+#pragma unroll
+        for (int k = 0; k < GBK; ++k) {
+            const float4 a = *reinterpret_cast<const float4*>(&As[k][4 * ty]);
+            const float4 b = *reinterpret_cast<const float4*>(&Bs[k][4 * tx]);
+            const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
         }
         __syncthreads();
     }
 #pragma unroll
-    for (int i = 0; i < 2; ++i)
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-            const int m = m0 + ty + 16 * i, n = n0 + tx + 16 * j;
-            if (m < M && n < N) out[m * ldo + n] = acc[i][j] + (bias ? bias[n] : 0.f);
+        for (int j = 0; j < 4; ++j) {
+            const int m = m0 + 4 * ty + i, n = n0 + 4 * tx + j;
+            if (m < M && n < N) out[(int64_t)m * ldo + n] = acc[i][j] + (bias ? bias[n] : 0.f);
         }
 }
 
@@ -301,6 +383,31 @@ int dbl_maxpool_fwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* x, v
     return launch_check("maxpool_fwd launch");
 }
 
+int dbl_bn_relu_maxpool_fwd(const dbl_bn_shape* s, int32_t n, int32_t h, int32_t w, const void* x,
+                            const float* ch_sum, const float* ch_sumsq, const float* gamma, const float* beta,
+                            float* save_mean, float* save_invstd, void* y, uint8_t* argmax, void* stream)
+{
+    using namespace dbl;
+    if (!s || n <= 0 || h <= 0 || w <= 0 || !x || !y || !argmax || !ch_sum || !ch_sumsq || !gamma || !beta ||
+        !save_mean || !save_invstd)
+        return set_error(DBL_ERR_INVALID, "bn_relu_maxpool_fwd: bad arguments");
+    const int c = s->c;
+    if (c <= 0 || c % 8 || !s->relu || s->count != (int64_t)n * h * w)
+        return set_error(DBL_ERR_INVALID, "bn_relu_maxpool_fwd: shape must be [n*h*w, c], c a multiple of 8, relu set");
+    if (!aligned16(x) || !aligned16(y) || (reinterpret_cast<uintptr_t>(argmax) & 7))
+        return set_error(DBL_ERR_INVALID, "bn_relu_maxpool_fwd: misaligned pointer");
+    const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
+    if ((int64_t)n * h * w * (c / 8) >= (int64_t)1 << 31)
+        return set_error(DBL_ERR_UNSUPPORTED, "bn_relu_maxpool_fwd: tensor too large for 32-bit indexing");
+    cudaStream_t st = as_stream(stream);
+    int rc = bn_fwd_finalize(s->count, c, s->eps, ch_sum, ch_sumsq, save_mean, save_invstd, st);
+    if (rc) return rc;
+    bn_relu_maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q * (c / 8), 256), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(x), gamma, beta, save_mean, save_invstd, static_cast<__nv_bfloat16*>(y),
+        argmax, n, h, w, c, P, Q);
+    return launch_check("bn_relu_maxpool_fwd launch");
+}
+
 int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, const void* dy2,
                     const uint8_t* argmax, void* dx, void* stream)
 {
@@ -351,7 +458,7 @@ int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const vo
                                                                        hw, c);
     if ((rc = launch_check("avgpool launch"))) return rc;
     // logits = feat * W^T + b
-    dim3 g1((classes + GT - 1) / GT, (n + GT - 1) / GT);
+    dim3 g1((classes + GBN - 1) / GBN, (n + GBM - 1) / GBM);
     gemm_f32_kernel<<<g1, 256, 0, s>>>(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c);
     if ((rc = launch_check("fc fwd launch"))) return rc;
     softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss);
@@ -359,11 +466,11 @@ int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const vo
     head_reduce_kernel<<<1 + (classes + 255) / 256, 256, 0, s>>>(row_loss, logits, n, classes, loss, dfc_b);
     if ((rc = launch_check("head reduce launch"))) return rc;
     // dW[j, c] = sum_n dl[n, j] feat[n, c]
-    dim3 g2((c + GT - 1) / GT, (classes + GT - 1) / GT);
+    dim3 g2((c + GBN - 1) / GBN, (classes + GBM - 1) / GBM);
     gemm_f32_kernel<<<g2, 256, 0, s>>>(logits, 1, classes, feat, 1, c, nullptr, dfc_w, c, classes, c, n);
     if ((rc = launch_check("fc dW launch"))) return rc;
     // df[n, c] = sum_j dl[n, j] W[j, c]
-    dim3 g3((c + GT - 1) / GT, (n + GT - 1) / GT);
+    dim3 g3((c + GBN - 1) / GBN, (n + GBM - 1) / GBM);
     gemm_f32_kernel<<<g3, 256, 0, s>>>(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes);
     if ((rc = launch_check("fc dX launch"))) return rc;
     avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(df, static_cast<__nv_bfloat16*>(dx), n,

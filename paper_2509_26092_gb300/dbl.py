@@ -72,6 +72,7 @@ def lib():
             "dbl_bn_relu_fused_bwd_noalloc": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 13),
             "dbl_maxpool_fwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V]),
             "dbl_maxpool_bwd": (ctypes.c_int, [_I32] * 4 + [_V, _V, _V, _V, _V]),
+            "dbl_bn_relu_maxpool_fwd": (ctypes.c_int, [ctypes.POINTER(BnShape), _I32, _I32, _I32] + [_V] * 10),
             "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
             "dbl_head_fwd_bwd": (ctypes.c_int, [_I32] * 4 + [_V] * 8 + [_V, _SZ, _V]),
             "dbl_ps_dual_batch_merge": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams), _V]),
@@ -194,6 +195,13 @@ def dbl_bn_relu_fused_bwd_noalloc(shape, dout, dout2, y, out, gamma, save_mean, 
     _check(lib().dbl_bn_relu_fused_bwd_noalloc(ctypes.byref(shape), _ptr(dout), _ptr(dout2), _ptr(y), _ptr(out),
                                                _ptr(gamma), _ptr(beta), _ptr(save_mean), _ptr(save_invstd), _ptr(dy),
                                                _ptr(dresidual), _ptr(dgamma), _ptr(dbeta), _stream(stream)))
+
+
+def dbl_bn_relu_maxpool_fwd(shape, n, h, w, x, ch_sum, ch_sumsq, gamma, beta, save_mean, save_invstd, y, argmax,
+                            stream=None):
+    _check(lib().dbl_bn_relu_maxpool_fwd(ctypes.byref(shape), n, h, w, _ptr(x), _ptr(ch_sum), _ptr(ch_sumsq),
+                                         _ptr(gamma), _ptr(beta), _ptr(save_mean), _ptr(save_invstd), _ptr(y),
+                                         _ptr(argmax), _stream(stream)))
 
 
 def dbl_maxpool_fwd(n, h, w, c, x, y, argmax, stream=None):

@@ -243,7 +243,9 @@ class Worker:
         # stem input unrolled (StemLayout): [B, rows, P, 64]
         self.stem_rows = spec.stem_layout.rows(res, p)
         self.x0 = torch.empty((B, self.stem_rows, p, 64), dtype=bf, device=dev)
-        self.stem_y, self.stem_a, self.stem_da, self.stem_dy = act(p, st.cout), act(p, st.cout), None, act(p, st.cout)
+        # the ImageNet stem's BatchNorm output is pooled on the fly and never stored
+        self.stem_a = act(p, st.cout) if spec.variant != "imagenet" else None
+        self.stem_y, self.stem_da, self.stem_dy = act(p, st.cout), None, act(p, st.cout)
         self.stem_stats = [vec(st.cout) for _ in range(4)]  # sum, sumsq, mean, invstd
         h = p
         if spec.variant == "imagenet":
@@ -363,12 +365,16 @@ class Worker:
         s_sum, s_sq, s_mean, s_istd = self.stem_stats
         D.dbl_conv_fwd(shp, self.x0, wv("conv1.w"), self.stem_y, s_sum, s_sq, ws, wsb, s)
         bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)
-        D.dbl_bn_relu_fused(bns, self.stem_y, s_sum, s_sq, pv("bn1.g"), pv("bn1.b"), None, self.stem_a, s_mean, s_istd,
-                            s)
-        cur = self.stem_a
         if spec.variant == "imagenet":
-            D.dbl_maxpool_fwd(B, self.stem_hw, self.stem_hw, st.cout, self.stem_a, self.pool_out, self.pool_arg, s)
+            # BatchNorm + ReLU + max pool in one pass: the BatchNorm output is never stored (its
+            # ReLU mask is recomputed in the backward pass)
+            D.dbl_bn_relu_maxpool_fwd(bns, B, self.stem_hw, self.stem_hw, self.stem_y, s_sum, s_sq, pv("bn1.g"),
+                                      pv("bn1.b"), s_mean, s_istd, self.pool_out, self.pool_arg, s)
             cur = self.pool_out
+        else:
+            D.dbl_bn_relu_fused(bns, self.stem_y, s_sum, s_sq, pv("bn1.g"), pv("bn1.b"), None, self.stem_a, s_mean,
+                                s_istd, s)
+            cur = self.stem_a
         for d in self.blocks:
             b = d["spec"]
             d["x"] = cur

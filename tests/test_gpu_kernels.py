@@ -235,6 +235,30 @@ def test_bn_fwd_bwd_match_oracle(D, count, C, relu, res):
     check_status(D)
 
 
+def test_bn_relu_maxpool_equals_bn_then_maxpool(D):
+    """The fused stem pass equals the BatchNorm pass followed by the max pool, bit for bit."""
+    n, H, W, C = 3, 20, 18, 64
+    g = rng(77)
+    y = bf16_values(g.standard_normal((n, H, W, C)) * 2.0 + 0.3)
+    gamma = (1.0 + 0.2 * g.standard_normal(C)).astype(np.float32)
+    beta = (0.1 * g.standard_normal(C)).astype(np.float32)
+    yd, gd, bd = to_bf16_dev(y), to_f32_dev(gamma), to_f32_dev(beta)
+    shape = D.bn_shape(n * H * W, C, 1e-5, True)
+    s1, s2 = torch.empty(C, device="cuda"), torch.empty(C, device="cuda")
+    D.dbl_bn_stats(shape, yd, s1, s2)
+    P, Q = (H - 1) // 2 + 1, (W - 1) // 2 + 1
+    out = torch.empty((n, H, W, C), dtype=torch.bfloat16, device="cuda")
+    m1, i1, m2, i2 = (torch.empty(C, device="cuda") for _ in range(4))
+    D.dbl_bn_relu_fused(shape, yd, s1, s2, gd, bd, None, out, m1, i1)
+    y1 = torch.empty((n, P, Q, C), dtype=torch.bfloat16, device="cuda")
+    a1 = torch.empty((n, P, Q, C), dtype=torch.uint8, device="cuda")
+    D.dbl_maxpool_fwd(n, H, W, C, out, y1, a1)
+    y2, a2 = torch.empty_like(y1), torch.empty_like(a1)
+    D.dbl_bn_relu_maxpool_fwd(shape, n, H, W, yd, s1, s2, gd, bd, m2, i2, y2, a2)
+    assert torch.equal(y1, y2) and torch.equal(a1, a2) and torch.equal(m1, m2) and torch.equal(i1, i2)
+    check_status(D)
+
+
 # ----------------------------------------------------------------------------- max pool
 @pytest.mark.parametrize("n,h,w,c,zeros", [(2, 9, 10, 64, False), (2, 16, 16, 64, True), (1, 112, 112, 64, True)])
 def test_maxpool_matches_oracle(D, n, h, w, c, zeros):

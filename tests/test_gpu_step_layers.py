@@ -56,12 +56,17 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
     w_stem = W16["conv1.w"][:, :st.r, :st.r, :3]
     chk("stem.conv", h(wk.stem_y), orc.conv2d_fwd(x0, w_stem, st.stride, st.pad))
     o, m, s = orc.bn_fwd(h(wk.stem_y), P["bn1.g"], P["bn1.b"], eps, relu=True)
-    chk("stem.bn", h(wk.stem_a), o)
     chk("stem.bn.mean", h(wk.stem_stats[2]), m, 1e-4)
     if variant == "imagenet":
-        y, arg = orc.maxpool_fwd(h(wk.stem_a))
-        chk("stem.pool", h(wk.pool_out), y, 0.0)
-        np.testing.assert_array_equal(wk.pool_arg.cpu().numpy().astype(np.int32), arg)
+        # the BatchNorm output is pooled on the fly (never stored): pool the oracle's stored values
+        stem_a = orc.round_bf16(o)
+        y, arg = orc.maxpool_fwd(stem_a)
+        chk("stem.bn.pool", h(wk.pool_out), y)
+        agree = np.mean(wk.pool_arg.cpu().numpy().astype(np.int32) == arg)
+        assert agree > 0.999, f"argmax agreement {agree}"  # ties may fall either way within one bf16 ulp
+    else:
+        stem_a = h(wk.stem_a)
+        chk("stem.bn", stem_a, o)
     for d in wk.blocks:
         b = d["spec"]
         x = h(d["x"])
@@ -126,12 +131,11 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
         dout, dout2 = h(d["din"]), h(d["din2"])
     s_stats = [h(t) for t in wk.stem_stats]
     if variant == "imagenet":
-        da = orc.maxpool_bwd(dout + dout2, wk.pool_arg.cpu().numpy().astype(np.int32), wk.stem_a.shape)
+        da = orc.maxpool_bwd(dout + dout2, wk.pool_arg.cpu().numpy().astype(np.int32), stem_a.shape)
         chk("stem.pool.bwd", h(wk.stem_da), da)
-        dys, dgs, dbs, _ = orc.bn_bwd(h(wk.stem_da), h(wk.stem_a), h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3])
+        dys, dgs, dbs, _ = orc.bn_bwd(h(wk.stem_da), stem_a, h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3])
     else:
-        dys, dgs, dbs, _ = orc.bn_bwd(dout, h(wk.stem_a), h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3],
-                                      dout2=dout2)
+        dys, dgs, dbs, _ = orc.bn_bwd(dout, stem_a, h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3], dout2=dout2)
     chk("stem.bn.bwd", h(wk.stem_dy), dys)
     wst = orc.conv2d_wgrad(x0, h(wk.stem_dy), w_stem.shape, st.stride, st.pad)
     chk("stem.wgrad", G["conv1.w"][:, :st.r, :st.r, :3], wst)
