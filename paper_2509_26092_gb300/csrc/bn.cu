@@ -216,13 +216,17 @@ __device__ __forceinline__ void combine_g(const Vec8& raw, const float (&y)[8], 
 }
 
 // sg += g, sgc += g*(y - mean)  (the 1/std factor is applied once per partial)
-template <int MASK>
+// WRITE_G: also store g (bf16) at vector v of g_out.  The sums are of the fp32 g (the
+// dgamma, dbeta outputs keep fp32 accuracy); the apply pass then reads the stored g.
+template <int MASK, bool WRITE_G>
 __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw, bool two, const ReluMask<MASK>& relu,
-                                             const float (&mu)[8], float (&sg)[8], float (&sgc)[8])
+                                             const float (&mu)[8], float (&sg)[8], float (&sgc)[8],
+                                             __nv_bfloat16* g_out, int v)
 {
     float gg[8], yy[8];
     unpack8(yraw.y, yy);
     combine_g(graw, yy, two, relu, gg);
+    if constexpr (WRITE_G) __stcs(reinterpret_cast<uint4*>(g_out) + v, pack8(gg));
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         sg[k] += gg[k];
@@ -233,13 +237,13 @@ __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw,
 // Partial blk reduces a contiguous range of rows into partial[blk][0..C) (sum g)
 // and partial[blk][C..2C) (sum g*xhat); CTA b computes partials b, b + gridDim.x, ...
 // (each in a fixed order, so the result does not depend on the grid).
-template <int MASK>
+template <int MASK, bool WRITE_G>
 __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
                          const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
                          int C, const float* __restrict__ gamma, const float* __restrict__ beta,
                          const float* __restrict__ mean, const float* __restrict__ invstd, int rows_per_blk, int nblk,
-                         float* __restrict__ partial)
+                         float* __restrict__ partial, __nv_bfloat16* __restrict__ g_out)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
@@ -261,12 +265,14 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) load_g_raw<MASK>(dout, dout2, out, y, (r + u * rstep) * groups + g, gg[u], yy[u]);
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) accumulate_g(gg[u], yy[u], dout2 != nullptr, rm, mu, sg, sgx);
+        for (int u = 0; u < kUnroll; ++u)
+            accumulate_g<MASK, WRITE_G>(gg[u], yy[u], dout2 != nullptr, rm, mu, sg, sgx, g_out,
+                                        (r + u * rstep) * groups + g);
     }
     for (; r < r1; r += rstep) {
         Vec8 gg, yy;
         load_g_raw<MASK>(dout, dout2, out, y, r * groups + g, gg, yy);
-        accumulate_g(gg, yy, dout2 != nullptr, rm, mu, sg, sgx);
+        accumulate_g<MASK, WRITE_G>(gg, yy, dout2 != nullptr, rm, mu, sg, sgx, g_out, r * groups + g);
     }
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -410,17 +416,30 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
     using namespace dbl;
     const int C = s->c;
     auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
-    bn_bwd_reduce_kernel<MASK><<<reduce_grid(nblk), kThreads, 0, st>>>(bd(dout), bd(dout2), bd(out), bd(y),
-                                                                       (int)s->count, C, gamma, beta, mean, invstd,
-                                                                       rows, (int)nblk, partial);
+    // When the caller wants g (the residual branch's gradient), the reduce pass stores it and the
+    // apply pass reads it back instead of re-reading dout, dout2 and out.
+    __nv_bfloat16* g_store = static_cast<__nv_bfloat16*>(dresidual);
+    if (g_store)
+        bn_bwd_reduce_kernel<MASK, true><<<reduce_grid(nblk), kThreads, 0, st>>>(
+            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, rows, (int)nblk, partial,
+            g_store);
+    else
+        bn_bwd_reduce_kernel<MASK, false><<<reduce_grid(nblk), kThreads, 0, st>>>(
+            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, rows, (int)nblk, partial,
+            nullptr);
     int rc = launch_check("bn_bwd_reduce launch");
     if (rc) return rc;
     bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
                                                                          invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
-    bn_bwd_apply_kernel<MASK><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
-        bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
-        static_cast<__nv_bfloat16*>(dy), static_cast<__nv_bfloat16*>(dresidual));
+    if (g_store)
+        bn_bwd_apply_kernel<kMaskNone><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
+            g_store, nullptr, nullptr, bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
+            static_cast<__nv_bfloat16*>(dy), nullptr);
+    else
+        bn_bwd_apply_kernel<MASK><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
+            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
+            static_cast<__nv_bfloat16*>(dy), nullptr);
     return launch_check("bn_bwd_apply launch");
 }
 

@@ -262,6 +262,7 @@ class Worker:
                 d[k] = act(ho if k not in ("din", "din2") else h, b.cout if k not in ("din", "din2") else b.cin)
             if b.proj:
                 d["hs"], d["sc"], d["dhs"] = act(ho, b.cout), act(ho, b.cout), act(ho, b.cout)
+                d["gout"] = act(ho, b.cout)  # the masked output gradient, input of the shortcut BatchNorm
             for k in ("bn1", "bn2", "downbn"):
                 d[k] = [vec(b.cout) for _ in range(4)]
             self.blocks.append(d)
@@ -409,9 +410,11 @@ class Worker:
             b = d["spec"]
             cnt = B * d["hout"] ** 2
             st1, st2, std = d["bn1"], d["bn2"], d["downbn"]
-            dres = None if b.proj else d["din2"]
+            # g = (dout + dout2) * [out > 0] is kept: the identity shortcut's gradient, or the
+            # projection shortcut BatchNorm's incoming gradient
+            g = d["gout"] if b.proj else d["din2"]
             D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), dout, dout2, d["h2"], d["out"],
-                                    pv(b.pre + ".bn2.g"), st2[2], st2[3], d["dh2"], dres, gv(b.pre + ".bn2.g"),
+                                    pv(b.pre + ".bn2.g"), st2[2], st2[3], d["dh2"], g, gv(b.pre + ".bn2.g"),
                                     gv(b.pre + ".bn2.b"), ws, wsb, s)
             s2 = D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)
             D.dbl_conv_wgrad(s2, d["o1"], d["dh2"], gv(b.pre + ".conv2.w"), False, ws, wsb, s)
@@ -424,8 +427,8 @@ class Worker:
             D.dbl_conv_wgrad(s1, d["x"], d["dh1"], gv(b.pre + ".conv1.w"), False, ws, wsb, s)
             D.dbl_conv_dgrad(s1, d["dh1"], wv(b.pre + ".conv1.w"), d["din"], None, 0, s)
             if b.proj:
-                # the shortcut BatchNorm sees the same masked gradient as bn2
-                D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, True), dout, dout2, d["hs"], d["out"],
+                # the shortcut BatchNorm sees the same masked gradient g as bn2 (no ReLU of its own)
+                D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, False), g, None, d["hs"], None,
                                         pv(b.pre + ".downbn.g"), std[2], std[3], d["dhs"], None,
                                         gv(b.pre + ".downbn.g"), gv(b.pre + ".downbn.b"), ws, wsb, s)
                 sd = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)
