@@ -34,7 +34,6 @@ namespace {
 using namespace dbl::dev;
 
 constexpr int BM = 128;        // tile rows = TMEM lanes
-constexpr int kTargetCTAs = 304;  // 2 x 152 SMs: split-K sizing target (device independent)
 
 enum Mode : int { kFwd = 0, kDgrad = 1, kWgrad = 2, kFwdC8 = 3, kWgradC8 = 4 };
 
@@ -1184,6 +1183,34 @@ int validate(const dbl_conv_shape* s, const char* who)
     return DBL_OK;
 }
 
+// Split-K slices of the implicit-GEMM weight gradient: the count that minimises the
+// modelled time of the persistent grid on a 152-SM GPU, where the busiest CTA runs
+// ceil(units / 152) units of (K-blocks per slice + ~2 K-blocks of epilogue) and the
+// fixed-order reduce afterwards reads every slice (one K-block of a 128 x BN tile is
+// ~4 BN tensor cycles, in which the GPU streams ~10.5 KB x BN).  At least 4 K-blocks
+// (512 pixels) per slice.  A fixed function of the shape, so the summation order, and
+// with it the result, does not depend on the device the plan runs on.
+int wgrad_splits(int tiles, int num_kb, int rows, int cols, int BN)
+{
+    constexpr int kPlanSMs = 152;
+    const double slice_cost = (double)rows * cols * 4 / (10.5e3 * BN);  // K-block times to reduce one slice
+    int best = 1;
+    double best_cost = 1e300;
+    const int max_splits = std::max(1, num_kb / 4);
+    for (int sp = 1; sp <= max_splits; ++sp) {
+        const int kbs = (num_kb + sp - 1) / sp;
+        const int eff = (num_kb + kbs - 1) / kbs;  // slices actually used
+        if (eff != sp) continue;
+        const int rounds = (tiles * sp + kPlanSMs - 1) / kPlanSMs;
+        const double cost = rounds * (kbs + 2.0) + (sp > 1 ? sp * slice_cost : 0.0);
+        if (cost < best_cost) {
+            best_cost = cost;
+            best = sp;
+        }
+    }
+    return best;
+}
+
 // Persistent grid: one CTA per SM (the kernel uses ~225 KB of shared memory), never more
 // CTAs than tiles, never more than kMaxGrid (the workspace is sized for that bound).
 int grid_size(int total_tiles)
@@ -1440,14 +1467,8 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         const int64_t pix = (int64_t)s->n * P * Q;
         if ((pix + 127) / 128 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
         p.num_kb = (int)((pix + 127) / 128);  // K-blocks of 128 output pixels
-        const int tiles = p.m_tiles * p.n_tiles;
-        // split the pixel reduction so that there are about two tiles per SM of a 152-SM GPU,
-        // keeping at least 4 K-blocks (512 pixels) per slice (a fixed function of the shape)
-        int splits = (kTargetCTAs + tiles - 1) / tiles;
-        if (splits > p.num_kb / 4) splits = p.num_kb / 4;
-        if (splits < 1) splits = 1;
+        const int splits = wgrad_splits(p.m_tiles * p.n_tiles, p.num_kb, p.M, s->k, pl.BN);
         p.kb_per_split = (p.num_kb + splits - 1) / splits;
-        splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
         p.zdim = splits;
         pl.ws_main = splits > 1 ? (size_t)splits * p.M * s->k * sizeof(float) : 0;
     }
