@@ -252,14 +252,16 @@ def build_pipeline(cfg, device):
                 lab_s=lab_s)
 
 
-def conv_roofline(stage, reps=3, table=None):
-    """Time each convolution pass of the stage's workers alone with CUDA events;
-    return (algorithmic conv FLOPs of one iteration, seconds per iteration).
-    If table is a list, append (worker batch, layer, pass, FLOPs, seconds) per pass."""
+def conv_roofline(stage, reps=4, replays=2, table=None):
+    """Time each convolution pass of the stage's workers alone with CUDA events:
+    `reps` calls of the pass are captured in one CUDA graph (as in the training
+    iteration, so no host-side launch gap sits between the events) and the graph
+    is replayed `replays` times.  Return (algorithmic conv FLOPs of one iteration,
+    seconds per iteration, algorithmic bytes).  If table is a list, append
+    (worker batch, layer, pass, FLOPs, seconds) per pass."""
     import torch
 
     from paper_2509_26092_gb300 import dbl as D
-    s = torch.cuda.current_stream()
     flops, secs = 0.0, 0.0
     nbytes = lambda *ts: sum(t.numel() * t.element_size() for t in ts)
     algo_bytes = 0  # unique operand bytes of every pass (inputs + weights + outputs)
@@ -273,22 +275,30 @@ def conv_roofline(stage, reps=3, table=None):
             st_sum = torch.empty(shp.k, device=x.device)
             st_sq = torch.empty(shp.k, device=x.device)
             f1 = float(wk.layer_flops(name, shp))
-            passes = [("fwd", lambda: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            passes = [("fwd", lambda s: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
             algo_bytes += nbytes(x, w16, y)
             if name != stem:
-                passes.append(("dgrad", lambda: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
+                passes.append(("dgrad", lambda s: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
                 algo_bytes += nbytes(dy, w16, dx)
-            passes.append(("wgrad", lambda: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
+            passes.append(("wgrad", lambda s: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
             algo_bytes += nbytes(x, dy, g)
             for pname, fn in passes:
-                fn()
+                fn(torch.cuda.current_stream())
+                torch.cuda.synchronize()
+                graph = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph):
+                    for _ in range(reps):
+                        fn(torch.cuda.current_stream())
+                graph.replay()
+                s = torch.cuda.current_stream()
                 ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
                 ev[0].record(s)
-                for _ in range(reps):
-                    fn()
+                for _ in range(replays):
+                    graph.replay()
                 ev[1].record(s)
                 torch.cuda.synchronize()
-                t1 = ev[0].elapsed_time(ev[1]) / 1000.0 / reps
+                del graph
+                t1 = ev[0].elapsed_time(ev[1]) / 1000.0 / (reps * replays)
                 secs += t1
                 flops += f1
                 if table is not None:
@@ -536,8 +546,10 @@ def run_ours(args, cfg):
                 "scope": f"one dual-batch iteration at {top['res']} px: every conv pass of both workers "
                          "(achieved = algorithmic FLOPs / summed CUDA-event time of the passes; traffic = ncu "
                          "DRAM bytes of the same launches, null if the kernel changed since the capture)",
-                "kernel": "conv_igemm_kernel (fwd/dgrad/wgrad, every layer of both workers at "
-                          f"{top['res']} px, each ABI call timed alone)", "peak_source": src}
+                "kernel": "conv_igemm_kernel, conv_win_kernel, conv_wgwin_kernel with their channel-sum and "
+                          f"split-K reduce kernels (fwd/dgrad/wgrad, every layer of both workers at {top['res']} px, "
+                          "each pass timed alone as CUDA-graph replays of its ABI calls)",
+                "peak_source": src}
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         v, dt, images, sample = time_oracle(cfg)

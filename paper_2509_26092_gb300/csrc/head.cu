@@ -8,6 +8,8 @@
 // products are done by a small tiled fp32 GEMM on the CUDA cores.
 #include <float.h>
 
+#include <algorithm>
+
 #include "dbl_internal.cuh"
 
 namespace {
@@ -242,62 +244,137 @@ __global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __res
 
 // out[m, n] = sum_k A(m,k) * B(n,k) (+ bias[n]); A(m,k) = A[m*sam + k*sak], B(n,k) = B[n*sbn + k*sbk].
 // fp32 on the CUDA cores (the head is fp32 end to end): 64 x 64 output tiles, 16-deep K tiles
-// stored K-major in shared memory, 4 x 4 outputs per thread from float4 reads.  Each output is a
-// sequential fmaf over k = 0..K-1.  Tile loads are coalesced along whichever index of an operand
-// has unit stride.
+// stored K-major in shared memory (double-buffered: the next tile is fetched into registers
+// while the current one is multiplied), 4 x 4 outputs per thread from float4 reads.  The
+// reduction is cut into gridDim.z fixed chunks of kchunk (a function of the shape only), each a
+// sequential fmaf over its k; with more than one chunk the partial sums go to part[z][M][N] and
+// gemm_chunk_reduce_kernel adds them in chunk order.  Tile loads are coalesced along whichever
+// index of an operand has unit stride.
 constexpr int GBM = 64, GBN = 64, GBK = 16;
+constexpr int kGemmThreads = 256;
+constexpr int kGemmTargetCTAs = 304;  // two 64 x 64 tiles per SM of a 152-SM GPU
 
-__device__ __forceinline__ void gemm_load_tile(const float* __restrict__ X, int64_t s_row, int64_t s_k, int row0,
-                                               int rows, int k0, int K, float (*dst)[GBM + 4])
+struct GemmTileRegs {
+    float v[GBM * GBK / kGemmThreads];
+};
+
+// Thread's share of the K tile [k0, k0 + GBK) of rows [row0, row0 + GBM): element e = tid + 256 q.
+__device__ __forceinline__ void gemm_fetch(const float* __restrict__ X, int64_t s_row, int64_t s_k, int row0, int rows,
+                                           int k0, int kend, GemmTileRegs& t)
 {
-    // dst[k][r] = X(row0 + r, k0 + k), zero outside
-    if (s_k == 1) {  // consecutive threads along k
-        for (int e = threadIdx.x; e < GBM * GBK; e += blockDim.x) {
-            const int r = e / GBK, k = e % GBK;
-            const int row = row0 + r, kk = k0 + k;
-            dst[k][r] = (row < rows && kk < K) ? __ldg(X + (int64_t)row * s_row + kk) : 0.f;
-        }
-    } else {  // consecutive threads along the row index
-        for (int e = threadIdx.x; e < GBM * GBK; e += blockDim.x) {
-            const int k = e / GBM, r = e % GBM;
-            const int row = row0 + r, kk = k0 + k;
-            dst[k][r] = (row < rows && kk < K) ? __ldg(X + (int64_t)row * s_row + (int64_t)kk * s_k) : 0.f;
-        }
+#pragma unroll
+    for (int q = 0; q < GBM * GBK / kGemmThreads; ++q) {
+        const int e = threadIdx.x + kGemmThreads * q;
+        const int r = s_k == 1 ? e / GBK : e % GBM, k = s_k == 1 ? e % GBK : e / GBM;
+        const int row = row0 + r, kk = k0 + k;
+        t.v[q] = (row < rows && kk < kend) ? __ldg(X + (int64_t)row * s_row + (int64_t)kk * s_k) : 0.f;
     }
 }
 
-__global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__ A, int64_t sam, int64_t sak,
-                                                       const float* __restrict__ B, int64_t sbn, int64_t sbk,
-                                                       const float* __restrict__ bias, float* __restrict__ out,
-                                                       int64_t ldo, int M, int N, int K)
+__device__ __forceinline__ void gemm_stash(int64_t s_k, const GemmTileRegs& t, float (*dst)[GBM + 4])
 {
-    __shared__ __align__(16) float As[GBK][GBM + 4], Bs[GBK][GBN + 4];
+#pragma unroll
+    for (int q = 0; q < GBM * GBK / kGemmThreads; ++q) {
+        const int e = threadIdx.x + kGemmThreads * q;
+        const int r = s_k == 1 ? e / GBK : e % GBM, k = s_k == 1 ? e % GBK : e / GBM;
+        dst[k][r] = t.v[q];
+    }
+}
+
+__global__ void __launch_bounds__(kGemmThreads) gemm_f32_kernel(const float* __restrict__ A, int64_t sam, int64_t sak,
+                                                                const float* __restrict__ B, int64_t sbn, int64_t sbk,
+                                                                const float* __restrict__ bias, float* __restrict__ out,
+                                                                int64_t ldo, int M, int N, int K, int kchunk,
+                                                                float* __restrict__ part)
+{
+    __shared__ __align__(16) float As[2][GBK][GBM + 4], Bs[2][GBK][GBN + 4];
     const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;  // thread owns rows 4ty.., columns 4tx..
     const int m0 = blockIdx.y * GBM, n0 = blockIdx.x * GBN;
+    const int kb = blockIdx.z * kchunk, ke = min(K, kb + kchunk);
     float acc[4][4] = {};
-    for (int k0 = 0; k0 < K; k0 += GBK) {
-        gemm_load_tile(A, sam, sak, m0, M, k0, K, As);
-        gemm_load_tile(B, sbn, sbk, n0, N, k0, K, Bs);
+    GemmTileRegs ra, rb;
+    gemm_fetch(A, sam, sak, m0, M, kb, ke, ra);
+    gemm_fetch(B, sbn, sbk, n0, N, kb, ke, rb);
+    int buf = 0;
+    for (int k0 = kb; k0 < ke; k0 += GBK, buf ^= 1) {
+        gemm_stash(sak, ra, As[buf]);
+        gemm_stash(sbk, rb, Bs[buf]);
         __syncthreads();
+        if (k0 + GBK < ke) {  // next tile in flight during the multiply
+            gemm_fetch(A, sam, sak, m0, M, k0 + GBK, ke, ra);
+            gemm_fetch(B, sbn, sbk, n0, N, k0 + GBK, ke, rb);
+        }
 #pragma unroll
         for (int k = 0; k < GBK; ++k) {
-            const float4 a = *reinterpret_cast<const float4*>(&As[k][4 * ty]);
-            const float4 b = *reinterpret_cast<const float4*>(&Bs[k][4 * tx]);
+            const float4 a = *reinterpret_cast<const float4*>(&As[buf][k][4 * ty]);
+            const float4 b = *reinterpret_cast<const float4*>(&Bs[buf][k][4 * tx]);
             const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
             for (int i = 0; i < 4; ++i)
 #pragma unroll
                 for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
         }
-        __syncthreads();
     }
+    float* dst = part ? part + (int64_t)blockIdx.z * M * N : out;
+    const int64_t ld = part ? N : ldo;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int m = m0 + 4 * ty + i, n = n0 + 4 * tx + j;
-            if (m < M && n < N) out[(int64_t)m * ldo + n] = acc[i][j] + (bias ? bias[n] : 0.f);
+            if (m < M && n < N) dst[(int64_t)m * ld + n] = part ? acc[i][j] : acc[i][j] + (bias ? bias[n] : 0.f);
         }
+}
+
+// out[m, n] = sum over chunks z = 0..nz-1 in order of part[z][m][n] (+ bias[n]).
+__global__ void __launch_bounds__(256) gemm_chunk_reduce_kernel(const float* __restrict__ part, int nz, int M, int N,
+                                                                const float* __restrict__ bias, float* __restrict__ out,
+                                                                int64_t ldo)
+{
+    const int64_t total = (int64_t)M * N;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+        float v = part[i];
+        for (int z = 1; z < nz; ++z) v += part[z * total + i];
+        const int m = (int)(i / N), n = (int)(i % N);
+        out[(int64_t)m * ldo + n] = v + (bias ? bias[n] : 0.f);
+    }
+}
+
+// K-chunking of an M x N x K head GEMM: enough chunks for ~kGemmTargetCTAs CTAs, at least
+// four K tiles per chunk.  Returns the chunk length; *nz receives the chunk count.
+int gemm_chunking(int M, int N, int K, int* nz)
+{
+    const int tiles = ((M + GBM - 1) / GBM) * ((N + GBN - 1) / GBN);
+    int z = (kGemmTargetCTAs + tiles - 1) / tiles;
+    const int zmax = std::max(1, (K + 4 * GBK - 1) / (4 * GBK));
+    z = std::min(std::max(z, 1), zmax);
+    int kchunk = (K + z - 1) / z;
+    kchunk = (kchunk + GBK - 1) / GBK * GBK;
+    *nz = (K + kchunk - 1) / kchunk;
+    return kchunk;
+}
+
+size_t gemm_part_floats(int M, int N, int K)
+{
+    int nz;
+    gemm_chunking(M, N, K, &nz);
+    return nz > 1 ? (size_t)nz * M * N : 0;
+}
+
+int gemm_f32(const float* A, int64_t sam, int64_t sak, const float* B, int64_t sbn, int64_t sbk, const float* bias,
+             float* out, int64_t ldo, int M, int N, int K, float* part, cudaStream_t s, const char* what)
+{
+    int nz;
+    const int kchunk = gemm_chunking(M, N, K, &nz);
+    dim3 g((N + GBN - 1) / GBN, (M + GBM - 1) / GBM, nz);
+    gemm_f32_kernel<<<g, kGemmThreads, 0, s>>>(A, sam, sak, B, sbn, sbk, bias, out, ldo, M, N, K, kchunk,
+                                                nz > 1 ? part : nullptr);
+    int rc = dbl::launch_check(what);
+    if (rc || nz == 1) return rc;
+    const int64_t total = (int64_t)M * N;
+    const int blocks = (int)std::min<int64_t>((total + 255) / 256, (int64_t)dbl::sm_count() * 8);
+    gemm_chunk_reduce_kernel<<<blocks, 256, 0, s>>>(part, nz, M, N, bias, out, ldo);
+    return dbl::launch_check(what);
 }
 
 // One warp per row: loss_n = logsumexp(l) - l[label]; dl = (softmax - onehot)/n (in place).
@@ -431,9 +508,12 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
 size_t dbl_head_workspace_bytes(int32_t n, int32_t c, int32_t classes)
 {
     if (n <= 0 || c <= 0 || classes <= 0) return 0;
-    // feat [n,c], logits/dlogits [n,classes], df [n,c], row_loss [n]
+    // feat [n,c], logits/dlogits [n,classes], df [n,c], row_loss [n], then the K-chunk partial
+    // sums of the largest of the three GEMMs
     const size_t f = (size_t)n * c * 2 + (size_t)n * classes + (size_t)n;
-    return (f * sizeof(float) + 255) / 256 * 256;
+    const size_t part = std::max({gemm_part_floats(n, classes, c), gemm_part_floats(classes, c, n),
+                                  gemm_part_floats(n, c, classes)});
+    return (((f + 3) / 4 * 4 + part) * sizeof(float) + 255) / 256 * 256;
 }
 
 int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
@@ -452,27 +532,25 @@ int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const vo
     float* logits = feat + (size_t)n * c;
     float* df = logits + (size_t)n * classes;
     float* row_loss = df + (size_t)n * c;
+    float* part = feat + ((size_t)n * c * 2 + (size_t)n * classes + (size_t)n + 3) / 4 * 4;
     cudaStream_t s = as_stream(stream);
     int rc;
     avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(x), feat, n,
                                                                        hw, c);
     if ((rc = launch_check("avgpool launch"))) return rc;
     // logits = feat * W^T + b
-    dim3 g1((classes + GBN - 1) / GBN, (n + GBM - 1) / GBM);
-    gemm_f32_kernel<<<g1, 256, 0, s>>>(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c);
-    if ((rc = launch_check("fc fwd launch"))) return rc;
+    if ((rc = gemm_f32(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c, part, s, "fc fwd launch")))
+        return rc;
     softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss);
     if ((rc = launch_check("softmax_ce launch"))) return rc;
     head_reduce_kernel<<<1 + (classes + 255) / 256, 256, 0, s>>>(row_loss, logits, n, classes, loss, dfc_b);
     if ((rc = launch_check("head reduce launch"))) return rc;
     // dW[j, c] = sum_n dl[n, j] feat[n, c]
-    dim3 g2((c + GBN - 1) / GBN, (classes + GBM - 1) / GBM);
-    gemm_f32_kernel<<<g2, 256, 0, s>>>(logits, 1, classes, feat, 1, c, nullptr, dfc_w, c, classes, c, n);
-    if ((rc = launch_check("fc dW launch"))) return rc;
+    if ((rc = gemm_f32(logits, 1, classes, feat, 1, c, nullptr, dfc_w, c, classes, c, n, part, s, "fc dW launch")))
+        return rc;
     // df[n, c] = sum_j dl[n, j] W[j, c]
-    dim3 g3((c + GBN - 1) / GBN, (n + GBM - 1) / GBM);
-    gemm_f32_kernel<<<g3, 256, 0, s>>>(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes);
-    if ((rc = launch_check("fc dX launch"))) return rc;
+    if ((rc = gemm_f32(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes, part, s, "fc dX launch")))
+        return rc;
     avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(df, static_cast<__nv_bfloat16*>(dx), n,
                                                                                 hw, c);
     return launch_check("avgpool_bwd launch");

@@ -284,7 +284,8 @@ def test_maxpool_matches_oracle(D, n, h, w, c, zeros):
 
 
 # ----------------------------------------------------------------------------- head
-@pytest.mark.parametrize("n,hw,c,classes", [(4, 16, 64, 10), (8, 49, 512, 1000), (256, 16, 512, 100)])
+@pytest.mark.parametrize("n,hw,c,classes", [(4, 16, 64, 10), (8, 49, 512, 1000), (256, 16, 512, 100),
+                                            (512, 49, 512, 1000), (128, 49, 512, 1000)])  # the two worker batches
 def test_head_matches_oracle(D, n, hw, c, classes):
     g = rng(n * classes)
     x = bf16_values(np.maximum(g.standard_normal((n, hw, c)), 0))
