@@ -26,6 +26,7 @@
 // Every mbarrier wait is bounded (see dbl_internal.cuh); a wait that gives up
 // records DBL_ERR_TIMEOUT in the device status word and the CTA winds down.
 #include <algorithm>
+#include <cstdlib>
 
 #include "dbl_internal.cuh"
 
@@ -95,16 +96,18 @@ enum Family : int { kFamFwd = 0, kFamWgrad = 1 };  // fwd/dgrad/stem-fwd, and th
 //   forward family, BN <= 128: a tile is 256 rows in two 128-row accumulators
 //     that share one B tile; one 256-pixel im2col op feeds both;
 //   weight-gradient family: a K-block is 128 pixels (8 MMA K-steps).
-template <int BN, int FAM>
+template <int BN, int FAM, int CG = 1>
 struct Cfg {
     static constexpr int ACC = (FAM == kFamFwd && BN <= 128) ? 2 : 1;  // 128-row accumulators per tile
-    static constexpr int BMT = 128 * ACC;                               // tile rows
+    static constexpr int BMT = 128 * ACC;                               // tile rows per CTA
     static constexpr int KB = FAM == kFamFwd ? 64 : 128;                // reduction elements per stage
     static constexpr int KSTEPS = KB / 16;
+    static constexpr int BNC = BN / CG;                                 // B columns held by one CTA
     static constexpr int A_BYTES = BMT * KB * 2;
-    static constexpr int B_BYTES = BN * KB * 2;
+    static constexpr int B_BYTES = BNC * KB * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = (196608 / STAGE_BYTES) < 4 ? (196608 / STAGE_BYTES) : 4;
+    static constexpr int MAX_STAGES = CG == 2 ? 6 : 4;
+    static constexpr int STAGES = (196608 / STAGE_BYTES) < MAX_STAGES ? (196608 / STAGE_BYTES) : MAX_STAGES;
     static constexpr int RING = STAGES * STAGE_BYTES;
     static constexpr int EPI_TILE = 4 * 32 * 33 * 4;           // per-warp 32x32 transpose scratch
     static constexpr int EPI_SUM = 4 * 2 * kMaxNcols * 4;      // per-warp channel sums (fwd)
@@ -114,16 +117,31 @@ struct Cfg {
     static constexpr int MMA_WARP = 4 + kProducers;
     static_assert(STAGES >= 2, "ring too shallow");
     static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
+    static_assert(SMEM <= 232448 - 1024, "shared memory per CTA");
 };
 
 struct TileCoord {
     int m_tile, n_tile, z;
 };
 
-__device__ __forceinline__ TileCoord decode_tile(const ConvParams& p, int t)
+// Weight gradient: split-K slice outermost, so that the CTAs running at one time
+// share the slice's dy K-blocks.  Stride-2 data gradient: the four phases of one
+// m-tile are adjacent, so that the dy rows they all read are fetched from DRAM
+// once; the phase index is rotated by one per wave of the persistent grid, so
+// that every CTA gets a mix of the 4-, 2- and 1-tap phases.
+// units: the number of tiles the persistent grid processes at one time.
+__device__ __forceinline__ TileCoord decode_tile(const ConvParams& p, int t, int units)
 {
-    const int mn = p.m_tiles * p.n_tiles;
     TileCoord c;
+    if (p.mode == kDgrad && p.zdim > 1) {
+        const int g = t / p.zdim, l = t - g * p.zdim;
+        const int per_wave = max(1, units / p.zdim);
+        c.z = (l + g / per_wave) % p.zdim;
+        c.m_tile = g / p.n_tiles;
+        c.n_tile = g - c.m_tile * p.n_tiles;
+        return c;
+    }
+    const int mn = p.m_tiles * p.n_tiles;
     c.z = t / mn;
     const int r = t - c.z * mn;
     c.m_tile = r / p.n_tiles;
@@ -147,36 +165,41 @@ __device__ __forceinline__ void kb_range(const ConvParams& p, int z, int& kb0, i
     }
 }
 
-// Issue the TMA loads of one K-block of one tile into ring stage (sa, sb).
-template <int BN, int FAM>
+// Issue the TMA loads of one K-block of one tile into ring stage (sa, sb); fb is
+// the shared::cluster address of the stage's full barrier.  With CTA pairs
+// (CG = 2) CTA `rank` loads its own 128-row (fwd family: BMT-row) part of A and
+// columns rank*BN/2 .. (rank+1)*BN/2-1 of B, and both CTAs' loads complete on
+// rank 0's barrier.
+template <int BN, int FAM, int CG>
 __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorMap* tmA, const CUtensorMap* tmB,
-                                            uint8_t* sa, uint8_t* sb, uint64_t* fb, const TileCoord& tc, int kb, int tn,
-                                            int tp, int tq)
+                                            uint8_t* sa, uint8_t* sb, uint32_t fb, const TileCoord& tc, int kb, int tn,
+                                            int tp, int tq, int rank)
 {
-    using C = Cfg<BN, FAM>;
+    using C = Cfg<BN, FAM, CG>;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
+    const int ncol0 = tc.n_tile * BN + rank * C::BNC;  // first B column this CTA loads
     if constexpr (FAM == kFamFwd) {
         if (p.mode == kFwd) {
             const int tap = kb / p.cblocks, cb = kb - tap * p.cblocks;
             const int r = tap / p.S, sx = tap - r * p.S;
-            tma_load_im2col_4d_elect(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
-                               (uint16_t)sx, (uint16_t)r);
-            tma_load_2d_elect(sb, tmB, fb, tap * p.Cin + cb * 64, tc.n_tile * BN);
+            tma_load_im2col_4d_cg<CG>(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
+                                      (uint16_t)sx, (uint16_t)r);
+            tma_load_2d_cg<CG>(sb, tmB, fb, tap * p.Cin + cb * 64, ncol0);
         } else if (p.mode == kDgrad) {
             const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
-            tma_load_im2col_4d_elect(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
-                               (uint16_t)p.tap_oh[t]);
+            tma_load_im2col_4d_cg<CG>(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
+                                      (uint16_t)p.tap_oh[t]);
             const int wtap = p.tap_r[t] * p.S + p.tap_s[t];
-            for (int j = 0; j < BN / 64; ++j)
-                tma_load_3d_elect(sb + j * 8192, tmB, fb, tc.n_tile * BN + 64 * j, wtap, kbk * 64);
+            for (int j = 0; j < C::BNC / 64; ++j)
+                tma_load_3d_cg<CG>(sb + j * 8192, tmB, fb, ncol0 + 64 * j, wtap, kbk * 64);
         } else {  // kFwdC8: 8 taps of 8 channels; taps past R*S read a valid tap and meet zero weights
             for (int j = 0; j < 8; ++j) {
                 int tap = kb * 8 + j;
                 const int wcol = tap * 8;
                 if (tap >= p.ntaps) tap = p.ntaps - 1;
-                tma_load_im2col_4d_elect(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride_w + p.base_w,
-                                   tp * p.tstride_h + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
-                tma_load_2d_elect(sb + j * (BN * 16), tmB, fb, wcol, tc.n_tile * BN);
+                tma_load_im2col_4d_cg<CG>(sa + j * (C::BMT * 16), tmA, fb, 0, tq * p.tstride_w + p.base_w,
+                                          tp * p.tstride_h + p.base_h, tn, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_2d_cg<CG>(sb + j * (C::BNC * 16), tmB, fb, wcol, ncol0);
             }
         }
     } else {
@@ -187,22 +210,22 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
         const int pp = (int)(rem / p.gQ), qq = (int)(rem - (int64_t)pp * p.gQ);
         if (p.mode == kWgrad) {
             for (int h = 0; h < 2; ++h) {
-                const int mrow = tc.m_tile * BM + 64 * h;
+                const int mrow = (tc.m_tile * CG + rank) * BM + 64 * h;
                 int tap = mrow / p.Cin;
                 const int c0 = mrow - tap * p.Cin;
                 if (tap >= p.ntaps) tap = 0;  // rows past R*S*C: loaded, never stored
-                tma_load_im2col_4d_elect(sa + h * 16384, tmA, fb, c0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
-                                   (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_im2col_4d_cg<CG>(sa + h * 16384, tmA, fb, c0, qq * p.tstride_w + p.base_w,
+                                          pp * p.tstride_h + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         } else {  // kWgradC8: 16 taps x 8 channels of rows
             for (int j = 0; j < 16; ++j) {
                 int tap = tc.m_tile * 16 + j;
                 if (tap >= p.ntaps) tap = 0;
-                tma_load_im2col_4d_elect(sa + j * 2048, tmA, fb, 0, qq * p.tstride_w + p.base_w, pp * p.tstride_h + p.base_h, n,
-                                   (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
+                tma_load_im2col_4d_cg<CG>(sa + j * 2048, tmA, fb, 0, qq * p.tstride_w + p.base_w,
+                                          pp * p.tstride_h + p.base_h, n, (uint16_t)(tap % p.S), (uint16_t)(tap / p.S));
             }
         }
-        for (int j = 0; j < BN / 64; ++j) tma_load_2d_elect(sb + j * 16384, tmB, fb, tc.n_tile * BN + 64 * j, (int)pix0);
+        for (int j = 0; j < C::BNC / 64; ++j) tma_load_2d_cg<CG>(sb + j * 16384, tmB, fb, ncol0 + 64 * j, (int)pix0);
     }
 }
 
@@ -308,15 +331,25 @@ struct RowStats {
 };
 
 // Persistent kernel: CTA b processes tiles b, b + gridDim.x, ...  The ring of
-// STAGES shared-memory stages (two K-blocks each) runs continuously across
-// tiles; two producer warps fill alternate stages; two TMEM accumulators let
-// the epilogue of one tile overlap the MMAs of the next.
-template <int BN, int FAM>
-__global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
+// STAGES shared-memory stages runs continuously across tiles; two producer
+// warps fill alternate stages; two TMEM accumulators let the epilogue of one
+// tile overlap the MMAs of the next.
+//
+// CG = 2 (clusters of two CTAs): a tile is processed by a CTA pair with
+// M = 256 MMAs (tcgen05 .cta_group::2).  Each CTA stages its own BMT rows of A
+// and half of the B columns, so a CTA's shared memory carries half of the B
+// bytes (TMA writes and MMA reads) of the single-CTA form; shared-memory
+// bandwidth is what limits the single-CTA form.  Rank 0 issues the MMAs and owns
+// the stage-full barriers, which both CTAs' loads complete on; its commits
+// arrive on the stage-empty and accumulator-full barriers of both CTAs; the
+// epilogues of both CTAs arrive on rank 0's accumulator-empty barriers.  Each
+// CTA drains its own TMEM (its own rows, all BN columns).
+template <int BN, int FAM, int CG>
+__global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const ConvParams p)
 {
-    using C = Cfg<BN, FAM>;
+    using C = Cfg<BN, FAM, CG>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accf_bar[2], acce_bar[2], drain_bar;
@@ -328,6 +361,8 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
     uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
     float* epi_tile = reinterpret_cast<float*>(sgen + C::RING);
     float* epi_sum = reinterpret_cast<float*>(sgen + C::RING + C::EPI_TILE);
+    const int rank = CG == 2 ? (int)cluster_ctarank() : 0;
+    const int unit0 = blockIdx.x / CG, nunits = gridDim.x / CG;  // this pair's first tile, tiles' stride
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -336,7 +371,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
-            mbar_init(&acce_bar[b], 4);  // one arrival per epilogue warp
+            mbar_init(&acce_bar[b], 4 * CG);  // one arrival per epilogue warp of the pair
         }
         mbar_init(&drain_bar, 1);
         abort_flag = 0;
@@ -350,11 +385,12 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         tma_prefetch_desc(&tmB);
     }
     if (warp == C::MMA_WARP) {
-        tmem_alloc(&tmem_slot, C::TMEM_COLS);
-        tmem_relinquish();
+        tmem_alloc_cg<CG>(&tmem_slot, C::TMEM_COLS);
+        tmem_relinquish_cg<CG>();
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (CG == 2) cluster_sync_all();  // both CTAs' barriers initialised, TMEM allocated
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
@@ -364,13 +400,13 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         const int prod = warp - 4;
         int it = 0, last_it = -1;
         bool failed = false;
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
-            const TileCoord tc = decode_tile(p, t);
+        for (int t = unit0; t < p.total_tiles; t += nunits) {
+            const TileCoord tc = decode_tile(p, t, nunits);
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
             int tn = 0, tp = 0, tq = 0;
             if (FAM == kFamFwd) {
-                const int64_t m0 = (int64_t)tc.m_tile * C::BMT;
+                const int64_t m0 = ((int64_t)tc.m_tile * CG + rank) * C::BMT;
                 tn = (int)(m0 / gPQ);
                 const int64_t rem = m0 - (int64_t)tn * gPQ;
                 tp = (int)(rem / p.gQ);
@@ -385,85 +421,128 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
                     break;
                 }
                 uint8_t* sa = sgen + s * C::STAGE_BYTES;
-                mbar_arrive_expect_tx_elect(&full_bar[s], (uint32_t)C::STAGE_BYTES);
-                load_kblock<BN, FAM>(p, &tmA, &tmB, sa, sa + C::A_BYTES, &full_bar[s], tc, kb0 + k, tn, tp, tq);
+                uint32_t fb = smem_u32(&full_bar[s]);
+                if (CG == 1 || rank == 0)
+                    mbar_arrive_expect_tx_elect(&full_bar[s], (uint32_t)(CG * C::STAGE_BYTES));
+                if (CG == 2) fb = mapa_shared(fb, 0);
+                load_kblock<BN, FAM, CG>(p, &tmA, &tmB, sa, sa + C::A_BYTES, fb, tc, kb0 + k, tn, tp, tq, rank);
                 last_it = it;
             }
             if (failed) break;
         }
         if (failed) {
             if (lane == 0) report_timeout(&abort_flag);
-            // let copies this producer issued land before the CTA's shared memory goes away
-            for (int i = last_it; i >= 0 && i > last_it - STAGES * kProducers; i -= kProducers)
-                (void)mbar_drain_warp(&full_bar[i % STAGES], (i / STAGES) & 1);
+            if (CG == 1 || rank == 0) {
+                // let copies this producer issued land before the CTA's shared memory goes away
+                for (int i = last_it; i >= 0 && i > last_it - STAGES * kProducers; i -= kProducers)
+                    (void)mbar_drain_warp(&full_bar[i % STAGES], (i / STAGES) & 1);
+            } else {
+                // rank 1's copies complete on rank 0's barriers: give them a fixed time instead
+                const uint64_t t0 = globaltimer();
+                while (globaltimer() - t0 < 1000000ull) {
+                }
+            }
         }
     } else if (warp == C::MMA_WARP) {
         // ------------------------------------------------------------------ MMA issuer (whole warp, one lane issues)
         const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
         const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
-        const uint32_t idesc = idesc_bf16(BM, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
-        int it = 0, lt = 0;
+        const uint32_t idesc = idesc_bf16(BM * CG, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
+        constexpr uint16_t kAll = CG == 2 ? 3 : 1;  // commits reach both CTAs of a pair
+        // Operand descriptors without their start address, and the start-address steps
+        // (in 16-byte units) per K-step and per accumulator:
+        //   kFwd / kDgrad: A K-major, 128-byte swizzle, one K-step = 32 bytes of a row;
+        //     B K-major (fwd) or MN-major with 64-wide atoms 8 KB apart (dgrad, 2 KB per K-step);
+        //   kFwdC8: K-major without swizzle: core matrices of 8 rows x 16 B, rows 16 B apart,
+        //     8-row groups 128 B apart (SBO), the two taps of one K-step LBO apart;
+        //   kWgrad: both MN-major, 128-byte swizzle, 64-wide atoms 16 KB apart (LBO);
+        //   kWgradC8: A MN-major without swizzle, 8 pixels x 8 channels per core matrix,
+        //     next 8 pixels 128 B apart (LBO), next tap 2 KB apart (SBO).
+        uint64_t dA, dB;
+        int a_step16, b_step16, a_acc16 = 16384 / 16;
+        if (p.mode == kFwd || p.mode == kDgrad) {
+            dA = smem_desc(0, 16, 1024, kSwizzle128B);
+            a_step16 = 2;
+            if (p.mode == kFwd) {
+                dB = smem_desc(0, 16, 1024, kSwizzle128B);
+                b_step16 = 2;
+            } else {
+                dB = smem_desc(0, 8192, 1024, kSwizzle128B);
+                b_step16 = 2048 / 16;
+            }
+        } else if (p.mode == kFwdC8) {
+            dA = smem_desc(0, C::BMT * 16, 128, kSwizzleNone);
+            dB = smem_desc(0, C::BNC * 16, 128, kSwizzleNone);
+            a_step16 = 2 * C::BMT;
+            b_step16 = 2 * C::BNC;
+            a_acc16 = 2048 / 16;
+        } else if (p.mode == kWgrad) {
+            dA = smem_desc(0, 16384, 1024, kSwizzle128B);
+            dB = smem_desc(0, 16384, 1024, kSwizzle128B);
+            a_step16 = b_step16 = 2048 / 16;
+        } else {
+            dA = smem_desc(0, 128, 2048, kSwizzleNone);
+            dB = smem_desc(0, 16384, 1024, kSwizzle128B);
+            a_step16 = 256 / 16;
+            b_step16 = 2048 / 16;
+        }
+        // The MMA issue is on the critical path: every cycle this warp spends polling a
+        // barrier while the tensor pipe has nothing queued is lost.  So the wait for the next
+        // stage is made before the last K-step of the current stage is issued, while the
+        // tensor pipe still has work.
         bool failed = false;
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t);
+        auto wait_ok = [&](uint64_t* bar, uint32_t parity) -> bool {
+            const uint32_t ok = mbar_wait_warp(bar, parity, &abort_flag);
+            return !__any_sync(0xffffffffu, ok == 0u);
+        };
+        // Only waits inside a tile are made ahead: waiting for the next tile's accumulator or
+        // data before this tile's last K-step would delay this tile's completion, and with it
+        // the epilogue, behind an earlier epilogue or a later load.
+        int it = 0, lt = 0;
+        for (int t = unit0; t < p.total_tiles && (CG == 1 || rank == 0) && !failed; t += nunits, ++lt) {
+            const TileCoord tc = decode_tile(p, t, nunits);
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
             const int buf = lt & 1;
-            const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
-            if (__any_sync(0xffffffffu, ok == 0u)) {
+            if (!wait_ok(&acce_bar[buf], ((lt >> 1) & 1) ^ 1) ||
+                (nkb > 0 && !wait_ok(&full_bar[it % STAGES], (it / STAGES) & 1))) {
                 failed = true;
                 break;
             }
-            tc_fence_after();
             const uint32_t d = tmem + (uint32_t)(buf * C::ACC * BN);
             for (int k = 0; k < nkb; ++k, ++it) {
-                const int s = it % STAGES;
-                const uint32_t okk = mbar_wait_warp(&full_bar[s], (it / STAGES) & 1, &abort_flag);
-                if (__any_sync(0xffffffffu, okk == 0u)) {
-                    failed = true;
-                    break;
-                }
                 tc_fence_after();
+                const int s = it % STAGES;
                 const uint32_t sa = sbase + s * C::STAGE_BYTES;
                 const uint32_t sb = sa + C::A_BYTES;
+                const uint64_t ad0 = dA | (uint64_t)((sa >> 4) & 0x3FFFu), bd0 = dB | (uint64_t)((sb >> 4) & 0x3FFFu);
 #pragma unroll
-                for (int j = 0; j < C::KSTEPS; ++j) {
+                for (int j = 0; j < C::KSTEPS - 1; ++j) {
 #pragma unroll
-                    for (int a = 0; a < C::ACC; ++a) {
-                        uint64_t ad, bd;
-                        if (p.mode == kFwd) {
-                            ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
-                        } else if (p.mode == kDgrad) {
-                            ad = smem_desc(sa + a * 16384 + 32 * j, 16, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B);
-                        } else if (p.mode == kFwdC8) {
-                            // K-major, no swizzle: core matrices of 8 rows x 16 B; rows 16 B apart,
-                            // 8-row groups 128 B apart (SBO), the two taps of one MMA apart by LBO
-                            ad = smem_desc(sa + a * 2048 + 2 * (C::BMT * 16) * j, C::BMT * 16, 128, kSwizzleNone);
-                            bd = smem_desc(sb + 2 * (BN * 16) * j, BN * 16, 128, kSwizzleNone);
-                        } else if (p.mode == kWgrad) {
-                            // MN-major, 128-byte swizzle: 64-wide atoms 16 KB apart (LBO)
-                            ad = smem_desc(sa + 2048 * j, 16384, 1024, kSwizzle128B);
-                            bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
-                        } else {
-                            // MN-major, no swizzle: 8 pixels x 8 channels per core matrix;
-                            // next 8 pixels 128 B apart (LBO), next tap 2 KB apart (SBO)
-                            ad = smem_desc(sa + 256 * j, 128, 2048, kSwizzleNone);
-                            bd = smem_desc(sb + 2048 * j, 16384, 1024, kSwizzle128B);
-                        }
-                        mma_bf16_elect(d + a * BN, ad, bd, idesc, (k > 0 || j > 0) ? 1u : 0u);
-                    }
+                    for (int a = 0; a < C::ACC; ++a)
+                        mma_bf16_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + j * a_step16),
+                                              bd0 + (uint64_t)(j * b_step16), idesc, (k > 0 || j > 0) ? 1u : 0u);
                 }
-                mma_commit_elect(&empty_bar[s]);
+                if (k + 1 < nkb) failed = !wait_ok(&full_bar[(it + 1) % STAGES], ((it + 1) / STAGES) & 1);
+                constexpr int jl = C::KSTEPS - 1;
+#pragma unroll
+                for (int a = 0; a < C::ACC; ++a)
+                    mma_bf16_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + jl * a_step16),
+                                          bd0 + (uint64_t)(jl * b_step16), idesc, (k > 0 || jl > 0) ? 1u : 0u);
+                mma_commit_elect_cg<CG>(&empty_bar[s], kAll);
+                if (failed) {
+                    ++it;
+                    break;
+                }
             }
-            mma_commit_elect(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
-            if (failed) break;
+            mma_commit_elect_cg<CG>(&accf_bar[buf], kAll);  // arrives when this tile's MMAs have completed
         }
         if (failed && lane == 0) report_timeout(&abort_flag);
-        // every MMA issued above completes before the accumulators are freed
-        mma_commit_elect(&drain_bar);
-        (void)mbar_drain_warp(&drain_bar, 0);
+        if (CG == 1 || rank == 0) {
+            // every MMA issued above completes before the accumulators are freed
+            mma_commit_elect_cg<CG>(&drain_bar, 1);
+            (void)mbar_drain_warp(&drain_bar, 0);
+        }
     } else {
         // ------------------------------------------------------------------ epilogue (warps 0-3)
         float* st_tile = epi_tile + warp * 32 * 33;
@@ -472,8 +551,8 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
         rs.zero();
         int stats_ntile = -1;  // column tile the register sums belong to
         int lt = 0;
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t);
+        for (int t = unit0; t < p.total_tiles; t += nunits, ++lt) {
+            const TileCoord tc = decode_tile(p, t, nunits);
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
             const int buf = lt & 1;
@@ -491,7 +570,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
             }
 #pragma unroll 1
             for (int a = 0; a < C::ACC; ++a) {
-                const int64_t m = (int64_t)tc.m_tile * C::BMT + a * 128 + row;
+                const int64_t m = ((int64_t)tc.m_tile * CG + rank) * C::BMT + a * 128 + row;
                 const bool valid = m < p.M;
                 const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * C::ACC + a) * BN);
                 if constexpr (FAM == kFamWgrad) {
@@ -545,7 +624,12 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&acce_bar[buf]);
+            if (lane == 0) {
+                if constexpr (CG == 2)
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&acce_bar[buf]), 0));
+                else
+                    mbar_arrive(&acce_bar[buf]);
+            }
         }
         if (want_stats && stats_ntile >= 0) rs.flush(st_tile, wsum, p.Ncols, stats_ntile * BN, lane);
         if (want_stats) {
@@ -557,9 +641,11 @@ __global__ void __launch_bounds__(Cfg<BN, FAM>::THREADS, 1)
     }
     tc_fence_before();
     __syncthreads();
+    // neither CTA of a pair leaves while the other may still signal its barriers or read its TMEM
+    if constexpr (CG == 2) cluster_sync_all();
     if (warp == C::MMA_WARP) {
         tc_fence_after();
-        tmem_dealloc(tmem, C::TMEM_COLS);
+        tmem_dealloc_cg<CG>(tmem, C::TMEM_COLS);
     }
 }
 
@@ -667,7 +753,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         bool failed = false;
         const uint32_t strip_tx = (uint32_t)(p.win_srows * Wp * 128);
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
-            const TileCoord tc = decode_tile(p, t);
+            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
             const int g0 = tc.m_tile * p.win_tile / Wp;
             for (int cb = 0; cb < CB; ++cb, ++it) {
                 const int s = it & 1;
@@ -704,7 +790,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             int bt = 0;
             bool failed = false;
             for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
-                const TileCoord tc = decode_tile(p, t);
+                const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
                 for (int cb = 0; cb < CB && !failed; ++cb)
                     for (int tap = 0; tap < ntaps; ++tap, ++bt) {
                         const int s = bt % kWinBStages;
@@ -734,7 +820,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             failed = __any_sync(0xffffffffu, ok == 0u);
         }
         for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t);
+            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
             const int buf = lt & 1;
             const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
@@ -807,7 +893,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const int img = p.win_Hp * Wp;
         int lt = 0;
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t);
+            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
             const int buf = lt & 1;
             const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
@@ -1133,6 +1219,7 @@ __global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restri
 struct Plan {
     int mode;
     int BN;
+    int cg = 1;          // conv_igemm_kernel CTAs per tile (2: CTA pairs with M = 256 MMAs)
     ConvParams p;
     size_t ws_main = 0;  // bytes: fwd channel-sum partials, or wgrad split-K slices
     bool win = false;    // conv_win_kernel (3x3 stride-1 correlation over padded strips)
@@ -1190,9 +1277,9 @@ int validate(const dbl_conv_shape* s, const char* who)
 // ~4 BN tensor cycles, in which the GPU streams ~10.5 KB x BN).  At least 4 K-blocks
 // (512 pixels) per slice.  A fixed function of the shape, so the summation order, and
 // with it the result, does not depend on the device the plan runs on.
-int wgrad_splits(int tiles, int num_kb, int rows, int cols, int BN)
+int wgrad_splits(int tiles, int num_kb, int rows, int cols, int BN, int cg)
 {
-    constexpr int kPlanSMs = 152;
+    const int kPlanSMs = 152 / cg;  // tile processors: SMs, or SM pairs
     const double slice_cost = (double)rows * cols * 4 / (10.5e3 * BN);  // K-block times to reduce one slice
     int best = 1;
     double best_cost = 1e300;
@@ -1340,6 +1427,17 @@ bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
     return true;
 }
 
+// Tiles of BN = 256 columns run on CTA pairs (see conv_igemm_kernel), unless the
+// environment variable DBL_CONV_CTA_PAIRS is set to 0.
+bool pair_tiles(int BN)
+{
+    static const bool enabled = [] {
+        const char* e = getenv("DBL_CONV_CTA_PAIRS");
+        return !(e && e[0] == '0');
+    }();
+    return enabled && BN == 256;
+}
+
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
 {
     using dbl::set_error;
@@ -1370,7 +1468,8 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.M = (int)M;
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
-        p.m_tiles = (p.M + fwd_tile_rows(pl.BN) - 1) / fwd_tile_rows(pl.BN);
+        pl.cg = pair_tiles(pl.BN) ? 2 : 1;
+        p.m_tiles = (p.M + pl.cg * fwd_tile_rows(pl.BN) - 1) / (pl.cg * fwd_tile_rows(pl.BN));
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;
         p.gP = P;
@@ -1449,13 +1548,15 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
             }
             p.phase_off[4] = t;
         }
-        p.m_tiles = (p.M + fwd_tile_rows(pl.BN) - 1) / fwd_tile_rows(pl.BN);
+        pl.cg = pair_tiles(pl.BN) ? 2 : 1;
+        p.m_tiles = (p.M + pl.cg * fwd_tile_rows(pl.BN) - 1) / (pl.cg * fwd_tile_rows(pl.BN));
     } else {
         pl.mode = p.mode = c8 ? kWgradC8 : kWgrad;
         p.M = p.ntaps * s->c;  // D rows = (tap, c)
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
-        p.m_tiles = c8 ? (p.ntaps + 15) / 16 : (p.M + BM - 1) / BM;
+        pl.cg = !c8 && pair_tiles(pl.BN) ? 2 : 1;
+        p.m_tiles = c8 ? (p.ntaps + 15) / 16 : (p.M + pl.cg * BM - 1) / (pl.cg * BM);
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;
         p.gP = P;
@@ -1467,7 +1568,7 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         const int64_t pix = (int64_t)s->n * P * Q;
         if ((pix + 127) / 128 > INT32_MAX / 2) return set_error(DBL_ERR_UNSUPPORTED, "conv_wgrad: too many pixels");
         p.num_kb = (int)((pix + 127) / 128);  // K-blocks of 128 output pixels
-        const int splits = wgrad_splits(p.m_tiles * p.n_tiles, p.num_kb, p.M, s->k, pl.BN);
+        const int splits = wgrad_splits(p.m_tiles * p.n_tiles, p.num_kb, p.M, s->k, pl.BN, pl.cg);
         p.kb_per_split = (p.num_kb + splits - 1) / splits;
         p.zdim = splits;
         pl.ws_main = splits > 1 ? (size_t)splits * p.M * s->k * sizeof(float) : 0;
@@ -1512,34 +1613,114 @@ int enc_tiled(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims
     return DBL_OK;
 }
 
-template <int BN, int FAM>
-int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+template <int BN, int FAM, int CG>
+int set_igemm_smem()
 {
-    using Cf = Cfg<BN, FAM>;
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN, FAM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             Cf::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<BN, FAM, CG>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN, FAM, CG>::SMEM);
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_igemm_kernel<BN, FAM><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
+    return DBL_OK;
+}
+
+// CTA pairs of conv_igemm_kernel<BN, FAM, 2> that fit on the device at once
+// (cached per device); at most half the SMs and kMaxGrid / 2.
+template <int BN, int FAM>
+int resident_pairs()
+{
+    static int cached[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+    int pairs = std::min(dbl::sm_count() / 2, kMaxGrid / 2);
+    if (set_igemm_smem<BN, FAM, 2>() == DBL_OK) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(2 * pairs);
+        cfg.blockDim = dim3(Cfg<BN, FAM, 2>::THREADS);
+        cfg.dynamicSmemBytes = Cfg<BN, FAM, 2>::SMEM;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, conv_igemm_kernel<BN, FAM, 2>, &cfg) == cudaSuccess && n > 0)
+            pairs = std::min(pairs, n);
+        else
+            (void)cudaGetLastError();
+    }
+    if (pairs < 1) pairs = 1;
+    if (dev >= 0 && dev < 64) cached[dev] = pairs;
+    return pairs;
+}
+
+// Persistent grid of a conv_igemm_kernel plan: one CTA per SM, or one CTA pair
+// per two SMs, never more CTAs (pairs) than tiles.
+int plan_grid(const Plan& pl)
+{
+    if (pl.cg == 1) return grid_size(pl.p.total_tiles);
+    const bool wg = pl.mode == kWgrad || pl.mode == kWgradC8;
+    int pairs = pl.BN == 256 ? (wg ? resident_pairs<256, kFamWgrad>() : resident_pairs<256, kFamFwd>())
+                             : (wg ? resident_pairs<128, kFamWgrad>() : resident_pairs<128, kFamFwd>());
+    if (pairs > pl.p.total_tiles) pairs = pl.p.total_tiles;
+    return 2 * std::max(pairs, 1);
+}
+
+template <int BN, int FAM, int CG>
+int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+{
+    using Cf = Cfg<BN, FAM, CG>;
+    int rc = set_igemm_smem<BN, FAM, CG>();
+    if (rc) return rc;
+    if constexpr (CG == 1) {
+        conv_igemm_kernel<BN, FAM, 1><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
+    } else {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(Cf::THREADS);
+        cfg.dynamicSmemBytes = Cf::SMEM;
+        cfg.stream = st;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        cudaError_t e = cudaLaunchKernelEx(&cfg, conv_igemm_kernel<BN, FAM, 2>, a, b, pl.p);
+        if (e != cudaSuccess) {
+            dbl::count_launch();
+            return dbl::cuda_check(e, "conv_igemm pair launch");
+        }
+    }
     return dbl::launch_check("conv_igemm launch");
 }
 
 int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
     const bool wg = pl.mode == kWgrad || pl.mode == kWgradC8;
-    if (wg) {
-        if (pl.BN == 256) return launch_cfg<256, kFamWgrad>(pl, a, b, grid, st);
-        if (pl.BN == 128) return launch_cfg<128, kFamWgrad>(pl, a, b, grid, st);
-        return launch_cfg<64, kFamWgrad>(pl, a, b, grid, st);
+    if (pl.cg == 2) {
+        if (pl.BN == 256) return wg ? launch_cfg<256, kFamWgrad, 2>(pl, a, b, grid, st)
+                                    : launch_cfg<256, kFamFwd, 2>(pl, a, b, grid, st);
+        if (pl.BN == 128) return wg ? launch_cfg<128, kFamWgrad, 2>(pl, a, b, grid, st)
+                                    : launch_cfg<128, kFamFwd, 2>(pl, a, b, grid, st);
+        return dbl::set_error(DBL_ERR_UNSUPPORTED, "conv: CTA pairs need 128 or 256 columns per tile");
     }
-    if (pl.BN == 256) return launch_cfg<256, kFamFwd>(pl, a, b, grid, st);
-    if (pl.BN == 128) return launch_cfg<128, kFamFwd>(pl, a, b, grid, st);
-    return launch_cfg<64, kFamFwd>(pl, a, b, grid, st);
+    if (wg) {
+        if (pl.BN == 256) return launch_cfg<256, kFamWgrad, 1>(pl, a, b, grid, st);
+        if (pl.BN == 128) return launch_cfg<128, kFamWgrad, 1>(pl, a, b, grid, st);
+        return launch_cfg<64, kFamWgrad, 1>(pl, a, b, grid, st);
+    }
+    if (pl.BN == 256) return launch_cfg<256, kFamFwd, 1>(pl, a, b, grid, st);
+    if (pl.BN == 128) return launch_cfg<128, kFamFwd, 1>(pl, a, b, grid, st);
+    return launch_cfg<64, kFamFwd, 1>(pl, a, b, grid, st);
 }
 
 template <int BN, bool DG, bool RES>
@@ -1647,12 +1828,12 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
         const int64_t rsc = (int64_t)s->r * s->s * s->c;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
         cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
+        cuuint32_t box[2] = {64, (cuuint32_t)(pl.BN / pl.cg)};
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
     }
     pl.p.out = y;
     pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
-    const int grid = grid_size(pl.p.total_tiles);
+    const int grid = plan_grid(pl);
     cudaStream_t st = as_stream(stream);
     if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, grid, st))) return rc;
     if (stats) {
@@ -1694,7 +1875,7 @@ int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void*
     cuuint32_t box[3] = {64, 1, 64};
     if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
     pl.p.out = dx;
-    const int grid = grid_size(pl.p.total_tiles);
+    const int grid = plan_grid(pl);
     return pl.win ? launch_win(pl, ta, tb, grid, as_stream(stream)) : launch(pl, ta, tb, grid, as_stream(stream));
 }
 
@@ -1732,7 +1913,7 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
     pl.p.out = sliced ? ws : static_cast<void*>(dw);
     pl.p.wg_accumulate = accumulate;
-    if ((rc = launch(pl, ta, tb, grid_size(pl.p.total_tiles), st))) return rc;
+    if ((rc = launch(pl, ta, tb, plan_grid(pl), st))) return rc;
     }
     if (!sliced) return DBL_OK;
     const int64_t n = (int64_t)pl.p.M * s->k;

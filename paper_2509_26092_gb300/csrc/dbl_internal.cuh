@@ -383,6 +383,187 @@ __device__ __forceinline__ void tma_load_im2col_4d_elect(void* dst, const void* 
         : "memory");
 }
 
+// ---------------------------------------------------------------------------- CTA pairs (clusters of 2)
+// A kernel whose MMAs span a CTA pair (tcgen05 .cta_group::2) uses these forms
+// throughout: PTX forbids mixing .cta_group::1 and ::2 tcgen05 instructions in
+// one kernel.
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Shared::cluster address of the variable at shared::cta address addr in CTA rank.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// Every thread of every CTA of the cluster: release this CTA's prior writes
+// (barrier inits included), acquire the others'.
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Arrive once on an mbarrier given by its shared::cluster address (possibly in the peer CTA).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// TMA loads whose completion is signalled on the mbarrier at shared::cluster
+// address bar.  CG = 2 (.cta_group::2): bar may be in the peer CTA of the pair,
+// which is how both CTAs' operand halves complete on the MMA-issuing CTA's barrier.
+template <int CG>
+__device__ __forceinline__ void tma_load_2d_cg(void* dst, const void* tmap, uint32_t bar, int32_t c0, int32_t c1)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1)
+            : "memory");
+}
+
+template <int CG>
+__device__ __forceinline__ void tma_load_3d_cg(void* dst, const void* tmap, uint32_t bar, int32_t c0, int32_t c1,
+                                               int32_t c2)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+            : "memory");
+}
+
+template <int CG>
+__device__ __forceinline__ void tma_load_im2col_4d_cg(void* dst, const void* tmap, uint32_t bar, int32_t c, int32_t w,
+                                                      int32_t h, int32_t n, uint16_t off_w, uint16_t off_h)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8};\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w), "h"(off_h)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8};\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w), "h"(off_h)
+            : "memory");
+}
+
+// TMEM allocation for CG-CTA MMAs.  CG = 2: one warp of each CTA of the pair
+// executes it; both CTAs get the same columns.
+template <int CG>
+__device__ __forceinline__ void tmem_alloc_cg(uint32_t* slot_smem, uint32_t ncols)
+{
+    if constexpr (CG == 2)
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot_smem)),
+                     "r"(ncols)
+                     : "memory");
+    else
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot_smem)),
+                     "r"(ncols)
+                     : "memory");
+}
+
+template <int CG>
+__device__ __forceinline__ void tmem_relinquish_cg()
+{
+    if constexpr (CG == 2)
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    else
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+template <int CG>
+__device__ __forceinline__ void tmem_dealloc_cg(uint32_t taddr, uint32_t ncols)
+{
+    if constexpr (CG == 2)
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+    else
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// Elected-lane MMA.  CG = 2: M = 256 across the pair; A rows 0-127 and B columns
+// 0..N/2-1 come from the shared memory of CTA rank 0, A rows 128-255 and B columns
+// N/2..N-1 from rank 1, at the same addresses; D rows 0-127 land in rank 0's TMEM,
+// rows 128-255 in rank 1's, at the same column address.  Issued by rank 0 only.
+template <int CG>
+__device__ __forceinline__ void mma_bf16_elect_cg(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t accumulate)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E, P;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "setp.ne.b32 P, %4, 0;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, P;\n\t}" ::"r"(d_tmem),
+            "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E, P;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "setp.ne.b32 P, %4, 0;\n\t"
+            "@E tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, P;\n\t}" ::"r"(d_tmem),
+            "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+            : "memory");
+}
+
+// Elected-lane commit: arrive once on the mbarrier at shared::cta offset bar
+// when the MMAs issued so far complete.  CG = 2: the arrival goes to the
+// barrier at that offset in every CTA of cta_mask (bit r = rank r).
+template <int CG>
+__device__ __forceinline__ void mma_commit_elect_cg(uint64_t* bar, uint16_t cta_mask)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n\t}" ::
+                "r"(smem_u32(bar)),
+            "h"(cta_mask)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(smem_u32(bar))
+            : "memory");
+}
+
 // ---------------------------------------------------------------------------- tcgen05 / TMEM
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot_smem, uint32_t ncols)
 {

@@ -323,6 +323,9 @@ FWD_CASES = [  # n, h, w, c, k, r, stride, pad
     (1, 4, 4, 256, 256, 3, 1, 1),    # deep layer, small image, 256-wide tile
     (4, 14, 14, 256, 512, 3, 2, 1),  # two 256-wide column tiles, stride 2
     (32, 56, 56, 64, 64, 3, 1, 1),   # 784 tiles: every persistent CTA loops over several
+    # 256-wide tiles on CTA pairs (M = 256 across two SMs, half of B in each)
+    (32, 14, 14, 256, 256, 3, 1, 1),  # 24.5 pair tiles: the second CTA of the last pair has no rows
+    (64, 14, 14, 256, 512, 3, 2, 1),  # stride 2, two column tiles, several tiles per pair
     # 3x3 stride-1 window kernel: strips of zero-padded rows, taps as shifted descriptors
     (4, 28, 28, 128, 128, 3, 1, 1),  # streamed 128-wide weight tiles, two channel blocks
     (5, 5, 13, 128, 64, 3, 1, 1),    # streamed 64-wide tiles; a tile spans several small images
@@ -371,6 +374,8 @@ DGRAD_CASES = [
     (1, 4, 4, 256, 256, 3, 1, 1),
     (2, 8, 8, 512, 512, 3, 1, 1),    # 256-wide tiles, 8 channel blocks of dy
     (16, 28, 28, 128, 128, 3, 1, 1), # many tiles per CTA
+    (24, 14, 14, 256, 256, 3, 1, 1), # CTA pairs, ragged last pair tile
+    (6, 28, 28, 256, 512, 3, 2, 1),  # CTA pairs over stride-2 phases (4, 2, 2, 1 taps)
     (5, 5, 13, 64, 128, 3, 1, 1),    # window kernel, 64-wide streamed tiles over two dy channel blocks
     (2, 9, 30, 64, 64, 3, 1, 1),     # window kernel, resident flipped weights, non-square image
 ]
@@ -403,6 +408,8 @@ WGRAD_CASES = [
     (8, 16, 16, 64, 64, 3, 1, 1),
     (2, 8, 8, 256, 512, 3, 2, 1),    # 256-wide tiles
     (16, 28, 28, 128, 128, 3, 1, 1), # split-K slices reduced in order
+    (16, 14, 14, 256, 256, 3, 1, 1), # CTA pairs: 9 pair tiles of 256 (tap, c) rows, split-K
+    (8, 7, 7, 512, 512, 3, 1, 1),    # CTA pairs, two column tiles
     (1, 3, 3, 64, 64, 3, 1, 1),      # a single slice, written straight into dw
     # window weight gradient (64 -> 64, 3x3 stride 1): x and dy strips, five tap-pair accumulators
     (32, 56, 56, 64, 64, 3, 1, 1),   # the layer1 shape at batch 32: one K-range per CTA
