@@ -858,16 +858,13 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                         sb = sbase + (uint32_t)(bs * C::B_TILE);
                     }
                     const uint32_t a0 = sa + (uint32_t)((off0 + r * Wp + sx) * 128);
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-#pragma unroll
-                        for (int a = 0; a < kWinACC; ++a) {
-                            const uint64_t ad = smem_desc(a0 + a * 128 * 128 + 32 * j, 16, 1024, kSwizzle128B);
-                            const uint64_t bd = DG ? smem_desc(sb + 2048 * j, 8192, 1024, kSwizzle128B)
-                                                   : smem_desc(sb + 32 * j, 16, 1024, kSwizzle128B);
-                            mma_bf16_elect(d + a * BN, ad, bd, idesc, (cb > 0 || tap > 0 || j > 0) ? 1u : 0u);
-                        }
-                    }
+                    // K-step j of accumulator a: A rows a*128.. of the shifted strip, 32 bytes per K-step;
+                    // B K-major (32 bytes per K-step) or, for the data gradient, MN-major (2 KB per K-step)
+                    static_assert(kWinACC == 2, "two accumulators per MMA group");
+                    const uint64_t ad = smem_desc(a0, 16, 1024, kSwizzle128B);
+                    const uint64_t bd = DG ? smem_desc(sb, 8192, 1024, kSwizzle128B) : smem_desc(sb, 16, 1024, kSwizzle128B);
+                    mma_bf16_x8_elect(d, d + BN, ad, (128 * 128) >> 4, 32 >> 4, bd, DG ? (2048 >> 4) : (32 >> 4), idesc,
+                                      (cb > 0 || tap > 0) ? 1u : 0u);
                     if (!RES) {
                         mma_commit_elect(&bempty[bs]);
                         ++bt;
@@ -902,24 +899,33 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             }
             tc_fence_after();
             const int row = warp * 32 + lane;
-#pragma unroll 1
+            bool valid[kWinACC];
+            int64_t out_row[kWinACC];
+#pragma unroll
             for (int a = 0; a < kWinACC; ++a) {
                 const int L = tc.m_tile * p.win_tile + a * 128 + row;
                 const int n = L / img, rem = L - n * img;
                 const int hp = rem / Wp, wp = rem - hp * Wp;
                 // rows past the tile belong to the next tile (row-aligned tiles are shorter than 256)
-                const bool valid = a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P && wp < p.win_Q;
-                const int64_t out_row = ((int64_t)n * p.win_P + hp) * p.win_Q + wp;
-                const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)((buf * kWinACC + a) * BN);
+                valid[a] = a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P && wp < p.win_Q;
+                out_row[a] = ((int64_t)n * p.win_P + hp) * p.win_Q + wp;
+            }
+            // chunks c = (accumulator, 32 columns), the next chunk's TMEM load in flight while
+            // this one is converted and stored
+            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * kWinACC * BN);
+            constexpr int NCH = BN / 32, NC = kWinACC * NCH;
+            uint32_t va[32], vb[32];
+            tmem_ld_32x32b_x32(taddr, va);
 #pragma unroll
-                for (int ch = 0; ch < BN / 32; ++ch) {
-                    uint32_t v[32];
-                    tmem_ld_32x32b_x32(taddr + ch * 32, v);
-                    tmem_ld_wait();
-                    float back[32];
-                    store_row_chunk_bf16(p, v, valid, out_row, tc.n_tile * BN + ch * 32, back);
-                    if (want_stats) rs.add(ch, back, lane);
-                }
+            for (int c = 0; c < NC; ++c) {
+                uint32_t(&cur)[32] = (c & 1) ? vb : va;
+                uint32_t(&nxt)[32] = (c & 1) ? va : vb;
+                tmem_ld_wait_regs(cur);
+                if (c + 1 < NC) tmem_ld_32x32b_x32(taddr + (uint32_t)((c + 1) * 32), nxt);
+                const int a = c / NCH, ch = c % NCH;
+                float back[32];
+                store_row_chunk_bf16(p, cur, valid[a], out_row[a], tc.n_tile * BN + ch * 32, back);
+                if (want_stats) rs.add(ch, back, lane);
             }
             tc_fence_before();
             __syncwarp();
@@ -1427,15 +1433,19 @@ bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
     return true;
 }
 
-// Tiles of BN = 256 columns run on CTA pairs (see conv_igemm_kernel), unless the
-// environment variable DBL_CONV_CTA_PAIRS is set to 0.
-bool pair_tiles(int BN)
+// Which tiles run on CTA pairs (see conv_igemm_kernel): 256-column tiles, and the
+// 128-column tiles of the weight gradient (its long K-blocks amortise the pair's
+// extra synchronisation; the short-K forward and data-gradient passes of 128
+// columns measured slower on pairs).  The environment variable DBL_CONV_CTA_PAIRS
+// overrides this: 0 = never, 2 = every 128- and 256-column tile.
+bool pair_tiles(int BN, bool wgrad)
 {
-    static const bool enabled = [] {
+    static const int level = [] {
         const char* e = getenv("DBL_CONV_CTA_PAIRS");
-        return !(e && e[0] == '0');
+        return e && (e[0] == '0' || e[0] == '2') ? e[0] - '0' : 1;
     }();
-    return enabled && BN == 256;
+    if (level == 0) return false;
+    return BN == 256 || (BN == 128 && (wgrad || level == 2));
 }
 
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
@@ -1468,7 +1478,7 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
         p.M = (int)M;
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
-        pl.cg = pair_tiles(pl.BN) ? 2 : 1;
+        pl.cg = !c8 && pair_tiles(pl.BN, false) ? 2 : 1;
         p.m_tiles = (p.M + pl.cg * fwd_tile_rows(pl.BN) - 1) / (pl.cg * fwd_tile_rows(pl.BN));
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;
@@ -1548,14 +1558,14 @@ int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
             }
             p.phase_off[4] = t;
         }
-        pl.cg = pair_tiles(pl.BN) ? 2 : 1;
+        pl.cg = pair_tiles(pl.BN, false) ? 2 : 1;
         p.m_tiles = (p.M + pl.cg * fwd_tile_rows(pl.BN) - 1) / (pl.cg * fwd_tile_rows(pl.BN));
     } else {
         pl.mode = p.mode = c8 ? kWgradC8 : kWgrad;
         p.M = p.ntaps * s->c;  // D rows = (tap, c)
         p.Ncols = s->k;
         pl.BN = c8 ? 64 : choose_bn(s->k);
-        pl.cg = !c8 && pair_tiles(pl.BN) ? 2 : 1;
+        pl.cg = !c8 && pair_tiles(pl.BN, true) ? 2 : 1;
         p.m_tiles = c8 ? (p.ntaps + 15) / 16 : (p.M + pl.cg * BM - 1) / (pl.cg * BM);
         p.n_tiles = s->k / pl.BN;
         p.gN = s->n;

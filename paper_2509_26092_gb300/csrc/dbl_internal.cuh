@@ -542,6 +542,38 @@ __device__ __forceinline__ void mma_bf16_elect_cg(uint32_t d_tmem, uint64_t a_de
             : "memory");
 }
 
+// Four K-steps of two accumulators (8 MMAs, cta_group::1) from one elected lane in
+// one asm block: D[d0] and D[d1] (+)= A * B for K-step j = 0..3 with descriptors
+// a0 + j*a_step (accumulator 0), a0 + a1_off + j*a_step (accumulator 1) and
+// b0 + j*b_step (all in descriptor units of 16 bytes).  K-step 0 accumulates only
+// if acc0 != 0; K-steps 1..3 always accumulate.  Keeping the whole group inside
+// one asm block (no per-MMA elect or predicate set-up in between) is what lets
+// N = 64 MMAs, which the tensor pipe finishes in 48 cycles, issue back to back.
+__device__ __forceinline__ void mma_bf16_x8_elect(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
+                                                  uint64_t a_step, uint64_t b0, uint64_t b_step, uint32_t idesc,
+                                                  uint32_t acc0)
+{
+    asm volatile(
+        "{\n\t.reg .pred E, P, T;\n\t.reg .b32 l;\n\t.reg .b64 a, c, b;\n\t"
+        "elect.sync l|E, 0xffffffff;\n\t"
+        "setp.ne.b32 P, %8, 0;\n\t"
+        "setp.eq.b32 T, 0, 0;\n\t"
+        "add.s64 c, %2, %3;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %5, %7, P;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%1], c, %5, %7, P;\n\t"
+        "add.s64 a, %2, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, %5, %6;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %7, T;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%1], c, b, %7, T;\n\t"
+        "add.s64 a, a, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, b, %6;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %7, T;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%1], c, b, %7, T;\n\t"
+        "add.s64 a, a, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, b, %6;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %7, T;\n\t"
+        "@E tcgen05.mma.cta_group::1.kind::f16 [%1], c, b, %7, T;\n\t}" ::"r"(d0),
+        "r"(d1), "l"(a0), "l"(a1_off), "l"(a_step), "l"(b0), "l"(b_step), "r"(idesc), "r"(acc0)
+        : "memory");
+}
+
 // Elected-lane commit: arrive once on the mbarrier at shared::cta offset bar
 // when the MMAs issued so far complete.  CG = 2: the arrival goes to the
 // barrier at that offset in every CTA of cta_mask (bit r = rank r).
@@ -645,6 +677,21 @@ __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)
 }
 
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Wait for this thread's outstanding tcgen05.ld; r (the destination of one of them)
+// is passed through the wait so that the compiler reads it only afterwards.  With
+// it a thread can keep the next chunk's load in flight while it works on this one.
+__device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32])
+{
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                   "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                   "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+                 :
+                 : "memory");
+}
 
 // ---------------------------------------------------------------------------- UMMA descriptors
 // Shared-memory matrix descriptor (tcgen05): start address, leading and

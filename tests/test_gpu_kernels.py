@@ -376,6 +376,7 @@ DGRAD_CASES = [
     (16, 28, 28, 128, 128, 3, 1, 1), # many tiles per CTA
     (24, 14, 14, 256, 256, 3, 1, 1), # CTA pairs, ragged last pair tile
     (6, 28, 28, 256, 512, 3, 2, 1),  # CTA pairs over stride-2 phases (4, 2, 2, 1 taps)
+    (8, 28, 28, 128, 256, 3, 2, 1),  # 128-wide tiles over stride-2 phases
     (5, 5, 13, 64, 128, 3, 1, 1),    # window kernel, 64-wide streamed tiles over two dy channel blocks
     (2, 9, 30, 64, 64, 3, 1, 1),     # window kernel, resident flipped weights, non-square image
 ]
