@@ -270,19 +270,28 @@ def conv_roofline(stage, reps=4, replays=2, table=None):
             continue
         stem = wk.spec.stem.name
         bufs = _conv_buffers(wk)
+        shapes = dict(wk.conv_shapes())
         for name, shp in wk.conv_shapes():
             x, y, dy, dx, w16, g = bufs[name]
             st_sum = torch.empty(shp.k, device=x.device)
             st_sq = torch.empty(shp.k, device=x.device)
             f1 = float(wk.layer_flops(name, shp))
-            passes = [("fwd", lambda s: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            passes = [("fwd", f1, lambda s: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
             algo_bytes += nbytes(x, w16, y)
-            if name != stem:
-                passes.append(("dgrad", lambda s: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
+            proj = name.replace(".conv1", ".down") if name.endswith(".conv1") else None
+            if proj in bufs:
+                # a downsampling block's input gradient: conv1's and the projection's in one pass
+                _, _, dy2, _, w2, _ = bufs[proj]
+                fd = f1 + float(wk.layer_flops(proj, shapes[proj]))
+                passes.append(("dgrad+proj", fd, lambda s: D.dbl_conv_dgrad_proj(shp, dy, w16, shapes[proj].k, dy2, w2,
+                                                                                 dx, None, 0, s)))
+                algo_bytes += nbytes(dy, w16, dy2, w2, dx)
+            elif name != stem and dx is not None:
+                passes.append(("dgrad", f1, lambda s: D.dbl_conv_dgrad(shp, dy, w16, dx, None, 0, s)))
                 algo_bytes += nbytes(dy, w16, dx)
-            passes.append(("wgrad", lambda s: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
+            passes.append(("wgrad", f1, lambda s: D.dbl_conv_wgrad(shp, x, dy, g, False, wk.ws, wk.ws.numel(), s)))
             algo_bytes += nbytes(x, dy, g)
-            for pname, fn in passes:
+            for pname, fp, fn in passes:
                 fn(torch.cuda.current_stream())
                 torch.cuda.synchronize()
                 graph = torch.cuda.CUDAGraph()
@@ -300,9 +309,9 @@ def conv_roofline(stage, reps=4, replays=2, table=None):
                 del graph
                 t1 = ev[0].elapsed_time(ev[1]) / 1000.0 / (reps * replays)
                 secs += t1
-                flops += f1
+                flops += fp
                 if table is not None:
-                    table.append((wk.batch, name, pname, f1, t1))
+                    table.append((wk.batch, name, pname, fp, t1))
     return flops, secs, algo_bytes
 
 
@@ -321,7 +330,7 @@ def _conv_buffers(wk):
         out[b.pre + ".conv2"] = (d["o1"], d["h2"], d["dh2"], d["do1"], spec.view(srv_w16, b.pre + ".conv2.w"),
                                  spec.view(wk.grad, b.pre + ".conv2.w"))
         if b.proj:
-            out[b.pre + ".down"] = (cur, d["hs"], d["dhs"], d["din2"], spec.view(srv_w16, b.pre + ".down.w"),
+            out[b.pre + ".down"] = (cur, d["hs"], d["dhs"], None, spec.view(srv_w16, b.pre + ".down.w"),
                                     spec.view(wk.grad, b.pre + ".down.w"))
         cur = d["out"]
     return out

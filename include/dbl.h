@@ -110,6 +110,18 @@ DBL_API int dbl_conv_fwd(const dbl_conv_shape* shape, const void* x_bf16, const 
 DBL_API int dbl_conv_dgrad(const dbl_conv_shape* shape, const void* dy_bf16, const void* w_bf16, void* dx_bf16, void* ws,
                    size_t ws_bytes, void* stream);
 
+/* Data gradient of a downsampling ResNet-18 block input (Sec. 5.1.1): the
+ * block's first convolution (shape, stride 2) and its 1x1 stride-2 pad-0
+ * projection shortcut both read the same input x, so
+ *   dx = dgrad(shape; dy, w) + dgrad(1x1/2; dy2, w2),
+ * computed in one pass (the projection term reaches only the even rows and
+ * columns of dx, where it is accumulated with the main term).
+ * dy2: [n, h/2, w/2, k2] bf16, w2: [k2, 1, 1, c] bf16; k2 a multiple of 64.
+ * Requires stride 2 and even h, w.  dx is fully overwritten. */
+DBL_API int dbl_conv_dgrad_proj(const dbl_conv_shape* shape, const void* dy_bf16, const void* w_bf16, int32_t k2,
+                                const void* dy2_bf16, const void* w2_bf16, void* dx_bf16, void* ws, size_t ws_bytes,
+                                void* stream);
+
 /* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*stride+r-pad, q*stride+s-pad, c],
  * fp32 [k,r,s,c].  accumulate != 0 adds to dw instead of overwriting it.
  * The split over n*P*Q is reduced in a fixed order (deterministic). */

@@ -64,6 +64,7 @@ struct ConvParams {
     int out_h, out_w;   // full dx spatial size
     int phase_off[5];
     int8_t tap_r[16], tap_s[16], tap_oh[16], tap_ow[16];
+    int proj_kb;        // dgrad phase (0,0): extra K-blocks of a 1x1 stride-2 projection's dy2 . w2
     // outputs
     void* out;          // bf16 rows (fwd, dgrad); fp32 dw (wgrad, one slice) or fp32 slices [z][Ncols][M]
     int64_t ldo;        // elements between output rows (fwd, dgrad)
@@ -154,7 +155,7 @@ __device__ __forceinline__ void kb_range(const ConvParams& p, int z, int& kb0, i
 {
     if (p.mode == kDgrad) {
         kb0 = 0;
-        nkb = (p.phase_off[z + 1] - p.phase_off[z]) * p.cblocks;
+        nkb = (p.phase_off[z + 1] - p.phase_off[z]) * p.cblocks + (z == 0 ? p.proj_kb : 0);
     } else if (p.mode == kWgrad || p.mode == kWgradC8) {
         kb0 = z * p.kb_per_split;
         nkb = min(p.num_kb, kb0 + p.kb_per_split) - kb0;
@@ -172,8 +173,9 @@ __device__ __forceinline__ void kb_range(const ConvParams& p, int z, int& kb0, i
 // rank 0's barrier.
 template <int BN, int FAM, int CG>
 __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorMap* tmA, const CUtensorMap* tmB,
-                                            uint8_t* sa, uint8_t* sb, uint32_t fb, const TileCoord& tc, int kb, int tn,
-                                            int tp, int tq, int rank)
+                                            const CUtensorMap* tmA2, const CUtensorMap* tmB2, uint8_t* sa,
+                                            uint8_t* sb, uint32_t fb, const TileCoord& tc, int kb, int tn, int tp,
+                                            int tq, int rank)
 {
     using C = Cfg<BN, FAM, CG>;
     const int64_t gPQ = (int64_t)p.gP * p.gQ;
@@ -185,6 +187,14 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
             tma_load_im2col_4d_cg<CG>(sa, tmA, fb, cb * 64, tq * p.tstride_w + p.base_w, tp * p.tstride_h + p.base_h, tn,
                                       (uint16_t)sx, (uint16_t)r);
             tma_load_2d_cg<CG>(sb, tmB, fb, tap * p.Cin + cb * 64, ncol0);
+        } else if (p.mode == kDgrad && kb >= (p.phase_off[tc.z + 1] - p.phase_off[tc.z]) * p.cblocks) {
+            // phase (0,0) of a stride-2 data gradient with a 1x1 stride-2 projection shortcut on
+            // the same input: dx[n, 2i, 2j] also receives dy2[n, i, j] . w2, the dy2 rows of this
+            // tile being the tile's own rows m0.. (tmA2: dy2 as [n*P*Q][k2], tmB2: w2 as [k2][1][c])
+            const int e = kb - (p.phase_off[tc.z + 1] - p.phase_off[tc.z]) * p.cblocks;
+            const int m0 = (tn * p.gP + tp) * p.gQ + tq;
+            tma_load_2d_cg<CG>(sa, tmA2, fb, e * 64, m0);
+            for (int j = 0; j < C::BNC / 64; ++j) tma_load_3d_cg<CG>(sb + j * 8192, tmB2, fb, ncol0 + 64 * j, 0, e * 64);
         } else if (p.mode == kDgrad) {
             const int t = p.phase_off[tc.z] + kb / p.cblocks, kbk = kb % p.cblocks;
             tma_load_im2col_4d_cg<CG>(sa, tmA, fb, kbk * 64, tq + p.base_w, tp + p.base_h, tn, (uint16_t)p.tap_ow[t],
@@ -347,6 +357,7 @@ struct RowStats {
 template <int BN, int FAM, int CG>
 __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
                       const ConvParams p)
 {
     using C = Cfg<BN, FAM, CG>;
@@ -383,6 +394,10 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
     if (warp >= 4 && warp < 4 + kProducers && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
+        if (p.proj_kb) {
+            tma_prefetch_desc(&tmA2);
+            tma_prefetch_desc(&tmB2);
+        }
     }
     if (warp == C::MMA_WARP) {
         tmem_alloc_cg<CG>(&tmem_slot, C::TMEM_COLS);
@@ -425,7 +440,8 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
                 if (CG == 1 || rank == 0)
                     mbar_arrive_expect_tx_elect(&full_bar[s], (uint32_t)(CG * C::STAGE_BYTES));
                 if (CG == 2) fb = mapa_shared(fb, 0);
-                load_kblock<BN, FAM, CG>(p, &tmA, &tmB, sa, sa + C::A_BYTES, fb, tc, kb0 + k, tn, tp, tq, rank);
+                load_kblock<BN, FAM, CG>(p, &tmA, &tmB, &tmA2, &tmB2, sa, sa + C::A_BYTES, fb, tc, kb0 + k, tn, tp, tq,
+                                         rank);
                 last_it = it;
             }
             if (failed) break;
@@ -1684,13 +1700,14 @@ int plan_grid(const Plan& pl)
 }
 
 template <int BN, int FAM, int CG>
-int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& a2,
+               const CUtensorMap& b2, int grid, cudaStream_t st)
 {
     using Cf = Cfg<BN, FAM, CG>;
     int rc = set_igemm_smem<BN, FAM, CG>();
     if (rc) return rc;
     if constexpr (CG == 1) {
-        conv_igemm_kernel<BN, FAM, 1><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, pl.p);
+        conv_igemm_kernel<BN, FAM, 1><<<grid, Cf::THREADS, Cf::SMEM, st>>>(a, b, a2, b2, pl.p);
     } else {
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute at[1];
@@ -1704,7 +1721,7 @@ int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int g
         cfg.stream = st;
         cfg.attrs = at;
         cfg.numAttrs = 1;
-        cudaError_t e = cudaLaunchKernelEx(&cfg, conv_igemm_kernel<BN, FAM, 2>, a, b, pl.p);
+        cudaError_t e = cudaLaunchKernelEx(&cfg, conv_igemm_kernel<BN, FAM, 2>, a, b, a2, b2, pl.p);
         if (e != cudaSuccess) {
             dbl::count_launch();
             return dbl::cuda_check(e, "conv_igemm pair launch");
@@ -1713,24 +1730,26 @@ int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int g
     return dbl::launch_check("conv_igemm launch");
 }
 
-int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+// a2, b2: the projection operands of a fused data gradient (unused otherwise).
+int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& a2, const CUtensorMap& b2,
+           int grid, cudaStream_t st)
 {
     const bool wg = pl.mode == kWgrad || pl.mode == kWgradC8;
     if (pl.cg == 2) {
-        if (pl.BN == 256) return wg ? launch_cfg<256, kFamWgrad, 2>(pl, a, b, grid, st)
-                                    : launch_cfg<256, kFamFwd, 2>(pl, a, b, grid, st);
-        if (pl.BN == 128) return wg ? launch_cfg<128, kFamWgrad, 2>(pl, a, b, grid, st)
-                                    : launch_cfg<128, kFamFwd, 2>(pl, a, b, grid, st);
+        if (pl.BN == 256) return wg ? launch_cfg<256, kFamWgrad, 2>(pl, a, b, a2, b2, grid, st)
+                                    : launch_cfg<256, kFamFwd, 2>(pl, a, b, a2, b2, grid, st);
+        if (pl.BN == 128) return wg ? launch_cfg<128, kFamWgrad, 2>(pl, a, b, a2, b2, grid, st)
+                                    : launch_cfg<128, kFamFwd, 2>(pl, a, b, a2, b2, grid, st);
         return dbl::set_error(DBL_ERR_UNSUPPORTED, "conv: CTA pairs need 128 or 256 columns per tile");
     }
     if (wg) {
-        if (pl.BN == 256) return launch_cfg<256, kFamWgrad, 1>(pl, a, b, grid, st);
-        if (pl.BN == 128) return launch_cfg<128, kFamWgrad, 1>(pl, a, b, grid, st);
-        return launch_cfg<64, kFamWgrad, 1>(pl, a, b, grid, st);
+        if (pl.BN == 256) return launch_cfg<256, kFamWgrad, 1>(pl, a, b, a2, b2, grid, st);
+        if (pl.BN == 128) return launch_cfg<128, kFamWgrad, 1>(pl, a, b, a2, b2, grid, st);
+        return launch_cfg<64, kFamWgrad, 1>(pl, a, b, a2, b2, grid, st);
     }
-    if (pl.BN == 256) return launch_cfg<256, kFamFwd, 1>(pl, a, b, grid, st);
-    if (pl.BN == 128) return launch_cfg<128, kFamFwd, 1>(pl, a, b, grid, st);
-    return launch_cfg<64, kFamFwd, 1>(pl, a, b, grid, st);
+    if (pl.BN == 256) return launch_cfg<256, kFamFwd, 1>(pl, a, b, a2, b2, grid, st);
+    if (pl.BN == 128) return launch_cfg<128, kFamFwd, 1>(pl, a, b, a2, b2, grid, st);
+    return launch_cfg<64, kFamFwd, 1>(pl, a, b, a2, b2, grid, st);
 }
 
 template <int BN, bool DG, bool RES>
@@ -1787,6 +1806,60 @@ int enc_win_rows(CUtensorMap* m, const void* base, int N, int H, int W, int C, i
 
 // Rows of one tile of the forward family (see Cfg).
 int fwd_tile_rows(int BN) { return BN <= 128 ? 256 : 128; }
+
+// Data gradient, optionally with the projection shortcut of a ResNet block fused in:
+// k2 > 0 adds dgrad of a 1x1 stride-2 pad-0 convolution of the same input (dy2:
+// [n, h/2, w/2, k2], w2: [k2][c]) to phase (0,0), the only phase it reaches.
+int conv_dgrad_impl(const dbl_conv_shape* s, const void* dy, const void* w, int k2, const void* dy2, const void* w2,
+                    void* dx, void* stream, const char* who)
+{
+    using namespace dbl;
+    Plan pl;
+    int rc = make_plan(s, DBL_PASS_DGRAD, pl);
+    if (rc) return rc;
+    if (!dy || !w || !dx || !aligned16(dy) || !aligned16(w) || !aligned16(dx))
+        return set_error(DBL_ERR_INVALID, "%s: null or misaligned tensor", who);
+    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
+    CUtensorMap ta, tb, ta2, tb2;
+    if (pl.win) {
+        if ((rc = enc_win_rows(&ta, dy, s->n, P, Q, s->k, pl.p.win_Wp))) return rc;
+    } else {
+        // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
+        int lower = 0, upper = 0;
+        if (s->stride == 1) {
+            lower = -(s->r - 1 - s->pad);
+            upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
+        }
+        if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, lower, upper, 1, 1, 64, fwd_tile_rows(pl.BN),
+                             true)))
+            return rc;
+    }
+    // w viewed as [k][r*s][c]: inner c, then tap, then k
+    cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
+    cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
+    cuuint32_t box[3] = {64, 1, 64};
+    if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
+    ta2 = ta;
+    tb2 = tb;
+    if (k2 > 0) {
+        if (pl.win || pl.p.phase_div != 2)
+            return set_error(DBL_ERR_UNSUPPORTED, "%s: the projection needs the stride-2 phase path", who);
+        // dy2 [n, h/2, w/2, k2] = the phase grid's rows, as [n*P*Q][k2]
+        cuuint64_t d2[2] = {(cuuint64_t)k2, (cuuint64_t)s->n * pl.p.gP * pl.p.gQ};
+        cuuint64_t s2[1] = {(cuuint64_t)k2 * 2};
+        cuuint32_t bx2[2] = {64, (cuuint32_t)fwd_tile_rows(pl.BN)};
+        if ((rc = enc_tiled(&ta2, dy2, 2, d2, s2, bx2, true))) return rc;
+        // w2 [k2][c] viewed as [k2][1][c], loaded like one tap of w
+        cuuint64_t d3[3] = {(cuuint64_t)s->c, 1, (cuuint64_t)k2};
+        cuuint64_t s3[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->c * 2};
+        if ((rc = enc_tiled(&tb2, w2, 3, d3, s3, box, true))) return rc;
+        pl.p.proj_kb = k2 / 64;
+    }
+    pl.p.out = dx;
+    const int grid = plan_grid(pl);
+    return pl.win ? launch_win(pl, ta, tb, grid, as_stream(stream))
+                  : launch(pl, ta, tb, ta2, tb2, grid, as_stream(stream));
+}
 
 }  // namespace
 
@@ -1845,7 +1918,7 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
     pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
     const int grid = plan_grid(pl);
     cudaStream_t st = as_stream(stream);
-    if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, grid, st))) return rc;
+    if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, ta, tb, grid, st))) return rc;
     if (stats) {
         stats_reduce_kernel<<<(s->k + 31) / 32, 32 * kColsumGroups, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
         if ((rc = launch_check("conv stats reduce"))) return rc;
@@ -1856,37 +1929,26 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
 int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void* dx, void* ws, size_t ws_bytes,
                    void* stream)
 {
-    using namespace dbl;
     (void)ws;
     (void)ws_bytes;
-    Plan pl;
-    int rc = make_plan(s, DBL_PASS_DGRAD, pl);
-    if (rc) return rc;
-    if (!dy || !w || !dx || !aligned16(dy) || !aligned16(w) || !aligned16(dx))
-        return set_error(DBL_ERR_INVALID, "conv_dgrad: null or misaligned tensor");
-    const int P = out_dim(s->h, s->r, s->stride, s->pad), Q = out_dim(s->w, s->s, s->stride, s->pad);
-    CUtensorMap ta, tb;
-    if (pl.win) {
-        if ((rc = enc_win_rows(&ta, dy, s->n, P, Q, s->k, pl.p.win_Wp))) return rc;
-    } else {
-        // im2col over dy [n, P, Q, k]: origins cover the dx grid (stride 1) or one phase grid (stride 2)
-        int lower = 0, upper = 0;
-        if (s->stride == 1) {
-            lower = -(s->r - 1 - s->pad);
-            upper = (s->h - 1 + lower) - (P - 1);  // origin range [lower, H-1+lower] against dy's extent P
-        }
-        if ((rc = enc_im2col(&ta, dy, s->n, P, Q, s->k, lower, upper, lower, upper, 1, 1, 64, fwd_tile_rows(pl.BN),
-                             true)))
-            return rc;
-    }
-    // w viewed as [k][r*s][c]: inner c, then tap, then k
-    cuuint64_t dims[3] = {(cuuint64_t)s->c, (cuuint64_t)s->r * s->s, (cuuint64_t)s->k};
-    cuuint64_t str[2] = {(cuuint64_t)s->c * 2, (cuuint64_t)s->r * s->s * s->c * 2};
-    cuuint32_t box[3] = {64, 1, 64};
-    if ((rc = enc_tiled(&tb, w, 3, dims, str, box, true))) return rc;
-    pl.p.out = dx;
-    const int grid = plan_grid(pl);
-    return pl.win ? launch_win(pl, ta, tb, grid, as_stream(stream)) : launch(pl, ta, tb, grid, as_stream(stream));
+    return conv_dgrad_impl(s, dy, w, 0, nullptr, nullptr, dx, stream, "conv_dgrad");
+}
+
+int dbl_conv_dgrad_proj(const dbl_conv_shape* s, const void* dy, const void* w, int32_t k2, const void* dy2,
+                        const void* w2, void* dx, void* ws, size_t ws_bytes, void* stream)
+{
+    (void)ws;
+    (void)ws_bytes;
+    using dbl::set_error;
+    if (!s) return set_error(DBL_ERR_INVALID, "conv_dgrad_proj: null shape");
+    if (s->stride != 2 || (s->stride_w && s->stride_w != 2))
+        return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad_proj: the main convolution must have stride 2");
+    if (k2 <= 0 || k2 % 64 || k2 > kMaxNcols)
+        return set_error(DBL_ERR_UNSUPPORTED, "conv_dgrad_proj: projection channels must be a multiple of 64, <= %d",
+                         kMaxNcols);
+    if (!dy2 || !w2 || !dbl::aligned16(dy2) || !dbl::aligned16(w2))
+        return set_error(DBL_ERR_INVALID, "conv_dgrad_proj: null or misaligned projection tensor");
+    return conv_dgrad_impl(s, dy, w, k2, dy2, w2, dx, stream, "conv_dgrad_proj");
 }
 
 int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float* dw, int accumulate, void* ws,
@@ -1923,7 +1985,7 @@ int dbl_conv_wgrad(const dbl_conv_shape* s, const void* x, const void* dy, float
     if ((rc = enc_tiled(&tb, dy, 2, dims, str, box, true))) return rc;
     pl.p.out = sliced ? ws : static_cast<void*>(dw);
     pl.p.wg_accumulate = accumulate;
-    if ((rc = launch(pl, ta, tb, plan_grid(pl), st))) return rc;
+    if ((rc = launch(pl, ta, tb, ta, tb, plan_grid(pl), st))) return rc;
     }
     if (!sliced) return DBL_OK;
     const int64_t n = (int64_t)pl.p.M * s->k;

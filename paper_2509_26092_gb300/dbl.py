@@ -65,6 +65,7 @@ def lib():
             "dbl_conv_fwd": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _V, _V, _SZ, _V]),
             "dbl_conv_dgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _SZ, _V]),
             "dbl_conv_wgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, ctypes.c_int, _V, _SZ, _V]),
+            "dbl_conv_dgrad_proj": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _I32, _V, _V, _V, _V, _SZ, _V]),
             "dbl_bn_stats": (ctypes.c_int, [ctypes.POINTER(BnShape), _V, _V, _V, _V]),
             "dbl_bn_relu_fused": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 10),
             "dbl_bn_workspace_bytes": (_SZ, [ctypes.POINTER(BnShape)]),
@@ -155,6 +156,11 @@ def dbl_conv_fwd(shape, x, w, y, ch_sum=None, ch_sumsq=None, ws=None, ws_bytes=0
 def dbl_conv_dgrad(shape, dy, w, dx, ws=None, ws_bytes=0, stream=None):
     _check(lib().dbl_conv_dgrad(ctypes.byref(shape), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws), ws_bytes,
                                 _stream(stream)))
+
+
+def dbl_conv_dgrad_proj(shape, dy, w, k2, dy2, w2, dx, ws=None, ws_bytes=0, stream=None):
+    _check(lib().dbl_conv_dgrad_proj(ctypes.byref(shape), _ptr(dy), _ptr(w), int(k2), _ptr(dy2), _ptr(w2), _ptr(dx),
+                                     _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def dbl_conv_wgrad(shape, x, dy, dw, accumulate=False, ws=None, ws_bytes=0, stream=None):

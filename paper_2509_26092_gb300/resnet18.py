@@ -258,7 +258,9 @@ class Worker:
         for b in spec.blocks:
             ho = conv_out(h, 3, b.stride, 1)
             d = dict(spec=b, hin=h, hout=ho)
-            for k in ("h1", "o1", "h2", "out", "dh2", "do1", "dh1", "din", "din2"):
+            # din: the block input's gradient through conv1 (with the projection shortcut's gradient
+            # fused in, for a downsampling block); din2: the identity shortcut's gradient
+            for k in ("h1", "o1", "h2", "out", "dh2", "do1", "dh1", "din") + (() if b.proj else ("din2",)):
                 d[k] = act(ho if k not in ("din", "din2") else h, b.cout if k not in ("din", "din2") else b.cin)
             if b.proj:
                 d["hs"], d["sc"], d["dhs"] = act(ho, b.cout), act(ho, b.cout), act(ho, b.cout)
@@ -425,7 +427,6 @@ class Worker:
                                     gv(b.pre + ".bn1.b"), ws, wsb, s, beta=pv(b.pre + ".bn1.b"))
             s1 = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)
             D.dbl_conv_wgrad(s1, d["x"], d["dh1"], gv(b.pre + ".conv1.w"), False, ws, wsb, s)
-            D.dbl_conv_dgrad(s1, d["dh1"], wv(b.pre + ".conv1.w"), d["din"], None, 0, s)
             if b.proj:
                 # the shortcut BatchNorm sees the same masked gradient g as bn2 (no ReLU of its own)
                 D.dbl_bn_relu_fused_bwd(D.bn_shape(cnt, b.cout, eps, False), g, None, d["hs"], None,
@@ -433,8 +434,13 @@ class Worker:
                                         gv(b.pre + ".downbn.g"), gv(b.pre + ".downbn.b"), ws, wsb, s)
                 sd = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)
                 D.dbl_conv_wgrad(sd, d["x"], d["dhs"], gv(b.pre + ".down.w"), False, ws, wsb, s)
-                D.dbl_conv_dgrad(sd, d["dhs"], wv(b.pre + ".down.w"), d["din2"], None, 0, s)
-            dout, dout2 = d["din"], d["din2"]
+                # the block input's gradient through conv1 and the projection, in one pass
+                D.dbl_conv_dgrad_proj(s1, d["dh1"], wv(b.pre + ".conv1.w"), b.cout, d["dhs"], wv(b.pre + ".down.w"),
+                                      d["din"], None, 0, s)
+                dout, dout2 = d["din"], None
+            else:
+                D.dbl_conv_dgrad(s1, d["dh1"], wv(b.pre + ".conv1.w"), d["din"], None, 0, s)
+                dout, dout2 = d["din"], d["din2"]
         bns = D.bn_shape(B * self.stem_hw ** 2, st.cout, eps, True)
         if spec.variant == "imagenet":
             D.dbl_maxpool_bwd(B, self.stem_hw, self.stem_hw, st.cout, dout, dout2, self.pool_arg, self.stem_da, s)

@@ -98,6 +98,13 @@ def test_invalid_arguments_rejected_before_launch(D):
     assert L.dbl_conv_wgrad(ctypes.byref(s), 16, 16, 16, 0, None, 0, None) == D.DBL_ERR_WORKSPACE
     s = D.ConvShape(2, 8, 8, 8, 64, 7, 7, 2, 3)
     assert L.dbl_conv_dgrad(ctypes.byref(s), 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
+    # fused projection data gradient: stride 2 only, 64-multiple projection channels, both tensors given
+    s = D.ConvShape(2, 8, 8, 64, 128, 3, 3, 1, 1)
+    assert L.dbl_conv_dgrad_proj(ctypes.byref(s), 16, 16, 128, 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
+    s = D.ConvShape(2, 8, 8, 64, 128, 3, 3, 2, 1)
+    assert L.dbl_conv_dgrad_proj(ctypes.byref(s), 16, 16, 96, 16, 16, 16, None, 0, None) == D.DBL_ERR_UNSUPPORTED
+    assert L.dbl_conv_dgrad_proj(ctypes.byref(s), 16, 16, 128, None, 16, 16, None, 0, None) == D.DBL_ERR_INVALID
+    assert L.dbl_conv_dgrad_proj(ctypes.byref(s), 16, 16, 128, 24, 16, 16, None, 0, None) == D.DBL_ERR_INVALID
     # resize: upsampling
     assert L.dbl_progressive_resize(16, 0, 1, 8, 8, 3, 16, 1, 16, 16, 8, None) == D.DBL_ERR_UNSUPPORTED
     assert L.dbl_progressive_resize_stem(16, 1, 8, 8, 3, 16, 16, 16, 7, 2, 3, 1, 0, 16, None) == D.DBL_ERR_UNSUPPORTED

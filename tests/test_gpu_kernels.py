@@ -398,6 +398,31 @@ def test_conv_dgrad_matches_oracle(D, case):
     check_status(D)
 
 
+@pytest.mark.parametrize("n,h,c,k,k2", [(2, 8, 64, 128, 128), (3, 14, 128, 256, 256), (4, 14, 256, 512, 512),
+                                        (2, 10, 64, 128, 64)])
+def test_conv_dgrad_with_projection_matches_oracle(D, n, h, c, k, k2):
+    """Block-input gradient of a downsampling block: the 3x3 stride-2 convolution's data
+    gradient plus that of the 1x1 stride-2 projection shortcut, in one pass."""
+    g = rng(n * 1000 + c)
+    x = bf16_values(g.standard_normal((n, h, h, c)))
+    wt = bf16_values(g.standard_normal((k, 3, 3, c)) * np.sqrt(2.0 / (9 * c)))
+    w2 = bf16_values(g.standard_normal((k2, 1, 1, c)) * np.sqrt(2.0 / c))
+    P = h // 2
+    dy = bf16_values(g.standard_normal((n, P, P, k)))
+    dy2 = bf16_values(g.standard_normal((n, P, P, k2)))
+    ref = orc.conv2d_dgrad(dy, wt, x.shape, 2, 1) + orc.conv2d_dgrad(dy2, w2, x.shape, 2, 0)
+    shape = D.conv_shape(n, h, h, c, k, 3, 2, 1)
+    dx = torch.full((n, h, h, c), float("nan"), dtype=torch.bfloat16, device="cuda")
+    D.dbl_conv_dgrad_proj(shape, to_bf16_dev(dy), to_bf16_dev(wt), k2, to_bf16_dev(dy2), to_bf16_dev(w2), dx)
+    got = host(dx)
+    assert np.all(np.isfinite(got))
+    assert max_norm_rel(got, ref) <= CONV_TOL
+    # the odd rows and columns carry the main term only
+    ref_main = orc.conv2d_dgrad(dy, wt, x.shape, 2, 1)
+    assert max_norm_rel(got[:, 1::2, :, :], ref_main[:, 1::2, :, :]) <= CONV_TOL
+    check_status(D)
+
+
 WGRAD_CASES = [
     (2, 8, 8, 64, 64, 3, 1, 1),
     (5, 7, 7, 64, 64, 3, 1, 1),      # ragged pixel count

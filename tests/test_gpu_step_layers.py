@@ -114,8 +114,7 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
         chk(b.pre + ".conv1.wgrad", G[b.pre + ".conv1.w"], orc.conv2d_wgrad(x, h(d["dh1"]),
                                                                               W16[b.pre + ".conv1.w"].shape, b.stride,
                                                                               1))
-        chk(b.pre + ".conv1.dgrad", h(d["din"]), orc.conv2d_dgrad(h(d["dh1"]), W16[b.pre + ".conv1.w"], x.shape,
-                                                                  b.stride, 1))
+        din_ref = orc.conv2d_dgrad(h(d["dh1"]), W16[b.pre + ".conv1.w"], x.shape, b.stride, 1)
         if b.proj:
             std = [h(t) for t in d["downbn"]]
             dhs, dgs, dbs, _ = orc.bn_bwd(dout, h(d["out"]), h(d["hs"]), P[b.pre + ".downbn.g"], std[2], std[3],
@@ -124,14 +123,17 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
             chk(b.pre + ".down.wgrad", G[b.pre + ".down.w"], orc.conv2d_wgrad(x, h(d["dhs"]),
                                                                                 W16[b.pre + ".down.w"].shape,
                                                                                 b.stride, 0))
-            chk(b.pre + ".down.dgrad", h(d["din2"]), orc.conv2d_dgrad(h(d["dhs"]), W16[b.pre + ".down.w"], x.shape,
-                                                                      b.stride, 0))
+            # the projection's data gradient is accumulated into conv1's in one pass
+            din_ref = din_ref + orc.conv2d_dgrad(h(d["dhs"]), W16[b.pre + ".down.w"], x.shape, b.stride, 0)
+            chk(b.pre + ".conv1+down.dgrad", h(d["din"]), din_ref)
+            dout, dout2 = h(d["din"]), None
         else:
+            chk(b.pre + ".conv1.dgrad", h(d["din"]), din_ref)
             chk(b.pre + ".dres", h(d["din2"]), dres)
-        dout, dout2 = h(d["din"]), h(d["din2"])
+            dout, dout2 = h(d["din"]), h(d["din2"])
     s_stats = [h(t) for t in wk.stem_stats]
     if variant == "imagenet":
-        da = orc.maxpool_bwd(dout + dout2, wk.pool_arg.cpu().numpy().astype(np.int32), stem_a.shape)
+        da = orc.maxpool_bwd(dout + (dout2 if dout2 is not None else 0), wk.pool_arg.cpu().numpy().astype(np.int32), stem_a.shape)
         chk("stem.pool.bwd", h(wk.stem_da), da)
         dys, dgs, dbs, _ = orc.bn_bwd(h(wk.stem_da), stem_a, h(wk.stem_y), P["bn1.g"], s_stats[2], s_stats[3])
     else:
