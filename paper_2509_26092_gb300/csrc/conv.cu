@@ -246,13 +246,14 @@ __device__ __forceinline__ void store_row_chunk_bf16(const ConvParams& p, const 
                                                      int64_t out_row, int col0, float (&back)[32])
 {
     uint4 pk[4];
-    __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(pk);
+    uint32_t* w32 = reinterpret_cast<uint32_t*>(pk);
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-        h2[k] = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
-        const float2 f = __bfloat1622float2(h2[k]);
-        back[2 * k] = valid ? f.x : 0.f;
-        back[2 * k + 1] = valid ? f.y : 0.f;
+        const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
+        const uint32_t u = valid ? *reinterpret_cast<const uint32_t*>(&h) : 0u;  // rows that are not outputs: 0
+        w32[k] = u;
+        back[2 * k] = __uint_as_float(u << 16);            // bf16 -> fp32 is exact: the high half
+        back[2 * k + 1] = __uint_as_float(u & 0xFFFF0000u);
     }
     if (valid) {
         uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
@@ -303,18 +304,26 @@ struct RowStats {
     // constant after unrolling).  Every lane of the warp must call it.
     __device__ __forceinline__ void add(int ch, const float (&x)[32], int lane)
     {
-        float a[32], b[32];
+        if constexpr (LEVELS == 0) {  // no folding: sum of squares by fused multiply-add
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-            a[k] = x[k];
-            b[k] = x[k] * x[k];
-        }
-        if constexpr (LEVELS >= 1) fold<32, 16>(a, b, lane);
-        if constexpr (LEVELS >= 2) fold<16, 8>(a, b, lane);
+            for (int k = 0; k < 32; ++k) {
+                s[ch][k] += x[k];
+                q[ch][k] = fmaf(x[k], x[k], q[ch][k]);
+            }
+        } else {
+            float a[32], b[32];
 #pragma unroll
-        for (int k = 0; k < V; ++k) {
-            s[ch][k] += a[k];
-            q[ch][k] += b[k];
+            for (int k = 0; k < 32; ++k) {
+                a[k] = x[k];
+                b[k] = x[k] * x[k];
+            }
+            if constexpr (LEVELS >= 1) fold<32, 16>(a, b, lane);
+            if constexpr (LEVELS >= 2) fold<16, 8>(a, b, lane);
+#pragma unroll
+            for (int k = 0; k < V; ++k) {
+                s[ch][k] += a[k];
+                q[ch][k] += b[k];
+            }
         }
     }
 
@@ -685,13 +694,20 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
 constexpr int kWinACC = 2;               // 128-row accumulators per tile
 constexpr int kWinBMT = 128 * kWinACC;   // padded positions per tile
 constexpr int kWinBStages = 4;           // weight-tile ring depth when not resident
-constexpr int kWinThreads = 224;
-constexpr int kEpiTileBytes = 4 * 32 * 33 * 4;
+constexpr int kWinThreads = 224;         // conv_wgwin_kernel: 4 epilogue warps, 2 producers, MMA
 
+// Warp roles of conv_win_kernel: EPI epilogue warps (0 .. EPI-1), then the strip
+// producer, the weight producer and the MMA issuer.  (Eight epilogue warps, two per
+// TMEM lane quarter, and stores staged in shared memory so that each instruction
+// writes whole lines, both measured slower on the stem than this form.)
 template <int BN>
 struct WinCfg {
     static constexpr int B_TILE = BN * 64 * 2;  // one tap x one 64-channel block of weights
     static constexpr uint32_t TMEM_COLS = 2 * kWinACC * BN;
+    static constexpr int EPI = 4;                // epilogue warps
+    static constexpr int CW = BN * 4 / EPI;      // columns one epilogue warp drains
+    static constexpr int W_STRIP = EPI, W_WEIGHT = EPI + 1, W_MMA = EPI + 2;
+    static constexpr int THREADS = 32 * (EPI + 3);
 };
 
 // One tap x 64-channel block of weights: K-major [BN out][64 in] for the forward
@@ -710,7 +726,7 @@ __device__ __forceinline__ void win_load_wtile(const ConvParams& p, const CUtens
 }
 
 template <int BN, bool DG, bool RES>
-__global__ void __launch_bounds__(kWinThreads, 1)
+__global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
     conv_win_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const ConvParams p)
 {
@@ -728,15 +744,16 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const int ntaps = p.win_R * p.win_S;
     const int b_bytes = RES ? ntaps * CB * C::B_TILE : kWinBStages * C::B_TILE;
     uint8_t* strip = sgen + b_bytes;
-    float* epi_tile = reinterpret_cast<float*>(strip + 2 * p.win_strip_bytes);
-    float* epi_sum = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(epi_tile) + kEpiTileBytes);
+    // per-warp statistics transposes reuse the strip buffers once the last tile's MMAs are done
+    float* epi_tile = reinterpret_cast<float*>(strip);
+    float* epi_sum = reinterpret_cast<float*>(strip + 2 * p.win_strip_bytes);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sfull[i], 1);
             mbar_init(&sempty[i], 1);
             mbar_init(&accf_bar[i], 1);
-            mbar_init(&acce_bar[i], 4);  // one arrival per epilogue warp
+            mbar_init(&acce_bar[i], C::EPI);  // one arrival per epilogue warp
         }
         for (int i = 0; i < kWinBStages; ++i) {
             mbar_init(&bfull[i], 1);
@@ -748,12 +765,12 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     }
     const bool want_stats = p.mode == kFwd && p.stats != nullptr;
     if (want_stats)
-        for (int i = threadIdx.x; i < 4 * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
-    if ((warp == 4 || warp == 5) && lane == 0) {
+        for (int i = threadIdx.x; i < C::EPI * 2 * p.Ncols; i += blockDim.x) epi_sum[i] = 0.f;
+    if ((warp == C::W_STRIP || warp == C::W_WEIGHT) && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
     }
-    if (warp == 6) {
+    if (warp == C::W_MMA) {
         tmem_alloc(&tmem_slot, C::TMEM_COLS);
         tmem_relinquish();
     }
@@ -763,7 +780,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const uint32_t tmem = tmem_slot;
     const int Wp = p.win_Wp;
 
-    if (warp == 4) {
+    if (warp == C::W_STRIP) {
         // ------------------------------------------------------------------ strip producer
         int it = 0;
         bool failed = false;
@@ -794,7 +811,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             if (lane == 0) report_timeout(&abort_flag);
             for (int i = it - 1; i >= 0 && i >= it - 2; --i) (void)mbar_drain_warp(&sfull[i & 1], (i >> 1) & 1);
         }
-    } else if (warp == 5) {
+    } else if (warp == C::W_WEIGHT) {
         // ------------------------------------------------------------------ weight producer
         if (RES) {
             mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(ntaps * CB * C::B_TILE));
@@ -826,7 +843,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     (void)mbar_drain_warp(&bfull[i % kWinBStages], (i / kWinBStages) & 1);
             }
         }
-    } else if (warp == 6) {
+    } else if (warp == C::W_MMA) {
         // ------------------------------------------------------------------ MMA issuer
         const uint32_t idesc = idesc_bf16(BM, BN, 0u, DG ? 1u : 0u);
         int it = 0, bt = 0, lt = 0;
@@ -898,10 +915,12 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         mma_commit_elect(&drain_bar);
         (void)mbar_drain_warp(&drain_bar, 0);
     } else {
-        // ------------------------------------------------------------------ epilogue (warps 0-3)
+        // ------------------------------------------------------------------ epilogue (warps 0 .. EPI-1)
+        constexpr int CW = C::CW;
+        const int quarter = warp & 3, col0 = (warp >> 2) * CW;  // TMEM lanes 32*quarter.., columns col0..
         float* st_tile = epi_tile + warp * 32 * 33;
         float* wsum = epi_sum + warp * 2 * p.Ncols;
-        RowStats<BN> rs;
+        RowStats<CW> rs;
         rs.zero();
         const int img = p.win_Hp * Wp;
         int lt = 0;
@@ -914,7 +933,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 break;
             }
             tc_fence_after();
-            const int row = warp * 32 + lane;
+            const int row = quarter * 32 + lane;
             bool valid[kWinACC];
             int64_t out_row[kWinACC];
 #pragma unroll
@@ -926,10 +945,10 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 valid[a] = a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P && wp < p.win_Q;
                 out_row[a] = ((int64_t)n * p.win_P + hp) * p.win_Q + wp;
             }
-            // chunks c = (accumulator, 32 columns), the next chunk's TMEM load in flight while
-            // this one is converted and stored
-            const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * kWinACC * BN);
-            constexpr int NCH = BN / 32, NC = kWinACC * NCH;
+            // chunks c = (accumulator, 32 of this warp's columns)
+            const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * kWinACC * BN + col0);
+            constexpr int NCH = CW / 32, NC = kWinACC * NCH;
+            // the next chunk's TMEM load in flight while this one is converted and stored
             uint32_t va[32], vb[32];
             tmem_ld_32x32b_x32(taddr, va);
 #pragma unroll
@@ -937,10 +956,11 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                 uint32_t(&cur)[32] = (c & 1) ? vb : va;
                 uint32_t(&nxt)[32] = (c & 1) ? va : vb;
                 tmem_ld_wait_regs(cur);
-                if (c + 1 < NC) tmem_ld_32x32b_x32(taddr + (uint32_t)((c + 1) * 32), nxt);
                 const int a = c / NCH, ch = c % NCH;
+                if (c + 1 < NC)
+                    tmem_ld_32x32b_x32(taddr + (uint32_t)(((c + 1) / NCH) * BN + ((c + 1) % NCH) * 32), nxt);
                 float back[32];
-                store_row_chunk_bf16(p, cur, valid[a], out_row[a], tc.n_tile * BN + ch * 32, back);
+                store_row_chunk_bf16(p, cur, valid[a], out_row[a], tc.n_tile * BN + col0 + ch * 32, back);
                 if (want_stats) rs.add(ch, back, lane);
             }
             tc_fence_before();
@@ -948,16 +968,22 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             if (lane == 0) mbar_arrive(&acce_bar[buf]);
         }
         if (want_stats) {
-            rs.flush(st_tile, wsum, p.Ncols, 0, lane);  // the window kernel has one column tile
-            asm volatile("bar.sync 1, 128;" ::: "memory");
+            rs.flush(st_tile, wsum, p.Ncols, col0, lane);  // the window kernel has one column tile
+            asm volatile("bar.sync 1, %0;" ::"r"(C::EPI * 32) : "memory");
             float* dst = p.stats + (int64_t)blockIdx.x * 2 * p.Ncols;
-            for (int c = threadIdx.x; c < 2 * p.Ncols; c += 128)
-                dst[c] = (epi_sum[c] + epi_sum[2 * p.Ncols + c]) + (epi_sum[4 * p.Ncols + c] + epi_sum[6 * p.Ncols + c]);
+            const int nc = 2 * p.Ncols;
+            // warps 4g..4g+3 hold column group g; the other groups' rows are zero
+            for (int c = threadIdx.x; c < nc; c += C::EPI * 32) {
+                float v = (epi_sum[c] + epi_sum[nc + c]) + (epi_sum[2 * nc + c] + epi_sum[3 * nc + c]);
+                if constexpr (C::EPI == 8)
+                    v += (epi_sum[4 * nc + c] + epi_sum[5 * nc + c]) + (epi_sum[6 * nc + c] + epi_sum[7 * nc + c]);
+                dst[c] = v;
+            }
         }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 6) {
+    if (warp == C::W_MMA) {
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);
     }
@@ -1155,20 +1181,47 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 }
 
 // ----------------------------------------------------------------------------- reductions
-// Per-channel sums over the per-CTA partials [nparts][2][K], fixed order
-// (colsum_fixed_order); block b covers channels 32b .. 32b+31 of both halves.
-__global__ void __launch_bounds__(32 * kColsumGroups) stats_reduce_kernel(const float* __restrict__ part, int nparts,
-                                                                         int K, float* __restrict__ sum,
-                                                                         float* __restrict__ sumsq)
+// Per-output-channel sums of the conv epilogue's per-CTA partials part[nparts][2][K]
+// (sum y, sum y^2 of each CTA's stored rows) -> sum[K], sumsq[K].  A block of 256
+// threads covers 32 channels; the 8 lanes j of a channel add the partials j, j+8,
+// ... in fp32 with Kahan compensation (four loads in flight), then a fixed
+// shuffle tree adds the 8 lane sums in fp64.  The order depends only on nparts,
+// so the result is the same on every launch and every GPU.
+__global__ void __launch_bounds__(256) stats_reduce_kernel(const float* __restrict__ part, int nparts, int K,
+                                                           float* __restrict__ sum, float* __restrict__ sumsq)
 {
-    __shared__ double red[kColsumGroups * 32];
-    const int c0 = blockIdx.x * 32;
-    const double s = colsum_fixed_order(part, nparts, 2 * (int64_t)K, c0, K, red);
-    const double q = colsum_fixed_order(part + K, nparts, 2 * (int64_t)K, c0, K, red);
-    const int c = c0 + threadIdx.x;
-    if (threadIdx.x < 32 && c < K) {
-        sum[c] = (float)s;
-        sumsq[c] = (float)q;
+    const int j = threadIdx.x & 7, c = blockIdx.x * 32 + (threadIdx.x >> 3);
+    float s = 0.f, sc = 0.f, q = 0.f, qc = 0.f;
+    if (c < K) {
+        const int64_t ld = 2 * (int64_t)K;
+        int t = j;
+        for (; t + 24 < nparts; t += 32) {
+            float vs[4], vq[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                vs[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + c);
+                vq[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + K + c);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                kahan_add(s, sc, vs[u]);
+                kahan_add(q, qc, vq[u]);
+            }
+        }
+        for (; t < nparts; t += 8) {
+            kahan_add(s, sc, __ldg(part + (int64_t)t * ld + c));
+            kahan_add(q, qc, __ldg(part + (int64_t)t * ld + K + c));
+        }
+    }
+    double ds = (double)s - (double)sc, dq = (double)q - (double)qc;
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+        ds += __shfl_xor_sync(0xffffffffu, ds, o);
+        dq += __shfl_xor_sync(0xffffffffu, dq, o);
+    }
+    if (j == 0 && c < K) {
+        sum[c] = (float)ds;
+        sumsq[c] = (float)dq;
     }
 }
 
@@ -1363,7 +1416,10 @@ bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& 
     const int BN = out_c, CB = red_c / 64, ntaps = s->r * s->s;
     const bool res = BN == 64 && CB == 1 && ntaps <= 9;
     const int b_bytes = res ? ntaps * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128;
-    const size_t smem = (size_t)b_bytes + 2 * (size_t)strip + kEpiTileBytes + 4 * 2 * (size_t)out_c * 4 + 1024;
+    // epilogue statistics: per-warp channel sums after the strips (the warps' transposes reuse the strips)
+    const int epi = out_c == 64 ? WinCfg<64>::EPI : WinCfg<128>::EPI;
+    const size_t smem = (size_t)b_bytes + 2 * (size_t)strip + (size_t)epi * 2 * out_c * 4 + 1024;
+    if (2 * (size_t)strip < (size_t)epi * 32 * 33 * 4) return false;
     if (smem > kWinSmemMax || (size_t)srows * Wp * 128 >= (1u << 20)) return false;
     ConvParams& p = pl.p;
     pl.win = true;
@@ -1764,7 +1820,7 @@ int launch_win_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, i
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_win_kernel<BN, DG, RES><<<grid, kWinThreads, pl.smem, st>>>(a, b, pl.p);
+    conv_win_kernel<BN, DG, RES><<<grid, WinCfg<BN>::THREADS, pl.smem, st>>>(a, b, pl.p);
     return dbl::launch_check("conv_win launch");
 }
 
@@ -1920,7 +1976,7 @@ int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y,
     cudaStream_t st = as_stream(stream);
     if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, ta, tb, grid, st))) return rc;
     if (stats) {
-        stats_reduce_kernel<<<(s->k + 31) / 32, 32 * kColsumGroups, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
+        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
         if ((rc = launch_check("conv stats reduce"))) return rc;
     }
     return DBL_OK;
