@@ -276,7 +276,13 @@ def conv_roofline(stage, reps=4, replays=2, table=None):
             st_sum = torch.empty(shp.k, device=x.device)
             st_sq = torch.empty(shp.k, device=x.device)
             f1 = float(wk.layer_flops(name, shp))
-            passes = [("fwd", f1, lambda s: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            if name == stem:
+                passes = [("fwd", f1, lambda s: D.dbl_conv_fwd(shp, x, w16, y, st_sum, st_sq, wk.ws, wk.ws.numel(), s))]
+            else:
+                # as in the training step: the BatchNorm statistics are left as per-CTA partials,
+                # which the BatchNorm finalize reduces
+                parts = wk.ws
+                passes = [("fwd", f1, lambda s: D.dbl_conv_fwd_parts(shp, x, w16, y, parts, parts.numel(), s))]
             algo_bytes += nbytes(x, w16, y)
             proj = name.replace(".conv1", ".down") if name.endswith(".conv1") else None
             if proj in bufs:

@@ -104,6 +104,18 @@ DBL_API size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass);
 DBL_API int dbl_conv_fwd(const dbl_conv_shape* shape, const void* x_bf16, const void* w_bf16, void* y_bf16,
                  float* ch_sum, float* ch_sumsq, void* ws, size_t ws_bytes, void* stream);
 
+/* Forward pass that leaves the BatchNorm statistics as partial sums for
+ * dbl_bn_relu_fused_parts to reduce (one kernel launch fewer per layer than
+ * dbl_conv_fwd + dbl_bn_relu_fused).  Writes y as dbl_conv_fwd does, and into
+ * parts ([*nparts][2][k] fp32, caller-owned, at least
+ * dbl_conv_stats_parts_bytes(shape) bytes) the sums of the stored y and of its
+ * squares over the rows each of *nparts thread blocks stored.  *nparts (host
+ * memory) is set at call time; the same shape on the same device always gives
+ * the same value. */
+DBL_API size_t dbl_conv_stats_parts_bytes(const dbl_conv_shape* shape);
+DBL_API int dbl_conv_fwd_parts(const dbl_conv_shape* shape, const void* x_bf16, const void* w_bf16, void* y_bf16,
+                               float* parts, size_t parts_bytes, int32_t* nparts, void* stream);
+
 /* Data gradient: dx = d(sum y*dy)/dx, the adjoint of the forward pass in its
  * input.  dy: [n,P,Q,k] bf16; dx: [n,h,w,c] bf16 (fully overwritten).
  * Supported for stride 1, and for stride 2 with even h and w. */
@@ -155,6 +167,14 @@ DBL_API int dbl_bn_stats(const dbl_bn_shape* shape, const void* y_bf16, float* c
 DBL_API int dbl_bn_relu_fused(const dbl_bn_shape* shape, const void* y_bf16, const float* ch_sum, const float* ch_sumsq,
                       const float* gamma, const float* beta, const void* residual_bf16 /* or NULL */,
                       void* out_bf16, float* save_mean, float* save_invstd, void* stream);
+
+/* dbl_bn_relu_fused with the batch statistics given as the partial sums of
+ * dbl_conv_fwd_parts (parts [nparts][2][c]); they are reduced in the same fixed
+ * order as dbl_conv_fwd reduces them, so the result is bit-identical to
+ * dbl_conv_fwd + dbl_bn_relu_fused. */
+DBL_API int dbl_bn_relu_fused_parts(const dbl_bn_shape* shape, const void* y_bf16, const float* parts, int32_t nparts,
+                                    const float* gamma, const float* beta, const void* residual_bf16 /* or NULL */,
+                                    void* out_bf16, float* save_mean, float* save_invstd, void* stream);
 
 /* Bytes of scratch dbl_bn_relu_fused_bwd needs.  Host. */
 DBL_API size_t dbl_bn_workspace_bytes(const dbl_bn_shape* shape);

@@ -103,6 +103,26 @@ __global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const fl
 }
 
 
+// The same finalize from a convolution's per-CTA partials part[nparts][2][C]: the
+// fixed-order partial sums (partials_colsum, rounded to fp32 as dbl_conv_fwd stores
+// them), then mean and 1/std exactly as above.  256 threads per 32 channels.
+__global__ void __launch_bounds__(256) bn_fwd_finalize_parts_kernel(int64_t count, int C, float eps,
+                                                                    const float* __restrict__ part, int nparts,
+                                                                    float* __restrict__ save_mean,
+                                                                    float* __restrict__ save_invstd)
+{
+    double ds, dq;
+    const int c = dbl::dev::partials_colsum(part, nparts, C, ds, dq);
+    if (c < 0) return;
+    const float sum = (float)ds, sumsq = (float)dq;
+    const double inv_n = 1.0 / (double)count;
+    const double mean = (double)sum * inv_n;
+    double var = (double)sumsq * inv_n - mean * mean;
+    if (var < 0.0) var = 0.0;
+    save_mean[c] = (float)mean;
+    save_invstd[c] = (float)(1.0 / sqrt(var + (double)eps));
+}
+
 // Thread t of a CTA owns channel group g = t % (C/8) (8 channels, one 16-byte
 // vector) and visits rows t / (C/8), + rows-per-CTA-step, ...; a warp covers
 // consecutive vectors of consecutive rows, so every access is coalesced, and the
@@ -299,20 +319,17 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     }
 }
 
-// Fixed-order sum of the partials [nblk][2][C] (colsum_fixed_order; block b
-// covers channels 32b .. 32b+31), then dgamma, dbeta and the three per-channel
-// coefficients (A, B, C) of the apply pass dy = A*g + B*y + C.
-__global__ void __launch_bounds__(32 * kColsumGroups) bn_bwd_finalize_kernel(
+// Fixed-order sum of the partials [nblk][2][C] (partials_colsum: 256 threads per 32
+// channels), then dgamma, dbeta and the three per-channel coefficients (A, B, C) of
+// the apply pass dy = A*g + B*y + C.
+__global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(
     const float* __restrict__ partial, int nblk, int C, int64_t count, const float* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ invstd, float* __restrict__ dgamma,
     float* __restrict__ dbeta, float* __restrict__ coef)
 {
-    __shared__ double red[kColsumGroups * 32];
-    const int c0 = blockIdx.x * 32;
-    const double sg = colsum_fixed_order(partial, nblk, 2 * (int64_t)C, c0, C, red);
-    const double sgx = colsum_fixed_order(partial + C, nblk, 2 * (int64_t)C, c0, C, red);
-    const int c = c0 + threadIdx.x;
-    if (threadIdx.x >= 32 || c >= C) return;
+    double sg, sgx;
+    const int c = dbl::dev::partials_colsum(partial, nblk, C, sg, sgx);
+    if (c < 0) return;
     dbeta[c] = (float)sg;
     dgamma[c] = (float)sgx;
     // dy = k1*(g - sum(g)/n - xhat*sum(g*xhat)/n), xhat = (y - mean)*invstd, as A*g + B*y + C
@@ -429,7 +446,7 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
             nullptr);
     int rc = launch_check("bn_bwd_reduce launch");
     if (rc) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 32 * kColsumGroups, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
+    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
                                                                          invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     if (g_store)
@@ -507,6 +524,29 @@ int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum,
         static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
         static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
     return launch_check("bn_relu_fused launch");
+}
+
+int dbl_bn_relu_fused_parts(const dbl_bn_shape* s, const void* y, const float* parts, int32_t nparts,
+                            const float* gamma, const float* beta, const void* residual, void* out, float* save_mean,
+                            float* save_invstd, void* stream)
+{
+    using namespace dbl;
+    int rc = check_shape(s, "bn_relu_fused_parts");
+    if (rc) return rc;
+    if (!y || !out || !parts || !gamma || !beta || !save_mean || !save_invstd)
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: null pointer");
+    if (nparts <= 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: no partials");
+    if (!aligned16(y) || !aligned16(out) || (residual && !aligned16(residual)))
+        return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: tensors must be 16-byte aligned");
+    if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: empty batch has no statistics");
+    cudaStream_t st = as_stream(stream);
+    bn_fwd_finalize_parts_kernel<<<(s->c + 31) / 32, 256, 0, st>>>(s->count, s->c, s->eps, parts, nparts, save_mean,
+                                                                   save_invstd);
+    if ((rc = launch_check("bn_fwd_finalize_parts launch"))) return rc;
+    bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
+        static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
+    return launch_check("bn_relu_fused_parts launch");
 }
 
 size_t dbl_bn_workspace_bytes(const dbl_bn_shape* s)

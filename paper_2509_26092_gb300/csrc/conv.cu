@@ -1182,46 +1182,15 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 
 // ----------------------------------------------------------------------------- reductions
 // Per-output-channel sums of the conv epilogue's per-CTA partials part[nparts][2][K]
-// (sum y, sum y^2 of each CTA's stored rows) -> sum[K], sumsq[K].  A block of 256
-// threads covers 32 channels; the 8 lanes j of a channel add the partials j, j+8,
-// ... in fp32 with Kahan compensation (four loads in flight), then a fixed
-// shuffle tree adds the 8 lane sums in fp64.  The order depends only on nparts,
-// so the result is the same on every launch and every GPU.
+// (partials_colsum: 256-thread blocks of 32 channels, fixed order).
 __global__ void __launch_bounds__(256) stats_reduce_kernel(const float* __restrict__ part, int nparts, int K,
                                                            float* __restrict__ sum, float* __restrict__ sumsq)
 {
-    const int j = threadIdx.x & 7, c = blockIdx.x * 32 + (threadIdx.x >> 3);
-    float s = 0.f, sc = 0.f, q = 0.f, qc = 0.f;
-    if (c < K) {
-        const int64_t ld = 2 * (int64_t)K;
-        int t = j;
-        for (; t + 24 < nparts; t += 32) {
-            float vs[4], vq[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                vs[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + c);
-                vq[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + K + c);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                kahan_add(s, sc, vs[u]);
-                kahan_add(q, qc, vq[u]);
-            }
-        }
-        for (; t < nparts; t += 8) {
-            kahan_add(s, sc, __ldg(part + (int64_t)t * ld + c));
-            kahan_add(q, qc, __ldg(part + (int64_t)t * ld + K + c));
-        }
-    }
-    double ds = (double)s - (double)sc, dq = (double)q - (double)qc;
-#pragma unroll
-    for (int o = 1; o < 8; o <<= 1) {
-        ds += __shfl_xor_sync(0xffffffffu, ds, o);
-        dq += __shfl_xor_sync(0xffffffffu, dq, o);
-    }
-    if (j == 0 && c < K) {
-        sum[c] = (float)ds;
-        sumsq[c] = (float)dq;
+    double s, q;
+    const int c = partials_colsum(part, nparts, K, s, q);
+    if (c >= 0) {
+        sum[c] = (float)s;
+        sumsq[c] = (float)q;
     }
 }
 
@@ -1863,6 +1832,66 @@ int enc_win_rows(CUtensorMap* m, const void* base, int N, int H, int W, int C, i
 // Rows of one tile of the forward family (see Cfg).
 int fwd_tile_rows(int BN) { return BN <= 128 ? 256 : 128; }
 
+// Forward pass.  nparts == nullptr: the channel sums are reduced into ch_sum/ch_sumsq
+// (NULL: no statistics).  nparts != nullptr: the per-CTA partials are left in ws
+// ([*nparts][2][k]) for the BatchNorm finalize to reduce (dbl_bn_relu_fused_parts).
+int conv_fwd_impl(const dbl_conv_shape* s, const void* x, const void* w, void* y, float* ch_sum, float* ch_sumsq,
+                  void* ws, size_t ws_bytes, int32_t* nparts, void* stream, const char* who)
+{
+    using namespace dbl;
+    Plan pl;
+    int rc = make_plan(s, DBL_PASS_FWD, pl);
+    if (rc) return rc;
+    if (!x || !w || !y || !aligned16(x) || !aligned16(w) || !aligned16(y))
+        return set_error(DBL_ERR_INVALID, "%s: null or misaligned tensor", who);
+    if ((ch_sum == nullptr) != (ch_sumsq == nullptr))
+        return set_error(DBL_ERR_INVALID, "%s: ch_sum and ch_sumsq go together", who);
+    const bool stats = ch_sum != nullptr || nparts != nullptr;
+    if (stats && (!ws || ws_bytes < plan_ws(pl)))
+        return set_error(DBL_ERR_WORKSPACE, "%s: workspace %zu < %zu bytes", who, ws_bytes, plan_ws(pl));
+    CUtensorMap ta, tb;
+    const Geom g = geom(s);
+    if (pl.win) {
+        if ((rc = enc_win_rows(&ta, x, s->n, s->h, s->w, s->c, pl.p.win_Wp))) return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * s->c;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
+    } else if (pl.mode == kFwdC8) {
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
+                             g.sw, 8, fwd_tile_rows(pl.BN), false)))
+            return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * 8;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {8, (cuuint32_t)pl.BN};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, false))) return rc;
+    } else {
+        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
+                             g.sw, 64, fwd_tile_rows(pl.BN), true)))
+            return rc;
+        const int64_t rsc = (int64_t)s->r * s->s * s->c;
+        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
+        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)(pl.BN / pl.cg)};
+        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
+    }
+    pl.p.out = y;
+    pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
+    const int grid = plan_grid(pl);
+    cudaStream_t st = as_stream(stream);
+    if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, ta, tb, grid, st))) return rc;
+    if (nparts) {
+        *nparts = grid;
+    } else if (stats) {
+        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
+        if ((rc = launch_check("conv stats reduce"))) return rc;
+    }
+    return DBL_OK;
+}
+
+
 // Data gradient, optionally with the projection shortcut of a ResNet block fused in:
 // k2 > 0 adds dgrad of a 1x1 stride-2 pad-0 convolution of the same input (dy2:
 // [n, h/2, w/2, k2], w2: [k2][c]) to phase (0,0), the only phase it reaches.
@@ -1931,55 +1960,22 @@ size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass)
 int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y, float* ch_sum, float* ch_sumsq,
                  void* ws, size_t ws_bytes, void* stream)
 {
-    using namespace dbl;
+    return conv_fwd_impl(s, x, w, y, ch_sum, ch_sumsq, ws, ws_bytes, nullptr, stream, "conv_fwd");
+}
+
+size_t dbl_conv_stats_parts_bytes(const dbl_conv_shape* shape)
+{
     Plan pl;
-    int rc = make_plan(s, DBL_PASS_FWD, pl);
-    if (rc) return rc;
-    if (!x || !w || !y || !aligned16(x) || !aligned16(w) || !aligned16(y))
-        return set_error(DBL_ERR_INVALID, "conv_fwd: null or misaligned tensor");
-    if ((ch_sum == nullptr) != (ch_sumsq == nullptr))
-        return set_error(DBL_ERR_INVALID, "conv_fwd: ch_sum and ch_sumsq go together");
-    const bool stats = ch_sum != nullptr;
-    if (stats && (!ws || ws_bytes < plan_ws(pl)))
-        return set_error(DBL_ERR_WORKSPACE, "conv_fwd: workspace %zu < %zu bytes", ws_bytes, plan_ws(pl));
-    CUtensorMap ta, tb;
-    const Geom g = geom(s);
-    if (pl.win) {
-        if ((rc = enc_win_rows(&ta, x, s->n, s->h, s->w, s->c, pl.p.win_Wp))) return rc;
-        const int64_t rsc = (int64_t)s->r * s->s * s->c;
-        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
-        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
-        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
-    } else if (pl.mode == kFwdC8) {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
-                             g.sw, 8, fwd_tile_rows(pl.BN), false)))
-            return rc;
-        const int64_t rsc = (int64_t)s->r * s->s * 8;
-        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
-        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
-        cuuint32_t box[2] = {8, (cuuint32_t)pl.BN};
-        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, false))) return rc;
-    } else {
-        if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, s->c, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,
-                             g.sw, 64, fwd_tile_rows(pl.BN), true)))
-            return rc;
-        const int64_t rsc = (int64_t)s->r * s->s * s->c;
-        cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
-        cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)(pl.BN / pl.cg)};
-        if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
-    }
-    pl.p.out = y;
-    pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
-    const int grid = plan_grid(pl);
-    cudaStream_t st = as_stream(stream);
-    if ((rc = pl.win ? launch_win(pl, ta, tb, grid, st) : launch(pl, ta, tb, ta, tb, grid, st))) return rc;
-    if (stats) {
-        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
-        if ((rc = launch_check("conv stats reduce"))) return rc;
-    }
-    return DBL_OK;
+    if (make_plan(shape, DBL_PASS_FWD, pl) != DBL_OK) return 0;
+    return (size_t)kMaxGrid * 2 * shape->k * sizeof(float);
+}
+
+int dbl_conv_fwd_parts(const dbl_conv_shape* s, const void* x, const void* w, void* y, float* parts,
+                       size_t parts_bytes, int32_t* nparts, void* stream)
+{
+    using dbl::set_error;
+    if (!parts || !nparts) return set_error(DBL_ERR_INVALID, "conv_fwd_parts: null partials or count");
+    return conv_fwd_impl(s, x, w, y, nullptr, nullptr, parts, parts_bytes, nparts, stream, "conv_fwd_parts");
 }
 
 int dbl_conv_dgrad(const dbl_conv_shape* s, const void* dy, const void* w, void* dx, void* ws, size_t ws_bytes,

@@ -294,6 +294,52 @@ __device__ __forceinline__ double colsum_fixed_order(const float* __restrict__ p
     return total;
 }
 
+// ---------------------------------------------------------------------------- per-block partial sums
+// Fixed-order column sums of per-block partials part[nparts][2][K] (row p: the two
+// sums block p produced for every channel: a convolution epilogue's sum y and sum
+// y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called by all 256
+// threads of a block covering channels 32*blockIdx.x ..: the 8 lanes j of a channel
+// add the partials j, j+8, ... in fp32 with Kahan compensation (four loads in
+// flight), then a fixed shuffle tree adds the 8 lane sums in fp64.  The order
+// depends only on nparts, so the result is the same on every launch and GPU.
+// Returns the channel (or -1 for lanes j != 0 and channels past K) and its sums.
+__device__ __forceinline__ int partials_colsum(const float* __restrict__ part, int nparts, int K, double& sum0,
+                                               double& sum1)
+{
+    const int j = threadIdx.x & 7, c = blockIdx.x * 32 + (threadIdx.x >> 3);
+    float s = 0.f, sc = 0.f, q = 0.f, qc = 0.f;
+    if (c < K) {
+        const int64_t ld = 2 * (int64_t)K;
+        int t = j;
+        for (; t + 24 < nparts; t += 32) {
+            float vs[4], vq[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                vs[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + c);
+                vq[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + K + c);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                kahan_add(s, sc, vs[u]);
+                kahan_add(q, qc, vq[u]);
+            }
+        }
+        for (; t < nparts; t += 8) {
+            kahan_add(s, sc, __ldg(part + (int64_t)t * ld + c));
+            kahan_add(q, qc, __ldg(part + (int64_t)t * ld + K + c));
+        }
+    }
+    double ds = (double)s - (double)sc, dq = (double)q - (double)qc;
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+        ds += __shfl_xor_sync(0xffffffffu, ds, o);
+        dq += __shfl_xor_sync(0xffffffffu, dq, o);
+    }
+    sum0 = ds;
+    sum1 = dq;
+    return (j == 0 && c < K) ? c : -1;
+}
+
 // ---------------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* tmap)
 {

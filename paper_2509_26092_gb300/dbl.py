@@ -66,6 +66,10 @@ def lib():
             "dbl_conv_dgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _SZ, _V]),
             "dbl_conv_wgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, ctypes.c_int, _V, _SZ, _V]),
             "dbl_conv_dgrad_proj": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _I32, _V, _V, _V, _V, _SZ, _V]),
+            "dbl_conv_stats_parts_bytes": (_SZ, [ctypes.POINTER(ConvShape)]),
+            "dbl_conv_fwd_parts": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _SZ,
+                                                  ctypes.POINTER(_I32), _V]),
+            "dbl_bn_relu_fused_parts": (ctypes.c_int, [ctypes.POINTER(BnShape), _V, _V, _I32] + [_V] * 7),
             "dbl_bn_stats": (ctypes.c_int, [ctypes.POINTER(BnShape), _V, _V, _V, _V]),
             "dbl_bn_relu_fused": (ctypes.c_int, [ctypes.POINTER(BnShape)] + [_V] * 10),
             "dbl_bn_workspace_bytes": (_SZ, [ctypes.POINTER(BnShape)]),
@@ -151,6 +155,25 @@ def dbl_conv_workspace_bytes(shape, pass_):
 def dbl_conv_fwd(shape, x, w, y, ch_sum=None, ch_sumsq=None, ws=None, ws_bytes=0, stream=None):
     _check(lib().dbl_conv_fwd(ctypes.byref(shape), _ptr(x), _ptr(w), _ptr(y), _ptr(ch_sum), _ptr(ch_sumsq), _ptr(ws),
                               ws_bytes, _stream(stream)))
+
+
+def dbl_conv_stats_parts_bytes(shape):
+    return lib().dbl_conv_stats_parts_bytes(ctypes.byref(shape))
+
+
+def dbl_conv_fwd_parts(shape, x, w, y, parts, parts_bytes, stream=None):
+    """Returns the number of partial rows written to parts (see dbl_bn_relu_fused_parts)."""
+    n = _I32(0)
+    _check(lib().dbl_conv_fwd_parts(ctypes.byref(shape), _ptr(x), _ptr(w), _ptr(y), _ptr(parts), parts_bytes,
+                                    ctypes.byref(n), _stream(stream)))
+    return n.value
+
+
+def dbl_bn_relu_fused_parts(shape, y, parts, nparts, gamma, beta, residual, out, save_mean, save_invstd,
+                            stream=None):
+    _check(lib().dbl_bn_relu_fused_parts(ctypes.byref(shape), _ptr(y), _ptr(parts), int(nparts), _ptr(gamma),
+                                         _ptr(beta), _ptr(residual), _ptr(out), _ptr(save_mean), _ptr(save_invstd),
+                                         _stream(stream)))
 
 
 def dbl_conv_dgrad(shape, dy, w, dx, ws=None, ws_bytes=0, stream=None):

@@ -267,6 +267,9 @@ class Worker:
                 d["gout"] = act(ho, b.cout)  # the masked output gradient, input of the shortcut BatchNorm
             for k in ("bn1", "bn2", "downbn"):
                 d[k] = [vec(b.cout) for _ in range(4)]
+                # the BatchNorm's per-CTA partial statistics from its convolution (dbl_conv_fwd_parts)
+                d[k + ".parts"] = torch.empty(D.dbl_conv_stats_parts_bytes(D.conv_shape(1, 8, 8, 64, b.cout, 1, 1, 0))
+                                              // 4, dtype=torch.float32, device=dev)
             self.blocks.append(d)
             h = ho
         self.final_hw = h
@@ -382,25 +385,28 @@ class Worker:
             b = d["spec"]
             d["x"] = cur
             cnt = B * d["hout"] ** 2
+            # each convolution leaves its BatchNorm statistics as per-CTA partials, which the
+            # BatchNorm's finalize reduces (one launch per layer fewer than reducing them apart)
             s1 = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 3, b.stride, 1)
-            st1 = d["bn1"]
-            D.dbl_conv_fwd(s1, cur, wv(b.pre + ".conv1.w"), d["h1"], st1[0], st1[1], ws, wsb, s)
-            D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, True), d["h1"], st1[0], st1[1], pv(b.pre + ".bn1.g"),
-                                pv(b.pre + ".bn1.b"), None, d["o1"], st1[2], st1[3], s)
+            st1, p1 = d["bn1"], d["bn1.parts"]
+            n1 = D.dbl_conv_fwd_parts(s1, cur, wv(b.pre + ".conv1.w"), d["h1"], p1, p1.numel() * 4, s)
+            D.dbl_bn_relu_fused_parts(D.bn_shape(cnt, b.cout, eps, True), d["h1"], p1, n1, pv(b.pre + ".bn1.g"),
+                                      pv(b.pre + ".bn1.b"), None, d["o1"], st1[2], st1[3], s)
             s2 = D.conv_shape(B, d["hout"], d["hout"], b.cout, b.cout, 3, 1, 1)
-            st2 = d["bn2"]
-            D.dbl_conv_fwd(s2, d["o1"], wv(b.pre + ".conv2.w"), d["h2"], st2[0], st2[1], ws, wsb, s)
+            st2, p2 = d["bn2"], d["bn2.parts"]
+            n2 = D.dbl_conv_fwd_parts(s2, d["o1"], wv(b.pre + ".conv2.w"), d["h2"], p2, p2.numel() * 4, s)
             if b.proj:
                 sd = D.conv_shape(B, d["hin"], d["hin"], b.cin, b.cout, 1, b.stride, 0)
-                std = d["downbn"]
-                D.dbl_conv_fwd(sd, cur, wv(b.pre + ".down.w"), d["hs"], std[0], std[1], ws, wsb, s)
-                D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, False), d["hs"], std[0], std[1],
-                                    pv(b.pre + ".downbn.g"), pv(b.pre + ".downbn.b"), None, d["sc"], std[2], std[3], s)
+                std, pd = d["downbn"], d["downbn.parts"]
+                nd = D.dbl_conv_fwd_parts(sd, cur, wv(b.pre + ".down.w"), d["hs"], pd, pd.numel() * 4, s)
+                D.dbl_bn_relu_fused_parts(D.bn_shape(cnt, b.cout, eps, False), d["hs"], pd, nd,
+                                          pv(b.pre + ".downbn.g"), pv(b.pre + ".downbn.b"), None, d["sc"], std[2],
+                                          std[3], s)
                 res = d["sc"]
             else:
                 res = cur
-            D.dbl_bn_relu_fused(D.bn_shape(cnt, b.cout, eps, True), d["h2"], st2[0], st2[1], pv(b.pre + ".bn2.g"),
-                                pv(b.pre + ".bn2.b"), res, d["out"], st2[2], st2[3], s)
+            D.dbl_bn_relu_fused_parts(D.bn_shape(cnt, b.cout, eps, True), d["h2"], p2, n2, pv(b.pre + ".bn2.g"),
+                                      pv(b.pre + ".bn2.b"), res, d["out"], st2[2], st2[3], s)
             cur = d["out"]
         # ---- head: pooling, FC, softmax cross-entropy and their backward
         C = spec.widths[-1]

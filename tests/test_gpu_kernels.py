@@ -365,6 +365,47 @@ def test_conv_fwd_matches_oracle(D, case):
     check_status(D)
 
 
+@pytest.mark.parametrize("case", [(2, 8, 8, 64, 64, 3, 1, 1), (4, 14, 14, 256, 512, 3, 2, 1), (32, 14, 14, 256, 256, 3, 1, 1),
+                                  (8, 16, 16, 64, 128, 3, 1, 1), (2, 8, 8, 64, 128, 1, 2, 0)])
+def test_conv_fwd_parts_then_bn_matches_two_step_path(D, case):
+    """Statistics left as per-CTA partials and reduced in the BatchNorm finalize give
+    the same bits as dbl_conv_fwd's own reduction followed by dbl_bn_relu_fused."""
+    n, h, w, c, k, r, st, pad = case
+    x, wt = _conv_inputs(case, 21)
+    shape = D.conv_shape(n, h, w, c, k, r, st, pad)
+    P, Q = orc.out_dim(h, r, st, pad), orc.out_dim(w, r, st, pad)
+    xd, wd = to_bf16_dev(x), to_bf16_dev(wt)
+    y1 = torch.empty((n, P, Q, k), dtype=torch.bfloat16, device="cuda")
+    y2 = torch.empty_like(y1)
+    s1, s2 = torch.empty(k, device="cuda"), torch.empty(k, device="cuda")
+    wsb = D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_FWD)
+    D.dbl_conv_fwd(shape, xd, wd, y1, s1, s2, ws(wsb), wsb)
+    pb = D.dbl_conv_stats_parts_bytes(shape)
+    parts = torch.empty(pb // 4, device="cuda")
+    nparts = D.dbl_conv_fwd_parts(shape, xd, wd, y2, parts, pb)
+    assert nparts >= 1 and torch.equal(y1, y2)
+    g = rng(22)
+    gamma = to_f32_dev(g.uniform(0.5, 1.5, k).astype(np.float32))
+    beta = to_f32_dev((0.1 * g.standard_normal(k)).astype(np.float32))
+    res = to_bf16_dev(bf16_values(g.standard_normal((n, P, Q, k))))
+    bs = D.bn_shape(n * P * Q, k, 1e-5, True)
+    outs = []
+    for use_parts in (False, True):
+        out = torch.empty_like(y1)
+        mean, istd = torch.empty(k, device="cuda"), torch.empty(k, device="cuda")
+        if use_parts:
+            D.dbl_bn_relu_fused_parts(bs, y2, parts, nparts, gamma, beta, res, out, mean, istd)
+        else:
+            D.dbl_bn_relu_fused(bs, y1, s1, s2, gamma, beta, res, out, mean, istd)
+        outs.append((out, mean, istd))
+    for a, b in zip(outs[0], outs[1]):
+        assert torch.equal(a, b)
+    # and both are the oracle's BatchNorm of the stored y
+    ref, _, _ = orc.bn_fwd(host(y1), host(gamma), host(beta), 1e-5, res=host(res))
+    assert max_norm_rel(host(outs[1][0]), ref) <= CONV_TOL
+    check_status(D)
+
+
 DGRAD_CASES = [
     (2, 8, 8, 64, 64, 3, 1, 1),
     (3, 6, 10, 64, 64, 3, 1, 1),     # ragged
