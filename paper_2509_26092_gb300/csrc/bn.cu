@@ -105,8 +105,8 @@ __global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const fl
 
 // The same finalize from a convolution's per-CTA partials part[nparts][2][C]: the
 // fixed-order partial sums (partials_colsum, rounded to fp32 as dbl_conv_fwd stores
-// them), then mean and 1/std exactly as above.  256 threads per 32 channels.
-__global__ void __launch_bounds__(256) bn_fwd_finalize_parts_kernel(int64_t count, int C, float eps,
+// them), then mean and 1/std exactly as above.  One warp per channel.
+__global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_parts_kernel(int64_t count, int C, float eps,
                                                                     const float* __restrict__ part, int nparts,
                                                                     float* __restrict__ save_mean,
                                                                     float* __restrict__ save_invstd)
@@ -319,10 +319,10 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     }
 }
 
-// Fixed-order sum of the partials [nblk][2][C] (partials_colsum: 256 threads per 32
-// channels), then dgamma, dbeta and the three per-channel coefficients (A, B, C) of
+// Fixed-order sum of the partials [nblk][2][C] (partials_colsum: one warp per
+// channel), then dgamma, dbeta and the three per-channel coefficients (A, B, C) of
 // the apply pass dy = A*g + B*y + C.
-__global__ void __launch_bounds__(256) bn_bwd_finalize_kernel(
+__global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_bwd_finalize_kernel(
     const float* __restrict__ partial, int nblk, int C, int64_t count, const float* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ invstd, float* __restrict__ dgamma,
     float* __restrict__ dbeta, float* __restrict__ coef)
@@ -446,7 +446,8 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
             nullptr);
     int rc = launch_check("bn_bwd_reduce launch");
     if (rc) return rc;
-    bn_bwd_finalize_kernel<<<(C + 31) / 32, 256, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
+    bn_bwd_finalize_kernel<<<(C + dbl::dev::kPartialsChannels - 1) / dbl::dev::kPartialsChannels,
+                             dbl::dev::kPartialsThreads, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
                                                                          invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     if (g_store)
@@ -540,7 +541,8 @@ int dbl_bn_relu_fused_parts(const dbl_bn_shape* s, const void* y, const float* p
         return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: tensors must be 16-byte aligned");
     if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: empty batch has no statistics");
     cudaStream_t st = as_stream(stream);
-    bn_fwd_finalize_parts_kernel<<<(s->c + 31) / 32, 256, 0, st>>>(s->count, s->c, s->eps, parts, nparts, save_mean,
+    bn_fwd_finalize_parts_kernel<<<(s->c + dbl::dev::kPartialsChannels - 1) / dbl::dev::kPartialsChannels,
+                                   dbl::dev::kPartialsThreads, 0, st>>>(s->count, s->c, s->eps, parts, nparts, save_mean,
                                                                    save_invstd);
     if ((rc = launch_check("bn_fwd_finalize_parts launch"))) return rc;
     bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(

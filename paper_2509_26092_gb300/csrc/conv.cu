@@ -1182,8 +1182,8 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 
 // ----------------------------------------------------------------------------- reductions
 // Per-output-channel sums of the conv epilogue's per-CTA partials part[nparts][2][K]
-// (partials_colsum: 256-thread blocks of 32 channels, fixed order).
-__global__ void __launch_bounds__(256) stats_reduce_kernel(const float* __restrict__ part, int nparts, int K,
+// (partials_colsum: one warp per channel, fixed order).
+__global__ void __launch_bounds__(kPartialsThreads) stats_reduce_kernel(const float* __restrict__ part, int nparts, int K,
                                                            float* __restrict__ sum, float* __restrict__ sumsq)
 {
     double s, q;
@@ -1885,7 +1885,7 @@ int conv_fwd_impl(const dbl_conv_shape* s, const void* x, const void* w, void* y
     if (nparts) {
         *nparts = grid;
     } else if (stats) {
-        stats_reduce_kernel<<<(s->k + 31) / 32, 256, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
+        stats_reduce_kernel<<<(s->k + kPartialsChannels - 1) / kPartialsChannels, kPartialsThreads, 0, st>>>(pl.p.stats, grid, s->k, ch_sum, ch_sumsq);
         if ((rc = launch_check("conv stats reduce"))) return rc;
     }
     return DBL_OK;

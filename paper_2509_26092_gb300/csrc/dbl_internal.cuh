@@ -297,26 +297,30 @@ __device__ __forceinline__ double colsum_fixed_order(const float* __restrict__ p
 // ---------------------------------------------------------------------------- per-block partial sums
 // Fixed-order column sums of per-block partials part[nparts][2][K] (row p: the two
 // sums block p produced for every channel: a convolution epilogue's sum y and sum
-// y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called by all 256
-// threads of a block covering channels 32*blockIdx.x ..: the 8 lanes j of a channel
-// add the partials j, j+8, ... in fp32 with Kahan compensation (four loads in
-// flight), then a fixed shuffle tree adds the 8 lane sums in fp64.  The order
-// depends only on nparts, so the result is the same on every launch and GPU.
-// Returns the channel (or -1 for lanes j != 0 and channels past K) and its sums.
+// y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called by all threads of
+// a block of kPartialsThreads covering channels kPartialsChannels*blockIdx.x ..:
+// the 32 lanes j of a warp (one channel) add the partials j, j+32, ... in fp32 with
+// Kahan compensation (four loads in flight), then a fixed shuffle tree adds the 32
+// lane sums in fp64.  The order depends only on nparts, so the result is the same
+// on every launch and GPU.  Returns the channel (or -1 for lanes j != 0 and
+// channels past K) and its two sums.
+constexpr int kPartialsThreads = 256;
+constexpr int kPartialsChannels = kPartialsThreads / 32;
+
 __device__ __forceinline__ int partials_colsum(const float* __restrict__ part, int nparts, int K, double& sum0,
                                                double& sum1)
 {
-    const int j = threadIdx.x & 7, c = blockIdx.x * 32 + (threadIdx.x >> 3);
+    const int j = threadIdx.x & 31, c = blockIdx.x * kPartialsChannels + (threadIdx.x >> 5);
     float s = 0.f, sc = 0.f, q = 0.f, qc = 0.f;
     if (c < K) {
         const int64_t ld = 2 * (int64_t)K;
         int t = j;
-        for (; t + 24 < nparts; t += 32) {
+        for (; t + 96 < nparts; t += 128) {
             float vs[4], vq[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                vs[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + c);
-                vq[u] = __ldg(part + (int64_t)(t + 8 * u) * ld + K + c);
+                vs[u] = __ldg(part + (int64_t)(t + 32 * u) * ld + c);
+                vq[u] = __ldg(part + (int64_t)(t + 32 * u) * ld + K + c);
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
@@ -324,14 +328,14 @@ __device__ __forceinline__ int partials_colsum(const float* __restrict__ part, i
                 kahan_add(q, qc, vq[u]);
             }
         }
-        for (; t < nparts; t += 8) {
+        for (; t < nparts; t += 32) {
             kahan_add(s, sc, __ldg(part + (int64_t)t * ld + c));
             kahan_add(q, qc, __ldg(part + (int64_t)t * ld + K + c));
         }
     }
     double ds = (double)s - (double)sc, dq = (double)q - (double)qc;
 #pragma unroll
-    for (int o = 1; o < 8; o <<= 1) {
+    for (int o = 1; o < 32; o <<= 1) {
         ds += __shfl_xor_sync(0xffffffffu, ds, o);
         dq += __shfl_xor_sync(0xffffffffu, dq, o);
     }
