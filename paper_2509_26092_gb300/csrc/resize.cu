@@ -112,7 +112,9 @@ int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, 
 // One CTA per unrolled row (n, m): it interpolates the rg resized rows once
 // into shared memory (with pw zero columns on each side), then writes the
 // row's Q positions as 16-byte chunks (8 elements), consecutive threads on
-// consecutive chunks.
+// consecutive chunks, each chunk gathered from the staged pixels with 16-byte
+// loads.  A resolution equal to the source's (lambda = 0, i0 = j: the
+// interpolation returns the pixel itself, bit for bit) skips the taps.
 constexpr int kStemMaxW = 1024;  // widest resized row a CTA stages (host-checked)
 
 // Per-channel affine map of 8-bit pixels to the network's input values,
@@ -147,6 +149,7 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict_
     const int32_t wst = wo + 2 * pw + 8;
     const int32_t m = blockIdx.x % M, b = blockIdx.x / M;
     const Tin* base = in + (int64_t)b * hi * wi * c;
+    const bool ident = hi == ho && wi == wo;
     // the RG source rows of this unrolled row: taps once per CTA
     Taps ty[RG];
     bool yin[RG];
@@ -173,43 +176,54 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict_
                 in_y = yin[k];
             }
         if (in_y && x >= 0 && x < wo) {
-            const Taps tx = axis_taps(x, wi, wo);
-            const Tin* r0 = base + (int64_t)tyy.i0 * wi * c;
-            const Tin* r1 = base + (int64_t)tyy.i1 * wi * c;
+            if (ident) {
+                const Tin* p = base + ((int64_t)tyy.i0 * wi + x) * c;
 #pragma unroll
-            for (int ch = 0; ch < cu; ++ch)
-                if (ch < c) {
-                    const float top = (1.f - tx.lam) * stem_pixel(r0 + tx.i0 * c + ch, ch, nm) +
-                                      tx.lam * stem_pixel(r0 + tx.i1 * c + ch, ch, nm);
-                    const float bot = (1.f - tx.lam) * stem_pixel(r1 + tx.i0 * c + ch, ch, nm) +
-                                      tx.lam * stem_pixel(r1 + tx.i1 * c + ch, ch, nm);
-                    v[ch] = (1.f - tyy.lam) * top + tyy.lam * bot;
-                }
-        }
-        float* dst = rows + (int64_t)i * cu;
-        if constexpr (cu == 4) {
-            *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
-        } else {
+                for (int ch = 0; ch < cu; ++ch)
+                    if (ch < c) v[ch] = stem_pixel(p + ch, ch, nm);
+            } else {
+                const Taps tx = axis_taps(x, wi, wo);
+                const Tin* r0 = base + (int64_t)tyy.i0 * wi * c;
+                const Tin* r1 = base + (int64_t)tyy.i1 * wi * c;
 #pragma unroll
-            for (int ch = 0; ch < cu; ++ch) dst[ch] = v[ch];
+                for (int ch = 0; ch < cu; ++ch)
+                    if (ch < c) {
+                        const float top = (1.f - tx.lam) * stem_pixel(r0 + tx.i0 * c + ch, ch, nm) +
+                                          tx.lam * stem_pixel(r0 + tx.i1 * c + ch, ch, nm);
+                        const float bot = (1.f - tx.lam) * stem_pixel(r1 + tx.i0 * c + ch, ch, nm) +
+                                          tx.lam * stem_pixel(r1 + tx.i1 * c + ch, ch, nm);
+                        v[ch] = (1.f - tyy.lam) * top + tyy.lam * bot;
+                    }
+            }
         }
+        float4* dst = reinterpret_cast<float4*>(rows + (int64_t)i * cu);
+#pragma unroll
+        for (int k = 0; k < cu / 4; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
     }
     __syncthreads();
     uint4* orow = reinterpret_cast<uint4*>(out) + ((int64_t)b * M + m) * Q * 8;
+    const float4* srow = reinterpret_cast<const float4*>(rows);  // staged pixel (e, xs): cu/4 float4 at (e*wst+xs)*cu/4
+    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int32_t idx = threadIdx.x; idx < Q * 8; idx += blockDim.x) {
         const int32_t q = idx >> 3, chunk = idx & 7;
-        const int32_t e = chunk / cu, tap0 = (chunk % cu) * (8 / cu);
-        float v[8];
-#pragma unroll
-        for (int u = 0; u < 8 / cu; ++u) {
-            const int32_t t = tap0 + u;
-            const int32_t xs = q * sw + t;  // staged column of image column q*sw + t - pw
-#pragma unroll
-            for (int ch = 0; ch < cu; ++ch) v[u * cu + ch] = t < taps ? rows[(e * wst + xs) * cu + ch] : 0.f;
+        float4 f[2];
+        if constexpr (RG == 2) {
+            // chunk = (row e, tap pair): taps t0, t0+1 of 4 channels each
+            const int32_t e = chunk >> 2, t0 = (chunk & 3) * 2;
+            const float4* pp = srow + (e * wst + q * sw + t0);
+            f[0] = t0 < taps ? pp[0] : zero;
+            f[1] = t0 + 1 < taps ? pp[1] : zero;
+        } else {
+            // chunk = tap t of 8 channels
+            const float4* pp = srow + 2 * (q * sw + chunk);
+            f[0] = chunk < taps ? pp[0] : zero;
+            f[1] = chunk < taps ? pp[1] : zero;
         }
         __nv_bfloat162 qv[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) qv[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+        qv[0] = __floats2bfloat162_rn(f[0].x, f[0].y);
+        qv[1] = __floats2bfloat162_rn(f[0].z, f[0].w);
+        qv[2] = __floats2bfloat162_rn(f[1].x, f[1].y);
+        qv[3] = __floats2bfloat162_rn(f[1].z, f[1].w);
         orow[idx] = *reinterpret_cast<uint4*>(qv);
     }
 }
@@ -242,7 +256,7 @@ int resize_stem_impl(const Tin* in, int32_t n, int32_t h_in, int32_t w_in, int32
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: rows wider than %d pixels", kStemMaxW);
     if (n == 0) return DBL_OK;
     const int blocks = n * rows_out;  // one CTA per unrolled row
-    const size_t smem = (size_t)row_group * (w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels
+    const size_t smem = (size_t)(w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels of fp32
     if (row_group == 2)
         resize_stem_kernel<2, Tin><<<blocks, 256, smem, as_stream(stream)>>>(
             in, static_cast<__nv_bfloat16*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
