@@ -94,6 +94,27 @@ __global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* _
 // BatchNorm pass would store it, bf16(relu(y*scale + shift)) with the same
 // fp32 operations, and then pooled, so the pooled values and the argmax are
 // those of pooling the stored BatchNorm output.
+// One pair of channels of one input vector through BatchNorm + ReLU, as
+// bf16x2: each lane is bf16(y*scale + shift) from one fp32 fma, then
+// max(., 0) in bf16, which maps negatives and NaN to zero like the stored
+// pass's relu.  A result may be -0 where that pass stores +0; the pool's
+// comparisons treat the two alike and the stored maximum is made +0.
+__device__ __forceinline__ uint32_t bn_relu_pair(uint32_t w, float2 sc, float2 sh)
+{
+    const float o0 = __fmaf_rn(__uint_as_float(w << 16), sc.x, sh.x);
+    const float o1 = __fmaf_rn(__uint_as_float(w & 0xffff0000u), sc.y, sh.y);
+    uint32_t v;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(v) : "f"(o1), "f"(o0));
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(v) : "r"(v), "r"(0u));
+    return v;
+}
+
+// The taps of a window are visited last to first with a >= comparison, so the
+// index left is the first maximum in (r, s) order, as in the plain max pool.
+// A thread keeps one channel group g for all its windows (the block size is a
+// multiple of C/8), so the per-channel scale and shift are computed once, and
+// it walks its windows by a fixed pixel stride with carries instead of
+// divisions.
 __global__ void __launch_bounds__(256)
     bn_relu_maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ gamma,
                                const float* __restrict__ beta, const float* __restrict__ mean,
@@ -101,120 +122,202 @@ __global__ void __launch_bounds__(256)
                                uint8_t* __restrict__ arg, int n, int H, int W, int C, int P, int Q)
 {
     const unsigned groups = (unsigned)C / 8u;
-    const unsigned total = (unsigned)n * P * Q * groups;
-    // a thread keeps its channel group across the grid-stride loop when the stride is a multiple of groups
-    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
-        const unsigned g = t % groups;
-        unsigned pix = t / groups;
-        const int q = (int)(pix % (unsigned)Q);
-        pix /= (unsigned)Q;
-        const int p = (int)(pix % (unsigned)P);
-        const int b = (int)(pix / (unsigned)P);
-        float sc[8], sh[8];
+    const unsigned per_block = blockDim.x / groups;
+    if (threadIdx.x >= per_block * groups) return;
+    const unsigned g = threadIdx.x % groups;
+    const unsigned npix = (unsigned)n * P * Q;
+    unsigned pix = blockIdx.x * per_block + threadIdx.x / groups;
+    const unsigned stride = gridDim.x * per_block;
+    int q = (int)(pix % (unsigned)Q), p = (int)((pix / (unsigned)Q) % (unsigned)P),
+        b = (int)(pix / ((unsigned)Q * P));
+    const int step_q = (int)(stride % (unsigned)Q), step_p = (int)((stride / (unsigned)Q) % (unsigned)P),
+              step_b = (int)(stride / ((unsigned)Q * P));
+    float2 sc[4], sh[4];
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
-            dbl::dev::bn_scale_shift(gamma[8 * g + k], beta[8 * g + k], mean[8 * g + k], invstd[8 * g + k], sc[k],
-                                     sh[k]);
-        float best[8];
-        uint8_t bi[8];
+    for (int k = 0; k < 4; ++k) {
+        const int c0 = 8 * g + 2 * k;
+        dbl::dev::bn_scale_shift(gamma[c0], beta[c0], mean[c0], invstd[c0], sc[k].x, sh[k].x);
+        dbl::dev::bn_scale_shift(gamma[c0 + 1], beta[c0 + 1], mean[c0 + 1], invstd[c0 + 1], sc[k].y, sh[k].y);
+    }
+    const int64_t row_vecs = (int64_t)W * groups;  // uint4 vectors per input row
+    for (; pix < npix; pix += stride) {
+        const uint4* xv = reinterpret_cast<const uint4*>(x) + ((int64_t)b * H + 2 * p - 1) * row_vecs +
+                          (int64_t)(2 * q - 1) * groups + g;
+        const bool r_ok[3] = {p > 0, true, 2 * p + 1 < H};
+        const bool s_ok[3] = {q > 0, true, 2 * q + 1 < W};
+        // rows last to first, the next row's loads in flight while one is pooled
+        uint32_t best[4] = {0u, 0u, 0u, 0u}, idx[4] = {0u, 0u, 0u, 0u};
+        uint4 cur[3], nxt[3];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            best[k] = -INFINITY;
-            bi[k] = 0;
+        for (int s = 0; s < 3; ++s) {
+            cur[s] = (r_ok[2] && s_ok[s]) ? __ldg(xv + 2 * row_vecs + s * (int64_t)groups) : make_uint4(0u, 0u, 0u, 0u);
+            nxt[s] = s_ok[s] ? __ldg(xv + row_vecs + s * (int64_t)groups) : make_uint4(0u, 0u, 0u, 0u);
         }
-        for (int r = 0; r < 3; ++r) {
-            const int h = 2 * p + r - 1;
-            if (h < 0 || h >= H) continue;
-            for (int s = 0; s < 3; ++s) {
-                const int w = 2 * q + s - 1;
-                if (w < 0 || w >= W) continue;
-                float f[8];
-                unpack8(__ldg(reinterpret_cast<const uint4*>(x + (((int64_t)b * H + h) * W + w) * C) + g), f);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    const float o = __fadd_rn(__fmaf_rn(f[k], sc[k], sh[k]), 0.f);
-                    const float a = __bfloat162float(__float2bfloat16_rn(o > 0.f ? o : 0.f));
-                    if (a > best[k]) {  // strict: the first maximum in (r, s) order wins ties
-                        best[k] = a;
-                        bi[k] = (uint8_t)(r * 3 + s);
+        for (int r = 2; r >= 0; --r) {
+            if (r_ok[r]) {
+#pragma unroll
+                for (int s = 2; s >= 0; --s) {
+                    if (!s_ok[s]) continue;
+                    const uint32_t tap = (uint32_t)(3 * r + s) * 0x10001u;
+                    const uint32_t w[4] = {cur[s].x, cur[s].y, cur[s].z, cur[s].w};
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const uint32_t a = bn_relu_pair(w[k], sc[k], sh[k]);
+                        uint32_t ge, m;
+                        asm("set.ge.u32.bf16x2 %0, %1, %2;" : "=r"(ge) : "r"(a), "r"(best[k]));
+                        asm("max.bf16x2 %0, %1, %2;" : "=r"(m) : "r"(best[k]), "r"(a));
+                        best[k] = m;
+                        idx[k] = (ge & tap) | (~ge & idx[k]);
                     }
                 }
             }
+            if (r > 0) {
+#pragma unroll
+                for (int s = 0; s < 3; ++s) {
+                    cur[s] = nxt[s];
+                    if (r == 2)
+                        nxt[s] = (r_ok[0] && s_ok[s]) ? __ldg(xv + s * (int64_t)groups) : make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
         }
-        const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
-        *reinterpret_cast<uint4*>(y + o) = pack8(best);
-        uint2 packed;
-        packed.x = bi[0] | (bi[1] << 8) | (bi[2] << 16) | ((uint32_t)bi[3] << 24);
-        packed.y = bi[4] | (bi[5] << 8) | (bi[6] << 16) | ((uint32_t)bi[7] << 24);
-        *reinterpret_cast<uint2*>(arg + o) = packed;
+        uint4 out;
+        // +0 for a maximum of zero (a -0 lane is negative as a signed 16-bit value)
+        asm("max.s16x2 %0, %1, %2;" : "=r"(out.x) : "r"(best[0]), "r"(0u));
+        asm("max.s16x2 %0, %1, %2;" : "=r"(out.y) : "r"(best[1]), "r"(0u));
+        asm("max.s16x2 %0, %1, %2;" : "=r"(out.z) : "r"(best[2]), "r"(0u));
+        asm("max.s16x2 %0, %1, %2;" : "=r"(out.w) : "r"(best[3]), "r"(0u));
+        const int64_t o = (int64_t)pix * C + 8 * g;
+        *reinterpret_cast<uint4*>(y + o) = out;
+        *reinterpret_cast<uint2*>(arg + o) = make_uint2(__byte_perm(idx[0], idx[1], 0x6420),
+                                                         __byte_perm(idx[2], idx[3], 0x6420));
+        q += step_q;
+        if (q >= Q) {
+            q -= Q;
+            ++p;
+        }
+        p += step_p;
+        if (p >= P) {
+            p -= P;
+            ++b;
+        }
+        b += step_b;
+    }
+}
+
+// dst[k] += src[k] where byte k of the argmax word pair equals tap (fp32; a
+// skipped term leaves dst as it is)
+__device__ __forceinline__ void add_if_tap(float (&dst)[8], const float (&src)[8], uint2 a, uint32_t tap)
+{
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const uint32_t byte = ((k < 4 ? a.x : a.y) >> (8 * (k & 3))) & 0xffu;
+        if (byte == tap) dst[k] += src[k];
     }
 }
 
 // Gather form over 2x2 blocks of input pixels: block (i, j) = rows 2i..2i+1,
 // cols 2j..2j+1 is covered by windows (i..i+1, j..j+1); window (p, q) reaches
-// input (h, w) at tap (h - 2p + 1, w - 2q + 1).  Each window's argmax and
-// gradient are read once per block, and every input pixel sums its windows in
-// (p, q) order.
+// input (h, w) at tap (h - 2p + 1, w - 2q + 1).  So pixel (2i, 2j) takes tap 4
+// of window (i, j); (2i, 2j+1) taps 5 and 3 of windows (i, j), (i, j+1);
+// (2i+1, 2j) taps 7 and 1 of (i, j), (i+1, j); (2i+1, 2j+1) taps 8, 6, 2, 0
+// of the four.  Each pixel sums its windows in (p, q) order, in fp32 from
+// zero.  A thread keeps one channel group and steps through the blocks with
+// carries, as in the forward pass.
 __global__ void __launch_bounds__(256)
     maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dy, const __nv_bfloat16* __restrict__ dy2,
                        const uint8_t* __restrict__ arg, __nv_bfloat16* __restrict__ dx, int n, int H, int W, int C,
                        int P, int Q)
 {
     const unsigned groups = (unsigned)C / 8u;
-    const int BH = (H + 1) / 2, BW = (W + 1) / 2;
-    const unsigned total = (unsigned)n * BH * BW * groups;
-    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
-        const unsigned g = t % groups;
-        unsigned pix = t / groups;
-        const int j = (int)(pix % (unsigned)BW);
-        pix /= (unsigned)BW;
-        const int i = (int)(pix % (unsigned)BH);
-        const int b = (int)(pix / (unsigned)BH);
-        float acc[4][8] = {};
-        for (int dp = 0; dp < 2; ++dp) {
-            const int p = i + dp;
-            if (p >= P) continue;
-            for (int dq = 0; dq < 2; ++dq) {
-                const int q = j + dq;
-                if (q >= Q) continue;
-                const int64_t o = (((int64_t)b * P + p) * Q + q) * C + 8 * g;
-                const uint2 a = __ldg(reinterpret_cast<const uint2*>(arg + o));
-                const uint8_t* ab = reinterpret_cast<const uint8_t*>(&a);
-                float f[8];
-                unpack8(__ldg(reinterpret_cast<const uint4*>(dy + o)), f);
-                if (dy2) {
-                    float f2[8];
-                    unpack8(__ldg(reinterpret_cast<const uint4*>(dy2 + o)), f2);
+    const unsigned per_block = blockDim.x / groups;
+    if (threadIdx.x >= per_block * groups) return;
+    const unsigned g = threadIdx.x % groups;
+    const int BH = (H + 1) / 2, BW = (W + 1) / 2;  // BH == P and BW == Q
+    const unsigned nblk = (unsigned)n * BH * BW;
+    unsigned blk = blockIdx.x * per_block + threadIdx.x / groups;
+    const unsigned stride = gridDim.x * per_block;
+    int j = (int)(blk % (unsigned)BW), i = (int)((blk / (unsigned)BW) % (unsigned)BH),
+        b = (int)(blk / ((unsigned)BW * BH));
+    const int step_j = (int)(stride % (unsigned)BW), step_i = (int)((stride / (unsigned)BW) % (unsigned)BH),
+              step_b = (int)(stride / ((unsigned)BW * BH));
+    const int64_t win_row = (int64_t)Q * C;
+    for (; blk < nblk; blk += stride) {
+        const bool ok[4] = {true, j + 1 < Q, i + 1 < P, i + 1 < P && j + 1 < Q};
+        const int64_t o = (((int64_t)b * P + i) * Q + j) * C + 8 * g;  // window (i, j)
+        uint4 gv[4], gv2[4];
+        uint2 av[4];
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) f[k] += f2[k];
-                }
-#pragma unroll
-                for (int dh = 0; dh < 2; ++dh) {
-                    const int r = 2 * i + dh - 2 * p + 1;  // tap row of input row 2i+dh in window row p
-                    if (r < 0 || r > 2) continue;
-#pragma unroll
-                    for (int dw = 0; dw < 2; ++dw) {
-                        const int sx = 2 * j + dw - 2 * q + 1;
-                        if (sx < 0 || sx > 2) continue;
-                        const uint8_t me = (uint8_t)(r * 3 + sx);
-#pragma unroll
-                        for (int k = 0; k < 8; ++k)
-                            if (ab[k] == me) acc[dh * 2 + dw][k] += f[k];
-                    }
-                }
-            }
+        for (int t = 0; t < 4; ++t) {
+            const int64_t ot = o + (t >> 1) * win_row + (t & 1) * (int64_t)C;
+            gv[t] = ok[t] ? __ldg(reinterpret_cast<const uint4*>(dy + ot)) : make_uint4(0u, 0u, 0u, 0u);
+            gv2[t] = (ok[t] && dy2) ? __ldg(reinterpret_cast<const uint4*>(dy2 + ot)) : make_uint4(0u, 0u, 0u, 0u);
+            av[t] = ok[t] ? __ldg(reinterpret_cast<const uint2*>(arg + ot)) : make_uint2(~0u, ~0u);
         }
+        const bool h1 = 2 * i + 1 < H, w1 = 2 * j + 1 < W;
+        __nv_bfloat16* px = dx + (((int64_t)b * H + 2 * i) * W + 2 * j) * C + 8 * g;
+        const int64_t px_row = (int64_t)W * C;
+        float acc01[8] = {}, acc10[8] = {}, acc11[8] = {};
+        {
+            float f[8], f2[8], acc00[8] = {};
+            unpack8(gv[0], f);
+            if (dy2) {
+                unpack8(gv2[0], f2);
 #pragma unroll
-        for (int dh = 0; dh < 2; ++dh) {
-            const int h = 2 * i + dh;
-            if (h >= H) continue;
-#pragma unroll
-            for (int dw = 0; dw < 2; ++dw) {
-                const int w = 2 * j + dw;
-                if (w >= W) continue;
-                *reinterpret_cast<uint4*>(dx + (((int64_t)b * H + h) * W + w) * C + 8 * g) = pack8(acc[dh * 2 + dw]);
+                for (int k = 0; k < 8; ++k) f[k] += f2[k];
             }
+            add_if_tap(acc00, f, av[0], 4);
+            add_if_tap(acc01, f, av[0], 5);
+            add_if_tap(acc10, f, av[0], 7);
+            add_if_tap(acc11, f, av[0], 8);
+            *reinterpret_cast<uint4*>(px) = pack8(acc00);
         }
+        {
+            float f[8], f2[8];
+            unpack8(gv[1], f);
+            if (dy2) {
+                unpack8(gv2[1], f2);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) f[k] += f2[k];
+            }
+            add_if_tap(acc01, f, av[1], 3);
+            add_if_tap(acc11, f, av[1], 6);
+            if (w1) *reinterpret_cast<uint4*>(px + C) = pack8(acc01);
+        }
+        {
+            float f[8], f2[8];
+            unpack8(gv[2], f);
+            if (dy2) {
+                unpack8(gv2[2], f2);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) f[k] += f2[k];
+            }
+            add_if_tap(acc10, f, av[2], 1);
+            add_if_tap(acc11, f, av[2], 2);
+            if (h1) *reinterpret_cast<uint4*>(px + px_row) = pack8(acc10);
+        }
+        {
+            float f[8], f2[8];
+            unpack8(gv[3], f);
+            if (dy2) {
+                unpack8(gv2[3], f2);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) f[k] += f2[k];
+            }
+            add_if_tap(acc11, f, av[3], 0);
+            if (h1 && w1) *reinterpret_cast<uint4*>(px + px_row + C) = pack8(acc11);
+        }
+        j += step_j;
+        if (j >= BW) {
+            j -= BW;
+            ++i;
+        }
+        i += step_i;
+        if (i >= BH) {
+            i -= BH;
+            ++b;
+        }
+        b += step_b;
     }
 }
 
@@ -471,6 +574,7 @@ int dbl_bn_relu_maxpool_fwd(const dbl_bn_shape* s, int32_t n, int32_t h, int32_t
     const int c = s->c;
     if (c <= 0 || c % 8 || !s->relu || s->count != (int64_t)n * h * w)
         return set_error(DBL_ERR_INVALID, "bn_relu_maxpool_fwd: shape must be [n*h*w, c], c a multiple of 8, relu set");
+    if (c > 8192) return set_error(DBL_ERR_UNSUPPORTED, "bn_relu_maxpool_fwd: at most 8192 channels");
     if (!aligned16(x) || !aligned16(y) || (reinterpret_cast<uintptr_t>(argmax) & 7))
         return set_error(DBL_ERR_INVALID, "bn_relu_maxpool_fwd: misaligned pointer");
     const int P = (h + 2 - 3) / 2 + 1, Q = (w + 2 - 3) / 2 + 1;
@@ -479,7 +583,9 @@ int dbl_bn_relu_maxpool_fwd(const dbl_bn_shape* s, int32_t n, int32_t h, int32_t
     cudaStream_t st = as_stream(stream);
     int rc = bn_fwd_finalize(s->count, c, s->eps, ch_sum, ch_sumsq, save_mean, save_invstd, st);
     if (rc) return rc;
-    bn_relu_maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q * (c / 8), 256), 256, 0, st>>>(
+    // a block size that is a multiple of the channel groups: each thread keeps its group
+    const int groups = c / 8, block = groups * std::max(1, 256 / groups);
+    bn_relu_maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q, block / groups), block, 0, st>>>(
         static_cast<const __nv_bfloat16*>(x), gamma, beta, save_mean, save_invstd, static_cast<__nv_bfloat16*>(y),
         argmax, n, h, w, c, P, Q);
     return launch_check("bn_relu_maxpool_fwd launch");
@@ -498,7 +604,10 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
     if ((int64_t)n * h * w * (c / 8) >= (int64_t)1 << 31)
         return set_error(DBL_ERR_UNSUPPORTED, "maxpool_bwd: tensor too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
-    maxpool_bwd_kernel<<<grid_for((int64_t)n * ((h + 1) / 2) * ((w + 1) / 2) * (c / 8), 256), 256, 0,
+    if (c > 8192) return set_error(DBL_ERR_UNSUPPORTED, "maxpool_bwd: at most 8192 channels");
+    // a block size that is a multiple of the channel groups: each thread keeps its group
+    const int groups = c / 8, block = groups * std::max(1, 256 / groups);
+    maxpool_bwd_kernel<<<grid_for((int64_t)n * ((h + 1) / 2) * ((w + 1) / 2), block / groups), block, 0,
                          as_stream(stream)>>>(
         static_cast<const __nv_bfloat16*>(dy), static_cast<const __nv_bfloat16*>(dy2), argmax,
         static_cast<__nv_bfloat16*>(dx), n, h, w, c, P, Q);

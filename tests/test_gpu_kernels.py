@@ -235,11 +235,20 @@ def test_bn_fwd_bwd_match_oracle(D, count, C, relu, res):
     check_status(D)
 
 
-def test_bn_relu_maxpool_equals_bn_then_maxpool(D):
-    """The fused stem pass equals the BatchNorm pass followed by the max pool, bit for bit."""
-    n, H, W, C = 3, 20, 18, 64
+@pytest.mark.parametrize("n,H,W,C,coarse", [(3, 20, 18, 64, False), (2, 21, 17, 64, False), (1, 112, 112, 64, False),
+                                            (2, 14, 14, 128, False), (2, 30, 26, 8, True), (16, 112, 112, 64, True),
+                                            (4, 48, 48, 2048, False)])
+def test_bn_relu_maxpool_equals_bn_then_maxpool(D, n, H, W, C, coarse):
+    """The fused stem pass equals the BatchNorm pass followed by the max pool, bit for bit.
+
+    Odd sizes clip windows at the bottom and right; 8 channels make one channel group a
+    window; 16 x 112 x 112 has more windows than the grid, so threads step on through the
+    batch; coarse inputs sit on a grid of quarters, so windows hold exact positive ties."""
     g = rng(77)
-    y = bf16_values(g.standard_normal((n, H, W, C)) * 2.0 + 0.3)
+    y = g.standard_normal((n, H, W, C)) * 2.0 + 0.3
+    if coarse:
+        y = np.round(y * 4.0) / 4.0
+    y = bf16_values(y)
     gamma = (1.0 + 0.2 * g.standard_normal(C)).astype(np.float32)
     beta = (0.1 * g.standard_normal(C)).astype(np.float32)
     yd, gd, bd = to_bf16_dev(y), to_f32_dev(gamma), to_f32_dev(beta)
@@ -281,6 +290,39 @@ def test_maxpool_matches_oracle(D, n, h, w, c, zeros):
     D.dbl_maxpool_bwd(n, h, w, c, to_bf16_dev(dy), to_bf16_dev(dy2), arg, dx)
     rdx = orc.maxpool_bwd(dy + dy2, rarg, x.shape, 3, 2, 1)
     assert max_norm_rel(host(dx), rdx) <= CONV_TOL
+
+
+@pytest.mark.parametrize("n,h,w,c", [(2, 9, 10, 64), (3, 13, 16, 128), (16, 112, 112, 64)])
+def test_maxpool_bwd_equals_fp32_window_order_gather(D, n, h, w, c):
+    """The max-pool gradient is, bit for bit, the fp32 sum from zero of each input pixel's
+    window gradients (dy + dy2 in fp32) in (p, q) window order, rounded to bf16 once; odd
+    sizes clip windows, and 16 x 112 x 112 has more 2x2 blocks than the grid."""
+    g = rng(n * h + c)
+    x = np.maximum(g.standard_normal((n, h, w, c)), 0.0)  # ties at zero
+    xd = to_bf16_dev(bf16_values(x))
+    P, Q = (h - 1) // 2 + 1, (w - 1) // 2 + 1
+    y = torch.empty((n, P, Q, c), dtype=torch.bfloat16, device="cuda")
+    arg = torch.empty((n, P, Q, c), dtype=torch.uint8, device="cuda")
+    D.dbl_maxpool_fwd(n, h, w, c, xd, y, arg)
+    dy = to_bf16_dev(bf16_values(g.standard_normal((n, P, Q, c))))
+    dy2 = to_bf16_dev(bf16_values(g.standard_normal((n, P, Q, c))))
+    dx = torch.empty_like(xd)
+    D.dbl_maxpool_bwd(n, h, w, c, dy, dy2, arg, dx)
+    f = torch.nn.functional.pad(dy.float() + dy2.float(), (0, 0, 0, 1, 0, 1))
+    a = torch.nn.functional.pad(arg.int(), (0, 0, 0, 1, 0, 1), value=255)
+    ref = torch.empty_like(dx)
+    for dh in range(2):
+        for dw in range(2):
+            acc = torch.zeros((n, P, Q, c), device="cuda")
+            for dp in range(2):
+                for dq in range(2):
+                    r, s = dh - 2 * dp + 1, dw - 2 * dq + 1
+                    if 0 <= r <= 2 and 0 <= s <= 2:
+                        win = (slice(None), slice(dp, dp + P), slice(dq, dq + Q))
+                        acc = acc + torch.where(a[win] == 3 * r + s, f[win], torch.zeros_like(acc))
+            ref[:, dh::2, dw::2] = acc[:, : (h - dh + 1) // 2, : (w - dw + 1) // 2].to(torch.bfloat16)
+    assert torch.equal(dx, ref)
+    check_status(D)
 
 
 # ----------------------------------------------------------------------------- head
