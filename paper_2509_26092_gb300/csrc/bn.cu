@@ -23,7 +23,9 @@ constexpr int kThreads = 256;
 constexpr int kMaxC = 2048;
 constexpr int kUnroll = 2;  // rows per thread whose loads are in flight together
 constexpr int kBlocksPerSM = 4;     // forward apply: 256-thread CTAs resident per SM (64 registers per thread)
-constexpr int kBwdBlocksPerSM = 3;  // backward passes (85 registers per thread)
+constexpr int kBwdBlocksPerSM = 3;  // backward apply pass (85 registers per thread)
+constexpr int kReduceBlocksPerSM = 2;  // backward reduce pass: four rows' loads in flight per thread
+constexpr int kReduceUnroll = 4;
 
 __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 {
@@ -105,7 +107,7 @@ __global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const fl
 
 // The same finalize from a convolution's per-CTA partials part[nparts][2][C]: the
 // fixed-order partial sums (partials_colsum, rounded to fp32 as dbl_conv_fwd stores
-// them), then mean and 1/std exactly as above.  One warp per channel.
+// them), then mean and 1/std exactly as above.
 __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_parts_kernel(int64_t count, int C, float eps,
                                                                     const float* __restrict__ part, int nparts,
                                                                     float* __restrict__ save_mean,
@@ -254,15 +256,18 @@ __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw,
     }
 }
 
-// Partial blk reduces a contiguous range of rows into partial[blk][0..C) (sum g)
-// and partial[blk][C..2C) (sum g*xhat); CTA b computes partials b, b + gridDim.x, ...
-// (each in a fixed order, so the result does not depend on the grid).
+// Partial blk reduces the row chunks blk, blk + nblk, blk + 2*nblk, ... (a chunk
+// is the kThreads/(C/8) rows one CTA covers in one step) into partial[blk][0..C)
+// (sum g) and partial[blk][C..2C) (sum g*xhat); CTA b computes partials b,
+// b + gridDim.x, ....  Interleaved chunks keep all CTAs streaming through the same
+// region of the tensors, and each partial adds its rows in a fixed order, so the
+// result does not depend on the grid.
 template <int MASK, bool WRITE_G>
-__global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
+__global__ void __launch_bounds__(kThreads, kReduceBlocksPerSM)
     bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
                          const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
                          int C, const float* __restrict__ gamma, const float* __restrict__ beta,
-                         const float* __restrict__ mean, const float* __restrict__ invstd, int rows_per_blk, int nblk,
+                         const float* __restrict__ mean, const float* __restrict__ invstd, int nblk,
                          float* __restrict__ partial, __nv_bfloat16* __restrict__ g_out)
 {
     const int groups = C / 8;
@@ -274,22 +279,21 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
 #pragma unroll
     for (int k = 0; k < 8; ++k) mu[k] = mean[8 * g + k];
     __shared__ float red[kThreads][17];
+    const int cstep = nblk * rstep;  // rows from one chunk of a partial to its next
+    constexpr int U = kReduceUnroll;  // chunks whose loads are in flight together
     for (int blk = blockIdx.x; blk < nblk; blk += gridDim.x) {
     float sg[8] = {}, sgx[8] = {};
-    const int r0 = blk * rows_per_blk;
-    const int r1 = min(count, r0 + rows_per_blk);
-    // kUnroll rows per iteration: all their loads are issued before any is used
-    int r = r0 + threadIdx.x / groups;
-    for (; r + (kUnroll - 1) * rstep < r1; r += kUnroll * rstep) {
-        Vec8 gg[kUnroll], yy[kUnroll];
+    int r = blk * rstep + threadIdx.x / groups;
+    for (; r + (U - 1) * cstep < count; r += U * cstep) {
+        Vec8 gg[U], yy[U];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) load_g_raw<MASK>(dout, dout2, out, y, (r + u * rstep) * groups + g, gg[u], yy[u]);
+        for (int u = 0; u < U; ++u) load_g_raw<MASK>(dout, dout2, out, y, (r + u * cstep) * groups + g, gg[u], yy[u]);
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u)
+        for (int u = 0; u < U; ++u)
             accumulate_g<MASK, WRITE_G>(gg[u], yy[u], dout2 != nullptr, rm, mu, sg, sgx, g_out,
-                                        (r + u * rstep) * groups + g);
+                                        (r + u * cstep) * groups + g);
     }
-    for (; r < r1; r += rstep) {
+    for (; r < count; r += cstep) {
         Vec8 gg, yy;
         load_g_raw<MASK>(dout, dout2, out, y, r * groups + g, gg, yy);
         accumulate_g<MASK, WRITE_G>(gg, yy, dout2 != nullptr, rm, mu, sg, sgx, g_out, r * groups + g);
@@ -319,9 +323,9 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
     }
 }
 
-// Fixed-order sum of the partials [nblk][2][C] (partials_colsum: one warp per
-// channel), then dgamma, dbeta and the three per-channel coefficients (A, B, C) of
-// the apply pass dy = A*g + B*y + C.
+// Fixed-order sum of the partials [nblk][2][C] (partials_colsum), then dgamma,
+// dbeta and the three per-channel coefficients (A, B, C) of the apply pass
+// dy = A*g + B*y + C.
 __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_bwd_finalize_kernel(
     const float* __restrict__ partial, int nblk, int C, int64_t count, const float* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ invstd, float* __restrict__ dgamma,
@@ -395,10 +399,13 @@ int bn_grid(int64_t nvec, int per_sm = kBlocksPerSM)
     return (int)(b < 1 ? 1 : b);
 }
 
+// One wave of CTAs that take the same number of partials each (512 partials on
+// 304 resident CTAs would leave 208 of them a second round alone).
 int reduce_grid(int64_t nblk)
 {
-    const int64_t cap = (int64_t)dbl::sm_count() * kBwdBlocksPerSM;
-    return (int)(nblk < cap ? nblk : cap);
+    const int64_t cap = (int64_t)dbl::sm_count() * kReduceBlocksPerSM;
+    const int64_t per_cta = (nblk + cap - 1) / cap;
+    return (int)((nblk + per_cta - 1) / per_cta);
 }
 
 int check_shape(const dbl_bn_shape* s, const char* who)
@@ -407,8 +414,11 @@ int check_shape(const dbl_bn_shape* s, const char* who)
     if (s->c % 8 != 0 || s->c > kMaxC || (kThreads % (s->c / 8)) != 0)
         return dbl::set_error(DBL_ERR_UNSUPPORTED, "%s: channel count %d (need a multiple of 8 dividing 2048)", who,
                               s->c);
-    // the streaming kernels index 16-byte vectors (and rows, plus one grid step) in 32 bits
-    if (s->count * (s->c / 8) + (int64_t)kThreads * dbl::sm_count() * kBlocksPerSM * kUnroll >= ((int64_t)1 << 31))
+    // the streaming kernels index 16-byte vectors (and rows, plus one grid step, or the
+    // reduce's kReduceUnroll chunk strides of at most 512 partials) in 32 bits
+    if (s->count * (s->c / 8) + (int64_t)kThreads * dbl::sm_count() * kBlocksPerSM * kUnroll +
+            (int64_t)kThreads * 512 * kReduceUnroll >=
+        ((int64_t)1 << 31))
         return dbl::set_error(DBL_ERR_UNSUPPORTED, "%s: %lld x %d elements exceed the 2^31-vector limit", who,
                               (long long)s->count, s->c);
     return DBL_OK;
@@ -427,7 +437,7 @@ int64_t bwd_blocks(int64_t count, int C)
 template <int MASK>
 int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
                     const float* gamma, const float* beta, const float* mean, const float* invstd, void* dy,
-                    void* dresidual, float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk, int rows,
+                    void* dresidual, float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk,
                     cudaStream_t st)
 {
     using namespace dbl;
@@ -438,11 +448,11 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
     __nv_bfloat16* g_store = static_cast<__nv_bfloat16*>(dresidual);
     if (g_store)
         bn_bwd_reduce_kernel<MASK, true><<<reduce_grid(nblk), kThreads, 0, st>>>(
-            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, rows, (int)nblk, partial,
+            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, (int)nblk, partial,
             g_store);
     else
         bn_bwd_reduce_kernel<MASK, false><<<reduce_grid(nblk), kThreads, 0, st>>>(
-            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, rows, (int)nblk, partial,
+            bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, (int)nblk, partial,
             nullptr);
     int rc = launch_check("bn_bwd_reduce launch");
     if (rc) return rc;
@@ -465,16 +475,16 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
 // with the ReLU mask taken from out, recomputed from y (out == NULL), or none.
 int bwd_launch(const dbl_bn_shape* s, const void* dout, const void* dout2, const void* y, const void* out,
                const float* gamma, const float* beta, const float* mean, const float* invstd, void* dy, void* dresidual,
-               float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk, int rows, cudaStream_t st)
+               float* dgamma, float* dbeta, float* partial, float* coef, int64_t nblk, cudaStream_t st)
 {
     if (!s->relu)
         return bwd_launch_mask<kMaskNone>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma,
-                                          dbeta, partial, coef, nblk, rows, st);
+                                          dbeta, partial, coef, nblk, st);
     if (out)
         return bwd_launch_mask<kMaskOut>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma,
-                                         dbeta, partial, coef, nblk, rows, st);
+                                         dbeta, partial, coef, nblk, st);
     return bwd_launch_mask<kMaskY>(s, dout, dout2, y, out, gamma, beta, mean, invstd, dy, dresidual, dgamma, dbeta,
-                                   partial, coef, nblk, rows, st);
+                                   partial, coef, nblk, st);
 }
 
 }  // namespace
@@ -575,12 +585,11 @@ int dbl_bn_relu_fused_bwd(const dbl_bn_shape* s, const void* dout, const void* d
         return set_error(DBL_ERR_WORKSPACE, "bn_relu_fused_bwd: workspace %zu < %zu bytes", ws_bytes, need);
     const int C = s->c;
     const int64_t nblk = bwd_blocks(s->count, s->c);
-    const int rows = (int)((s->count + nblk - 1) / nblk);
     float* partial = static_cast<float*>(ws);
     float* coef = partial + nblk * 2 * C;
     cudaStream_t st = as_stream(stream);
     return bwd_launch(s, dout, dout2, y, out, gamma, beta, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
-                      partial, coef, nblk, rows, st);
+                      partial, coef, nblk, st);
 }
 
 }  // extern "C"
@@ -648,8 +657,7 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
     float* partial = noalloc_scratch(&rc);
     if (rc) return rc;
     float* coef = partial + nblk * 2 * C;  // written by the finalize kernel before the apply kernel reads it
-    const int rows = (int)((s->count + nblk - 1) / nblk);
     cudaStream_t st = as_stream(stream);
     return bwd_launch(s, dout, dout2, y, out, gamma, beta, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
-                      partial, coef, nblk, rows, st);
+                      partial, coef, nblk, st);
 }

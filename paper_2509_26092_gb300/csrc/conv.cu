@@ -1182,7 +1182,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
 
 // ----------------------------------------------------------------------------- reductions
 // Per-output-channel sums of the conv epilogue's per-CTA partials part[nparts][2][K]
-// (partials_colsum: one warp per channel, fixed order).
+// (partials_colsum, fixed order).
 __global__ void __launch_bounds__(kPartialsThreads) stats_reduce_kernel(const float* __restrict__ part, int nparts, int K,
                                                            float* __restrict__ sum, float* __restrict__ sumsq)
 {

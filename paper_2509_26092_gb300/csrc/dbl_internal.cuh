@@ -297,51 +297,70 @@ __device__ __forceinline__ double colsum_fixed_order(const float* __restrict__ p
 // ---------------------------------------------------------------------------- per-block partial sums
 // Fixed-order column sums of per-block partials part[nparts][2][K] (row p: the two
 // sums block p produced for every channel: a convolution epilogue's sum y and sum
-// y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called by all threads of
-// a block of kPartialsThreads covering channels kPartialsChannels*blockIdx.x ..:
-// the 32 lanes j of a warp (one channel) add the partials j, j+32, ... in fp32 with
-// Kahan compensation (four loads in flight), then a fixed shuffle tree adds the 32
-// lane sums in fp64.  The order depends only on nparts, so the result is the same
-// on every launch and GPU.  Returns the channel (or -1 for lanes j != 0 and
-// channels past K) and its two sums.
+// y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called once by all
+// threads of a block of kPartialsThreads covering the kPartialsChannels channels
+// from kPartialsChannels*blockIdx.x: thread t takes channel t % 8 and stream
+// s = t / 8 of 32, and stream s adds the partials s, s+32, ... in fp32 with Kahan
+// compensation (sixteen loads in flight).  A warp's load then reads four partial
+// rows of eight adjacent channels, four whole 32-byte sectors.  The 32 stream sums
+// are added in fp64 by a fixed binary tree over the stream index, lowest bit first
+// (shuffles across lanes 8 and 16 apart, then pairs of warps through shared
+// memory).  The order depends only on nparts, so the result is the same on every
+// launch and GPU.  Returns the channel (for threads t < 8 whose channel is below
+// K, else -1) and its two sums.
 constexpr int kPartialsThreads = 256;
-constexpr int kPartialsChannels = kPartialsThreads / 32;
+constexpr int kPartialsChannels = 8;
+static_assert(kPartialsThreads == 32 * kPartialsChannels, "32 streams of 8 channels");
 
 __device__ __forceinline__ int partials_colsum(const float* __restrict__ part, int nparts, int K, double& sum0,
                                                double& sum1)
 {
-    const int j = threadIdx.x & 31, c = blockIdx.x * kPartialsChannels + (threadIdx.x >> 5);
+    __shared__ double red[2][kPartialsThreads / 32][kPartialsChannels];
+    const int cl = threadIdx.x % kPartialsChannels, stream = threadIdx.x / kPartialsChannels;
+    const int c = blockIdx.x * kPartialsChannels + cl;
     float s = 0.f, sc = 0.f, q = 0.f, qc = 0.f;
     if (c < K) {
         const int64_t ld = 2 * (int64_t)K;
-        int t = j;
-        for (; t + 96 < nparts; t += 128) {
-            float vs[4], vq[4];
+        for (int t = stream; t < nparts; t += 512) {
+            float vs[16], vq[16];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                vs[u] = __ldg(part + (int64_t)(t + 32 * u) * ld + c);
-                vq[u] = __ldg(part + (int64_t)(t + 32 * u) * ld + K + c);
+            for (int u = 0; u < 16; ++u) {
+                const bool in = t + 32 * u < nparts;
+                vs[u] = in ? __ldg(part + (int64_t)(t + 32 * u) * ld + c) : 0.f;
+                vq[u] = in ? __ldg(part + (int64_t)(t + 32 * u) * ld + K + c) : 0.f;
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                kahan_add(s, sc, vs[u]);
-                kahan_add(q, qc, vq[u]);
-            }
-        }
-        for (; t < nparts; t += 32) {
-            kahan_add(s, sc, __ldg(part + (int64_t)t * ld + c));
-            kahan_add(q, qc, __ldg(part + (int64_t)t * ld + K + c));
+            for (int u = 0; u < 16; ++u)
+                if (t + 32 * u < nparts) {
+                    kahan_add(s, sc, vs[u]);
+                    kahan_add(q, qc, vq[u]);
+                }
         }
     }
     double ds = (double)s - (double)sc, dq = (double)q - (double)qc;
+    // stream bits 0 and 1 are lane bits 3 and 4
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
+    for (int o = 8; o < 32; o <<= 1) {
         ds += __shfl_xor_sync(0xffffffffu, ds, o);
         dq += __shfl_xor_sync(0xffffffffu, dq, o);
     }
+    const int w = threadIdx.x / 32;
+    if ((threadIdx.x & 31) < kPartialsChannels) {
+        red[0][w][cl] = ds;
+        red[1][w][cl] = dq;
+    }
+    __syncthreads();
+    if (threadIdx.x < kPartialsChannels) {
+        // stream bits 2, 3 and 4 are warp bits 0, 1 and 2
+        const double(&a)[8][kPartialsChannels] = red[0];
+        const double(&b)[8][kPartialsChannels] = red[1];
+        ds = ((a[0][cl] + a[1][cl]) + (a[2][cl] + a[3][cl])) + ((a[4][cl] + a[5][cl]) + (a[6][cl] + a[7][cl]));
+        dq = ((b[0][cl] + b[1][cl]) + (b[2][cl] + b[3][cl])) + ((b[4][cl] + b[5][cl]) + (b[6][cl] + b[7][cl]));
+    }
+    __syncthreads();
     sum0 = ds;
     sum1 = dq;
-    return (j == 0 && c < K) ? c : -1;
+    return (threadIdx.x < kPartialsChannels && c < K) ? c : -1;
 }
 
 // ---------------------------------------------------------------------------- TMA
