@@ -79,6 +79,7 @@ struct ConvParams {
     int win_srows;            // padded rows loaded per strip (weight gradient: x strip)
     int win_dyrows;           // weight gradient: padded rows of the dy strip
     int win_strip_bytes;      // bytes of one strip buffer, or of one x + dy stage (a multiple of 1024)
+    int win_margin;           // CTA pairs: bytes before and after each strip buffer (0 for single CTAs)
 };
 
 __device__ __forceinline__ void report_timeout(volatile int* abort)
@@ -712,25 +713,44 @@ struct WinCfg {
 
 // One tap x 64-channel block of weights: K-major [BN out][64 in] for the forward
 // pass, MN-major [64 k][BN c] blocks of 64 for the data gradient (flipped tap).
-template <int BN, bool DG>
-__device__ __forceinline__ void win_load_wtile(const ConvParams& p, const CUtensorMap* tmB, uint8_t* dst, uint64_t* bar,
-                                               int tap, int cb, int n_tile)
+// CG = 2: this CTA's half of the BN columns (rank r: columns r*BN/2 ..), completing
+// on the barrier at shared::cluster address bar (the leader's).
+template <int BN, bool DG, int CG>
+__device__ __forceinline__ void win_load_wtile(const ConvParams& p, const CUtensorMap* tmB, uint8_t* dst, uint32_t bar,
+                                               int tap, int cb, int n_tile, int rank)
 {
     if constexpr (DG) {
         const int wtap = p.win_R * p.win_S - 1 - tap;  // flipped filter
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tma_load_3d_elect(dst + j * 8192, tmB, bar, n_tile * BN + 64 * j, wtap, cb * 64);
+        for (int j = 0; j < BN / 64 / CG; ++j)
+            tma_load_3d_cg<CG>(dst + j * 8192, tmB, bar, n_tile * BN + rank * (BN / CG) + 64 * j, wtap, cb * 64);
     } else {
-        tma_load_2d_elect(dst, tmB, bar, tap * p.Cin + cb * 64, n_tile * BN);
+        tma_load_2d_cg<CG>(dst, tmB, bar, tap * p.Cin + cb * 64, n_tile * BN + rank * (BN / CG));
     }
 }
 
-template <int BN, bool DG, bool RES>
+// CG = 2 (a cluster of two CTAs, tcgen05 .cta_group::2): CTA rank r computes tile
+// 2u + r of pair unit u.  Rank 0 issues M = 256 MMAs whose A rows 0-127 come from
+// its strip and rows 128-255 from rank 1's, at the same shared-memory address, and
+// whose B columns are split between the two CTAs' halves of the weights, so each SM
+// reads half of B per MMA.  The two tiles start at different offsets within a
+// padded row (off0), so rank 1 places its strip (off0 of rank 0 - off0 of rank 1)
+// rows away from rank 0's (inside a margin of one padded row on either side): the
+// descriptors rank 0 builds from its own off0 then read rank 1's tile at the same
+// rows.  Rank 0 owns the strip-full, weight-full and accumulator-empty barriers;
+// both CTAs' copies complete on rank 0's full barriers, rank 0's commits arrive on
+// both CTAs' empty and accumulator-full barriers, and both CTAs' epilogues arrive on
+// rank 0's accumulator-empty barrier.  A pair unit past the last tile loads zeros
+// (images past the batch) and stores nothing.
+template <int BN, bool DG, bool RES, int CG>
 __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
     conv_win_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const ConvParams p)
 {
     using C = WinCfg<BN>;
+    static_assert(CG == 1 || BN == 128, "CTA pairs split the weights in 64-column halves");
+    constexpr int BT = C::B_TILE / CG;  // this CTA's bytes of one tap x 64-channel block of weights
+    constexpr uint16_t kAll = CG == 2 ? 3 : 1;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t sfull[2], sempty[2], bfull[kWinBStages], bempty[kWinBStages], accf_bar[2],
         acce_bar[2], drain_bar;
@@ -740,20 +760,24 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
     uint8_t* sgen = smem_raw + (sbase - smem_u32(smem_raw));
+    const int rank = CG == 2 ? (int)cluster_ctarank() : 0;
+    const int unit0 = blockIdx.x / CG, nunits = gridDim.x / CG;
+    const int total_units = (p.total_tiles + CG - 1) / CG;
     const int CB = p.cblocks;
     const int ntaps = p.win_R * p.win_S;
-    const int b_bytes = RES ? ntaps * CB * C::B_TILE : kWinBStages * C::B_TILE;
-    uint8_t* strip = sgen + b_bytes;
+    const int b_bytes = RES ? ntaps * CB * BT : kWinBStages * BT;
+    const int strip_stride = p.win_strip_bytes + 2 * p.win_margin;
+    uint8_t* strip = sgen + b_bytes + p.win_margin;  // stage s at strip + s * strip_stride
     // per-warp statistics transposes reuse the strip buffers once the last tile's MMAs are done
-    float* epi_tile = reinterpret_cast<float*>(strip);
-    float* epi_sum = reinterpret_cast<float*>(strip + 2 * p.win_strip_bytes);
+    float* epi_tile = reinterpret_cast<float*>(sgen + b_bytes);
+    float* epi_sum = reinterpret_cast<float*>(sgen + b_bytes + 2 * strip_stride);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sfull[i], 1);
             mbar_init(&sempty[i], 1);
             mbar_init(&accf_bar[i], 1);
-            mbar_init(&acce_bar[i], C::EPI);  // one arrival per epilogue warp
+            mbar_init(&acce_bar[i], C::EPI * CG);  // one arrival per epilogue warp of the pair
         }
         for (int i = 0; i < kWinBStages; ++i) {
             mbar_init(&bfull[i], 1);
@@ -771,11 +795,12 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         tma_prefetch_desc(&tmB);
     }
     if (warp == C::W_MMA) {
-        tmem_alloc(&tmem_slot, C::TMEM_COLS);
-        tmem_relinquish();
+        tmem_alloc_cg<CG>(&tmem_slot, C::TMEM_COLS);
+        tmem_relinquish_cg<CG>();
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (CG == 2) cluster_sync_all();  // both CTAs' barriers initialised, TMEM allocated
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
     const int Wp = p.win_Wp;
@@ -785,9 +810,12 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         int it = 0;
         bool failed = false;
         const uint32_t strip_tx = (uint32_t)(p.win_srows * Wp * 128);
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
-            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
-            const int g0 = tc.m_tile * p.win_tile / Wp;
+        for (int t = unit0; t < total_units; t += nunits) {
+            const int m_tile = t * CG + rank;
+            const int L0 = m_tile * p.win_tile;
+            const int g0 = L0 / Wp;
+            // rank 1: rows between its strip and rank 0's, so that both tiles sit at rank 0's offsets
+            const int shift = (CG == 2 && rank == 1) ? ((L0 - p.win_tile) % Wp) - (L0 % Wp) : 0;
             for (int cb = 0; cb < CB; ++cb, ++it) {
                 const int s = it & 1;
                 const uint32_t ok = mbar_wait_warp(&sempty[s], ((it >> 1) & 1) ^ 1, &abort_flag);
@@ -795,35 +823,45 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                     failed = true;
                     break;
                 }
-                uint8_t* dst = strip + s * p.win_strip_bytes;
-                mbar_arrive_expect_tx_elect(&sfull[s], strip_tx);
+                uint8_t* dst = strip + s * strip_stride + shift * 128;
+                uint32_t fb = smem_u32(&sfull[s]);
+                if (CG == 1 || rank == 0) mbar_arrive_expect_tx_elect(&sfull[s], (uint32_t)CG * strip_tx);
+                if (CG == 2) fb = mapa_shared(fb, 0);
                 for (int r = 0; r < p.win_srows; ++r) {
                     const int g = g0 + r;
                     const int n = g / p.win_Hp, hp = g - n * p.win_Hp;
                     // padded row hp of image n = input row hp - ph from column -pw (padding rows and
                     // columns, and images past the batch, are outside the tensor and arrive as zeros)
-                    tma_load_4d_elect(dst + r * Wp * 128, &tmA, &sfull[s], cb * 64, -p.win_pw, hp - p.win_ph, n);
+                    tma_load_4d_cg<CG>(dst + r * Wp * 128, &tmA, fb, cb * 64, -p.win_pw, hp - p.win_ph, n);
                 }
             }
             if (failed) break;
         }
         if (failed) {
             if (lane == 0) report_timeout(&abort_flag);
-            for (int i = it - 1; i >= 0 && i >= it - 2; --i) (void)mbar_drain_warp(&sfull[i & 1], (i >> 1) & 1);
+            if (CG == 1 || rank == 0) {
+                for (int i = it - 1; i >= 0 && i >= it - 2; --i) (void)mbar_drain_warp(&sfull[i & 1], (i >> 1) & 1);
+            } else {
+                // rank 1's copies complete on rank 0's barriers: give them a fixed time instead
+                const uint64_t t0 = globaltimer();
+                while (globaltimer() - t0 < 1000000ull) {
+                }
+            }
         }
     } else if (warp == C::W_WEIGHT) {
         // ------------------------------------------------------------------ weight producer
         if (RES) {
-            mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(ntaps * CB * C::B_TILE));
+            uint32_t fb = smem_u32(&bfull[0]);
+            if (CG == 1 || rank == 0) mbar_arrive_expect_tx_elect(&bfull[0], (uint32_t)(CG * ntaps * CB * BT));
+            if (CG == 2) fb = mapa_shared(fb, 0);
             for (int tap = 0; tap < ntaps; ++tap)
                 for (int cb = 0; cb < CB; ++cb)
-                    win_load_wtile<BN, DG>(p, &tmB, sgen + (tap * CB + cb) * C::B_TILE, &bfull[0], tap, cb, 0);
-            (void)mbar_drain_warp(&bfull[0], 0);
+                    win_load_wtile<BN, DG, CG>(p, &tmB, sgen + (tap * CB + cb) * BT, fb, tap, cb, 0, rank);
+            if (CG == 1 || rank == 0) (void)mbar_drain_warp(&bfull[0], 0);
         } else {
             int bt = 0;
             bool failed = false;
-            for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x) {
-                const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
+            for (int t = unit0; t < total_units && !failed; t += nunits)
                 for (int cb = 0; cb < CB && !failed; ++cb)
                     for (int tap = 0; tap < ntaps; ++tap, ++bt) {
                         const int s = bt % kWinBStages;
@@ -833,27 +871,33 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                             failed = true;
                             break;
                         }
-                        mbar_arrive_expect_tx_elect(&bfull[s], (uint32_t)C::B_TILE);
-                        win_load_wtile<BN, DG>(p, &tmB, sgen + s * C::B_TILE, &bfull[s], tap, cb, tc.n_tile);
+                        uint32_t fb = smem_u32(&bfull[s]);
+                        if (CG == 1 || rank == 0) mbar_arrive_expect_tx_elect(&bfull[s], (uint32_t)(CG * BT));
+                        if (CG == 2) fb = mapa_shared(fb, 0);
+                        win_load_wtile<BN, DG, CG>(p, &tmB, sgen + s * BT, fb, tap, cb, 0, rank);
                     }
-            }
             if (failed) {
                 if (lane == 0) report_timeout(&abort_flag);
-                for (int i = bt - 1; i >= 0 && i >= bt - kWinBStages; --i)
-                    (void)mbar_drain_warp(&bfull[i % kWinBStages], (i / kWinBStages) & 1);
+                if (CG == 1 || rank == 0) {
+                    for (int i = bt - 1; i >= 0 && i >= bt - kWinBStages; --i)
+                        (void)mbar_drain_warp(&bfull[i % kWinBStages], (i / kWinBStages) & 1);
+                } else {
+                    const uint64_t t0 = globaltimer();
+                    while (globaltimer() - t0 < 1000000ull) {
+                    }
+                }
             }
         }
     } else if (warp == C::W_MMA) {
-        // ------------------------------------------------------------------ MMA issuer
-        const uint32_t idesc = idesc_bf16(BM, BN, 0u, DG ? 1u : 0u);
+        // ------------------------------------------------------------------ MMA issuer (rank 0 of a pair)
+        const uint32_t idesc = idesc_bf16(BM * CG, BN, 0u, DG ? 1u : 0u);
         int it = 0, bt = 0, lt = 0;
         bool failed = false;
-        if (RES) {
+        if (RES && (CG == 1 || rank == 0)) {
             const uint32_t ok = mbar_wait_warp(&bfull[0], 0, &abort_flag);
             failed = __any_sync(0xffffffffu, ok == 0u);
         }
-        for (int t = blockIdx.x; t < p.total_tiles && !failed; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
+        for (int t = unit0; t < total_units && (CG == 1 || rank == 0) && !failed; t += nunits, ++lt) {
             const int buf = lt & 1;
             const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
@@ -861,7 +905,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                 break;
             }
             tc_fence_after();
-            const int L0 = tc.m_tile * p.win_tile;
+            const int L0 = t * CG * p.win_tile;  // this CTA's (rank 0's) tile
             const int off0 = L0 - (L0 / Wp) * Wp;  // tile start within the strip's first row
             const uint32_t d = tmem + (uint32_t)(buf * kWinACC * BN);
             for (int cb = 0; cb < CB && !failed; ++cb, ++it) {
@@ -872,14 +916,14 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = sbase + (uint32_t)(b_bytes + s * p.win_strip_bytes);
+                const uint32_t sa = smem_u32(strip + s * strip_stride);
                 int r = 0, sx = 0;  // (tap / S, tap % S), stepped without divisions
 #pragma unroll 1
                 for (int tap = 0; tap < ntaps; ++tap) {
                     uint32_t sb;
                     int bs = 0;
                     if (RES) {
-                        sb = sbase + (uint32_t)((tap * CB + cb) * C::B_TILE);
+                        sb = sbase + (uint32_t)((tap * CB + cb) * BT);
                     } else {
                         bs = bt % kWinBStages;
                         const uint32_t okb = mbar_wait_warp(&bfull[bs], (bt / kWinBStages) & 1, &abort_flag);
@@ -888,7 +932,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                             break;
                         }
                         tc_fence_after();
-                        sb = sbase + (uint32_t)(bs * C::B_TILE);
+                        sb = sbase + (uint32_t)(bs * BT);
                     }
                     const uint32_t a0 = sa + (uint32_t)((off0 + r * Wp + sx) * 128);
                     // K-step j of accumulator a: A rows a*128.. of the shifted strip, 32 bytes per K-step;
@@ -896,10 +940,10 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                     static_assert(kWinACC == 2, "two accumulators per MMA group");
                     const uint64_t ad = smem_desc(a0, 16, 1024, kSwizzle128B);
                     const uint64_t bd = DG ? smem_desc(sb, 8192, 1024, kSwizzle128B) : smem_desc(sb, 16, 1024, kSwizzle128B);
-                    mma_bf16_x8_elect(d, d + BN, ad, (128 * 128) >> 4, 32 >> 4, bd, DG ? (2048 >> 4) : (32 >> 4), idesc,
-                                      (cb > 0 || tap > 0) ? 1u : 0u);
+                    mma_bf16_x8_elect_cg<CG>(d, d + BN, ad, (128 * 128) >> 4, 32 >> 4, bd, DG ? (2048 >> 4) : (32 >> 4),
+                                             idesc, (cb > 0 || tap > 0) ? 1u : 0u);
                     if (!RES) {
-                        mma_commit_elect(&bempty[bs]);
+                        mma_commit_elect_cg<CG>(&bempty[bs], kAll);
                         ++bt;
                     }
                     if (++sx == p.win_S) {
@@ -907,13 +951,15 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                         ++r;
                     }
                 }
-                mma_commit_elect(&sempty[s]);
+                mma_commit_elect_cg<CG>(&sempty[s], kAll);
             }
-            mma_commit_elect(&accf_bar[buf]);  // arrives when this tile's MMAs have completed
+            mma_commit_elect_cg<CG>(&accf_bar[buf], kAll);  // arrives when this unit's MMAs have completed
         }
-        if (failed && lane == 0) report_timeout(&abort_flag);
-        mma_commit_elect(&drain_bar);
-        (void)mbar_drain_warp(&drain_bar, 0);
+        if (CG == 1 || rank == 0) {
+            if (failed && lane == 0) report_timeout(&abort_flag);
+            mma_commit_elect_cg<CG>(&drain_bar, 1);
+            (void)mbar_drain_warp(&drain_bar, 0);
+        }
     } else {
         // ------------------------------------------------------------------ epilogue (warps 0 .. EPI-1)
         constexpr int CW = C::CW;
@@ -924,8 +970,8 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         rs.zero();
         const int img = p.win_Hp * Wp;
         int lt = 0;
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++lt) {
-            const TileCoord tc = decode_tile(p, t, (int)gridDim.x);
+        for (int t = unit0; t < total_units; t += nunits, ++lt) {
+            const int m_tile = t * CG + rank;
             const int buf = lt & 1;
             const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
@@ -938,11 +984,12 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
             int64_t out_row[kWinACC];
 #pragma unroll
             for (int a = 0; a < kWinACC; ++a) {
-                const int L = tc.m_tile * p.win_tile + a * 128 + row;
+                const int L = m_tile * p.win_tile + a * 128 + row;
                 const int n = L / img, rem = L - n * img;
                 const int hp = rem / Wp, wp = rem - hp * Wp;
                 // rows past the tile belong to the next tile (row-aligned tiles are shorter than 256)
-                valid[a] = a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P && wp < p.win_Q;
+                valid[a] = m_tile < p.total_tiles && a * 128 + row < p.win_tile && n < p.gN && hp < p.win_P &&
+                           wp < p.win_Q;
                 out_row[a] = ((int64_t)n * p.win_P + hp) * p.win_Q + wp;
             }
             // chunks c = (accumulator, 32 of this warp's columns)
@@ -960,12 +1007,17 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                 if (c + 1 < NC)
                     tmem_ld_32x32b_x32(taddr + (uint32_t)(((c + 1) / NCH) * BN + ((c + 1) % NCH) * 32), nxt);
                 float back[32];
-                store_row_chunk_bf16(p, cur, valid[a], out_row[a], tc.n_tile * BN + col0 + ch * 32, back);
+                store_row_chunk_bf16(p, cur, valid[a], out_row[a], col0 + ch * 32, back);
                 if (want_stats) rs.add(ch, back, lane);
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&acce_bar[buf]);
+            if (lane == 0) {
+                if constexpr (CG == 2)
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&acce_bar[buf]), 0));
+                else
+                    mbar_arrive(&acce_bar[buf]);
+            }
         }
         if (want_stats) {
             rs.flush(st_tile, wsum, p.Ncols, col0, lane);  // the window kernel has one column tile
@@ -983,9 +1035,11 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
     }
     tc_fence_before();
     __syncthreads();
+    // neither CTA of a pair leaves while the other may still signal its barriers or read its TMEM
+    if constexpr (CG == 2) cluster_sync_all();
     if (warp == C::W_MMA) {
         tc_fence_after();
-        tmem_dealloc(tmem, C::TMEM_COLS);
+        tmem_dealloc_cg<CG>(tmem, C::TMEM_COLS);
     }
 }
 
@@ -1365,6 +1419,8 @@ int win_tile_positions(int Wp) { return Wp >= 64 ? (kWinBMT / Wp) * Wp : kWinBMT
 // axes, 64-channel blocks of the reduced operand (red_c), 64 or 128 output
 // channels, padded rows of 10..256 positions; the data gradient (dgrad) for
 // 3x3 filters with pad 1 only (its taps are the forward taps flipped).
+bool win_pairs();
+
 bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& pl)
 {
     const Geom g = geom(s);
@@ -1384,17 +1440,31 @@ bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& 
     const int strip = ((srows * Wp * 128 + 1023) / 1024) * 1024;
     const int BN = out_c, CB = red_c / 64, ntaps = s->r * s->s;
     const bool res = BN == 64 && CB == 1 && ntaps <= 9;
-    const int b_bytes = res ? ntaps * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128;
-    // epilogue statistics: per-warp channel sums after the strips (the warps' transposes reuse the strips)
+    // CTA pairs for 128-column tiles: each SM stages half of the weights; rank 1's strip is
+    // shifted by up to a padded row either way, so each strip buffer gets a margin of one padded
+    // row on both sides (single CTAs when the pair layout does not fit in shared memory).  The
+    // 64-column forward pass measured slower on pairs (818 against 959 TFLOP/s at layer1).
+    if ((size_t)srows * Wp * 128 >= (1u << 20)) return false;
     const int epi = out_c == 64 ? WinCfg<64>::EPI : WinCfg<128>::EPI;
-    const size_t smem = (size_t)b_bytes + 2 * (size_t)strip + (size_t)epi * 2 * out_c * 4 + 1024;
-    if (2 * (size_t)strip < (size_t)epi * 32 * 33 * 4) return false;
-    if (smem > kWinSmemMax || (size_t)srows * Wp * 128 >= (1u << 20)) return false;
+    int cg = win_pairs() && BN == 128 ? 2 : 1;
+    int margin = 0;
+    size_t smem = 0;
+    for (;; cg = 1) {
+        margin = cg == 2 ? (Wp * 128 + 1023) / 1024 * 1024 : 0;
+        const int b_bytes = (res ? ntaps * CB * WinCfg<64>::B_TILE : kWinBStages * BN * 128) / cg;
+        // epilogue statistics: per-warp channel sums after the strips (the warps' transposes reuse the strips)
+        const size_t strips = 2 * ((size_t)strip + 2 * (size_t)margin);
+        smem = (size_t)b_bytes + strips + (size_t)epi * 2 * out_c * 4 + 1024;
+        if (strips >= (size_t)epi * 32 * 33 * 4 && smem <= kWinSmemMax) break;
+        if (cg == 1) return false;
+    }
     ConvParams& p = pl.p;
     pl.win = true;
     pl.res = res;
     pl.BN = BN;
+    pl.cg = cg;
     pl.smem = smem;
+    p.win_margin = margin;
     p.win_R = s->r;
     p.win_S = s->s;
     p.win_ph = g.ph;
@@ -1487,6 +1557,17 @@ bool pair_tiles(int BN, bool wgrad)
     }();
     if (level == 0) return false;
     return BN == 256 || (BN == 128 && (wgrad || level == 2));
+}
+
+// Window-kernel CTA pairs (128-column tiles); DBL_CONV_CTA_PAIRS=0 turns them off with
+// the others.
+bool win_pairs()
+{
+    static const bool on = [] {
+        const char* e = getenv("DBL_CONV_CTA_PAIRS");
+        return !(e && e[0] == '0');
+    }();
+    return on;
 }
 
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
@@ -1714,8 +1795,11 @@ int resident_pairs()
 
 // Persistent grid of a conv_igemm_kernel plan: one CTA per SM, or one CTA pair
 // per two SMs, never more CTAs (pairs) than tiles.
+int win_grid(const Plan& pl);
+
 int plan_grid(const Plan& pl)
 {
+    if (pl.win) return win_grid(pl);
     if (pl.cg == 1) return grid_size(pl.p.total_tiles);
     const bool wg = pl.mode == kWgrad || pl.mode == kWgradC8;
     int pairs = pl.BN == 256 ? (wg ? resident_pairs<256, kFamWgrad>() : resident_pairs<256, kFamFwd>())
@@ -1777,30 +1861,109 @@ int launch(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, const CUt
     return launch_cfg<64, kFamFwd, 1>(pl, a, b, a2, b2, grid, st);
 }
 
-template <int BN, bool DG, bool RES>
-int launch_win_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+template <int BN, bool DG, bool RES, int CG>
+int set_win_smem()
 {
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(conv_win_kernel<BN, DG, RES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kWinSmemMax);
+        cudaError_t e = cudaFuncSetAttribute(conv_win_kernel<BN, DG, RES, CG>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWinSmemMax);
         if (e != cudaSuccess) return dbl::cuda_check(e, "conv: set smem attribute");
         attr_set[dev] = true;
     }
-    conv_win_kernel<BN, DG, RES><<<grid, WinCfg<BN>::THREADS, pl.smem, st>>>(a, b, pl.p);
+    return DBL_OK;
+}
+
+// CTA pairs of conv_win_kernel<BN, DG, RES, 2> that fit on the device at once with
+// `smem` bytes each (one CTA per SM; cached per device), at most half the SMs.
+template <int BN, bool DG, bool RES>
+int resident_win_pairs(size_t smem)
+{
+    static int cached[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+    int pairs = std::min(dbl::sm_count() / 2, kMaxGrid / 2);
+    if (set_win_smem<BN, DG, RES, 2>() == DBL_OK) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(2 * pairs);
+        cfg.blockDim = dim3(WinCfg<BN>::THREADS);
+        cfg.dynamicSmemBytes = smem;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, conv_win_kernel<BN, DG, RES, 2>, &cfg) == cudaSuccess && n > 0)
+            pairs = std::min(pairs, n);
+        else
+            (void)cudaGetLastError();
+    }
+    if (pairs < 1) pairs = 1;
+    if (dev >= 0 && dev < 64) cached[dev] = pairs;
+    return pairs;
+}
+
+// Grid of a window-kernel plan: one CTA per SM (never more than tiles), or one CTA
+// pair per two SMs (never more pairs than pair units).
+int win_grid(const Plan& pl)
+{
+    if (pl.cg == 1) return grid_size(pl.p.total_tiles);
+    const bool dg = pl.mode == kDgrad;
+    int pairs = dg ? resident_win_pairs<128, true, false>(pl.smem) : resident_win_pairs<128, false, false>(pl.smem);
+    const int units = (pl.p.total_tiles + 1) / 2;
+    if (pairs > units) pairs = units;
+    return 2 * std::max(pairs, 1);
+}
+
+template <int BN, bool DG, bool RES, int CG>
+int launch_win_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
+{
+    int rc = set_win_smem<BN, DG, RES, CG>();
+    if (rc) return rc;
+    if constexpr (CG == 1) {
+        conv_win_kernel<BN, DG, RES, 1><<<grid, WinCfg<BN>::THREADS, pl.smem, st>>>(a, b, pl.p);
+    } else {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(WinCfg<BN>::THREADS);
+        cfg.dynamicSmemBytes = pl.smem;
+        cfg.stream = st;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        cudaError_t e = cudaLaunchKernelEx(&cfg, conv_win_kernel<BN, DG, RES, 2>, a, b, pl.p);
+        if (e != cudaSuccess) {
+            dbl::count_launch();
+            return dbl::cuda_check(e, "conv_win pair launch");
+        }
+    }
     return dbl::launch_check("conv_win launch");
 }
 
 int launch_win(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int grid, cudaStream_t st)
 {
     const bool dg = pl.mode == kDgrad;
-    if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false>(pl, a, b, grid, st)
-                                : launch_win_cfg<128, false, false>(pl, a, b, grid, st);
-    if (pl.res) return dg ? launch_win_cfg<64, true, true>(pl, a, b, grid, st)
-                          : launch_win_cfg<64, false, true>(pl, a, b, grid, st);
-    return dg ? launch_win_cfg<64, true, false>(pl, a, b, grid, st) : launch_win_cfg<64, false, false>(pl, a, b, grid, st);
+    if (pl.cg == 2) {
+        if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false, 2>(pl, a, b, grid, st)
+                                    : launch_win_cfg<128, false, false, 2>(pl, a, b, grid, st);
+        return dbl::set_error(DBL_ERR_UNSUPPORTED, "conv: CTA-pair window kernels need 128 columns");
+    }
+    if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false, 1>(pl, a, b, grid, st)
+                                : launch_win_cfg<128, false, false, 1>(pl, a, b, grid, st);
+    if (pl.res) return dg ? launch_win_cfg<64, true, true, 1>(pl, a, b, grid, st)
+                          : launch_win_cfg<64, false, true, 1>(pl, a, b, grid, st);
+    return dg ? launch_win_cfg<64, true, false, 1>(pl, a, b, grid, st)
+              : launch_win_cfg<64, false, false, 1>(pl, a, b, grid, st);
 }
 
 template <int NACC>
@@ -1856,7 +2019,7 @@ int conv_fwd_impl(const dbl_conv_shape* s, const void* x, const void* w, void* y
         const int64_t rsc = (int64_t)s->r * s->s * s->c;
         cuuint64_t dims[2] = {(cuuint64_t)rsc, (cuuint64_t)s->k};
         cuuint64_t str[1] = {(cuuint64_t)rsc * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)pl.BN};
+        cuuint32_t box[2] = {64, (cuuint32_t)(pl.BN / pl.cg)};  // a CTA pair stages half the columns each
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
     } else if (pl.mode == kFwdC8) {
         if ((rc = enc_im2col(&ta, x, s->n, s->h, s->w, 8, -g.ph, g.ph - (s->r - 1), -g.pw, g.pw - (s->s - 1), g.sh,

@@ -531,6 +531,28 @@ __device__ __forceinline__ void tma_load_3d_cg(void* dst, const void* tmap, uint
 }
 
 template <int CG>
+__device__ __forceinline__ void tma_load_4d_cg(void* dst, const void* tmap, uint32_t bar, int32_t c0, int32_t c1,
+                                               int32_t c2, int32_t c3)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5, %6}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "@E cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+            " [%0], [%1, {%3, %4, %5, %6}], [%2];\n\t}" ::"r"(smem_u32(dst)),
+            "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+            : "memory");
+}
+
+template <int CG>
 __device__ __forceinline__ void tma_load_im2col_4d_cg(void* dst, const void* tmap, uint32_t bar, int32_t c, int32_t w,
                                                       int32_t h, int32_t n, uint16_t off_w, uint16_t off_h)
 {
@@ -641,6 +663,37 @@ __device__ __forceinline__ void mma_bf16_x8_elect(uint32_t d0, uint32_t d1, uint
         "@E tcgen05.mma.cta_group::1.kind::f16 [%1], c, b, %7, T;\n\t}" ::"r"(d0),
         "r"(d1), "l"(a0), "l"(a1_off), "l"(a_step), "l"(b0), "l"(b_step), "r"(idesc), "r"(acc0)
         : "memory");
+}
+
+// mma_bf16_x8_elect for CG-CTA MMAs (CG = 2: M = 256 across the pair, issued by rank 0,
+// A and B halves at the same shared-memory addresses in both CTAs, as in mma_bf16_elect_cg).
+template <int CG>
+__device__ __forceinline__ void mma_bf16_x8_elect_cg(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
+                                                     uint64_t a_step, uint64_t b0, uint64_t b_step, uint32_t idesc,
+                                                     uint32_t acc0)
+{
+    if constexpr (CG == 2)
+        asm volatile(
+            "{\n\t.reg .pred E, P, T;\n\t.reg .b32 l;\n\t.reg .b64 a, c, b;\n\t"
+            "elect.sync l|E, 0xffffffff;\n\t"
+            "setp.ne.b32 P, %8, 0;\n\t"
+            "setp.eq.b32 T, 0, 0;\n\t"
+            "add.s64 c, %2, %3;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%0], %2, %5, %7, P;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%1], c, %5, %7, P;\n\t"
+            "add.s64 a, %2, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, %5, %6;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %7, T;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%1], c, b, %7, T;\n\t"
+            "add.s64 a, a, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, b, %6;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %7, T;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%1], c, b, %7, T;\n\t"
+            "add.s64 a, a, %4;\n\tadd.s64 c, c, %4;\n\tadd.s64 b, b, %6;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%0], a, b, %7, T;\n\t"
+            "@E tcgen05.mma.cta_group::2.kind::f16 [%1], c, b, %7, T;\n\t}" ::"r"(d0),
+            "r"(d1), "l"(a0), "l"(a1_off), "l"(a_step), "l"(b0), "l"(b_step), "r"(idesc), "r"(acc0)
+            : "memory");
+    else
+        mma_bf16_x8_elect(d0, d1, a0, a1_off, a_step, b0, b_step, idesc, acc0);
 }
 
 // Elected-lane commit: arrive once on the mbarrier at shared::cta offset bar
