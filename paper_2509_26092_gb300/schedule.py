@@ -15,9 +15,9 @@ own streams, each from its own pulled copy of the weights, so their steps
 overlap; the merges are serialised in push order by CUDA events.  The step times
 come from the calibrated time model (``time_model``: t = a*B + b, Eq. 2).
 
-``hybrid_schedule`` gives the paper's hybrid schemes (the training-configuration
-tables of Sec. 5 for CIFAR-100 and ImageNet: three stages of decreasing learning
-rate, each cycling through increasing resolutions), and ``run_schedule`` runs one
+``hybrid_schedule`` gives the paper's hybrid schemes (Table 7 for CIFAR-100 and
+Table 9 for ImageNet, Sec. 5.2: three stages of decreasing learning rate, each
+cycling through increasing resolutions), and ``run_schedule`` runs one
 on synthetic data for a fraction of each epoch; the synthetic source images have
 the schedule's largest resolution, so every sub-stage downsamples or passes them
 through.  The dropout rates of those tables are listed but not applied (the step
@@ -143,8 +143,8 @@ class SubStage:
 
 
 def hybrid_schedule(variant):
-    """The hybrid scheme's sub-stages (Sec. 5): CIFAR-100, 140 epochs at 24 and 32 px, or ImageNet,
-    105 epochs at 160, 224 and 288 px."""
+    """The hybrid scheme's sub-stages: Table 7 (CIFAR-100, 140 epochs at 24 and 32 px) or Table 9
+    (ImageNet, 105 epochs at 160, 224 and 288 px)."""
     if variant == "cifar":
         rows = [(1, 40, 0.2, 24, 600, 0.1), (1, 40, 0.2, 32, 560, 0.2), (2, 20, 0.02, 24, 600, 0.1),
                 (2, 20, 0.02, 32, 560, 0.2), (3, 10, 0.002, 24, 600, 0.1), (3, 10, 0.002, 32, 560, 0.2)]
