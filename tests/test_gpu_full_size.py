@@ -1,11 +1,14 @@
-"""Convolution passes at the full sizes the bench times: the 224 px layers of the
+"""The step's kernels at the full sizes the bench times: the 224 px layers of the
 ImageNet-shaped ResNet-18 at the large worker's batch of 512, through the same
-library calls and launch configurations as the training step (window kernels,
-the 128-column window tiles and the 256-column tiles on CTA pairs, phase-split
-stride-2 data gradients, split-K weight gradients).  The oracle computes sampled
-outputs one by one in fp64 from the same inputs; the corners of every output
-tensor are always among the samples.  Tolerance: max-norm relative 1e-2 over the
-samples."""
+library calls and launch configurations as the training step.
+
+Convolutions (window kernels, the 128-column window tiles and the 256-column tiles
+on CTA pairs, phase-split stride-2 data gradients, split-K weight gradients): the
+oracle computes sampled outputs one by one in fp64 from the same inputs, the corners
+of every output tensor always among them; tolerance max-norm relative 1e-2 over the
+samples.  A layer1 BatchNorm: the oracle over the whole tensor.  The stem's pool at
+batch 512: the fused forward equals the two-step path and the gradient equals the
+fp32 window-order gather, bit for bit."""
 import numpy as np
 import pytest
 import torch
@@ -81,3 +84,86 @@ def test_conv_passes_at_full_size(case):
     _check([dxh[i] for i in dg], [orc.conv2d_dgrad_at(dy64, w64, x64.shape, st, pad, *i) for i in dg], f"{case} dgrad")
     wg = _indices((k, r, r, c), g)
     _check([dwh[i] for i in wg], [orc.conv2d_wgrad_at(x64, dy64, w64.shape, st, pad, *i) for i in wg], f"{case} wgrad")
+
+
+def test_batchnorm_at_full_size():
+    """A layer1 BatchNorm with residual and ReLU at batch 512 (1.6 M rows x 64 channels), forward
+    and backward with two upstream gradients, against the oracle over the whole tensor."""
+    from conftest import max_norm_rel
+    D = load_dbl()
+    count, C = 512 * 56 * 56, 64
+    g = rng(2024)
+    y64, yd = _bf16((count, C), g, scale=2.0)
+    r64, rd = _bf16((count, C), g)
+    gamma = (1.0 + 0.2 * g.standard_normal(C)).astype(np.float32)
+    beta = (0.1 * g.standard_normal(C)).astype(np.float32)
+    gd, bd = torch.from_numpy(gamma).cuda(), torch.from_numpy(beta).cuda()
+    shape = D.bn_shape(count, C, 1e-5, True)
+    s1, s2 = torch.empty(C, device="cuda"), torch.empty(C, device="cuda")
+    D.dbl_bn_stats(shape, yd, s1, s2)
+    out = torch.empty_like(yd)
+    mean, istd = torch.empty(C, device="cuda"), torch.empty(C, device="cuda")
+    D.dbl_bn_relu_fused(shape, yd, s1, s2, gd, bd, rd, out, mean, istd)
+    do64, dod = _bf16((count, C), g)
+    do264, do2d = _bf16((count, C), g)
+    dy, dres = torch.empty_like(yd), torch.empty_like(yd)
+    dg, db = torch.empty(C, device="cuda"), torch.empty(C, device="cuda")
+    wsb = D.dbl_bn_workspace_bytes(shape)
+    D.dbl_bn_relu_fused_bwd(shape, dod, do2d, yd, out, gd, mean, istd, dy, dres, dg, db, ws(wsb), wsb)
+    torch.cuda.synchronize()
+    check_status(D)
+    ro, rm, ri = orc.bn_fwd(y64, gamma, beta, 1e-5, res=r64, relu=True)
+    assert max_norm_rel(out.double().cpu().numpy(), ro) <= TOL
+    np.testing.assert_allclose(mean.cpu().numpy(), rm, rtol=1e-5, atol=1e-5)
+    np.testing.assert_allclose(istd.cpu().numpy(), ri, rtol=1e-4)
+    rdy, rdg, rdb, rdres = orc.bn_bwd(do64, out.double().cpu().numpy(), y64, gamma, mean.double().cpu().numpy(),
+                                      istd.double().cpu().numpy(), relu=True, dout2=do264, want_dres=True)
+    assert max_norm_rel(dy.double().cpu().numpy(), rdy) <= TOL
+    assert max_norm_rel(dres.double().cpu().numpy(), rdres) <= TOL
+    assert max_norm_rel(dg.double().cpu().numpy(), rdg) <= 1e-4
+    assert max_norm_rel(db.double().cpu().numpy(), rdb) <= 1e-4
+
+
+def test_stem_pool_at_full_size():
+    """The stem's fused BatchNorm + ReLU + max pool at batch 512 (112 x 112 x 64) equals the
+    BatchNorm pass followed by the max pool bit for bit, and the pool gradient equals the fp32
+    window-order gather of the two upstream gradients."""
+    D = load_dbl()
+    n, H, C = 512, 112, 64
+    P = (H - 1) // 2 + 1
+    gen = torch.Generator(device="cuda").manual_seed(7)
+    x = (torch.randn((n, H, H, C), device="cuda", generator=gen) * 2.0 + 0.3).to(torch.bfloat16)
+    shape = D.bn_shape(n * H * H, C, 1e-5, True)
+    s1, s2 = torch.empty(C, device="cuda"), torch.empty(C, device="cuda")
+    D.dbl_bn_stats(shape, x, s1, s2)
+    gd = (1.0 + 0.2 * torch.randn(C, device="cuda", generator=gen)).float()
+    bd = (0.1 * torch.randn(C, device="cuda", generator=gen)).float()
+    m1, i1, m2, i2 = (torch.empty(C, device="cuda") for _ in range(4))
+    a = torch.empty_like(x)
+    D.dbl_bn_relu_fused(shape, x, s1, s2, gd, bd, None, a, m1, i1)
+    y1 = torch.empty((n, P, P, C), dtype=torch.bfloat16, device="cuda")
+    a1 = torch.empty((n, P, P, C), dtype=torch.uint8, device="cuda")
+    D.dbl_maxpool_fwd(n, H, H, C, a, y1, a1)
+    del a
+    y2, a2 = torch.empty_like(y1), torch.empty_like(a1)
+    D.dbl_bn_relu_maxpool_fwd(shape, n, H, H, x, s1, s2, gd, bd, m2, i2, y2, a2)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2) and torch.equal(a1, a2) and torch.equal(m1, m2) and torch.equal(i1, i2)
+    dp = torch.randn((n, P, P, C), device="cuda", generator=gen).to(torch.bfloat16)
+    dp2 = torch.randn((n, P, P, C), device="cuda", generator=gen).to(torch.bfloat16)
+    dx = torch.empty_like(x)
+    D.dbl_maxpool_bwd(n, H, H, C, dp, dp2, a2, dx)
+    torch.cuda.synchronize()
+    check_status(D)
+    f = torch.nn.functional.pad(dp.float() + dp2.float(), (0, 0, 0, 1, 0, 1))
+    am = torch.nn.functional.pad(a2.int(), (0, 0, 0, 1, 0, 1), value=255)
+    for dh in range(2):
+        for dw in range(2):
+            acc = torch.zeros((n, P, P, C), device="cuda")
+            for dpp in range(2):
+                for dq in range(2):
+                    r, s = dh - 2 * dpp + 1, dw - 2 * dq + 1
+                    if 0 <= r <= 2 and 0 <= s <= 2:
+                        win = (slice(None), slice(dpp, dpp + P), slice(dq, dq + P))
+                        acc = acc + torch.where(am[win] == 3 * r + s, f[win], torch.zeros_like(acc))
+            assert torch.equal(dx[:, dh::2, dw::2], acc.to(torch.bfloat16)), (dh, dw)
