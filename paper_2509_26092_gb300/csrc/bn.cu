@@ -16,8 +16,6 @@
 namespace {
 
 using dbl::dev::bn_scale_shift;
-using dbl::dev::colsum_fixed_order;
-using dbl::dev::kColsumGroups;
 
 constexpr int kThreads = 256;
 constexpr int kMaxC = 2048;

@@ -248,18 +248,8 @@ __device__ __forceinline__ void bn_scale_shift(float gamma, float beta, float me
     shift = __fsub_rn(beta, __fmul_rn(mean, scale));
 }
 
-// ---------------------------------------------------------------------------- fixed-order column sums
-// Column sums of a row-major fp32 matrix part[nrows][ld] for the 32 columns
-// col0 .. col0+31, by a block of 32 x kColsumGroups threads: thread (g, lane)
-// sums rows g, g + kColsumGroups, ... of column col0 + lane in fp32 with
-// Kahan compensation (16 loads in flight before the adds), then one thread
-// per column adds the groups 0..kColsumGroups-1 in order, in double.  (FP64
-// arithmetic is slow on this GPU, so only the last kColsumGroups adds use it.)
-// The order depends only on nrows, so the result is the same on every launch
-// and every GPU.  Returns the column sum in threads with g == 0 (other threads
-// return 0); every thread of the block must call it (it synchronises the block).
-constexpr int kColsumGroups = 32;
-
+// ---------------------------------------------------------------------------- per-block partial sums
+// sum += v with Kahan compensation (comp carries the lost low-order part)
 __device__ __forceinline__ void kahan_add(float& sum, float& comp, float v)
 {
     const float y = v - comp;
@@ -268,33 +258,6 @@ __device__ __forceinline__ void kahan_add(float& sum, float& comp, float v)
     sum = t;
 }
 
-__device__ __forceinline__ double colsum_fixed_order(const float* __restrict__ part, int nrows, int64_t ld,
-                                                     int col0, int ncols, double* red /* [kColsumGroups][32] */)
-{
-    const int lane = threadIdx.x % 32, g = threadIdx.x / 32;
-    const int col = col0 + lane;
-    float sum = 0.f, comp = 0.f;
-    if (col < ncols) {
-        int t = g;
-        for (; t + 15 * kColsumGroups < nrows; t += 16 * kColsumGroups) {
-            float v[16];
-#pragma unroll
-            for (int u = 0; u < 16; ++u) v[u] = __ldg(part + (int64_t)(t + u * kColsumGroups) * ld + col);
-#pragma unroll
-            for (int u = 0; u < 16; ++u) kahan_add(sum, comp, v[u]);
-        }
-        for (; t < nrows; t += kColsumGroups) kahan_add(sum, comp, __ldg(part + (int64_t)t * ld + col));
-    }
-    red[g * 32 + lane] = (double)sum - (double)comp;
-    __syncthreads();
-    double total = 0.0;
-    if (g == 0)
-        for (int k = 0; k < kColsumGroups; ++k) total += red[k * 32 + lane];
-    __syncthreads();
-    return total;
-}
-
-// ---------------------------------------------------------------------------- per-block partial sums
 // Fixed-order column sums of per-block partials part[nparts][2][K] (row p: the two
 // sums block p produced for every channel: a convolution epilogue's sum y and sum
 // y^2, or the BatchNorm backward's sum g and sum g*xhat).  Called once by all
@@ -403,29 +366,6 @@ __device__ __forceinline__ void tma_load_im2col_4d(void* dst, const void* tmap, 
 }
 
 // Elected-lane forms of the TMA loads above (whole warp calls, one lane issues).
-__device__ __forceinline__ void tma_load_2d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1)
-{
-    asm volatile(
-        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
-        "elect.sync l|E, 0xffffffff;\n\t"
-        "@E cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%3, %4}], [%2];\n\t}" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
-        : "memory");
-}
-
-__device__ __forceinline__ void tma_load_3d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1,
-                                                  int32_t c2)
-{
-    asm volatile(
-        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
-        "elect.sync l|E, 0xffffffff;\n\t"
-        "@E cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%3, %4, %5}], [%2];\n\t}" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
-        : "memory");
-}
-
 __device__ __forceinline__ void tma_load_4d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c0, int32_t c1,
                                                   int32_t c2, int32_t c3)
 {
@@ -435,20 +375,6 @@ __device__ __forceinline__ void tma_load_4d_elect(void* dst, const void* tmap, u
         "@E cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%3, %4, %5, %6}], [%2];\n\t}" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
-        : "memory");
-}
-
-__device__ __forceinline__ void tma_load_im2col_4d_elect(void* dst, const void* tmap, uint64_t* bar, int32_t c,
-                                                         int32_t w, int32_t h, int32_t n, uint16_t off_w,
-                                                         uint16_t off_h)
-{
-    asm volatile(
-        "{\n\t.reg .pred E;\n\t.reg .b32 l;\n\t"
-        "elect.sync l|E, 0xffffffff;\n\t"
-        "@E cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8};\n\t}" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w),
-        "h"(off_h)
         : "memory");
 }
 
