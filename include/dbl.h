@@ -96,6 +96,28 @@ enum { DBL_PASS_FWD = 0, DBL_PASS_DGRAD = 1, DBL_PASS_WGRAD = 2 };
 /* Bytes of scratch the given pass needs for this shape (0 if none).  Host. */
 DBL_API size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass);
 
+/* How a convolution pass runs on the current device, without launching it
+ * (host): the kernel (implicit GEMM, the 3x3 stride-1 window kernel, or the
+ * window weight gradient), output columns per tile, CTAs per MMA (2: a CTA
+ * pair with M = 256 MMAs across two SMs), tiles of the persistent loop, the
+ * split-K slices of a weight gradient or the phases of a stride-2 data
+ * gradient (else 1), the CTAs launched, and the window kernels' dynamic shared
+ * memory per CTA (0 for the implicit GEMM).  The pass functions make the same
+ * plan.  Errors: DBL_ERR_INVALID (null info, bad pass), and the shape errors of
+ * the pass functions. */
+enum { DBL_KERNEL_IGEMM = 0, DBL_KERNEL_WINDOW = 1, DBL_KERNEL_WINDOW_WGRAD = 2 };
+typedef struct {
+    int32_t kernel;
+    int32_t tile_cols;
+    int32_t ctas_per_mma;
+    int32_t tiles;
+    int32_t zdim;
+    int32_t grid;
+    int64_t smem_bytes;
+} dbl_conv_plan_info;
+
+DBL_API int dbl_conv_plan(const dbl_conv_shape* shape, int pass, dbl_conv_plan_info* info);
+
 /* Forward pass.  Writes y (bf16, rounded to nearest even from the fp32
  * accumulator).  If ch_sum/ch_sumsq are non-NULL, also writes the per-output-
  * channel sums of the stored (rounded) y and of its squares over all n*P*Q

@@ -2120,6 +2120,24 @@ size_t dbl_conv_workspace_bytes(const dbl_conv_shape* shape, int pass)
     return plan_ws(pl);
 }
 
+int dbl_conv_plan(const dbl_conv_shape* s, int pass, dbl_conv_plan_info* info)
+{
+    using namespace dbl;
+    if (!info || pass < 0 || pass > 2) return set_error(DBL_ERR_INVALID, "conv_plan: bad arguments");
+    Plan pl;
+    int rc = make_plan(s, pass, pl);
+    if (rc) return rc;
+    const bool wgwin = pl.win && pass == DBL_PASS_WGRAD;
+    info->kernel = wgwin ? DBL_KERNEL_WINDOW_WGRAD : pl.win ? DBL_KERNEL_WINDOW : DBL_KERNEL_IGEMM;
+    info->tile_cols = wgwin ? s->k : pl.BN;
+    info->ctas_per_mma = pl.cg;
+    info->tiles = pl.p.total_tiles;
+    info->zdim = pl.p.zdim;
+    info->grid = wgwin ? grid_size(pl.p.zdim) : plan_grid(pl);
+    info->smem_bytes = pl.win ? (int64_t)pl.smem : 0;
+    return DBL_OK;
+}
+
 int dbl_conv_fwd(const dbl_conv_shape* s, const void* x, const void* w, void* y, float* ch_sum, float* ch_sumsq,
                  void* ws, size_t ws_bytes, void* stream)
 {

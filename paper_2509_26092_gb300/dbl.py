@@ -27,6 +27,15 @@ class ConvShape(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int32) for f in ("n", "h", "w", "c", "k", "r", "s", "stride", "pad", "stride_w", "pad_w")]
 
 
+class ConvPlanInfo(ctypes.Structure):
+    _fields_ = [("kernel", ctypes.c_int32), ("tile_cols", ctypes.c_int32), ("ctas_per_mma", ctypes.c_int32),
+                ("tiles", ctypes.c_int32), ("zdim", ctypes.c_int32), ("grid", ctypes.c_int32),
+                ("smem_bytes", ctypes.c_int64)]
+
+
+DBL_KERNEL_IGEMM, DBL_KERNEL_WINDOW, DBL_KERNEL_WINDOW_WGRAD = 0, 1, 2
+
+
 class BnShape(ctypes.Structure):
     _fields_ = [("count", ctypes.c_int64), ("c", ctypes.c_int32), ("eps", ctypes.c_float), ("relu", ctypes.c_int32)]
 
@@ -62,6 +71,7 @@ def lib():
             "dbl_kernel_launches": (_I64, []),
             "dbl_device_status": (ctypes.c_int, [ctypes.POINTER(_I32)]),
             "dbl_conv_workspace_bytes": (_SZ, [ctypes.POINTER(ConvShape), ctypes.c_int]),
+            "dbl_conv_plan": (ctypes.c_int, [ctypes.POINTER(ConvShape), ctypes.c_int, ctypes.POINTER(ConvPlanInfo)]),
             "dbl_conv_fwd": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _V, _V, _SZ, _V]),
             "dbl_conv_dgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, _V, _SZ, _V]),
             "dbl_conv_wgrad": (ctypes.c_int, [ctypes.POINTER(ConvShape), _V, _V, _V, ctypes.c_int, _V, _SZ, _V]),
@@ -150,6 +160,13 @@ def conv_shape(n, h, w, c, k, r, stride, pad, s=None, stride_w=0, pad_w=0):
 
 def dbl_conv_workspace_bytes(shape, pass_):
     return lib().dbl_conv_workspace_bytes(ctypes.byref(shape), pass_)
+
+
+def dbl_conv_plan(shape, pass_):
+    """How the pass runs on the current device (host): a ConvPlanInfo."""
+    info = ConvPlanInfo()
+    _check(lib().dbl_conv_plan(ctypes.byref(shape), pass_, ctypes.byref(info)))
+    return info
 
 
 def dbl_conv_fwd(shape, x, w, y, ch_sum=None, ch_sumsq=None, ws=None, ws_bytes=0, stream=None):

@@ -117,3 +117,64 @@ def test_invalid_arguments_rejected_before_launch(D):
     b = D.BnShape(100, 12, 1e-5, 1)
     assert L.dbl_bn_relu_fused(ctypes.byref(b), 16, 16, 16, 16, 16, None, 16, 16, 16, None) == D.DBL_ERR_UNSUPPORTED
     assert "channel" in D.dbl_last_error()
+
+
+def _resnet18_convs(variant, batch, res):
+    """(n, h, w, c, k, r, stride, pad) of every non-stem convolution of ResNet-18."""
+    h = res // 4 if variant == "imagenet" else res  # after the ImageNet stem's stride 2 and max pool
+    out, cin = [], 64
+    for cout, st in ((64, 1), (128, 2), (256, 2), (512, 2)):
+        for b in range(2):
+            s = st if b == 0 else 1
+            ho = (h + 2 - 3) // s + 1
+            out.append((batch, h, h, cin, cout, 3, s, 1))
+            out.append((batch, ho, ho, cout, cout, 3, 1, 1))
+            if b == 0 and (s != 1 or cin != cout):
+                out.append((batch, h, h, cin, cout, 1, s, 0))
+            h, cin = ho, cout
+    return out
+
+
+def test_conv_plans_of_the_resnet18_layers(D):
+    """The host-side plan (dbl_conv_plan): which kernel each layer of the step uses, and the
+    invariants every plan keeps (grid within the workspace bound, even grids for CTA pairs,
+    window kernels within shared memory)."""
+    plan = lambda shp, p: D.dbl_conv_plan(D.conv_shape(*shp), p)
+    FWD, DG, WG = D.DBL_PASS_FWD, D.DBL_PASS_DGRAD, D.DBL_PASS_WGRAD
+    l1, l2, l3 = (512, 56, 56, 64, 64, 3, 1, 1), (512, 28, 28, 128, 128, 3, 1, 1), (512, 14, 14, 256, 256, 3, 1, 1)
+    for p in (FWD, DG):
+        i = plan(l1, p)
+        assert (i.kernel, i.tile_cols, i.ctas_per_mma) == (D.DBL_KERNEL_WINDOW, 64, 1)
+        i = plan(l2, p)
+        assert (i.kernel, i.tile_cols, i.ctas_per_mma) == (D.DBL_KERNEL_WINDOW, 128, 2)
+        i = plan(l3, p)
+        assert (i.kernel, i.tile_cols, i.ctas_per_mma) == (D.DBL_KERNEL_IGEMM, 256, 2)
+    assert plan(l1, WG).kernel == D.DBL_KERNEL_WINDOW_WGRAD
+    assert plan((512, 56, 56, 64, 128, 3, 2, 1), DG).zdim == 4  # stride-2 data gradient: four phases
+    for variant, batch, res in (("imagenet", 512, 224), ("imagenet", 128, 224), ("imagenet", 512, 160),
+                                ("imagenet", 512, 128), ("cifar", 256, 32), ("cifar", 1024, 16)):
+        for shp in _resnet18_convs(variant, batch, res):
+            for p in (FWD, DG, WG):
+                i = plan(shp, p)
+                assert 1 <= i.grid <= 256 and i.tiles >= 1 and i.zdim >= 1, (shp, p)
+                assert i.ctas_per_mma in (1, 2) and (i.ctas_per_mma == 1 or i.grid % 2 == 0), (shp, p)
+                if i.kernel == D.DBL_KERNEL_IGEMM:
+                    assert i.smem_bytes == 0
+                else:
+                    assert 0 < i.smem_bytes <= 232448 - 2048, (shp, p, i.smem_bytes)
+    with pytest.raises(Exception):
+        D.dbl_conv_plan(D.conv_shape(2, 8, 8, 24, 64, 3, 1, 1), FWD)  # 24 input channels: unsupported
+
+
+def test_cta_pairs_can_be_switched_off():
+    """DBL_CONV_CTA_PAIRS=0 plans every pass on single CTAs (read once per process)."""
+    import subprocess
+    import sys
+    code = ("from paper_2509_26092_gb300 import build_lib\nbuild_lib.build()\n"
+            "from paper_2509_26092_gb300 import dbl as D\n"
+            "for shp in ((512, 28, 28, 128, 128, 3, 1, 1), (512, 14, 14, 256, 256, 3, 1, 1)):\n"
+            "    for p in (0, 1, 2):\n"
+            "        assert D.dbl_conv_plan(D.conv_shape(*shp), p).ctas_per_mma == 1\n")
+    env = dict(os.environ, DBL_CONV_CTA_PAIRS="0")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
