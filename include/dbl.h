@@ -230,10 +230,15 @@ DBL_API int dbl_bn_relu_fused_bwd(const dbl_bn_shape* shape, const void* dout_bf
  * The scratch lives in one statically sized device array inside libdbl.so
  * (2.1 MB, held on every device that loads the library until the process
  * exits).  Limit: c <= DBL_BN_NOALLOC_MAX_C (512); larger c returns
- * DBL_ERR_UNSUPPORTED before anything is launched.  The first call on a
- * device looks up the array's device address (cudaGetSymbolAddress) with that
- * device current; make that first call before any stream capture.  No
- * device memory is allocated or freed by any call.  All calls share the one
+ * DBL_ERR_UNSUPPORTED before anything is launched.  The first call in a CUDA
+ * context looks up the array's device address (cudaGetSymbolAddress) with
+ * that context current and caches it under the context's unique ID; a context
+ * destroyed and created again (cudaDeviceReset) gets a new ID, so its first
+ * call looks the address up again.  That lookup may load the library's
+ * module, so it must not run inside a stream capture: a first call while the
+ * stream is capturing returns DBL_ERR_INVALID and launches nothing; make one
+ * call outside capture first.  No device memory is allocated or freed by any
+ * call.  All calls share the one
  * array, so calls whose kernels overlap on the GPU (two streams, two host
  * threads) race on it; serialise them.  Nothing in the array needs to start
  * at zero: each call writes every element it later reads. */

@@ -604,28 +604,47 @@ constexpr size_t kNoallocFloats =
 
 static __device__ __align__(256) float g_bn_noalloc_scratch[kNoallocFloats];
 
-// Device address of the array, looked up once per device with that device current.
-// (In host code the array's name is only a stand-in, never a device address.)
-float* noalloc_scratch(int* rc)
+// Device address of the array in the calling thread's current context.  It is
+// looked up (cudaGetSymbolAddress) the first time a context calls, and cached
+// under that context's unique ID: a context destroyed and created again
+// (cudaDeviceReset) loads the library's module again, the array may move, and
+// the new ID forces a fresh lookup.  A lookup may load the module, which must
+// not happen inside a stream capture, so a first call while `st` is capturing
+// is refused.  (In host code the array's name is only a stand-in, never a
+// device address.)
+float* noalloc_scratch(cudaStream_t st, int* rc)
 {
+    struct Entry {
+        unsigned long long ctx;
+        float* ptr;
+    };
     static std::mutex mu;
-    static float* ptr[64] = {nullptr};
-    int dev = 0;
-    if ((*rc = dbl::cuda_check(cudaGetDevice(&dev), "bn_bwd_noalloc: cudaGetDevice"))) return nullptr;
-    if (dev < 0 || dev >= 64) {
-        *rc = dbl::set_error(DBL_ERR_UNSUPPORTED, "bn_bwd_noalloc: device index %d out of range", dev);
+    static Entry cache[64] = {};
+    static int used = 0;
+    unsigned long long ctx = 0;
+    if ((*rc = dbl::current_context_id(&ctx))) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; ctx && i < used; ++i)
+        if (cache[i].ctx == ctx) {
+            *rc = DBL_OK;
+            return cache[i].ptr;
+        }
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(st, &cs);
+    if (e != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+        (void)cudaGetLastError();
+        *rc = dbl::set_error(DBL_ERR_INVALID,
+                             "bn_bwd_noalloc: the first call in a CUDA context looks up the static scratch and "
+                             "must come before any stream capture; call it once outside capture first");
         return nullptr;
     }
-    std::lock_guard<std::mutex> lock(mu);
-    if (!ptr[dev]) {
-        void* p = nullptr;
-        if ((*rc = dbl::cuda_check(cudaGetSymbolAddress(&p, g_bn_noalloc_scratch),
-                                   "bn_bwd_noalloc: cudaGetSymbolAddress")))
-            return nullptr;
-        ptr[dev] = static_cast<float*>(p);
-    }
+    void* p = nullptr;
+    if ((*rc = dbl::cuda_check(cudaGetSymbolAddress(&p, g_bn_noalloc_scratch), "bn_bwd_noalloc: cudaGetSymbolAddress")))
+        return nullptr;
+    if (!ctx && (*rc = dbl::current_context_id(&ctx))) return nullptr;  // the lookup made the context current
+    if (ctx && used < 64) cache[used++] = Entry{ctx, static_cast<float*>(p)};  // beyond 64 contexts: no cache
     *rc = DBL_OK;
-    return ptr[dev];
+    return static_cast<float*>(p);
 }
 
 }  // namespace
@@ -652,10 +671,10 @@ extern "C" int dbl_bn_relu_fused_bwd_noalloc(const dbl_bn_shape* s, const void* 
     const int64_t nblk = bwd_blocks(s->count, s->c);
     if (nblk > kNoallocMaxBlocks || (size_t)nblk * 2 * C + 3 * (size_t)C > kNoallocFloats)
         return set_error(DBL_ERR_UNSUPPORTED, "bn_relu_fused_bwd_noalloc: shape exceeds the static scratch");
-    float* partial = noalloc_scratch(&rc);
+    cudaStream_t st = as_stream(stream);
+    float* partial = noalloc_scratch(st, &rc);
     if (rc) return rc;
     float* coef = partial + nblk * 2 * C;  // written by the finalize kernel before the apply kernel reads it
-    cudaStream_t st = as_stream(stream);
     return bwd_launch(s, dout, dout2, y, out, gamma, beta, save_mean, save_invstd, dy, dresidual, dgamma, dbeta,
                       partial, coef, nblk, st);
 }

@@ -1766,9 +1766,13 @@ template <int BN, int FAM>
 int resident_pairs()
 {
     static int cached[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        dev = -1;
+    }
     if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+    bool queried = false;  // only a plan the device itself answered for is cached
     int pairs = std::min(dbl::sm_count() / 2, kMaxGrid / 2);
     if (set_igemm_smem<BN, FAM, 2>() == DBL_OK) {
         cudaLaunchConfig_t cfg = {};
@@ -1784,12 +1788,15 @@ int resident_pairs()
         cfg.numAttrs = 1;
         int n = 0;
         if (cudaOccupancyMaxActiveClusters(&n, conv_igemm_kernel<BN, FAM, 2>, &cfg) == cudaSuccess && n > 0)
+        {
             pairs = std::min(pairs, n);
-        else
+            queried = true;
+        } else {
             (void)cudaGetLastError();
+        }
     }
     if (pairs < 1) pairs = 1;
-    if (dev >= 0 && dev < 64) cached[dev] = pairs;
+    if (queried && dev >= 0 && dev < 64) cached[dev] = pairs;
     return pairs;
 }
 
@@ -1882,9 +1889,13 @@ template <int BN, bool DG, bool RES>
 int resident_win_pairs(size_t smem)
 {
     static int cached[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        dev = -1;
+    }
     if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+    bool queried = false;  // only a plan the device itself answered for is cached
     int pairs = std::min(dbl::sm_count() / 2, kMaxGrid / 2);
     if (set_win_smem<BN, DG, RES, 2>() == DBL_OK) {
         cudaLaunchConfig_t cfg = {};
@@ -1900,12 +1911,15 @@ int resident_win_pairs(size_t smem)
         cfg.numAttrs = 1;
         int n = 0;
         if (cudaOccupancyMaxActiveClusters(&n, conv_win_kernel<BN, DG, RES, 2>, &cfg) == cudaSuccess && n > 0)
+        {
             pairs = std::min(pairs, n);
-        else
+            queried = true;
+        } else {
             (void)cudaGetLastError();
+        }
     }
     if (pairs < 1) pairs = 1;
-    if (dev >= 0 && dev < 64) cached[dev] = pairs;
+    if (queried && dev >= 0 && dev < 64) cached[dev] = pairs;
     return pairs;
 }
 

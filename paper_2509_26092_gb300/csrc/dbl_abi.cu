@@ -33,7 +33,10 @@ int sm_count()
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
     if (dev < 64 && cached[dev]) return cached[dev];
     int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+        (void)cudaGetLastError();
+        return 148;  // no device answered: a nominal count, never cached
+    }
     if (dev < 64) cached[dev] = n;
     return n;
 }
@@ -62,6 +65,26 @@ PFN_encodeIm2col encode_im2col()
     static PFN_encodeIm2col fn = nullptr;
     std::call_once(once, [] { fn = reinterpret_cast<PFN_encodeIm2col>(driver_entry("cuTensorMapEncodeIm2col")); });
     return fn;
+}
+
+int current_context_id(unsigned long long* id)
+{
+    typedef CUresult (*PFN_ctxGetCurrent)(CUcontext*);
+    typedef CUresult (*PFN_ctxGetId)(CUcontext, unsigned long long*);
+    static std::once_flag once;
+    static PFN_ctxGetCurrent get_current = nullptr;
+    static PFN_ctxGetId get_id = nullptr;
+    std::call_once(once, [] {
+        get_current = reinterpret_cast<PFN_ctxGetCurrent>(driver_entry("cuCtxGetCurrent"));
+        get_id = reinterpret_cast<PFN_ctxGetId>(driver_entry("cuCtxGetId"));
+    });
+    *id = 0;
+    if (!get_current || !get_id) return set_error(DBL_ERR_CUDA, "driver entry points cuCtxGetCurrent/cuCtxGetId missing");
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS) return set_error(DBL_ERR_CUDA, "cuCtxGetCurrent failed");
+    if (!ctx) return DBL_OK;
+    if (get_id(ctx, id) != CUDA_SUCCESS) return set_error(DBL_ERR_CUDA, "cuCtxGetId failed");
+    return DBL_OK;
 }
 
 }  // namespace dbl

@@ -49,6 +49,10 @@ typedef CUresult (*PFN_encodeIm2col)(CUtensorMap*, CUtensorMapDataType, cuuint32
                                      CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 PFN_encodeTiled encode_tiled();
 PFN_encodeIm2col encode_im2col();
+// Unique ID of the calling thread's current CUDA context (cuCtxGetId), 0 if no
+// context is current yet.  IDs are never reused within a process, so a context
+// destroyed and created again (cudaDeviceReset) gets a new one.
+int current_context_id(unsigned long long* id);
 
 // BatchNorm forward finalize (bn.cu): channel sums over count rows -> saved mean and
 // 1/sqrt(var + eps), once per channel in fp64.  Launches on st; returns a status.

@@ -138,7 +138,10 @@ def _resnet18_convs(variant, batch, res):
 def test_conv_plans_of_the_resnet18_layers(D):
     """The host-side plan (dbl_conv_plan): which kernel each layer of the step uses, and the
     invariants every plan keeps (grid within the workspace bound, even grids for CTA pairs,
-    window kernels within shared memory)."""
+    window kernels within shared memory).  Without a GPU the grid and tile counts come from a
+    nominal SM count (never cached), so on a CPU host this pins only the choices that do not
+    depend on the device: kernel, tile width, CTAs per MMA and phase count; the invariants hold
+    for any SM count."""
     plan = lambda shp, p: D.dbl_conv_plan(D.conv_shape(*shp), p)
     FWD, DG, WG = D.DBL_PASS_FWD, D.DBL_PASS_DGRAD, D.DBL_PASS_WGRAD
     l1, l2, l3 = (512, 56, 56, 64, 64, 3, 1, 1), (512, 28, 28, 128, 128, 3, 1, 1), (512, 14, 14, 256, 256, 3, 1, 1)

@@ -9,7 +9,7 @@ with respect to storage rounding (ReLU masks flip and BatchNorm backward
 subtracts nearly equal terms), so the oracle's own bf16-storage gradients
 differ from its fp64 gradients by about 30% (median over tensors).  With
 spread = |oracle_bf16 - oracle_fp64| per tensor (max norm), the GPU's error
-|gpu - oracle_bf16| must be at most max(3 * spread, 1e-2 * |oracle_bf16|) for
+|gpu - oracle_bf16| must be at most max(2 * spread, 1e-2 * |oracle_bf16|) for
 every tensor, and its median ratio to the spread over all tensors at most 1:
 the GPU is no further from the oracle than the oracle's own rounding moves it.  Each layer on its own is held to 1e-2 at the same shapes in
 test_gpu_step_layers.py.  The merge is compared on the GPU's own pushed
@@ -45,7 +45,7 @@ def _compare_grads(spec, grad_flat, ref_bf16, ref_f64, tag=""):
         scale = float(np.max(np.abs(g))) or 1.0
         err = float(np.max(np.abs(got[name] - g))) / scale
         spread = float(np.max(np.abs(ref_f64[name] - g))) / scale
-        rows.append((name, err, spread, max(3.0 * spread, TOL)))
+        rows.append((name, err, spread, max(2.0 * spread, TOL)))
     ratio = [r[1] / max(r[2], 1e-12) for r in rows]
     print(f"\n{tag}: median gpu-vs-oracle {np.median([r[1] for r in rows]):.2e}, median bf16-vs-fp64 spread "
           f"{np.median([r[2] for r in rows]):.2e}, median ratio {np.median(ratio):.2f}, max ratio {max(ratio):.2f}")
@@ -116,7 +116,7 @@ def test_dual_batch_iteration_matches_oracle(R):
         d_ref, d64 = nw[name] - p64[name], nw64[name] - p64[name]
         scale = float(np.max(np.abs(d_ref))) or 1.0
         spread = float(np.max(np.abs(d64 - d_ref))) / scale
-        assert float(np.max(np.abs(got_w[name] - p64[name] - d_ref))) / scale <= max(3 * spread, TOL), name
+        assert float(np.max(np.abs(got_w[name] - p64[name] - d_ref))) / scale <= max(2 * spread, TOL), name
 
 
 def test_graph_replay_equals_eager(R):
