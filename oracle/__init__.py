@@ -51,6 +51,13 @@ def lib():
         L.orc_softmax_ce.argtypes = [_D, _I32, _i, _i, _D]
         L.orc_softmax_ce.restype = _d
         L.orc_ps_merge.argtypes = [_D, _D, _D, _D, _i64, _d, _d, _d, _d, _i]
+        _U64 = ctypes.POINTER(ctypes.c_uint64)
+        L.orc_philox4x64_10.argtypes = [_U64, _U64, _U64]
+        L.orc_philox4x64_10.restype = None
+        L.orc_dropout_mask.argtypes = [_i, _i, _d, ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(ctypes.c_uint8)]
+        L.orc_dropout_mask.restype = None
+        L.orc_dropout_apply.argtypes = [_D, ctypes.POINTER(ctypes.c_uint8), _i64, _d, _D]
+        L.orc_dropout_apply.restype = None
         L.orc_resize_taps.argtypes = [_i, _i, _I32, _I32, _D]
         L.orc_resize_taps.restype = _i
         L.orc_bilinear_resize.argtypes = [_D, _i, _i, _i, _i, _D, _i, _i]
@@ -195,6 +202,33 @@ def avgpool_bwd(df, x_shape):
     dx = np.empty((N, H, W, C))
     lib().orc_avgpool_bwd(_p(df), N, H * W, C, _p(dx))
     return dx
+
+
+def philox4x64_10(counter, key):
+    """Philox4x64-10 of a 4-word counter and 2-word key (uint64 words) -> 4 uint64 words."""
+    c = np.ascontiguousarray(counter, dtype=np.uint64)
+    k = np.ascontiguousarray(key, dtype=np.uint64)
+    out = np.empty(4, dtype=np.uint64)
+    U = ctypes.POINTER(ctypes.c_uint64)
+    lib().orc_philox4x64_10(c.ctypes.data_as(U), k.ctypes.data_as(U), out.ctypes.data_as(U))
+    return out
+
+
+def dropout_mask(N, C, d, seed, step):
+    """keep [N, C] uint8 (1 = kept) of the dropout before the FC layer (see dbl_oracle.c)."""
+    keep = np.empty((N, C), dtype=np.uint8)
+    lib().orc_dropout_mask(N, C, float(d), int(seed), int(step), keep.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
+    return keep
+
+
+def dropout_apply(x, keep, d):
+    """keep * x / (1 - d), elementwise (forward of the features, backward of their gradient)."""
+    x = _f64(x)
+    keep = np.ascontiguousarray(keep, dtype=np.uint8)
+    assert keep.shape == x.shape
+    out = np.empty_like(x)
+    lib().orc_dropout_apply(_p(x), keep.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)), x.size, float(d), _p(out))
+    return out
 
 
 def fc_fwd(f, Wt, b):

@@ -397,6 +397,82 @@ double orc_softmax_ce(const double* logits, const int32_t* labels, int N, int J,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Dropout before the fully connected layer.  Cyclic progressive learning   */
+/* raises the dropout rate d with the resolution inside each stage          */
+/* (Sec. 4.1; Tables 7 and 9 give 0.1 / 0.2 / 0.3).  The paper gives no     */
+/* formula; the reading is inverted dropout on the pooled features, as in   */
+/* the framework it used: each feature is kept with probability 1 - d and */
+/* a kept feature is divided by 1 - d, so its expectation is unchanged.     */
+/*                                                                          */
+/* The random draw is the counter-based generator Philox4x64-10 (Salmon,    */
+/* Moraes, Dror and Shaw, "Parallel random numbers: as easy as 1, 2, 3",    */
+/* SC 2011), written from that definition: a 256-bit counter and a 128-bit  */
+/* key, ten rounds, each multiplying counter words 0 and 2 by the two round */
+/* multipliers (full 128-bit products), then                                */
+/*     (c0, c1, c2, c3) <- (hi(M1*c2) ^ c1 ^ k0, lo(M1*c2),                 */
+/*                          hi(M0*c0) ^ c3 ^ k1, lo(M0*c0)),                */
+/* with the key advanced by the two Weyl constants between rounds.          */
+/* ------------------------------------------------------------------------ */
+static void mul_hilo64(uint64_t a, uint64_t b, uint64_t* hi, uint64_t* lo)
+{
+    /* schoolbook product of 32-bit halves */
+    const uint64_t a0 = a & 0xffffffffu, a1 = a >> 32, b0 = b & 0xffffffffu, b1 = b >> 32;
+    const uint64_t p00 = a0 * b0, p01 = a0 * b1, p10 = a1 * b0, p11 = a1 * b1;
+    const uint64_t mid = (p00 >> 32) + (p01 & 0xffffffffu) + (p10 & 0xffffffffu);
+    *lo = (mid << 32) | (p00 & 0xffffffffu);
+    *hi = p11 + (p01 >> 32) + (p10 >> 32) + (mid >> 32);
+}
+
+void orc_philox4x64_10(const uint64_t ctr[4], const uint64_t key[2], uint64_t out[4])
+{
+    const uint64_t M0 = 0xD2E7470EE14C6C93ull, M1 = 0xCA5A826395121157ull;
+    const uint64_t W0 = 0x9E3779B97F4A7C15ull, W1 = 0xBB67AE8584CAA73Bull;
+    uint64_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3], k0 = key[0], k1 = key[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) {
+            k0 += W0;
+            k1 += W1;
+        }
+        uint64_t hi0, lo0, hi1, lo1;
+        mul_hilo64(M0, c0, &hi0, &lo0);
+        mul_hilo64(M1, c2, &hi1, &lo1);
+        const uint64_t n0 = hi1 ^ c1 ^ k0, n1 = lo1, n2 = hi0 ^ c3 ^ k1, n3 = lo0;
+        c0 = n0;
+        c1 = n1;
+        c2 = n2;
+        c3 = n3;
+    }
+    out[0] = c0;
+    out[1] = c1;
+    out[2] = c2;
+    out[3] = c3;
+}
+
+/* keep[n,c] for N samples of C features (C a multiple of 4): feature c of   */
+/* sample n takes word c % 4 of Philox4x64-10 at counter                     */
+/* (n*C/4 + c/4, step, 0, 0) with key (seed, 0), and is kept when the word's */
+/* upper 32 bits, as an integer, are at least floor(d * 2^32).               */
+void orc_dropout_mask(int N, int C, double d, uint64_t seed, uint64_t step, uint8_t* keep)
+{
+    const uint64_t thr = (uint64_t)floor(d * 4294967296.0);
+    const uint64_t key[2] = {seed, 0};
+    for (int n = 0; n < N; ++n)
+        for (int g = 0; g < C / 4; ++g) {
+            const uint64_t ctr[4] = {(uint64_t)n * (uint64_t)(C / 4) + (uint64_t)g, step, 0, 0};
+            uint64_t r[4];
+            orc_philox4x64_10(ctr, key, r);
+            for (int j = 0; j < 4; ++j) keep[(int64_t)n * C + 4 * g + j] = (uint8_t)((r[j] >> 32) >= thr);
+        }
+}
+
+/* out = keep * x / (1 - d): the forward map, and (it is linear and          */
+/* diagonal) also the backward map of a gradient.                           */
+void orc_dropout_apply(const double* x, const uint8_t* keep, int64_t n, double d, double* out)
+{
+    for (int64_t i = 0; i < n; ++i) out[i] = keep[i] ? x[i] / (1.0 - d) : 0.0;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Parameter-server merge of the two workers' pushes (Sec. 3.4 with Eq. 1). */
 /* Each push i carries its worker's batch-mean gradient g_i and is scaled by */
 /* the model-update factor f_i (f_L = 1, f_S = d_S/d_L or its square root).  */

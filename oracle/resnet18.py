@@ -34,7 +34,7 @@ import math
 import numpy as np
 
 from . import (avgpool_bwd, avgpool_fwd, bilinear_resize, bn_bwd, bn_fwd, conv2d_dgrad, conv2d_fwd, conv2d_wgrad,
-               fc_bwd, fc_fwd, maxpool_bwd, maxpool_fwd, ps_merge, round_bf16, softmax_ce)
+               dropout_apply, dropout_mask, fc_bwd, fc_fwd, maxpool_bwd, maxpool_fwd, ps_merge, round_bf16, softmax_ce)
 
 WIDTHS = (64, 128, 256, 512)
 
@@ -95,11 +95,13 @@ def _check_params(params, variant, classes, widths):
             raise ValueError(f"{name}: shape {params[name].shape} != {shape}")
 
 
-def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths=WIDTHS, keep=False):
+def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths=WIDTHS, keep=False, dropout=None):
     """One worker's forward + backward on a batch.
 
     params: dict name -> fp32-valued array (the master weights the worker pulled);
     img: [N, H, W, 3] float, already at the training resolution; labels: [N] int.
+    dropout: None, or (d, seed, step): dropout of rate d on the pooled features before
+    the FC layer (Sec. 4.1), with the mask of ``dropout_mask(N, C, d, seed, step)``.
     Returns dict(loss=float, grads={name: array}, acts={...} if keep).
     """
     classes = params["fc.w"].shape[0]
@@ -153,11 +155,17 @@ def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths
             blocks.append(blk)
             c_in = wdt
     feat = avgpool_fwd(cur)
+    mask = None
+    if dropout is not None and dropout[0] > 0.0:
+        mask = dropout_mask(feat.shape[0], feat.shape[1], dropout[0], dropout[1], dropout[2])
+        feat = dropout_apply(feat, mask, dropout[0])
     logits = fc_fwd(feat, P["fc.w"], P["fc.b"])
     loss, dl = softmax_ce(logits, labels)
 
     grads = {}
     grads["fc.w"], grads["fc.b"], dfeat = fc_bwd(dl, feat, P["fc.w"])
+    if mask is not None:
+        dfeat = dropout_apply(dfeat, mask, dropout[0])
     dout = R(avgpool_bwd(dfeat, cur.shape))
     dout2 = None
     for blk in reversed(blocks):
@@ -197,28 +205,31 @@ def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths
     grads["conv1.w"] = conv2d_wgrad(x0, dys, wq["conv1.w"].shape, stem["stride"], stem["pad"])
     res = dict(loss=loss, grads=grads, logits=logits)
     if keep:
-        res["acts"] = dict(stem=stem, blocks=blocks, feat=feat, dlogits=dl)
+        res["acts"] = dict(stem=stem, blocks=blocks, feat=feat, dlogits=dl, dropout_keep=mask)
     return res
 
 
 def dual_batch_iteration(params, velocity, img_large, labels_large, img_small, labels_small, resolution, variant,
-                         lr, momentum, f_large, f_small, order=0, bf16_storage=True, widths=WIDTHS):
+                         lr, momentum, f_large, f_small, order=0, bf16_storage=True, widths=WIDTHS,
+                         dropout_large=None, dropout_small=None):
     """One emulated parameter-server iteration of the hybrid scheme (Sec. 3-4).
 
     Both workers pull the same model version, resize their images to the
     sub-stage resolution (Sec. 4.1), run one training step each, and the server
     applies their pushes with the model-update factors (Sec. 3.4).
+    dropout_large / dropout_small: each worker's (d, seed, step) for ``train_step``, or None.
     Returns (new_params, new_velocity, loss_large, loss_small, grads_large, grads_small).
     """
     out = {}
-    for tag, img, lab in (("L", img_large, labels_large), ("S", img_small, labels_small)):
+    for tag, img, lab, drop in (("L", img_large, labels_large, dropout_large),
+                                ("S", img_small, labels_small, dropout_small)):
         if img is None:
             out[tag] = None
             continue
         x = np.asarray(img, dtype=np.float64)
         if x.shape[1] != resolution or x.shape[2] != resolution:
             x = bilinear_resize(x, resolution, resolution)
-        out[tag] = train_step(params, x, lab, variant, bf16_storage=bf16_storage, widths=widths)
+        out[tag] = train_step(params, x, lab, variant, bf16_storage=bf16_storage, widths=widths, dropout=drop)
     new_w, new_u = {}, {}
     for name in params:
         gl = out["L"]["grads"][name] if out["L"] else None
