@@ -32,20 +32,29 @@ if ROOT not in sys.path:
 METRIC = "ResNet-18 train-step images/s per resolution; conv TFLOP/s vs bf16 peak"
 
 CONFIGS = {
-    # variant, classes, native resolution, sub-stage resolutions, large / small batch per stage
+    # variant, classes, native resolution, sub-stage resolutions, large / small batch per stage, and the
+    # rate of the dropout before the FC layer per stage (Sec. 4.1: it rises with the resolution of the
+    # sub-stage, 0.1 / 0.2 / 0.3 in Tables 7 and 9)
     "imagenet_hybrid": dict(variant="imagenet", classes=1000, native=224, stages=(128, 160, 224),
-                            large=(512, 512, 512), small=(128, 128, 128),
+                            large=(512, 512, 512), small=(128, 128, 128), dropout=(0.1, 0.2, 0.3),
                             desc="ImageNet-shaped ResNet-18 hybrid: 224 px images resized to 128/160/224, "
                                  "large worker 512 + small worker 128 on two streams, PS merge each iteration"),
+    "imagenet_paper": dict(variant="imagenet", classes=1000, native=288, stages=(160, 224, 288),
+                           large=(2330, 1110, 740), small=(582, 277, 185), dropout=(0.1, 0.2, 0.3),
+                           desc="the paper's ImageNet hybrid sub-stages (Table 9): 288 px images resized to "
+                                "160/224/288, large-batch worker 2330/1110/740 and a small-batch worker of a "
+                                "quarter of that on two streams, PS merge each iteration"),
     "cifar_hybrid": dict(variant="cifar", classes=100, native=32, stages=(16, 24, 32), large=(1024, 512, 256),
-                         small=(256, 128, 64),
+                         small=(256, 128, 64), dropout=(0.1, 0.1, 0.2),
                          desc="CIFAR-shaped ResNet-18 cyclic progressive sweep 16/24/32 px, dual batch, PS merge"),
     "cifar_step": dict(variant="cifar", classes=100, native=32, stages=(32,), large=(256,), small=(None,),
+                       dropout=(0.2,),
                        desc="CIFAR-shaped ResNet-18, one train step at 32x32, batch 256, single push"),
     "imagenet_step": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(256,), small=(None,),
+                          dropout=(0.2,),
                           desc="ImageNet-shaped ResNet-18, one train step at 224x224, batch 256, single push"),
     "imagenet_small": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(32,), small=(8,),
-                           desc="small ImageNet-shaped dual-batch iteration for profiling"),
+                           dropout=(0.2,), desc="small ImageNet-shaped dual-batch iteration for profiling"),
 }
 DEFAULT_CONFIG = "imagenet_hybrid"
 F_SMALL = 19.0 / 21.0  # d_S/d_L for one large and one small worker at k = 1.05 (Eqs. 4-6)
@@ -164,11 +173,17 @@ def _oracle_setup(cfg):
 
 def _oracle_iteration(cfg, st, res):
     """One dual-batch iteration of the fp64 oracle at resolution res: large batch 2, small batch 1."""
+    import numpy as np
+
     from oracle import resnet18 as OR
+    d = float(np.float32(cfg["dropout"][list(cfg["stages"]).index(res)]))
+    st["step"] = st.get("step", -1) + 1
     t0 = time.perf_counter()
     st["params"], st["vel"], *_ = OR.dual_batch_iteration(st["params"], st["vel"], st["img"][:2], st["lab"][:2],
                                                           st["img"][2:], st["lab"][2:], res, cfg["variant"], LR,
-                                                          MOMENTUM, 1.0, F_SMALL, order=0)
+                                                          MOMENTUM, 1.0, F_SMALL, order=0,
+                                                          dropout_large=(d, 2 * res + 1, st["step"]),
+                                                          dropout_small=(d, 2 * res + 2, st["step"]))
     return 3, time.perf_counter() - t0
 
 
@@ -236,9 +251,9 @@ def build_pipeline(cfg, device):
     lab_l = torch.from_numpy(synth.labels(bl_max, cfg["classes"], seed=1, name="large")).pin_memory()
     lab_s = torch.from_numpy(synth.labels(bs_max, cfg["classes"], seed=1, name="small")).pin_memory() if bs_max else None
     stages = []
-    for res, bl, bs in zip(cfg["stages"], cfg["large"], cfg["small"]):
-        large = R.Worker(spec, bl, res, device)
-        small = R.Worker(spec, bs, res, device) if bs else None
+    for res, bl, bs, drop in zip(cfg["stages"], cfg["large"], cfg["small"], cfg["dropout"]):
+        large = R.Worker(spec, bl, res, device, dropout=drop, dropout_seed=2 * res + 1)
+        small = R.Worker(spec, bs, res, device, dropout=drop, dropout_seed=2 * res + 2) if bs else None
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_large=1.0, f_small=F_SMALL)
         it.set_inputs(host_l[:bl].to(device), lab_l[:bl].to(device),
                       host_s[:bs].to(device) if bs else None, lab_s[:bs].to(device) if bs else None)
@@ -358,11 +373,11 @@ def run_profile_iteration(args, cfg):
     server = R.ServerState(spec, synth.params(spec.table(), seed=0))
     nat = cfg["native"]
     n0 = D.dbl_kernel_launches()
-    for res, bl, bs in zip(cfg["stages"], cfg["large"], cfg["small"]):
+    for res, bl, bs, drop in zip(cfg["stages"], cfg["large"], cfg["small"], cfg["dropout"]):
         if args.profile_res and res != args.profile_res:
             continue
-        large = R.Worker(spec, bl, res)
-        small = R.Worker(spec, bs, res) if bs else None
+        large = R.Worker(spec, bl, res, dropout=drop, dropout_seed=2 * res + 1)
+        small = R.Worker(spec, bs, res, dropout=drop, dropout_seed=2 * res + 2) if bs else None
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_small=F_SMALL)
         it.set_inputs(torch.from_numpy(synth.images_u8(bl, nat, nat, 3, seed=1)).cuda(),
                       torch.from_numpy(synth.labels(bl, cfg["classes"], seed=1)).cuda(),
@@ -577,7 +592,8 @@ def run_ours(args, cfg):
                 "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
                 "config": {"workload": args.config, "description": cfg["desc"],
                            "stages_px": list(cfg["stages"]), "large_batch": list(cfg["large"]),
-                           "small_batch": list(cfg["small"]), "images_per_step": images_per_step,
+                           "small_batch": list(cfg["small"]), "dropout": list(cfg["dropout"]),
+                           "images_per_step": images_per_step,
                            "params": pipe["spec"].n_params(), "f_small": F_SMALL, "lr": LR, "momentum": MOMENTUM,
                            "l2": "working set (activations, several GB) larger than L2; no explicit flush",
                            "input": f"uint8 images {cfg['native']}x{cfg['native']}x3 from pinned host memory, "

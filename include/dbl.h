@@ -292,6 +292,34 @@ DBL_API int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, 
                      const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx_bf16,
                      void* ws, size_t ws_bytes, void* stream);
 
+/* Head with dropout of the pooled features before the FC layer.  Cyclic
+ * progressive learning raises the dropout rate d with the resolution of each
+ * sub-stage (Sec. 4.1; 0.1 / 0.2 / 0.3 in Tables 7 and 9).  Inverted dropout:
+ *   featd[n,c] = feat[n,c] * keep[n,c] / (1 - d),
+ * logits, loss, dfc_w, dfc_b as dbl_head_fwd_bwd with featd in place of feat,
+ * and dx[n,i,c] = (dlogits*fc_w)[n,c] * keep[n,c] / (1 - d) / hw.
+ * keep[n,c] is the mask dbl_dropout_mask writes for the same (d, seed, *step)
+ * (a counter-based draw, so the mask depends on nothing else).  step: device
+ * pointer to one uint64 (8-byte aligned) read by the kernels; after the call's
+ * last kernel it is incremented by one on the stream, so consecutive calls
+ * (and replays of a captured graph) draw fresh masks.  drop_rate = 0 is
+ * dbl_head_fwd_bwd exactly (step may then be NULL and is not touched).
+ * drop_rate outside [0, 1): DBL_ERR_INVALID.  Workspace as dbl_head_fwd_bwd. */
+DBL_API int dbl_head_fwd_bwd_dropout(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x_bf16,
+                                     const float* fc_w, const float* fc_b, const int32_t* labels, float drop_rate,
+                                     uint64_t seed, uint64_t* step, float* loss, float* dfc_w, float* dfc_b,
+                                     void* dx_bf16, void* ws, size_t ws_bytes, void* stream);
+
+/* The dropout mask of dbl_head_fwd_bwd_dropout: keep[n,c] (uint8, 1 = kept)
+ * for n samples of c features (c a multiple of 4; keep 4-byte aligned).
+ * Feature c of sample n takes word c % 4 of the Philox4x64-10 block (Salmon
+ * et al., SC 2011) at counter (n*c/4 + c/4, *step, 0, 0) with key (seed, 0),
+ * and is kept when the word's upper 32 bits are at least
+ * floor(drop_rate * 2^32) (an integer comparison, so the mask is exact).
+ * step is read on the device and not changed.  drop_rate = 0 keeps all. */
+DBL_API int dbl_dropout_mask(int32_t n, int32_t c, float drop_rate, uint64_t seed, const uint64_t* step,
+                             uint8_t* keep, void* stream);
+
 /* ========================================================================
  * Parameter-server merge of the two workers' pushes (Sec. 3.4, with the SGD
  * of Eq. 1 and momentum).  Each push i brings its worker's batch-mean
@@ -311,6 +339,27 @@ typedef struct {
 
 DBL_API int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const float* g_large, const float* g_small, int64_t n,
                             const dbl_merge_params* params, void* stream);
+
+/* Late and missing pushes.  Under ASP the server applies each push as it
+ * arrives and does not wait for a worker that has stopped (Sec. 2.4); a
+ * missing push is merged as g = NULL above.  With the workers on streams,
+ * "has pushed" means "the worker's step event has completed".
+ *
+ * dbl_event_wait (host): DBL_OK once the cudaEvent_t `event` has completed,
+ * DBL_ERR_TIMEOUT if it has not after timeout_s seconds (polling
+ * cudaEventQuery; nothing is enqueued and the device is not synchronised),
+ * DBL_ERR_CUDA if the query fails.  An event never recorded counts as
+ * complete, as for cudaEventQuery.
+ *
+ * dbl_hold: holds `stream` until the host writes a non-zero value to *flag
+ * (host-pinned memory the device can read, 4-byte aligned), or until
+ * timeout_s (in (0, 10] s) has passed, whichever comes first; then writes
+ * DBL_OK (released) or DBL_ERR_TIMEOUT (gave up) to *status (device or
+ * pinned memory, may be NULL).  It emulates a worker whose push is delayed,
+ * as a straggler on the paper's network would be; the wait is bounded, so
+ * the stream always moves on.  Not a step of the method. */
+DBL_API int dbl_event_wait(void* event, double timeout_s);
+DBL_API int dbl_hold(const uint32_t* flag, double timeout_s, int32_t* status, void* stream);
 
 /* ========================================================================
  * Progressive resizing for the low-resolution sub-stages of cyclic

@@ -321,13 +321,75 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// ----------------------------------------------------------------------------- dropout
+// Dropout of the pooled features before the FC layer (Sec. 4.1: the rate rises with the
+// resolution, Tables 7 and 9), inverted: a kept feature is scaled by 1/(1 - d).  The draw is
+// the counter-based generator Philox4x64-10 (Salmon et al., SC 2011): ten rounds over a
+// 256-bit counter with a 128-bit key; a round takes the full 128-bit products of counter
+// words 0 and 2 with the two round multipliers and moves the words to
+//   (hi(M1*c2) ^ c1 ^ k0, lo(M1*c2), hi(M0*c0) ^ c3 ^ k1, lo(M0*c0)),
+// and the key is advanced by the two Weyl increments between rounds.  Feature c of sample n
+// takes word c % 4 of the block at counter (n*C/4 + c/4, step, 0, 0), key (seed, 0), and is
+// kept when the word's upper 32 bits are >= thr = floor(d * 2^32).
+struct Dropout {
+    uint32_t thr;          // 0: no dropout
+    float scale;           // 1/(1 - d), rounded to fp32
+    uint64_t seed;
+    const uint64_t* step;  // device counter, read when the kernel runs
+    float* mult;           // [n, C] per-feature multiplier (0 or scale) for the backward pass
+};
+
+__device__ __forceinline__ void philox4x64_10(uint64_t c[4], uint64_t k0, uint64_t k1)
+{
+    constexpr uint64_t kM0 = 0xD2E7470EE14C6C93ull, kM1 = 0xCA5A826395121157ull;
+    constexpr uint64_t kW0 = 0x9E3779B97F4A7C15ull, kW1 = 0xBB67AE8584CAA73Bull;
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint64_t p0 = kM0 * c[0], q0 = __umul64hi(kM0, c[0]);
+        const uint64_t p1 = kM1 * c[2], q1 = __umul64hi(kM1, c[2]);
+        const uint64_t a = q1 ^ c[1] ^ k0, b = q0 ^ c[3] ^ k1;
+        c[0] = a;
+        c[1] = p1;
+        c[2] = b;
+        c[3] = p0;
+        k0 += kW0;
+        k1 += kW1;
+    }
+}
+
+// keep bits (bit j: feature 4*group + j) of one Philox block
+__device__ __forceinline__ unsigned dropout_keep4(uint64_t seed, uint64_t step, uint64_t group, uint32_t thr)
+{
+    uint64_t c[4] = {group, step, 0, 0};
+    philox4x64_10(c, seed, 0);
+    unsigned bits = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) bits |= (uint32_t)(c[j] >> 32) >= thr ? 1u << j : 0u;
+    return bits;
+}
+
+__global__ void __launch_bounds__(256) dropout_mask_kernel(int n, int C, uint32_t thr, uint64_t seed,
+                                                           const uint64_t* __restrict__ step, uint8_t* __restrict__ keep)
+{
+    const int64_t groups = (int64_t)n * (C / 4);
+    const uint64_t st = thr ? *step : 0;
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += (int64_t)gridDim.x * blockDim.x) {
+        const unsigned b = thr ? dropout_keep4(seed, st, (uint64_t)g, thr) : 0xFu;
+        uchar4 v = make_uchar4(b & 1, (b >> 1) & 1, (b >> 2) & 1, (b >> 3) & 1);
+        reinterpret_cast<uchar4*>(keep)[g] = v;
+    }
+}
+
+__global__ void dropout_advance_kernel(uint64_t* step) { *step += 1; }
+
 // ----------------------------------------------------------------------------- head
-// feat[n, c] = mean over hw of x[n, hw, c]
+// feat[n, c] = mean over hw of x[n, hw, c], then (with dropout) times the feature's multiplier
 __global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __restrict__ x, float* __restrict__ feat,
-                                                      int n, int hw, int C)
+                                                      int n, int hw, int C, Dropout dp)
 {
     const int groups = C / 8;
     const int64_t total = (int64_t)n * groups;
+    const uint64_t st = dp.thr ? *dp.step : 0;
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
          t += (int64_t)gridDim.x * blockDim.x) {
         const int g = (int)(t % groups);
@@ -340,8 +402,19 @@ __global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __res
             for (int k = 0; k < 8; ++k) acc[k] += f[k];
         }
         const float inv = 1.0f / (float)hw;
+        if (dp.thr) {
+            const uint64_t q = (uint64_t)b * (uint64_t)(C / 4) + 2 * (uint64_t)g;
+            const unsigned bits = dropout_keep4(dp.seed, st, q, dp.thr) | dropout_keep4(dp.seed, st, q + 1, dp.thr) << 4;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv;
+            for (int k = 0; k < 8; ++k) {
+                const float m = (bits >> k) & 1 ? dp.scale : 0.f;
+                dp.mult[(int64_t)b * C + 8 * g + k] = m;
+                feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv * m;
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv;
+        }
     }
 }
 
@@ -524,9 +597,9 @@ __global__ void head_reduce_kernel(const float* __restrict__ row_loss, const flo
     db[j] = s;
 }
 
-// dx[n, i, c] = df[n, c] / hw
+// dx[n, i, c] = df[n, c] / hw, with dropout (df[n, c] * mult[n, c]) / hw
 __global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, __nv_bfloat16* __restrict__ dx,
-                                                          int n, int hw, int C)
+                                                          int n, int hw, int C, const float* __restrict__ mult)
 {
     const int groups = C / 8;
     const int64_t total = (int64_t)n * hw * groups;
@@ -537,7 +610,10 @@ __global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restric
         const int b = (int)(t / groups / hw);
         float f[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) f[k] = df[(int64_t)b * C + 8 * g + k] * inv;
+        for (int k = 0; k < 8; ++k) {
+            const int64_t e = (int64_t)b * C + 8 * g + k;
+            f[k] = (mult ? df[e] * mult[e] : df[e]) * inv;
+        }
         reinterpret_cast<uint4*>(dx)[t] = pack8(f);
     }
 }
@@ -617,35 +693,49 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
 size_t dbl_head_workspace_bytes(int32_t n, int32_t c, int32_t classes)
 {
     if (n <= 0 || c <= 0 || classes <= 0) return 0;
-    // feat [n,c], logits/dlogits [n,classes], df [n,c], row_loss [n], then the K-chunk partial
-    // sums of the largest of the three GEMMs
-    const size_t f = (size_t)n * c * 2 + (size_t)n * classes + (size_t)n;
+    // feat [n,c], logits/dlogits [n,classes], df [n,c], row_loss [n], dropout multipliers [n,c],
+    // then the K-chunk partial sums of the largest of the three GEMMs
+    const size_t f = (size_t)n * c * 3 + (size_t)n * classes + (size_t)n;
     const size_t part = std::max({gemm_part_floats(n, classes, c), gemm_part_floats(classes, c, n),
                                   gemm_part_floats(n, c, classes)});
     return (((f + 3) / 4 * 4 + part) * sizeof(float) + 255) / 256 * 256;
 }
 
-int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
-                     const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx,
-                     void* ws, size_t ws_bytes, void* stream)
+}  // extern "C"
+
+namespace {
+
+int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w, const float* fc_b,
+                 const int32_t* labels, float drop_rate, uint64_t seed, uint64_t* step, float* loss, float* dfc_w,
+                 float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream, const char* name)
 {
     using namespace dbl;
     if (n <= 0 || hw <= 0 || c <= 0 || classes <= 0 || !x || !fc_w || !fc_b || !labels || !loss || !dfc_w || !dfc_b ||
         !dx)
-        return set_error(DBL_ERR_INVALID, "head_fwd_bwd: bad arguments");
+        return set_error(DBL_ERR_INVALID, "%s: bad arguments", name);
     if (c % 8 || !aligned16(x) || !aligned16(dx))
-        return set_error(DBL_ERR_INVALID, "head_fwd_bwd: channels must be a multiple of 8, tensors 16-byte aligned");
+        return set_error(DBL_ERR_INVALID, "%s: channels must be a multiple of 8, tensors 16-byte aligned", name);
+    if (!(drop_rate >= 0.f && drop_rate < 1.f))
+        return set_error(DBL_ERR_INVALID, "%s: dropout rate %g outside [0, 1)", name, (double)drop_rate);
+    if (drop_rate > 0.f && (!step || (reinterpret_cast<uintptr_t>(step) & 7)))
+        return set_error(DBL_ERR_INVALID, "%s: dropout needs an 8-byte aligned device step counter", name);
     const size_t need = dbl_head_workspace_bytes(n, c, classes);
-    if (!ws || ws_bytes < need) return set_error(DBL_ERR_WORKSPACE, "head_fwd_bwd: workspace %zu < %zu", ws_bytes, need);
+    if (!ws || ws_bytes < need) return set_error(DBL_ERR_WORKSPACE, "%s: workspace %zu < %zu", name, ws_bytes, need);
     float* feat = static_cast<float*>(ws);
     float* logits = feat + (size_t)n * c;
     float* df = logits + (size_t)n * classes;
     float* row_loss = df + (size_t)n * c;
-    float* part = feat + ((size_t)n * c * 2 + (size_t)n * classes + (size_t)n + 3) / 4 * 4;
+    float* mult = row_loss + (size_t)n;
+    float* part = feat + ((size_t)n * c * 3 + (size_t)n * classes + (size_t)n + 3) / 4 * 4;
+    Dropout dp{0u, 1.f, seed, step, mult};
+    if (drop_rate > 0.f) {
+        dp.thr = (uint32_t)floor((double)drop_rate * 4294967296.0);
+        dp.scale = (float)(1.0 / (1.0 - (double)drop_rate));
+    }
     cudaStream_t s = as_stream(stream);
     int rc;
     avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(x), feat, n,
-                                                                       hw, c);
+                                                                       hw, c, dp);
     if ((rc = launch_check("avgpool launch"))) return rc;
     // logits = feat * W^T + b
     if ((rc = gemm_f32(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c, part, s, "fc fwd launch")))
@@ -660,9 +750,47 @@ int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const vo
     // df[n, c] = sum_j dl[n, j] W[j, c]
     if ((rc = gemm_f32(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes, part, s, "fc dX launch")))
         return rc;
-    avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(df, static_cast<__nv_bfloat16*>(dx), n,
-                                                                                hw, c);
-    return launch_check("avgpool_bwd launch");
+    avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(
+        df, static_cast<__nv_bfloat16*>(dx), n, hw, c, dp.thr ? mult : nullptr);
+    if ((rc = launch_check("avgpool_bwd launch")) || !dp.thr) return rc;
+    dropout_advance_kernel<<<1, 1, 0, s>>>(step);  // the next call draws a fresh mask
+    return launch_check("dropout advance launch");
+}
+
+}  // namespace
+
+extern "C" {
+
+int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
+                     const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx,
+                     void* ws, size_t ws_bytes, void* stream)
+{
+    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, 0.f, 0, nullptr, loss, dfc_w, dfc_b, dx, ws, ws_bytes,
+                        stream, "head_fwd_bwd");
+}
+
+int dbl_head_fwd_bwd_dropout(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
+                             const float* fc_b, const int32_t* labels, float drop_rate, uint64_t seed, uint64_t* step,
+                             float* loss, float* dfc_w, float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream)
+{
+    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, drop_rate, seed, step, loss, dfc_w, dfc_b, dx, ws,
+                        ws_bytes, stream, "head_fwd_bwd_dropout");
+}
+
+int dbl_dropout_mask(int32_t n, int32_t c, float drop_rate, uint64_t seed, const uint64_t* step, uint8_t* keep,
+                     void* stream)
+{
+    using namespace dbl;
+    if (n < 0 || c <= 0 || c % 4 || !keep || (reinterpret_cast<uintptr_t>(keep) & 3))
+        return set_error(DBL_ERR_INVALID, "dropout_mask: bad arguments (c a multiple of 4, keep 4-byte aligned)");
+    if (!(drop_rate >= 0.f && drop_rate < 1.f))
+        return set_error(DBL_ERR_INVALID, "dropout_mask: rate %g outside [0, 1)", (double)drop_rate);
+    const uint32_t thr = drop_rate > 0.f ? (uint32_t)floor((double)drop_rate * 4294967296.0) : 0u;
+    if (thr && (!step || (reinterpret_cast<uintptr_t>(step) & 7)))
+        return set_error(DBL_ERR_INVALID, "dropout_mask: needs an 8-byte aligned device step counter");
+    if (n == 0) return DBL_OK;
+    dropout_mask_kernel<<<grid_for((int64_t)n * (c / 4), 256), 256, 0, as_stream(stream)>>>(n, c, thr, seed, step, keep);
+    return launch_check("dropout_mask launch");
 }
 
 }  // extern "C"

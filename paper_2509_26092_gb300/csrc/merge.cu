@@ -6,6 +6,9 @@
 // writes w, u (8 B) and the bf16 w16 (2 B), 26 B in all.  The kernel is
 // HBM-bound; it moves 4 parameters per thread per step with 128-bit loads,
 // streaming (evict-first) cache hints, and two steps in flight per thread.
+#include <chrono>
+#include <thread>
+
 #include "dbl_internal.cuh"
 
 namespace {
@@ -148,4 +151,63 @@ extern "C" int dbl_zero_f32_2d(float* base, int64_t rows, int64_t cols, int64_t 
     return cuda_check(cudaMemset2DAsync(base, (size_t)ld * sizeof(float), 0, (size_t)cols * sizeof(float), (size_t)rows,
                                         as_stream(stream)),
                       "zero_f32_2d");
+}
+
+// ----------------------------------------------------------------------------- late and missing pushes
+// Under ASP the server applies whatever push arrives and does not wait for a worker that
+// has stopped (Sec. 2.4).  On one GPU a worker is a stream, so "has not pushed" is an
+// event that has not completed by the server's deadline; dbl_event_wait gives the host
+// that deadline.  dbl_hold holds a worker's stream until the host releases it: a push
+// delayed as on the paper's network (a straggler), bounded so that it always ends.
+namespace {
+
+__device__ __forceinline__ uint64_t global_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__global__ void hold_kernel(const volatile uint32_t* flag, uint64_t timeout_ns, int32_t* status)
+{
+    const uint64_t t0 = global_ns();
+    int32_t rc = DBL_ERR_TIMEOUT;
+    // bounded twice: by the timeout, and by an iteration count that takes far longer at
+    // the sleep's minimum of 1 us per poll
+    for (uint32_t it = 0; it < (1u << 30); ++it) {
+        if (*flag) {
+            rc = DBL_OK;
+            break;
+        }
+        if (global_ns() - t0 >= timeout_ns) break;
+        __nanosleep(1000);
+    }
+    if (status) *status = rc;
+}
+
+}  // namespace
+
+extern "C" int dbl_hold(const uint32_t* flag, double timeout_s, int32_t* status, void* stream)
+{
+    using namespace dbl;
+    if (!flag || (reinterpret_cast<uintptr_t>(flag) & 3)) return set_error(DBL_ERR_INVALID, "hold: flag must be 4-byte aligned");
+    if (!(timeout_s > 0.0 && timeout_s <= 10.0)) return set_error(DBL_ERR_INVALID, "hold: timeout must be in (0, 10] s");
+    hold_kernel<<<1, 1, 0, as_stream(stream)>>>(flag, (uint64_t)(timeout_s * 1e9), status);
+    return launch_check("hold launch");
+}
+
+extern "C" int dbl_event_wait(void* event, double timeout_s)
+{
+    using namespace dbl;
+    if (!event || !(timeout_s >= 0.0)) return set_error(DBL_ERR_INVALID, "event_wait: null event or negative timeout");
+    const auto t0 = std::chrono::steady_clock::now();
+    for (;;) {
+        const cudaError_t e = cudaEventQuery(static_cast<cudaEvent_t>(event));
+        if (e == cudaSuccess) return DBL_OK;
+        if (e != cudaErrorNotReady) return cuda_check(e, "event_wait: cudaEventQuery");
+        const double waited = std::chrono::duration<double>(std::chrono::steady_clock::now() - t0).count();
+        if (waited >= timeout_s)
+            return set_error(DBL_ERR_TIMEOUT, "event_wait: not complete after %.3f s", timeout_s);
+        std::this_thread::sleep_for(std::chrono::microseconds(50));
+    }
 }

@@ -90,6 +90,11 @@ def lib():
             "dbl_bn_relu_maxpool_fwd": (ctypes.c_int, [ctypes.POINTER(BnShape), _I32, _I32, _I32] + [_V] * 10),
             "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
             "dbl_head_fwd_bwd": (ctypes.c_int, [_I32] * 4 + [_V] * 8 + [_V, _SZ, _V]),
+            "dbl_head_fwd_bwd_dropout": (ctypes.c_int, [_I32] * 4 + [_V] * 4 + [ctypes.c_float, ctypes.c_uint64]
+                                         + [_V] * 6 + [_SZ, _V]),
+            "dbl_dropout_mask": (ctypes.c_int, [_I32, _I32, ctypes.c_float, ctypes.c_uint64, _V, _V, _V]),
+            "dbl_event_wait": (ctypes.c_int, [_V, _D]),
+            "dbl_hold": (ctypes.c_int, [_V, _D, _V, _V]),
             "dbl_ps_dual_batch_merge": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams), _V]),
             "dbl_progressive_resize": (ctypes.c_int, [_V, ctypes.c_int, _I32, _I32, _I32, _I32, _V, ctypes.c_int,
                                                       _I32, _I32, _I32, _V]),
@@ -265,6 +270,36 @@ def dbl_head_workspace_bytes(n, c, classes):
 def dbl_head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, loss, dfc_w, dfc_b, dx, ws, ws_bytes, stream=None):
     _check(lib().dbl_head_fwd_bwd(n, hw, c, classes, _ptr(x), _ptr(fc_w), _ptr(fc_b), _ptr(labels), _ptr(loss),
                                   _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, fc_w, fc_b, labels, drop_rate, seed, step, loss, dfc_w, dfc_b, dx,
+                             ws, ws_bytes, stream=None):
+    """The head with dropout of rate drop_rate before the FC layer; step: device uint64 counter
+    (incremented by one on the stream after the call's kernels)."""
+    _check(lib().dbl_head_fwd_bwd_dropout(n, hw, c, classes, _ptr(x), _ptr(fc_w), _ptr(fc_b), _ptr(labels),
+                                          float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(loss),
+                                          _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def dbl_dropout_mask(n, c, drop_rate, seed, step, keep, stream=None):
+    """keep [n, c] uint8: the mask dbl_head_fwd_bwd_dropout draws for (drop_rate, seed, *step)."""
+    _check(lib().dbl_dropout_mask(n, c, float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(keep),
+                                  _stream(stream)))
+
+
+def dbl_event_wait(event, timeout_s):
+    """DBL_OK once the torch.cuda.Event (or raw cudaEvent_t) has completed, DBL_ERR_TIMEOUT if it
+    has not after timeout_s seconds; other failures raise DblError."""
+    handle = event.cuda_event if hasattr(event, "cuda_event") else event
+    rc = lib().dbl_event_wait(ctypes.c_void_p(handle), float(timeout_s))
+    if rc not in (DBL_OK, DBL_ERR_TIMEOUT):
+        _check(rc)
+    return rc
+
+
+def dbl_hold(flag, timeout_s, status=None, stream=None):
+    """Hold the stream until the pinned host uint32 `flag` is non-zero or timeout_s passes."""
+    _check(lib().dbl_hold(_ptr(flag), float(timeout_s), _ptr(status), _stream(stream)))
 
 
 def dbl_ps_dual_batch_merge(w, u, w16_out, g_large, g_small, n, lr, momentum, f_large, f_small, order=0,

@@ -38,9 +38,11 @@ zero-padded in every direction.
 Convolutions read the bf16 weights ``w16``; BatchNorm and the fully connected
 layer read the fp32 master weights directly (they are tiny).
 """
+import time
 from dataclasses import dataclass, field
 
 import numpy as np
+
 import torch
 
 from . import dbl as D
@@ -225,8 +227,12 @@ class ServerState:
 class Worker:
     """Activations, gradients and scratch of one worker at one (batch, resolution)."""
 
-    def __init__(self, spec, batch, res, device="cuda", eps=1e-5):
+    def __init__(self, spec, batch, res, device="cuda", eps=1e-5, dropout=0.0, dropout_seed=0):
         self.spec, self.batch, self.res, self.eps = spec, batch, res, eps
+        # dropout before the FC layer (Sec. 4.1): rate, the worker's seed, and the device step
+        # counter the head reads and advances once per step
+        self.dropout, self.dropout_seed = float(dropout), int(dropout_seed)
+        self.dropout_step = torch.zeros(1, dtype=torch.int64, device=device)
         dev = device
         bf = torch.bfloat16
         B = batch
@@ -410,8 +416,13 @@ class Worker:
             cur = d["out"]
         # ---- head: pooling, FC, softmax cross-entropy and their backward
         C = spec.widths[-1]
-        D.dbl_head_fwd_bwd(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"), self.labels, self.loss,
-                           gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
+        if self.dropout > 0.0:
+            D.dbl_head_fwd_bwd_dropout(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"),
+                                       self.labels, self.dropout, self.dropout_seed, self.dropout_step, self.loss,
+                                       gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
+        else:
+            D.dbl_head_fwd_bwd(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"), self.labels,
+                               self.loss, gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
         # ---- backward
         dout, dout2 = self.dfeat, None
         for d in reversed(self.blocks):
@@ -456,6 +467,26 @@ class Worker:
             D.dbl_bn_relu_fused_bwd(bns, dout, dout2, self.stem_y, None, pv("bn1.g"), s_mean, s_istd,
                                     self.stem_dy, None, gv("bn1.g"), gv("bn1.b"), ws, wsb, s, beta=pv("bn1.b"))
         self.stem_wgrad(self.stem_dy, gv("conv1.w"), ws, wsb, s)
+
+
+def collect_pushes(done, deadline_s, wait, clock=time.monotonic):
+    """The server's side of a deadline (host): ``done`` maps worker tags to their step
+    events, in the order the server checks them; all share one deadline of ``deadline_s``
+    seconds from the call.  ``wait(event, seconds)`` returns DBL_OK once the event has
+    completed or DBL_ERR_TIMEOUT if it has not within the given seconds.  Returns
+    (arrived, failed): lists of tags."""
+    t0 = clock()
+    arrived, failed = [], []
+    for tag, ev in done.items():
+        left = max(0.0, deadline_s - (clock() - t0))
+        rc = wait(ev, left)
+        if rc == D.DBL_OK:
+            arrived.append(tag)
+        elif rc == D.DBL_ERR_TIMEOUT:
+            failed.append(tag)
+        else:
+            raise D.DblError(rc, f"waiting for worker {tag}")
+    return arrived, failed
 
 
 class DualBatchIteration:
@@ -542,6 +573,45 @@ class DualBatchIteration:
             self._enqueue()
         self._consumed = torch.cuda.Event()
         self._consumed.record(cur)
+
+    def run_with_deadline(self, deadline_s, wait=None):
+        """One iteration in which the server waits at most ``deadline_s`` seconds of host time
+        (counted from when both workers' steps are enqueued) for the pushes, and merges those
+        that arrived: under ASP the server does not wait for a worker that has stopped
+        (Sec. 2.4).  A worker whose step has not completed by then is reported failed and its
+        push is left out of this iteration; its stream finishes in its own time, and the next
+        iteration's steps queue behind it.  Runs eagerly, not as the captured graph.
+        Returns (status, failed): (DBL_OK, []) when every worker pushed, otherwise
+        (DBL_ERR_TIMEOUT, tags) with the tags ('L', 'S') of the workers that missed the
+        deadline.  ``wait(event, seconds) -> status`` defaults to ``dbl_event_wait``.
+        Run the iteration once (``run`` or ``capture``) before the first call: the first launch
+        of a kernel loads it, and loading waits for every stream, a stalled one included."""
+        wait = wait or D.dbl_event_wait
+        cur = torch.cuda.current_stream()
+        if self._inputs_ready is not None:
+            cur.wait_event(self._inputs_ready)
+            self._inputs_ready = None
+        done = {}
+        for tag, wk, st, img in (("L", self.large, self.stream_l, self.images_l),
+                                 ("S", self.small, self.stream_s, self.images_s)):
+            if wk is None:
+                continue
+            st.wait_stream(cur)
+            wk.enqueue_step(self.server, img, self.native_res, st)
+            ev = torch.cuda.Event()
+            ev.record(st)
+            done[tag] = ev
+        arrived, failed = collect_pushes(done, deadline_s, wait)
+        if arrived:
+            for tag in arrived:
+                cur.wait_event(done[tag])
+            srv = self.server
+            D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, self.large.grad if "L" in arrived else None,
+                                      self.small.grad if "S" in arrived else None, srv.spec.n_flat, self.lr,
+                                      self.momentum, self.f_large, self.f_small, self.order, cur.cuda_stream)
+        self._consumed = torch.cuda.Event()
+        self._consumed.record(cur)
+        return (D.DBL_OK if not failed else D.DBL_ERR_TIMEOUT), failed
 
     def capture(self):
         """Record one iteration (both workers, the join and the merge) as a CUDA graph."""

@@ -20,8 +20,8 @@ Table 9 for ImageNet, Sec. 5.2: three stages of decreasing learning rate, each
 cycling through increasing resolutions), and ``run_schedule`` runs one
 on synthetic data for a fraction of each epoch; the synthetic source images have
 the schedule's largest resolution, so every sub-stage downsamples or passes them
-through.  The dropout rates of those tables are listed but not applied (the step
-has no dropout layer).
+through.  Each sub-stage's workers apply the tables' dropout rate before the FC
+layer (inverted dropout with a counter-based mask; each worker has its own seed).
 """
 import argparse
 import json
@@ -81,6 +81,8 @@ class AsyncDualBatch:
         self.streams = {"L": torch.cuda.Stream(), "S": torch.cuda.Stream()}
         self.pulled = {"L": PulledWeights(server), "S": PulledWeights(server)}
         self.losses = {"L": [], "S": []}
+        self.done = {}     # tag -> event after the worker's latest step
+        self.failed = []   # workers that missed the server's deadline (no further pushes)
 
     def _launch(self, tag):
         import torch
@@ -91,14 +93,22 @@ class AsyncDualBatch:
         with torch.cuda.stream(s):
             wk.labels.copy_(labs[b], non_blocking=True)
         wk.enqueue_step(self.pulled[tag], imgs[b], self.native_res, s)
+        self.done[tag] = torch.cuda.Event()
+        self.done[tag].record(s)
 
-    def run(self, t_large, t_small, n_large, n_small, on_push=None):
+    def run(self, t_large, t_small, n_large, n_small, on_push=None, deadline_s=None, wait=None):
         """Run n_large + n_small pushes in ``push_order``; returns that order.
         ``on_push(tag, worker, pulled)``, if given, is called when a push has been
-        enqueued, after its merge and before the worker pulls (stream ``self.streams[tag]``)."""
+        enqueued, after its merge and before the worker pulls (stream ``self.streams[tag]``).
+        With ``deadline_s`` the server (the host) waits at most that long for each push's step
+        to complete (``wait(event, seconds)``, default ``dbl_event_wait``); a worker that misses
+        it is taken as stopped: that push and all its later ones are left out (ASP does not
+        wait for it, Sec. 2.4) and its tag is listed in ``self.failed``."""
         import torch
 
         from . import dbl as D
+        from .resnet18 import collect_pushes
+        wait = wait or D.dbl_event_wait
         order = push_order(t_large, t_small, n_large, n_small)
         remaining = {"L": n_large, "S": n_small}
         cur = torch.cuda.current_stream()
@@ -110,6 +120,11 @@ class AsyncDualBatch:
                 self._launch(tag)
         last = None  # event after the previous push's merge and pull
         for _, tag, _ in order:
+            if tag in self.failed:
+                continue
+            if deadline_s is not None and collect_pushes({tag: self.done[tag]}, deadline_s, wait)[1]:
+                self.failed.append(tag)
+                continue
             s, wk = self.streams[tag], self.workers[tag]
             if last is not None:
                 s.wait_event(last)
@@ -139,7 +154,7 @@ class SubStage:
     lr: float
     res: int
     batch_large: int
-    dropout: float  # listed by the paper's tables; not applied
+    dropout: float  # rate of the dropout before the FC layer
 
 
 def hybrid_schedule(variant):
@@ -190,7 +205,8 @@ def run_schedule(variant, fits, k=1.05, data_fraction=1e-3, batch_large=None, ma
         if max_batch_small:
             pl["batch_small"] = min(pl["batch_small"], max_batch_small)
         bl, bs = pl["batch_large"], pl["batch_small"]
-        large, small = R.Worker(spec, bl, sub.res, device), R.Worker(spec, bs, sub.res, device)
+        large = R.Worker(spec, bl, sub.res, device, dropout=sub.dropout, dropout_seed=2 * seed + 1)
+        small = R.Worker(spec, bs, sub.res, device, dropout=sub.dropout, dropout_seed=2 * seed + 2)
         imgs = {t: [torch.from_numpy(synth.images_u8(n, native, native, 3, seed=seed + 10 * i + j,
                                                      name=t)).to(device) for i in range(2)]
                 for j, (t, n) in enumerate((("L", bl), ("S", bs)))}
@@ -207,7 +223,7 @@ def run_schedule(variant, fits, k=1.05, data_fraction=1e-3, batch_large=None, ma
         images = pl["pushes_large"] * bl + pl["pushes_small"] * bs
         loss = {t: [float(x) for x in torch.stack(run.losses[t]).cpu()] for t in ("L", "S")}
         out.append({"stage": sub.stage, "res": sub.res, "lr": sub.lr, "epochs": sub.epochs,
-                    "dropout_listed": sub.dropout, **pl, "pushes": len(order),
+                    "dropout": sub.dropout, **pl, "pushes": len(order),
                     "first_pushes": "".join(t for _, t, _ in order[:12]), "seconds": secs,
                     "images_per_s": images / secs, "loss_first": {t: v[0] for t, v in loss.items() if v},
                     "loss_last": {t: v[-1] for t, v in loss.items() if v}})

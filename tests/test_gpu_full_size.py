@@ -1,5 +1,6 @@
 """The step's kernels at the full sizes the bench times: the 224 px layers of the
-ImageNet-shaped ResNet-18 at the large worker's batch of 512, through the same
+ImageNet-shaped ResNet-18 at the large worker's batch of 512, and the 288 px layers
+of the paper's last ImageNet sub-stage at its batch of 740, through the same
 library calls and launch configurations as the training step.
 
 Convolutions (window kernels, the 128-column window tiles and the 256-column tiles
@@ -28,6 +29,13 @@ SHAPES = [  # n, h, w, c, k, r, stride, pad
     (512, 14, 14, 256, 256, 3, 1, 1),  # layer3: 256-column tiles on CTA pairs
     (512, 7, 7, 512, 512, 3, 1, 1),    # layer4: two 256-column tiles
     (512, 56, 56, 64, 128, 1, 2, 0),   # layer2.0.down: 1x1 stride-2 projection
+    # the paper's 288 px ImageNet sub-stage (Table 9) at its large-batch worker's batch of 740
+    (740, 72, 72, 64, 64, 3, 1, 1),    # layer1
+    (740, 72, 72, 64, 128, 3, 2, 1),   # layer2.0.conv1
+    (740, 36, 36, 128, 128, 3, 1, 1),  # layer2
+    (740, 18, 18, 256, 256, 3, 1, 1),  # layer3
+    (740, 9, 9, 512, 512, 3, 1, 1),    # layer4: 59,940 rows, a ragged last tile
+    (740, 18, 18, 256, 512, 1, 2, 0),  # layer4.0.down
 ]
 
 

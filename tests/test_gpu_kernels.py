@@ -139,6 +139,7 @@ STEM_CASES = [  # n, h (square input), r, stride, pad
     (4, 64, 7, 2, 3),    # several tiles
     (2, 224, 7, 2, 3),   # full size: window tiles of two 112-wide rows, two-row weight-gradient K-blocks
     (1, 160, 7, 2, 3),   # tiles of three 80-wide rows
+    (1, 288, 7, 2, 3),   # the paper's 288 px sub-stage: 144-wide rows
 ]
 
 
@@ -351,6 +352,78 @@ def test_head_matches_oracle(D, n, hw, c, classes):
     assert max_norm_rel(host(dW), rdW) <= 1e-4
     assert max_norm_rel(host(db), rdb) <= 1e-4
     assert max_norm_rel(host(dx), rdx) <= CONV_TOL
+
+
+@pytest.mark.parametrize("n,hw,c,classes,rate", [(6, 4, 64, 10, 0.3), (128, 49, 512, 1000, 0.1),
+                                                 (37, 16, 512, 100, 0.2)])
+def test_head_dropout_matches_oracle(D, n, hw, c, classes, rate):
+    """Dropout before the FC layer: the mask bit for bit against the oracle's Philox draw,
+    the head's outputs against the oracle applying that mask, the step counter advanced by
+    one per call, and a second call drawing a new mask."""
+    g = rng(n + classes)
+    x = bf16_values(np.maximum(g.standard_normal((n, hw, c)), 0))
+    W = (0.05 * g.standard_normal((classes, c))).astype(np.float32)
+    b = (0.01 * g.standard_normal(classes)).astype(np.float32)
+    lab = g.integers(0, classes, n).astype(np.int32)
+    d = float(np.float32(rate))  # the rate as the fp32 value the library receives
+    seed, step0 = 0x9E3779B97F4A7C15 ^ n, 5
+    step = torch.tensor([step0], dtype=torch.int64, device="cuda")
+    keep = torch.empty((n, c), dtype=torch.uint8, device="cuda")
+    D.dbl_dropout_mask(n, c, rate, seed, step, keep)
+    rkeep = orc.dropout_mask(n, c, d, seed, step0)
+    torch.cuda.synchronize()
+    assert np.array_equal(keep.cpu().numpy(), rkeep)
+    loss = torch.empty(1, device="cuda")
+    dW = torch.empty((classes, c), device="cuda")
+    db = torch.empty(classes, device="cuda")
+    dx = torch.empty((n, hw, c), dtype=torch.bfloat16, device="cuda")
+    wsb = D.dbl_head_workspace_bytes(n, c, classes)
+    work = ws(wsb)
+    xd, Wd, bd, labd = to_bf16_dev(x), to_f32_dev(W), to_f32_dev(b), torch.from_numpy(lab).cuda()
+    D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, xd, Wd, bd, labd, rate, seed, step, loss, dW, db, dx, work, wsb)
+    x4 = x.reshape(n, 1, hw, c)
+    feat = orc.dropout_apply(orc.avgpool_fwd(x4), rkeep, d)
+    logits = orc.fc_fwd(feat, W, b)
+    rl, dl = orc.softmax_ce(logits, lab)
+    rdW, rdb, rdf = orc.fc_bwd(dl, feat, W)
+    rdx = orc.avgpool_bwd(orc.dropout_apply(rdf, rkeep, d), x4.shape).reshape(n, hw, c)
+    assert int(step.item()) == step0 + 1
+    assert abs(loss.item() - rl) <= 1e-5 * abs(rl)
+    assert max_norm_rel(host(dW), rdW) <= 1e-4
+    assert max_norm_rel(host(db), rdb) <= 1e-4
+    assert max_norm_rel(host(dx), rdx) <= CONV_TOL
+    dropped = np.broadcast_to((rkeep == 0)[:, None, :], (n, hw, c))
+    assert np.all(host(dx)[dropped] == 0.0)  # a dropped feature passes no gradient back
+    # the next call draws the mask of step 6
+    D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, xd, Wd, bd, labd, rate, seed, step, loss, dW, db, dx, work, wsb)
+    rkeep6 = orc.dropout_mask(n, c, d, seed, step0 + 1)
+    feat6 = orc.dropout_apply(orc.avgpool_fwd(x4), rkeep6, d)
+    rl6, _ = orc.softmax_ce(orc.fc_fwd(feat6, W, b), lab)
+    assert int(step.item()) == step0 + 2 and not np.array_equal(rkeep6, rkeep)
+    assert abs(loss.item() - rl6) <= 1e-5 * abs(rl6)
+
+
+def test_head_dropout_rate_zero_is_the_plain_head(D):
+    n, hw, c, classes = 9, 16, 64, 10
+    g = rng(3)
+    x = to_bf16_dev(bf16_values(np.maximum(g.standard_normal((n, hw, c)), 0)))
+    W, b = to_f32_dev(0.05 * g.standard_normal((classes, c))), to_f32_dev(0.01 * g.standard_normal(classes))
+    lab = torch.from_numpy(g.integers(0, classes, n).astype(np.int32)).cuda()
+    wsb = D.dbl_head_workspace_bytes(n, c, classes)
+    outs = []
+    for drop in (False, True):
+        o = (torch.empty(1, device="cuda"), torch.empty((classes, c), device="cuda"), torch.empty(classes, device="cuda"),
+             torch.empty((n, hw, c), dtype=torch.bfloat16, device="cuda"))
+        if drop:
+            D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, W, b, lab, 0.0, 1, None, *o, ws(wsb), wsb)
+        else:
+            D.dbl_head_fwd_bwd(n, hw, c, classes, x, W, b, lab, *o, ws(wsb), wsb)
+        outs.append(o)
+    torch.cuda.synchronize()
+    for a, b_ in zip(*outs):
+        assert torch.equal(a, b_)
+    with pytest.raises(D.DblError):
+        D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, W, b, lab, 1.0, 1, None, *outs[0], ws(wsb), wsb)
 
 
 # ----------------------------------------------------------------------------- convolutions

@@ -77,15 +77,20 @@ def test_train_step_matches_oracle(R, variant, classes, batch, res):
     _compare_grads(spec, wk.grad, ref["grads"], ref64["grads"], variant)
 
 
-def test_dual_batch_iteration_matches_oracle(R):
-    # native 32x32 images, sub-stage resolution 24: large worker batch 6, small worker batch 2
+@pytest.mark.parametrize("dropout", [0.0, 0.2])
+def test_dual_batch_iteration_matches_oracle(R, dropout):
+    # native 32x32 images, sub-stage resolution 24: large worker batch 6, small worker batch 2;
+    # with dropout before the FC layer (Sec. 4.1), each worker drawing its own mask
     spec = R.ResNet18Spec("cifar", 100)
     params = synth.params(spec.table(), seed=5, random_bn=True)
     u0 = synth.momentum_state(spec.table(), 0.01, seed=5)
     img = synth.images(8, 32, 32, 3, seed=5)
     lab = synth.labels(8, 100, seed=5)
     server = R.ServerState(spec, params, u0)
-    large, small = R.Worker(spec, 6, 24), R.Worker(spec, 2, 24)
+    large = R.Worker(spec, 6, 24, dropout=dropout, dropout_seed=101)
+    small = R.Worker(spec, 2, 24, dropout=dropout, dropout_seed=202)
+    d = float(np.float32(dropout))  # the rate as the fp32 value the library receives
+    drops = dict(dropout_large=(d, 101, 0), dropout_small=(d, 202, 0)) if dropout else {}
     fS = 19.0 / 21.0
     it = R.DualBatchIteration(server, large, small, 32, lr=0.2, momentum=0.9, f_large=1.0, f_small=fS, order=0)
     it.set_inputs(torch.from_numpy(img[2:]).cuda(), torch.from_numpy(lab[2:]).cuda(), torch.from_numpy(img[:2]).cuda(),
@@ -97,9 +102,15 @@ def test_dual_batch_iteration_matches_oracle(R):
     p64 = {k: v.astype(np.float64) for k, v in params.items()}
     u64 = {k: v.astype(np.float64) for k, v in u0.items()}
     nw, nu, lL, lS, gL, gS = OR.dual_batch_iteration(p64, u64, img[2:], lab[2:], img[:2], lab[:2], 24, "cifar", 0.2,
-                                                     0.9, 1.0, fS, order=0, bf16_storage=True)
+                                                     0.9, 1.0, fS, order=0, bf16_storage=True, **drops)
     nw64, _, _, _, gL64, gS64 = OR.dual_batch_iteration(p64, u64, img[2:], lab[2:], img[:2], lab[:2], 24, "cifar",
-                                                        0.2, 0.9, 1.0, fS, order=0, bf16_storage=False)
+                                                        0.2, 0.9, 1.0, fS, order=0, bf16_storage=False, **drops)
+    if dropout:
+        # each worker's step counter advanced once; the FC gradient of a feature no sample kept is zero
+        assert int(large.dropout_step.item()) == 1 and int(small.dropout_step.item()) == 1
+        keep = orc.dropout_mask(2, 512, d, 202, 0)
+        dead = np.where(keep.sum(axis=0) == 0)[0]
+        assert dead.size > 0 and np.all(spec.unpack(small.grad)["fc.w"][:, dead] == 0.0)
     assert abs(large.loss.item() - lL) <= TOL * abs(lL)
     assert abs(small.loss.item() - lS) <= TOL * abs(lS)
     _compare_grads(spec, large.grad, gL, gL64, "large worker")
@@ -186,3 +197,48 @@ def test_8bit_images_give_the_same_iteration_as_standardized_fp32(R):
         torch.cuda.synchronize()
         outs.append(server.w.clone())
     assert torch.equal(outs[0], outs[1])
+
+
+def test_a_late_push_is_left_out_of_the_merge(R):
+    """A small-batch worker held back on its stream (a straggler) misses the server's deadline:
+    the iteration reports DBL_ERR_TIMEOUT with the small worker as failed and merges the large
+    worker's push alone, as ASP does (Sec. 2.4).  Released afterwards, the held stream finishes,
+    and the next iteration merges both pushes again."""
+    D = load_dbl()
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=6)
+    u0 = synth.momentum_state(spec.table(), 0.01, seed=6)
+    img = torch.from_numpy(synth.images(8, 32, 32, 3, seed=6)).cuda()
+    lab = torch.from_numpy(synth.labels(8, 100, seed=6)).cuda()
+    server = R.ServerState(spec, params, u0)
+    large, small = R.Worker(spec, 6, 24), R.Worker(spec, 2, 24)
+    fS = 19.0 / 21.0
+    it = R.DualBatchIteration(server, large, small, 32, lr=0.2, momentum=0.9, f_large=1.0, f_small=fS, order=0)
+    it.set_inputs(img[2:], lab[2:], img[:2], lab[:2])
+    it.run()  # warm-up: the first launches load the library's kernels, which waits for every stream
+    torch.cuda.synchronize()
+    w0, u0d = server.w.double().cpu().numpy(), server.u.double().cpu().numpy()
+    flag = torch.zeros(1, dtype=torch.int32).pin_memory()
+    status = torch.full((1,), 7, dtype=torch.int32).pin_memory()
+    D.dbl_hold(flag, 5.0, status, it.stream_s)  # the small worker's step queues behind this
+    rc, failed = it.run_with_deadline(0.5)
+    held = int(status[0])  # still 7 while the hold waits
+    assert (rc, failed, held) == (D.DBL_ERR_TIMEOUT, ["S"], 7)
+    it.stream_l.synchronize()
+    torch.cuda.current_stream().synchronize()  # the merge, which did not wait for the held stream
+    rw, ru = orc.ps_merge(w0, u0d, large.grad.double().cpu().numpy(), None, 0.2, 0.9, 1.0, fS, 0)
+    assert max_norm_rel(server.w.double().cpu().numpy(), rw) <= 1e-6
+    assert max_norm_rel(server.u.double().cpu().numpy(), ru) <= 1e-6
+    flag[0] = 1  # release the straggler
+    torch.cuda.synchronize()
+    assert int(status[0]) == D.DBL_OK  # released by the host, not by the hold's own timeout
+    assert D.dbl_device_status() == D.DBL_OK
+    # a normal iteration afterwards: both pushes arrive and are merged
+    w1, u1 = server.w.double().cpu().numpy(), server.u.double().cpu().numpy()
+    rc, failed = it.run_with_deadline(60.0)
+    torch.cuda.synchronize()
+    assert rc == D.DBL_OK and failed == []
+    rw, ru = orc.ps_merge(w1, u1, large.grad.double().cpu().numpy(), small.grad.double().cpu().numpy(), 0.2, 0.9,
+                          1.0, fS, 0)
+    assert max_norm_rel(server.w.double().cpu().numpy(), rw) <= 1e-6
+    assert max_norm_rel(server.u.double().cpu().numpy(), ru) <= 1e-6
