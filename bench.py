@@ -147,6 +147,22 @@ class ClockSampler:
         return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def max_over_ranks(x, device="cpu"):
+    """The largest of each rank's x (the job's time is its slowest rank's); x itself on one rank."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(images_per_step, world, steps, ms):
+    """images/s of the whole job: every rank's images over the slowest rank's time."""
+    return images_per_step * world * steps / (ms / 1000.0)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -336,6 +352,70 @@ def conv_roofline(stage, reps=4, replays=2, table=None):
     return flops, secs, algo_bytes
 
 
+def bandwidth_kernels(pipe, hbm, reps=10):
+    """The HBM-bound kernels timed alone with L2 flushed before each launch (a 256 MB buffer,
+    larger than the 129 MB L2, written on the same stream): the parameter-server merge of both
+    pushes (26 B per parameter: read w, u, g_L, g_S, write w, u and the bf16 copy; 22 B with one
+    push) and, per stage, the large worker's resize of its uint8 source images into the stem's
+    unrolled bf16 input (bytes: the source read once plus the unrolled tensor written once).
+    Median of `reps` launches, CUDA events on the launching stream."""
+    import torch
+
+    from paper_2509_26092_gb300 import dbl as D
+    s = torch.cuda.current_stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=pipe["server"].w.device)
+
+    def timed(fn):
+        out = []
+        for _ in range(reps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            fn()
+            e1.record(s)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) * 1e-3)
+        out.sort()
+        return out[len(out) // 2]
+
+    srv, top = pipe["server"], pipe["stages"][-1]
+    gl, gs = top["large"].grad, top["small"].grad if top["small"] else None
+    n = srv.spec.n_flat
+    nbytes = n * (26 if gs is not None else 22)
+    t = timed(lambda: D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, gl, gs, n, LR, MOMENTUM, 1.0, F_SMALL, 0, s))
+    merge = {"us": round(t * 1e6, 2), "bytes": nbytes, "gbs": round(nbytes / t / 1e9, 1),
+             "frac": round(nbytes / t / 1e9 / hbm, 4), "params": n, "pushes": 2 if gs is not None else 1,
+             "l2": "flushed before each launch"}
+    resize = {}
+    for st in pipe["stages"]:
+        wk, it = st["large"], st["it"]
+        nb = it.images_l.numel() * it.images_l.element_size() + wk.x0.numel() * wk.x0.element_size()
+        t = timed(lambda: wk.stem_prepare(it.images_l, it.native_res, s))
+        resize[str(st["res"])] = {"us": round(t * 1e6, 2), "bytes": nb, "gbs": round(nb / t / 1e9, 1),
+                                  "frac": round(nb / t / 1e9 / hbm, 4), "batch": wk.batch}
+    return {"merge": merge, "resize": resize}
+
+
+def time_oracle_single_thread(config):
+    """The oracle on one host thread (OMP_NUM_THREADS=1, a child process): one dual-batch
+    iteration (large batch 2, small batch 1) at the smallest sub-stage resolution."""
+    code = ("import json, sys; sys.path.insert(0, sys.argv[1]); import bench\n"
+            "cfg = bench.CONFIGS[sys.argv[2]]; st = bench._oracle_setup(cfg)\n"
+            "n, dt = bench._oracle_iteration(cfg, st, min(cfg['stages']))\n"
+            "print(json.dumps({'images': n, 'seconds': dt}))\n")
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    try:
+        r = subprocess.run([sys.executable, "-c", code, ROOT, config], env=env, capture_output=True, text=True,
+                           timeout=600)
+        rec = json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception as e:  # the figure is a reported baseline; its absence must not fail the bench
+        return {"error": str(e)[:200]}
+    cfg = CONFIGS[config]
+    return {"value": round(rec["images"] / rec["seconds"], 4), "unit": "images/s", "cores": 1,
+            "seconds": round(rec["seconds"], 2),
+            "sample": f"one dual-batch iteration (large batch 2, small batch 1) at {min(cfg['stages'])} px, fp64"}
+
+
 def _conv_buffers(wk):
     """Per conv layer: (input, output, output-gradient, input-gradient, bf16 weights, fp32 gradient slice)."""
     spec = wk.spec
@@ -491,13 +571,9 @@ def run_ours(args, cfg):
     t1.record(stream)
     barrier()
     clk = clocks.stop()
-    ms = t0.elapsed_time(t1)
-    if ws > 1:
-        tt = torch.tensor([ms], device=device)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(t0.elapsed_time(t1), device)
     ms_per_step = ms / args.steps
-    value = images_per_step * ws * args.steps / (ms / 1000.0)
+    value = whole_job_rate(images_per_step, ws, args.steps, ms)
     gpu_launches = sum(s["launches"] for s in stages) * args.steps
 
     # per-resolution throughput (each stage's graph replayed alone)
@@ -549,12 +625,8 @@ def run_ours(args, cfg):
     e1.record(stream)
     barrier()
     assert len(loss_seen) == args.steps and all(np.isfinite(v).all() for v in map(np.asarray, loss_seen))
-    e2e_ms = e0.elapsed_time(e1)
-    if ws > 1:
-        tt = torch.tensor([e2e_ms], device=device)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_value = images_per_step * ws * args.steps / (e2e_ms / 1000.0)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), device)
+    e2e_value = whole_job_rate(images_per_step, ws, args.steps, e2e_ms)
     assert D.dbl_device_status() == D.DBL_OK, "a device-side wait timed out during the timed region"
 
     # roofline of the dominant kernel: the implicit-GEMM convolution, full-resolution stage, timed alone
@@ -580,12 +652,14 @@ def run_ours(args, cfg):
                           f"split-K reduce kernels (fwd/dgrad/wgrad, every layer of both workers at {top['res']} px, "
                           "each pass timed alone as CUDA-graph replays of its ABI calls)",
                 "peak_source": src}
+    bw = bandwidth_kernels(pipe, hbm)
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         v, dt, images, sample = time_oracle(cfg)
         cpu = {"value": round(v, 4), "unit": "images/s", "cores": int(os.environ.get("OMP_NUM_THREADS",
                                                                                       os.cpu_count() or 1)),
-               "kind": "oracle", "sample": sample, "seconds": round(dt, 2)}
+               "kind": "oracle", "sample": sample, "seconds": round(dt, 2),
+               "single_thread": time_oracle_single_thread(args.config)}
     if rank == 0:
         line = {"metric": METRIC, "value": round(value, 1), "unit": "images/s", "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3), "higher_is_better": True,
@@ -599,7 +673,8 @@ def run_ours(args, cfg):
                            "input": f"uint8 images {cfg['native']}x{cfg['native']}x3 from pinned host memory, "
                                     "standardized per channel on the GPU",
                            "parallelism": f"{ws} independent replica(s), 2 worker streams each"},
-                "per_resolution": per_res, "roofline": roofline, "cpu_baseline": cpu,
+                "per_resolution": per_res, "roofline": roofline, "merge": bw["merge"], "resize": bw["resize"],
+                "cpu_baseline": cpu,
                 "e2e": {"value": round(e2e_value, 1), "unit": "images/s", "h2d_bytes_per_step": h2d,
                         "d2h_bytes_per_step": d2h},
                 "clocks": clk, "gpu_launches": gpu_launches,

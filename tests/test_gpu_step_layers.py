@@ -25,7 +25,8 @@ def h(t):
     return t.detach().double().cpu().numpy()
 
 
-@pytest.mark.parametrize("variant,classes,batch,res", [("cifar", 100, 8, 32), ("imagenet", 1000, 4, 96)])
+@pytest.mark.parametrize("variant,classes,batch,res", [("cifar", 100, 8, 32), ("imagenet", 1000, 4, 96),
+                                                       ("cifar", 100, 256, 32)])  # the CIFAR step at its batch
 def test_every_layer_of_the_step(variant, classes, batch, res):
     load_dbl()
     from paper_2509_26092_gb300 import resnet18 as R
