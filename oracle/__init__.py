@@ -40,6 +40,13 @@ def lib():
         L.orc_round_bf16.argtypes = [_d]
         L.orc_round_bf16.restype = _d
         L.orc_round_bf16_array.argtypes = [_D, _i64]
+        L.orc_round_f16.argtypes = [_d]
+        L.orc_round_f16.restype = _d
+        L.orc_round_f16_array.argtypes = [_D, _i64]
+        L.orc_ps_merge_scaled.argtypes = [_D, _D, _D, _D, _i64, _d, _d, _d, _d, _i, _d, _d]
+        L.orc_ps_merge_scaled.restype = _i
+        L.orc_loss_scale_update.argtypes = [_D, ctypes.POINTER(ctypes.c_int), _i, _i]
+        L.orc_loss_scale_update.restype = None
         L.orc_bn_fwd.argtypes = [_D, _i64, _i, _D, _D, _d, _D, _i, _D, _D, _D]
         L.orc_bn_bwd.argtypes = [_D, _D, _D, _i, _D, _i64, _i, _D, _D, _D, _D, _D, _D, _D]
         L.orc_maxpool_fwd.argtypes = [_D, _i, _i, _i, _i, _i, _i, _i, _D, _I32]
@@ -87,6 +94,13 @@ def round_bf16(a):
     """Round-to-nearest-even onto the bfloat16 grid (returned as float64)."""
     a = _f64(a).copy()
     lib().orc_round_bf16_array(_p(a), a.size)
+    return a
+
+
+def round_f16(a):
+    """Round-to-nearest-even onto the IEEE binary16 grid (returned as float64)."""
+    a = _f64(a).copy()
+    lib().orc_round_f16_array(_p(a), a.size)
     return a
 
 
@@ -267,6 +281,25 @@ def ps_merge(w, u, g_large, g_small, lr, momentum, f_large, f_small, order=0):
     gs = None if g_small is None else _f64(g_small)
     lib().orc_ps_merge(_p(w), _p(u), _p(gl), _p(gs), w.size, lr, momentum, f_large, f_small, order)
     return w, u
+
+
+def ps_merge_scaled(w, u, g_large, g_small, lr, momentum, f_large, f_small, order, scale_large, scale_small):
+    """The merge of pushes made under loss scaling (see orc_ps_merge_scaled): returns new
+    (w, u, applied); applied is False (and w, u unchanged) when a pushed value is not finite."""
+    w, u = _f64(w).copy(), _f64(u).copy()
+    gl = None if g_large is None else _f64(g_large)
+    gs = None if g_small is None else _f64(g_small)
+    ok = lib().orc_ps_merge_scaled(_p(w), _p(u), _p(gl), _p(gs), w.size, lr, momentum, f_large, f_small, order,
+                                   float(scale_large), float(scale_small))
+    return w, u, bool(ok)
+
+
+def loss_scale_update(scale, good, found_inf, interval):
+    """One step of the dynamic loss scale; returns (scale, good)."""
+    s_ = ctypes.c_double(scale)
+    g_ = ctypes.c_int(good)
+    lib().orc_loss_scale_update(ctypes.byref(s_), ctypes.byref(g_), int(bool(found_inf)), int(interval))
+    return s_.value, g_.value
 
 
 # --------------------------------------------------------------------------- resize

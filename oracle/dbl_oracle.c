@@ -60,6 +60,33 @@ double orc_round_bf16(double x)
     return y;
 }
 
+/* ------------------------------------------------------------------------ */
+/* fp16 (IEEE 754 binary16) storage rounding, for the mixed-precision runs   */
+/* of the paper's ImageNet experiments (Sec. 5.2.3).  binary16 has a 5-bit   */
+/* exponent and 11 significand bits (10 stored): for |x| in [2^(e-1), 2^e)   */
+/* with e - 1 >= -14 the quantum is 2^(e-11); below 2^-14 (subnormals) it is */
+/* fixed at 2^-24.  Round to nearest, ties to even; the largest finite value */
+/* is 65504 = (2 - 2^-10) * 2^15, and anything that rounds above it is       */
+/* infinite.                                                                 */
+/* ------------------------------------------------------------------------ */
+double orc_round_f16(double x)
+{
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    frexp(x, &e); /* |x| in [2^(e-1), 2^e) */
+    int qexp = e - 11;
+    if (e - 1 < -14) qexp = -24;
+    double r = nearbyint(ldexp(x, -qexp)); /* ties to even */
+    double y = ldexp(r, qexp);
+    if (fabs(y) > 65504.0) y = copysign(INFINITY, x);
+    return y;
+}
+
+void orc_round_f16_array(double* a, int64_t n)
+{
+    for (int64_t i = 0; i < n; ++i) a[i] = orc_round_f16(a[i]);
+}
+
 void orc_round_bf16_array(double* a, int64_t n)
 {
     for (int64_t i = 0; i < n; ++i) a[i] = orc_round_bf16(a[i]);
@@ -511,6 +538,48 @@ void orc_ps_merge(double* w, double* u, const double* gL, const double* gS, int6
         }
         w[i] = wi;
         u[i] = ui;
+    }
+}
+
+/* The merge under mixed precision with loss scaling (Micikevicius et al.,   */
+/* the method the paper cites for its fp16 runs, Sec. 5.2.3).  A worker      */
+/* computes its gradient from a loss multiplied by its scale S_i, so it      */
+/* pushes S_i * g_i; the server divides each push by its scale before the   */
+/* momentum update above.  If any pushed value is not finite (the scaled    */
+/* gradient overflowed fp16 somewhere), the server applies nothing: w and u  */
+/* are left as they are.  Returns 1 when the update was applied, 0 when it  */
+/* was skipped.                                                              */
+int orc_ps_merge_scaled(double* w, double* u, const double* gL, const double* gS, int64_t n, double lr, double mu,
+                        double fL, double fS, int order, double sL, double sS)
+{
+    for (int64_t i = 0; i < n; ++i)
+        if ((gL && !isfinite(gL[i])) || (gS && !isfinite(gS[i]))) return 0;
+    double* uL = gL ? (double*)malloc(sizeof(double) * (size_t)(n ? n : 1)) : NULL;
+    double* uS = gS ? (double*)malloc(sizeof(double) * (size_t)(n ? n : 1)) : NULL;
+    for (int64_t i = 0; i < n; ++i) {
+        if (uL) uL[i] = gL[i] / sL;
+        if (uS) uS[i] = gS[i] / sS;
+    }
+    orc_ps_merge(w, u, uL, uS, n, lr, mu, fL, fS, order);
+    free(uL);
+    free(uS);
+    return 1;
+}
+
+/* Dynamic loss scale: after a step whose gradients overflowed, halve the   */
+/* scale and restart the count of good steps; after `interval` good steps   */
+/* in a row, double it.                                                     */
+void orc_loss_scale_update(double* scale, int* good, int found_inf, int interval)
+{
+    if (found_inf) {
+        *scale = *scale / 2.0;
+        *good = 0;
+        return;
+    }
+    *good += 1;
+    if (*good >= interval) {
+        *scale = *scale * 2.0;
+        *good = 0;
     }
 }
 

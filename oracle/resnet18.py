@@ -34,7 +34,8 @@ import math
 import numpy as np
 
 from . import (avgpool_bwd, avgpool_fwd, bilinear_resize, bn_bwd, bn_fwd, conv2d_dgrad, conv2d_fwd, conv2d_wgrad,
-               dropout_apply, dropout_mask, fc_bwd, fc_fwd, maxpool_bwd, maxpool_fwd, ps_merge, round_bf16, softmax_ce)
+               dropout_apply, dropout_mask, fc_bwd, fc_fwd, maxpool_bwd, maxpool_fwd, ps_merge, ps_merge_scaled,
+               round_bf16, round_f16, softmax_ce)
 
 WIDTHS = (64, 128, 256, 512)
 
@@ -80,11 +81,14 @@ def n_params(variant, classes, widths=WIDTHS):
 
 
 class _Rounder:
-    def __init__(self, on):
-        self.on = on
+    """Rounding at the points where the GPU stores 16-bit values: bf16, fp16 (IEEE binary16),
+    or none (fp64 throughout)."""
+
+    def __init__(self, mode):
+        self.fn = {"bf16": round_bf16, "f16": round_f16, None: None}[mode]
 
     def __call__(self, a):
-        return round_bf16(a) if self.on else a
+        return self.fn(a) if self.fn else a
 
 
 def _check_params(params, variant, classes, widths):
@@ -95,18 +99,23 @@ def _check_params(params, variant, classes, widths):
             raise ValueError(f"{name}: shape {params[name].shape} != {shape}")
 
 
-def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths=WIDTHS, keep=False, dropout=None):
+def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths=WIDTHS, keep=False, dropout=None,
+               storage="", loss_scale=1.0):
     """One worker's forward + backward on a batch.
 
     params: dict name -> fp32-valued array (the master weights the worker pulled);
     img: [N, H, W, 3] float, already at the training resolution; labels: [N] int.
     dropout: None, or (d, seed, step): dropout of rate d on the pooled features before
     the FC layer (Sec. 4.1), with the mask of ``dropout_mask(N, C, d, seed, step)``.
+    storage: "bf16", "f16" or None picks the 16-bit format rounded to at the GPU's storage
+    points (the default "" follows bf16_storage).  loss_scale: the backward pass starts from
+    loss_scale * dloss, as mixed-precision training with loss scaling does (Sec. 5.2.3), so
+    the returned gradients are loss_scale times the loss's; the loss itself is unscaled.
     Returns dict(loss=float, grads={name: array}, acts={...} if keep).
     """
     classes = params["fc.w"].shape[0]
     _check_params(params, variant, classes, widths)
-    R = _Rounder(bf16_storage)
+    R = _Rounder(storage if storage != "" else ("bf16" if bf16_storage else None))
     P = {k: np.asarray(v, dtype=np.float64) for k, v in params.items()}
     wq = {k: R(v) for k, v in P.items() if k.endswith(".w") and v.ndim == 4}  # bf16 conv weights
     acts = {}
@@ -161,6 +170,7 @@ def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths
         feat = dropout_apply(feat, mask, dropout[0])
     logits = fc_fwd(feat, P["fc.w"], P["fc.b"])
     loss, dl = softmax_ce(logits, labels)
+    dl = dl * loss_scale
 
     grads = {}
     grads["fc.w"], grads["fc.b"], dfeat = fc_bwd(dl, feat, P["fc.w"])
@@ -211,13 +221,16 @@ def train_step(params, img, labels, variant, bf16_storage=True, eps=1e-5, widths
 
 def dual_batch_iteration(params, velocity, img_large, labels_large, img_small, labels_small, resolution, variant,
                          lr, momentum, f_large, f_small, order=0, bf16_storage=True, widths=WIDTHS,
-                         dropout_large=None, dropout_small=None):
+                         dropout_large=None, dropout_small=None, storage="", loss_scale=None):
     """One emulated parameter-server iteration of the hybrid scheme (Sec. 3-4).
 
     Both workers pull the same model version, resize their images to the
     sub-stage resolution (Sec. 4.1), run one training step each, and the server
     applies their pushes with the model-update factors (Sec. 3.4).
     dropout_large / dropout_small: each worker's (d, seed, step) for ``train_step``, or None.
+    loss_scale: None, or the scale both workers multiply their loss by (storage then usually
+    "f16"); the server divides each push by it and skips the update if a pushed value is not
+    finite (``ps_merge_scaled``).
     Returns (new_params, new_velocity, loss_large, loss_small, grads_large, grads_small).
     """
     out = {}
@@ -229,13 +242,25 @@ def dual_batch_iteration(params, velocity, img_large, labels_large, img_small, l
         x = np.asarray(img, dtype=np.float64)
         if x.shape[1] != resolution or x.shape[2] != resolution:
             x = bilinear_resize(x, resolution, resolution)
-        out[tag] = train_step(params, x, lab, variant, bf16_storage=bf16_storage, widths=widths, dropout=drop)
+        out[tag] = train_step(params, x, lab, variant, bf16_storage=bf16_storage, widths=widths, dropout=drop,
+                              storage=storage, loss_scale=1.0 if loss_scale is None else loss_scale)
     new_w, new_u = {}, {}
+    if loss_scale is not None:
+        # one server decision for the whole push: any non-finite value anywhere skips the update
+        finite = all(np.all(np.isfinite(out[t]["grads"][name])) for t in ("L", "S") if out[t] for name in params)
+        if not finite:
+            return (dict(params), dict(velocity), out["L"]["loss"] if out["L"] else None,
+                    out["S"]["loss"] if out["S"] else None, out["L"]["grads"] if out["L"] else None,
+                    out["S"]["grads"] if out["S"] else None)
     for name in params:
         gl = out["L"]["grads"][name] if out["L"] else None
         gs = out["S"]["grads"][name] if out["S"] else None
-        new_w[name], new_u[name] = ps_merge(params[name], velocity[name], gl, gs, lr, momentum, f_large, f_small,
-                                            order)
+        if loss_scale is not None:
+            new_w[name], new_u[name], _ = ps_merge_scaled(params[name], velocity[name], gl, gs, lr, momentum,
+                                                          f_large, f_small, order, loss_scale, loss_scale)
+        else:
+            new_w[name], new_u[name] = ps_merge(params[name], velocity[name], gl, gs, lr, momentum, f_large,
+                                                f_small, order)
     return (new_w, new_u, out["L"]["loss"] if out["L"] else None, out["S"]["loss"] if out["S"] else None,
             out["L"]["grads"] if out["L"] else None, out["S"]["grads"] if out["S"] else None)
 
