@@ -249,7 +249,7 @@ def run_reference(args, cfg):
 
 
 # ------------------------------------------------------------------------------------------ GPU arm
-def build_pipeline(cfg, device):
+def build_pipeline(cfg, device, precision="bf16"):
     import torch
 
     from paper_2509_26092_gb300 import dbl as D
@@ -257,7 +257,8 @@ def build_pipeline(cfg, device):
     from paper_2509_26092_gb300 import synth
 
     spec = R.ResNet18Spec(cfg["variant"], cfg["classes"])
-    server = R.ServerState(spec, synth.params(spec.table(), seed=0), synth.momentum_state(spec.table(), 0.0, seed=0))
+    server = R.ServerState(spec, synth.params(spec.table(), seed=0), synth.momentum_state(spec.table(), 0.0, seed=0),
+                           precision=precision)
     bl_max = max(cfg["large"])
     bs_max = max([b for b in cfg["small"] if b] or [0])
     nat = cfg["native"]
@@ -268,8 +269,9 @@ def build_pipeline(cfg, device):
     lab_s = torch.from_numpy(synth.labels(bs_max, cfg["classes"], seed=1, name="small")).pin_memory() if bs_max else None
     stages = []
     for res, bl, bs, drop in zip(cfg["stages"], cfg["large"], cfg["small"], cfg["dropout"]):
-        large = R.Worker(spec, bl, res, device, dropout=drop, dropout_seed=2 * res + 1)
-        small = R.Worker(spec, bs, res, device, dropout=drop, dropout_seed=2 * res + 2) if bs else None
+        large = R.Worker(spec, bl, res, device, dropout=drop, dropout_seed=2 * res + 1, precision=precision)
+        small = (R.Worker(spec, bs, res, device, dropout=drop, dropout_seed=2 * res + 2, precision=precision)
+                 if bs else None)
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_large=1.0, f_small=F_SMALL)
         it.set_inputs(host_l[:bl].to(device), lab_l[:bl].to(device),
                       host_s[:bs].to(device) if bs else None, lab_s[:bs].to(device) if bs else None)
@@ -543,7 +545,7 @@ def run_ours(args, cfg):
     build_lib.build()
     from paper_2509_26092_gb300 import dbl as D
 
-    pipe = build_pipeline(cfg, device)
+    pipe = build_pipeline(cfg, device, args.precision)
     stages = pipe["stages"]
     images_per_step = sum(s["images"] for s in stages)
 
@@ -636,7 +638,8 @@ def run_ours(args, cfg):
         if wk is not None:
             wk._bench_w16 = pipe["server"].w16
     table = [] if args.conv_table else None
-    flops, secs, algo_bytes = conv_roofline(top, table=table)
+    with D.precision(args.precision):
+        flops, secs, algo_bytes = conv_roofline(top, table=table)
     if table is not None:
         for b, name, pname, f1, t1 in table:
             print(f"conv {b:4d} {name:16s} {pname:5s} {t1 * 1e6:9.1f} us {f1 / t1 / 1e12:7.1f} TFLOP/s",
@@ -652,7 +655,8 @@ def run_ours(args, cfg):
                           f"split-K reduce kernels (fwd/dgrad/wgrad, every layer of both workers at {top['res']} px, "
                           "each pass timed alone as CUDA-graph replays of its ABI calls)",
                 "peak_source": src}
-    bw = bandwidth_kernels(pipe, hbm)
+    with D.precision(args.precision):
+        bw = bandwidth_kernels(pipe, hbm)
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         v, dt, images, sample = time_oracle(cfg)
@@ -663,8 +667,10 @@ def run_ours(args, cfg):
     if rank == 0:
         line = {"metric": METRIC, "value": round(value, 1), "unit": "images/s", "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3), "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": args.config, "description": cfg["desc"],
+                "scaling": "weak", "vs_baseline": None, "dtype": args.precision, "data": "synthetic",
+                "config": {"workload": args.config, "description": cfg["desc"], "precision": args.precision,
+                           "loss_scaling": ("dynamic: initial 2^15, halved on overflow, doubled after 2000 good "
+                                            "steps" if args.precision == "f16" else None),
                            "stages_px": list(cfg["stages"]), "large_batch": list(cfg["large"]),
                            "small_batch": list(cfg["small"]), "dropout": list(cfg["dropout"]),
                            "images_per_step": images_per_step,
@@ -694,6 +700,8 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "f16"],
+                    help="16-bit storage format: bf16, or f16 with dynamic loss scaling (the paper's mixed precision)")
     ap.add_argument("--conv-table", action="store_true",
                     help="print each convolution pass's time and TFLOP/s (largest stage) to stderr")
     ap.add_argument("--profile-conv", default=None, metavar="LAYER:PASS",

@@ -22,6 +22,15 @@
  *  - Kernels that wait on an asynchronous copy give up after a bounded time,
  *    record DBL_ERR_TIMEOUT in a device-side status word and return; read it
  *    with dbl_device_status().
+ *  - Storage format.  The library is built twice from the same sources, with
+ *    the same entry points: libdbl.so stores activations, activation gradients
+ *    and the convolutions' weight copies as bfloat16; libdbl_f16.so (built
+ *    with DBL_ACT_F16) stores them as IEEE binary16, the format of the
+ *    paper's mixed-precision ImageNet runs (Sec. 5.2.3), to be used with the
+ *    loss scaling below.  Every parameter named *_bf16 (and DBL_BF16) denotes
+ *    the library's 16-bit format; fp32 arguments are fp32 in both.  The
+ *    tensor cores multiply the two operands in that one format (never mixed)
+ *    and accumulate in fp32.
  */
 #ifndef DBL_H
 #define DBL_H
@@ -292,25 +301,37 @@ DBL_API int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, 
                      const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx_bf16,
                      void* ws, size_t ws_bytes, void* stream);
 
-/* Head with dropout of the pooled features before the FC layer.  Cyclic
- * progressive learning raises the dropout rate d with the resolution of each
- * sub-stage (Sec. 4.1; 0.1 / 0.2 / 0.3 in Tables 7 and 9).  Inverted dropout:
- *   featd[n,c] = feat[n,c] * keep[n,c] / (1 - d),
- * logits, loss, dfc_w, dfc_b as dbl_head_fwd_bwd with featd in place of feat,
- * and dx[n,i,c] = (dlogits*fc_w)[n,c] * keep[n,c] / (1 - d) / hw.
- * keep[n,c] is the mask dbl_dropout_mask writes for the same (d, seed, *step)
- * (a counter-based draw, so the mask depends on nothing else).  step: device
- * pointer to one uint64 (8-byte aligned) read by the kernels; after the call's
- * last kernel it is incremented by one on the stream, so consecutive calls
- * (and replays of a captured graph) draw fresh masks.  drop_rate = 0 is
- * dbl_head_fwd_bwd exactly (step may then be NULL and is not touched).
- * drop_rate outside [0, 1): DBL_ERR_INVALID.  Workspace as dbl_head_fwd_bwd. */
-DBL_API int dbl_head_fwd_bwd_dropout(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x_bf16,
-                                     const float* fc_w, const float* fc_b, const int32_t* labels, float drop_rate,
-                                     uint64_t seed, uint64_t* step, float* loss, float* dfc_w, float* dfc_b,
-                                     void* dx_bf16, void* ws, size_t ws_bytes, void* stream);
+/* Head with the options of the hybrid scheme's training step:
+ *  - dropout of the pooled features before the FC layer.  Cyclic progressive
+ *    learning raises the dropout rate d with the resolution of each sub-stage
+ *    (Sec. 4.1; 0.1 / 0.2 / 0.3 in Tables 7 and 9).  Inverted dropout:
+ *      featd[n,c] = feat[n,c] * keep[n,c] / (1 - d),
+ *    logits, loss, dfc_w, dfc_b as dbl_head_fwd_bwd with featd in place of
+ *    feat, and dx[n,i,c] = (dlogits*fc_w)[n,c] * keep[n,c] / (1 - d) / hw, with
+ *    keep[n,c] the mask dbl_dropout_mask writes for the same (d, seed, *step).
+ *    step: device pointer to one uint64 (8-byte aligned) read by the kernels;
+ *    after the call's last kernel it is incremented by one on the stream, so
+ *    consecutive calls (and replays of a captured graph) draw fresh masks.
+ *    drop_rate = 0: no dropout (step may be NULL and is not touched);
+ *    outside [0, 1): DBL_ERR_INVALID.
+ *  - loss scaling for mixed-precision training (Sec. 5.2.3): loss_scale is a
+ *    device pointer to one fp32 S read by the kernels (NULL: S = 1); the
+ *    backward pass starts from dlogits = (softmax - onehot) * S/n, so dfc_w,
+ *    dfc_b and dx (and every gradient computed from dx) are S times the
+ *    loss's gradients.  loss is reported unscaled.
+ * With drop_rate 0 and loss_scale NULL this is dbl_head_fwd_bwd exactly.
+ * Workspace as dbl_head_fwd_bwd. */
+typedef struct {
+    float drop_rate;
+    uint64_t seed;
+    uint64_t* step;
+    const float* loss_scale;
+} dbl_head_opts;
+DBL_API int dbl_head_fwd_bwd_ex(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x_bf16, const float* fc_w,
+                                const float* fc_b, const int32_t* labels, const dbl_head_opts* opts, float* loss,
+                                float* dfc_w, float* dfc_b, void* dx_bf16, void* ws, size_t ws_bytes, void* stream);
 
-/* The dropout mask of dbl_head_fwd_bwd_dropout: keep[n,c] (uint8, 1 = kept)
+/* The dropout mask of dbl_head_fwd_bwd_ex: keep[n,c] (uint8, 1 = kept)
  * for n samples of c features (c a multiple of 4; keep 4-byte aligned).
  * Feature c of sample n takes word c % 4 of the Philox4x64-10 block (Salmon
  * et al., SC 2011) at counter (n*c/4 + c/4, *step, 0, 0) with key (seed, 0),
@@ -339,6 +360,36 @@ typedef struct {
 
 DBL_API int dbl_ps_dual_batch_merge(float* w, float* u, void* w16_out, const float* g_large, const float* g_small, int64_t n,
                             const dbl_merge_params* params, void* stream);
+
+/* The merge under mixed precision with loss scaling (Micikevicius et al., the
+ * method of the paper's fp16 runs, Sec. 5.2.3).  A worker that scaled its loss
+ * by S_i pushes S_i * g_i; this merge divides each push by its scale
+ * (scale_large / scale_small: device pointers to the fp32 scale each worker
+ * used; required for each non-NULL push), then applies the update of
+ * dbl_ps_dual_batch_merge.  If *found_inf (device int32) is non-zero, nothing
+ * is written: w, u and w16 keep their values.  Scales are powers of two (the
+ * dynamic scale below keeps them so), so the division is exact. */
+DBL_API int dbl_ps_dual_batch_merge_scaled(float* w, float* u, void* w16_out, const float* g_large,
+                                           const float* g_small, int64_t n, const dbl_merge_params* params,
+                                           const float* scale_large, const float* scale_small,
+                                           const int32_t* found_inf, void* stream);
+
+/* Sets *found_inf (device int32) to 1 if any of g[0, n) (fp32, device, 16-byte
+ * aligned) is infinite or NaN; never clears it. */
+DBL_API int dbl_grads_finite(const float* g, int64_t n, int32_t* found_inf, void* stream);
+
+/* Dynamic loss scale, in device memory (16 bytes).  After the merge of a step:
+ * if found_inf, the scale halves, good_steps restarts at 0 and skipped counts
+ * the skipped update; otherwise good_steps counts up, and the scale doubles
+ * when it reaches growth_interval (then restarts).  found_inf is cleared.
+ * One thread, stream ordered. */
+typedef struct {
+    float scale;
+    int32_t good_steps;
+    int32_t found_inf;
+    int32_t skipped;
+} dbl_loss_scale;
+DBL_API int dbl_loss_scale_update(dbl_loss_scale* state, int32_t growth_interval, void* stream);
 
 /* Late and missing pushes.  Under ASP the server applies each push as it
  * arrives and does not wait for a worker that has stopped (Sec. 2.4); a

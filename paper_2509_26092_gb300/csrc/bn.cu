@@ -27,10 +27,10 @@ constexpr int kReduceUnroll = 4;
 
 __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 {
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+    const act2_t* h = reinterpret_cast<const act2_t*>(&v);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        const float2 t = __bfloat1622float2(h[k]);
+        const float2 t = dbl::act::unpack2(h[k]);
         f[2 * k] = t.x;
         f[2 * k + 1] = t.y;
     }
@@ -39,14 +39,14 @@ __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 __device__ __forceinline__ uint4 pack8(const float (&f)[8])
 {
     uint4 v;
-    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
+    act2_t* h = reinterpret_cast<act2_t*>(&v);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(f[2 * k], f[2 * k + 1]);
+    for (int k = 0; k < 4; ++k) h[k] = dbl::act::pack2(f[2 * k], f[2 * k + 1]);
     return v;
 }
 
 // ----------------------------------------------------------------------------- statistics
-__global__ void __launch_bounds__(kThreads) bn_stats_kernel(const __nv_bfloat16* __restrict__ y, int64_t count, int C,
+__global__ void __launch_bounds__(kThreads) bn_stats_kernel(const act_t* __restrict__ y, int64_t count, int C,
                                                             float* __restrict__ sum, float* __restrict__ sumsq)
 {
     const int groups = C / 8;
@@ -128,8 +128,8 @@ __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_pa
 // consecutive vectors of consecutive rows, so every access is coalesced, and the
 // channel's scale and shift stay in registers.
 __global__ void __launch_bounds__(kThreads, kBlocksPerSM)
-    bn_apply_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ res,
-                    __nv_bfloat16* __restrict__ out, int count, int C, int relu, const float* __restrict__ gamma,
+    bn_apply_kernel(const act_t* __restrict__ y, const act_t* __restrict__ res,
+                    act_t* __restrict__ out, int count, int C, int relu, const float* __restrict__ gamma,
                     const float* __restrict__ beta, const float* __restrict__ mean, const float* __restrict__ invstd)
 {
     const int groups = C / 8;
@@ -187,8 +187,8 @@ struct Vec8 {
 };
 
 template <int MASK>
-__device__ __forceinline__ void load_g_raw(const __nv_bfloat16* dout, const __nv_bfloat16* dout2,
-                                           const __nv_bfloat16* out, const __nv_bfloat16* y, int v, Vec8& g, Vec8& yv)
+__device__ __forceinline__ void load_g_raw(const act_t* dout, const act_t* dout2,
+                                           const act_t* out, const act_t* y, int v, Vec8& g, Vec8& yv)
 {
     g.d = __ldcs(reinterpret_cast<const uint4*>(dout) + v);
     g.d2 = dout2 ? __ldcs(reinterpret_cast<const uint4*>(dout2) + v) : make_uint4(0, 0, 0, 0);
@@ -241,7 +241,7 @@ __device__ __forceinline__ void combine_g(const Vec8& raw, const float (&y)[8], 
 template <int MASK, bool WRITE_G>
 __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw, bool two, const ReluMask<MASK>& relu,
                                              const float (&mu)[8], float (&sg)[8], float (&sgc)[8],
-                                             __nv_bfloat16* g_out, int v)
+                                             act_t* g_out, int v)
 {
     float gg[8], yy[8];
     unpack8(yraw.y, yy);
@@ -262,11 +262,11 @@ __device__ __forceinline__ void accumulate_g(const Vec8& graw, const Vec8& yraw,
 // result does not depend on the grid.
 template <int MASK, bool WRITE_G>
 __global__ void __launch_bounds__(kThreads, kReduceBlocksPerSM)
-    bn_bwd_reduce_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
-                         const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
+    bn_bwd_reduce_kernel(const act_t* __restrict__ dout, const act_t* __restrict__ dout2,
+                         const act_t* __restrict__ out, const act_t* __restrict__ y, int count,
                          int C, const float* __restrict__ gamma, const float* __restrict__ beta,
                          const float* __restrict__ mean, const float* __restrict__ invstd, int nblk,
-                         float* __restrict__ partial, __nv_bfloat16* __restrict__ g_out)
+                         float* __restrict__ partial, act_t* __restrict__ g_out)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
@@ -345,11 +345,11 @@ __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_bwd_finalize_ke
 
 template <int MASK>
 __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
-    bn_bwd_apply_kernel(const __nv_bfloat16* __restrict__ dout, const __nv_bfloat16* __restrict__ dout2,
-                        const __nv_bfloat16* __restrict__ out, const __nv_bfloat16* __restrict__ y, int count,
+    bn_bwd_apply_kernel(const act_t* __restrict__ dout, const act_t* __restrict__ dout2,
+                        const act_t* __restrict__ out, const act_t* __restrict__ y, int count,
                         int C, const float* __restrict__ gamma, const float* __restrict__ beta,
                         const float* __restrict__ mean, const float* __restrict__ invstd,
-                        const float* __restrict__ coef, __nv_bfloat16* __restrict__ dy, __nv_bfloat16* __restrict__ dres)
+                        const float* __restrict__ coef, act_t* __restrict__ dy, act_t* __restrict__ dres)
 {
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
@@ -440,10 +440,10 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
 {
     using namespace dbl;
     const int C = s->c;
-    auto bd = [](const void* p) { return static_cast<const __nv_bfloat16*>(p); };
+    auto bd = [](const void* p) { return static_cast<const act_t*>(p); };
     // When the caller wants g (the residual branch's gradient), the reduce pass stores it and the
     // apply pass reads it back instead of re-reading dout, dout2 and out.
-    __nv_bfloat16* g_store = static_cast<__nv_bfloat16*>(dresidual);
+    act_t* g_store = static_cast<act_t*>(dresidual);
     if (g_store)
         bn_bwd_reduce_kernel<MASK, true><<<reduce_grid(nblk), kThreads, 0, st>>>(
             bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, (int)nblk, partial,
@@ -461,11 +461,11 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
     if (g_store)
         bn_bwd_apply_kernel<kMaskNone><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
             g_store, nullptr, nullptr, bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
-            static_cast<__nv_bfloat16*>(dy), nullptr);
+            static_cast<act_t*>(dy), nullptr);
     else
         bn_bwd_apply_kernel<MASK><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
             bd(dout), bd(dout2), bd(out), bd(y), (int)s->count, C, gamma, beta, mean, invstd, coef,
-            static_cast<__nv_bfloat16*>(dy), nullptr);
+            static_cast<act_t*>(dy), nullptr);
     return launch_check("bn_bwd_apply launch");
 }
 
@@ -510,7 +510,7 @@ int dbl_bn_stats(const dbl_bn_shape* s, const void* y, float* ch_sum, float* ch_
     if ((rc = cuda_check(cudaMemsetAsync(ch_sum, 0, sizeof(float) * s->c, st), "bn_stats memset"))) return rc;
     if ((rc = cuda_check(cudaMemsetAsync(ch_sumsq, 0, sizeof(float) * s->c, st), "bn_stats memset"))) return rc;
     if (s->count == 0) return DBL_OK;
-    bn_stats_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(y), s->count,
+    bn_stats_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(static_cast<const act_t*>(y), s->count,
                                                                        s->c, ch_sum, ch_sumsq);
     return launch_check("bn_stats launch");
 }
@@ -530,8 +530,8 @@ int dbl_bn_relu_fused(const dbl_bn_shape* s, const void* y, const float* ch_sum,
     cudaStream_t st = as_stream(stream);
     if ((rc = bn_fwd_finalize(s->count, s->c, s->eps, ch_sum, ch_sumsq, save_mean, save_invstd, st))) return rc;
     bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
-        static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
+        static_cast<const act_t*>(y), static_cast<const act_t*>(residual),
+        static_cast<act_t*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
     return launch_check("bn_relu_fused launch");
 }
 
@@ -554,8 +554,8 @@ int dbl_bn_relu_fused_parts(const dbl_bn_shape* s, const void* y, const float* p
                                                                    save_invstd);
     if ((rc = launch_check("bn_fwd_finalize_parts launch"))) return rc;
     bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(residual),
-        static_cast<__nv_bfloat16*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
+        static_cast<const act_t*>(y), static_cast<const act_t*>(residual),
+        static_cast<act_t*>(out), (int)s->count, s->c, s->relu, gamma, beta, save_mean, save_invstd);
     return launch_check("bn_relu_fused_parts launch");
 }
 

@@ -240,24 +240,25 @@ __device__ __forceinline__ void load_kblock(const ConvParams& p, const CUtensorM
     }
 }
 
-// Epilogue of the bf16-output passes for one 32-column chunk of this thread's
-// accumulator row: round to bf16 and store the row chunk (if the row is a real
+// Epilogue of the 16-bit-output passes for one 32-column chunk of this thread's
+// accumulator row: round to the storage format (bf16, or f16) and store the row chunk (if the row is a real
 // output); back[] receives the stored values (zeros for rows that are not outputs).
-__device__ __forceinline__ void store_row_chunk_bf16(const ConvParams& p, const uint32_t (&v)[32], bool valid,
+__device__ __forceinline__ void store_row_chunk_act(const ConvParams& p, const uint32_t (&v)[32], bool valid,
                                                      int64_t out_row, int col0, float (&back)[32])
 {
     uint4 pk[4];
     uint32_t* w32 = reinterpret_cast<uint32_t*>(pk);
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-        const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]));
-        const uint32_t u = valid ? *reinterpret_cast<const uint32_t*>(&h) : 0u;  // rows that are not outputs: 0
+        const uint32_t u = valid ? dbl::act::pack2_u32(__uint_as_float(v[2 * k]), __uint_as_float(v[2 * k + 1]))
+                                 : 0u;  // rows that are not outputs: 0
         w32[k] = u;
-        back[2 * k] = __uint_as_float(u << 16);            // bf16 -> fp32 is exact: the high half
-        back[2 * k + 1] = __uint_as_float(u & 0xFFFF0000u);
+        const float2 f = dbl::act::unpack2_u32(u);  // the stored values (16-bit -> fp32 is exact)
+        back[2 * k] = f.x;
+        back[2 * k + 1] = f.y;
     }
     if (valid) {
-        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + out_row * p.ldo + col0);
+        uint4* o = reinterpret_cast<uint4*>(static_cast<act_t*>(p.out) + out_row * p.ldo + col0);
 #pragma unroll
         for (int k = 0; k < 4; ++k) o[k] = pk[k];
     }
@@ -473,7 +474,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
         // ------------------------------------------------------------------ MMA issuer (whole warp, one lane issues)
         const bool a_mn = (p.mode == kWgrad || p.mode == kWgradC8);
         const bool b_mn = (p.mode != kFwd && p.mode != kFwdC8);
-        const uint32_t idesc = idesc_bf16(BM * CG, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
+        const uint32_t idesc = idesc_act(BM * CG, BN, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
         constexpr uint16_t kAll = CG == 2 ? 3 : 1;  // commits reach both CTAs of a pair
         // Operand descriptors without their start address, and the start-address steps
         // (in 16-byte units) per K-step and per accumulator:
@@ -546,14 +547,14 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
                 for (int j = 0; j < C::KSTEPS - 1; ++j) {
 #pragma unroll
                     for (int a = 0; a < C::ACC; ++a)
-                        mma_bf16_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + j * a_step16),
+                        mma_act_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + j * a_step16),
                                               bd0 + (uint64_t)(j * b_step16), idesc, (k > 0 || j > 0) ? 1u : 0u);
                 }
                 if (k + 1 < nkb) failed = !wait_ok(&full_bar[(it + 1) % STAGES], ((it + 1) / STAGES) & 1);
                 constexpr int jl = C::KSTEPS - 1;
 #pragma unroll
                 for (int a = 0; a < C::ACC; ++a)
-                    mma_bf16_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + jl * a_step16),
+                    mma_act_elect_cg<CG>(d + a * BN, ad0 + (uint64_t)(a * a_acc16 + jl * a_step16),
                                           bd0 + (uint64_t)(jl * b_step16), idesc, (k > 0 || jl > 0) ? 1u : 0u);
                 mma_commit_elect_cg<CG>(&empty_bar[s], kAll);
                 if (failed) {
@@ -643,7 +644,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
                             for (int k = 0; k < 32; ++k) v[k] = 0u;
                         }
                         float back[32];
-                        store_row_chunk_bf16(p, v, valid, out_row, tc.n_tile * BN + ch * 32, back);
+                        store_row_chunk_act(p, v, valid, out_row, tc.n_tile * BN + ch * 32, back);
                         if (want_stats) rs.add(ch, back, lane);
                     }
                 }
@@ -890,7 +891,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         }
     } else if (warp == C::W_MMA) {
         // ------------------------------------------------------------------ MMA issuer (rank 0 of a pair)
-        const uint32_t idesc = idesc_bf16(BM * CG, BN, 0u, DG ? 1u : 0u);
+        const uint32_t idesc = idesc_act(BM * CG, BN, 0u, DG ? 1u : 0u);
         int it = 0, bt = 0, lt = 0;
         bool failed = false;
         if (RES && (CG == 1 || rank == 0)) {
@@ -940,7 +941,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                     static_assert(kWinACC == 2, "two accumulators per MMA group");
                     const uint64_t ad = smem_desc(a0, 16, 1024, kSwizzle128B);
                     const uint64_t bd = DG ? smem_desc(sb, 8192, 1024, kSwizzle128B) : smem_desc(sb, 16, 1024, kSwizzle128B);
-                    mma_bf16_x8_elect_cg<CG>(d, d + BN, ad, (128 * 128) >> 4, 32 >> 4, bd, DG ? (2048 >> 4) : (32 >> 4),
+                    mma_act_x8_elect_cg<CG>(d, d + BN, ad, (128 * 128) >> 4, 32 >> 4, bd, DG ? (2048 >> 4) : (32 >> 4),
                                              idesc, (cb > 0 || tap > 0) ? 1u : 0u);
                     if (!RES) {
                         mma_commit_elect_cg<CG>(&bempty[bs], kAll);
@@ -1007,7 +1008,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
                 if (c + 1 < NC)
                     tmem_ld_32x32b_x32(taddr + (uint32_t)(((c + 1) / NCH) * BN + ((c + 1) % NCH) * 32), nxt);
                 float back[32];
-                store_row_chunk_bf16(p, cur, valid[a], out_row[a], col0 + ch * 32, back);
+                store_row_chunk_act(p, cur, valid[a], out_row[a], col0 + ch * 32, back);
                 if (want_stats) rs.add(ch, back, lane);
             }
             tc_fence_before();
@@ -1132,7 +1133,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         }
     } else if (warp == 6) {
         // ------------------------------------------------------------------ MMA issuer
-        const uint32_t idesc = idesc_bf16(BM, 64, 1u, 1u);
+        const uint32_t idesc = idesc_act(BM, 64, 1u, 1u);
         // strip-row offsets of each tap pair's two halves (the unused half of an odd last pair
         // reads the row after its first half), once per CTA
         int o0[NACC], o1[NACC];
@@ -1170,7 +1171,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     for (int pp = 0; pp < NACC; ++pp) {
                         const uint64_t ad = smem_desc(xa + (uint32_t)((off + o0[pp] + 16 * j) * 128),
                                                       (uint32_t)((o1[pp] - o0[pp]) * 128), 1024, kSwizzle128B);
-                        mma_bf16_elect(tmem + (uint32_t)(pp * 64), ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
+                        mma_act_elect(tmem + (uint32_t)(pp * 64), ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
                     }
                 }
                 mma_commit_elect(&empty_bar[s]);
@@ -1723,7 +1724,7 @@ int enc_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int
     cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
     int lo[2] = {lower_w, lower_h}, hi[2] = {upper_w, upper_h};
     cuuint32_t es[4] = {1, (cuuint32_t)stride_w, (cuuint32_t)stride_h, 1};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, lo, hi,
+    CUresult r = fn(m, (dbl::act::kF16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16), 4, const_cast<void*>(base), dims, strides, lo, hi,
                     (cuuint32_t)channels, (cuuint32_t)pixels, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -1737,7 +1738,7 @@ int enc_tiled(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims
     auto fn = dbl::encode_tiled();
     if (!fn) return dbl::set_error(DBL_ERR_CUDA, "conv: cuTensorMapEncodeTiled unavailable from the driver");
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims,
+    CUresult r = fn(m, (dbl::act::kF16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16), (cuuint32_t)rank, const_cast<void*>(base), dims,
                     strides_bytes, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);

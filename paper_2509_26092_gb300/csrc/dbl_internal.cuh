@@ -5,10 +5,12 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "../../include/dbl.h"
+#include "dbl_act.cuh"
 
 // ---------------------------------------------------------------------------- host-side errors
 namespace dbl {
@@ -542,7 +544,7 @@ __device__ __forceinline__ void tmem_dealloc_cg(uint32_t taddr, uint32_t ncols)
 // N/2..N-1 from rank 1, at the same addresses; D rows 0-127 land in rank 0's TMEM,
 // rows 128-255 in rank 1's, at the same column address.  Issued by rank 0 only.
 template <int CG>
-__device__ __forceinline__ void mma_bf16_elect_cg(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+__device__ __forceinline__ void mma_act_elect_cg(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                                   uint32_t accumulate)
 {
     if constexpr (CG == 2)
@@ -570,7 +572,7 @@ __device__ __forceinline__ void mma_bf16_elect_cg(uint32_t d_tmem, uint64_t a_de
 // if acc0 != 0; K-steps 1..3 always accumulate.  Keeping the whole group inside
 // one asm block (no per-MMA elect or predicate set-up in between) is what lets
 // N = 64 MMAs, which the tensor pipe finishes in 48 cycles, issue back to back.
-__device__ __forceinline__ void mma_bf16_x8_elect(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
+__device__ __forceinline__ void mma_act_x8_elect(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
                                                   uint64_t a_step, uint64_t b0, uint64_t b_step, uint32_t idesc,
                                                   uint32_t acc0)
 {
@@ -595,10 +597,10 @@ __device__ __forceinline__ void mma_bf16_x8_elect(uint32_t d0, uint32_t d1, uint
         : "memory");
 }
 
-// mma_bf16_x8_elect for CG-CTA MMAs (CG = 2: M = 256 across the pair, issued by rank 0,
-// A and B halves at the same shared-memory addresses in both CTAs, as in mma_bf16_elect_cg).
+// mma_act_x8_elect for CG-CTA MMAs (CG = 2: M = 256 across the pair, issued by rank 0,
+// A and B halves at the same shared-memory addresses in both CTAs, as in mma_act_elect_cg).
 template <int CG>
-__device__ __forceinline__ void mma_bf16_x8_elect_cg(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
+__device__ __forceinline__ void mma_act_x8_elect_cg(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1_off,
                                                      uint64_t a_step, uint64_t b0, uint64_t b_step, uint32_t idesc,
                                                      uint32_t acc0)
 {
@@ -623,7 +625,7 @@ __device__ __forceinline__ void mma_bf16_x8_elect_cg(uint32_t d0, uint32_t d1, u
             "r"(d1), "l"(a0), "l"(a1_off), "l"(a_step), "l"(b0), "l"(b_step), "r"(idesc), "r"(acc0)
             : "memory");
     else
-        mma_bf16_x8_elect(d0, d1, a0, a1_off, a_step, b0, b_step, idesc, acc0);
+        mma_act_x8_elect(d0, d1, a0, a1_off, a_step, b0, b_step, idesc, acc0);
 }
 
 // Elected-lane commit: arrive once on the mbarrier at shared::cta offset bar
@@ -669,8 +671,8 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// D[tmem] (+)= A[smem desc] * B[smem desc]^T, kind::f16 (bf16 inputs, fp32 accumulate).
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, kind::f16 (16-bit inputs of the storage format, fp32 accumulate).
+__device__ __forceinline__ void mma_act(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                          uint32_t accumulate)
 {
     asm volatile(
@@ -690,8 +692,8 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar)
 
 // Elected-lane forms: the whole warp calls, one lane issues.  The commit
 // tracks the MMAs issued by the elected lane, which is the same lane that
-// mma_bf16_elect uses in a converged warp.
-__device__ __forceinline__ void mma_bf16_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+// mma_act_elect uses in a converged warp.
+__device__ __forceinline__ void mma_act_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                                uint32_t accumulate)
 {
     asm volatile(
@@ -763,13 +765,14 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo_bytes
     return d;
 }
 
-// Instruction descriptor, kind::f16 with bf16 A/B and fp32 D.
+// Instruction descriptor, kind::f16 with A and B both in the storage format (bf16, or f16 in the
+// fp16 build: one MMA never mixes the two) and fp32 D.
 // a_mn / b_mn: 1 if that operand is MN-major (transposed) in shared memory.
-__host__ __device__ constexpr uint32_t idesc_bf16(uint32_t M, uint32_t N, uint32_t a_mn, uint32_t b_mn)
+__host__ __device__ constexpr uint32_t idesc_act(uint32_t M, uint32_t N, uint32_t a_mn, uint32_t b_mn)
 {
     return (1u << 4)            // D: fp32
-           | (1u << 7)          // A: bf16
-           | (1u << 10)         // B: bf16
+           | (dbl::act::kMmaFormat << 7)    // A: bf16 (1) or f16 (0), the storage format
+           | (dbl::act::kMmaFormat << 10)   // B: the same format as A
            | (a_mn << 15) | (b_mn << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 

@@ -16,10 +16,10 @@ namespace {
 
 __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 {
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+    const act2_t* h = reinterpret_cast<const act2_t*>(&v);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        const float2 t = __bfloat1622float2(h[k]);
+        const float2 t = dbl::act::unpack2(h[k]);
         f[2 * k] = t.x;
         f[2 * k + 1] = t.y;
     }
@@ -28,9 +28,9 @@ __device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8])
 __device__ __forceinline__ uint4 pack8(const float (&f)[8])
 {
     uint4 v;
-    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
+    act2_t* h = reinterpret_cast<act2_t*>(&v);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) h[k] = __floats2bfloat162_rn(f[2 * k], f[2 * k + 1]);
+    for (int k = 0; k < 4; ++k) h[k] = dbl::act::pack2(f[2 * k], f[2 * k + 1]);
     return v;
 }
 
@@ -43,8 +43,8 @@ int grid_for(int64_t items, int threads, int per_sm = 8)
 }
 
 // ----------------------------------------------------------------------------- max pool 3x3 / 2, pad 1
-__global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ x,
-                                                          __nv_bfloat16* __restrict__ y, uint8_t* __restrict__ arg,
+__global__ void __launch_bounds__(256) maxpool_fwd_kernel(const act_t* __restrict__ x,
+                                                          act_t* __restrict__ y, uint8_t* __restrict__ arg,
                                                           int n, int H, int W, int C, int P, int Q)
 {
     // 32-bit index math: the host checks that n*P*Q*C/8 fits
@@ -95,17 +95,18 @@ __global__ void __launch_bounds__(256) maxpool_fwd_kernel(const __nv_bfloat16* _
 // fp32 operations, and then pooled, so the pooled values and the argmax are
 // those of pooling the stored BatchNorm output.
 // One pair of channels of one input vector through BatchNorm + ReLU, as
-// bf16x2: each lane is bf16(y*scale + shift) from one fp32 fma, then
-// max(., 0) in bf16, which maps negatives and NaN to zero like the stored
+// 16-bit pairs of the storage format: each lane is the rounded y*scale + shift from one
+// fp32 fma, then max(., 0) in that format, which maps negatives and NaN to zero like the stored
 // pass's relu.  A result may be -0 where that pass stores +0; the pool's
 // comparisons treat the two alike and the stored maximum is made +0.
 __device__ __forceinline__ uint32_t bn_relu_pair(uint32_t w, float2 sc, float2 sh)
 {
-    const float o0 = __fmaf_rn(__uint_as_float(w << 16), sc.x, sh.x);
-    const float o1 = __fmaf_rn(__uint_as_float(w & 0xffff0000u), sc.y, sh.y);
+    const float2 x = dbl::act::unpack2_u32(w);
+    const float o0 = __fmaf_rn(x.x, sc.x, sh.x);
+    const float o1 = __fmaf_rn(x.y, sc.y, sh.y);
     uint32_t v;
-    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(v) : "f"(o1), "f"(o0));
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(v) : "r"(v), "r"(0u));
+    asm("cvt.rn." DBL_ACT_X2 ".f32 %0, %1, %2;" : "=r"(v) : "f"(o1), "f"(o0));
+    asm("max." DBL_ACT_X2 " %0, %1, %2;" : "=r"(v) : "r"(v), "r"(0u));
     return v;
 }
 
@@ -116,9 +117,9 @@ __device__ __forceinline__ uint32_t bn_relu_pair(uint32_t w, float2 sc, float2 s
 // it walks its windows by a fixed pixel stride with carries instead of
 // divisions.
 __global__ void __launch_bounds__(256)
-    bn_relu_maxpool_fwd_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ gamma,
+    bn_relu_maxpool_fwd_kernel(const act_t* __restrict__ x, const float* __restrict__ gamma,
                                const float* __restrict__ beta, const float* __restrict__ mean,
-                               const float* __restrict__ invstd, __nv_bfloat16* __restrict__ y,
+                               const float* __restrict__ invstd, act_t* __restrict__ y,
                                uint8_t* __restrict__ arg, int n, int H, int W, int C, int P, int Q)
 {
     const unsigned groups = (unsigned)C / 8u;
@@ -165,8 +166,8 @@ __global__ void __launch_bounds__(256)
                     for (int k = 0; k < 4; ++k) {
                         const uint32_t a = bn_relu_pair(w[k], sc[k], sh[k]);
                         uint32_t ge, m;
-                        asm("set.ge.u32.bf16x2 %0, %1, %2;" : "=r"(ge) : "r"(a), "r"(best[k]));
-                        asm("max.bf16x2 %0, %1, %2;" : "=r"(m) : "r"(best[k]), "r"(a));
+                        asm("set.ge.u32." DBL_ACT_X2 " %0, %1, %2;" : "=r"(ge) : "r"(a), "r"(best[k]));
+                        asm("max." DBL_ACT_X2 " %0, %1, %2;" : "=r"(m) : "r"(best[k]), "r"(a));
                         best[k] = m;
                         idx[k] = (ge & tap) | (~ge & idx[k]);
                     }
@@ -225,8 +226,8 @@ __device__ __forceinline__ void add_if_tap(float (&dst)[8], const float (&src)[8
 // zero.  A thread keeps one channel group and steps through the blocks with
 // carries, as in the forward pass.
 __global__ void __launch_bounds__(256)
-    maxpool_bwd_kernel(const __nv_bfloat16* __restrict__ dy, const __nv_bfloat16* __restrict__ dy2,
-                       const uint8_t* __restrict__ arg, __nv_bfloat16* __restrict__ dx, int n, int H, int W, int C,
+    maxpool_bwd_kernel(const act_t* __restrict__ dy, const act_t* __restrict__ dy2,
+                       const uint8_t* __restrict__ arg, act_t* __restrict__ dx, int n, int H, int W, int C,
                        int P, int Q)
 {
     const unsigned groups = (unsigned)C / 8u;
@@ -255,7 +256,7 @@ __global__ void __launch_bounds__(256)
             av[t] = ok[t] ? __ldg(reinterpret_cast<const uint2*>(arg + ot)) : make_uint2(~0u, ~0u);
         }
         const bool h1 = 2 * i + 1 < H, w1 = 2 * j + 1 < W;
-        __nv_bfloat16* px = dx + (((int64_t)b * H + 2 * i) * W + 2 * j) * C + 8 * g;
+        act_t* px = dx + (((int64_t)b * H + 2 * i) * W + 2 * j) * C + 8 * g;
         const int64_t px_row = (int64_t)W * C;
         float acc01[8] = {}, acc10[8] = {}, acc11[8] = {};
         {
@@ -384,7 +385,7 @@ __global__ void dropout_advance_kernel(uint64_t* step) { *step += 1; }
 
 // ----------------------------------------------------------------------------- head
 // feat[n, c] = mean over hw of x[n, hw, c], then (with dropout) times the feature's multiplier
-__global__ void __launch_bounds__(256) avgpool_kernel(const __nv_bfloat16* __restrict__ x, float* __restrict__ feat,
+__global__ void __launch_bounds__(256) avgpool_kernel(const act_t* __restrict__ x, float* __restrict__ feat,
                                                       int n, int hw, int C, Dropout dp)
 {
     const int groups = C / 8;
@@ -553,9 +554,10 @@ int gemm_f32(const float* A, int64_t sam, int64_t sak, const float* B, int64_t s
     return dbl::launch_check(what);
 }
 
-// One warp per row: loss_n = logsumexp(l) - l[label]; dl = (softmax - onehot)/n (in place).
+// One warp per row: loss_n = logsumexp(l) - l[label]; dl = (softmax - onehot) * S/n (in place), S the
+// loss scale (1 without loss scaling).
 __global__ void softmax_ce_kernel(float* __restrict__ logits, const int32_t* __restrict__ labels, int n, int J,
-                                  float* __restrict__ row_loss)
+                                  float* __restrict__ row_loss, const float* __restrict__ loss_scale)
 {
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
     if (warp >= n) return;
@@ -569,7 +571,7 @@ __global__ void softmax_ce_kernel(float* __restrict__ logits, const int32_t* __r
     const float lse = mx + logf(z);
     const int lab = labels[warp];
     if (lane == 0) row_loss[warp] = lse - l[lab];
-    const float invn = 1.0f / (float)n;
+    const float invn = (loss_scale ? *loss_scale : 1.0f) / (float)n;
     for (int j = lane; j < J; j += 32) l[j] = (expf(l[j] - lse) - (j == lab ? 1.f : 0.f)) * invn;
 }
 
@@ -598,7 +600,7 @@ __global__ void head_reduce_kernel(const float* __restrict__ row_loss, const flo
 }
 
 // dx[n, i, c] = df[n, c] / hw, with dropout (df[n, c] * mult[n, c]) / hw
-__global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, __nv_bfloat16* __restrict__ dx,
+__global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, act_t* __restrict__ dx,
                                                           int n, int hw, int C, const float* __restrict__ mult)
 {
     const int groups = C / 8;
@@ -635,7 +637,7 @@ int dbl_maxpool_fwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* x, v
         return set_error(DBL_ERR_UNSUPPORTED, "maxpool_fwd: tensor too large for 32-bit indexing");
     if (n == 0) return DBL_OK;
     maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q * (c / 8), 256), 256, 0, as_stream(stream)>>>(
-        static_cast<const __nv_bfloat16*>(x), static_cast<__nv_bfloat16*>(y), argmax, n, h, w, c, P, Q);
+        static_cast<const act_t*>(x), static_cast<act_t*>(y), argmax, n, h, w, c, P, Q);
     return launch_check("maxpool_fwd launch");
 }
 
@@ -662,7 +664,7 @@ int dbl_bn_relu_maxpool_fwd(const dbl_bn_shape* s, int32_t n, int32_t h, int32_t
     // a block size that is a multiple of the channel groups: each thread keeps its group
     const int groups = c / 8, block = groups * std::max(1, 256 / groups);
     bn_relu_maxpool_fwd_kernel<<<grid_for((int64_t)n * P * Q, block / groups), block, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(x), gamma, beta, save_mean, save_invstd, static_cast<__nv_bfloat16*>(y),
+        static_cast<const act_t*>(x), gamma, beta, save_mean, save_invstd, static_cast<act_t*>(y),
         argmax, n, h, w, c, P, Q);
     return launch_check("bn_relu_maxpool_fwd launch");
 }
@@ -685,8 +687,8 @@ int dbl_maxpool_bwd(int32_t n, int32_t h, int32_t w, int32_t c, const void* dy, 
     const int groups = c / 8, block = groups * std::max(1, 256 / groups);
     maxpool_bwd_kernel<<<grid_for((int64_t)n * ((h + 1) / 2) * ((w + 1) / 2), block / groups), block, 0,
                          as_stream(stream)>>>(
-        static_cast<const __nv_bfloat16*>(dy), static_cast<const __nv_bfloat16*>(dy2), argmax,
-        static_cast<__nv_bfloat16*>(dx), n, h, w, c, P, Q);
+        static_cast<const act_t*>(dy), static_cast<const act_t*>(dy2), argmax,
+        static_cast<act_t*>(dx), n, h, w, c, P, Q);
     return launch_check("maxpool_bwd launch");
 }
 
@@ -706,8 +708,9 @@ size_t dbl_head_workspace_bytes(int32_t n, int32_t c, int32_t classes)
 namespace {
 
 int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w, const float* fc_b,
-                 const int32_t* labels, float drop_rate, uint64_t seed, uint64_t* step, float* loss, float* dfc_w,
-                 float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream, const char* name)
+                 const int32_t* labels, float drop_rate, uint64_t seed, uint64_t* step, const float* loss_scale,
+                 float* loss, float* dfc_w, float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream,
+                 const char* name)
 {
     using namespace dbl;
     if (n <= 0 || hw <= 0 || c <= 0 || classes <= 0 || !x || !fc_w || !fc_b || !labels || !loss || !dfc_w || !dfc_b ||
@@ -734,13 +737,13 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
     }
     cudaStream_t s = as_stream(stream);
     int rc;
-    avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(x), feat, n,
+    avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const act_t*>(x), feat, n,
                                                                        hw, c, dp);
     if ((rc = launch_check("avgpool launch"))) return rc;
     // logits = feat * W^T + b
     if ((rc = gemm_f32(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c, part, s, "fc fwd launch")))
         return rc;
-    softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss);
+    softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss, loss_scale);
     if ((rc = launch_check("softmax_ce launch"))) return rc;
     head_reduce_kernel<<<1 + (classes + 255) / 256, 256, 0, s>>>(row_loss, logits, n, classes, loss, dfc_b);
     if ((rc = launch_check("head reduce launch"))) return rc;
@@ -751,7 +754,7 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
     if ((rc = gemm_f32(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes, part, s, "fc dX launch")))
         return rc;
     avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(
-        df, static_cast<__nv_bfloat16*>(dx), n, hw, c, dp.thr ? mult : nullptr);
+        df, static_cast<act_t*>(dx), n, hw, c, dp.thr ? mult : nullptr);
     if ((rc = launch_check("avgpool_bwd launch")) || !dp.thr) return rc;
     dropout_advance_kernel<<<1, 1, 0, s>>>(step);  // the next call draws a fresh mask
     return launch_check("dropout advance launch");
@@ -765,16 +768,17 @@ int dbl_head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const vo
                      const float* fc_b, const int32_t* labels, float* loss, float* dfc_w, float* dfc_b, void* dx,
                      void* ws, size_t ws_bytes, void* stream)
 {
-    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, 0.f, 0, nullptr, loss, dfc_w, dfc_b, dx, ws, ws_bytes,
-                        stream, "head_fwd_bwd");
+    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, 0.f, 0, nullptr, nullptr, loss, dfc_w, dfc_b, dx, ws,
+                        ws_bytes, stream, "head_fwd_bwd");
 }
 
-int dbl_head_fwd_bwd_dropout(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
-                             const float* fc_b, const int32_t* labels, float drop_rate, uint64_t seed, uint64_t* step,
-                             float* loss, float* dfc_w, float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream)
+int dbl_head_fwd_bwd_ex(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* x, const float* fc_w,
+                        const float* fc_b, const int32_t* labels, const dbl_head_opts* opts, float* loss, float* dfc_w,
+                        float* dfc_b, void* dx, void* ws, size_t ws_bytes, void* stream)
 {
-    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, drop_rate, seed, step, loss, dfc_w, dfc_b, dx, ws,
-                        ws_bytes, stream, "head_fwd_bwd_dropout");
+    if (!opts) return dbl::set_error(DBL_ERR_INVALID, "head_fwd_bwd_ex: null options");
+    return head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, opts->drop_rate, opts->seed, opts->step,
+                        opts->loss_scale, loss, dfc_w, dfc_b, dx, ws, ws_bytes, stream, "head_fwd_bwd_ex");
 }
 
 int dbl_dropout_mask(int32_t n, int32_t c, float drop_rate, uint64_t seed, const uint64_t* step, uint8_t* keep,

@@ -36,9 +36,9 @@ __device__ __forceinline__ float ld_in<float>(const float* p)
     return __ldg(p);
 }
 template <>
-__device__ __forceinline__ float ld_in<__nv_bfloat16>(const __nv_bfloat16* p)
+__device__ __forceinline__ float ld_in<act_t>(const act_t* p)
 {
-    return __bfloat162float(*p);
+    return dbl::act::to_f(*p);
 }
 
 // One thread per output pixel; channels 0..c-1 interpolated, c..cs-1 zeroed.
@@ -73,9 +73,9 @@ __global__ void __launch_bounds__(256) resize_kernel(const Tin* __restrict__ in,
         Tout* o = out + (int64_t)pix * cs;
         if constexpr (sizeof(Tout) == 2 && CMAX == 8) {
             if (cs == 8) {  // one 16-byte store per pixel
-                __nv_bfloat162 q[4];
+                act2_t q[4];
 #pragma unroll
-                for (int k = 0; k < 4; ++k) q[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+                for (int k = 0; k < 4; ++k) q[k] = dbl::act::pack2(v[2 * k], v[2 * k + 1]);
                 *reinterpret_cast<uint4*>(o) = *reinterpret_cast<uint4*>(q);
                 continue;
             }
@@ -83,7 +83,7 @@ __global__ void __launch_bounds__(256) resize_kernel(const Tin* __restrict__ in,
         for (int ch = 0; ch < cs; ++ch) {
             const float val = ch < CMAX ? v[ch < CMAX ? ch : 0] : 0.f;
             if constexpr (sizeof(Tout) == 2)
-                o[ch] = __float2bfloat16_rn(val);
+                o[ch] = dbl::act::from_f(val);
             else
                 o[ch] = val;
         }
@@ -138,7 +138,7 @@ __device__ __forceinline__ float stem_pixel<uint8_t>(const uint8_t* p, int ch, c
 }
 
 template <int RG, typename Tin>
-__global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict__ in, __nv_bfloat16* __restrict__ out,
+__global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict__ in, act_t* __restrict__ out,
                                                           int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
                                                           int32_t M, int32_t Q, int32_t taps, int32_t sw, int32_t pw,
                                                           int32_t ph, const PixelNorm nm)
@@ -219,11 +219,11 @@ __global__ void __launch_bounds__(256) resize_stem_kernel(const Tin* __restrict_
             f[0] = chunk < taps ? pp[0] : zero;
             f[1] = chunk < taps ? pp[1] : zero;
         }
-        __nv_bfloat162 qv[4];
-        qv[0] = __floats2bfloat162_rn(f[0].x, f[0].y);
-        qv[1] = __floats2bfloat162_rn(f[0].z, f[0].w);
-        qv[2] = __floats2bfloat162_rn(f[1].x, f[1].y);
-        qv[3] = __floats2bfloat162_rn(f[1].z, f[1].w);
+        act2_t qv[4];
+        qv[0] = dbl::act::pack2(f[0].x, f[0].y);
+        qv[1] = dbl::act::pack2(f[0].z, f[0].w);
+        qv[2] = dbl::act::pack2(f[1].x, f[1].y);
+        qv[3] = dbl::act::pack2(f[1].z, f[1].w);
         orow[idx] = *reinterpret_cast<uint4*>(qv);
     }
 }
@@ -259,11 +259,11 @@ int resize_stem_impl(const Tin* in, int32_t n, int32_t h_in, int32_t w_in, int32
     const size_t smem = (size_t)(w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels of fp32
     if (row_group == 2)
         resize_stem_kernel<2, Tin><<<blocks, 256, smem, as_stream(stream)>>>(
-            in, static_cast<__nv_bfloat16*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
+            in, static_cast<act_t*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
             nm);
     else
         resize_stem_kernel<1, Tin><<<blocks, 256, smem, as_stream(stream)>>>(
-            in, static_cast<__nv_bfloat16*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
+            in, static_cast<act_t*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
             nm);
     return launch_check("progressive_resize_stem launch");
 }
@@ -318,10 +318,10 @@ extern "C" int dbl_progressive_resize(const void* in, int in_dtype, int32_t n, i
     if (n == 0) return DBL_OK;
     cudaStream_t s = as_stream(stream);
     if (in_dtype == DBL_F32 && out_dtype == DBL_BF16)
-        return launch_resize<float, __nv_bfloat16>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+        return launch_resize<float, act_t>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
     if (in_dtype == DBL_F32 && out_dtype == DBL_F32)
         return launch_resize<float, float>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
     if (in_dtype == DBL_BF16 && out_dtype == DBL_BF16)
-        return launch_resize<__nv_bfloat16, __nv_bfloat16>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
-    return launch_resize<__nv_bfloat16, float>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+        return launch_resize<act_t, act_t>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
+    return launch_resize<act_t, float>(in, out, n, h_in, w_in, c, h_out, w_out, c_out_stride, s);
 }

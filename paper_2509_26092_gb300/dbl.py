@@ -1,4 +1,4 @@
-"""ctypes binding of ``libdbl.so`` (see ``include/dbl.h``).
+"""ctypes binding of ``libdbl.so`` and ``libdbl_f16.so`` (see ``include/dbl.h``).
 
 Argument marshalling only: every function here calls the C entry point of
 the same name, passing device pointers, sizes and the CUDA stream.  Tensors
@@ -6,7 +6,13 @@ may be given as torch tensors (their ``data_ptr()`` is passed) or as raw
 integer addresses.  A nonzero status raises ``DblError`` with the library's
 error text.  There is no fallback: if the library is not built, importing
 the functions fails.
+
+The two libraries differ only in the 16-bit storage format (bfloat16, or
+IEEE binary16); calls go to the bfloat16 one unless made inside
+``with precision("f16"):``.
 """
+import contextlib
+import contextvars
 import ctypes
 import os
 
@@ -40,12 +46,25 @@ class BnShape(ctypes.Structure):
     _fields_ = [("count", ctypes.c_int64), ("c", ctypes.c_int32), ("eps", ctypes.c_float), ("relu", ctypes.c_int32)]
 
 
+class HeadOpts(ctypes.Structure):
+    _fields_ = [("drop_rate", ctypes.c_float), ("seed", ctypes.c_uint64), ("step", ctypes.c_void_p),
+                ("loss_scale", ctypes.c_void_p)]
+
+
+class LossScale(ctypes.Structure):
+    """dbl_loss_scale: its device copy is a 4-element tensor (fp32 scale, int32 good, found_inf, skipped)."""
+    _fields_ = [("scale", ctypes.c_float), ("good_steps", ctypes.c_int32), ("found_inf", ctypes.c_int32),
+                ("skipped", ctypes.c_int32)]
+
+
 class MergeParams(ctypes.Structure):
     _fields_ = [("lr", ctypes.c_float), ("momentum", ctypes.c_float), ("f_large", ctypes.c_float),
                 ("f_small", ctypes.c_float), ("order", ctypes.c_int32)]
 
 
-_lib = None
+_libs = {}
+_precision = contextvars.ContextVar("dbl_precision", default="bf16")
+PRECISIONS = ("bf16", "f16")
 _V = ctypes.c_void_p
 _I32 = ctypes.c_int32
 _I64 = ctypes.c_int64
@@ -53,15 +72,32 @@ _SZ = ctypes.c_size_t
 _D = ctypes.c_double
 
 
-def lib_path():
-    return build_lib.LIB
+def lib_path(p=None):
+    return build_lib.library_path(p or _precision.get())
 
 
-def lib():
-    """Load libdbl.so (it must have been built by ``build_lib.build()``)."""
-    global _lib
-    if _lib is None:
-        path = build_lib.LIB
+@contextlib.contextmanager
+def precision(p):
+    """Route the calls made inside the block to the library of storage format p ("bf16" or "f16")."""
+    if p not in PRECISIONS:
+        raise ValueError(f"precision must be one of {PRECISIONS}, not {p!r}")
+    tok = _precision.set(p)
+    try:
+        yield
+    finally:
+        _precision.reset(tok)
+
+
+def current_precision():
+    return _precision.get()
+
+
+def lib(p=None):
+    """Load the library of storage format p (default: the current one); it must have been built
+    by ``build_lib.build()``."""
+    p = p or _precision.get()
+    if p not in _libs:
+        path = build_lib.library_path(p)
         if not os.path.exists(path):
             raise ImportError(f"{path} is missing: build it with paper_2509_26092_gb300.build_lib.build()")
         L = ctypes.CDLL(path)
@@ -90,8 +126,12 @@ def lib():
             "dbl_bn_relu_maxpool_fwd": (ctypes.c_int, [ctypes.POINTER(BnShape), _I32, _I32, _I32] + [_V] * 10),
             "dbl_head_workspace_bytes": (_SZ, [_I32, _I32, _I32]),
             "dbl_head_fwd_bwd": (ctypes.c_int, [_I32] * 4 + [_V] * 8 + [_V, _SZ, _V]),
-            "dbl_head_fwd_bwd_dropout": (ctypes.c_int, [_I32] * 4 + [_V] * 4 + [ctypes.c_float, ctypes.c_uint64]
-                                         + [_V] * 6 + [_SZ, _V]),
+            "dbl_head_fwd_bwd_ex": (ctypes.c_int, [_I32] * 4 + [_V] * 4 + [ctypes.POINTER(HeadOpts)] + [_V] * 5
+                                    + [_SZ, _V]),
+            "dbl_ps_dual_batch_merge_scaled": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams),
+                                                              _V, _V, _V, _V]),
+            "dbl_grads_finite": (ctypes.c_int, [_V, _I64, _V, _V]),
+            "dbl_loss_scale_update": (ctypes.c_int, [_V, _I32, _V]),
             "dbl_dropout_mask": (ctypes.c_int, [_I32, _I32, ctypes.c_float, ctypes.c_uint64, _V, _V, _V]),
             "dbl_event_wait": (ctypes.c_int, [_V, _D]),
             "dbl_hold": (ctypes.c_int, [_V, _D, _V, _V]),
@@ -112,8 +152,8 @@ def lib():
             f = getattr(L, name)
             f.restype = res
             f.argtypes = args
-        _lib = L
-    return _lib
+        _libs[p] = L
+    return _libs[p]
 
 
 def _ptr(t):
@@ -147,15 +187,23 @@ def dbl_version():
 
 
 def dbl_kernel_launches():
-    """Kernel launches issued by the library from the host so far."""
-    return lib().dbl_kernel_launches()
+    """Kernel launches issued so far by the libraries loaded in this process (both formats)."""
+    lib()
+    return sum(L.dbl_kernel_launches() for L in _libs.values())
 
 
 def dbl_device_status():
-    """Synchronous: device-side status word (DBL_OK or DBL_ERR_TIMEOUT), then cleared."""
-    v = _I32(0)
-    _check(lib().dbl_device_status(ctypes.byref(v)))
-    return v.value
+    """Synchronous: the device-side status words of the loaded libraries (DBL_OK, or the first
+    DBL_ERR_TIMEOUT), then cleared."""
+    lib()
+    out = DBL_OK
+    for p, L in _libs.items():
+        v = _I32(0)
+        rc = L.dbl_device_status(ctypes.byref(v))
+        if rc != DBL_OK:
+            raise DblError(rc, L.dbl_last_error().decode(errors="replace"))
+        out = out if out != DBL_OK else v.value
+    return out
 
 
 def conv_shape(n, h, w, c, k, r, stride, pad, s=None, stride_w=0, pad_w=0):
@@ -272,17 +320,37 @@ def dbl_head_fwd_bwd(n, hw, c, classes, x, fc_w, fc_b, labels, loss, dfc_w, dfc_
                                   _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
 
 
-def dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, fc_w, fc_b, labels, drop_rate, seed, step, loss, dfc_w, dfc_b, dx,
-                             ws, ws_bytes, stream=None):
-    """The head with dropout of rate drop_rate before the FC layer; step: device uint64 counter
-    (incremented by one on the stream after the call's kernels)."""
-    _check(lib().dbl_head_fwd_bwd_dropout(n, hw, c, classes, _ptr(x), _ptr(fc_w), _ptr(fc_b), _ptr(labels),
-                                          float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(loss),
-                                          _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws), ws_bytes, _stream(stream)))
+def head_opts(drop_rate=0.0, seed=0, step=None, loss_scale=None):
+    """dbl_head_opts: dropout of rate drop_rate (step: device uint64 counter, incremented by one on
+    the stream after each call) and loss_scale (device fp32 pointer/tensor, or None)."""
+    return HeadOpts(float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(loss_scale))
+
+
+def dbl_head_fwd_bwd_ex(n, hw, c, classes, x, fc_w, fc_b, labels, opts, loss, dfc_w, dfc_b, dx, ws, ws_bytes,
+                        stream=None):
+    _check(lib().dbl_head_fwd_bwd_ex(n, hw, c, classes, _ptr(x), _ptr(fc_w), _ptr(fc_b), _ptr(labels),
+                                     ctypes.byref(opts), _ptr(loss), _ptr(dfc_w), _ptr(dfc_b), _ptr(dx), _ptr(ws),
+                                     ws_bytes, _stream(stream)))
+
+
+def dbl_ps_dual_batch_merge_scaled(w, u, w16_out, g_large, g_small, n, lr, momentum, f_large, f_small, order,
+                                   scale_large, scale_small, found_inf, stream=None):
+    p = MergeParams(lr, momentum, f_large, f_small, order)
+    _check(lib().dbl_ps_dual_batch_merge_scaled(_ptr(w), _ptr(u), _ptr(w16_out), _ptr(g_large), _ptr(g_small), n,
+                                                ctypes.byref(p), _ptr(scale_large), _ptr(scale_small),
+                                                _ptr(found_inf), _stream(stream)))
+
+
+def dbl_grads_finite(g, n, found_inf, stream=None):
+    _check(lib().dbl_grads_finite(_ptr(g), n, _ptr(found_inf), _stream(stream)))
+
+
+def dbl_loss_scale_update(state, growth_interval, stream=None):
+    _check(lib().dbl_loss_scale_update(_ptr(state), growth_interval, _stream(stream)))
 
 
 def dbl_dropout_mask(n, c, drop_rate, seed, step, keep, stream=None):
-    """keep [n, c] uint8: the mask dbl_head_fwd_bwd_dropout draws for (drop_rate, seed, *step)."""
+    """keep [n, c] uint8: the mask dbl_head_fwd_bwd_ex draws for (drop_rate, seed, *step)."""
     _check(lib().dbl_dropout_mask(n, c, float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(keep),
                                   _stream(stream)))
 

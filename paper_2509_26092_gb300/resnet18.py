@@ -213,28 +213,69 @@ def conv_out(n, r, st, pad):
     return (n + 2 * pad - r) // st + 1
 
 
-class ServerState:
-    """The parameter server's global model: fp32 master w, momentum u, bf16 pull copy w16."""
+ACT_DTYPE = {"bf16": torch.bfloat16, "f16": torch.float16}
 
-    def __init__(self, spec, params, momentum_state=None, device="cuda"):
-        self.spec = spec
+
+class ServerState:
+    """The parameter server's global model: fp32 master w, momentum u, and the 16-bit pull copy
+    w16 in the storage format of ``precision`` ("bf16", or "f16" for the fp16 mixed precision of
+    the paper's ImageNet runs, Sec. 5.2.3).  With ``loss_scale`` (an initial scale, 2^15 for fp16
+    by default) the workers scale their loss and the server keeps the dynamic scale state
+    (``dbl_loss_scale``: fp32 scale, int32 good steps, found_inf, skipped updates) on the device."""
+
+    def __init__(self, spec, params, momentum_state=None, device="cuda", precision="bf16", loss_scale="auto",
+                 growth_interval=2000):
+        self.spec, self.precision = spec, precision
         self.w = spec.pack(params, device)
         self.u = (spec.pack(momentum_state, device) if momentum_state is not None
                   else torch.zeros_like(self.w))
-        self.w16 = self.w.to(torch.bfloat16)
+        self.w16 = self.w.to(ACT_DTYPE[precision])
+        if loss_scale == "auto":
+            loss_scale = 2.0 ** 15 if precision == "f16" else None
+        self.scaled = loss_scale is not None
+        self.growth_interval = int(growth_interval)
+        self.scale_state = torch.zeros(4, dtype=torch.int32, device=device)
+        if self.scaled:
+            self.scale_state[0:1].view(torch.float32).fill_(float(loss_scale))
+
+    def loss_scale(self):
+        """(scale, good steps, skipped updates), read back from the device (synchronous)."""
+        st = self.scale_state.cpu()
+        return float(st[0:1].view(torch.float32).item()), int(st[1]), int(st[3])
+
+    def apply_pushes(self, g_large, g_small, scale_large, scale_small, lr, momentum, f_large, f_small, order, stream):
+        """The server's update from the pushed gradients (either may be None): the merge of Sec. 3.4,
+        and under loss scaling first the finiteness check of the pushes, the merge of the unscaled
+        pushes (skipped when a value is not finite) and the dynamic scale's update."""
+        n = self.spec.n_flat
+        with D.precision(self.precision):
+            if not self.scaled:
+                D.dbl_ps_dual_batch_merge(self.w, self.u, self.w16, g_large, g_small, n, lr, momentum, f_large,
+                                          f_small, order, stream)
+                return
+            found_inf = self.scale_state.data_ptr() + 8
+            for g in (g_large, g_small):
+                if g is not None:
+                    D.dbl_grads_finite(g, n, found_inf, stream)
+            D.dbl_ps_dual_batch_merge_scaled(self.w, self.u, self.w16, g_large, g_small, n, lr, momentum, f_large,
+                                             f_small, order, scale_large, scale_small, found_inf, stream)
+            D.dbl_loss_scale_update(self.scale_state, self.growth_interval, stream)
 
 
 class Worker:
     """Activations, gradients and scratch of one worker at one (batch, resolution)."""
 
-    def __init__(self, spec, batch, res, device="cuda", eps=1e-5, dropout=0.0, dropout_seed=0):
+    def __init__(self, spec, batch, res, device="cuda", eps=1e-5, dropout=0.0, dropout_seed=0, precision="bf16"):
         self.spec, self.batch, self.res, self.eps = spec, batch, res, eps
+        self.precision = precision
+        # under loss scaling: the scale this worker's step used, copied from the server's at its start
+        self.scale_used = torch.ones(1, dtype=torch.float32, device=device)
         # dropout before the FC layer (Sec. 4.1): rate, the worker's seed, and the device step
         # counter the head reads and advances once per step
         self.dropout, self.dropout_seed = float(dropout), int(dropout_seed)
         self.dropout_step = torch.zeros(1, dtype=torch.int64, device=device)
         dev = device
-        bf = torch.bfloat16
+        bf = ACT_DTYPE[precision]
         B = batch
 
         def act(h, c):
@@ -352,10 +393,22 @@ class Worker:
 
     # ------------------------------------------------------------------ the step
     def enqueue_step(self, server, images, native_res, stream):
-        """Resize, forward, loss, backward; gradients land in self.grad (batch means).
+        """Resize, forward, loss, backward; gradients land in self.grad (batch means, times the
+        loss scale under loss scaling).
 
-        images: fp32 [B, native_res, native_res, 3] on the device; labels in self.labels.
+        images: fp32 [B, native_res, native_res, 3] (or uint8 pixels) on the device; labels in
+        self.labels.  server: the model to compute on (a ServerState or a worker's pulled copy).
         """
+        if server.precision != self.precision:
+            raise ValueError(f"worker stores {self.precision}, the model's copy is {server.precision}")
+        with D.precision(self.precision):
+            if server.scaled:
+                st = stream if isinstance(stream, torch.cuda.Stream) else torch.cuda.ExternalStream(stream)
+                with torch.cuda.stream(st):
+                    self.scale_used.copy_(server.scale_state[0:1].view(torch.float32))
+            self._enqueue_step(server, images, native_res, stream)
+
+    def _enqueue_step(self, server, images, native_res, stream):
         spec, B, eps = self.spec, self.batch, self.eps
         s = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
         ws, wsb = self.ws, self.ws.numel()
@@ -416,10 +469,11 @@ class Worker:
             cur = d["out"]
         # ---- head: pooling, FC, softmax cross-entropy and their backward
         C = spec.widths[-1]
-        if self.dropout > 0.0:
-            D.dbl_head_fwd_bwd_dropout(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"),
-                                       self.labels, self.dropout, self.dropout_seed, self.dropout_step, self.loss,
-                                       gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
+        if self.dropout > 0.0 or server.scaled:
+            opts = D.head_opts(self.dropout, self.dropout_seed, self.dropout_step if self.dropout > 0.0 else None,
+                               self.scale_used if server.scaled else None)
+            D.dbl_head_fwd_bwd_ex(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"), self.labels,
+                                  opts, self.loss, gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
         else:
             D.dbl_head_fwd_bwd(B, self.final_hw ** 2, C, spec.classes, cur, pv("fc.w"), pv("fc.b"), self.labels,
                                self.loss, gv("fc.w"), gv("fc.b"), self.dfeat, ws, wsb, s)
@@ -556,11 +610,15 @@ class DualBatchIteration:
         if self.small is not None:
             self.small.enqueue_step(self.server, self.images_s, self.native_res, sS)
         sL.wait_stream(sS)  # the server applies the pushes once both have arrived
-        srv = self.server
-        D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, self.large.grad if self.large else None,
-                                  self.small.grad if self.small else None, srv.spec.n_flat, self.lr, self.momentum,
-                                  self.f_large, self.f_small, self.order, sL.cuda_stream)
+        self._merge(["L", "S"], sL)
         cur.wait_stream(sL)
+
+    def _merge(self, tags, stream):
+        wl = self.large if "L" in tags else None
+        ws_ = self.small if "S" in tags else None
+        self.server.apply_pushes(wl.grad if wl else None, ws_.grad if ws_ else None,
+                                 wl.scale_used if wl else None, ws_.scale_used if ws_ else None, self.lr,
+                                 self.momentum, self.f_large, self.f_small, self.order, stream.cuda_stream)
 
     def run(self):
         cur = torch.cuda.current_stream()
@@ -605,10 +663,7 @@ class DualBatchIteration:
         if arrived:
             for tag in arrived:
                 cur.wait_event(done[tag])
-            srv = self.server
-            D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, self.large.grad if "L" in arrived else None,
-                                      self.small.grad if "S" in arrived else None, srv.spec.n_flat, self.lr,
-                                      self.momentum, self.f_large, self.f_small, self.order, cur.cuda_stream)
+            self._merge(arrived, cur)
         self._consumed = torch.cuda.Event()
         self._consumed.record(cur)
         return (D.DBL_OK if not failed else D.DBL_ERR_TIMEOUT), failed

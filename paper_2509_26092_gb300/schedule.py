@@ -52,9 +52,11 @@ class PulledWeights:
     refreshed by ``pull`` on the worker's stream."""
 
     def __init__(self, server):
-        self.spec = server.spec
+        self.spec, self.precision = server.spec, server.precision
         self.w = server.w.clone()
         self.w16 = server.w16.clone()
+        # the loss scale is the server's live state: a worker copies it when its step starts
+        self.scaled, self.scale_state = server.scaled, server.scale_state
 
     def pull(self, server, stream):
         import torch
@@ -130,8 +132,8 @@ class AsyncDualBatch:
                 s.wait_event(last)
             g_l = wk.grad if tag == "L" else None
             g_s = wk.grad if tag == "S" else None
-            D.dbl_ps_dual_batch_merge(srv.w, srv.u, srv.w16, g_l, g_s, srv.spec.n_flat, self.lr, self.momentum,
-                                      self.factor["L"], self.factor["S"], 0, s.cuda_stream)
+            srv.apply_pushes(g_l, g_s, wk.scale_used if tag == "L" else None, wk.scale_used if tag == "S" else None,
+                             self.lr, self.momentum, self.factor["L"], self.factor["S"], 0, s.cuda_stream)
             with torch.cuda.stream(s):
                 self.losses[tag].append(wk.loss.clone())
             if on_push is not None:

@@ -28,12 +28,25 @@ def declared_symbols():
     return sorted(set(re.findall(r"\b(dbl_[a-z0-9_]+)\s*\(", src)))
 
 
-def test_every_declared_symbol_is_exported(D):
-    L = D.lib()
+@pytest.mark.parametrize("precision", ["bf16", "f16"])
+def test_every_declared_symbol_is_exported(D, precision):
+    """Both builds (bfloat16 and binary16 storage) export every entry point dbl.h declares."""
+    L = D.lib(precision)
     names = declared_symbols()
     assert len(names) >= 20
     for name in names:
         assert hasattr(L, name), name
+
+
+def test_calls_go_to_the_library_of_the_current_precision(D):
+    assert D.current_precision() == "bf16" and D.lib_path().endswith("libdbl.so")
+    with D.precision("f16"):
+        assert D.current_precision() == "f16" and D.lib_path().endswith("libdbl_f16.so")
+        assert D.lib() is D.lib("f16") and D.lib("f16") is not D.lib("bf16")
+    assert D.current_precision() == "bf16"
+    with pytest.raises(ValueError):
+        with D.precision("fp8"):
+            pass
 
 
 def test_version(D):

@@ -380,7 +380,8 @@ def test_head_dropout_matches_oracle(D, n, hw, c, classes, rate):
     wsb = D.dbl_head_workspace_bytes(n, c, classes)
     work = ws(wsb)
     xd, Wd, bd, labd = to_bf16_dev(x), to_f32_dev(W), to_f32_dev(b), torch.from_numpy(lab).cuda()
-    D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, xd, Wd, bd, labd, rate, seed, step, loss, dW, db, dx, work, wsb)
+    opts = D.head_opts(rate, seed, step)
+    D.dbl_head_fwd_bwd_ex(n, hw, c, classes, xd, Wd, bd, labd, opts, loss, dW, db, dx, work, wsb)
     x4 = x.reshape(n, 1, hw, c)
     feat = orc.dropout_apply(orc.avgpool_fwd(x4), rkeep, d)
     logits = orc.fc_fwd(feat, W, b)
@@ -395,7 +396,7 @@ def test_head_dropout_matches_oracle(D, n, hw, c, classes, rate):
     dropped = np.broadcast_to((rkeep == 0)[:, None, :], (n, hw, c))
     assert np.all(host(dx)[dropped] == 0.0)  # a dropped feature passes no gradient back
     # the next call draws the mask of step 6
-    D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, xd, Wd, bd, labd, rate, seed, step, loss, dW, db, dx, work, wsb)
+    D.dbl_head_fwd_bwd_ex(n, hw, c, classes, xd, Wd, bd, labd, opts, loss, dW, db, dx, work, wsb)
     rkeep6 = orc.dropout_mask(n, c, d, seed, step0 + 1)
     feat6 = orc.dropout_apply(orc.avgpool_fwd(x4), rkeep6, d)
     rl6, _ = orc.softmax_ce(orc.fc_fwd(feat6, W, b), lab)
@@ -415,7 +416,7 @@ def test_head_dropout_rate_zero_is_the_plain_head(D):
         o = (torch.empty(1, device="cuda"), torch.empty((classes, c), device="cuda"), torch.empty(classes, device="cuda"),
              torch.empty((n, hw, c), dtype=torch.bfloat16, device="cuda"))
         if drop:
-            D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, W, b, lab, 0.0, 1, None, *o, ws(wsb), wsb)
+            D.dbl_head_fwd_bwd_ex(n, hw, c, classes, x, W, b, lab, D.head_opts(0.0, 1), *o, ws(wsb), wsb)
         else:
             D.dbl_head_fwd_bwd(n, hw, c, classes, x, W, b, lab, *o, ws(wsb), wsb)
         outs.append(o)
@@ -423,7 +424,7 @@ def test_head_dropout_rate_zero_is_the_plain_head(D):
     for a, b_ in zip(*outs):
         assert torch.equal(a, b_)
     with pytest.raises(D.DblError):
-        D.dbl_head_fwd_bwd_dropout(n, hw, c, classes, x, W, b, lab, 1.0, 1, None, *outs[0], ws(wsb), wsb)
+        D.dbl_head_fwd_bwd_ex(n, hw, c, classes, x, W, b, lab, D.head_opts(1.0, 1), *outs[0], ws(wsb), wsb)
 
 
 # ----------------------------------------------------------------------------- convolutions

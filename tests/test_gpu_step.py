@@ -242,3 +242,70 @@ def test_a_late_push_is_left_out_of_the_merge(R):
                           1.0, fS, 0)
     assert max_norm_rel(server.w.double().cpu().numpy(), rw) <= 1e-6
     assert max_norm_rel(server.u.double().cpu().numpy(), ru) <= 1e-6
+
+
+def test_fp16_dual_batch_iteration_matches_oracle(R):
+    """The dual-batch iteration in fp16 mixed precision with loss scaling (Sec. 5.2.3): binary16
+    storage, loss scale 2^15, the server's scaled merge.  Losses and the pushed (scaled) gradients
+    against the oracle rounding to binary16 at the same storage points, the merge against the
+    oracle's scaled merge of the GPU's own pushes, and the dynamic scale's first good step."""
+    D = load_dbl()
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=8, random_bn=True)
+    u0 = synth.momentum_state(spec.table(), 0.01, seed=8)
+    img = synth.images(8, 32, 32, 3, seed=8)
+    lab = synth.labels(8, 100, seed=8)
+    S = 2.0 ** 15
+    server = R.ServerState(spec, params, u0, precision="f16", loss_scale=S)
+    large = R.Worker(spec, 6, 24, dropout=0.2, dropout_seed=11, precision="f16")
+    small = R.Worker(spec, 2, 24, dropout=0.2, dropout_seed=12, precision="f16")
+    fS = 19.0 / 21.0
+    it = R.DualBatchIteration(server, large, small, 32, lr=0.2, momentum=0.9, f_large=1.0, f_small=fS, order=0)
+    it.set_inputs(torch.from_numpy(img[2:]).cuda(), torch.from_numpy(lab[2:]).cuda(), torch.from_numpy(img[:2]).cuda(),
+                  torch.from_numpy(lab[:2]).cuda())
+    w_before, u_before = server.w.clone(), server.u.clone()
+    it.run()
+    torch.cuda.synchronize()
+    assert D.dbl_device_status() == D.DBL_OK
+    assert server.w16.dtype == torch.float16 and large.x0.dtype == torch.float16
+    d = float(np.float32(0.2))
+    p64 = {k: v.astype(np.float64) for k, v in params.items()}
+    u64 = {k: v.astype(np.float64) for k, v in u0.items()}
+    kw = dict(order=0, dropout_large=(d, 11, 0), dropout_small=(d, 12, 0), loss_scale=S)
+    nw, nu, lL, lS, gL, gS = OR.dual_batch_iteration(p64, u64, img[2:], lab[2:], img[:2], lab[:2], 24, "cifar", 0.2,
+                                                     0.9, 1.0, fS, storage="f16", **kw)
+    _, _, _, _, gL64, gS64 = OR.dual_batch_iteration(p64, u64, img[2:], lab[2:], img[:2], lab[:2], 24, "cifar", 0.2,
+                                                     0.9, 1.0, fS, storage=None, **kw)
+    assert abs(large.loss.item() - lL) <= TOL * abs(lL)
+    assert abs(small.loss.item() - lS) <= TOL * abs(lS)
+    _compare_grads(spec, large.grad, gL, gL64, "fp16 large worker")
+    _compare_grads(spec, small.grad, gS, gS64, "fp16 small worker")
+    rw, ru, ok = orc.ps_merge_scaled(w_before.double().cpu().numpy(), u_before.double().cpu().numpy(),
+                                     large.grad.double().cpu().numpy(), small.grad.double().cpu().numpy(), 0.2, 0.9,
+                                     1.0, fS, 0, S, S)
+    assert ok
+    assert max_norm_rel(server.w.double().cpu().numpy(), rw) <= 1e-6
+    assert max_norm_rel(server.u.double().cpu().numpy(), ru) <= 1e-6
+    assert torch.equal(server.w16, server.w.to(torch.float16))
+    assert server.loss_scale() == (S, 1, 0)
+
+
+def test_fp16_overflow_skips_the_update_and_halves_the_scale(R):
+    """A loss scale far too large makes the scaled gradients overflow binary16: the server finds
+    the non-finite push, leaves the model as it was, halves the scale and counts the skip."""
+    D = load_dbl()
+    spec = R.ResNet18Spec("cifar", 100)
+    params = synth.params(spec.table(), seed=9)
+    server = R.ServerState(spec, params, precision="f16", loss_scale=2.0 ** 60)
+    it = R.DualBatchIteration(server, R.Worker(spec, 6, 24, precision="f16"), R.Worker(spec, 2, 24, precision="f16"),
+                              32)
+    img = torch.from_numpy(synth.images(8, 32, 32, 3, seed=9)).cuda()
+    lab = torch.from_numpy(synth.labels(8, 100, seed=9)).cuda()
+    it.set_inputs(img[2:], lab[2:], img[:2], lab[:2])
+    w0, u0, w160 = server.w.clone(), server.u.clone(), server.w16.clone()
+    it.run()
+    torch.cuda.synchronize()
+    assert D.dbl_device_status() == D.DBL_OK
+    assert not torch.isfinite(it.large.grad).all()
+    assert torch.equal(server.w, w0) and torch.equal(server.u, u0) and torch.equal(server.w16, w160)
+    assert server.loss_scale() == (2.0 ** 59, 0, 1)

@@ -25,15 +25,18 @@ def h(t):
     return t.detach().double().cpu().numpy()
 
 
-@pytest.mark.parametrize("variant,classes,batch,res", [("cifar", 100, 8, 32), ("imagenet", 1000, 4, 96),
-                                                       ("cifar", 100, 256, 32)])  # the CIFAR step at its batch
-def test_every_layer_of_the_step(variant, classes, batch, res):
+@pytest.mark.parametrize("variant,classes,batch,res,precision", [
+    ("cifar", 100, 8, 32, "bf16"), ("imagenet", 1000, 4, 96, "bf16"),
+    ("cifar", 100, 256, 32, "bf16"),                                     # the CIFAR step at its batch
+    ("imagenet", 1000, 4, 96, "f16")])                                   # fp16 storage, loss scale 2^15
+def test_every_layer_of_the_step(variant, classes, batch, res, precision):
     load_dbl()
     from paper_2509_26092_gb300 import resnet18 as R
     spec = R.ResNet18Spec(variant, classes)
     params = synth.params(spec.table(), seed=11, random_bn=True)
-    server = R.ServerState(spec, params)
-    wk = R.Worker(spec, batch, res)
+    server = R.ServerState(spec, params, precision=precision)
+    wk = R.Worker(spec, batch, res, precision=precision)
+    scale = server.loss_scale()[0] if server.scaled else 1.0  # every gradient is the loss's times this
     img = torch.from_numpy(synth.images(batch, res, res, 3, seed=11)).cuda()
     wk.labels.copy_(torch.from_numpy(synth.labels(batch, classes, seed=11)).cuda())
     wk.enqueue_step(server, img, res, torch.cuda.current_stream())
@@ -60,7 +63,7 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
     chk("stem.bn.mean", h(wk.stem_stats[2]), m, 1e-4)
     if variant == "imagenet":
         # the BatchNorm output is pooled on the fly (never stored): pool the oracle's stored values
-        stem_a = orc.round_bf16(o)
+        stem_a = (orc.round_f16 if precision == "f16" else orc.round_bf16)(o)
         y, arg = orc.maxpool_fwd(stem_a)
         chk("stem.bn.pool", h(wk.pool_out), y)
         agree = np.mean(wk.pool_arg.cpu().numpy().astype(np.int32) == arg)
@@ -88,7 +91,7 @@ def test_every_layer_of_the_step(variant, classes, batch, res):
     feat = orc.avgpool_fwd(last)
     logits = orc.fc_fwd(feat, P["fc.w"], P["fc.b"])
     loss, dl = orc.softmax_ce(logits, wk.labels.cpu().numpy())
-    dW, db, df = orc.fc_bwd(dl, feat, P["fc.w"])
+    dW, db, df = orc.fc_bwd(dl * scale, feat, P["fc.w"])
     assert abs(wk.loss.item() - loss) <= 1e-5 * abs(loss)
     chk("fc.w.grad", G["fc.w"], dW, 1e-4)
     chk("fc.b.grad", G["fc.b"], db, 1e-4)
