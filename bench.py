@@ -55,6 +55,10 @@ CONFIGS = {
                           desc="ImageNet-shaped ResNet-18, one train step at 224x224, batch 256, single push"),
     "imagenet_small": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(32,), small=(8,),
                            dropout=(0.2,), desc="small ImageNet-shaped dual-batch iteration for profiling"),
+    "imagenet_profile": dict(variant="imagenet", classes=1000, native=224, stages=(224,), large=(128,), small=(None,),
+                             dropout=(0.3,),
+                             desc="one 224 px worker of batch 128 (a fifth of the imagenet_hybrid 224 px iteration's "
+                                  "640 images), the size DRAM-traffic captures are taken at"),
 }
 DEFAULT_CONFIG = "imagenet_hybrid"
 F_SMALL = 19.0 / 21.0  # d_S/d_L for one large and one small worker at k = 1.05 (Eqs. 4-6)
@@ -72,7 +76,7 @@ def _peaks():
 
 def _conv_source_hash():
     h = hashlib.sha256()
-    for name in ("conv.cu", "dbl_internal.cuh"):
+    for name in ("conv.cu", "dbl_internal.cuh", "dbl_act.cuh"):
         with open(os.path.join(ROOT, "paper_2509_26092_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -80,14 +84,16 @@ def _conv_source_hash():
 
 def _traffic_record(config):
     """DRAM bytes (read + write) of all conv-kernel launches of one iteration at the largest
-    stage, from a committed ncu summary, if it was taken on the current kernel source."""
+    stage of `config`, from a committed ncu summary taken on the current kernel source: the
+    capture ran a smaller configuration and is scaled by the images processed (conv traffic
+    is per image: activations and their gradients, the weights being a small share)."""
     path = os.path.join(ROOT, "profiles", "conv_traffic_imagenet_hybrid_224.json")
     try:
         with open(path) as f:
             rec = json.load(f)
-        if rec.get("source_hash") != _conv_source_hash() or rec.get("config") != config:
+        if rec.get("source_hash") != _conv_source_hash() or rec.get("applies_to") != config:
             return None
-        return rec.get("dram_bytes_per_iteration")
+        return int(rec["dram_bytes_per_iteration"] * rec.get("scale", 1.0))
     except Exception:
         return None
 
@@ -486,6 +492,13 @@ def run_profile_conv(args):
     from paper_2509_26092_gb300 import resnet18 as R
 
     torch.cuda.set_device(0)
+    with D.precision(args.precision):
+        return _profile_conv(args, D, R)
+
+
+def _profile_conv(args, D, R):
+    import torch
+    act = {"bf16": torch.bfloat16, "f16": torch.float16}[args.precision]
     layer, pname = args.profile_conv.split(":")
     spec = R.ResNet18Spec("imagenet", 1000)
     n = args.profile_batch
@@ -508,14 +521,14 @@ def run_profile_conv(args):
     P = R.conv_out(s.h, s.r, s.stride, s.pad)
     Q = R.conv_out(s.w, s.s, s.stride_w or s.stride, s.pad_w if s.stride_w else s.pad)
     g = torch.Generator(device="cuda").manual_seed(0)
-    x = torch.randn(s.n, s.h, s.w, s.c, device="cuda", generator=g).to(torch.bfloat16)
-    w = (0.05 * torch.randn(s.k, s.r, s.s, s.c, device="cuda", generator=g)).to(torch.bfloat16)
-    dy = torch.randn(s.n, P, Q, s.k, device="cuda", generator=g).to(torch.bfloat16)
+    x = torch.randn(s.n, s.h, s.w, s.c, device="cuda", generator=g).to(act)
+    w = (0.05 * torch.randn(s.k, s.r, s.s, s.c, device="cuda", generator=g)).to(act)
+    dy = torch.randn(s.n, P, Q, s.k, device="cuda", generator=g).to(act)
     ps = {"fwd": D.DBL_PASS_FWD, "dgrad": D.DBL_PASS_DGRAD, "wgrad": D.DBL_PASS_WGRAD}[pname]
     ws = torch.empty(max(int(D.dbl_conv_workspace_bytes(s, ps)), 16), dtype=torch.uint8, device="cuda")
     st = torch.cuda.current_stream()
     if pname == "fwd":
-        y = torch.empty(s.n, P, Q, s.k, dtype=torch.bfloat16, device="cuda")
+        y = torch.empty(s.n, P, Q, s.k, dtype=act, device="cuda")
         ssum, ssq = torch.empty(s.k, device="cuda"), torch.empty(s.k, device="cuda")
         fn = lambda: D.dbl_conv_fwd(s, x, w, y, ssum, ssq, ws, ws.numel(), st)
     elif pname == "dgrad":
@@ -528,7 +541,7 @@ def run_profile_conv(args):
         fn()
     torch.cuda.synchronize()
     assert D.dbl_device_status() == D.DBL_OK
-    print(json.dumps({"profile_conv": args.profile_conv, "batch": n}), flush=True)
+    print(json.dumps({"profile_conv": args.profile_conv, "batch": n, "precision": args.precision}), flush=True)
     return 0
 
 
