@@ -16,6 +16,9 @@ from gpu_common import bf16_values, check_status, host, load_dbl, rng, stem_fold
 pytestmark = pytest.mark.gpu
 
 CONV_TOL = 1e-2
+# fp32 weight gradients: the products of two bf16 values are exact in fp32, so the only error
+# against the fp64 oracle is that of fp32 summation (relative ~1e-6 at these sizes)
+WGRAD_TOL = 1e-4
 MERGE_TOL = 1e-6
 
 
@@ -180,7 +183,7 @@ def test_unrolled_stem_fwd_and_wgrad_match_oracle(D, case):
     assert np.all(got[:, :, r:, :] == 0.0) and np.all(got[..., 3:] == 0.0)  # padding gets no gradient
     assert np.all(got[:, r:] == 0.0)
     rdw = orc.conv2d_wgrad(x, dy, wt.shape, st, pad)
-    assert max_norm_rel(got[:, :r, :r, :3], rdw) <= CONV_TOL
+    assert max_norm_rel(got[:, :r, :r, :3], rdw) <= WGRAD_TOL
     check_status(D)
 
 
@@ -614,8 +617,8 @@ def test_conv_wgrad_matches_oracle(D, case):
     D.dbl_conv_wgrad(shape, xd, dyd, dw, False, ws(wsb), wsb)
     got = host(dw)
     assert np.all(np.isfinite(got))
-    assert max_norm_rel(got, ref) <= CONV_TOL
+    assert max_norm_rel(got, ref) <= WGRAD_TOL
     # accumulate mode adds onto what is there
     D.dbl_conv_wgrad(shape, xd, dyd, dw, True, ws(wsb), wsb)
-    assert max_norm_rel(host(dw), 2 * ref) <= CONV_TOL
+    assert max_norm_rel(host(dw), 2 * ref) <= WGRAD_TOL
     check_status(D)

@@ -309,3 +309,21 @@ def test_fp16_overflow_skips_the_update_and_halves_the_scale(R):
     assert not torch.isfinite(it.large.grad).all()
     assert torch.equal(server.w, w0) and torch.equal(server.u, u0) and torch.equal(server.w16, w160)
     assert server.loss_scale() == (2.0 ** 59, 0, 1)
+
+
+def test_a_hold_that_is_never_released_times_out_on_the_device(R):
+    """A bounded device wait that runs out: the hold gives up after its limit, reports
+    DBL_ERR_TIMEOUT in its status word, and the stream (and the context) carry on."""
+    D = load_dbl()
+    flag = torch.zeros(1, dtype=torch.int32).pin_memory()  # nothing ever sets it
+    status = torch.full((1,), 7, dtype=torch.int32).pin_memory()
+    after = torch.ones(4, device="cuda")
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    D.dbl_hold(flag, 0.2, status, s)
+    with torch.cuda.stream(s):
+        after.mul_(3.0)  # queued behind the hold
+    s.synchronize()
+    assert int(status[0]) == D.DBL_ERR_TIMEOUT
+    assert torch.equal(after, torch.full((4,), 3.0, device="cuda"))
+    assert D.dbl_device_status() == D.DBL_OK  # the hold reports through its own word only
