@@ -110,12 +110,14 @@ def test_resize_stem_unrolls_the_resized_image(D, n, hin, hout, r, st, pad):
     check_status(D)
 
 
-@pytest.mark.parametrize("n,hin,hout", [(2, 224, 160), (3, 40, 40)])
-def test_resize_stem_from_8bit_pixels(D, n, hin, hout):
+@pytest.mark.parametrize("n,hin,hout,r,st,pad", [
+    (2, 224, 160, 7, 2, 3), (2, 224, 128, 7, 2, 3), (1, 288, 160, 7, 2, 3), (2, 224, 224, 7, 2, 3),
+    (3, 40, 40, 7, 2, 3),
+    (3, 32, 24, 3, 1, 1), (2, 32, 32, 3, 1, 1)])           # the CIFAR stem's layout (one row per position)
+def test_resize_stem_from_8bit_pixels(D, n, hin, hout, r, st, pad):
     """8-bit pixels standardized on the GPU: the same bits as the fp32 path on pixels
     standardized on the host with the same two fp32 operations, and the oracle's resize."""
     from paper_2509_26092_gb300.resnet18 import PIXEL_BIAS, PIXEL_SCALE
-    r, st, pad = 7, 2, 3
     lay = _stem_layout(r, st, pad)
     u8 = rng(hin + 5).integers(0, 256, size=(n, hin, hin, 3), dtype=np.uint8)
     x32 = u8.astype(np.float32) * np.asarray(PIXEL_SCALE, np.float32) + np.asarray(PIXEL_BIAS, np.float32)
