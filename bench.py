@@ -294,9 +294,9 @@ def build_pipeline(cfg, device, precision="bf16"):
 def conv_roofline(stage, reps=4, replays=2, table=None, cold_reps=5):
     """Time each convolution pass of the stage's workers alone with CUDA events, two ways.
     Cold: L2 flushed before each launch (a 512 MB buffer, larger than the 129 MB L2, written on
-    the stream first, which also covers the host's launch of the pass), the median of
-    `cold_reps` launches, as in the training step where every pass's operands come from DRAM
-    (its working set is many GB).  Warm: `reps` calls of the pass captured in one CUDA graph
+    the stream first), the pass replayed from a one-call CUDA graph, the median of `cold_reps`
+    launches, as in the training step where every pass's operands come from DRAM (its working
+    set is many GB).  Warm: `reps` calls of the pass captured in one CUDA graph
     and replayed `replays` times, so repeats 2.. find operands of the smaller layers in L2.
     Return (algorithmic conv FLOPs of one iteration, cold seconds per iteration, warm seconds
     per iteration, algorithmic bytes).  If table is a list, append (worker batch, layer, pass,
@@ -358,15 +358,21 @@ def conv_roofline(stage, reps=4, replays=2, table=None, cold_reps=5):
                 torch.cuda.synchronize()
                 del graph
                 tw = ev[0].elapsed_time(ev[1]) / 1000.0 / (reps * replays)
+                # cold: one call of the pass as a CUDA graph (its replay is enqueued in microseconds,
+                # so the host never holds up the GPU between the events), after the flush
+                one = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(one):
+                    fn(torch.cuda.current_stream())
                 cold = []
                 for _ in range(cold_reps):
                     flush.zero_()
                     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                     e0.record(s)
-                    fn(s)
+                    one.replay()
                     e1.record(s)
                     torch.cuda.synchronize()
                     cold.append(e0.elapsed_time(e1) / 1000.0)
+                del one
                 tc = sorted(cold)[len(cold) // 2]
                 secs += tc
                 warm_secs += tw
