@@ -92,6 +92,13 @@ DBL_API int dbl_device_status(int32_t* status);
  * channels zero-padded to 8) for the forward and weight passes.  The stem of
  * ResNet-18 is run as an r x 1 convolution over the input unrolled along W
  * (see dbl_progressive_resize_stem).
+ *
+ * Environment (read once per process): DBL_CONV_CTA_PAIRS=0 runs every pass on
+ * single CTAs, =2 puts every 128/256-column tile on CTA pairs; DBL_CONV_PDL=1
+ * launches the passes with programmatic stream serialization, so that a
+ * kernel's set-up overlaps the end of the kernel before it on the stream
+ * (faster with one stream of work, slower when another stream competes for
+ * the SMs).  Neither changes what is computed.
  * ======================================================================== */
 typedef struct {
     int32_t n, h, w, c; /* input activation shape (NHWC)                    */

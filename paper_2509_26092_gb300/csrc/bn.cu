@@ -132,6 +132,7 @@ __global__ void __launch_bounds__(kThreads, kBlocksPerSM)
                     act_t* __restrict__ out, int count, int C, int relu, const float* __restrict__ gamma,
                     const float* __restrict__ beta, const float* __restrict__ mean, const float* __restrict__ invstd)
 {
+    dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;
@@ -351,6 +352,7 @@ __global__ void __launch_bounds__(kThreads, kBwdBlocksPerSM)
                         const float* __restrict__ mean, const float* __restrict__ invstd,
                         const float* __restrict__ coef, act_t* __restrict__ dy, act_t* __restrict__ dres)
 {
+    dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     const int groups = C / 8;
     const int g = threadIdx.x % groups;
     const int rstep = kThreads / groups;

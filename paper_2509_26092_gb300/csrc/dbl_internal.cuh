@@ -765,6 +765,16 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo_bytes
     return d;
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream serialization may
+// start while the kernel before it on the stream is still running; this waits (once per
+// thread) until that kernel has completed and its memory operations are visible.  Without the
+// launch attribute it returns at once.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel on the stream (if launched with programmatic stream serialization) be
+// scheduled once every CTA of this one has issued this or exited; it still waits for this
+// kernel's completion before touching memory.
+__device__ __forceinline__ void grid_dependency_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Instruction descriptor, kind::f16 with A and B both in the storage format (bf16, or f16 in the
 // fp16 build: one MMA never mixes the two) and fp32 D.
 // a_mn / b_mn: 1 if that operand is MN-major (transposed) in shared memory.

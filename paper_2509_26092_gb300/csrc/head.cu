@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(256)
                                const float* __restrict__ invstd, act_t* __restrict__ y,
                                uint8_t* __restrict__ arg, int n, int H, int W, int C, int P, int Q)
 {
+    dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     const unsigned groups = (unsigned)C / 8u;
     const unsigned per_block = blockDim.x / groups;
     if (threadIdx.x >= per_block * groups) return;

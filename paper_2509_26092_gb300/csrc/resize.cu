@@ -147,6 +147,7 @@ __global__ void __launch_bounds__(kStemThreads) resize_stem_kernel(const Tin* __
                                                           int32_t M, int32_t Q, int32_t taps, int32_t sw, int32_t pw,
                                                           int32_t ph, const PixelNorm nm)
 {
+    dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     constexpr int32_t cu = 8 / RG;  // channels per tap
     // staged rows: [RG][wo + 2*pw + 8][cu] fp32, column x at index x + pw (dynamic shared memory)
     extern __shared__ __align__(16) float rows[];

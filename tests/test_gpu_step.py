@@ -327,3 +327,38 @@ def test_a_hold_that_is_never_released_times_out_on_the_device(R):
     assert int(status[0]) == D.DBL_ERR_TIMEOUT
     assert torch.equal(after, torch.full((4,), 3.0, device="cuda"))
     assert D.dbl_device_status() == D.DBL_OK  # the hold reports through its own word only
+
+
+_STEP_IN_CHILD = r"""
+import sys, torch
+sys.path.insert(0, sys.argv[1])
+from paper_2509_26092_gb300 import build_lib
+build_lib.build()
+from paper_2509_26092_gb300 import resnet18 as R, synth
+spec = R.ResNet18Spec("imagenet", 1000)
+server = R.ServerState(spec, synth.params(spec.table(), seed=21, random_bn=True))
+wk = R.Worker(spec, 8, 96)
+wk.labels.copy_(torch.from_numpy(synth.labels(8, 1000, seed=21)).cuda())
+img = torch.from_numpy(synth.images(8, 96, 96, 3, seed=21)).cuda()
+for _ in range(2):
+    wk.enqueue_step(server, img, 96, torch.cuda.current_stream())
+torch.cuda.synchronize()
+torch.save(wk.grad.cpu(), sys.argv[2])
+"""
+
+
+def test_programmatic_dependent_launch_gives_the_same_step(R, tmp_path):
+    """Convolutions launched with programmatic stream serialization (DBL_CONV_PDL=1, read once per
+    process, hence a child process) give the same gradients, bit for bit, as in plain stream order."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = {}
+    for flag in ("0", "1"):
+        path = str(tmp_path / f"grad{flag}.pt")
+        r = subprocess.run([sys.executable, "-c", _STEP_IN_CHILD, root, path], capture_output=True, text=True,
+                           timeout=600, env=dict(os.environ, DBL_CONV_PDL=flag))
+        assert r.returncode == 0, r.stderr[-2000:]
+        out[flag] = torch.load(path)
+    assert torch.isfinite(out["1"]).all() and torch.equal(out["0"], out["1"])
