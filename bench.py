@@ -255,7 +255,7 @@ def run_reference(args, cfg):
 
 
 # ------------------------------------------------------------------------------------------ GPU arm
-def build_pipeline(cfg, device, precision="bf16"):
+def build_pipeline(cfg, device, precision="bf16", pdl="auto"):
     import torch
 
     from paper_2509_26092_gb300 import dbl as D
@@ -278,6 +278,10 @@ def build_pipeline(cfg, device, precision="bf16"):
         large = R.Worker(spec, bl, res, device, dropout=drop, dropout_seed=2 * res + 1, precision=precision)
         small = (R.Worker(spec, bs, res, device, dropout=drop, dropout_seed=2 * res + 2, precision=precision)
                  if bs else None)
+        if pdl != "auto":  # programmatic dependent launch per worker: on, off, or the large worker only
+            large.pdl = pdl in ("on", "large")
+            if small is not None:
+                small.pdl = pdl == "on"
         it = R.DualBatchIteration(server, large, small, nat, lr=LR, momentum=MOMENTUM, f_large=1.0, f_small=F_SMALL)
         it.set_inputs(host_l[:bl].to(device), lab_l[:bl].to(device),
                       host_s[:bs].to(device) if bs else None, lab_s[:bs].to(device) if bs else None)
@@ -571,7 +575,7 @@ def run_ours(args, cfg):
     import numpy as np
     import torch
     ws, rank, local = _dist()
-    if all(b is None for b in cfg["small"]):
+    if args.pdl == "auto" and all(b is None for b in cfg["small"]):
         # one worker, one stream: let each convolution's set-up overlap the kernel before it
         # (programmatic dependent launch; with two worker streams it measured slower)
         os.environ.setdefault("DBL_CONV_PDL", "1")
@@ -584,7 +588,7 @@ def run_ours(args, cfg):
     build_lib.build()
     from paper_2509_26092_gb300 import dbl as D
 
-    pipe = build_pipeline(cfg, device, args.precision)
+    pipe = build_pipeline(cfg, device, args.precision, args.pdl)
     stages = pipe["stages"]
     images_per_step = sum(s["images"] for s in stages)
 
@@ -718,7 +722,8 @@ def run_ours(args, cfg):
                            "small_batch": list(cfg["small"]), "dropout": list(cfg["dropout"]),
                            "images_per_step": images_per_step,
                            "params": pipe["spec"].n_params(), "f_small": F_SMALL, "lr": LR, "momentum": MOMENTUM,
-                           "conv_pdl": os.environ.get("DBL_CONV_PDL") == "1",
+                           "conv_pdl": (args.pdl if args.pdl != "auto" else
+                                        "on" if os.environ.get("DBL_CONV_PDL") == "1" else "off"),
                            "l2": "working set (activations, several GB) larger than L2; no explicit flush",
                            "input": f"uint8 images {cfg['native']}x{cfg['native']}x3 from pinned host memory, "
                                     "standardized per channel on the GPU",
@@ -744,6 +749,9 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--pdl", default="auto", choices=["auto", "off", "on", "large"],
+                    help="programmatic dependent launch of the convolutions: auto (one-worker workloads only), "
+                         "off, on, or the large worker only")
     ap.add_argument("--precision", default="bf16", choices=["bf16", "f16"],
                     help="16-bit storage format: bf16, or f16 with dynamic loss scaling (the paper's mixed precision)")
     ap.add_argument("--conv-table", action="store_true",

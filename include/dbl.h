@@ -100,6 +100,12 @@ DBL_API int dbl_device_status(int32_t* status);
  * (faster with one stream of work, slower when another stream competes for
  * the SMs).  Neither changes what is computed.
  * ======================================================================== */
+
+/* Host: overrides DBL_CONV_PDL for the convolution launches that follow, in
+ * this process, from any thread: 1 = programmatic stream serialization on,
+ * 0 = off, -1 = back to the environment's choice.  Launches already enqueued
+ * (or captured) keep the attribute they were launched with. */
+DBL_API int dbl_set_conv_pdl(int32_t mode);
 typedef struct {
     int32_t n, h, w, c; /* input activation shape (NHWC)                    */
     int32_t k, r, s;    /* output channels and filter size (KRSC weights)   */

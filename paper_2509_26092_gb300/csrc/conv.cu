@@ -28,6 +28,8 @@
 #include <algorithm>
 #include <cstdlib>
 
+#include <atomic>
+
 #include "dbl_internal.cuh"
 
 namespace {
@@ -1830,13 +1832,16 @@ int plan_grid(const Plan& pl)
 // GB300: one worker's 224 px step 1.2% faster with it; two workers' iteration on two streams
 // 1.1% slower, because CTAs launched early wait on SMs the other stream's kernels need.  Off by
 // default.
+std::atomic<int> g_conv_pdl_override{-1};  // dbl_set_conv_pdl: -1 = the environment's choice
+
 bool conv_pdl()
 {
-    static const bool on = [] {
+    static const bool env_on = [] {
         const char* e = getenv("DBL_CONV_PDL");
         return e && e[0] == '1';
     }();
-    return on;
+    const int o = g_conv_pdl_override.load(std::memory_order_relaxed);
+    return o < 0 ? env_on : o != 0;
 }
 
 int conv_attrs(int cg, cudaLaunchAttribute (&at)[2])
@@ -2300,3 +2305,10 @@ int dbl_device_status(int32_t* status)
 }
 
 }  // extern "C"
+
+extern "C" int dbl_set_conv_pdl(int32_t mode)
+{
+    if (mode < -1 || mode > 1) return dbl::set_error(DBL_ERR_INVALID, "set_conv_pdl: mode must be -1, 0 or 1");
+    g_conv_pdl_override.store(mode, std::memory_order_relaxed);
+    return DBL_OK;
+}

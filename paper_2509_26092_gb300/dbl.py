@@ -134,6 +134,7 @@ def lib(p=None):
             "dbl_loss_scale_update": (ctypes.c_int, [_V, _I32, _V]),
             "dbl_dropout_mask": (ctypes.c_int, [_I32, _I32, ctypes.c_float, ctypes.c_uint64, _V, _V, _V]),
             "dbl_event_wait": (ctypes.c_int, [_V, _D]),
+            "dbl_set_conv_pdl": (ctypes.c_int, [_I32]),
             "dbl_hold": (ctypes.c_int, [_V, _D, _V, _V]),
             "dbl_ps_dual_batch_merge": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams), _V]),
             "dbl_progressive_resize": (ctypes.c_int, [_V, ctypes.c_int, _I32, _I32, _I32, _I32, _V, ctypes.c_int,
@@ -353,6 +354,18 @@ def dbl_dropout_mask(n, c, drop_rate, seed, step, keep, stream=None):
     """keep [n, c] uint8: the mask dbl_head_fwd_bwd_ex draws for (drop_rate, seed, *step)."""
     _check(lib().dbl_dropout_mask(n, c, float(drop_rate), int(seed) & (2**64 - 1), _ptr(step), _ptr(keep),
                                   _stream(stream)))
+
+
+def dbl_set_conv_pdl(mode):
+    """Programmatic dependent launch of the convolutions that follow: 1 on, 0 off, -1 the
+    environment's choice (DBL_CONV_PDL), in both storage formats' libraries."""
+    for p in PRECISIONS:
+        _check_lib(lib(p), lib(p).dbl_set_conv_pdl(int(mode)))
+
+
+def _check_lib(L, rc):
+    if rc != DBL_OK:
+        raise DblError(rc, L.dbl_last_error().decode(errors="replace"))
 
 
 def dbl_event_wait(event, timeout_s):

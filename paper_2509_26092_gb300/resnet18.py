@@ -268,6 +268,9 @@ class Worker:
     def __init__(self, spec, batch, res, device="cuda", eps=1e-5, dropout=0.0, dropout_seed=0, precision="bf16"):
         self.spec, self.batch, self.res, self.eps = spec, batch, res, eps
         self.precision = precision
+        # programmatic dependent launch of this worker's convolutions: None leaves the library's
+        # setting (DBL_CONV_PDL), True / False override it while the step is enqueued
+        self.pdl = None
         # under loss scaling: the scale this worker's step used, copied from the server's at its start
         self.scale_used = torch.ones(1, dtype=torch.float32, device=device)
         # dropout before the FC layer (Sec. 4.1): rate, the worker's seed, and the device step
@@ -406,7 +409,13 @@ class Worker:
                 st = stream if isinstance(stream, torch.cuda.Stream) else torch.cuda.ExternalStream(stream)
                 with torch.cuda.stream(st):
                     self.scale_used.copy_(server.scale_state[0:1].view(torch.float32))
-            self._enqueue_step(server, images, native_res, stream)
+            if self.pdl is not None:
+                D.dbl_set_conv_pdl(1 if self.pdl else 0)
+            try:
+                self._enqueue_step(server, images, native_res, stream)
+            finally:
+                if self.pdl is not None:
+                    D.dbl_set_conv_pdl(-1)
 
     def _enqueue_step(self, server, images, native_res, stream):
         spec, B, eps = self.spec, self.batch, self.eps

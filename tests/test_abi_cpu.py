@@ -194,3 +194,11 @@ def test_cta_pairs_can_be_switched_off():
     env = dict(os.environ, DBL_CONV_CTA_PAIRS="0")
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
+
+
+def test_conv_pdl_setter_validates_its_mode(D):
+    """dbl_set_conv_pdl (host): 1, 0 and -1 are accepted by both libraries, anything else refused."""
+    for mode in (1, 0, -1):
+        D.dbl_set_conv_pdl(mode)
+    for p in D.PRECISIONS:
+        assert D.lib(p).dbl_set_conv_pdl(2) == D.DBL_ERR_INVALID
