@@ -110,10 +110,13 @@ int launch_resize(const void* in, void* out, int32_t n, int32_t hi, int32_t wi, 
 // element (e, t, ch) is the resized pixel at (y, q*sw + t - pw), channel ch
 // (zero outside the image, for t >= taps and for ch >= c).
 // One CTA per unrolled row (n, m): it interpolates the rg resized rows once
-// into shared memory (with pw zero columns on each side), then writes the
-// row's Q positions as 16-byte chunks (8 elements), consecutive threads on
-// consecutive chunks, each chunk gathered from the staged pixels with 16-byte
-// loads.  A resolution equal to the source's (lambda = 0, i0 = j: the
+// into shared memory (with pw zero columns on each side), each pixel rounded
+// to the storage format there, then writes the row's Q positions as 16-byte
+// chunks (8 elements), consecutive threads on consecutive chunks, each chunk
+// one 16-byte shared-memory load of two staged pixels (a tap pair) or of one
+// (8 channels).  Staging fp32 values and rounding every copy of a pixel in the
+// write phase issued twice the instructions there, with 8.7-way bank
+// conflicts.  A resolution equal to the source's (lambda = 0, i0 = j: the
 // interpolation returns the pixel itself, bit for bit) skips the taps.
 constexpr int kStemMaxW = 1024;  // widest resized row a CTA stages (host-checked)
 // Threads per CTA.  A CTA's two phases are short chains of dependent memory operations, so
@@ -141,6 +144,20 @@ __device__ __forceinline__ float stem_pixel<uint8_t>(const uint8_t* p, int ch, c
     return __fadd_rn(__fmul_rn((float)__ldg(p), nm.scale[ch]), nm.bias[ch]);
 }
 
+
+// Bilinear value from the four taps (a, b) on the upper source row and (c, d) on the lower one:
+// (1-l)*p + l*q as one rounded product (l*q) and one fused multiply-add, written out so that the
+// bits do not depend on how the compiler contracts the expression.
+__device__ __forceinline__ float lerp_rn(float p, float q, float l) { return __fmaf_rn(1.f - l, p, __fmul_rn(l, q)); }
+__device__ __forceinline__ float bilerp(float a, float b, float c, float d, float lx, float ly)
+{
+    return lerp_rn(lerp_rn(a, b, lx), lerp_rn(c, d, lx), ly);
+}
+
+// Staged row width in pixels: the resized row with pw zero columns on each side and 8 more for
+// the taps past its end, rounded up to an even count so that pixel pairs start on 16 bytes.
+__host__ __device__ __forceinline__ int32_t stem_staged_width(int32_t wo, int32_t pw) { return (wo + 2 * pw + 9) & ~1; }
+
 template <int RG, typename Tin>
 __global__ void __launch_bounds__(kStemThreads) resize_stem_kernel(const Tin* __restrict__ in, act_t* __restrict__ out,
                                                           int32_t hi, int32_t wi, int32_t c, int32_t ho, int32_t wo,
@@ -149,9 +166,9 @@ __global__ void __launch_bounds__(kStemThreads) resize_stem_kernel(const Tin* __
 {
     dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     constexpr int32_t cu = 8 / RG;  // channels per tap
-    // staged rows: [RG][wo + 2*pw + 8][cu] fp32, column x at index x + pw (dynamic shared memory)
-    extern __shared__ __align__(16) float rows[];
-    const int32_t wst = wo + 2 * pw + 8;
+    // staged rows: [RG][wst][cu] in the storage format (cu*2 bytes per pixel), column x at index x + pw
+    extern __shared__ __align__(16) uint8_t staged[];
+    const int32_t wst = stem_staged_width(wo, pw);
     const int32_t m = blockIdx.x % M, b = blockIdx.x / M;
     const Tin* base = in + (int64_t)b * hi * wi * c;
     const bool ident = hi == ho && wi == wo;
@@ -164,72 +181,71 @@ __global__ void __launch_bounds__(kStemThreads) resize_stem_kernel(const Tin* __
         yin[e] = y >= 0 && y < ho;
         ty[e] = axis_taps(yin[e] ? y : 0, hi, ho);
     }
-    // one staged pixel (all its channels) per thread and iteration
-#pragma unroll 2
-    for (int32_t i = threadIdx.x; i < RG * wst; i += blockDim.x) {
-        const int32_t xs = i % wst, e = i / wst;
+    // one staged column (its RG pixels, all channels) per thread and iteration: the column taps
+    // once for the RG rows, each pixel rounded to the storage format once (not once per copy)
+    for (int32_t xs = threadIdx.x; xs < wst; xs += blockDim.x) {
         const int32_t x = xs - pw;
-        float v[cu];
+        const bool in_x = x >= 0 && x < wo;
+        const Taps tx = axis_taps(in_x && !ident ? x : 0, wi, wo);
 #pragma unroll
-        for (int ch = 0; ch < cu; ++ch) v[ch] = 0.f;
-        Taps tyy = ty[0];
-        bool in_y = yin[0];
+        for (int e = 0; e < RG; ++e) {
+            float v[cu];
 #pragma unroll
-        for (int k = 1; k < RG; ++k)
-            if (e == k) {
-                tyy = ty[k];
-                in_y = yin[k];
+            for (int ch = 0; ch < cu; ++ch) v[ch] = 0.f;
+            if (yin[e] && in_x) {
+                if (ident) {
+                    const Tin* p = base + ((int64_t)ty[e].i0 * wi + x) * c;
+#pragma unroll
+                    for (int ch = 0; ch < cu; ++ch)
+                        if (ch < c) v[ch] = stem_pixel(p + ch, ch, nm);
+                } else {
+                    const Tin* r0 = base + (int64_t)ty[e].i0 * wi * c;
+                    const Tin* r1 = base + (int64_t)ty[e].i1 * wi * c;
+#pragma unroll
+                    for (int ch = 0; ch < cu; ++ch)
+                        if (ch < c)
+                            v[ch] = bilerp(stem_pixel(r0 + tx.i0 * c + ch, ch, nm),
+                                           stem_pixel(r0 + tx.i1 * c + ch, ch, nm),
+                                           stem_pixel(r1 + tx.i0 * c + ch, ch, nm),
+                                           stem_pixel(r1 + tx.i1 * c + ch, ch, nm), tx.lam, ty[e].lam);
+                }
             }
-        if (in_y && x >= 0 && x < wo) {
-            if (ident) {
-                const Tin* p = base + ((int64_t)tyy.i0 * wi + x) * c;
+            act2_t h[cu / 2];
 #pragma unroll
-                for (int ch = 0; ch < cu; ++ch)
-                    if (ch < c) v[ch] = stem_pixel(p + ch, ch, nm);
-            } else {
-                const Taps tx = axis_taps(x, wi, wo);
-                const Tin* r0 = base + (int64_t)tyy.i0 * wi * c;
-                const Tin* r1 = base + (int64_t)tyy.i1 * wi * c;
-#pragma unroll
-                for (int ch = 0; ch < cu; ++ch)
-                    if (ch < c) {
-                        const float top = (1.f - tx.lam) * stem_pixel(r0 + tx.i0 * c + ch, ch, nm) +
-                                          tx.lam * stem_pixel(r0 + tx.i1 * c + ch, ch, nm);
-                        const float bot = (1.f - tx.lam) * stem_pixel(r1 + tx.i0 * c + ch, ch, nm) +
-                                          tx.lam * stem_pixel(r1 + tx.i1 * c + ch, ch, nm);
-                        v[ch] = (1.f - tyy.lam) * top + tyy.lam * bot;
-                    }
-            }
+            for (int k = 0; k < cu / 2; ++k) h[k] = dbl::act::pack2(v[2 * k], v[2 * k + 1]);
+            uint8_t* dst = staged + ((size_t)e * wst + xs) * cu * 2;
+            if constexpr (cu == 4)
+                *reinterpret_cast<uint2*>(dst) = *reinterpret_cast<const uint2*>(h);
+            else
+                *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(h);
         }
-        float4* dst = reinterpret_cast<float4*>(rows + (int64_t)i * cu);
-#pragma unroll
-        for (int k = 0; k < cu / 4; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
     }
     __syncthreads();
+    // the unrolled row: 16-byte chunks gathered from the staged pixels, consecutive threads on
+    // consecutive chunks; a chunk is 16 staged bytes (two pixels of one row, or one of 8 channels)
     uint4* orow = reinterpret_cast<uint4*>(out) + ((int64_t)b * M + m) * Q * 8;
-    const float4* srow = reinterpret_cast<const float4*>(rows);  // staged pixel (e, xs): cu/4 float4 at (e*wst+xs)*cu/4
-    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+    const uint4 zero = make_uint4(0u, 0u, 0u, 0u);  // +0 in every lane of either format
+    const bool pairs16 = (sw & 1) == 0;  // pixel pairs q*sw + t0 (t0 even) start on 16 bytes
     for (int32_t idx = threadIdx.x; idx < Q * 8; idx += blockDim.x) {
         const int32_t q = idx >> 3, chunk = idx & 7;
-        float4 f[2];
+        uint4 val;
         if constexpr (RG == 2) {
             // chunk = (row e, tap pair): taps t0, t0+1 of 4 channels each
             const int32_t e = chunk >> 2, t0 = (chunk & 3) * 2;
-            const float4* pp = srow + (e * wst + q * sw + t0);
-            f[0] = t0 < taps ? pp[0] : zero;
-            f[1] = t0 + 1 < taps ? pp[1] : zero;
+            const uint8_t* pp = staged + ((size_t)e * wst + q * sw + t0) * 8;
+            if (pairs16) {
+                val = *reinterpret_cast<const uint4*>(pp);
+            } else {
+                const uint2 lo = *reinterpret_cast<const uint2*>(pp), hi2 = *reinterpret_cast<const uint2*>(pp + 8);
+                val = make_uint4(lo.x, lo.y, hi2.x, hi2.y);
+            }
+            if (t0 >= taps) val = zero;
+            if (t0 + 1 >= taps) val.z = val.w = 0u;
         } else {
             // chunk = tap t of 8 channels
-            const float4* pp = srow + 2 * (q * sw + chunk);
-            f[0] = chunk < taps ? pp[0] : zero;
-            f[1] = chunk < taps ? pp[1] : zero;
+            val = chunk < taps ? *reinterpret_cast<const uint4*>(staged + ((size_t)q * sw + chunk) * 16) : zero;
         }
-        act2_t qv[4];
-        qv[0] = dbl::act::pack2(f[0].x, f[0].y);
-        qv[1] = dbl::act::pack2(f[0].z, f[0].w);
-        qv[2] = dbl::act::pack2(f[1].x, f[1].y);
-        qv[3] = dbl::act::pack2(f[1].z, f[1].w);
-        orow[idx] = *reinterpret_cast<uint4*>(qv);
+        orow[idx] = val;
     }
 }
 
@@ -261,7 +277,7 @@ int resize_stem_impl(const Tin* in, int32_t n, int32_t h_in, int32_t w_in, int32
         return set_error(DBL_ERR_UNSUPPORTED, "progressive_resize_stem: rows wider than %d pixels", kStemMaxW);
     if (n == 0) return DBL_OK;
     const int blocks = n * rows_out;  // one CTA per unrolled row
-    const size_t smem = (size_t)(w_out + 2 * pad_w + 8) * 8 * sizeof(float);  // rg rows x 8/rg channels of fp32
+    const size_t smem = (size_t)stem_staged_width(w_out, pad_w) * 8 * sizeof(act_t);  // rg rows x 8/rg channels
     if (row_group == 2)
         resize_stem_kernel<2, Tin><<<blocks, kStemThreads, smem, as_stream(stream)>>>(
             in, static_cast<act_t*>(out), h_in, w_in, c, h_out, w_out, rows_out, Q, taps, stride_w, pad_w, pad_h,
