@@ -399,8 +399,8 @@ int bn_grid(int64_t nvec, int per_sm = kBlocksPerSM)
     return (int)(b < 1 ? 1 : b);
 }
 
-// One wave of CTAs that take the same number of partials each (512 partials on
-// 304 resident CTAs would leave 208 of them a second round alone).
+// One wave of CTAs that take the same number of partials each (more partials than
+// resident CTAs would leave some of them a second round alone).
 int reduce_grid(int64_t nblk)
 {
     const int64_t cap = (int64_t)dbl::sm_count() * kReduceBlocksPerSM;
@@ -426,12 +426,16 @@ int check_shape(const dbl_bn_shape* s, const char* who)
 
 // Backward reduce split: a fixed function of the shape (so the workspace size
 // and the summation order do not depend on the device): one partial per 2048
-// 8-channel vectors (8 per thread), at most 512 partials.
+// 8-channel vectors (8 per thread), at most kMaxBwdParts.  The cap is below the
+// reduce's resident CTAs on this GPU (two per SM), so a large tensor gets one
+// partial per CTA; a cap of 512 gave those CTAs two partials each and the
+// finalize twice the partials to add (8 us per call at layer4, batch 512).
+constexpr int64_t kMaxBwdParts = 256;
 int64_t bwd_blocks(int64_t count, int C)
 {
     if (count <= 0 || C <= 0) return 1;
     const int64_t b = (count * (C / 8) + 2047) / 2048;
-    return b < 1 ? 1 : b > 512 ? 512 : b;
+    return b < 1 ? 1 : b > kMaxBwdParts ? kMaxBwdParts : b;
 }
 
 template <int MASK>

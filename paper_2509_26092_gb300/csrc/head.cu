@@ -576,12 +576,15 @@ __global__ void softmax_ce_kernel(float* __restrict__ logits, const int32_t* __r
     for (int j = lane; j < J; j += 32) l[j] = (expf(l[j] - lse) - (j == lab ? 1.f : 0.f)) * invn;
 }
 
-// loss = mean(row_loss) (one block, fixed order); db[j] = sum_n dl[n, j].
-__global__ void head_reduce_kernel(const float* __restrict__ row_loss, const float* __restrict__ dl, int n, int J,
-                                   float* __restrict__ loss, float* __restrict__ db)
+// loss = mean(row_loss) (block 0, fixed order); db[j] = sum_n dl[n, j] (blocks 1..: 32 columns each,
+// warp w adding rows w, w + 8, ... in order, then the eight warp sums added in warp order).  Each
+// column's rows are spread over eight warps instead of one thread's chain of n dependent adds.
+constexpr int kHeadRedCols = 32;
+__global__ void __launch_bounds__(256) head_reduce_kernel(const float* __restrict__ row_loss, const float* __restrict__ dl,
+                                                          int n, int J, float* __restrict__ loss, float* __restrict__ db)
 {
+    __shared__ float red[256];
     if (blockIdx.x == 0) {
-        __shared__ float red[256];
         float s = 0.f;
         for (int i = threadIdx.x; i < n; i += blockDim.x) s += row_loss[i];
         red[threadIdx.x] = s;
@@ -593,11 +596,19 @@ __global__ void head_reduce_kernel(const float* __restrict__ row_loss, const flo
         if (threadIdx.x == 0) *loss = red[0] / (float)n;
         return;
     }
-    const int j = (blockIdx.x - 1) * blockDim.x + threadIdx.x;
-    if (j >= J) return;
+    const int lane = threadIdx.x % 32, w = threadIdx.x / 32;
+    const int j = (blockIdx.x - 1) * kHeadRedCols + lane;
     float s = 0.f;
-    for (int i = 0; i < n; ++i) s += dl[(int64_t)i * J + j];
-    db[j] = s;
+    if (j < J)
+        for (int i = w; i < n; i += 8) s += dl[(int64_t)i * J + j];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    if (w == 0 && j < J) {
+        float t = red[lane];
+#pragma unroll
+        for (int k = 1; k < 8; ++k) t += red[k * 32 + lane];
+        db[j] = t;
+    }
 }
 
 // dx[n, i, c] = df[n, c] / hw, with dropout (df[n, c] * mult[n, c]) / hw
@@ -746,7 +757,8 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
         return rc;
     softmax_ce_kernel<<<(n * 32 + 255) / 256, 256, 0, s>>>(logits, labels, n, classes, row_loss, loss_scale);
     if ((rc = launch_check("softmax_ce launch"))) return rc;
-    head_reduce_kernel<<<1 + (classes + 255) / 256, 256, 0, s>>>(row_loss, logits, n, classes, loss, dfc_b);
+    head_reduce_kernel<<<1 + (classes + kHeadRedCols - 1) / kHeadRedCols, 256, 0, s>>>(row_loss, logits, n, classes,
+                                                                                        loss, dfc_b);
     if ((rc = launch_check("head reduce launch"))) return rc;
     // dW[j, c] = sum_n dl[n, j] feat[n, c]
     if ((rc = gemm_f32(logits, 1, classes, feat, 1, c, nullptr, dfc_w, c, classes, c, n, part, s, "fc dW launch")))
