@@ -611,6 +611,70 @@ __global__ void __launch_bounds__(256) head_reduce_kernel(const float* __restric
     }
 }
 
+// The same two passes with one CTA per image, blockDim = S slices x (C/8) channel groups: thread
+// (slice s, group g) takes the rows i = s, s + S, ... of its image (consecutive threads on
+// consecutive 16-byte vectors of a row).  Forward: each slice adds its rows in order, then the S
+// slice sums are added in slice order.  Backward: each thread computes its 8 gradients once and
+// writes them to its rows.  (One thread per (image, group) walking all hw rows, or loading its
+// 16 fp32 factors again for every row, left these passes at a fifth of HBM.)
+__device__ __forceinline__ int pool_slices(int groups) { return groups >= 1024 ? 1 : min(8, 1024 / groups); }
+
+__global__ void __launch_bounds__(1024) avgpool_img_kernel(const act_t* __restrict__ x, float* __restrict__ feat,
+                                                           int hw, int C, Dropout dp)
+{
+    extern __shared__ float slice_sum[];  // [S][C]
+    const int groups = C / 8, S = pool_slices(groups);
+    const int g = threadIdx.x % groups, sl = threadIdx.x / groups;
+    const int b = blockIdx.x;
+    float acc[8] = {};
+    for (int i = sl; i < hw; i += S) {
+        float f[8];
+        unpack8(__ldg(reinterpret_cast<const uint4*>(x + ((int64_t)b * hw + i) * C) + g), f);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] += f[k];
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) slice_sum[sl * C + 8 * g + k] = acc[k];
+    __syncthreads();
+    if (sl != 0) return;
+    for (int q = 1; q < S; ++q)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] += slice_sum[q * C + 8 * g + k];
+    const float inv = 1.0f / (float)hw;
+    if (dp.thr) {
+        const uint64_t st = *dp.step;
+        const uint64_t q = (uint64_t)b * (uint64_t)(C / 4) + 2 * (uint64_t)g;
+        const unsigned bits = dropout_keep4(dp.seed, st, q, dp.thr) | dropout_keep4(dp.seed, st, q + 1, dp.thr) << 4;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const float m = (bits >> k) & 1 ? dp.scale : 0.f;
+            dp.mult[(int64_t)b * C + 8 * g + k] = m;
+            feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv * m;
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) feat[(int64_t)b * C + 8 * g + k] = acc[k] * inv;
+    }
+}
+
+__global__ void __launch_bounds__(1024) avgpool_bwd_img_kernel(const float* __restrict__ df, act_t* __restrict__ dx,
+                                                               int hw, int C, const float* __restrict__ mult)
+{
+    const int groups = C / 8, S = pool_slices(groups);
+    const int g = threadIdx.x % groups, sl = threadIdx.x / groups;
+    const int b = blockIdx.x;
+    const float inv = 1.0f / (float)hw;
+    float f[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int64_t e = (int64_t)b * C + 8 * g + k;
+        f[k] = (mult ? df[e] * mult[e] : df[e]) * inv;
+    }
+    const uint4 v = pack8(f);
+    uint4* row = reinterpret_cast<uint4*>(dx + (int64_t)b * hw * C) + g;
+    for (int i = sl; i < hw; i += S) row[(int64_t)i * groups] = v;
+}
+
 // dx[n, i, c] = df[n, c] / hw, with dropout (df[n, c] * mult[n, c]) / hw
 __global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, act_t* __restrict__ dx,
                                                           int n, int hw, int C, const float* __restrict__ mult)
@@ -749,8 +813,15 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
     }
     cudaStream_t s = as_stream(stream);
     int rc;
-    avgpool_kernel<<<grid_for((int64_t)n * (c / 8), 256), 256, 0, s>>>(static_cast<const act_t*>(x), feat, n,
-                                                                       hw, c, dp);
+    const int groups = c / 8;
+    const bool per_image = groups <= 1024;  // one CTA per image (at most 1024 threads)
+    const int S = groups >= 1024 ? 1 : std::min(8, 1024 / groups);
+    if (per_image)
+        avgpool_img_kernel<<<n, S * groups, (size_t)S * c * sizeof(float), s>>>(static_cast<const act_t*>(x), feat,
+                                                                                 hw, c, dp);
+    else
+        avgpool_kernel<<<grid_for((int64_t)n * groups, 256), 256, 0, s>>>(static_cast<const act_t*>(x), feat, n, hw,
+                                                                           c, dp);
     if ((rc = launch_check("avgpool launch"))) return rc;
     // logits = feat * W^T + b
     if ((rc = gemm_f32(feat, c, 1, fc_w, c, 1, fc_b, logits, classes, n, classes, c, part, s, "fc fwd launch")))
@@ -766,8 +837,11 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
     // df[n, c] = sum_j dl[n, j] W[j, c]
     if ((rc = gemm_f32(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes, part, s, "fc dX launch")))
         return rc;
-    avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * (c / 8), 256), 256, 0, s>>>(
-        df, static_cast<act_t*>(dx), n, hw, c, dp.thr ? mult : nullptr);
+    if (per_image)
+        avgpool_bwd_img_kernel<<<n, S * groups, 0, s>>>(df, static_cast<act_t*>(dx), hw, c, dp.thr ? mult : nullptr);
+    else
+        avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * groups, 256), 256, 0, s>>>(df, static_cast<act_t*>(dx), n, hw,
+                                                                                    c, dp.thr ? mult : nullptr);
     if ((rc = launch_check("avgpool_bwd launch")) || !dp.thr) return rc;
     dropout_advance_kernel<<<1, 1, 0, s>>>(step);  // the next call draws a fresh mask
     return launch_check("dropout advance launch");
