@@ -116,7 +116,8 @@ struct Cfg {
     static constexpr int EPI_TILE = 4 * 32 * 33 * 4;           // per-warp 32x32 transpose scratch
     static constexpr int EPI_SUM = 4 * 2 * kMaxNcols * 4;      // per-warp channel sums (fwd)
     static constexpr int SMEM = RING + EPI_TILE + EPI_SUM + 1024;  // + 1 KB alignment slack
-    static constexpr uint32_t TMEM_COLS = 2 * ACC * BN;         // two tiles in flight
+    static constexpr int NB = ACC * BN <= 128 ? 4 : 2;          // tiles in flight (TMEM accumulator buffers)
+    static constexpr uint32_t TMEM_COLS = NB * ACC * BN;
     static constexpr int THREADS = 32 * (4 + kProducers + 1);   // epilogue, producers, MMA
     static constexpr int MMA_WARP = 4 + kProducers;
     static_assert(STAGES >= 2, "ring too shallow");
@@ -377,7 +378,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
     using C = Cfg<BN, FAM, CG>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accf_bar[2], acce_bar[2], drain_bar;
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES], accf_bar[C::NB], acce_bar[C::NB], drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
 
@@ -394,7 +395,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::NB; ++b) {
             mbar_init(&accf_bar[b], 1);
             mbar_init(&acce_bar[b], 4 * CG);  // one arrival per epilogue warp of the pair
         }
@@ -534,8 +535,8 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
             const TileCoord tc = decode_tile(p, t, nunits);
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
-            const int buf = lt & 1;
-            if (!wait_ok(&acce_bar[buf], ((lt >> 1) & 1) ^ 1) ||
+            const int buf = lt % C::NB;
+            if (!wait_ok(&acce_bar[buf], ((lt / C::NB) & 1) ^ 1) ||
                 (nkb > 0 && !wait_ok(&full_bar[it % STAGES], (it / STAGES) & 1))) {
                 failed = true;
                 break;
@@ -586,8 +587,8 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
             const TileCoord tc = decode_tile(p, t, nunits);
             int kb0, nkb;
             kb_range(p, tc.z, kb0, nkb);
-            const int buf = lt & 1;
-            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
+            const int buf = lt % C::NB;
+            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt / C::NB) & 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
                 if (lane == 0) report_timeout(&abort_flag);
                 break;
@@ -709,7 +710,8 @@ constexpr int kWinThreads = 224;         // conv_wgwin_kernel: 4 epilogue warps,
 template <int BN>
 struct WinCfg {
     static constexpr int B_TILE = BN * 64 * 2;  // one tap x one 64-channel block of weights
-    static constexpr uint32_t TMEM_COLS = 2 * kWinACC * BN;
+    static constexpr int NB = BN == 64 ? 4 : 2;  // accumulator buffers (tiles in flight)
+    static constexpr uint32_t TMEM_COLS = NB * kWinACC * BN;
     static constexpr int EPI = 4;                // epilogue warps
     static constexpr int CW = BN * 4 / EPI;      // columns one epilogue warp drains
     static constexpr int W_STRIP = EPI, W_WEIGHT = EPI + 1, W_MMA = EPI + 2;
@@ -758,8 +760,8 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
     constexpr int BT = C::B_TILE / CG;  // this CTA's bytes of one tap x 64-channel block of weights
     constexpr uint16_t kAll = CG == 2 ? 3 : 1;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t sfull[2], sempty[2], bfull[kWinBStages], bempty[kWinBStages], accf_bar[2],
-        acce_bar[2], drain_bar;
+    __shared__ __align__(8) uint64_t sfull[2], sempty[2], bfull[kWinBStages], bempty[kWinBStages], accf_bar[4],
+        acce_bar[4], drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
 
@@ -782,6 +784,8 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sfull[i], 1);
             mbar_init(&sempty[i], 1);
+        }
+        for (int i = 0; i < C::NB; ++i) {
             mbar_init(&accf_bar[i], 1);
             mbar_init(&acce_bar[i], C::EPI * CG);  // one arrival per epilogue warp of the pair
         }
@@ -905,8 +909,8 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
             failed = __any_sync(0xffffffffu, ok == 0u);
         }
         for (int t = unit0; t < total_units && (CG == 1 || rank == 0) && !failed; t += nunits, ++lt) {
-            const int buf = lt & 1;
-            const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt >> 1) & 1) ^ 1, &abort_flag);
+            const int buf = lt % C::NB;
+            const uint32_t ok = mbar_wait_warp(&acce_bar[buf], ((lt / C::NB) & 1) ^ 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
                 failed = true;
                 break;
@@ -979,8 +983,8 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
         int lt = 0;
         for (int t = unit0; t < total_units; t += nunits, ++lt) {
             const int m_tile = t * CG + rank;
-            const int buf = lt & 1;
-            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt >> 1) & 1, &abort_flag);
+            const int buf = lt % C::NB;
+            const uint32_t ok = mbar_wait_warp(&accf_bar[buf], (lt / C::NB) & 1, &abort_flag);
             if (__any_sync(0xffffffffu, ok == 0u)) {
                 if (lane == 0) report_timeout(&abort_flag);
                 break;
