@@ -70,6 +70,7 @@ struct ConvParams {
     // outputs
     void* out;          // bf16 rows (fwd, dgrad); fp32 dw (wgrad, one slice) or fp32 slices [z][Ncols][M]
     int64_t ldo;        // elements between output rows (fwd, dgrad)
+    int st32;           // 16-bit outputs whose base and row pitch are multiples of 32 bytes: 32-byte stores
     int wg_accumulate;  // wgrad with one slice: add into dw
     float* stats;       // fwd: [gridDim.x][2][Ncols] per-CTA channel sums, or nullptr
     // window kernel (3x3, stride 1, pad 1): the batch as one column of zero-padded images
@@ -261,9 +262,20 @@ __device__ __forceinline__ void store_row_chunk_act(const ConvParams& p, const u
         back[2 * k + 1] = f.y;
     }
     if (valid) {
-        uint4* o = reinterpret_cast<uint4*>(static_cast<act_t*>(p.out) + out_row * p.ldo + col0);
+        act_t* o = static_cast<act_t*>(p.out) + out_row * p.ldo + col0;
+        if (p.st32) {
+            // whole 32-byte sectors per instruction: half the store instructions and L2 write
+            // requests of 16-byte stores, each of which fills half a sector
 #pragma unroll
-        for (int k = 0; k < 4; ++k) o[k] = pk[k];
+            for (int k = 0; k < 2; ++k)
+                asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(o + 16 * k),
+                             "r"(pk[2 * k].x), "r"(pk[2 * k].y), "r"(pk[2 * k].z), "r"(pk[2 * k].w),
+                             "r"(pk[2 * k + 1].x), "r"(pk[2 * k + 1].y), "r"(pk[2 * k + 1].z), "r"(pk[2 * k + 1].w)
+                             : "memory");
+        } else {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) reinterpret_cast<uint4*>(o)[k] = pk[k];
+        }
     }
 }
 
@@ -2102,6 +2114,7 @@ int conv_fwd_impl(const dbl_conv_shape* s, const void* x, const void* w, void* y
         if ((rc = enc_tiled(&tb, w, 2, dims, str, box, true))) return rc;
     }
     pl.p.out = y;
+    pl.p.st32 = (reinterpret_cast<uintptr_t>(y) % 32 == 0) && (pl.p.ldo * (int64_t)sizeof(act_t)) % 32 == 0;
     pl.p.stats = stats ? static_cast<float*>(ws) : nullptr;
     const int grid = plan_grid(pl);
     cudaStream_t st = as_stream(stream);
@@ -2165,6 +2178,7 @@ int conv_dgrad_impl(const dbl_conv_shape* s, const void* dy, const void* w, int 
         pl.p.proj_kb = k2 / 64;
     }
     pl.p.out = dx;
+    pl.p.st32 = (reinterpret_cast<uintptr_t>(dx) % 32 == 0) && (pl.p.ldo * (int64_t)sizeof(act_t)) % 32 == 0;
     const int grid = plan_grid(pl);
     return pl.win ? launch_win(pl, ta, tb, grid, as_stream(stream))
                   : launch(pl, ta, tb, ta2, tb2, grid, as_stream(stream));
