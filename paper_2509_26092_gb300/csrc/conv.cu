@@ -768,7 +768,7 @@ __global__ void __launch_bounds__(WinCfg<BN>::THREADS, 1)
 {
     dbl::dev::grid_dependency_trigger();  // a convolution launched next may start its set-up
     using C = WinCfg<BN>;
-    static_assert(CG == 1 || BN == 128, "CTA pairs split the weights in 64-column halves");
+    static_assert(CG == 1 || BN == 128 || !DG, "data-gradient pairs split the weights in 64-column halves");
     constexpr int BT = C::B_TILE / CG;  // this CTA's bytes of one tap x 64-channel block of weights
     constexpr uint16_t kAll = CG == 2 ? 3 : 1;
     extern __shared__ uint8_t smem_raw[];
@@ -1446,6 +1446,7 @@ int win_tile_positions(int Wp) { return Wp >= 64 ? (kWinBMT / Wp) * Wp : kWinBMT
 // channels, padded rows of 10..256 positions; the data gradient (dgrad) for
 // 3x3 filters with pad 1 only (its taps are the forward taps flipped).
 bool win_pairs();
+int cta_pair_level();
 
 bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& pl)
 {
@@ -1469,10 +1470,14 @@ bool win_setup(const dbl_conv_shape* s, int red_c, int out_c, bool dgrad, Plan& 
     // CTA pairs for 128-column tiles: each SM stages half of the weights; rank 1's strip is
     // shifted by up to a padded row either way, so each strip buffer gets a margin of one padded
     // row on both sides (single CTAs when the pair layout does not fit in shared memory).  The
-    // 64-column forward pass measured slower on pairs (818 against 959 TFLOP/s at layer1).
+    // 64-column forward pass with resident weights runs on pairs only with DBL_CONV_CTA_PAIRS=2:
+    // it halves each SM's weight reads (a sixth of its tensor-core shared-memory reads) but
+    // couples the two CTAs' loads and epilogues; with two accumulator buffers it measured slower
+    // (layer1 forward at batch 384: 113 against 97 us), with four the same (122 against 123 us
+    // at batch 512).
     if ((size_t)srows * Wp * 128 >= (1u << 20)) return false;
     const int epi = out_c == 64 ? WinCfg<64>::EPI : WinCfg<128>::EPI;
-    int cg = win_pairs() && BN == 128 ? 2 : 1;
+    int cg = win_pairs() && (BN == 128 || (BN == 64 && res && !dgrad && cta_pair_level() == 2)) ? 2 : 1;
     int margin = 0;
     size_t smem = 0;
     for (;; cg = 1) {
@@ -1575,26 +1580,26 @@ bool wgwin_setup(const dbl_conv_shape* s, Plan& pl)
 // extra synchronisation; the short-K forward and data-gradient passes of 128
 // columns measured slower on pairs).  The environment variable DBL_CONV_CTA_PAIRS
 // overrides this: 0 = never, 2 = every 128- and 256-column tile.
-bool pair_tiles(int BN, bool wgrad)
+int cta_pair_level()
 {
     static const int level = [] {
         const char* e = getenv("DBL_CONV_CTA_PAIRS");
         return e && (e[0] == '0' || e[0] == '2') ? e[0] - '0' : 1;
     }();
+    return level;
+}
+
+bool pair_tiles(int BN, bool wgrad)
+{
+    const int level = cta_pair_level();
     if (level == 0) return false;
     return BN == 256 || (BN == 128 && (wgrad || level == 2));
 }
 
-// Window-kernel CTA pairs (128-column tiles); DBL_CONV_CTA_PAIRS=0 turns them off with
-// the others.
-bool win_pairs()
-{
-    static const bool on = [] {
-        const char* e = getenv("DBL_CONV_CTA_PAIRS");
-        return !(e && e[0] == '0');
-    }();
-    return on;
-}
+// Window-kernel CTA pairs: 128-column tiles; with DBL_CONV_CTA_PAIRS=2 also the 64-column
+// forward pass with resident weights (measured no faster, for comparison); DBL_CONV_CTA_PAIRS=0
+// turns them off with the others.
+bool win_pairs() { return cta_pair_level() != 0; }
 
 int make_plan(const dbl_conv_shape* s, int pass, Plan& pl)
 {
@@ -1984,7 +1989,9 @@ int win_grid(const Plan& pl)
 {
     if (pl.cg == 1) return grid_size(pl.p.total_tiles);
     const bool dg = pl.mode == kDgrad;
-    int pairs = dg ? resident_win_pairs<128, true, false>(pl.smem) : resident_win_pairs<128, false, false>(pl.smem);
+    int pairs = pl.BN == 64 ? resident_win_pairs<64, false, true>(pl.smem)
+                : dg        ? resident_win_pairs<128, true, false>(pl.smem)
+                            : resident_win_pairs<128, false, false>(pl.smem);
     const int units = (pl.p.total_tiles + 1) / 2;
     if (pairs > units) pairs = units;
     return 2 * std::max(pairs, 1);
@@ -2017,7 +2024,8 @@ int launch_win(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, int g
     if (pl.cg == 2) {
         if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false, 2>(pl, a, b, grid, st)
                                     : launch_win_cfg<128, false, false, 2>(pl, a, b, grid, st);
-        return dbl::set_error(DBL_ERR_UNSUPPORTED, "conv: CTA-pair window kernels need 128 columns");
+        if (pl.BN == 64 && pl.res && !dg) return launch_win_cfg<64, false, true, 2>(pl, a, b, grid, st);
+        return dbl::set_error(DBL_ERR_UNSUPPORTED, "conv: no CTA-pair window kernel for this plan");
     }
     if (pl.BN == 128) return dg ? launch_win_cfg<128, true, false, 1>(pl, a, b, grid, st)
                                 : launch_win_cfg<128, false, false, 1>(pl, a, b, grid, st);

@@ -196,6 +196,26 @@ def test_cta_pairs_can_be_switched_off():
     assert r.returncode == 0, r.stderr[-2000:]
 
 
+def test_window_pairs_of_64_columns_only_for_comparison():
+    """The 64-column window forward pass with resident weights runs on CTA pairs only with
+    DBL_CONV_CTA_PAIRS=2 (measured no faster); its data gradient never does."""
+    import subprocess
+    import sys
+    code = ("from paper_2509_26092_gb300 import build_lib\nbuild_lib.build()\n"
+            "from paper_2509_26092_gb300 import dbl as D\nimport sys\n"
+            "i = D.dbl_conv_plan(D.conv_shape(512, 56, 56, 64, 64, 3, 1, 1), 0)\n"
+            "d = D.dbl_conv_plan(D.conv_shape(512, 56, 56, 64, 64, 3, 1, 1), 1)\n"
+            "assert i.kernel == D.DBL_KERNEL_WINDOW and d.ctas_per_mma == 1\n"
+            "print(i.ctas_per_mma)\n")
+    got = {}
+    for level in ("1", "2"):
+        r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=dict(os.environ, DBL_CONV_CTA_PAIRS=level),
+                           capture_output=True, text=True, timeout=300)
+        assert r.returncode == 0, r.stderr[-2000:]
+        got[level] = int(r.stdout.split()[-1])
+    assert got == {"1": 1, "2": 2}
+
+
 def test_conv_pdl_setter_validates_its_mode(D):
     """dbl_set_conv_pdl (host): 1, 0 and -1 are accepted by both libraries, anything else refused."""
     for mode in (1, 0, -1):

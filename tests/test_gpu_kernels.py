@@ -486,6 +486,54 @@ def test_conv_fwd_matches_oracle(D, case):
     check_status(D)
 
 
+_PAIR64_IN_CHILD = r"""
+import sys, torch, numpy as np
+sys.path.insert(0, sys.argv[1])
+from paper_2509_26092_gb300 import build_lib
+build_lib.build()
+from paper_2509_26092_gb300 import dbl as D
+cases = [(32, 56, 56), (3, 7, 9), (2, 8, 8)]
+out = []
+for i, (n, h, w) in enumerate(cases):
+    shape = D.conv_shape(n, h, w, 64, 64, 3, 1, 1)
+    assert D.dbl_conv_plan(shape, D.DBL_PASS_FWD).ctas_per_mma == int(sys.argv[3])
+    g = np.random.default_rng(100 + i)
+    x = torch.from_numpy(g.standard_normal((n, h, w, 64)).astype(np.float32)).cuda().to(torch.bfloat16)
+    wt = torch.from_numpy((0.05 * g.standard_normal((64, 3, 3, 64))).astype(np.float32)).cuda().to(torch.bfloat16)
+    y = torch.full((n, h, w, 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    s1, s2 = torch.empty(64, device="cuda"), torch.empty(64, device="cuda")
+    wsb = D.dbl_conv_workspace_bytes(shape, D.DBL_PASS_FWD)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    D.dbl_conv_fwd(shape, x, wt, y, s1, s2, ws, wsb)
+    out.append((y.cpu(), s1.cpu(), s2.cpu()))
+torch.cuda.synchronize()
+assert D.dbl_device_status() == D.DBL_OK
+torch.save(out, sys.argv[2])
+"""
+
+
+def test_window_pairs_of_64_columns_give_the_same_outputs(tmp_path):
+    """The 64-column window forward pass on CTA pairs (DBL_CONV_CTA_PAIRS=2, read once per process,
+    hence child processes; M = 256 MMAs across two SMs, half of the resident weights in each) stores
+    the same bits and channel sums as on single CTAs, on tiles that fill pairs, leave the second
+    CTA of the last pair without a tile, and span several small images."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    got = {}
+    for level, cg in (("1", "1"), ("2", "2")):
+        path = str(tmp_path / f"y{level}.pt")
+        r = subprocess.run([sys.executable, "-c", _PAIR64_IN_CHILD, root, path, cg], capture_output=True, text=True,
+                           timeout=600, env=dict(os.environ, DBL_CONV_CTA_PAIRS=level))
+        assert r.returncode == 0, r.stderr[-2000:]
+        got[level] = torch.load(path)
+    for a, b in zip(got["1"], got["2"]):
+        assert torch.isfinite(a[0].float()).all()
+        for t1, t2 in zip(a, b):
+            assert torch.equal(t1, t2)
+
+
 @pytest.mark.parametrize("case", [(2, 8, 8, 64, 64, 3, 1, 1), (4, 14, 14, 256, 512, 3, 2, 1), (32, 14, 14, 256, 256, 3, 1, 1),
                                   (8, 16, 16, 64, 128, 3, 1, 1), (2, 8, 8, 64, 128, 1, 2, 0)])
 def test_conv_fwd_parts_then_bn_matches_two_step_path(D, case):
