@@ -106,6 +106,18 @@ DBL_API int dbl_device_status(int32_t* status);
  * 0 = off, -1 = back to the environment's choice.  Launches already enqueued
  * (or captured) keep the attribute they were launched with. */
 DBL_API int dbl_set_conv_pdl(int32_t mode);
+
+/* Host, for tests of the bounded waits: arms the next implicit-GEMM
+ * convolution launch (a pass that dbl_conv_plan reports as
+ * DBL_KERNEL_IGEMM) of this process so that its thread block 0 never
+ * issues the load of its first K-block.  That block's MMA issuer then waits
+ * on a stage that never fills; the wait gives up after its limit (about 2 s),
+ * records DBL_ERR_TIMEOUT in the device status (dbl_device_status), and every
+ * role of the block winds down through its own bounded waits, letting the
+ * copies it issued land before it returns.  The other blocks finish normally;
+ * the launch's outputs are not valid.  No fault is raised and the context
+ * stays usable.  Applies to one launch, then disarms itself. */
+DBL_API int dbl_conv_test_stall_next(void);
 typedef struct {
     int32_t n, h, w, c; /* input activation shape (NHWC)                    */
     int32_t k, r, s;    /* output channels and filter size (KRSC weights)   */

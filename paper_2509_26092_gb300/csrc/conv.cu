@@ -83,6 +83,7 @@ struct ConvParams {
     int win_dyrows;           // weight gradient: padded rows of the dy strip
     int win_strip_bytes;      // bytes of one strip buffer, or of one x + dy stage (a multiple of 1024)
     int win_margin;           // CTA pairs: bytes before and after each strip buffer (0 for single CTAs)
+    int test_stall;           // dbl_conv_test_stall_next: block 0 never loads its first K-block
 };
 
 __device__ __forceinline__ void report_timeout(volatile int* abort)
@@ -457,6 +458,7 @@ __global__ void __launch_bounds__(Cfg<BN, FAM, CG>::THREADS, 1)
             }
             for (int k = 0; k < nkb; ++k, ++it) {
                 if (it % kProducers != prod) continue;
+                if (p.test_stall && blockIdx.x == 0 && it == 0) continue;  // stage 0 never fills (bounded-wait test)
                 const int s = it % STAGES;
                 const uint32_t ok = mbar_wait_warp(&empty_bar[s], ((it / STAGES) & 1) ^ 1, &abort_flag);
                 if (__any_sync(0xffffffffu, ok == 0u)) {
@@ -1854,6 +1856,7 @@ int plan_grid(const Plan& pl)
 // 1.1% slower, because CTAs launched early wait on SMs the other stream's kernels need.  Off by
 // default.
 std::atomic<int> g_conv_pdl_override{-1};  // dbl_set_conv_pdl: -1 = the environment's choice
+std::atomic<int> g_conv_stall_next{0};     // dbl_conv_test_stall_next: arms one implicit-GEMM launch
 
 bool conv_pdl()
 {
@@ -1898,7 +1901,9 @@ int launch_cfg(const Plan& pl, const CUtensorMap& a, const CUtensorMap& b, const
     cfg.stream = st;
     cfg.attrs = at;
     cfg.numAttrs = conv_attrs(CG, at);
-    cudaError_t e = cudaLaunchKernelEx(&cfg, conv_igemm_kernel<BN, FAM, CG>, a, b, a2, b2, pl.p);
+    ConvParams prm = pl.p;
+    if (g_conv_stall_next.exchange(0)) prm.test_stall = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, conv_igemm_kernel<BN, FAM, CG>, a, b, a2, b2, prm);
     if (e != cudaSuccess) {
         dbl::count_launch();
         return dbl::cuda_check(e, "conv_igemm launch");
@@ -2331,6 +2336,12 @@ int dbl_device_status(int32_t* status)
 }
 
 }  // extern "C"
+
+extern "C" int dbl_conv_test_stall_next(void)
+{
+    g_conv_stall_next.store(1);
+    return DBL_OK;
+}
 
 extern "C" int dbl_set_conv_pdl(int32_t mode)
 {

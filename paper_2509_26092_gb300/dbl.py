@@ -135,6 +135,7 @@ def lib(p=None):
             "dbl_dropout_mask": (ctypes.c_int, [_I32, _I32, ctypes.c_float, ctypes.c_uint64, _V, _V, _V]),
             "dbl_event_wait": (ctypes.c_int, [_V, _D]),
             "dbl_set_conv_pdl": (ctypes.c_int, [_I32]),
+            "dbl_conv_test_stall_next": (ctypes.c_int, []),
             "dbl_hold": (ctypes.c_int, [_V, _D, _V, _V]),
             "dbl_ps_dual_batch_merge": (ctypes.c_int, [_V, _V, _V, _V, _V, _I64, ctypes.POINTER(MergeParams), _V]),
             "dbl_progressive_resize": (ctypes.c_int, [_V, ctypes.c_int, _I32, _I32, _I32, _I32, _V, ctypes.c_int,
@@ -210,6 +211,12 @@ def dbl_device_status():
 def conv_shape(n, h, w, c, k, r, stride, pad, s=None, stride_w=0, pad_w=0):
     """dbl_conv_shape; s defaults to r, stride_w == 0 means the same stride and pad along W."""
     return ConvShape(n, h, w, c, k, r, r if s is None else s, stride, pad, stride_w, pad_w)
+
+
+def dbl_conv_test_stall_next():
+    """Test hook: the next implicit-GEMM convolution launch's block 0 never loads its first
+    K-block, so its bounded MMA wait runs out and the device status reports DBL_ERR_TIMEOUT."""
+    _check(lib().dbl_conv_test_stall_next())
 
 
 def dbl_conv_workspace_bytes(shape, pass_):
