@@ -87,14 +87,15 @@ __global__ void __launch_bounds__(kThreads) bn_stats_kernel(const act_t* __restr
 
 // ----------------------------------------------------------------------------- forward apply
 // Batch statistics -> saved mean and 1/std, once per channel (fp64: the
-// variance is E[y^2] - E[y]^2 of sums over up to 10^8 rows).
-__global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const float* __restrict__ sum,
+// variance is E[y^2] - E[y]^2 of sums over up to 10^8 rows).  inv_n = 1/count is
+// divided on the host (the same correctly rounded value; an fp64 division on the
+// device is a long chain of the GPU's slow fp64 operations).
+__global__ void bn_fwd_finalize_kernel(double inv_n, int C, float eps, const float* __restrict__ sum,
                                        const float* __restrict__ sumsq, float* __restrict__ save_mean,
                                        float* __restrict__ save_invstd)
 {
     const int c = blockIdx.x * blockDim.x + threadIdx.x;
     if (c >= C) return;
-    const double inv_n = 1.0 / (double)count;
     const double mean = (double)sum[c] * inv_n;
     double var = (double)sumsq[c] * inv_n - mean * mean;
     if (var < 0.0) var = 0.0;
@@ -106,7 +107,7 @@ __global__ void bn_fwd_finalize_kernel(int64_t count, int C, float eps, const fl
 // The same finalize from a convolution's per-CTA partials part[nparts][2][C]: the
 // fixed-order partial sums (partials_colsum, rounded to fp32 as dbl_conv_fwd stores
 // them), then mean and 1/std exactly as above.
-__global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_parts_kernel(int64_t count, int C, float eps,
+__global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_parts_kernel(double inv_n, int C, float eps,
                                                                     const float* __restrict__ part, int nparts,
                                                                     float* __restrict__ save_mean,
                                                                     float* __restrict__ save_invstd)
@@ -115,7 +116,6 @@ __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_fwd_finalize_pa
     const int c = dbl::dev::partials_colsum(part, nparts, C, ds, dq);
     if (c < 0) return;
     const float sum = (float)ds, sumsq = (float)dq;
-    const double inv_n = 1.0 / (double)count;
     const double mean = (double)sum * inv_n;
     double var = (double)sumsq * inv_n - mean * mean;
     if (var < 0.0) var = 0.0;
@@ -326,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, kReduceBlocksPerSM)
 // dbeta and the three per-channel coefficients (A, B, C) of the apply pass
 // dy = A*g + B*y + C.
 __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_bwd_finalize_kernel(
-    const float* __restrict__ partial, int nblk, int C, int64_t count, const float* __restrict__ gamma,
+    const float* __restrict__ partial, int nblk, int C, double inv_n, const float* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ invstd, float* __restrict__ dgamma,
     float* __restrict__ dbeta, float* __restrict__ coef)
 {
@@ -337,11 +337,11 @@ __global__ void __launch_bounds__(dbl::dev::kPartialsThreads) bn_bwd_finalize_ke
     dgamma[c] = (float)sgx;
     // dy = k1*(g - sum(g)/n - xhat*sum(g*xhat)/n), xhat = (y - mean)*invstd, as A*g + B*y + C
     const double k1 = (double)gamma[c] * (double)invstd[c];
-    const double k3 = sgx / (double)count;
+    const double k3 = sgx * inv_n;  // inv_n = 1/count, divided on the host
     const double b = -k1 * (double)invstd[c] * k3;
     coef[c] = (float)k1;
     coef[C + c] = (float)b;
-    coef[2 * C + c] = (float)(-k1 * (sg / (double)count) - b * (double)mean[c]);
+    coef[2 * C + c] = (float)(-k1 * (sg * inv_n) - b * (double)mean[c]);
 }
 
 template <int MASK>
@@ -461,8 +461,8 @@ int bwd_launch_mask(const dbl_bn_shape* s, const void* dout, const void* dout2, 
     int rc = launch_check("bn_bwd_reduce launch");
     if (rc) return rc;
     bn_bwd_finalize_kernel<<<(C + dbl::dev::kPartialsChannels - 1) / dbl::dev::kPartialsChannels,
-                             dbl::dev::kPartialsThreads, 0, st>>>(partial, (int)nblk, C, s->count, gamma, mean,
-                                                                         invstd, dgamma, dbeta, coef);
+                             dbl::dev::kPartialsThreads, 0, st>>>(partial, (int)nblk, C, 1.0 / (double)s->count,
+                                                                         gamma, mean, invstd, dgamma, dbeta, coef);
     if ((rc = launch_check("bn_bwd_finalize launch"))) return rc;
     if (g_store)
         bn_bwd_apply_kernel<kMaskNone><<<bn_grid(s->count * C / 8, kBwdBlocksPerSM), kThreads, 0, st>>>(
@@ -498,7 +498,8 @@ namespace dbl {
 int bn_fwd_finalize(int64_t count, int C, float eps, const float* sum, const float* sumsq, float* save_mean,
                     float* save_invstd, cudaStream_t st)
 {
-    bn_fwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(count, C, eps, sum, sumsq, save_mean, save_invstd);
+    bn_fwd_finalize_kernel<<<(C + 127) / 128, 128, 0, st>>>(1.0 / (double)count, C, eps, sum, sumsq, save_mean,
+                                                            save_invstd);
     return launch_check("bn_fwd_finalize launch");
 }
 
@@ -556,8 +557,8 @@ int dbl_bn_relu_fused_parts(const dbl_bn_shape* s, const void* y, const float* p
     if (s->count == 0) return set_error(DBL_ERR_INVALID, "bn_relu_fused_parts: empty batch has no statistics");
     cudaStream_t st = as_stream(stream);
     bn_fwd_finalize_parts_kernel<<<(s->c + dbl::dev::kPartialsChannels - 1) / dbl::dev::kPartialsChannels,
-                                   dbl::dev::kPartialsThreads, 0, st>>>(s->count, s->c, s->eps, parts, nparts, save_mean,
-                                                                   save_invstd);
+                                   dbl::dev::kPartialsThreads, 0, st>>>(1.0 / (double)s->count, s->c, s->eps, parts,
+                                                                   nparts, save_mean, save_invstd);
     if ((rc = launch_check("bn_fwd_finalize_parts launch"))) return rc;
     bn_apply_kernel<<<bn_grid(s->count * s->c / 8), kThreads, 0, st>>>(
         static_cast<const act_t*>(y), static_cast<const act_t*>(residual),
