@@ -382,8 +382,6 @@ __global__ void __launch_bounds__(256) dropout_mask_kernel(int n, int C, uint32_
     }
 }
 
-__global__ void dropout_advance_kernel(uint64_t* step) { *step += 1; }
-
 // ----------------------------------------------------------------------------- head
 // feat[n, c] = mean over hw of x[n, hw, c], then (with dropout) times the feature's multiplier
 __global__ void __launch_bounds__(256) avgpool_kernel(const act_t* __restrict__ x, float* __restrict__ feat,
@@ -657,9 +655,13 @@ __global__ void __launch_bounds__(1024) avgpool_img_kernel(const act_t* __restri
     }
 }
 
+// step (or nullptr): the dropout step counter, advanced once here so that the next call draws a
+// fresh mask (every read of it in this call has happened in the forward pool)
 __global__ void __launch_bounds__(1024) avgpool_bwd_img_kernel(const float* __restrict__ df, act_t* __restrict__ dx,
-                                                               int hw, int C, const float* __restrict__ mult)
+                                                               int hw, int C, const float* __restrict__ mult,
+                                                               uint64_t* __restrict__ step)
 {
+    if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;
     const int groups = C / 8, S = pool_slices(groups);
     const int g = threadIdx.x % groups, sl = threadIdx.x / groups;
     const int b = blockIdx.x;
@@ -677,8 +679,10 @@ __global__ void __launch_bounds__(1024) avgpool_bwd_img_kernel(const float* __re
 
 // dx[n, i, c] = df[n, c] / hw, with dropout (df[n, c] * mult[n, c]) / hw
 __global__ void __launch_bounds__(256) avgpool_bwd_kernel(const float* __restrict__ df, act_t* __restrict__ dx,
-                                                          int n, int hw, int C, const float* __restrict__ mult)
+                                                          int n, int hw, int C, const float* __restrict__ mult,
+                                                          uint64_t* __restrict__ step)
 {
+    if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;  // as in avgpool_bwd_img_kernel
     const int groups = C / 8;
     const int64_t total = (int64_t)n * hw * groups;
     const float inv = 1.0f / (float)hw;
@@ -837,14 +841,15 @@ int head_fwd_bwd(int32_t n, int32_t hw, int32_t c, int32_t classes, const void* 
     // df[n, c] = sum_j dl[n, j] W[j, c]
     if ((rc = gemm_f32(logits, classes, 1, fc_w, 1, c, nullptr, df, c, n, c, classes, part, s, "fc dX launch")))
         return rc;
+    // with dropout, the pool's backward also advances the step counter (the next call draws a fresh mask)
+    uint64_t* adv = dp.thr ? step : nullptr;
     if (per_image)
-        avgpool_bwd_img_kernel<<<n, S * groups, 0, s>>>(df, static_cast<act_t*>(dx), hw, c, dp.thr ? mult : nullptr);
+        avgpool_bwd_img_kernel<<<n, S * groups, 0, s>>>(df, static_cast<act_t*>(dx), hw, c, dp.thr ? mult : nullptr,
+                                                        adv);
     else
         avgpool_bwd_kernel<<<grid_for((int64_t)n * hw * groups, 256), 256, 0, s>>>(df, static_cast<act_t*>(dx), n, hw,
-                                                                                    c, dp.thr ? mult : nullptr);
-    if ((rc = launch_check("avgpool_bwd launch")) || !dp.thr) return rc;
-    dropout_advance_kernel<<<1, 1, 0, s>>>(step);  // the next call draws a fresh mask
-    return launch_check("dropout advance launch");
+                                                                                    c, dp.thr ? mult : nullptr, adv);
+    return launch_check("avgpool_bwd launch");
 }
 
 }  // namespace
